@@ -1,0 +1,72 @@
+"""The oracle's pins must catch plausible mistakes.
+
+Each case plants one mistake in a temporary copy of ``oracle/oracle.c`` (a
+dropped term, a wrong comparison, sign or bound, a lost reset), builds it on
+the CPU, routes the oracle wrappers to it and runs a battery of pins drawn from
+the other oracle tests.  At least one pin must fail for every planted mistake.
+The committed oracle is never modified.
+"""
+import os
+import subprocess
+
+import numpy as np
+import pytest
+
+import oracle
+import test_oracle_search as S
+import test_oracle_stopping as T
+
+SRC = os.path.join(os.path.dirname(oracle.__file__), "oracle.c")
+
+MUTATIONS = [
+    ("tau test strict", "if (s >= tau) {", "if (s > tau) {"),
+    ("hit does not reset the run", "if (f(ctx, searched))\n            stale = 0;",
+     "if (f(ctx, searched))\n            stale = stale;"),
+    ("id tie-break reversed", "(sa == sb && ia < ib)", "(sa == sb && ia > ib)"),
+    ("stop line one short", "int64_t reach = (int64_t)j + W;", "int64_t reach = (int64_t)j + W - 1;"),
+    ("first coordinate dropped", "for (int t = 0; t < d; ++t)", "for (int t = 1; t < d; ++t)"),
+    ("centroid order reversed", "if (x->score > y->score) return -1;",
+     "if (x->score > y->score) return 1;"),
+    ("self not excluded", "if (has_qid && id == qid)\n            continue;", ""),
+    ("initial stop line 1", "int64_t s = W < nprobe ? W : nprobe;", "int64_t s = 1;"),
+    ("merge drops last local entry", "m < (local_n[j] > 0 ? local_n[j] : 0)",
+     "m + 1 < (local_n[j] > 0 ? local_n[j] : 0)"),
+    ("window off by one", "while (searched < nprobe && stale < W)",
+     "while (searched < nprobe && stale <= W)"),
+]
+
+
+def _pins(tiny, deep):
+    """Each pin is a zero-argument callable that raises on failure."""
+    return [
+        T.test_golden_examples,
+        lambda: T.test_exhaustive_patterns(6),
+        S.test_tau_boundary_self_and_ties,
+        S.test_fig4_walk_end_to_end,
+        lambda: S.test_rank_matches_numpy_sort(tiny),
+        lambda: S.test_full_probe_equals_bruteforce(deep),
+        lambda: S.test_window_at_least_nprobe_is_fixed_probe(tiny, 16),
+        lambda: S.test_probes_follow_hit_pattern(deep),
+    ]
+
+
+@pytest.mark.parametrize("name,old,new", MUTATIONS, ids=[m[0] for m in MUTATIONS])
+def test_planted_mistake_is_caught(tmp_path, tiny, deep, name, old, new):
+    src = open(SRC).read()
+    assert src.count(old) == 1, f"mutation site for '{name}' not unique"
+    mutated = tmp_path / "oracle_mut.c"
+    mutated.write_text(src.replace(old, new))
+    lib = tmp_path / "liboracle_mut.so"
+    subprocess.run(["gcc", "-std=c11", "-O2", "-fopenmp", "-fPIC", "-shared", "-o", str(lib),
+                    str(mutated), "-lm"], check=True)
+    oracle.use_library(str(lib))
+    failed = []
+    try:
+        for pin in _pins(tiny, deep):
+            try:
+                pin()
+            except (AssertionError, ValueError):
+                failed.append(pin)
+    finally:
+        oracle.use_library(None)
+    assert failed, f"no pin caught the planted mistake '{name}'"
