@@ -1,0 +1,410 @@
+#!/usr/bin/env python
+"""Throughput of the threshold-aware IVF search on GB300 (one JSON line).
+
+A step is one ``sieve_search`` call over one batch of queries: centroid
+ranking, then device-resident rounds of issue / bucketing / grouped scan with
+the fused tau, top-k and stop-line epilogue / merge until every query has
+stopped.  The workload is the 1M x 256 configuration (1,024 partitions,
+100K database-drawn queries, tau 0.90, k 10, nprobe 64, W 8, lookahead on),
+synthetic and seeded (``synth``), with the index resident in HBM.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl sieve|reference]
+
+With N > 1 (torchrun) each rank searches its own query batch against its own
+replica of the index (queries shard with no data-path exchange: weak scaling);
+the step time is the maximum over ranks.  ``--impl reference`` times the fp64
+CPU oracle on the host cores instead (rank 0 only).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = ("queries/s at W=8 (tau-filtered top-10) + speedup vs fixed-probe; "
+          "% HBM/tensor roofline")
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=("sieve", "reference"), default="sieve")
+    ap.add_argument("--config", default="1m")
+    ap.add_argument("--skip-cpu-baseline", action="store_true")
+    ap.add_argument("--skip-e2e", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0,
+                    help="target CPU seconds for the oracle sample")
+    return ap.parse_args()
+
+
+def workload_desc(cfg):
+    return (f"{cfg.name}: {cfg.n:,} x {cfg.d} fp32 unit-norm rows, {cfg.ncomp} components"
+            f"{'' if cfg.zipf is None else f' Zipf({cfg.zipf})'}, planted near-duplicates, "
+            f"nlist {cfg.nlist}, {cfg.nq:,} database-drawn queries, tau {cfg.tau}, k {cfg.k}, "
+            f"nprobe {cfg.nprobe}, W {cfg.W}, lookahead on")
+
+
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    """nvidia-smi samples (every 200 ms) while the GPU is busy."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,utilization.gpu,"
+              "clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=self.fh, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.fh.close()
+        rows = []
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 10:
+                continue
+            try:
+                rows.append({"sm": float(parts[1]), "max": float(parts[2]), "util": float(parts[4]),
+                             "hw": parts[6], "hwt": parts[7], "swt": parts[8], "pcap": parts[9]})
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        busy = [r for r in rows if r["util"] >= 50] or rows
+        reasons = set()
+        for r in busy:
+            for key, name in (("hw", "hw_slowdown"), ("hwt", "hw_thermal_slowdown"),
+                              ("swt", "sw_thermal_slowdown"), ("pcap", "sw_power_cap")):
+                if r[key].lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(r["sm"] for r in busy),
+                "sm_max_mhz": max(r["max"] for r in busy), "reasons": sorted(reasons),
+                "samples": len(busy)}
+
+
+# ---------------------------------------------------------------------------
+def measured_peaks():
+    try:
+        return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except Exception:
+        return {}
+
+
+def kernel_source_sha():
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2608_03199_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        if f.endswith((".cu", ".cuh")):
+            h.update(open(os.path.join(csrc, f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def committed_traffic(kernel, workload):
+    """DRAM bytes per launch from the committed ncu summary, if the kernel
+    sources are unchanged since it was taken."""
+    try:
+        t = json.load(open(os.path.join(ROOT, "profiles", "traffic.json")))
+    except Exception:
+        return None
+    e = t.get(kernel, {}).get(workload)
+    if not e or e.get("source_sha") != kernel_source_sha():
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+def roofline(prof, cfg, dev):
+    """Roofline entry for the kernel with the largest share of the step."""
+    km, kl = prof["kernel_ms"], prof["kernel_launches"]
+    top = max(km, key=lambda k: km[k])
+    props = torch.cuda.get_device_properties(dev)
+    peaks = measured_peaks()
+    clock_mhz = peaks.get("sm_max_mhz", 2070.0)
+    fp32_tflops = props.multi_processor_count * 128 * 2 * clock_mhz * 1e6 / 1e12
+    hbm = peaks.get("hbm_gbs", 6800.0)
+    d = cfg.d
+    launches = max(1, kl[top])
+    ms_per_launch = km[top] / launches
+    out = {"kernel": f"k_{top}", "launches": kl[top], "ms_per_launch": ms_per_launch}
+    if top == "scan":
+        flops = 2.0 * d * prof["pairs"]
+        ach = flops / launches / (ms_per_launch * 1e-3) / 1e12
+        bytes_ = 4.0 * d * (prof["rows_read"] + prof["items"])
+        out.update(bound="alu", achieved=ach, peak=fp32_tflops, unit="TFLOP/s",
+                   frac=ach / fp32_tflops,
+                   peak_source=f"FP32 FMA: {props.multi_processor_count} SMs x 128 lanes x 2 "
+                               f"x {clock_mhz:.0f} MHz (measured max clock)",
+                   hbm_view={"achieved_gbs": bytes_ / launches / (ms_per_launch * 1e-3) / 1e9,
+                             "peak_gbs": hbm})
+    elif top == "rank":
+        flops = 2.0 * cfg.nq * cfg.nlist * d
+        ach = flops / (ms_per_launch * 1e-3) / 1e12
+        out.update(bound="alu", achieved=ach, peak=fp32_tflops, unit="TFLOP/s",
+                   frac=ach / fp32_tflops,
+                   peak_source=f"FP32 FMA: {props.multi_processor_count} SMs x 128 lanes x 2 "
+                               f"x {clock_mhz:.0f} MHz (measured max clock)")
+    else:
+        out.update(bound="hbm", achieved=None, peak=hbm, unit="GB/s", frac=None)
+    out["traffic"] = committed_traffic(out["kernel"], cfg.name)
+    return out
+
+
+# ---------------------------------------------------------------------------
+def dist_setup(gpus):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        torch.distributed.barrier()
+
+
+def max_over_ranks(x, world, dev):
+    if world == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def time_steps(fn, steps, warmup, world, dev):
+    for _ in range(warmup):
+        fn()
+    torch.cuda.synchronize()
+    barrier(world)
+    st = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(st)
+    for _ in range(steps):
+        fn()
+    e1.record(st)
+    torch.cuda.synchronize()
+    barrier(world)
+    ms = e0.elapsed_time(e1) / steps
+    return max_over_ranks(ms, world, dev)
+
+
+def cpu_baseline(w, cfg, target_s):
+    """The oracle (fp64, OpenMP over queries) on a bounded query sample."""
+    import oracle
+    idx = {k: w[k] for k in ("X", "ids", "assign", "centroids")}
+    threads = oracle.default_threads()
+    probe = min(cfg.nq, 64)
+    t0 = time.perf_counter()
+    oracle.search(idx, w["Q"][:probe], cfg.tau, cfg.k, cfg.nprobe, cfg.W, qids=w["qids"][:probe],
+                  threads=threads)
+    per_q = (time.perf_counter() - t0) / probe
+    sample = int(min(cfg.nq, max(probe, target_s / max(per_q, 1e-9))))
+    t0 = time.perf_counter()
+    oracle.search(idx, w["Q"][:sample], cfg.tau, cfg.k, cfg.nprobe, cfg.W,
+                  qids=w["qids"][:sample], threads=threads)
+    dt = time.perf_counter() - t0
+    return {"value": sample / dt, "unit": "queries/s", "cores": threads, "kind": "oracle",
+            "sample": f"first {sample:,} of the {cfg.nq:,} queries, W={cfg.W}, "
+                      f"{dt:.1f} s on {threads} host threads"}
+
+
+def host_arrays(wl):
+    return {k: wl[k].detach().cpu().numpy() for k in ("X", "ids", "assign", "centroids", "Q", "qids")}
+
+
+# ---------------------------------------------------------------------------
+def run_reference(args, cfg, world, rank):
+    if rank != 0:
+        return 0
+    import oracle
+    dev = torch.device("cuda:0") if torch.cuda.is_available() else torch.device("cpu")
+    wl = synth.make_workload(cfg, device=dev)
+    w = host_arrays(wl)
+    del wl
+    idx = {k: w[k] for k in ("X", "ids", "assign", "centroids")}
+    threads = oracle.default_threads()
+    probe = min(cfg.nq, 64)
+    t0 = time.perf_counter()
+    oracle.search(idx, w["Q"][:probe], cfg.tau, cfg.k, cfg.nprobe, cfg.W, qids=w["qids"][:probe],
+                  threads=threads)
+    per_q = (time.perf_counter() - t0) / probe
+    budget = 150.0 / max(1, args.steps + args.warmup)       # whole run within a few minutes
+    sample = int(min(cfg.nq, max(16, budget / max(per_q, 1e-9))))
+    times = []
+    for i in range(args.warmup + args.steps):
+        lo = (i * sample) % max(1, cfg.nq - sample + 1)
+        t0 = time.perf_counter()
+        oracle.search(idx, w["Q"][lo:lo + sample], cfg.tau, cfg.k, cfg.nprobe, cfg.W,
+                      qids=w["qids"][lo:lo + sample], threads=threads)
+        if i >= args.warmup:
+            times.append(time.perf_counter() - t0)
+    step_s = sum(times) / len(times)
+    value = sample / step_s
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "queries/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": workload_desc(cfg), "queries_per_step": sample},
+        "cpu_baseline": {"value": value, "unit": "queries/s", "cores": threads, "kind": "oracle",
+                         "sample": f"{sample:,} queries per step of the {cfg.nq:,}-query batch"},
+        "e2e": {"value": value, "unit": "queries/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
+def run_sieve(args, cfg, world, rank, local):
+    import paper_2608_03199_gb300 as sieve
+
+    assert torch.cuda.is_available(), "bench.py needs a CUDA device"
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        torch.distributed.init_process_group("nccl", device_id=dev)
+    sieve.lib()
+    wl = synth.make_workload(cfg, device=dev, query_stream=rank)
+    index = sieve.build_layout(wl["X"], wl["assign"], cfg.nlist, wl["centroids"])
+    Q, qids = wl["Q"], wl["qids"]
+    torch.cuda.synchronize()
+
+    ws = sieve.Workspace()
+    nq, k = cfg.nq, cfg.k
+    outs = (torch.empty((nq, k), dtype=torch.int64, device=dev),
+            torch.empty((nq, k), dtype=torch.float32, device=dev),
+            torch.empty(nq, dtype=torch.int32, device=dev),
+            torch.empty(nq, dtype=torch.int32, device=dev))
+
+    def step(W):
+        return lambda: sieve.search(index, Q, cfg.tau, k, cfg.nprobe, W, lookahead=True,
+                                    query_ids=qids, workspace=ws, out=outs)
+
+    clocks = ClockSampler(local)
+    clocks.start()
+    ms = time_steps(step(cfg.W), args.steps, args.warmup, world, dev)
+    clock_rec = clocks.stop()
+    ms_fixed = time_steps(step(cfg.nprobe), max(3, args.steps // 5), 2, world, dev)
+
+    # one profiled step (host-driven rounds, CUDA events around every launch)
+    prof = sieve.search(index, Q, cfg.tau, k, cfg.nprobe, cfg.W, lookahead=True, query_ids=qids,
+                        profile=True, workspace=ws)[4]
+    probes = outs[3]
+    sieve.search(index, Q, cfg.tau, k, cfg.nprobe, cfg.W, lookahead=True, query_ids=qids,
+                 workspace=ws, out=outs)
+    mean_probes = float(probes.float().mean().item())
+    hit_frac = float((outs[2] > 0).float().mean().item())
+
+    # end to end through the C ABI with host buffers
+    e2e = None
+    if not args.skip_e2e:
+        Qh = Q.cpu().pin_memory()
+        qh = qids.cpu().pin_memory()
+        houts = (torch.empty((nq, k), dtype=torch.int64, pin_memory=True),
+                 torch.empty((nq, k), dtype=torch.float32, pin_memory=True),
+                 torch.empty(nq, dtype=torch.int32, pin_memory=True),
+                 torch.empty(nq, dtype=torch.int32, pin_memory=True))
+        hws = sieve.Workspace()
+
+        def hstep():
+            sieve.search_host(index, Qh, cfg.tau, k, cfg.nprobe, cfg.W, lookahead=True,
+                              query_ids_host=qh, workspace=hws, out=houts)
+        hsteps = max(3, args.steps // 5)
+        for _ in range(2):
+            hstep()
+        barrier(world)
+        t0 = time.perf_counter()
+        for _ in range(hsteps):
+            hstep()
+        torch.cuda.synchronize()
+        barrier(world)
+        e2e_ms = max_over_ranks((time.perf_counter() - t0) / hsteps * 1e3, world, dev)
+        e2e = {"value": nq * world / (e2e_ms * 1e-3), "unit": "queries/s",
+               "ms_per_step": e2e_ms, "h2d_bytes_per_step": nq * cfg.d * 4 + nq * 8,
+               "d2h_bytes_per_step": nq * (k * 12 + 8)}
+
+    line = {
+        "metric": METRIC,
+        "value": nq * world / (ms * 1e-3),
+        "unit": "queries/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": ms,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f32",
+        "data": "synthetic",
+        "config": {"workload": workload_desc(cfg), "nq_per_gpu": nq, "parallelism": f"query-shard x{world}",
+                   "l2": "inputs larger than L2 (index 1.02 GB streamed per step)"},
+        "fixed_probe": {"value": nq * world / (ms_fixed * 1e-3), "ms_per_step": ms_fixed,
+                        "W": cfg.nprobe},
+        "speedup_vs_fixed": ms_fixed / ms,
+        "mean_probes": mean_probes,
+        "queries_with_results": hit_frac,
+        "roofline": roofline(prof, cfg, dev),
+        "profile": {"kernel_ms": prof["kernel_ms"], "kernel_launches": prof["kernel_launches"],
+                    "rounds": prof["rounds"], "items": prof["items"], "groups": prof["groups"],
+                    "mean_group": prof["items"] / max(1, prof["groups"]),
+                    "pairs": prof["pairs"], "rows_read": prof["rows_read"]},
+        "gpu_launches": args.steps * int(sum(prof["kernel_launches"].values())),
+        "clocks": clock_rec,
+        "e2e": e2e,
+    }
+    if rank == 0 and world == 1 and not args.skip_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(host_arrays(wl), cfg, args.cpu_seconds)
+    if rank == 0:
+        print(json.dumps(line))
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse()
+    cfg = synth.CONFIGS[args.config]
+    world, rank, local = dist_setup(args.gpus)
+    if args.impl == "reference":
+        return run_reference(args, cfg, world, rank)
+    return run_sieve(args, cfg, world, rank, local)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

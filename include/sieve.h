@@ -1,0 +1,224 @@
+/*
+ * sieve.h -- C ABI of libsieve, a single-GPU (sm_103a) implementation of the
+ * data-parallel hot path of SieveIVF's threshold-aware IVF search
+ * (arXiv 2608.03199).
+ *
+ * A query batch Q searches an IVF index: each query ranks the centroids
+ * (Sec. 2.3, Sec. 4.1), then visits partitions in that order.  A visit is a
+ * hit when the partition holds a row x with sim(q, x) >= tau (R(q, tau),
+ * Sec. 2.2).  A query stops after W consecutive empty visits or at nprobe
+ * (Sec. 4.1); equivalently it searches ranks 1..s, where the stop line s
+ * starts at min(W, nprobe) and a hit at rank j raises it to
+ * max(s, min(j + W, nprobe)) (Sec. 4.3).  Active queries are regrouped by
+ * partition every round (continuous batching, Algorithm 1); with lookahead
+ * every committed rank is issued at once (Algorithm 2).  The result is the
+ * top-k of the qualifying rows over the searched partitions (MergeTopK).
+ *
+ * Conventions for every call:
+ *   - similarity is the fp32 inner product of unit-norm vectors (cosine);
+ *   - "device" pointers are CUDA global memory of the current device;
+ *     "host" pointers are ordinary (ideally page-locked) host memory;
+ *   - the library allocates no device memory: scratch comes from the
+ *     caller's workspace (ws, ws_bytes), sized by the *_workspace_size calls,
+ *     256-byte aligned; the caller owns every buffer and must keep it alive
+ *     until the stream has passed the call;
+ *   - calls are asynchronous on `stream` (0 = the legacy default stream)
+ *     unless stated otherwise; they never abort and never print; a failure
+ *     returns a negative sieve_status and, for SIEVE_ECUDA, records the CUDA
+ *     error code (sieve_last_cuda_error, per host thread);
+ *   - calls on different streams may run concurrently when they use
+ *     different workspaces; one workspace must not be shared by calls that
+ *     may overlap.
+ */
+#ifndef SIEVE_H
+#define SIEVE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int32_t sieve_status;
+#define SIEVE_OK 0
+#define SIEVE_EINVAL (-1)       /* bad shape, parameter or null required pointer */
+#define SIEVE_ECUDA (-2)        /* a CUDA runtime call failed */
+#define SIEVE_EWORKSPACE (-3)   /* ws_bytes below the size the call needs, or ws misaligned */
+#define SIEVE_ELIMIT (-4)       /* the device round loop hit its round limit (see sieve_stats) */
+#define SIEVE_EUNSUPPORTED (-5) /* the current device is not sm_103 */
+
+/* The IVF index, resident on the device (Sec. 2.3).  Borrowed, read-only.
+ *   vectors      device [n][d] fp32, unit-norm, partition-contiguous: the rows
+ *                of partition p are list_offsets[p] .. list_offsets[p+1]-1
+ *   ids          device [n] int64, the external id of each stored row
+ *   list_offsets device [nlist+1] int64, nondecreasing, [0] = 0, [nlist] = n
+ *   centroids    device [nlist][d] fp32 (unit-norm for cosine ranking)
+ * d must be a multiple of 4 and at most 1024; every base pointer 16-byte
+ * aligned.  Every row must sit in the partition of its nearest centroid
+ * (exact assignment, the precondition of Sec. 4.4); the library does not
+ * check this. */
+typedef struct {
+    int64_t n;
+    int64_t nlist;
+    int32_t d;
+    int32_t reserved0;
+    const float *vectors;
+    const int64_t *ids;
+    const int64_t *list_offsets;
+    const float *centroids;
+} sieve_index_view;
+
+/* Search parameters (Sec. 4, Sec. 6.1).
+ *   tau        similarity threshold; a row qualifies iff sim >= tau; not NaN
+ *   k          results per query, 1..64
+ *   nprobe     maximum partitions per query, 1..min(nlist, 512)
+ *   W          consecutive-empty window, >= 1; W >= nprobe is fixed probing
+ *   lookahead  0 = continuous batching (one rank per query per round,
+ *              Algorithm 1), 1 = issue every committed rank (Algorithm 2)
+ *   max_items_per_round  cap on (query, rank) items issued in one round;
+ *              0 = automatic.  Only splits work into more rounds: the result
+ *              does not depend on it (Sec. 4.2).
+ *   loop       0 = device-resident round loop (a CUDA graph whose WHILE node
+ *              runs rounds until no item is left; no host sync per round),
+ *              1 = host-driven rounds (one stream sync per round; a debugging
+ *              aid that must give identical results)
+ *   profile    1 = also time every kernel launch with CUDA events recorded on
+ *              `stream` around it (implies host-driven rounds and needs a
+ *              stats pointer); 0 = no timing
+ *   reserved0  must be 0
+ */
+typedef struct {
+    float tau;
+    int32_t k;
+    int32_t nprobe;
+    int32_t W;
+    int32_t lookahead;
+    int32_t loop;
+    int32_t profile;
+    int32_t reserved0;
+    int64_t max_items_per_round;
+} sieve_params;
+
+/* Kernels of one search call, indexing sieve_stats.kernel_ms / kernel_launches:
+ * centroid ranking, state initialisation, the issuer, the ready-queue
+ * bucketing, the scatter into partition groups, the grouped scan with its
+ * fused epilogue, the per-query merge, the end-of-round step, finalisation. */
+enum {
+    SIEVE_K_RANK = 0,
+    SIEVE_K_INIT,
+    SIEVE_K_ISSUE,
+    SIEVE_K_BUCKET,
+    SIEVE_K_SCATTER,
+    SIEVE_K_SCAN,
+    SIEVE_K_MERGE,
+    SIEVE_K_ROUND_END,
+    SIEVE_K_FINALIZE,
+    SIEVE_NKERNELS
+};
+
+/* Counters of one search call (filled only when a stats pointer is given;
+ * that makes the call synchronize `stream`).
+ *   rounds       rounds executed
+ *   items        (query, rank) items searched = sum of probes over queries
+ *   groups       sum over rounds of partitions with at least one item
+ *                (partition groups, Sec. 4.2); items / groups = mean group
+ *   tiles        work tiles of the grouped scan
+ *   rows_read    partition rows streamed by the scan (one read per tile)
+ *   pairs        query-row similarities computed
+ *   status       device status word (0, or a SIEVE_E* code) */
+typedef struct {
+    int64_t rounds;
+    int64_t items;
+    int64_t groups;
+    int64_t tiles;
+    int64_t rows_read;
+    int64_t pairs;
+    int32_t status;
+    int32_t reserved0;
+    float kernel_ms[SIEVE_NKERNELS];          /* profile = 1: summed launch durations */
+    int32_t kernel_launches[SIEVE_NKERNELS];  /* launches per kernel in the call */
+} sieve_stats;
+
+/* Partition-contiguous layout of an index (the storage of Sec. 2.3):
+ * a stable counting sort of the rows of X by their partition.
+ *   X          device [n][d] fp32, rows in any order
+ *   assign     device [n] int32, partition of each row, 0 <= assign < nlist
+ *   X_sorted   device [n][d] fp32 out; ids_sorted device [n] int64 out (the
+ *              row index in X of each sorted row, so the ids are 0..n-1);
+ *   list_offsets device [nlist+1] int64 out
+ * Rows of one partition keep their order in X.  An out-of-range assign
+ * value makes the call return SIEVE_EINVAL after the kernels ran (the call
+ * synchronizes `stream`).  Workspace: sieve_layout_workspace_size. */
+sieve_status sieve_layout_workspace_size(int64_t n, int64_t nlist, size_t *bytes);
+sieve_status sieve_build_layout(const float *X, const int32_t *assign, int64_t n, int32_t d,
+                                int64_t nlist, float *X_sorted, int64_t *ids_sorted,
+                                int64_t *list_offsets, void *ws, size_t ws_bytes,
+                                void *stream);
+
+/* Centroid ranking (Sec. 2.3, Sec. 4.1): for every query, the nprobe
+ * centroids with the largest fp32 inner product, best first; equal scores
+ * rank the lower centroid id first.
+ *   Q        device [nq][d] fp32
+ *   order    device [nq][nprobe] int32 out, 0-based centroid ids
+ *   cscores  device [nq][nprobe] fp32 out (nullable): the matching scores
+ * Needs no workspace (ws may be NULL, ws_bytes 0). */
+sieve_status sieve_rank_partitions(const sieve_index_view *ix, const float *Q, int64_t nq,
+                                   int32_t nprobe, int32_t *order, float *cscores, void *ws,
+                                   size_t ws_bytes, void *stream);
+
+/* Workspace bytes sieve_search needs for nq queries with these parameters.
+ * host_io = 1 sizes it for sieve_search_host (adds device staging for the
+ * queries and results). */
+sieve_status sieve_search_workspace_size(const sieve_index_view *ix, int64_t nq,
+                                         const sieve_params *p, int32_t host_io,
+                                         size_t *bytes);
+
+/* Threshold-aware IVF search (Sec. 4, Algorithms 1 and 2), all on the device.
+ *   Q          device [nq][d] fp32 queries (unit-norm)
+ *   query_ids  device [nq] int64 (nullable): a row whose id equals its
+ *              query's id is neither a candidate nor a hit (self-join
+ *              deduplication with queries drawn from the indexed rows)
+ *   order      device [nq][nprobe] int32 (nullable): precomputed centroid
+ *              ranks; NULL ranks inside the call (sieve_rank_partitions)
+ *   out_ids    device [nq][k] int64: result ids by (score desc, id asc),
+ *              -1 past out_count
+ *   out_scores device [nq][k] fp32: their similarities, -inf past out_count
+ *   out_count  device [nq] int32: results per query (<= k)
+ *   out_probes device [nq] int32: partitions searched (the final stop line)
+ *   stats      host (nullable): counters; non-NULL synchronizes `stream`
+ * nq = 0 is valid and does nothing.  A list_offsets table that is not a
+ * partition of [0, n), or an order entry outside [0, nlist), is detected on
+ * the device: nothing past it is searched and, with stats, the call returns
+ * SIEVE_EINVAL (without stats the outputs are then undefined). */
+sieve_status sieve_search(const sieve_index_view *ix, const float *Q, int64_t nq,
+                          const int64_t *query_ids, const int32_t *order,
+                          const sieve_params *p, int64_t *out_ids, float *out_scores,
+                          int32_t *out_count, int32_t *out_probes, sieve_stats *stats,
+                          void *ws, size_t ws_bytes, void *stream);
+
+/* sieve_search with the queries and results in HOST memory: copies Q (and
+ * query_ids) to device staging inside the workspace, searches, copies the
+ * results back and synchronizes `stream` before returning.  Pointers as in
+ * sieve_search but host-side; workspace from
+ * sieve_search_workspace_size(..., host_io = 1, ...). */
+sieve_status sieve_search_host(const sieve_index_view *ix, const float *Q_host, int64_t nq,
+                               const int64_t *query_ids_host, const sieve_params *p,
+                               int64_t *out_ids_host, float *out_scores_host,
+                               int32_t *out_count_host, int32_t *out_probes_host,
+                               sieve_stats *stats, void *ws, size_t ws_bytes, void *stream);
+
+/* Human-readable name of a status code (static string). */
+const char *sieve_status_str(sieve_status s);
+
+/* The CUDA error code behind the calling thread's last SIEVE_ECUDA (0 if none). */
+int32_t sieve_last_cuda_error(void);
+
+/* Library version string. */
+const char *sieve_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SIEVE_H */

@@ -1,0 +1,320 @@
+"""Python binding of libsieve: threshold-aware IVF search on one GB300 (sm_103a).
+
+This module only marshals arguments: it takes torch tensors (device memory and
+streams come from PyTorch), passes raw pointers and sizes to the C ABI declared
+in ``include/sieve.h``, and returns tensors.  Every step of the search runs in
+libsieve's CUDA kernels; there is no CPU or PyTorch fallback.  If the library
+cannot be built or loaded the calls raise.
+
+Entry points (same names as the C ABI):
+
+* :func:`build_layout`      -- partition-contiguous storage of an IVF index
+* :func:`rank_partitions`   -- per-query top-nprobe centroid order
+* :func:`search`            -- SieveIVF search on device tensors
+* :func:`search_host`       -- the same with host queries and host results
+"""
+from __future__ import annotations
+
+import ctypes as C
+import threading
+from dataclasses import dataclass
+
+import torch
+
+from . import _build
+
+SIEVE_OK = 0
+_STATUS = {0: "ok", -1: "invalid argument", -2: "CUDA error", -3: "workspace", -4: "round limit",
+           -5: "unsupported device"}
+
+
+class SieveError(RuntimeError):
+    def __init__(self, status: int, what: str, cuda_error: int = 0):
+        msg = f"{what}: status {status} ({_STATUS.get(status, '?')})"
+        if status == -2:
+            msg += f", cudaError {cuda_error}"
+        super().__init__(msg)
+        self.status = status
+
+
+class IndexViewC(C.Structure):
+    _fields_ = [("n", C.c_int64), ("nlist", C.c_int64), ("d", C.c_int32), ("reserved0", C.c_int32),
+                ("vectors", C.c_void_p), ("ids", C.c_void_p), ("list_offsets", C.c_void_p),
+                ("centroids", C.c_void_p)]
+
+
+class ParamsC(C.Structure):
+    _fields_ = [("tau", C.c_float), ("k", C.c_int32), ("nprobe", C.c_int32), ("W", C.c_int32),
+                ("lookahead", C.c_int32), ("loop", C.c_int32), ("profile", C.c_int32),
+                ("reserved0", C.c_int32), ("max_items_per_round", C.c_int64)]
+
+
+class StatsC(C.Structure):
+    _fields_ = [("rounds", C.c_int64), ("items", C.c_int64), ("groups", C.c_int64),
+                ("tiles", C.c_int64), ("rows_read", C.c_int64), ("pairs", C.c_int64),
+                ("status", C.c_int32), ("reserved0", C.c_int32),
+                ("kernel_ms", C.c_float * 9), ("kernel_launches", C.c_int32 * 9)]
+
+
+KERNELS = ("rank", "init", "issue", "bucket", "scatter", "scan", "merge", "round_end", "finalize")
+
+
+_lib = None
+_lib_lock = threading.Lock()
+
+# every function include/sieve.h declares, with its ctypes signature
+_SIGNATURES = {
+    "sieve_layout_workspace_size": (C.c_int32, [C.c_int64, C.c_int64, C.POINTER(C.c_size_t)]),
+    "sieve_build_layout": (C.c_int32, [C.c_void_p, C.c_void_p, C.c_int64, C.c_int32, C.c_int64,
+                                       C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_size_t,
+                                       C.c_void_p]),
+    "sieve_rank_partitions": (C.c_int32, [C.POINTER(IndexViewC), C.c_void_p, C.c_int64, C.c_int32,
+                                          C.c_void_p, C.c_void_p, C.c_void_p, C.c_size_t,
+                                          C.c_void_p]),
+    "sieve_search_workspace_size": (C.c_int32, [C.POINTER(IndexViewC), C.c_int64,
+                                                C.POINTER(ParamsC), C.c_int32,
+                                                C.POINTER(C.c_size_t)]),
+    "sieve_search": (C.c_int32, [C.POINTER(IndexViewC), C.c_void_p, C.c_int64, C.c_void_p,
+                                 C.c_void_p, C.POINTER(ParamsC), C.c_void_p, C.c_void_p,
+                                 C.c_void_p, C.c_void_p, C.POINTER(StatsC), C.c_void_p,
+                                 C.c_size_t, C.c_void_p]),
+    "sieve_search_host": (C.c_int32, [C.POINTER(IndexViewC), C.c_void_p, C.c_int64, C.c_void_p,
+                                      C.POINTER(ParamsC), C.c_void_p, C.c_void_p, C.c_void_p,
+                                      C.c_void_p, C.POINTER(StatsC), C.c_void_p, C.c_size_t,
+                                      C.c_void_p]),
+    "sieve_status_str": (C.c_char_p, [C.c_int32]),
+    "sieve_last_cuda_error": (C.c_int32, []),
+    "sieve_version": (C.c_char_p, []),
+}
+
+
+def build(force: bool = False) -> str:
+    """Compile libsieve for sm_103a (in-tree); returns the library path."""
+    return _build.build(force=force)
+
+
+def lib():
+    """The loaded libsieve (built on first use)."""
+    global _lib
+    with _lib_lock:
+        if _lib is None:
+            path = _build.build()
+            handle = C.CDLL(path)
+            for name, (res, args) in _SIGNATURES.items():
+                fn = getattr(handle, name)
+                fn.restype = res
+                fn.argtypes = args
+            _lib = handle
+        return _lib
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def _check(status: int, what: str):
+    if status != SIEVE_OK:
+        raise SieveError(status, what, lib().sieve_last_cuda_error())
+
+
+def _ptr(t):
+    return None if t is None else C.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return C.c_void_p(stream.cuda_stream)
+
+
+def _need_cuda(t, dtype, name, ndim=None):
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if ndim is not None and t.dim() != ndim:
+        raise ValueError(f"{name} must have {ndim} dims")
+    return t
+
+
+@dataclass
+class Index:
+    """A device-resident IVF index in the layout libsieve reads."""
+    vectors: torch.Tensor        # [n][d] f32, partition-contiguous
+    ids: torch.Tensor            # [n] i64
+    list_offsets: torch.Tensor   # [nlist+1] i64
+    centroids: torch.Tensor      # [nlist][d] f32
+
+    def view(self) -> IndexViewC:
+        v = IndexViewC()
+        v.n = self.vectors.shape[0]
+        v.nlist = self.centroids.shape[0]
+        v.d = self.vectors.shape[1]
+        v.vectors = self.vectors.data_ptr()
+        v.ids = self.ids.data_ptr()
+        v.list_offsets = self.list_offsets.data_ptr()
+        v.centroids = self.centroids.data_ptr()
+        return v
+
+    @property
+    def nlist(self):
+        return self.centroids.shape[0]
+
+    @property
+    def d(self):
+        return self.vectors.shape[1]
+
+
+def build_layout(X, assign, nlist, centroids, stream=None) -> Index:
+    """Index from rows X [n][d] and their partitions assign [n] (sieve_build_layout).
+
+    ids of the index are the row numbers of X."""
+    _need_cuda(X, torch.float32, "X", 2)
+    _need_cuda(assign, torch.int32, "assign", 1)
+    _need_cuda(centroids, torch.float32, "centroids", 2)
+    n, d = X.shape
+    L = lib()
+    nbytes = C.c_size_t()
+    _check(L.sieve_layout_workspace_size(n, nlist, C.byref(nbytes)), "sieve_layout_workspace_size")
+    ws = torch.empty(max(nbytes.value, 1), dtype=torch.uint8, device=X.device)
+    Xs = torch.empty_like(X)
+    ids = torch.empty(n, dtype=torch.int64, device=X.device)
+    off = torch.empty(nlist + 1, dtype=torch.int64, device=X.device)
+    _check(L.sieve_build_layout(_ptr(X), _ptr(assign), n, d, nlist, _ptr(Xs), _ptr(ids), _ptr(off),
+                                _ptr(ws), nbytes.value, _stream(stream)), "sieve_build_layout")
+    return Index(Xs, ids, off, centroids.contiguous())
+
+
+def rank_partitions(index: Index, Q, nprobe, return_scores=False, stream=None):
+    """int32 [nq][nprobe] centroid order per query (sieve_rank_partitions)."""
+    _need_cuda(Q, torch.float32, "Q", 2)
+    nq = Q.shape[0]
+    order = torch.empty((nq, nprobe), dtype=torch.int32, device=Q.device)
+    sc = torch.empty((nq, nprobe), dtype=torch.float32, device=Q.device) if return_scores else None
+    v = index.view()
+    _check(lib().sieve_rank_partitions(C.byref(v), _ptr(Q), nq, nprobe, _ptr(order), _ptr(sc),
+                                       None, 0, _stream(stream)), "sieve_rank_partitions")
+    return (order, sc) if return_scores else order
+
+
+def _params(tau, k, nprobe, W, lookahead, loop, max_items_per_round, profile=0):
+    p = ParamsC()
+    p.profile = int(profile)
+    p.tau = float(tau)
+    p.k = int(k)
+    p.nprobe = int(nprobe)
+    p.W = int(min(W, 2**31 - 1))
+    p.lookahead = 1 if lookahead else 0
+    p.loop = int(loop)
+    p.max_items_per_round = int(max_items_per_round)
+    return p
+
+
+def workspace_size(index: Index, nq, tau, k, nprobe, W, lookahead=True, max_items_per_round=0,
+                   host_io=False) -> int:
+    v = index.view()
+    p = _params(tau, k, nprobe, W, lookahead, 0, max_items_per_round)
+    nbytes = C.c_size_t()
+    _check(lib().sieve_search_workspace_size(C.byref(v), nq, C.byref(p), 1 if host_io else 0,
+                                             C.byref(nbytes)), "sieve_search_workspace_size")
+    return nbytes.value
+
+
+class Workspace:
+    """A reusable device scratch buffer (grown on demand)."""
+
+    def __init__(self, device=None):
+        self.device = device
+        self.buf = None
+
+    def get(self, nbytes, device):
+        if self.buf is None or self.buf.numel() < nbytes or self.buf.device != device:
+            self.buf = torch.empty(max(nbytes, 256), dtype=torch.uint8, device=device)
+        return self.buf
+
+
+_default_ws = {}
+
+
+def _workspace(ws, nbytes, device):
+    if ws is None:
+        key = (device, torch.cuda.current_stream(device).cuda_stream)
+        ws = _default_ws.setdefault(key, Workspace())
+    return ws.get(nbytes, device)
+
+
+def _stats_dict(st):
+    out = {f: getattr(st, f) for f, _ in StatsC._fields_ if not f.startswith("kernel")}
+    out["kernel_ms"] = dict(zip(KERNELS, list(st.kernel_ms)))
+    out["kernel_launches"] = dict(zip(KERNELS, list(st.kernel_launches)))
+    return out
+
+
+def search(index: Index, Q, tau, k, nprobe, W, lookahead=True, query_ids=None, order=None,
+           max_items_per_round=0, loop=0, stats=False, profile=False, workspace=None, out=None,
+           stream=None):
+    """SieveIVF search on device tensors (sieve_search).
+
+    Returns (ids [nq][k] i64, scores [nq][k] f32, count [nq] i32, probes [nq] i32),
+    plus a dict of counters when ``stats`` or ``profile`` (both synchronize the
+    stream; ``profile`` also times every kernel launch with CUDA events)."""
+    stats = stats or profile
+    _need_cuda(Q, torch.float32, "Q", 2)
+    if query_ids is not None:
+        _need_cuda(query_ids, torch.int64, "query_ids", 1)
+    if order is not None:
+        _need_cuda(order, torch.int32, "order", 2)
+    nq = Q.shape[0]
+    dev = Q.device
+    p = _params(tau, k, nprobe, W, lookahead, loop, max_items_per_round, profile)
+    v = index.view()
+    nbytes = C.c_size_t()
+    _check(lib().sieve_search_workspace_size(C.byref(v), nq, C.byref(p), 0, C.byref(nbytes)),
+           "sieve_search_workspace_size")
+    ws = _workspace(workspace, nbytes.value, dev)
+    if out is None:
+        out = (torch.empty((nq, k), dtype=torch.int64, device=dev),
+               torch.empty((nq, k), dtype=torch.float32, device=dev),
+               torch.empty(nq, dtype=torch.int32, device=dev),
+               torch.empty(nq, dtype=torch.int32, device=dev))
+    ids, scores, count, probes = out
+    st = StatsC() if stats else None
+    _check(lib().sieve_search(C.byref(v), _ptr(Q), nq, _ptr(query_ids), _ptr(order), C.byref(p),
+                              _ptr(ids), _ptr(scores), _ptr(count), _ptr(probes),
+                              C.byref(st) if st is not None else None, _ptr(ws), ws.numel(),
+                              _stream(stream)), "sieve_search")
+    if stats:
+        return ids, scores, count, probes, _stats_dict(st)
+    return ids, scores, count, probes
+
+
+def search_host(index: Index, Q_host, tau, k, nprobe, W, lookahead=True, query_ids_host=None,
+                max_items_per_round=0, loop=0, workspace=None, out=None, stream=None):
+    """sieve_search_host: host (CPU, ideally pinned) queries in, host results out.
+
+    The call copies the queries to the device, searches, copies the results
+    back and synchronizes the stream."""
+    if Q_host.is_cuda or Q_host.dtype != torch.float32 or not Q_host.is_contiguous():
+        raise TypeError("Q_host must be a contiguous float32 CPU tensor")
+    if query_ids_host is not None and (query_ids_host.is_cuda or query_ids_host.dtype != torch.int64):
+        raise TypeError("query_ids_host must be an int64 CPU tensor")
+    nq = Q_host.shape[0]
+    dev = index.vectors.device
+    p = _params(tau, k, nprobe, W, lookahead, loop, max_items_per_round)
+    v = index.view()
+    nbytes = C.c_size_t()
+    _check(lib().sieve_search_workspace_size(C.byref(v), nq, C.byref(p), 1, C.byref(nbytes)),
+           "sieve_search_workspace_size")
+    ws = _workspace(workspace, nbytes.value, dev)
+    if out is None:
+        out = (torch.empty((nq, k), dtype=torch.int64, pin_memory=True),
+               torch.empty((nq, k), dtype=torch.float32, pin_memory=True),
+               torch.empty(nq, dtype=torch.int32, pin_memory=True),
+               torch.empty(nq, dtype=torch.int32, pin_memory=True))
+    ids, scores, count, probes = out
+    _check(lib().sieve_search_host(C.byref(v), _ptr(Q_host), nq, _ptr(query_ids_host), C.byref(p),
+                                   _ptr(ids), _ptr(scores), _ptr(count), _ptr(probes), None,
+                                   _ptr(ws), ws.numel(), _stream(stream)), "sieve_search_host")
+    return ids, scores, count, probes

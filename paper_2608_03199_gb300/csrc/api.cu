@@ -1,0 +1,523 @@
+// api.cu -- the C ABI of libsieve (declared in include/sieve.h): argument
+// checks, workspace layout, the device-resident round loop as a CUDA graph
+// with a WHILE conditional node, and the host-buffer variant.
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+#include "search.cuh"
+
+using namespace sieve;
+
+namespace {
+
+thread_local int32_t g_last_cuda_error = 0;
+
+sieve_status cuda_fail(cudaError_t e) {
+    g_last_cuda_error = (int32_t)e;
+    return SIEVE_ECUDA;
+}
+
+#define SIEVE_CUDA(call)                                  \
+    do {                                                  \
+        cudaError_t e_ = (call);                          \
+        if (e_ != cudaSuccess) return cuda_fail(e_);      \
+    } while (0)
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+sieve_status check_device() {
+    int dev = 0;
+    SIEVE_CUDA(cudaGetDevice(&dev));
+    static std::mutex m;
+    static std::vector<int> verdict;   // per device: 0 unknown, 1 ok, 2 unsupported
+    std::lock_guard<std::mutex> g(m);
+    if ((int)verdict.size() <= dev) verdict.resize(dev + 1, 0);
+    if (verdict[dev] == 0) {
+        int major = 0, minor = 0;
+        SIEVE_CUDA(cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev));
+        SIEVE_CUDA(cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev));
+        verdict[dev] = (major == 10 && minor == 3) ? 1 : 2;
+    }
+    return verdict[dev] == 1 ? SIEVE_OK : SIEVE_EUNSUPPORTED;
+}
+
+sieve_status check_index(const sieve_index_view *ix, bool need_centroids) {
+    if (!ix) return SIEVE_EINVAL;
+    if (ix->n < 0 || ix->nlist < 1 || ix->nlist > INT32_MAX) return SIEVE_EINVAL;
+    if (ix->d < 4 || ix->d > kMaxD || ix->d % 4) return SIEVE_EINVAL;
+    if (!ix->list_offsets) return SIEVE_EINVAL;
+    if (ix->n > 0 && (!ix->vectors || !ix->ids || !aligned16(ix->vectors))) return SIEVE_EINVAL;
+    if (need_centroids && (!ix->centroids || !aligned16(ix->centroids))) return SIEVE_EINVAL;
+    return SIEVE_OK;
+}
+
+sieve_status check_params(const sieve_index_view *ix, const sieve_params *p) {
+    if (!p) return SIEVE_EINVAL;
+    if (p->tau != p->tau) return SIEVE_EINVAL;   // NaN
+    if (p->k < 1 || p->k > kMaxK) return SIEVE_EINVAL;
+    if (p->nprobe < 1 || p->nprobe > kMaxNprobe || p->nprobe > ix->nlist) return SIEVE_EINVAL;
+    if (p->W < 1) return SIEVE_EINVAL;
+    if (p->lookahead != 0 && p->lookahead != 1) return SIEVE_EINVAL;
+    if (p->loop != 0 && p->loop != 1) return SIEVE_EINVAL;
+    if (p->max_items_per_round < 0) return SIEVE_EINVAL;
+    if (p->profile != 0 && p->profile != 1) return SIEVE_EINVAL;
+    if (p->reserved0 != 0) return SIEVE_EINVAL;
+    return SIEVE_OK;
+}
+
+constexpr int64_t kAutoCapMax = int64_t(1) << 24;
+constexpr int64_t kCapMax = int64_t(1) << 30;
+
+int64_t items_cap(int64_t nq, const sieve_params *p) {
+    const int64_t per = p->lookahead ? std::min<int64_t>(p->W, p->nprobe) : 1;
+    const int64_t most = std::max<int64_t>(1, nq * (p->lookahead ? p->nprobe : 1));
+    int64_t cap = p->max_items_per_round > 0 ? p->max_items_per_round
+                                             : std::min<int64_t>(nq * per, kAutoCapMax);
+    cap = std::min(cap, most);
+    cap = std::min(cap, kCapMax);
+    return std::max<int64_t>(cap, 1);
+}
+
+// Byte layout of the search workspace.
+struct Layout {
+    size_t ctl, order, S, E, counts, cursor, item_q, item_rank, item_p, bucketed, tiles, active,
+        res_cnt, res_s, res_id;
+    size_t h_Q, h_qids, h_ids, h_scores, h_count, h_probes;
+    size_t total;
+    int64_t cap, max_tiles;
+};
+
+Layout make_layout(const sieve_index_view *ix, int64_t nq, const sieve_params *p, bool host_io) {
+    Layout L{};
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        size_t at = off;
+        off += (size_t)round_up((int64_t)std::max<size_t>(bytes, 1), 256);
+        return at;
+    };
+    const int64_t cap = items_cap(nq, p);
+    const int64_t max_tiles = ceil_div(cap, QT) + ix->nlist + 1;
+    L.cap = cap;
+    L.max_tiles = max_tiles;
+    L.ctl = take(sizeof(Ctl));
+    L.order = take((size_t)nq * p->nprobe * 4);
+    L.S = take((size_t)nq * 4);
+    L.E = take((size_t)nq * 4);
+    L.counts = take((size_t)ix->nlist * 4);
+    L.cursor = take((size_t)ix->nlist * 4);
+    L.item_q = take((size_t)cap * 4);
+    L.item_rank = take((size_t)cap * 4);
+    L.item_p = take((size_t)cap * 4);
+    L.bucketed = take((size_t)cap * 4);
+    L.tiles = take((size_t)max_tiles * 16);
+    L.active = take((size_t)nq * 16);
+    L.res_cnt = take((size_t)cap * 4);
+    L.res_s = take((size_t)cap * p->k * 4);
+    L.res_id = take((size_t)cap * p->k * 8);
+    if (host_io) {
+        L.h_Q = take((size_t)nq * ix->d * 4);
+        L.h_qids = take((size_t)nq * 8);
+        L.h_ids = take((size_t)nq * p->k * 8);
+        L.h_scores = take((size_t)nq * p->k * 4);
+        L.h_count = take((size_t)nq * 4);
+        L.h_probes = take((size_t)nq * 4);
+    }
+    L.total = off;
+    return L;
+}
+
+// ---------------------------------------------------------------------------
+// CUDA-graph cache: one instantiated graph per distinct argument set (the
+// graph bakes every pointer and size in; replaying it for identical arguments
+// is exactly what a fresh build would do).
+struct GraphKey {
+    SearchArgs a;
+    int device;
+    int with_rank;
+    size_t scan_smem;
+    int scan_blocks;
+    bool operator==(const GraphKey &o) const { return std::memcmp(this, &o, sizeof(*this)) == 0; }
+};
+
+struct GraphEntry {
+    GraphKey key;
+    cudaGraph_t graph;
+    cudaGraphExec_t exec;
+    uint64_t last_use;
+};
+
+std::mutex g_graph_mu;
+std::vector<GraphEntry> g_graphs;
+uint64_t g_graph_clock = 0;
+constexpr size_t kGraphCacheMax = 8;
+
+sieve_status build_graph(const GraphKey &key, cudaGraph_t *g_out, cudaGraphExec_t *exec_out) {
+    const SearchArgs &a = key.a;
+    cudaStream_t cs = nullptr;
+    SIEVE_CUDA(cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking));
+    cudaGraph_t g = nullptr;
+    cudaError_t e = cudaSuccess;
+    cudaGraphConditionalHandle cond = 0;
+    cudaGraphNodeParams np{};
+    cudaGraphNode_t wnode = nullptr;
+    do {
+        // outer graph: [rank] -> init -> WHILE(rounds) -> finalize
+        if ((e = cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal)) != cudaSuccess) break;
+        if (key.with_rank)
+            e = enqueue_rank(a.Q, a.nq, a.C, a.nlist, a.d, a.nprobe, const_cast<int32_t *>(a.order),
+                             nullptr, cs);
+        if (e == cudaSuccess) e = launch_init(a, cs);
+        cudaStreamCaptureStatus cst;
+        cudaGraph_t cg = nullptr;
+        const cudaGraphNode_t *deps = nullptr;
+        size_t ndeps = 0;
+        if (e == cudaSuccess)
+            e = cudaStreamGetCaptureInfo(cs, &cst, nullptr, &cg, &deps, nullptr, &ndeps);
+        if (e == cudaSuccess)
+            e = cudaGraphConditionalHandleCreate(&cond, cg, 1, cudaGraphCondAssignDefault);
+        if (e == cudaSuccess) {
+            np.type = cudaGraphNodeTypeConditional;
+            np.conditional.handle = cond;
+            np.conditional.type = cudaGraphCondTypeWhile;
+            np.conditional.size = 1;
+            e = cudaGraphAddNode(&wnode, cg, deps, nullptr, ndeps, &np);
+        }
+        if (e == cudaSuccess)
+            e = cudaStreamUpdateCaptureDependencies(cs, &wnode, nullptr, 1,
+                                                    cudaStreamSetCaptureDependencies);
+        if (e == cudaSuccess) e = launch_finalize(a, cs);
+        cudaError_t e2 = cudaStreamEndCapture(cs, &g);
+        if (e == cudaSuccess) e = e2;
+        if (e != cudaSuccess) break;
+        // loop body: one round
+        cudaGraph_t body = np.conditional.phGraph_out[0];
+        if ((e = cudaStreamBeginCaptureToGraph(cs, body, nullptr, nullptr, 0,
+                                               cudaStreamCaptureModeThreadLocal)) != cudaSuccess)
+            break;
+        e = launch_round(a, key.scan_smem, key.scan_blocks, cond, 1, cs);
+        e2 = cudaStreamEndCapture(cs, &body);
+        if (e == cudaSuccess) e = e2;
+        if (e != cudaSuccess) break;
+        e = cudaGraphInstantiate(exec_out, g, 0);
+    } while (0);
+    cudaStreamDestroy(cs);
+    if (e != cudaSuccess) {
+        if (g) cudaGraphDestroy(g);
+        return cuda_fail(e);
+    }
+    *g_out = g;
+    return SIEVE_OK;
+}
+
+sieve_status run_graph(const GraphKey &key, cudaStream_t st) {
+    std::lock_guard<std::mutex> lk(g_graph_mu);
+    GraphEntry *hit = nullptr;
+    for (auto &ge : g_graphs)
+        if (ge.key == key) hit = &ge;
+    if (!hit) {
+        if (g_graphs.size() >= kGraphCacheMax) {
+            size_t victim = 0;
+            for (size_t i = 1; i < g_graphs.size(); ++i)
+                if (g_graphs[i].last_use < g_graphs[victim].last_use) victim = i;
+            cudaGraphExecDestroy(g_graphs[victim].exec);
+            cudaGraphDestroy(g_graphs[victim].graph);
+            g_graphs.erase(g_graphs.begin() + victim);
+        }
+        GraphEntry ge{};
+        ge.key = key;
+        sieve_status rc = build_graph(key, &ge.graph, &ge.exec);
+        if (rc != SIEVE_OK) return rc;
+        g_graphs.push_back(ge);
+        hit = &g_graphs.back();
+    }
+    hit->last_use = ++g_graph_clock;
+    SIEVE_CUDA(cudaGraphLaunch(hit->exec, st));
+    return SIEVE_OK;
+}
+
+// 14 CUDA events: 12 around the six kernels of a round, 2 for single launches
+struct EventSet {
+    cudaEvent_t e[14] = {};
+    cudaError_t create() {
+        for (auto &x : e) {
+            cudaError_t r = cudaEventCreate(&x);
+            if (r != cudaSuccess) return r;
+        }
+        return cudaSuccess;
+    }
+    ~EventSet() {
+        for (auto &x : e)
+            if (x) cudaEventDestroy(x);
+    }
+};
+
+// the device-side search on device buffers (shared by sieve_search and
+// sieve_search_host); arguments already checked
+sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t nq,
+                           const int64_t *qids, const int32_t *order, const sieve_params *p,
+                           int64_t *out_ids, float *out_scores, int32_t *out_count,
+                           int32_t *out_probes, sieve_stats *stats, unsigned char *ws,
+                           const Layout &L, cudaStream_t st) {
+    SearchArgs a;
+    std::memset(&a, 0, sizeof(a));   // padding takes part in the graph-cache key
+    a.X = ix->vectors;
+    a.ids = ix->ids;
+    a.off = ix->list_offsets;
+    a.C = ix->centroids;
+    a.n = ix->n;
+    a.nlist = ix->nlist;
+    a.d = ix->d;
+    a.Q = Q;
+    a.qids = qids;
+    a.order = order ? order : reinterpret_cast<const int32_t *>(ws + L.order);
+    a.nq = nq;
+    a.tau = p->tau;
+    a.k = p->k;
+    a.nprobe = p->nprobe;
+    a.W = p->W;
+    a.lookahead = p->lookahead;
+    a.cap = L.cap;
+    a.max_rounds = (int)std::min<int64_t>(INT32_MAX, p->nprobe + ceil_div(nq * p->nprobe, L.cap) + 2);
+    a.S = reinterpret_cast<int *>(ws + L.S);
+    a.E = reinterpret_cast<int *>(ws + L.E);
+    a.item_q = reinterpret_cast<int *>(ws + L.item_q);
+    a.item_rank = reinterpret_cast<int *>(ws + L.item_rank);
+    a.item_p = reinterpret_cast<int *>(ws + L.item_p);
+    a.counts = reinterpret_cast<int *>(ws + L.counts);
+    a.cursor = reinterpret_cast<int *>(ws + L.cursor);
+    a.bucketed = reinterpret_cast<int *>(ws + L.bucketed);
+    a.tiles = reinterpret_cast<int4 *>(ws + L.tiles);
+    a.active = reinterpret_cast<int4 *>(ws + L.active);
+    a.res_cnt = reinterpret_cast<int *>(ws + L.res_cnt);
+    a.res_s = reinterpret_cast<float *>(ws + L.res_s);
+    a.res_id = reinterpret_cast<long long *>(ws + L.res_id);
+    a.out_ids = reinterpret_cast<long long *>(out_ids);
+    a.out_scores = out_scores;
+    a.out_count = out_count;
+    a.out_probes = out_probes;
+    a.ctl = reinterpret_cast<Ctl *>(ws + L.ctl);
+
+    const bool with_rank = order == nullptr;
+    const size_t smem = scan_smem_bytes(ix->d, p->k);
+    SIEVE_CUDA(prepare_scan_kernel(smem));
+    if (with_rank) SIEVE_CUDA(prepare_rank(p->nprobe));
+    const int blocks = scan_blocks_for(smem);
+
+    float ms[SIEVE_NKERNELS] = {0};
+    if (p->loop == 0 && !p->profile) {
+        GraphKey key;
+        std::memset(&key, 0, sizeof(key));
+        key.a = a;
+        SIEVE_CUDA(cudaGetDevice(&key.device));
+        key.with_rank = with_rank;
+        key.scan_smem = smem;
+        key.scan_blocks = blocks;
+        sieve_status rc = run_graph(key, st);
+        if (rc != SIEVE_OK) return rc;
+    } else {
+        // host-driven rounds; with profile = 1 every launch is bracketed by
+        // CUDA events recorded on the launch stream
+        EventSet ev;
+        if (p->profile) SIEVE_CUDA(ev.create());
+        auto timed = [&](int slot, auto &&launch) -> cudaError_t {
+            if (p->profile) cudaEventRecord(ev.e[12], st);
+            cudaError_t e = launch();
+            if (p->profile) {
+                cudaEventRecord(ev.e[13], st);
+                cudaEventSynchronize(ev.e[13]);
+                float t = 0.f;
+                cudaEventElapsedTime(&t, ev.e[12], ev.e[13]);
+                ms[slot] += t;
+            }
+            return e;
+        };
+        if (with_rank)
+            SIEVE_CUDA(timed(SIEVE_K_RANK, [&] {
+                return enqueue_rank(Q, nq, ix->centroids, ix->nlist, ix->d, p->nprobe,
+                                    const_cast<int32_t *>(a.order), nullptr, st);
+            }));
+        SIEVE_CUDA(timed(SIEVE_K_INIT, [&] { return launch_init(a, st); }));
+        for (;;) {
+            SIEVE_CUDA(launch_round(a, smem, blocks, 0, 0, st, p->profile ? ev.e : nullptr));
+            int more = 0;
+            SIEVE_CUDA(cudaMemcpyAsync(&more, &a.ctl->more, sizeof(int), cudaMemcpyDeviceToHost, st));
+            SIEVE_CUDA(cudaStreamSynchronize(st));
+            if (p->profile) {
+                const int slot[6] = {SIEVE_K_ISSUE, SIEVE_K_BUCKET, SIEVE_K_SCATTER, SIEVE_K_SCAN,
+                                     SIEVE_K_MERGE, SIEVE_K_ROUND_END};
+                for (int i = 0; i < 6; ++i) {
+                    float t = 0.f;
+                    SIEVE_CUDA(cudaEventElapsedTime(&t, ev.e[2 * i], ev.e[2 * i + 1]));
+                    ms[slot[i]] += t;
+                }
+            }
+            if (!more) break;
+        }
+        SIEVE_CUDA(timed(SIEVE_K_FINALIZE, [&] { return launch_finalize(a, st); }));
+    }
+    if (stats) {
+        Ctl c;
+        SIEVE_CUDA(cudaMemcpyAsync(&c, a.ctl, sizeof(Ctl), cudaMemcpyDeviceToHost, st));
+        SIEVE_CUDA(cudaStreamSynchronize(st));
+        stats->rounds = c.round;
+        stats->items = (int64_t)c.tot_items;
+        stats->groups = (int64_t)c.tot_groups;
+        stats->tiles = (int64_t)c.tot_tiles;
+        stats->rows_read = (int64_t)c.tot_rows;
+        stats->pairs = (int64_t)c.tot_pairs;
+        stats->status = c.status;
+        stats->reserved0 = 0;
+        for (int i = 0; i < SIEVE_NKERNELS; ++i) stats->kernel_ms[i] = ms[i];
+        const int per_round[] = {SIEVE_K_ISSUE, SIEVE_K_BUCKET, SIEVE_K_SCATTER, SIEVE_K_SCAN,
+                                 SIEVE_K_MERGE, SIEVE_K_ROUND_END};
+        stats->kernel_launches[SIEVE_K_RANK] = with_rank ? 1 : 0;
+        stats->kernel_launches[SIEVE_K_INIT] = 1;
+        stats->kernel_launches[SIEVE_K_FINALIZE] = 1;
+        for (int slot : per_round) stats->kernel_launches[slot] = c.round;
+        if (c.status != 0) return c.status;
+    }
+    return SIEVE_OK;
+}
+
+sieve_status check_search(const sieve_index_view *ix, const float *Q, int64_t nq,
+                          const int32_t *order, const sieve_params *p, const void *o1,
+                          const void *o2, const void *o3, const void *o4) {
+    sieve_status rc = check_index(ix, order == nullptr);
+    if (rc != SIEVE_OK) return rc;
+    if ((rc = check_params(ix, p)) != SIEVE_OK) return rc;
+    if (nq < 0 || nq > INT32_MAX / 2) return SIEVE_EINVAL;
+    if (nq > 0 && (!Q || !o1 || !o2 || !o3 || !o4)) return SIEVE_EINVAL;
+    return SIEVE_OK;
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+extern "C" {
+
+const char *sieve_version(void) { return "libsieve 0.1 (sm_103a)"; }
+
+int32_t sieve_last_cuda_error(void) { return g_last_cuda_error; }
+
+const char *sieve_status_str(sieve_status s) {
+    switch (s) {
+        case SIEVE_OK: return "ok";
+        case SIEVE_EINVAL: return "invalid argument";
+        case SIEVE_ECUDA: return "CUDA error";
+        case SIEVE_EWORKSPACE: return "workspace too small or misaligned";
+        case SIEVE_ELIMIT: return "round limit reached";
+        case SIEVE_EUNSUPPORTED: return "unsupported device (needs sm_103)";
+        default: return "unknown status";
+    }
+}
+
+sieve_status sieve_layout_workspace_size(int64_t n, int64_t nlist, size_t *bytes) {
+    if (!bytes || n < 0 || nlist < 1) return SIEVE_EINVAL;
+    *bytes = layout_workspace_bytes(n, nlist);
+    return SIEVE_OK;
+}
+
+sieve_status sieve_build_layout(const float *X, const int32_t *assign, int64_t n, int32_t d,
+                                int64_t nlist, float *X_sorted, int64_t *ids_sorted,
+                                int64_t *list_offsets, void *ws, size_t ws_bytes, void *stream) {
+    if (n < 0 || nlist < 1 || nlist > INT32_MAX || d < 4 || d % 4 || d > kMaxD) return SIEVE_EINVAL;
+    if (!list_offsets) return SIEVE_EINVAL;
+    if (n > 0 && (!X || !assign || !X_sorted || !ids_sorted || !aligned16(X) || !aligned16(X_sorted)))
+        return SIEVE_EINVAL;
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u)) return SIEVE_EWORKSPACE;
+    if (ws_bytes < layout_workspace_bytes(n, nlist)) return SIEVE_EWORKSPACE;
+    sieve_status rc = check_device();
+    if (rc != SIEVE_OK) return rc;
+    int bad = 0;
+    SIEVE_CUDA(launch_layout(X, assign, n, d, nlist, X_sorted, ids_sorted, list_offsets, ws, &bad,
+                             static_cast<cudaStream_t>(stream)));
+    return bad ? SIEVE_EINVAL : SIEVE_OK;
+}
+
+sieve_status sieve_rank_partitions(const sieve_index_view *ix, const float *Q, int64_t nq,
+                                   int32_t nprobe, int32_t *order, float *cscores, void *ws,
+                                   size_t ws_bytes, void *stream) {
+    (void)ws;
+    (void)ws_bytes;
+    sieve_status rc = check_index(ix, true);
+    if (rc != SIEVE_OK) return rc;
+    if (nprobe < 1 || nprobe > kMaxNprobe || nprobe > ix->nlist) return SIEVE_EINVAL;
+    if (nq < 0 || nq > INT32_MAX / 2) return SIEVE_EINVAL;
+    if (nq > 0 && (!Q || !order || !aligned16(Q))) return SIEVE_EINVAL;
+    if ((rc = check_device()) != SIEVE_OK) return rc;
+    if (nq == 0) return SIEVE_OK;
+    SIEVE_CUDA(prepare_rank(nprobe));
+    SIEVE_CUDA(enqueue_rank(Q, nq, ix->centroids, ix->nlist, ix->d, nprobe, order, cscores,
+                            static_cast<cudaStream_t>(stream)));
+    return SIEVE_OK;
+}
+
+sieve_status sieve_search_workspace_size(const sieve_index_view *ix, int64_t nq,
+                                         const sieve_params *p, int32_t host_io, size_t *bytes) {
+    if (!bytes) return SIEVE_EINVAL;
+    sieve_status rc = check_index(ix, false);
+    if (rc != SIEVE_OK) return rc;
+    if ((rc = check_params(ix, p)) != SIEVE_OK) return rc;
+    if (nq < 0 || nq > INT32_MAX / 2) return SIEVE_EINVAL;
+    *bytes = make_layout(ix, nq, p, host_io != 0).total;
+    return SIEVE_OK;
+}
+
+sieve_status sieve_search(const sieve_index_view *ix, const float *Q, int64_t nq,
+                          const int64_t *query_ids, const int32_t *order, const sieve_params *p,
+                          int64_t *out_ids, float *out_scores, int32_t *out_count,
+                          int32_t *out_probes, sieve_stats *stats, void *ws, size_t ws_bytes,
+                          void *stream) {
+    sieve_status rc = check_search(ix, Q, nq, order, p, out_ids, out_scores, out_count, out_probes);
+    if (rc != SIEVE_OK) return rc;
+    if (nq > 0 && !aligned16(Q)) return SIEVE_EINVAL;
+    if (p->profile && !stats) return SIEVE_EINVAL;
+    if ((rc = check_device()) != SIEVE_OK) return rc;
+    if (stats) std::memset(stats, 0, sizeof(*stats));
+    if (nq == 0) return SIEVE_OK;
+    const Layout L = make_layout(ix, nq, p, false);
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < L.total)
+        return SIEVE_EWORKSPACE;
+    return search_device(ix, Q, nq, query_ids, order, p, out_ids, out_scores, out_count,
+                         out_probes, stats, static_cast<unsigned char *>(ws), L,
+                         static_cast<cudaStream_t>(stream));
+}
+
+sieve_status sieve_search_host(const sieve_index_view *ix, const float *Q_host, int64_t nq,
+                               const int64_t *query_ids_host, const sieve_params *p,
+                               int64_t *out_ids_host, float *out_scores_host,
+                               int32_t *out_count_host, int32_t *out_probes_host,
+                               sieve_stats *stats, void *ws, size_t ws_bytes, void *stream) {
+    sieve_status rc = check_search(ix, Q_host, nq, nullptr, p, out_ids_host, out_scores_host,
+                                   out_count_host, out_probes_host);
+    if (rc != SIEVE_OK) return rc;
+    if (p->profile && !stats) return SIEVE_EINVAL;
+    if ((rc = check_device()) != SIEVE_OK) return rc;
+    if (stats) std::memset(stats, 0, sizeof(*stats));
+    if (nq == 0) return SIEVE_OK;
+    const Layout L = make_layout(ix, nq, p, true);
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < L.total)
+        return SIEVE_EWORKSPACE;
+    unsigned char *w = static_cast<unsigned char *>(ws);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    float *dQ = reinterpret_cast<float *>(w + L.h_Q);
+    int64_t *dqids = query_ids_host ? reinterpret_cast<int64_t *>(w + L.h_qids) : nullptr;
+    int64_t *dids = reinterpret_cast<int64_t *>(w + L.h_ids);
+    float *dsc = reinterpret_cast<float *>(w + L.h_scores);
+    int32_t *dcnt = reinterpret_cast<int32_t *>(w + L.h_count);
+    int32_t *dpr = reinterpret_cast<int32_t *>(w + L.h_probes);
+    SIEVE_CUDA(cudaMemcpyAsync(dQ, Q_host, (size_t)nq * ix->d * 4, cudaMemcpyHostToDevice, st));
+    if (dqids)
+        SIEVE_CUDA(cudaMemcpyAsync(dqids, query_ids_host, (size_t)nq * 8, cudaMemcpyHostToDevice, st));
+    rc = search_device(ix, dQ, nq, dqids, nullptr, p, dids, dsc, dcnt, dpr, stats, w, L, st);
+    if (rc != SIEVE_OK) return rc;
+    SIEVE_CUDA(cudaMemcpyAsync(out_ids_host, dids, (size_t)nq * p->k * 8, cudaMemcpyDeviceToHost, st));
+    SIEVE_CUDA(cudaMemcpyAsync(out_scores_host, dsc, (size_t)nq * p->k * 4, cudaMemcpyDeviceToHost, st));
+    SIEVE_CUDA(cudaMemcpyAsync(out_count_host, dcnt, (size_t)nq * 4, cudaMemcpyDeviceToHost, st));
+    SIEVE_CUDA(cudaMemcpyAsync(out_probes_host, dpr, (size_t)nq * 4, cudaMemcpyDeviceToHost, st));
+    SIEVE_CUDA(cudaStreamSynchronize(st));
+    return SIEVE_OK;
+}
+
+}  // extern "C"

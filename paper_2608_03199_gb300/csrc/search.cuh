@@ -1,0 +1,72 @@
+// search.cuh -- arguments and launchers of the search rounds (internal).
+#pragma once
+
+#include <algorithm>
+
+#include "common.cuh"
+
+namespace sieve {
+
+// Everything the round kernels read or write.  Device pointers.
+struct SearchArgs {
+    // index
+    const float *X;            // [n][d] partition-contiguous rows
+    const int64_t *ids;        // [n]
+    const int64_t *off;        // [nlist+1]
+    const float *C;            // [nlist][d] centroids (ranking inside the call)
+    int64_t n;
+    int64_t nlist;
+    int d;
+    // queries
+    const float *Q;            // [nq][d]
+    const int64_t *qids;       // [nq] or nullptr
+    const int32_t *order;      // [nq][nprobe]
+    int64_t nq;
+    // parameters
+    float tau;
+    int k, nprobe, W, lookahead;
+    int64_t cap;               // items per round
+    int max_rounds;
+    // per-query state: stop line S (Sec. 4.3) and enqueue cursor E (first
+    // rank not yet issued), 1-based ranks
+    int *S, *E;
+    // per-round ready queue
+    int *item_q, *item_rank, *item_p;   // [cap]
+    int *counts, *cursor;               // [nlist]
+    int *bucketed;                      // [cap]
+    int4 *tiles;                        // [max_tiles]: partition, first bucketed slot, items
+    int4 *active;                       // [nq]: query, first item, items
+    // per-item local results
+    int *res_cnt;                       // [cap]
+    float *res_s;                       // [cap][k]
+    long long *res_id;                  // [cap][k]
+    // outputs (the running top-k lives here during the search)
+    long long *out_ids;
+    float *out_scores;
+    int *out_count, *out_probes;
+    Ctl *ctl;
+};
+
+size_t scan_smem_bytes(int d, int k);
+int num_sms();
+int scan_blocks_for(size_t smem);
+cudaError_t prepare_scan_kernel(size_t smem);
+cudaError_t launch_init(const SearchArgs &a, cudaStream_t st);
+cudaError_t launch_finalize(const SearchArgs &a, cudaStream_t st);
+cudaError_t launch_round(const SearchArgs &a, size_t scan_smem, int scan_blocks,
+                         cudaGraphConditionalHandle cond, int use_cond, cudaStream_t st,
+                         cudaEvent_t *ev = nullptr);
+
+// centroid ranking (rank_kernel.cu): prepare_rank once before launches or
+// stream capture, then enqueue_rank (a single kernel launch)
+cudaError_t prepare_rank(int nprobe);
+cudaError_t enqueue_rank(const float *Q, int64_t nq, const float *C, int64_t nlist, int d,
+                         int nprobe, int32_t *order, float *cscores, cudaStream_t st);
+
+// partition layout (layout_kernels.cu)
+size_t layout_workspace_bytes(int64_t n, int64_t nlist);
+cudaError_t launch_layout(const float *X, const int32_t *assign, int64_t n, int d, int64_t nlist,
+                          float *X_sorted, int64_t *ids_sorted, int64_t *list_offsets, void *ws,
+                          int *bad_flag_host, cudaStream_t st);
+
+}  // namespace sieve

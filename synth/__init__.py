@@ -189,16 +189,20 @@ def build_index(X: torch.Tensor, cfg: Workload, g: torch.Generator, chunk: int =
 
 
 @torch.no_grad()
-def make_workload(cfg: Workload | str, device="cpu"):
+def make_workload(cfg: Workload | str, device="cpu", query_stream: int = 0):
     """Everything one search call needs, on ``device``.
 
     Returns a dict: X [n][d] f32, ids [n] i64 (= row), centroids [nlist][d] f32,
     assign [n] i32, Q [nq][d] f32, qids [nq] i64, and the search parameters.
+    ``query_stream`` > 0 draws an independent query batch from the same index
+    (one batch per process when queries are sharded over GPUs).
     """
     if isinstance(cfg, str):
         cfg = CONFIGS[cfg]
     X, g = make_corpus(cfg, device)
     cent, assign = build_index(X, cfg, g)
+    if query_stream:
+        g = torch.Generator(device=device).manual_seed(cfg.seed * 1_000_003 + query_stream)
     qrows = torch.randperm(cfg.n, generator=g, device=device)[:cfg.nq]
     return {
         "cfg": cfg,

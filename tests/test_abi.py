@@ -1,0 +1,59 @@
+"""The C-ABI library builds for sm_103a, loads, and exports every function that
+include/*.h declares (no compute calls: this runs without a GPU)."""
+import ctypes
+import glob
+import os
+import re
+
+import paper_2608_03199_gb300 as sieve
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_functions():
+    names = set()
+    for h in glob.glob(os.path.join(ROOT, "include", "*.h")):
+        text = open(h).read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        for m in re.finditer(r"^[A-Za-z_][\w \*]*?\b(sieve_\w+)\s*\(", text, flags=re.M):
+            names.add(m.group(1))
+    return names
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("sieve_rank_partitions", "sieve_search", "sieve_search_host",
+                     "sieve_build_layout", "sieve_search_workspace_size", "sieve_status_str"):
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol():
+    path = sieve.build()
+    lib = ctypes.CDLL(path)
+    missing = [n for n in declared_functions() if not hasattr(lib, n)]
+    assert not missing, missing
+    assert set(declared_functions()) <= set(sieve._SIGNATURES), "binding lacks a declared call"
+
+
+def test_host_only_calls_without_gpu():
+    lib = sieve.lib()
+    assert lib.sieve_version().startswith(b"libsieve")
+    assert lib.sieve_status_str(-1) == b"invalid argument"
+    n = ctypes.c_size_t()
+    assert lib.sieve_layout_workspace_size(1000, 16, ctypes.byref(n)) == 0 and n.value > 0
+    assert lib.sieve_layout_workspace_size(-1, 16, ctypes.byref(n)) == -1
+    v = sieve.IndexViewC(n=1000, nlist=16, d=64, vectors=16, ids=16, list_offsets=16, centroids=16)
+    p = sieve._params(0.9, 10, 8, 4, True, 0, 0)
+    assert lib.sieve_search_workspace_size(ctypes.byref(v), 100, ctypes.byref(p), 0,
+                                           ctypes.byref(n)) == 0
+    small = n.value
+    assert lib.sieve_search_workspace_size(ctypes.byref(v), 100, ctypes.byref(p), 1,
+                                           ctypes.byref(n)) == 0 and n.value > small
+    for bad in (sieve._params(0.9, 0, 8, 4, True, 0, 0), sieve._params(0.9, 65, 8, 4, True, 0, 0),
+                sieve._params(0.9, 10, 17, 4, True, 0, 0), sieve._params(0.9, 10, 8, 0, True, 0, 0),
+                sieve._params(float("nan"), 10, 8, 4, True, 0, 0)):
+        assert lib.sieve_search_workspace_size(ctypes.byref(v), 100, ctypes.byref(bad), 0,
+                                               ctypes.byref(n)) == -1
+    v.d = 62
+    assert lib.sieve_search_workspace_size(ctypes.byref(v), 100, ctypes.byref(p), 0,
+                                           ctypes.byref(n)) == -1

@@ -1,0 +1,84 @@
+"""Parity at the benchmark's full size (1M x 256 rows, 1,024 partitions, 100K
+queries, tau 0.90, k 10, nprobe 64, W 8, lookahead on) in the launch
+configuration ``bench.py`` times.
+
+The whole batch runs on the GPU; the oracle recomputes a seeded sample of the
+queries one by one (per-query results do not depend on the batch, Sec. 4.3),
+and properties that hold at any size are checked on every query."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2608_03199_gb300 as sieve
+import synth
+from parity import assert_parity, compare
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def full():
+    assert torch.cuda.is_available()
+    dev = torch.device("cuda:0")
+    cfg = synth.CONFIGS["1m"]
+    wl = synth.make_workload(cfg, device=dev)
+    index = sieve.build_layout(wl["X"], wl["assign"], cfg.nlist, wl["centroids"])
+    host = {k: wl[k].cpu().numpy() for k in ("X", "ids", "assign", "centroids", "Q", "qids")}
+    return cfg, wl, index, host
+
+
+def _np(out):
+    return {"ids": out[0].cpu().numpy(), "scores": out[1].cpu().numpy(),
+            "count": out[2].cpu().numpy(), "probes": out[3].cpu().numpy()}
+
+
+def test_full_size_sampled_parity(full):
+    cfg, wl, index, h = full
+    out = sieve.search(index, wl["Q"], cfg.tau, cfg.k, cfg.nprobe, cfg.W, lookahead=True,
+                       query_ids=wl["qids"], stats=True)
+    got, st = _np(out), out[4]
+    assert st["status"] == 0
+    assert st["items"] == got["probes"].sum()
+    assert ((got["probes"] >= cfg.W) & (got["probes"] <= cfg.nprobe)).all()
+    rng = np.random.default_rng(1234)
+    sample = np.sort(rng.choice(cfg.nq, 1500, replace=False))
+    idx = {k: h[k] for k in ("X", "ids", "assign", "centroids")}
+    Q, qids = h["Q"][sample], h["qids"][sample]
+    ref = oracle.search(idx, Q, cfg.tau, cfg.k, cfg.nprobe, cfg.W, qids=qids)
+    order = oracle.rank(Q, h["centroids"], cfg.nprobe)
+    rep = compare({k: v[sample] for k, v in got.items()}, ref, idx, Q, qids, cfg.tau, cfg.k,
+                  cfg.nprobe, order)
+    assert_parity(rep)
+    # sorted output rows, padding
+    valid = np.arange(cfg.k)[None, :] < got["count"][:, None]
+    sc = got["scores"]
+    assert ((sc[:, 1:] <= sc[:, :-1]) | ~valid[:, 1:]).all()
+    assert ((got["ids"] == -1) == ~valid).all()
+    assert (got["scores"][valid] >= np.float32(cfg.tau)).all()
+
+
+def test_full_size_schedule_invariance_and_fixed_probe(full):
+    cfg, wl, index, h = full
+    a = _np(sieve.search(index, wl["Q"], cfg.tau, cfg.k, cfg.nprobe, cfg.W, lookahead=True,
+                         query_ids=wl["qids"]))
+    b = _np(sieve.search(index, wl["Q"], cfg.tau, cfg.k, cfg.nprobe, cfg.W, lookahead=False,
+                         query_ids=wl["qids"]))
+    c = _np(sieve.search(index, wl["Q"], cfg.tau, cfg.k, cfg.nprobe, cfg.W, lookahead=True,
+                         query_ids=wl["qids"], max_items_per_round=65536))
+    for key in a:
+        assert np.array_equal(a[key], b[key]) and np.array_equal(a[key], c[key]), key
+    fx = _np(sieve.search(index, wl["Q"], cfg.tau, cfg.k, cfg.nprobe, cfg.nprobe, lookahead=True,
+                          query_ids=wl["qids"]))
+    assert (fx["probes"] == cfg.nprobe).all()
+    # fixed probe sees a superset of partitions: it never returns fewer results
+    assert (fx["count"] >= a["count"]).all()
+    sample = np.arange(0, cfg.nq, 400)
+    idx = {k: h[k] for k in ("X", "ids", "assign", "centroids")}
+    Q, qids = h["Q"][sample], h["qids"][sample]
+    order = oracle.rank(Q, h["centroids"], cfg.nprobe)
+    ref = oracle.fixed_probe(idx, Q, cfg.tau, cfg.k, cfg.nprobe, order, qids=qids)
+    ref["probes"] = np.full(len(sample), cfg.nprobe, np.int32)
+    rep = compare({k: v[sample] for k, v in fx.items()}, ref, idx, Q, qids, cfg.tau, cfg.k,
+                  cfg.nprobe, order)
+    assert_parity(rep)

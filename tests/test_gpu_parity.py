@@ -1,0 +1,254 @@
+"""Parity of the CUDA path (through the C ABI) with the fp64 oracle.
+
+Element by element on seeded inputs that span many tiles with ragged tails:
+probe counts, result ids and counts identical (up to the counted, tagged
+rounding divergences of ``parity.py``), scores within 1e-5.  Also the
+invariances the paper fixes (lookahead / per-round caps / loop mode change
+nothing, Sec. 4.2-4.3; W >= nprobe is fixed probing; nprobe = nlist with
+W = infinity is brute force) and the edge cases of the boundary.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2608_03199_gb300 as sieve
+from conftest import index_of
+from parity import TOL, assert_parity, compare
+
+pytestmark = pytest.mark.gpu
+
+BIG_W = 2**31 - 1
+
+
+@pytest.fixture(scope="module")
+def dev():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    return torch.device("cuda:0")
+
+
+def gpu_index(w, dev):
+    X = torch.from_numpy(w["X"]).to(dev)
+    assign = torch.from_numpy(w["assign"]).to(dev)
+    cent = torch.from_numpy(w["centroids"]).to(dev)
+    return sieve.build_layout(X, assign, cent.shape[0], cent)
+
+
+@pytest.fixture(scope="module")
+def g_tiny(tiny, dev):
+    return gpu_index(tiny, dev)
+
+
+@pytest.fixture(scope="module")
+def g_deep(deep, dev):
+    return gpu_index(deep, dev)
+
+
+def run(index, Q, qids, tau, k, nprobe, W, **kw):
+    dev = index.vectors.device
+    Qd = torch.from_numpy(np.ascontiguousarray(Q)).to(dev)
+    qd = None if qids is None else torch.from_numpy(np.ascontiguousarray(qids)).to(dev)
+    out = sieve.search(index, Qd, tau, k, nprobe, W, query_ids=qd, **kw)
+    torch.cuda.synchronize()
+    res = {"ids": out[0].cpu().numpy(), "scores": out[1].cpu().numpy(),
+           "count": out[2].cpu().numpy(), "probes": out[3].cpu().numpy()}
+    if kw.get("stats"):
+        res["stats"] = out[4]
+    return res
+
+
+def check(w, gidx, Q, qids, tau, k, nprobe, W, lookahead, **kw):
+    ref = oracle.search(index_of(w), Q, tau, k, nprobe, W, qids=qids)
+    got = run(gidx, Q, qids, tau, k, nprobe, W, lookahead=lookahead, **kw)
+    order = oracle.rank(Q, w["centroids"], nprobe)
+    rep = compare(got, ref, index_of(w), Q, qids, tau, k, nprobe, order)
+    assert_parity(rep)
+    return got, ref, rep
+
+
+# ---------------------------------------------------------------------------
+def test_layout_is_a_stable_counting_sort(tiny, g_tiny):
+    perm = np.argsort(tiny["assign"], kind="stable")
+    assert (g_tiny.ids.cpu().numpy() == perm).all()
+    assert np.array_equal(g_tiny.vectors.cpu().numpy(), tiny["X"][perm])
+    off = np.concatenate([[0], np.cumsum(np.bincount(tiny["assign"], minlength=64))])
+    assert (g_tiny.list_offsets.cpu().numpy() == off).all()
+
+
+def test_rank_parity(tiny, g_tiny, dev):
+    Q = torch.from_numpy(tiny["Q"]).to(dev)
+    for nprobe in (1, 16, 63, 64):
+        order, sc = sieve.rank_partitions(g_tiny, Q, nprobe, return_scores=True)
+        order, sc = order.cpu().numpy(), sc.cpu().numpy()
+        ref, rsc = oracle.rank(tiny["Q"], tiny["centroids"], min(nprobe + 1, 64), return_scores=True)
+        assert np.abs(sc - rsc[:, :nprobe]).max() <= TOL
+        gaps = np.diff(rsc, axis=1).__neg__().min(axis=1) if rsc.shape[1] > 1 else np.full(len(rsc), np.inf)
+        bad = (order != ref[:, :nprobe]).any(axis=1)
+        assert (gaps[bad] < TOL).all()
+        assert bad.sum() <= 2
+
+
+@pytest.mark.parametrize("lookahead", [0, 1])
+def test_search_parity_tiny(tiny, g_tiny, lookahead):
+    c = tiny["cfg"]
+    got, ref, rep = check(tiny, g_tiny, tiny["Q"], tiny["qids"], c.tau, c.k, c.nprobe, c.W,
+                          lookahead)
+    assert rep["exact"] >= 0.99 * len(tiny["Q"])
+    assert (got["count"] > 0).any()
+
+
+@pytest.mark.parametrize("W", [1, 2, 3, 5, 24])
+@pytest.mark.parametrize("lookahead", [0, 1])
+def test_search_parity_deep(deep, g_deep, W, lookahead):
+    c = deep["cfg"]
+    check(deep, g_deep, deep["Q"], deep["qids"], c.tau, c.k, c.nprobe, W, lookahead)
+
+
+def test_schedule_changes_nothing(deep, g_deep):
+    """Lookahead on/off, per-round caps and the loop mode give bit-identical
+    output (Sec. 4.2: the microbatch cap only splits groups; Sec. 4.3)."""
+    c = deep["cfg"]
+    Q, qids = deep["Q"], deep["qids"]
+    base = run(g_deep, Q, qids, c.tau, c.k, c.nprobe, c.W, lookahead=1)
+    variants = [dict(lookahead=0), dict(lookahead=1, max_items_per_round=4096),
+                dict(lookahead=1, max_items_per_round=7), dict(lookahead=0, loop=1),
+                dict(lookahead=1, loop=1, max_items_per_round=100)]
+    for kw in variants:
+        got = run(g_deep, Q, qids, c.tau, c.k, c.nprobe, c.W, **kw)
+        for key in ("ids", "scores", "count", "probes"):
+            assert np.array_equal(got[key], base[key]), (kw, key)
+    sub = slice(0, 25)   # a cap of one item per round: one search per round
+    one = run(g_deep, Q[sub], qids[sub], c.tau, c.k, c.nprobe, c.W, lookahead=1,
+              max_items_per_round=1, stats=True)
+    for key in ("ids", "scores", "count", "probes"):
+        assert np.array_equal(one[key], base[key][sub]), key
+    assert one["stats"]["rounds"] >= one["probes"].sum()
+
+
+@pytest.mark.parametrize("W", [16, BIG_W])
+def test_window_at_least_nprobe_is_fixed_probe(tiny, g_tiny, W):
+    c = tiny["cfg"]
+    got = run(g_tiny, tiny["Q"], tiny["qids"], c.tau, c.k, c.nprobe, W, lookahead=1)
+    assert (got["probes"] == c.nprobe).all()
+    order = oracle.rank(tiny["Q"], tiny["centroids"], c.nprobe)
+    fp = oracle.fixed_probe(index_of(tiny), tiny["Q"], c.tau, c.k, c.nprobe, order,
+                            qids=tiny["qids"])
+    fp["probes"] = np.full(len(order), c.nprobe, np.int32)
+    assert_parity(compare(got, fp, index_of(tiny), tiny["Q"], tiny["qids"], c.tau, c.k,
+                          c.nprobe, order))
+
+
+def test_full_probe_is_bruteforce(tiny, g_tiny):
+    c = tiny["cfg"]
+    Q, qids = tiny["Q"][:300], tiny["qids"][:300]
+    got = run(g_tiny, Q, qids, c.tau, c.k, 64, BIG_W, lookahead=1)
+    bf = oracle.bruteforce(tiny["X"], tiny["ids"], Q, c.tau, c.k, qids=qids)
+    bf["probes"] = np.full(len(Q), 64, np.int32)
+    order = oracle.rank(Q, tiny["centroids"], 64)
+    assert_parity(compare(got, bf, index_of(tiny), Q, qids, c.tau, c.k, 64, order))
+
+
+def test_given_order_and_host_variant(tiny, g_tiny, dev):
+    c = tiny["cfg"]
+    Q = torch.from_numpy(tiny["Q"]).to(dev)
+    qids = torch.from_numpy(tiny["qids"]).to(dev)
+    base = sieve.search(g_tiny, Q, c.tau, c.k, c.nprobe, c.W, query_ids=qids)
+    order = sieve.rank_partitions(g_tiny, Q, c.nprobe)
+    given = sieve.search(g_tiny, Q, c.tau, c.k, c.nprobe, c.W, query_ids=qids, order=order)
+    host = sieve.search_host(g_tiny, torch.from_numpy(tiny["Q"]).pin_memory(), c.tau, c.k,
+                             c.nprobe, c.W, query_ids_host=torch.from_numpy(tiny["qids"]))
+    for a, b, h in zip(base, given, host):
+        assert torch.equal(a.cpu(), b.cpu())
+        assert torch.equal(a.cpu(), h)
+
+
+def test_stats_account_for_the_work(deep, g_deep):
+    c = deep["cfg"]
+    got = run(g_deep, deep["Q"], deep["qids"], c.tau, c.k, c.nprobe, c.W, lookahead=0, stats=True)
+    st = got["stats"]
+    assert st["status"] == 0
+    assert st["items"] == got["probes"].sum()           # each committed rank searched once
+    assert st["rounds"] == got["probes"].max() + 0      # one rank per query per round
+    sizes = np.bincount(deep["assign"], minlength=c.nlist)
+    order = oracle.rank(deep["Q"], deep["centroids"], c.nprobe)
+    want_pairs = sum(sizes[order[i, :got["probes"][i]]].sum() for i in range(len(order)))
+    assert st["pairs"] == want_pairs
+
+
+# ---------------------------------------------------------------------------
+# edge cases
+
+
+def test_empty_and_single_query(tiny, g_tiny, dev):
+    c = tiny["cfg"]
+    empty = torch.empty((0, 64), dtype=torch.float32, device=dev)
+    ids, sc, cnt, pr = sieve.search(g_tiny, empty, c.tau, c.k, c.nprobe, c.W)
+    assert ids.shape == (0, c.k) and pr.shape == (0,)
+    check(tiny, g_tiny, tiny["Q"][:1], tiny["qids"][:1], c.tau, c.k, c.nprobe, c.W, 1)
+
+
+@pytest.mark.parametrize("k", [1, 3, 33, 64])
+def test_k_range(deep, g_deep, k):
+    c = deep["cfg"]
+    check(deep, g_deep, deep["Q"], deep["qids"], c.tau, k, c.nprobe, c.W, 1)
+
+
+def test_no_query_ids_and_low_tau(deep, g_deep):
+    c = deep["cfg"]
+    check(deep, g_deep, deep["Q"][:100], None, 0.5, c.k, 8, 2, 1)
+
+
+def _hand_index(dev, X, assign, C):
+    Xd = torch.from_numpy(np.asarray(X, np.float32)).to(dev)
+    a = torch.from_numpy(np.asarray(assign, np.int32)).to(dev)
+    Cd = torch.from_numpy(np.asarray(C, np.float32)).to(dev)
+    return sieve.build_layout(Xd, a, Cd.shape[0], Cd)
+
+
+def test_tau_boundary_self_ties_padding(dev):
+    q = np.array([[1, 0, 0, 0]], np.float32)
+    X = np.array([[0.5, 0.5, 0.5, 0.5], [0.5, 0.5, 0.5, 0.5], [1, 0, 0, 0], [0, 1, 0, 0],
+                  [0.5, -0.5, 0.5, 0.5]], np.float32)
+    # external ids are row numbers; the query is row 2
+    idx = _hand_index(dev, X, [0] * 5, q)
+    Qd = torch.from_numpy(q).to(dev)
+    ids, sc, cnt, pr = sieve.search(idx, Qd, 0.5, 4, 1, 1, query_ids=torch.tensor([2], device=dev))
+    assert cnt.item() == 3 and pr.item() == 1
+    assert ids[0].tolist() == [0, 1, 4, -1]
+    assert sc[0, :3].tolist() == [0.5, 0.5, 0.5] and sc[0, 3].item() == float("-inf")
+    above = float(np.nextafter(np.float32(0.5), np.float32(1)))
+    ids, sc, cnt, pr = sieve.search(idx, Qd, above, 4, 1, 1, query_ids=torch.tensor([2], device=dev))
+    assert cnt.item() == 0 and ids[0].tolist() == [-1] * 4
+
+
+def test_empty_partitions_and_odd_dimension(dev):
+    rng = np.random.default_rng(5)
+    d, nlist = 36, 10
+    C = rng.normal(size=(nlist, d)).astype(np.float32)
+    C /= np.linalg.norm(C, axis=1, keepdims=True)
+    X = np.repeat(C[:6], 150, axis=0) + 0.05 * rng.normal(size=(900, d)).astype(np.float32)
+    X = (X / np.linalg.norm(X, axis=1, keepdims=True)).astype(np.float32)
+    assign = np.argmax(X @ C.T, axis=1).astype(np.int32)       # partitions 6..9 stay empty
+    w = {"X": X, "ids": np.arange(900, dtype=np.int64), "assign": assign, "centroids": C}
+    gidx = _hand_index(dev, X, assign, C)
+    Q = X[::9].copy()
+    qids = np.arange(0, 900, 9, dtype=np.int64)
+    for W in (1, 3, BIG_W):
+        check(w, gidx, Q, qids, 0.9, 7, nlist, W, 1)
+
+
+def test_invalid_arguments_raise(tiny, g_tiny, dev):
+    Q = torch.from_numpy(tiny["Q"][:4]).to(dev)
+    for kw in (dict(k=0), dict(k=65), dict(nprobe=65), dict(W=0)):
+        args = dict(tau=0.9, k=10, nprobe=16, W=4)
+        args.update(kw)
+        with pytest.raises(sieve.SieveError):
+            sieve.search(g_tiny, Q, **args)
+    with pytest.raises(sieve.SieveError):
+        sieve.search(g_tiny, Q, float("nan"), 10, 16, 4)
+    tiny_ws = sieve.Workspace()
+    tiny_ws.buf = torch.empty(256, dtype=torch.uint8, device=dev)
+    tiny_ws.get = lambda n, d: tiny_ws.buf     # hand the call a too-small buffer
+    with pytest.raises(sieve.SieveError) as e:
+        sieve.search(g_tiny, Q, 0.9, 10, 16, 4, workspace=tiny_ws)
+    assert e.value.status == -3
