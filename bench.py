@@ -128,12 +128,17 @@ def measured_peaks():
         return {}
 
 
+KERNEL_SOURCES = ("common.cuh", "search.cuh", "search_kernels.cu", "rank_kernel.cu")
+
+
 def kernel_source_sha():
+    """Hash of the files that define the search kernels (not the host API)."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2608_03199_gb300", "csrc")
-    for f in sorted(os.listdir(csrc)):
-        if f.endswith((".cu", ".cuh")):
-            h.update(open(os.path.join(csrc, f), "rb").read())
+    for f in KERNEL_SOURCES:
+        p = os.path.join(csrc, f)
+        if os.path.exists(p):
+            h.update(open(p, "rb").read())
     return h.hexdigest()[:16]
 
 
@@ -147,7 +152,7 @@ def committed_traffic(kernel, workload):
     e = t.get(kernel, {}).get(workload)
     if not e or e.get("source_sha") != kernel_source_sha():
         return None
-    return e.get("dram_bytes_per_launch")
+    return {"dram_bytes_per_launch": e.get("dram_bytes_per_launch"), "launch": e.get("launch")}
 
 
 def roofline(prof, cfg, dev):
