@@ -47,6 +47,8 @@ typedef int32_t sieve_status;
 #define SIEVE_EWORKSPACE (-3)   /* ws_bytes below the size the call needs, or ws misaligned */
 #define SIEVE_ELIMIT (-4)       /* the device round loop hit its round limit (see sieve_stats) */
 #define SIEVE_EUNSUPPORTED (-5) /* the current device is not sm_103 */
+#define SIEVE_ESCRATCH (-6)     /* sieve_search_noalloc: the call needs more scratch than
+                                   SIEVE_NOALLOC_SCRATCH_BYTES */
 
 /* The IVF index, resident on the device (Sec. 2.3).  Borrowed, read-only.
  *   vectors      device [n][d] fp32, unit-norm, partition-contiguous: the rows
@@ -207,6 +209,37 @@ sieve_status sieve_search_host(const sieve_index_view *ix, const float *Q_host, 
                                int64_t *out_ids_host, float *out_scores_host,
                                int32_t *out_count_host, int32_t *out_probes_host,
                                sieve_stats *stats, void *ws, size_t ws_bytes, void *stream);
+
+/* sieve_search for callers that cannot allocate device memory at all: a host
+ * process without a device allocator, a plug-in whose host application owns
+ * every allocation, code that runs while the caller's memory pool is being
+ * reset.  The paper has no counterpart; this is a deployment convenience.
+ *
+ * Arguments and results are those of sieve_search, without the workspace.
+ * The caller still provides (and owns) every input and output buffer; the
+ * call's scratch is a fixed array of SIEVE_NOALLOC_SCRATCH_BYTES inside the
+ * library image, so every GPU that loads the library holds that memory until
+ * the process exits.  The call allocates nothing: no cudaMalloc, no CUDA
+ * graph (rounds are host-driven, one stream sync per round, whatever
+ * p->loop says), no events (p->profile must be 0).
+ *   - A call whose scratch need (sieve_search_workspace_size with
+ *     host_io = 0) exceeds SIEVE_NOALLOC_SCRATCH_BYTES returns
+ *     SIEVE_ESCRATCH and touches nothing.
+ *   - The first call on a device looks up the array's device address on that
+ *     device (cudaGetSymbolAddress); make that first call before any stream
+ *     capture begins.
+ *   - Every call on a device uses the same array and leaves its contents
+ *     behind; each call initialises what it reads.  Calls that can overlap
+ *     on the GPU (other host threads, other streams) race on the array and
+ *     must be serialized by the caller.
+ * As with sieve_search, the outputs are complete once `stream` has passed
+ * the call (the host-driven rounds synchronize `stream` on the way). */
+#define SIEVE_NOALLOC_SCRATCH_BYTES ((size_t)64 << 20)
+sieve_status sieve_search_noalloc(const sieve_index_view *ix, const float *Q, int64_t nq,
+                                  const int64_t *query_ids, const int32_t *order,
+                                  const sieve_params *p, int64_t *out_ids, float *out_scores,
+                                  int32_t *out_count, int32_t *out_probes, sieve_stats *stats,
+                                  void *stream);
 
 /* Human-readable name of a status code (static string). */
 const char *sieve_status_str(sieve_status s);

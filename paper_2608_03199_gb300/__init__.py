@@ -25,7 +25,7 @@ from . import _build
 
 SIEVE_OK = 0
 _STATUS = {0: "ok", -1: "invalid argument", -2: "CUDA error", -3: "workspace", -4: "round limit",
-           -5: "unsupported device"}
+           -5: "unsupported device", -6: "exceeds the no-allocation scratch"}
 
 
 class SieveError(RuntimeError):
@@ -82,6 +82,10 @@ _SIGNATURES = {
                                       C.POINTER(ParamsC), C.c_void_p, C.c_void_p, C.c_void_p,
                                       C.c_void_p, C.POINTER(StatsC), C.c_void_p, C.c_size_t,
                                       C.c_void_p]),
+    "sieve_search_noalloc": (C.c_int32, [C.POINTER(IndexViewC), C.c_void_p, C.c_int64,
+                                         C.c_void_p, C.c_void_p, C.POINTER(ParamsC), C.c_void_p,
+                                         C.c_void_p, C.c_void_p, C.c_void_p, C.POINTER(StatsC),
+                                         C.c_void_p]),
     "sieve_status_str": (C.c_char_p, [C.c_int32]),
     "sieve_last_cuda_error": (C.c_int32, []),
     "sieve_version": (C.c_char_p, []),
@@ -317,4 +321,33 @@ def search_host(index: Index, Q_host, tau, k, nprobe, W, lookahead=True, query_i
     _check(lib().sieve_search_host(C.byref(v), _ptr(Q_host), nq, _ptr(query_ids_host), C.byref(p),
                                    _ptr(ids), _ptr(scores), _ptr(count), _ptr(probes), None,
                                    _ptr(ws), ws.numel(), _stream(stream)), "sieve_search_host")
+    return ids, scores, count, probes
+
+
+NOALLOC_SCRATCH_BYTES = 64 << 20
+
+
+def search_noalloc(index: Index, Q, tau, k, nprobe, W, lookahead=True, query_ids=None,
+                   order=None, max_items_per_round=0, out=None, stream=None):
+    """sieve_search_noalloc: the search with no device allocation in the call.
+
+    For callers that cannot allocate device memory: the scratch is a fixed
+    array inside libsieve (NOALLOC_SCRATCH_BYTES per GPU, held until exit);
+    the caller passes the output tensors in ``out`` to keep the call itself
+    allocation-free.  Returns (ids, scores, count, probes), complete once the
+    stream has passed the call."""
+    _need_cuda(Q, torch.float32, "Q", 2)
+    nq = Q.shape[0]
+    if out is None:
+        dev = Q.device
+        out = (torch.empty((nq, k), dtype=torch.int64, device=dev),
+               torch.empty((nq, k), dtype=torch.float32, device=dev),
+               torch.empty(nq, dtype=torch.int32, device=dev),
+               torch.empty(nq, dtype=torch.int32, device=dev))
+    ids, scores, count, probes = out
+    p = _params(tau, k, nprobe, W, lookahead, 1, max_items_per_round)
+    v = index.view()
+    _check(lib().sieve_search_noalloc(C.byref(v), _ptr(Q), nq, _ptr(query_ids), _ptr(order),
+                                      C.byref(p), _ptr(ids), _ptr(scores), _ptr(count),
+                                      _ptr(probes), None, _stream(stream)), "sieve_search_noalloc")
     return ids, scores, count, probes

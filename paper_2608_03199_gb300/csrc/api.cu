@@ -408,6 +408,7 @@ const char *sieve_status_str(sieve_status s) {
         case SIEVE_EWORKSPACE: return "workspace too small or misaligned";
         case SIEVE_ELIMIT: return "round limit reached";
         case SIEVE_EUNSUPPORTED: return "unsupported device (needs sm_103)";
+        case SIEVE_ESCRATCH: return "call needs more scratch than the fixed no-allocation array";
         default: return "unknown status";
     }
 }
@@ -521,3 +522,66 @@ sieve_status sieve_search_host(const sieve_index_view *ix, const float *Q_host, 
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// sieve_search_noalloc: sieve_search for callers that cannot allocate device
+// memory at all (an allocator-free host process, a plug-in running inside a
+// host application that owns every allocation, code between a caller's own
+// pool resets).  Its scratch is the fixed array below: part of the library
+// image, so every GPU that loads the library holds it until the process
+// exits, and every call on that GPU shares it.
+namespace {
+
+constexpr size_t kNoallocScratchBytes = size_t(64) << 20;   // SIEVE_NOALLOC_SCRATCH_BYTES
+constexpr int kNoallocMaxDevices = 64;
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocScratchBytes];
+
+std::mutex g_noalloc_mu;
+void *g_noalloc_ptr[kNoallocMaxDevices] = {};
+
+// Device address of the scratch array on the current device.  Host code only
+// sees a host-side stand-in under the array's name, so the address is asked
+// of the runtime once per device (with that device current) and kept.
+sieve_status noalloc_scratch(void **out) {
+    int dev = 0;
+    SIEVE_CUDA(cudaGetDevice(&dev));
+    if (dev < 0 || dev >= kNoallocMaxDevices) return SIEVE_EUNSUPPORTED;
+    std::lock_guard<std::mutex> lk(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+        void *p = nullptr;
+        cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess || !p) return cuda_fail(e != cudaSuccess ? e : cudaErrorInvalidSymbol);
+        g_noalloc_ptr[dev] = p;
+    }
+    *out = g_noalloc_ptr[dev];
+    return SIEVE_OK;
+}
+
+}  // namespace
+
+extern "C" sieve_status sieve_search_noalloc(const sieve_index_view *ix, const float *Q,
+                                             int64_t nq, const int64_t *query_ids,
+                                             const int32_t *order, const sieve_params *p,
+                                             int64_t *out_ids, float *out_scores,
+                                             int32_t *out_count, int32_t *out_probes,
+                                             sieve_stats *stats, void *stream) {
+    sieve_status rc = check_search(ix, Q, nq, order, p, out_ids, out_scores, out_count, out_probes);
+    if (rc != SIEVE_OK) return rc;
+    if (nq > 0 && !aligned16(Q)) return SIEVE_EINVAL;
+    if (p->profile) return SIEVE_EINVAL;   // event timing is not offered here
+    if ((rc = check_device()) != SIEVE_OK) return rc;
+    if (stats) std::memset(stats, 0, sizeof(*stats));
+    if (nq == 0) return SIEVE_OK;
+    const Layout L = make_layout(ix, nq, p, false);
+    if (L.total > kNoallocScratchBytes) return SIEVE_ESCRATCH;
+    void *ws = nullptr;
+    if ((rc = noalloc_scratch(&ws)) != SIEVE_OK) return rc;
+    // host-driven rounds: building and instantiating a CUDA graph could
+    // allocate, so this entry point never does
+    sieve_params hp = *p;
+    hp.loop = 1;
+    return search_device(ix, Q, nq, query_ids, order, &hp, out_ids, out_scores, out_count,
+                         out_probes, stats, static_cast<unsigned char *>(ws), L,
+                         static_cast<cudaStream_t>(stream));
+}
