@@ -128,7 +128,8 @@ def measured_peaks():
         return {}
 
 
-KERNEL_SOURCES = ("common.cuh", "search.cuh", "search_kernels.cu", "rank_kernel.cu")
+KERNEL_SOURCES = ("common.cuh", "search.cuh", "search_kernels.cu", "rank_kernel.cu",
+                  "scan_tc.cu", "tcgen05.cuh")
 
 
 def kernel_source_sha():
@@ -168,10 +169,22 @@ def roofline(prof, cfg, dev):
     launches = max(1, kl[top])
     ms_per_launch = km[top] / launches
     out = {"kernel": f"k_{top}", "launches": kl[top], "ms_per_launch": ms_per_launch}
-    if top == "scan":
-        flops = 2.0 * d * prof["pairs"]
+    # TF32 dense peak: the measured bf16 cuBLAS peak x the nominal TF32/BF16 ratio (1.1 / 2.25)
+    tf32_tflops = peaks.get("bf16_tflops", 1889.4) * (1.1 / 2.25)
+    if top == "scan_tc":
+        flops = 2.0 * d * prof["pairs_tc"]
         ach = flops / launches / (ms_per_launch * 1e-3) / 1e12
-        bytes_ = 4.0 * d * (prof["rows_read"] + prof["items"])
+        out.update(bound="tensor", achieved=ach, peak=tf32_tflops / 3, unit="TFLOP/s",
+                   frac=ach / (tf32_tflops / 3),
+                   peak_source=(f"3xTF32: three TF32 MMAs per product; TF32 dense peak "
+                                f"{tf32_tflops:.0f} TFLOP/s = measured bf16 "
+                                f"{peaks.get('bf16_tflops', 1889.4):.0f} x 1.1/2.25 (of measured), "
+                                f"so the algorithmic peak is a third of it"),
+                   tensor_pipe_tflops=3 * ach)
+    elif top == "scan":
+        flops = 2.0 * d * (prof["pairs"] - prof["pairs_tc"])
+        ach = flops / launches / (ms_per_launch * 1e-3) / 1e12
+        bytes_ = 4.0 * d * (prof["rows_read"] - prof["rows_read_tc"] + prof["items"])
         out.update(bound="alu", achieved=ach, peak=fp32_tflops, unit="TFLOP/s",
                    frac=ach / fp32_tflops,
                    peak_source=f"FP32 FMA: {props.multi_processor_count} SMs x 128 lanes x 2 "
@@ -388,7 +401,8 @@ def run_sieve(args, cfg, world, rank, local):
         "profile": {"kernel_ms": prof["kernel_ms"], "kernel_launches": prof["kernel_launches"],
                     "rounds": prof["rounds"], "items": prof["items"], "groups": prof["groups"],
                     "mean_group": prof["items"] / max(1, prof["groups"]),
-                    "pairs": prof["pairs"], "rows_read": prof["rows_read"]},
+                    "pairs": prof["pairs"], "rows_read": prof["rows_read"],
+                    "pairs_tc": prof["pairs_tc"], "rows_read_tc": prof["rows_read_tc"]},
         "gpu_launches": args.steps * int(sum(prof["kernel_launches"].values())),
         "clocks": clock_rec,
         "e2e": e2e,

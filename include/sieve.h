@@ -49,6 +49,7 @@ typedef int32_t sieve_status;
 #define SIEVE_EUNSUPPORTED (-5) /* the current device is not sm_103 */
 #define SIEVE_ESCRATCH (-6)     /* sieve_search_noalloc: the call needs more scratch than
                                    SIEVE_NOALLOC_SCRATCH_BYTES */
+#define SIEVE_ETIMEOUT (-7)     /* a bounded device-side wait gave up (reported in sieve_stats) */
 
 /* The IVF index, resident on the device (Sec. 2.3).  Borrowed, read-only.
  *   vectors      device [n][d] fp32, unit-norm, partition-contiguous: the rows
@@ -88,7 +89,12 @@ typedef struct {
  *   profile    1 = also time every kernel launch with CUDA events recorded on
  *              `stream` around it (implies host-driven rounds and needs a
  *              stats pointer); 0 = no timing
- *   reserved0  must be 0
+ *   scan_path  how partition groups are scanned; all paths give the same
+ *              decisions up to fp32 rounding (see the parity notes):
+ *              0 = automatic (groups of >= 24 items on the tensor cores with
+ *              the 3xTF32 split when k <= 16, the rest on FP32 FMA),
+ *              1 = FP32 FMA only, 2 = tensor cores for every group
+ *              (needs k <= 16)
  */
 typedef struct {
     float tau;
@@ -98,14 +104,15 @@ typedef struct {
     int32_t lookahead;
     int32_t loop;
     int32_t profile;
-    int32_t reserved0;
+    int32_t scan_path;
     int64_t max_items_per_round;
 } sieve_params;
 
 /* Kernels of one search call, indexing sieve_stats.kernel_ms / kernel_launches:
  * centroid ranking, state initialisation, the issuer, the ready-queue
  * bucketing, the scatter into partition groups, the grouped scan with its
- * fused epilogue, the per-query merge, the end-of-round step, finalisation. */
+ * fused epilogue on FP32 FMA, the per-query merge, the end-of-round step,
+ * finalisation, and the grouped scan on the tensor cores. */
 enum {
     SIEVE_K_RANK = 0,
     SIEVE_K_INIT,
@@ -116,6 +123,7 @@ enum {
     SIEVE_K_MERGE,
     SIEVE_K_ROUND_END,
     SIEVE_K_FINALIZE,
+    SIEVE_K_SCAN_TC,
     SIEVE_NKERNELS
 };
 
@@ -128,6 +136,7 @@ enum {
  *   tiles        work tiles of the grouped scan
  *   rows_read    partition rows streamed by the scan (one read per tile)
  *   pairs        query-row similarities computed
+ *   rows_read_tc, pairs_tc  the part of rows_read / pairs done on the tensor cores
  *   status       device status word (0, or a SIEVE_E* code) */
 typedef struct {
     int64_t rounds;
@@ -136,6 +145,8 @@ typedef struct {
     int64_t tiles;
     int64_t rows_read;
     int64_t pairs;
+    int64_t rows_read_tc;
+    int64_t pairs_tc;
     int32_t status;
     int32_t reserved0;
     float kernel_ms[SIEVE_NKERNELS];          /* profile = 1: summed launch durations */

@@ -25,7 +25,8 @@ from . import _build
 
 SIEVE_OK = 0
 _STATUS = {0: "ok", -1: "invalid argument", -2: "CUDA error", -3: "workspace", -4: "round limit",
-           -5: "unsupported device", -6: "exceeds the no-allocation scratch"}
+           -5: "unsupported device", -6: "exceeds the no-allocation scratch",
+           -7: "device wait timed out"}
 
 
 class SieveError(RuntimeError):
@@ -46,17 +47,20 @@ class IndexViewC(C.Structure):
 class ParamsC(C.Structure):
     _fields_ = [("tau", C.c_float), ("k", C.c_int32), ("nprobe", C.c_int32), ("W", C.c_int32),
                 ("lookahead", C.c_int32), ("loop", C.c_int32), ("profile", C.c_int32),
-                ("reserved0", C.c_int32), ("max_items_per_round", C.c_int64)]
+                ("scan_path", C.c_int32), ("max_items_per_round", C.c_int64)]
 
 
 class StatsC(C.Structure):
     _fields_ = [("rounds", C.c_int64), ("items", C.c_int64), ("groups", C.c_int64),
                 ("tiles", C.c_int64), ("rows_read", C.c_int64), ("pairs", C.c_int64),
+                ("rows_read_tc", C.c_int64), ("pairs_tc", C.c_int64),
                 ("status", C.c_int32), ("reserved0", C.c_int32),
-                ("kernel_ms", C.c_float * 9), ("kernel_launches", C.c_int32 * 9)]
+                ("kernel_ms", C.c_float * 10), ("kernel_launches", C.c_int32 * 10)]
 
 
-KERNELS = ("rank", "init", "issue", "bucket", "scatter", "scan", "merge", "round_end", "finalize")
+KERNELS = ("rank", "init", "issue", "bucket", "scatter", "scan", "merge", "round_end", "finalize",
+           "scan_tc")
+SCAN_PATHS = {"auto": 0, "simt": 1, "tensor": 2}
 
 
 _lib = None
@@ -203,9 +207,10 @@ def rank_partitions(index: Index, Q, nprobe, return_scores=False, stream=None):
     return (order, sc) if return_scores else order
 
 
-def _params(tau, k, nprobe, W, lookahead, loop, max_items_per_round, profile=0):
+def _params(tau, k, nprobe, W, lookahead, loop, max_items_per_round, profile=0, scan_path="auto"):
     p = ParamsC()
     p.profile = int(profile)
+    p.scan_path = SCAN_PATHS[scan_path] if isinstance(scan_path, str) else int(scan_path)
     p.tau = float(tau)
     p.k = int(k)
     p.nprobe = int(nprobe)
@@ -257,8 +262,8 @@ def _stats_dict(st):
 
 
 def search(index: Index, Q, tau, k, nprobe, W, lookahead=True, query_ids=None, order=None,
-           max_items_per_round=0, loop=0, stats=False, profile=False, workspace=None, out=None,
-           stream=None):
+           max_items_per_round=0, loop=0, stats=False, profile=False, scan_path="auto",
+           workspace=None, out=None, stream=None):
     """SieveIVF search on device tensors (sieve_search).
 
     Returns (ids [nq][k] i64, scores [nq][k] f32, count [nq] i32, probes [nq] i32),
@@ -272,7 +277,7 @@ def search(index: Index, Q, tau, k, nprobe, W, lookahead=True, query_ids=None, o
         _need_cuda(order, torch.int32, "order", 2)
     nq = Q.shape[0]
     dev = Q.device
-    p = _params(tau, k, nprobe, W, lookahead, loop, max_items_per_round, profile)
+    p = _params(tau, k, nprobe, W, lookahead, loop, max_items_per_round, profile, scan_path)
     v = index.view()
     nbytes = C.c_size_t()
     _check(lib().sieve_search_workspace_size(C.byref(v), nq, C.byref(p), 0, C.byref(nbytes)),

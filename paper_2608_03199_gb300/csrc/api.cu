@@ -62,7 +62,8 @@ sieve_status check_params(const sieve_index_view *ix, const sieve_params *p) {
     if (p->loop != 0 && p->loop != 1) return SIEVE_EINVAL;
     if (p->max_items_per_round < 0) return SIEVE_EINVAL;
     if (p->profile != 0 && p->profile != 1) return SIEVE_EINVAL;
-    if (p->reserved0 != 0) return SIEVE_EINVAL;
+    if (p->scan_path < 0 || p->scan_path > 2) return SIEVE_EINVAL;
+    if (p->scan_path == 2 && p->k > kTcMaxK) return SIEVE_EINVAL;
     return SIEVE_OK;
 }
 
@@ -81,8 +82,8 @@ int64_t items_cap(int64_t nq, const sieve_params *p) {
 
 // Byte layout of the search workspace.
 struct Layout {
-    size_t ctl, order, S, E, counts, cursor, item_q, item_rank, item_p, bucketed, tiles, active,
-        res_cnt, res_s, res_id;
+    size_t ctl, order, S, E, counts, cursor, item_q, item_rank, item_p, bucketed, tiles, tc_tiles,
+        active, res_cnt, res_s, res_id;
     size_t h_Q, h_qids, h_ids, h_scores, h_count, h_probes;
     size_t total;
     int64_t cap, max_tiles;
@@ -97,7 +98,10 @@ Layout make_layout(const sieve_index_view *ix, int64_t nq, const sieve_params *p
         return at;
     };
     const int64_t cap = items_cap(nq, p);
-    const int64_t max_tiles = ceil_div(cap, QT) + ix->nlist + 1;
+    // SIMT tiles: at most one per QT items plus one per partial chunk; tensor-core
+    // tiles: at most one per kTcTile items plus one per partition
+    const int64_t max_tiles = ceil_div(cap, QT) + ceil_div(cap, kTcTile) + ix->nlist + 1;
+    const int64_t max_tc_tiles = ceil_div(cap, kTcTile) + ix->nlist + 1;
     L.cap = cap;
     L.max_tiles = max_tiles;
     L.ctl = take(sizeof(Ctl));
@@ -111,6 +115,7 @@ Layout make_layout(const sieve_index_view *ix, int64_t nq, const sieve_params *p
     L.item_p = take((size_t)cap * 4);
     L.bucketed = take((size_t)cap * 4);
     L.tiles = take((size_t)max_tiles * 16);
+    L.tc_tiles = take((size_t)max_tc_tiles * 16);
     L.active = take((size_t)nq * 16);
     L.res_cnt = take((size_t)cap * 4);
     L.res_s = take((size_t)cap * p->k * 4);
@@ -236,9 +241,9 @@ sieve_status run_graph(const GraphKey &key, cudaStream_t st) {
     return SIEVE_OK;
 }
 
-// 14 CUDA events: 12 around the six kernels of a round, 2 for single launches
+// CUDA events: two around each kernel of a round, two for single launches
 struct EventSet {
-    cudaEvent_t e[14] = {};
+    cudaEvent_t e[2 * kRoundKernels + 2] = {};
     cudaError_t create() {
         for (auto &x : e) {
             cudaError_t r = cudaEventCreate(&x);
@@ -288,6 +293,8 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
     a.cursor = reinterpret_cast<int *>(ws + L.cursor);
     a.bucketed = reinterpret_cast<int *>(ws + L.bucketed);
     a.tiles = reinterpret_cast<int4 *>(ws + L.tiles);
+    a.tc_tiles = reinterpret_cast<int4 *>(ws + L.tc_tiles);
+    a.tc_min = p->scan_path == 1 ? 0 : p->scan_path == 2 ? 1 : (p->k <= kTcMaxK ? 24 : 0);
     a.active = reinterpret_cast<int4 *>(ws + L.active);
     a.res_cnt = reinterpret_cast<int *>(ws + L.res_cnt);
     a.res_s = reinterpret_cast<float *>(ws + L.res_s);
@@ -301,6 +308,7 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
     const bool with_rank = order == nullptr;
     const size_t smem = scan_smem_bytes(ix->d, p->k);
     SIEVE_CUDA(prepare_scan_kernel(smem));
+    if (a.tc_min > 0) SIEVE_CUDA(prepare_scan_tc(p->k));
     if (with_rank) SIEVE_CUDA(prepare_rank(p->nprobe));
     const int blocks = scan_blocks_for(smem);
 
@@ -321,13 +329,13 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
         EventSet ev;
         if (p->profile) SIEVE_CUDA(ev.create());
         auto timed = [&](int slot, auto &&launch) -> cudaError_t {
-            if (p->profile) cudaEventRecord(ev.e[12], st);
+            if (p->profile) cudaEventRecord(ev.e[2 * kRoundKernels], st);
             cudaError_t e = launch();
             if (p->profile) {
-                cudaEventRecord(ev.e[13], st);
-                cudaEventSynchronize(ev.e[13]);
+                cudaEventRecord(ev.e[2 * kRoundKernels + 1], st);
+                cudaEventSynchronize(ev.e[2 * kRoundKernels + 1]);
                 float t = 0.f;
-                cudaEventElapsedTime(&t, ev.e[12], ev.e[13]);
+                cudaEventElapsedTime(&t, ev.e[2 * kRoundKernels], ev.e[2 * kRoundKernels + 1]);
                 ms[slot] += t;
             }
             return e;
@@ -344,9 +352,10 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
             SIEVE_CUDA(cudaMemcpyAsync(&more, &a.ctl->more, sizeof(int), cudaMemcpyDeviceToHost, st));
             SIEVE_CUDA(cudaStreamSynchronize(st));
             if (p->profile) {
-                const int slot[6] = {SIEVE_K_ISSUE, SIEVE_K_BUCKET, SIEVE_K_SCATTER, SIEVE_K_SCAN,
-                                     SIEVE_K_MERGE, SIEVE_K_ROUND_END};
-                for (int i = 0; i < 6; ++i) {
+                const int slot[kRoundKernels] = {SIEVE_K_ISSUE, SIEVE_K_BUCKET, SIEVE_K_SCATTER,
+                                                 SIEVE_K_SCAN_TC, SIEVE_K_SCAN, SIEVE_K_MERGE,
+                                                 SIEVE_K_ROUND_END};
+                for (int i = 0; i < kRoundKernels; ++i) {
                     float t = 0.f;
                     SIEVE_CUDA(cudaEventElapsedTime(&t, ev.e[2 * i], ev.e[2 * i + 1]));
                     ms[slot[i]] += t;
@@ -366,6 +375,8 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
         stats->tiles = (int64_t)c.tot_tiles;
         stats->rows_read = (int64_t)c.tot_rows;
         stats->pairs = (int64_t)c.tot_pairs;
+        stats->rows_read_tc = (int64_t)c.tot_rows_tc;
+        stats->pairs_tc = (int64_t)c.tot_pairs_tc;
         stats->status = c.status;
         stats->reserved0 = 0;
         for (int i = 0; i < SIEVE_NKERNELS; ++i) stats->kernel_ms[i] = ms[i];
@@ -375,6 +386,7 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
         stats->kernel_launches[SIEVE_K_INIT] = 1;
         stats->kernel_launches[SIEVE_K_FINALIZE] = 1;
         for (int slot : per_round) stats->kernel_launches[slot] = c.round;
+        stats->kernel_launches[SIEVE_K_SCAN_TC] = a.tc_min > 0 ? c.round : 0;
         if (c.status != 0) return c.status;
     }
     return SIEVE_OK;
@@ -409,6 +421,7 @@ const char *sieve_status_str(sieve_status s) {
         case SIEVE_ELIMIT: return "round limit reached";
         case SIEVE_EUNSUPPORTED: return "unsupported device (needs sm_103)";
         case SIEVE_ESCRATCH: return "call needs more scratch than the fixed no-allocation array";
+        case SIEVE_ETIMEOUT: return "a bounded device-side wait gave up";
         default: return "unknown status";
     }
 }

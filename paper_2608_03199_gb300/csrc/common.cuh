@@ -31,8 +31,10 @@ struct Ctl {
     int round;         // rounds finished
     int status;        // 0 or a SIEVE_E* code
     int more;          // 1 while another round is needed
-    int pad[7];
+    int n_tc_tiles;    // tensor-core scan tiles this round
+    int pad[6];
     unsigned long long tot_items, tot_groups, tot_tiles, tot_rows, tot_pairs;
+    unsigned long long tot_rows_tc, tot_pairs_tc;   // the tensor-core share of the two above
 };
 
 __host__ __device__ inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }

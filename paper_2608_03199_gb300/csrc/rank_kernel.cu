@@ -21,7 +21,74 @@ size_t rank_smem_bytes(int nprobe) {
     b += (size_t)QT * (RT + 1) * sizeof(float);  // tile scores
     b += (size_t)QT * nprobe * sizeof(float);    // list scores
     b += (size_t)QT * nprobe * sizeof(int);      // list ids
+    b += (size_t)(kThreads / 32) * RT * 8;       // per-warp sorted tile
+    b += (size_t)(kThreads / 32) * nprobe * 8;   // per-warp merge output
     return round_up(b, 16);
+}
+
+// Sort the 64 entries of a warp (entry h*32 + lane in slot h) so that entry 0
+// ranks first (score desc, id asc): a bitonic network, shuffles within a half,
+// in-register exchange across the halves.
+__device__ __forceinline__ void warp_sort64(float (&s)[2], int (&c)[2]) {
+    const unsigned lane = lane_id();
+    for (int k = 2; k <= 64; k <<= 1) {
+        for (int j = k >> 1; j > 0; j >>= 1) {
+            if (j == 32) {
+                // pair (lane, lane + 32); k == 64 here, so the block sorts "first first"
+                if (!ranks_before(s[0], c[0], s[1], c[1])) {
+                    float ts = s[0]; s[0] = s[1]; s[1] = ts;
+                    int tc = c[0]; c[0] = c[1]; c[1] = tc;
+                }
+            } else {
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int e = h * 32 + (int)lane;
+                    const float ps = __shfl_xor_sync(0xffffffffu, s[h], j);
+                    const int pc = __shfl_xor_sync(0xffffffffu, c[h], j);
+                    const bool up = (e & k) == 0;       // this block sorts first-ranked first
+                    const bool lower = (e & j) == 0;    // the lower index of the pair
+                    const bool mine_first = ranks_before(s[h], c[h], ps, pc);
+                    if (mine_first != (lower == up)) {
+                        s[h] = ps;
+                        c[h] = pc;
+                    }
+                }
+            }
+        }
+    }
+}
+
+// Merge the sorted list L (n entries, capacity cap) with the sorted tile T
+// (its first m entries) and keep the first cap: merge-path co-ranks, one
+// output position per lane step.  O is per-warp scratch of cap entries.
+__device__ __forceinline__ void warp_merge_list(float *Ls, int *Lc, int *n_ptr, int cap,
+                                                const float *Ts, const int *Tc, int m,
+                                                float *Os, int *Oc) {
+    const unsigned lane = lane_id();
+    const int n = *n_ptr;
+    const int total = n + m < cap ? n + m : cap;
+    for (int j = lane; j < total; j += 32) {
+        int lo = j - m > 0 ? j - m : 0;
+        int hi = j < n ? j : n;
+        while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (ranks_before(Ls[mid], Lc[mid], Ts[j - mid - 1], Tc[j - mid - 1]))
+                lo = mid + 1;
+            else
+                hi = mid;
+        }
+        const int i = lo;
+        const bool take_l = i < n && (j - i >= m || ranks_before(Ls[i], Lc[i], Ts[j - i], Tc[j - i]));
+        Os[j] = take_l ? Ls[i] : Ts[j - i];
+        Oc[j] = take_l ? Lc[i] : Tc[j - i];
+    }
+    __syncwarp();
+    for (int j = lane; j < total; j += 32) {
+        Ls[j] = Os[j];
+        Lc[j] = Oc[j];
+    }
+    if (lane == 0) *n_ptr = total;
+    __syncwarp();
 }
 
 __global__ void __launch_bounds__(kThreads) k_rank(const float *__restrict__ Q, int64_t nq,
@@ -35,6 +102,11 @@ __global__ void __launch_bounds__(kThreads) k_rank(const float *__restrict__ Q, 
     float *Ss = Cst + 2 * RT * LDX;
     float *ls = Ss + QT * (RT + 1);
     int *lc = reinterpret_cast<int *>(ls + QT * nprobe);
+    float *ts_w = reinterpret_cast<float *>(lc + QT * nprobe) + (threadIdx.x >> 5) * (2 * RT);
+    int *tc_w = reinterpret_cast<int *>(ts_w + RT);
+    float *os_w = reinterpret_cast<float *>(lc + QT * nprobe) + (kThreads / 32) * 2 * RT +
+                  (threadIdx.x >> 5) * (2 * nprobe);
+    int *oc_w = reinterpret_cast<int *>(os_w + nprobe);
 
     const int tid = threadIdx.x, tq = tid & 7, tr = tid >> 3;
     const unsigned lane = lane_id(), warp = tid >> 5;
@@ -77,24 +149,49 @@ __global__ void __launch_bounds__(kThreads) k_rank(const float *__restrict__ Q, 
 #pragma unroll
                 for (int j = 0; j < 4; ++j) Ss[(tq + 8 * i) * (RT + 1) + tr + 16 * j] = acc[i][j];
             __syncthreads();
+            // merge the tile into each query's sorted top-nprobe list: entries
+            // that rank before the list's last entry are candidates; a few are
+            // inserted one by one, more are sorted and merged in one pass
             for (int i = warp; i < nqb; i += kThreads / 32) {
                 float *li_s = ls + i * nprobe;
                 int *li_c = lc + i * nprobe;
-                for (int half = 0; half < 2; ++half) {
-                    const int64_t cid = ct * RT + half * 32 + lane;
-                    const float sc = Ss[i * (RT + 1) + half * 32 + lane];
-                    const int n = list_n[i];
-                    bool cand = cid < nlist &&
-                                (n < nprobe || ranks_before(sc, (int)cid, li_s[nprobe - 1],
-                                                            li_c[nprobe - 1]));
-                    unsigned bal = __ballot_sync(0xffffffffu, cand);
-                    while (bal) {
-                        const int src = __ffs(bal) - 1;
-                        bal &= bal - 1;
-                        const float bs = __shfl_sync(0xffffffffu, sc, src);
-                        const int bc = __shfl_sync(0xffffffffu, (int)cid, src);
-                        warp_list_insert(li_s, li_c, &list_n[i], nprobe, bs, bc);
+                const int n = list_n[i];
+                float sv[2];
+                int cv[2];
+                bool cand[2];
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int64_t cid = ct * RT + h * 32 + lane;
+                    sv[h] = cid < nlist ? Ss[i * (RT + 1) + h * 32 + lane] : -__int_as_float(0x7f800000);
+                    cv[h] = cid < nlist ? (int)cid : INT32_MAX;
+                    cand[h] = cid < nlist &&
+                              (n < nprobe || ranks_before(sv[h], cv[h], li_s[nprobe - 1], li_c[nprobe - 1]));
+                }
+                const unsigned b0 = __ballot_sync(0xffffffffu, cand[0]);
+                const unsigned b1 = __ballot_sync(0xffffffffu, cand[1]);
+                const int m = __popc(b0) + __popc(b1);
+                if (m == 0) continue;
+                if (m <= 4) {
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        unsigned bal = h ? b1 : b0;
+                        while (bal) {
+                            const int src = __ffs(bal) - 1;
+                            bal &= bal - 1;
+                            const float bs = __shfl_sync(0xffffffffu, sv[h], src);
+                            const int bc = __shfl_sync(0xffffffffu, cv[h], src);
+                            warp_list_insert(li_s, li_c, &list_n[i], nprobe, bs, bc);
+                        }
                     }
+                } else {
+                    // candidates form a prefix of the sorted tile
+                    warp_sort64(sv, cv);
+                    ts_w[lane] = sv[0];
+                    tc_w[lane] = cv[0];
+                    ts_w[lane + 32] = sv[1];
+                    tc_w[lane + 32] = cv[1];
+                    __syncwarp();
+                    warp_merge_list(li_s, li_c, &list_n[i], nprobe, ts_w, tc_w, m, os_w, oc_w);
                 }
             }
         }

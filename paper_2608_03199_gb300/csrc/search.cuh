@@ -34,7 +34,10 @@ struct SearchArgs {
     int *item_q, *item_rank, *item_p;   // [cap]
     int *counts, *cursor;               // [nlist]
     int *bucketed;                      // [cap]
-    int4 *tiles;                        // [max_tiles]: partition, first bucketed slot, items
+    int4 *tiles;                        // SIMT tiles: partition, first bucketed slot, items
+    int4 *tc_tiles;                     // tensor-core tiles (up to 128 items each)
+    int tc_min;                         // groups chunks of >= tc_min items go to the
+                                        // tensor cores; 0 = SIMT only
     int4 *active;                       // [nq]: query, first item, items
     // per-item local results
     int *res_cnt;                       // [cap]
@@ -56,6 +59,14 @@ cudaError_t launch_finalize(const SearchArgs &a, cudaStream_t st);
 cudaError_t launch_round(const SearchArgs &a, size_t scan_smem, int scan_blocks,
                          cudaGraphConditionalHandle cond, int use_cond, cudaStream_t st,
                          cudaEvent_t *ev = nullptr);
+constexpr int kRoundKernels = 7;   // issue, bucket, scatter, scan_tc, scan, merge, round_end
+
+// tensor-core scan (scan_tc.cu)
+constexpr int kTcMaxK = 16;        // largest k the tensor-core epilogue keeps
+constexpr int kTcTile = 128;       // items per tensor-core tile
+size_t scan_tc_smem_bytes(int k);
+cudaError_t prepare_scan_tc(int k);
+void enqueue_scan_tc(const SearchArgs &a, cudaStream_t st);
 
 // centroid ranking (rank_kernel.cu): prepare_rank once before launches or
 // stream capture, then enqueue_rank (a single kernel launch)

@@ -133,25 +133,44 @@ __global__ void __launch_bounds__(kIssueThreads) k_issue(SearchArgs a) {
 // ---------------------------------------------------------------------------
 constexpr int kBucketThreads = 1024;
 
+// A group of c items is cut into chunks of up to kTcTile; a chunk with at
+// least tc_min items is one tensor-core tile, a smaller one is cut into SIMT
+// tiles of up to QT items.
+__device__ __forceinline__ void count_tiles(int c, int tc_min, int &n_tc, int &n_simt) {
+    n_tc = 0;
+    n_simt = 0;
+    for (int o = 0; o < c; o += kTcTile) {
+        const int sz = c - o < kTcTile ? c - o : kTcTile;
+        if (tc_min > 0 && sz >= tc_min)
+            ++n_tc;
+        else
+            n_simt += (sz + QT - 1) / QT;
+    }
+}
+
 __global__ void __launch_bounds__(kBucketThreads) k_bucket(SearchArgs a) {
     __shared__ int warp_tot[32];
-    __shared__ int sums[2];
+    __shared__ int sums[3];
     Ctl *ctl = a.ctl;
     const int64_t nl = a.nlist;
     const int per = (int)ceil_div(nl, kBucketThreads);
     const int64_t p0 = (int64_t)threadIdx.x * per;
-    int my_items = 0, my_tiles = 0, my_groups = 0;
+    int my[3] = {0, 0, 0};   // items, SIMT tiles, tensor-core tiles
+    int my_groups = 0;
     for (int64_t p = p0; p < p0 + per && p < nl; ++p) {
-        int c = a.counts[p];
-        my_items += c;
-        my_tiles += (c + QT - 1) / QT;
+        const int c = a.counts[p];
+        int ntc, ns;
+        count_tiles(c, a.tc_min, ntc, ns);
+        my[0] += c;
+        my[1] += ns;
+        my[2] += ntc;
         my_groups += c > 0;
     }
-    // two exclusive scans over threads (items, tiles)
+    // three exclusive scans over threads
     const unsigned lane = lane_id(), warp = threadIdx.x >> 5;
-    int xs[2] = {my_items, my_tiles}, ex[2];
-    for (int v = 0; v < 2; ++v) {
-        int x = xs[v];
+    int ex[3];
+    for (int v = 0; v < 3; ++v) {
+        int x = my[v];
         for (int o = 1; o < 32; o <<= 1) {
             int y = __shfl_up_sync(0xffffffffu, x, o);
             if (lane >= (unsigned)o) x += y;
@@ -168,16 +187,22 @@ __global__ void __launch_bounds__(kBucketThreads) k_bucket(SearchArgs a) {
             if (lane == 31) sums[v] = w;
         }
         __syncthreads();
-        ex[v] = (warp > 0 ? warp_tot[warp - 1] : 0) + x - xs[v];
+        ex[v] = (warp > 0 ? warp_tot[warp - 1] : 0) + x - my[v];
         __syncthreads();
     }
-    int ioff = ex[0], toff = ex[1];
+    int ioff = ex[0], soff = ex[1], toff = ex[2];
     for (int64_t p = p0; p < p0 + per && p < nl; ++p) {
-        int c = a.counts[p];
+        const int c = a.counts[p];
         a.cursor[p] = ioff;
-        for (int t = 0; t * QT < c; ++t)
-            a.tiles[toff + t] = make_int4((int)p, ioff + t * QT, c - t * QT < QT ? c - t * QT : QT, 0);
-        toff += (c + QT - 1) / QT;
+        for (int o = 0; o < c; o += kTcTile) {
+            const int sz = c - o < kTcTile ? c - o : kTcTile;
+            if (a.tc_min > 0 && sz >= a.tc_min) {
+                a.tc_tiles[toff++] = make_int4((int)p, ioff + o, sz, 0);
+            } else {
+                for (int u = 0; u < sz; u += QT)
+                    a.tiles[soff++] = make_int4((int)p, ioff + o + u, sz - u < QT ? sz - u : QT, 0);
+            }
+        }
         ioff += c;
         a.counts[p] = 0;   // ready for the next round's issue
     }
@@ -187,6 +212,7 @@ __global__ void __launch_bounds__(kBucketThreads) k_bucket(SearchArgs a) {
     if (lane == 0 && g) atomicAdd(&ctl->tot_groups, (unsigned long long)g);
     if (threadIdx.x == 0) {
         ctl->n_tiles = sums[1];
+        ctl->n_tc_tiles = sums[2];
         ctl->tile_next = 0;
     }
 }
@@ -456,7 +482,7 @@ __global__ void k_round_end(SearchArgs a, cudaGraphConditionalHandle cond, int u
     Ctl *c = a.ctl;
     const int items = c->n_items < a.cap ? c->n_items : (int)a.cap;
     c->tot_items += (unsigned long long)items;
-    c->tot_tiles += (unsigned long long)c->n_tiles;
+    c->tot_tiles += (unsigned long long)(c->n_tiles + c->n_tc_tiles);
     c->round += 1;
     int more = (c->n_continue > 0 || c->n_deferred > 0) && c->status == 0 ? 1 : 0;
     if (more && c->round >= a.max_rounds) {
@@ -467,6 +493,7 @@ __global__ void k_round_end(SearchArgs a, cudaGraphConditionalHandle cond, int u
     c->n_items = 0;
     c->n_active = 0;
     c->n_tiles = 0;
+    c->n_tc_tiles = 0;
     c->tile_next = 0;
     c->n_deferred = 0;
     c->n_continue = 0;
@@ -509,32 +536,40 @@ cudaError_t launch_finalize(const SearchArgs &a, cudaStream_t st) {
 cudaError_t launch_round(const SearchArgs &a, size_t scan_smem, int scan_blocks,
                          cudaGraphConditionalHandle cond, int use_cond, cudaStream_t st,
                          cudaEvent_t *ev) {
-    // ev (optional): 12 events, recorded before/after each of the 6 kernels
+    // ev (optional): 2 * kRoundKernels events, recorded before/after each kernel
     const int sms = num_sms();
-    auto mark = [&](int i) {
-        if (ev) cudaEventRecord(ev[i], st);
+    int slot = 0;
+    auto begin = [&] {
+        if (ev) cudaEventRecord(ev[2 * slot], st);
     };
-    int issue_blocks = (int)std::min<int64_t>(ceil_div(a.nq, kIssueThreads), 8 * sms);
-    mark(0);
+    auto end = [&] {
+        if (ev) cudaEventRecord(ev[2 * slot + 1], st);
+        ++slot;
+    };
+    const int issue_blocks = (int)std::min<int64_t>(ceil_div(a.nq, kIssueThreads), 8 * sms);
+    begin();
     k_issue<<<issue_blocks, kIssueThreads, 0, st>>>(a);
-    mark(1);
-    mark(2);
+    end();
+    begin();
     k_bucket<<<1, kBucketThreads, 0, st>>>(a);
-    mark(3);
-    int scatter_blocks = (int)std::min<int64_t>(ceil_div(a.cap, 256), 8 * sms);
-    mark(4);
+    end();
+    const int scatter_blocks = (int)std::min<int64_t>(ceil_div(a.cap, 256), 8 * sms);
+    begin();
     k_scatter<<<scatter_blocks, 256, 0, st>>>(a);
-    mark(5);
-    mark(6);
+    end();
+    begin();
+    if (a.tc_min > 0) enqueue_scan_tc(a, st);
+    end();
+    begin();
     k_scan<<<scan_blocks, kThreads, scan_smem, st>>>(a);
-    mark(7);
-    int merge_blocks = (int)std::min<int64_t>(ceil_div(a.nq * 32, kMergeThreads), 8 * sms);
-    mark(8);
+    end();
+    const int merge_blocks = (int)std::min<int64_t>(ceil_div(a.nq * 32, kMergeThreads), 8 * sms);
+    begin();
     k_merge<<<merge_blocks, kMergeThreads, 0, st>>>(a);
-    mark(9);
-    mark(10);
+    end();
+    begin();
     k_round_end<<<1, 1, 0, st>>>(a, cond, use_cond);
-    mark(11);
+    end();
     return cudaGetLastError();
 }
 

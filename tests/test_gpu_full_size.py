@@ -60,14 +60,14 @@ def test_full_size_sampled_parity(full):
 
 def test_full_size_schedule_invariance_and_fixed_probe(full):
     cfg, wl, index, h = full
+    runs = [_np(sieve.search(index, wl["Q"], cfg.tau, cfg.k, cfg.nprobe, cfg.W, query_ids=wl["qids"],
+                             scan_path="tensor", **kw))
+            for kw in (dict(lookahead=True), dict(lookahead=False),
+                       dict(lookahead=True, max_items_per_round=65536))]
+    for key in runs[0]:
+        assert all(np.array_equal(runs[0][key], r[key]) for r in runs[1:]), key
     a = _np(sieve.search(index, wl["Q"], cfg.tau, cfg.k, cfg.nprobe, cfg.W, lookahead=True,
                          query_ids=wl["qids"]))
-    b = _np(sieve.search(index, wl["Q"], cfg.tau, cfg.k, cfg.nprobe, cfg.W, lookahead=False,
-                         query_ids=wl["qids"]))
-    c = _np(sieve.search(index, wl["Q"], cfg.tau, cfg.k, cfg.nprobe, cfg.W, lookahead=True,
-                         query_ids=wl["qids"], max_items_per_round=65536))
-    for key in a:
-        assert np.array_equal(a[key], b[key]) and np.array_equal(a[key], c[key]), key
     fx = _np(sieve.search(index, wl["Q"], cfg.tau, cfg.k, cfg.nprobe, cfg.nprobe, lookahead=True,
                           query_ids=wl["qids"]))
     assert (fx["probes"] == cfg.nprobe).all()

@@ -104,25 +104,56 @@ def test_search_parity_deep(deep, g_deep, W, lookahead):
     check(deep, g_deep, deep["Q"], deep["qids"], c.tau, c.k, c.nprobe, W, lookahead)
 
 
-def test_schedule_changes_nothing(deep, g_deep):
+@pytest.mark.parametrize("path", ["simt", "tensor"])
+def test_schedule_changes_nothing(deep, g_deep, path):
     """Lookahead on/off, per-round caps and the loop mode give bit-identical
-    output (Sec. 4.2: the microbatch cap only splits groups; Sec. 4.3)."""
+    output (Sec. 4.2: the microbatch cap only splits groups; Sec. 4.3).  The
+    scan path is fixed: each path computes a pair's similarity the same way
+    whatever group it lands in, the two paths round differently."""
     c = deep["cfg"]
     Q, qids = deep["Q"], deep["qids"]
-    base = run(g_deep, Q, qids, c.tau, c.k, c.nprobe, c.W, lookahead=1)
+    base = run(g_deep, Q, qids, c.tau, c.k, c.nprobe, c.W, lookahead=1, scan_path=path)
     variants = [dict(lookahead=0), dict(lookahead=1, max_items_per_round=4096),
                 dict(lookahead=1, max_items_per_round=7), dict(lookahead=0, loop=1),
                 dict(lookahead=1, loop=1, max_items_per_round=100)]
     for kw in variants:
-        got = run(g_deep, Q, qids, c.tau, c.k, c.nprobe, c.W, **kw)
+        got = run(g_deep, Q, qids, c.tau, c.k, c.nprobe, c.W, scan_path=path, **kw)
         for key in ("ids", "scores", "count", "probes"):
             assert np.array_equal(got[key], base[key]), (kw, key)
     sub = slice(0, 25)   # a cap of one item per round: one search per round
     one = run(g_deep, Q[sub], qids[sub], c.tau, c.k, c.nprobe, c.W, lookahead=1,
-              max_items_per_round=1, stats=True)
+              max_items_per_round=1, stats=True, scan_path=path)
     for key in ("ids", "scores", "count", "probes"):
         assert np.array_equal(one[key], base[key][sub]), key
     assert one["stats"]["rounds"] >= one["probes"].sum()
+
+
+@pytest.mark.parametrize("path", ["simt", "tensor", "auto"])
+def test_scan_paths_parity(tiny, g_tiny, deep, g_deep, path):
+    """Both contraction paths (FP32 FMA, tensor-core 3xTF32) and the automatic
+    split meet the parity bar, on groups of every size."""
+    c = tiny["cfg"]
+    for la in (0, 1):
+        check(tiny, g_tiny, tiny["Q"], tiny["qids"], c.tau, c.k, c.nprobe, c.W, la, scan_path=path)
+    c = deep["cfg"]
+    check(deep, g_deep, deep["Q"], deep["qids"], c.tau, c.k, c.nprobe, c.W, 1, scan_path=path)
+    check(deep, g_deep, deep["Q"], deep["qids"], c.tau, c.k, c.nprobe, BIG_W, 1, scan_path=path)
+
+
+def test_tensor_path_scores_match_fp64(tiny, g_tiny, dev):
+    """Every returned similarity of the 3xTF32 path is within 1e-6 of the fp64
+    inner product of the same pair (the split's error bound, well inside the
+    1e-5 tolerance)."""
+    c = tiny["cfg"]
+    got = run(g_tiny, tiny["Q"], tiny["qids"], 0.5, 16, c.nprobe, BIG_W, lookahead=1,
+              scan_path="tensor")
+    ids, sc, cnt = got["ids"], got["scores"], got["count"]
+    valid = np.arange(16)[None, :] < cnt[:, None]
+    qi, kj = np.nonzero(valid)
+    exact = np.einsum("ij,ij->i", tiny["Q"][qi].astype(np.float64),
+                      tiny["X"][ids[qi, kj]].astype(np.float64))
+    assert len(qi) > 1000
+    assert np.abs(sc[qi, kj] - exact).max() <= 1e-6
 
 
 @pytest.mark.parametrize("W", [16, BIG_W])
@@ -239,6 +270,8 @@ def test_empty_partitions_and_odd_dimension(dev):
 
 def test_invalid_arguments_raise(tiny, g_tiny, dev):
     Q = torch.from_numpy(tiny["Q"][:4]).to(dev)
+    with pytest.raises(sieve.SieveError):
+        sieve.search(g_tiny, Q, 0.9, 17, 16, 4, scan_path="tensor")   # tensor path needs k <= 16
     for kw in (dict(k=0), dict(k=65), dict(nprobe=65), dict(W=0)):
         args = dict(tau=0.9, k=10, nprobe=16, W=4)
         args.update(kw)
