@@ -89,12 +89,12 @@ typedef struct {
  *   profile    1 = also time every kernel launch with CUDA events recorded on
  *              `stream` around it (implies host-driven rounds and needs a
  *              stats pointer); 0 = no timing
- *   scan_path  how partition groups are scanned; all paths give the same
+ *   scan_path  which units compute similarities; all paths give the same
  *              decisions up to fp32 rounding (see the parity notes):
- *              0 = automatic (groups of >= 24 items on the tensor cores with
- *              the 3xTF32 split when k <= 16, the rest on FP32 FMA),
- *              1 = FP32 FMA only, 2 = tensor cores for every group
- *              (needs k <= 16)
+ *              0 = automatic (ranking on the tensor cores when nlist <= 2048;
+ *              partition groups of >= 24 items on the tensor cores when
+ *              k <= 16, the rest on FP32 FMA), 1 = FP32 FMA only,
+ *              2 = tensor cores for every group (needs k <= 16)
  */
 typedef struct {
     float tau;
@@ -170,12 +170,17 @@ sieve_status sieve_build_layout(const float *X, const int32_t *assign, int64_t n
                                 void *stream);
 
 /* Centroid ranking (Sec. 2.3, Sec. 4.1): for every query, the nprobe
- * centroids with the largest fp32 inner product, best first; equal scores
- * rank the lower centroid id first.
+ * centroids with the largest inner product, best first; equal scores rank
+ * the lower centroid id first.  Scores are fp32-accurate: tensor cores with
+ * a 3xTF32 split and a score table in the workspace when nlist <= 2048,
+ * FP32 FMA with a fused selection otherwise.
  *   Q        device [nq][d] fp32
  *   order    device [nq][nprobe] int32 out, 0-based centroid ids
  *   cscores  device [nq][nprobe] fp32 out (nullable): the matching scores
- * Needs no workspace (ws may be NULL, ws_bytes 0). */
+ *   ws       workspace of sieve_rank_workspace_size bytes (0 bytes, ws may
+ *            be NULL, when nlist > 2048); SIEVE_EWORKSPACE if smaller */
+sieve_status sieve_rank_workspace_size(const sieve_index_view *ix, int64_t nq, int32_t nprobe,
+                                       size_t *bytes);
 sieve_status sieve_rank_partitions(const sieve_index_view *ix, const float *Q, int64_t nq,
                                    int32_t nprobe, int32_t *order, float *cscores, void *ws,
                                    size_t ws_bytes, void *stream);

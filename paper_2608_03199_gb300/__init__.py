@@ -72,6 +72,8 @@ _SIGNATURES = {
     "sieve_build_layout": (C.c_int32, [C.c_void_p, C.c_void_p, C.c_int64, C.c_int32, C.c_int64,
                                        C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_size_t,
                                        C.c_void_p]),
+    "sieve_rank_workspace_size": (C.c_int32, [C.POINTER(IndexViewC), C.c_int64, C.c_int32,
+                                              C.POINTER(C.c_size_t)]),
     "sieve_rank_partitions": (C.c_int32, [C.POINTER(IndexViewC), C.c_void_p, C.c_int64, C.c_int32,
                                           C.c_void_p, C.c_void_p, C.c_void_p, C.c_size_t,
                                           C.c_void_p]),
@@ -202,8 +204,12 @@ def rank_partitions(index: Index, Q, nprobe, return_scores=False, stream=None):
     order = torch.empty((nq, nprobe), dtype=torch.int32, device=Q.device)
     sc = torch.empty((nq, nprobe), dtype=torch.float32, device=Q.device) if return_scores else None
     v = index.view()
+    nbytes = C.c_size_t()
+    _check(lib().sieve_rank_workspace_size(C.byref(v), nq, nprobe, C.byref(nbytes)),
+           "sieve_rank_workspace_size")
+    ws = torch.empty(max(nbytes.value, 256), dtype=torch.uint8, device=Q.device)
     _check(lib().sieve_rank_partitions(C.byref(v), _ptr(Q), nq, nprobe, _ptr(order), _ptr(sc),
-                                       None, 0, _stream(stream)), "sieve_rank_partitions")
+                                       _ptr(ws), ws.numel(), _stream(stream)), "sieve_rank_partitions")
     return (order, sc) if return_scores else order
 
 

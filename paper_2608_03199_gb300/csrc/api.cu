@@ -83,7 +83,7 @@ int64_t items_cap(int64_t nq, const sieve_params *p) {
 // Byte layout of the search workspace.
 struct Layout {
     size_t ctl, order, S, E, counts, cursor, item_q, item_rank, item_p, bucketed, tiles, tc_tiles,
-        active, res_cnt, res_s, res_id;
+        active, res_cnt, res_s, res_id, rank_scratch;
     size_t h_Q, h_qids, h_ids, h_scores, h_count, h_probes;
     size_t total;
     int64_t cap, max_tiles;
@@ -120,6 +120,9 @@ Layout make_layout(const sieve_index_view *ix, int64_t nq, const sieve_params *p
     L.res_cnt = take((size_t)cap * 4);
     L.res_s = take((size_t)cap * p->k * 4);
     L.res_id = take((size_t)cap * p->k * 8);
+    L.rank_scratch = (p->scan_path != 1 && rank_tc_supported(ix->nlist, p->nprobe))
+                         ? take(rank_tc_scratch_bytes(nq, ix->nlist))
+                         : 0;
     if (host_io) {
         L.h_Q = take((size_t)nq * ix->d * 4);
         L.h_qids = take((size_t)nq * 8);
@@ -140,6 +143,7 @@ struct GraphKey {
     SearchArgs a;
     int device;
     int with_rank;
+    int rank_tc;
     size_t scan_smem;
     int scan_blocks;
     bool operator==(const GraphKey &o) const { return std::memcmp(this, &o, sizeof(*this)) == 0; }
@@ -157,6 +161,16 @@ std::vector<GraphEntry> g_graphs;
 uint64_t g_graph_clock = 0;
 constexpr size_t kGraphCacheMax = 8;
 
+// the centroid ranking of a search: the tensor-core kernel when it applies,
+// reporting a bounded wait that gives up in the search's status word
+cudaError_t launch_search_rank(const SearchArgs &a, int rank_tc, cudaStream_t st) {
+    int32_t *order = const_cast<int32_t *>(a.order);
+    if (rank_tc)
+        return enqueue_rank_tc(a.Q, a.nq, a.C, a.nlist, a.d, a.nprobe, order, nullptr,
+                               a.rank_scratch, &a.ctl->status, st);
+    return enqueue_rank(a.Q, a.nq, a.C, a.nlist, a.d, a.nprobe, order, nullptr, st);
+}
+
 sieve_status build_graph(const GraphKey &key, cudaGraph_t *g_out, cudaGraphExec_t *exec_out) {
     const SearchArgs &a = key.a;
     cudaStream_t cs = nullptr;
@@ -169,10 +183,8 @@ sieve_status build_graph(const GraphKey &key, cudaGraph_t *g_out, cudaGraphExec_
     do {
         // outer graph: [rank] -> init -> WHILE(rounds) -> finalize
         if ((e = cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal)) != cudaSuccess) break;
-        if (key.with_rank)
-            e = enqueue_rank(a.Q, a.nq, a.C, a.nlist, a.d, a.nprobe, const_cast<int32_t *>(a.order),
-                             nullptr, cs);
-        if (e == cudaSuccess) e = launch_init(a, cs);
+        e = launch_init(a, cs);
+        if (e == cudaSuccess && key.with_rank) e = launch_search_rank(a, key.rank_tc, cs);
         cudaStreamCaptureStatus cst;
         cudaGraph_t cg = nullptr;
         const cudaGraphNode_t *deps = nullptr;
@@ -296,6 +308,7 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
     a.tc_tiles = reinterpret_cast<int4 *>(ws + L.tc_tiles);
     a.tc_min = p->scan_path == 1 ? 0 : p->scan_path == 2 ? 1 : (p->k <= kTcMaxK ? 24 : 0);
     a.active = reinterpret_cast<int4 *>(ws + L.active);
+    a.rank_scratch = L.rank_scratch ? reinterpret_cast<float *>(ws + L.rank_scratch) : nullptr;
     a.res_cnt = reinterpret_cast<int *>(ws + L.res_cnt);
     a.res_s = reinterpret_cast<float *>(ws + L.res_s);
     a.res_id = reinterpret_cast<long long *>(ws + L.res_id);
@@ -306,10 +319,11 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
     a.ctl = reinterpret_cast<Ctl *>(ws + L.ctl);
 
     const bool with_rank = order == nullptr;
+    const int rank_tc = with_rank && a.rank_scratch != nullptr;
     const size_t smem = scan_smem_bytes(ix->d, p->k);
     SIEVE_CUDA(prepare_scan_kernel(smem));
     if (a.tc_min > 0) SIEVE_CUDA(prepare_scan_tc(p->k));
-    if (with_rank) SIEVE_CUDA(prepare_rank(p->nprobe));
+    if (with_rank) SIEVE_CUDA(rank_tc ? prepare_rank_tc(p->nprobe) : prepare_rank(p->nprobe));
     const int blocks = scan_blocks_for(smem);
 
     float ms[SIEVE_NKERNELS] = {0};
@@ -319,6 +333,7 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
         key.a = a;
         SIEVE_CUDA(cudaGetDevice(&key.device));
         key.with_rank = with_rank;
+        key.rank_tc = rank_tc;
         key.scan_smem = smem;
         key.scan_blocks = blocks;
         sieve_status rc = run_graph(key, st);
@@ -340,12 +355,9 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
             }
             return e;
         };
-        if (with_rank)
-            SIEVE_CUDA(timed(SIEVE_K_RANK, [&] {
-                return enqueue_rank(Q, nq, ix->centroids, ix->nlist, ix->d, p->nprobe,
-                                    const_cast<int32_t *>(a.order), nullptr, st);
-            }));
         SIEVE_CUDA(timed(SIEVE_K_INIT, [&] { return launch_init(a, st); }));
+        if (with_rank)
+            SIEVE_CUDA(timed(SIEVE_K_RANK, [&] { return launch_search_rank(a, rank_tc, st); }));
         for (;;) {
             SIEVE_CUDA(launch_round(a, smem, blocks, 0, 0, st, p->profile ? ev.e : nullptr));
             int more = 0;
@@ -449,11 +461,19 @@ sieve_status sieve_build_layout(const float *X, const int32_t *assign, int64_t n
     return bad ? SIEVE_EINVAL : SIEVE_OK;
 }
 
+sieve_status sieve_rank_workspace_size(const sieve_index_view *ix, int64_t nq, int32_t nprobe,
+                                       size_t *bytes) {
+    if (!bytes) return SIEVE_EINVAL;
+    sieve_status rc = check_index(ix, true);
+    if (rc != SIEVE_OK) return rc;
+    if (nprobe < 1 || nprobe > kMaxNprobe || nprobe > ix->nlist || nq < 0) return SIEVE_EINVAL;
+    *bytes = rank_tc_supported(ix->nlist, nprobe) && nq > 0 ? rank_tc_scratch_bytes(nq, ix->nlist) : 0;
+    return SIEVE_OK;
+}
+
 sieve_status sieve_rank_partitions(const sieve_index_view *ix, const float *Q, int64_t nq,
                                    int32_t nprobe, int32_t *order, float *cscores, void *ws,
                                    size_t ws_bytes, void *stream) {
-    (void)ws;
-    (void)ws_bytes;
     sieve_status rc = check_index(ix, true);
     if (rc != SIEVE_OK) return rc;
     if (nprobe < 1 || nprobe > kMaxNprobe || nprobe > ix->nlist) return SIEVE_EINVAL;
@@ -461,9 +481,19 @@ sieve_status sieve_rank_partitions(const sieve_index_view *ix, const float *Q, i
     if (nq > 0 && (!Q || !order || !aligned16(Q))) return SIEVE_EINVAL;
     if ((rc = check_device()) != SIEVE_OK) return rc;
     if (nq == 0) return SIEVE_OK;
-    SIEVE_CUDA(prepare_rank(nprobe));
-    SIEVE_CUDA(enqueue_rank(Q, nq, ix->centroids, ix->nlist, ix->d, nprobe, order, cscores,
-                            static_cast<cudaStream_t>(stream)));
+    if (rank_tc_supported(ix->nlist, nprobe)) {
+        if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) ||
+            ws_bytes < rank_tc_scratch_bytes(nq, ix->nlist))
+            return SIEVE_EWORKSPACE;
+        SIEVE_CUDA(prepare_rank_tc(nprobe));
+        SIEVE_CUDA(enqueue_rank_tc(Q, nq, ix->centroids, ix->nlist, ix->d, nprobe, order, cscores,
+                                   static_cast<float *>(ws), nullptr,
+                                   static_cast<cudaStream_t>(stream)));
+    } else {
+        SIEVE_CUDA(prepare_rank(nprobe));
+        SIEVE_CUDA(enqueue_rank(Q, nq, ix->centroids, ix->nlist, ix->d, nprobe, order, cscores,
+                                static_cast<cudaStream_t>(stream)));
+    }
     return SIEVE_OK;
 }
 

@@ -1,0 +1,247 @@
+// rank_tc.cu -- centroid ranking on the tcgen05 tensor cores (Sec. 2.3,
+// Sec. 4.1: P_i = the nprobe centroids with the largest inner product with
+// q_i, best first, equal scores by lower centroid id), for nlist <= 2048.
+//
+// Two kernels per chunk of queries:
+//   k_rank_tc  the 3xTF32 pipeline of tc_pipeline.cuh: 128 consecutive
+//              queries (A rows) against all centroids (B rows, 128 per
+//              chunk); each epilogue thread stores its query's scores into a
+//              score table [queries][ld] in the caller's workspace
+//   k_select   one warp per query: the query's scores sit in registers
+//              (nlist / 32 per lane); the exact nprobe-th largest score is
+//              found bit by bit (32 rounds of "how many scores are >= t"),
+//              the entries above it plus the lowest-id entries equal to it
+//              are gathered, and a warp bitonic network sorts them by
+//              (score desc, id asc).
+#include "tc_pipeline.cuh"
+
+namespace sieve {
+
+struct RankArgs {
+    const float *Q;
+    int64_t nq;
+    const float *C;
+    int64_t nlist;
+    int d;
+    float *scores;   // [nq][ld] score table
+    int64_t ld;      // row stride of the table, a multiple of 32
+    int *status;     // nullable: where a bounded wait that gives up is reported
+};
+
+__device__ int g_rank_status_sink;
+
+struct RankMode {
+    using Args = RankArgs;
+    static constexpr int kN = 128;
+    struct Tile {
+        int64_t q0;
+        int ni;
+        int64_t nb;
+    };
+    __device__ static int num_tiles(const Args &a) { return (int)ceil_div(a.nq, tcp::kM); }
+    __device__ static int d(const Args &a) { return a.d; }
+    __device__ static int *status(const Args &a) { return a.status ? a.status : &g_rank_status_sink; }
+    __device__ static Tile tile(const Args &a, int t) {
+        Tile T;
+        T.q0 = (int64_t)t * tcp::kM;
+        T.ni = (int)(a.nq - T.q0 < tcp::kM ? a.nq - T.q0 : tcp::kM);
+        T.nb = a.nlist;
+        return T;
+    }
+    __device__ static const float *a_row(const Args &a, const Tile &T, int i) {
+        return i < T.ni ? a.Q + (T.q0 + i) * a.d : nullptr;
+    }
+    __device__ static const float *b_row(const Args &a, const Tile &T, int64_t r) {
+        return r < T.nb ? a.C + r * a.d : nullptr;
+    }
+    struct Epi {
+        float *row;
+        __device__ void begin(const Args &a, const Tile &T, int slot, unsigned char *) {
+            row = slot < T.ni ? a.scores + (T.q0 + slot) * a.ld : nullptr;
+        }
+        __device__ void chunk(const Args &a, const Tile &, int64_t col0, const float (&v)[32], int ncol) {
+            if (!row || ncol <= 0) return;   // ld is a multiple of 32: whole 32-column groups fit
+            float4 *dst = reinterpret_cast<float4 *>(row + col0);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) dst[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+        }
+        __device__ void end(const Args &, const Tile &) {}
+    };
+};
+
+__global__ void __launch_bounds__(tcp::kThreads, 1) k_rank_tc(RankArgs a) {
+    extern __shared__ unsigned char smem_raw[];
+    tcp::run_pipeline<RankMode>(a, smem_raw);
+}
+
+// ---------------------------------------------------------------------------
+// selection: monotone map of fp32 to uint32 (larger float -> larger key)
+__device__ __forceinline__ uint32_t order_key(float s) {
+    const uint32_t u = __float_as_uint(s);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+constexpr int kSelectWarps = 4;
+
+template <int KPL>   // scores per lane: nlist <= 32 * KPL
+__global__ void __launch_bounds__(kSelectWarps * 32) k_select(const float *__restrict__ scores,
+                                                              int64_t ld, int64_t nq, int nlist,
+                                                              int nprobe, int P,
+                                                              int32_t *__restrict__ order,
+                                                              float *__restrict__ cscores) {
+    extern __shared__ __align__(16) unsigned char sel_smem[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    float *bs = reinterpret_cast<float *>(sel_smem) + warp * 2 * P;   // P scores, then P ids
+    int *bc = reinterpret_cast<int *>(bs + P);
+    const int64_t q = (int64_t)blockIdx.x * kSelectWarps + warp;
+    if (q >= nq) return;
+    const float *row = scores + q * ld;
+    float s[KPL];
+    uint32_t key[KPL];
+#pragma unroll
+    for (int j = 0; j < KPL; ++j) {
+        const int c = j * 32 + lane;
+        s[j] = c < nlist ? row[c] : 0.f;
+        key[j] = c < nlist ? order_key(s[j]) : 0u;   // padding ranks below every score
+    }
+    // the largest t with at least nprobe keys >= t is the nprobe-th largest key
+    uint32_t T = 0;
+    for (int b = 31; b >= 0; --b) {
+        const uint32_t t = T | (1u << b);
+        int cnt = 0;
+#pragma unroll
+        for (int j = 0; j < KPL; ++j) cnt += key[j] >= t;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, o);
+        if (cnt >= nprobe) T = t;
+    }
+    int gt = 0;
+#pragma unroll
+    for (int j = 0; j < KPL; ++j) gt += key[j] > T;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) gt += __shfl_xor_sync(0xffffffffu, gt, o);
+    const int ties_wanted = nprobe - gt;   // >= 1: equal keys, lowest ids first
+    // gather, in increasing id order (id = 32 j + lane)
+    const unsigned below = (1u << lane) - 1u;
+    int pos = 0, ties_seen = 0;
+#pragma unroll
+    for (int j = 0; j < KPL; ++j) {
+        const bool tie = key[j] == T && j * 32 + lane < nlist;
+        const unsigned tb = __ballot_sync(0xffffffffu, tie);
+        const bool sel = key[j] > T || (tie && ties_seen + __popc(tb & below) < ties_wanted);
+        const unsigned sb = __ballot_sync(0xffffffffu, sel);
+        if (sel) {
+            const int p = pos + __popc(sb & below);
+            bs[p] = s[j];
+            bc[p] = j * 32 + lane;
+        }
+        pos += __popc(sb);
+        ties_seen += __popc(tb);
+    }
+    for (int p = nprobe + lane; p < P; p += 32) {   // pad to a power of two
+        bs[p] = -__int_as_float(0x7f800000);
+        bc[p] = INT32_MAX;
+    }
+    __syncwarp();
+    // bitonic sort of P entries, first-ranked first
+    for (int k = 2; k <= P; k <<= 1) {
+        for (int j = k >> 1; j > 0; j >>= 1) {
+            for (int i = lane; i < P / 2; i += 32) {
+                const int lo = 2 * i - (i & (j - 1));
+                const int hi = lo + j;
+                const bool up = (lo & k) == 0;
+                const float s0 = bs[lo], s1 = bs[hi];
+                const int c0 = bc[lo], c1 = bc[hi];
+                if (ranks_before(s1, c1, s0, c0) == up) {
+                    bs[lo] = s1;
+                    bc[lo] = c1;
+                    bs[hi] = s0;
+                    bc[hi] = c0;
+                }
+            }
+            __syncwarp();
+        }
+    }
+    for (int p = lane; p < nprobe; p += 32) {
+        order[q * nprobe + p] = bc[p];
+        if (cscores) cscores[q * nprobe + p] = bs[p];
+    }
+}
+
+// ---------------------------------------------------------------------------
+bool rank_tc_supported(int64_t nlist, int nprobe) { return nlist <= kRankTcMaxNlist && nprobe <= nlist; }
+
+int64_t rank_tc_ld(int64_t nlist) { return round_up(nlist, 32); }
+
+int64_t rank_tc_chunk(int64_t nq, int64_t nlist) {
+    const int64_t per_q = rank_tc_ld(nlist) * (int64_t)sizeof(float);
+    int64_t c = kRankScratchBytes / per_q;
+    c = c / tcp::kM * tcp::kM;
+    if (c < tcp::kM) c = tcp::kM;
+    return nq < c ? nq : c;
+}
+
+size_t rank_tc_scratch_bytes(int64_t nq, int64_t nlist) {
+    return (size_t)(rank_tc_chunk(nq, nlist) * rank_tc_ld(nlist) * (int64_t)sizeof(float));
+}
+
+static size_t tc_smem() { return tcp::Geometry<RankMode::kN>::smem_bytes(0); }
+
+static int pow2_at_least(int x) {
+    int p = 1;
+    while (p < x) p <<= 1;
+    return p;
+}
+
+template <int KPL>
+static cudaError_t set_select_attr(int P) {
+    return cudaFuncSetAttribute(k_select<KPL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                kSelectWarps * 2 * P * 4);
+}
+
+cudaError_t prepare_rank_tc(int nprobe) {
+    cudaError_t e = cudaFuncSetAttribute(k_rank_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)tc_smem());
+    const int P = pow2_at_least(nprobe);
+    if (e == cudaSuccess) e = set_select_attr<1>(P);
+    if (e == cudaSuccess) e = set_select_attr<2>(P);
+    if (e == cudaSuccess) e = set_select_attr<4>(P);
+    if (e == cudaSuccess) e = set_select_attr<8>(P);
+    if (e == cudaSuccess) e = set_select_attr<16>(P);
+    if (e == cudaSuccess) e = set_select_attr<32>(P);
+    if (e == cudaSuccess) e = set_select_attr<64>(P);
+    return e;
+}
+
+cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t nlist, int d,
+                            int nprobe, int32_t *order, float *cscores, float *scratch, int *status,
+                            cudaStream_t st) {
+    const int64_t ld = rank_tc_ld(nlist);
+    const int64_t chunk = rank_tc_chunk(nq, nlist);
+    const int P = pow2_at_least(nprobe);
+    const int kpl = pow2_at_least((int)ceil_div(nlist, 32));
+    for (int64_t q0 = 0; q0 < nq; q0 += chunk) {
+        const int64_t n = nq - q0 < chunk ? nq - q0 : chunk;
+        RankArgs a{Q + q0 * d, n, C, nlist, d, scratch, ld, status};
+        const int tiles = (int)ceil_div(n, tcp::kM);
+        k_rank_tc<<<std::min(tiles, num_sms()), tcp::kThreads, tc_smem(), st>>>(a);
+        const unsigned blocks = (unsigned)ceil_div(n, kSelectWarps);
+        const size_t smem = (size_t)kSelectWarps * 2 * P * 4;
+        int32_t *o = order + q0 * nprobe;
+        float *cs = cscores ? cscores + q0 * nprobe : nullptr;
+        switch (kpl) {
+            case 1: k_select<1><<<blocks, kSelectWarps * 32, smem, st>>>(scratch, ld, n, (int)nlist, nprobe, P, o, cs); break;
+            case 2: k_select<2><<<blocks, kSelectWarps * 32, smem, st>>>(scratch, ld, n, (int)nlist, nprobe, P, o, cs); break;
+            case 4: k_select<4><<<blocks, kSelectWarps * 32, smem, st>>>(scratch, ld, n, (int)nlist, nprobe, P, o, cs); break;
+            case 8: k_select<8><<<blocks, kSelectWarps * 32, smem, st>>>(scratch, ld, n, (int)nlist, nprobe, P, o, cs); break;
+            case 16: k_select<16><<<blocks, kSelectWarps * 32, smem, st>>>(scratch, ld, n, (int)nlist, nprobe, P, o, cs); break;
+            case 32: k_select<32><<<blocks, kSelectWarps * 32, smem, st>>>(scratch, ld, n, (int)nlist, nprobe, P, o, cs); break;
+            default: k_select<64><<<blocks, kSelectWarps * 32, smem, st>>>(scratch, ld, n, (int)nlist, nprobe, P, o, cs); break;
+        }
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+}
+
+}  // namespace sieve

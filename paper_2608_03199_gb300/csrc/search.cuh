@@ -39,6 +39,7 @@ struct SearchArgs {
     int tc_min;                         // groups chunks of >= tc_min items go to the
                                         // tensor cores; 0 = SIMT only
     int4 *active;                       // [nq]: query, first item, items
+    float *rank_scratch;                // score table of the tensor-core ranking
     // per-item local results
     int *res_cnt;                       // [cap]
     float *res_s;                       // [cap][k]
@@ -73,6 +74,18 @@ void enqueue_scan_tc(const SearchArgs &a, cudaStream_t st);
 cudaError_t prepare_rank(int nprobe);
 cudaError_t enqueue_rank(const float *Q, int64_t nq, const float *C, int64_t nlist, int d,
                          int nprobe, int32_t *order, float *cscores, cudaStream_t st);
+
+// centroid ranking on the tensor cores (rank_tc.cu) for nlist <= kRankTcMaxNlist:
+// a score table of at most kRankScratchBytes per chunk of queries, then a
+// warp-per-query selection
+constexpr int64_t kRankTcMaxNlist = 2048;
+constexpr int64_t kRankScratchBytes = int64_t(512) << 20;
+bool rank_tc_supported(int64_t nlist, int nprobe);
+size_t rank_tc_scratch_bytes(int64_t nq, int64_t nlist);
+cudaError_t prepare_rank_tc(int nprobe);
+cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t nlist, int d,
+                            int nprobe, int32_t *order, float *cscores, float *scratch, int *status,
+                            cudaStream_t st);
 
 // partition layout (layout_kernels.cu)
 size_t layout_workspace_bytes(int64_t n, int64_t nlist);

@@ -163,7 +163,9 @@ def _nearest(X: torch.Tensor, Cn: torch.Tensor, chunk: int) -> torch.Tensor:
 def build_index(X: torch.Tensor, cfg: Workload, g: torch.Generator, chunk: int = 1 << 16):
     """Spherical k-means centroids [nlist][d] (unit) and exact assignment [n] int32."""
     prev = torch.backends.cuda.matmul.allow_tf32
+    prev_det = torch.are_deterministic_algorithms_enabled()
     torch.backends.cuda.matmul.allow_tf32 = False
+    torch.use_deterministic_algorithms(True, warn_only=True)   # same index on every run
     try:
         n = X.shape[0]
         cap = cfg.train_cap or n
@@ -185,6 +187,7 @@ def build_index(X: torch.Tensor, cfg: Workload, g: torch.Generator, chunk: int =
         assign = _nearest(X, Cn, chunk)
     finally:
         torch.backends.cuda.matmul.allow_tf32 = prev
+        torch.use_deterministic_algorithms(prev_det)
     return Cn.contiguous(), assign
 
 
