@@ -43,13 +43,14 @@ struct ScanMode {
     struct Epi {
         float *ks;
         long long *ki;
-        int kn, item, q, rank;
+        int kn, item, q, rank, slot;
         bool valid;
         long long qid;
         // entry j of thread slot's list sits at [j * kM + slot] (bank-conflict free)
         __device__ float &KS(int j) const { return ks[j * tcp::kM]; }
         __device__ long long &KI(int j) const { return ki[j * tcp::kM]; }
-        __device__ void begin(const Args &a, const Tile &T, int slot, unsigned char *smem) {
+        __device__ void begin(const Args &a, const Tile &T, int slot_, unsigned char *smem) {
+            slot = slot_;
             ks = reinterpret_cast<float *>(smem) + slot;
             ki = reinterpret_cast<long long *>(reinterpret_cast<float *>(smem) + tcp::kM * a.k) + slot;
             kn = 0;
@@ -98,7 +99,7 @@ struct ScanMode {
                     atomicMax(&a.S[q], reach < a.nprobe ? (int)reach : a.nprobe);
                 }
             }
-            if (threadIdx.x == 32 * 12) {   // one epilogue thread per tile counts the work
+            if (slot == 0) {   // one epilogue thread per tile counts the work
                 atomicAdd(&a.ctl->tot_rows, (unsigned long long)T.nb);
                 atomicAdd(&a.ctl->tot_pairs, (unsigned long long)T.nb * (unsigned long long)T.ni);
                 atomicAdd(&a.ctl->tot_rows_tc, (unsigned long long)T.nb);

@@ -1,31 +1,38 @@
 // tc_pipeline.cuh -- a persistent tcgen05 contraction pipeline shared by the
 // grouped scan and the centroid ranking: S = A * B^T for tiles of 128 rows
 // of A (queries) against all rows of a B range (partition rows or
-// centroids), in fp32 accuracy through a 3xTF32 split, handed chunk by chunk
-// to a per-row epilogue.
+// centroids), to fp32 accuracy through an error-compensated fp16 split,
+// handed chunk by chunk to a per-row epilogue.
 //
 // A tile's 128 A rows form the MMA's M side; B streams through in chunks of
-// Mode::kN rows (the MMA N); d is covered in K-blocks of 32 fp32 (one
-// 128-byte swizzle row).  Every operand x is stored as hi = tf32(x) and
-// lo = tf32(x - hi); each K step issues three kind::tf32 MMAs,
-// lo*hi + hi*lo + hi*hi, accumulated in fp32 in tensor memory.  The dropped
-// lo*lo term and the rounding of lo are about 2^-22 of |a_i b_i| each, so a
-// unit-vector similarity is off by at most a few 1e-7.
+// Mode::kN rows (the MMA N); d is covered in K-blocks of 64 elements (one
+// 128-byte swizzle row of fp16).  Every operand x is scaled by 2^8 and stored
+// as hi = fp16(256 x) and lo = fp16(256 x - hi); each K step issues three
+// kind::f16 MMAs, lo*hi + hi*lo + hi*hi, accumulated in fp32 in tensor
+// memory, and the epilogue multiplies by 2^-16 (exact).  For |x| <= 1,
+// |256 x - hi| <= 2^-12 |256 x|, the rounding of lo adds 2^-11 of that, and
+// the dropped lo*lo term is 2^-24 of |256 a 256 b|: a unit-vector similarity
+// is off by a few 1e-7 at most, as with a 3xTF32 split, at half the shared
+// memory bytes per product (the scale keeps lo out of fp16's subnormal range
+// whenever |x| >= 2^-11; below that its absolute error is under 2^-33).
 //
-// Warp roles (416 threads, one block per SM):
-//   warps 0-7   converters: load a stage (128 A half-rows and one K-block of
-//               the B chunk) from global memory, split hi/lo, store both in
-//               the swizzled layout, arrive on the stage's "full" barrier
-//   warp 8      allocates 2 * kN tensor-memory columns (two accumulators);
+// Warp roles (672 threads, one block per SM):
+//   warps 0-15  converters: load one K-block of the tile's 128 A rows and of
+//               the current B chunk from global memory (before waiting for
+//               the stage to free up), split hi/lo, store both in the
+//               swizzled layout, arrive on the stage's "full" barrier
+//   warp 16     allocates 2 * kN tensor-memory columns (two accumulators);
 //               lane 0 issues the MMAs, commits each stage to its "empty"
 //               barrier and each finished chunk to "dfull"
-//   warps 9-12  epilogue: thread i owns tensor-memory lane i = A row i of the
+//   warps 17-20 epilogue: thread i owns tensor-memory lane i = A row i of the
 //               tile; it reads that row's kN scores of a chunk (Mode::Epi),
 //               then releases the accumulator ("dempty")
 // Every mbarrier wait is bounded: a wait that gives up marks the block as
 // aborted (SIEVE_ETIMEOUT in the mode's status word), every role leaves its
 // loop, the issued MMAs are drained (bounded) and tensor memory is freed.
 #pragma once
+
+#include <cuda_fp16.h>
 
 #include "search.cuh"
 #include "tcgen05.cuh"
@@ -34,10 +41,13 @@ namespace sieve {
 namespace tcp {
 
 constexpr int kM = 128;                  // A rows per tile = tensor-memory lanes
-constexpr int kKB = 32;                  // fp32 per K-block
-constexpr int kConvWarps = 8;
-constexpr int kMmaWarp = 8;
-constexpr int kThreads = 13 * 32;
+constexpr int kKB = 64;                  // elements per K-block (128 bytes of fp16)
+constexpr int kConvWarps = 16;
+constexpr int kConvThreads = kConvWarps * 32;
+constexpr int kMmaWarp = 16;
+constexpr float kSplitScale = 256.f;               // operands scaled by 2^8 ...
+constexpr float kUnscale = 1.f / 65536.f;          // ... products by 2^16
+constexpr int kThreads = 21 * 32;
 constexpr int kStages = 2;
 constexpr uint32_t kWaitPolls = 1u << 24;
 constexpr uint32_t A_BYTES = kM * 128;   // one K-block of the tile's A rows
@@ -52,37 +62,34 @@ struct Geometry {
     }
 };
 
-// store NCHUNK 16-byte chunks of a row, starting at logical chunk chunk0, as
-// hi/lo tf32 pairs in the 128-byte swizzled layout (chunk c of row r sits
-// at chunk c ^ (r & 7))
-template <int NCHUNK>
-__device__ __forceinline__ void store_split(unsigned char *hi_tile, unsigned char *lo_tile, int row,
-                                            int chunk0, const float4 (&v)[NCHUNK]) {
-#pragma unroll
-    for (int c = 0; c < NCHUNK; ++c) {
-        const uint32_t off = (uint32_t)row * 128u + (uint32_t)(((chunk0 + c) ^ (row & 7)) << 4);
-        uint4 h, l;
-        h.x = tc::to_tf32(v[c].x);
-        h.y = tc::to_tf32(v[c].y);
-        h.z = tc::to_tf32(v[c].z);
-        h.w = tc::to_tf32(v[c].w);
-        l.x = tc::to_tf32(v[c].x - __uint_as_float(h.x));
-        l.y = tc::to_tf32(v[c].y - __uint_as_float(h.y));
-        l.z = tc::to_tf32(v[c].z - __uint_as_float(h.z));
-        l.w = tc::to_tf32(v[c].w - __uint_as_float(h.w));
-        *reinterpret_cast<uint4 *>(hi_tile + off) = h;
-        *reinterpret_cast<uint4 *>(lo_tile + off) = l;
-    }
+// One unit = 8 consecutive elements of a row = one 16-byte fp16 chunk of the
+// hi and of the lo tile.  Chunk c of row r sits at chunk c ^ (r & 7) (the
+// 128-byte swizzle the descriptors name).
+__device__ __forceinline__ void load_unit(const float *row, int col, int d, float4 &x0, float4 &x1) {
+    const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+    x0 = (row && col < d) ? __ldg(reinterpret_cast<const float4 *>(row + col)) : z;
+    x1 = (row && col + 4 < d) ? __ldg(reinterpret_cast<const float4 *>(row + col + 4)) : z;
 }
 
-template <int NCHUNK>
-__device__ __forceinline__ void load_chunks(const float *row, int col0, int d, float4 (&v)[NCHUNK]) {
-#pragma unroll
-    for (int c = 0; c < NCHUNK; ++c) {
-        const int col = col0 + 4 * c;
-        v[c] = (row && col < d) ? __ldg(reinterpret_cast<const float4 *>(row + col))
-                                : make_float4(0.f, 0.f, 0.f, 0.f);
-    }
+__device__ __forceinline__ void split2(float a, float b, uint32_t &hi, uint32_t &lo) {
+    const float2 f = make_float2(a * kSplitScale, b * kSplitScale);
+    const __half2 h = __float22half2_rn(f);
+    const float2 back = __half22float2(h);
+    const __half2 l = __float22half2_rn(make_float2(f.x - back.x, f.y - back.y));
+    hi = *reinterpret_cast<const uint32_t *>(&h);
+    lo = *reinterpret_cast<const uint32_t *>(&l);
+}
+
+__device__ __forceinline__ void store_unit(unsigned char *hi_tile, unsigned char *lo_tile, int row,
+                                           int chunk, const float4 &x0, const float4 &x1) {
+    const uint32_t off = (uint32_t)row * 128u + (uint32_t)((chunk ^ (row & 7)) << 4);
+    uint4 h, l;
+    split2(x0.x, x0.y, h.x, l.x);
+    split2(x0.z, x0.w, h.y, l.y);
+    split2(x1.x, x1.y, h.z, l.z);
+    split2(x1.z, x1.w, h.w, l.w);
+    *reinterpret_cast<uint4 *>(hi_tile + off) = h;
+    *reinterpret_cast<uint4 *>(lo_tile + off) = l;
 }
 
 // Mode provides: kN; Args; Tile; num_tiles(a); tile(a, t) with fields
@@ -94,10 +101,10 @@ template <class Mode>
 __device__ __forceinline__ void run_pipeline(const typename Mode::Args &a, unsigned char *smem_raw) {
     constexpr int kN = Mode::kN;
     using G = Geometry<kN>;
-    constexpr uint32_t kIdesc = tc::idesc_tf32(kM, kN);
-    constexpr int kBThreadsPerRow = (kConvWarps * 32) / kN;   // 1 (N = 256) or 2 (N = 128)
-    constexpr int kBChunks = 8 / kBThreadsPerRow;
-    static_assert(kBThreadsPerRow * kN == kConvWarps * 32, "one or two converters per B row");
+    constexpr uint32_t kIdesc = tc::idesc_f16(kM, kN);
+    constexpr int kAUnits = kM * 8 / kConvThreads;       // 2 units of A per converter
+    constexpr int kBUnits = kN * 8 / kConvThreads;       // 4 (N = 256) or 2 (N = 128)
+    static_assert(kAUnits * kConvThreads == kM * 8 && kBUnits * kConvThreads == kN * 8, "");
 
     __shared__ __align__(8) uint64_t full_bar[kStages], empty_bar[kStages], dfull_bar[2],
         dempty_bar[2], drain_bar;
@@ -116,7 +123,7 @@ __device__ __forceinline__ void run_pipeline(const typename Mode::Args &a, unsig
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
-            tc::mbar_init(&full_bar[s], kConvWarps * 32);
+            tc::mbar_init(&full_bar[s], kConvThreads);
             tc::mbar_init(&empty_bar[s], 1);
         }
         for (int b = 0; b < 2; ++b) {
@@ -147,8 +154,8 @@ __device__ __forceinline__ void run_pipeline(const typename Mode::Args &a, unsig
     if (warp < kConvWarps) {
         // ---------------- converters ----------------
         const int pt = threadIdx.x;
-        const int arow = pt >> 1, ahalf = pt & 1;
-        const int brow_l = pt / kBThreadsPerRow, bpart = pt % kBThreadsPerRow;
+        const int arow = pt / (8 / kAUnits), achunk0 = (pt % (8 / kAUnits)) * kAUnits;
+        const int brow_l = pt / (8 / kBUnits), bchunk0 = (pt % (8 / kBUnits)) * kBUnits;
         uint32_t s = 0;
         for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) {
             const typename Mode::Tile T = Mode::tile(a, t);
@@ -158,19 +165,22 @@ __device__ __forceinline__ void run_pipeline(const typename Mode::Args &a, unsig
                 const float *brow_p = Mode::b_row(a, T, (int64_t)ch * kN + brow_l);
                 for (int kb = 0; kb < nkb; ++kb, ++s) {
                     const uint32_t st = s & 1u, ph = (s >> 1) & 1u;
+                    float4 bx[kBUnits][2], ax[kAUnits][2];
+#pragma unroll
+                    for (int u = 0; u < kBUnits; ++u)
+                        load_unit(brow_p, kb * kKB + (bchunk0 + u) * 8, d, bx[u][0], bx[u][1]);
+#pragma unroll
+                    for (int u = 0; u < kAUnits; ++u)
+                        load_unit(arow_p, kb * kKB + (achunk0 + u) * 8, d, ax[u][0], ax[u][1]);
                     if (!wait(&empty_bar[st], ph ^ 1u)) goto conv_done;
                     unsigned char *stage = base + st * G::STAGE_BYTES;
-                    {
-                        float4 v[kBChunks];
-                        load_chunks<kBChunks>(brow_p, kb * kKB + bpart * kBChunks * 4, d, v);
-                        store_split<kBChunks>(stage + 2 * A_BYTES, stage + 2 * A_BYTES + G::B_BYTES,
-                                              brow_l, bpart * kBChunks, v);
-                    }
-                    {
-                        float4 u[4];
-                        load_chunks<4>(arow_p, kb * kKB + ahalf * 16, d, u);
-                        store_split<4>(stage, stage + A_BYTES, arow, ahalf * 4, u);
-                    }
+#pragma unroll
+                    for (int u = 0; u < kBUnits; ++u)
+                        store_unit(stage + 2 * A_BYTES, stage + 2 * A_BYTES + G::B_BYTES, brow_l,
+                                   bchunk0 + u, bx[u][0], bx[u][1]);
+#pragma unroll
+                    for (int u = 0; u < kAUnits; ++u)
+                        store_unit(stage, stage + A_BYTES, arow, achunk0 + u, ax[u][0], ax[u][1]);
                     tc::fence_proxy_async_smem();
                     tc::mbar_arrive(&full_bar[st]);
                 }
@@ -198,14 +208,14 @@ __device__ __forceinline__ void run_pipeline(const typename Mode::Args &a, unsig
                         const uint32_t a_hi = sa, a_lo = sa + A_BYTES;
                         const uint32_t b_hi = sa + 2 * A_BYTES, b_lo = b_hi + G::B_BYTES;
 #pragma unroll
-                        for (int ks = 0; ks < kKB / 8; ++ks) {
+                        for (int ks = 0; ks < kKB / 16; ++ks) {   // K = 16 fp16 = 32 bytes per MMA
                             const uint32_t o = ks * 32;
-                            tc::mma_tf32(dt, tc::desc_k_sw128(a_lo + o), tc::desc_k_sw128(b_hi + o),
-                                         kIdesc, (kb > 0 || ks > 0) ? 1u : 0u);
-                            tc::mma_tf32(dt, tc::desc_k_sw128(a_hi + o), tc::desc_k_sw128(b_lo + o),
-                                         kIdesc, 1u);
-                            tc::mma_tf32(dt, tc::desc_k_sw128(a_hi + o), tc::desc_k_sw128(b_hi + o),
-                                         kIdesc, 1u);
+                            tc::mma_f16(dt, tc::desc_k_sw128(a_lo + o), tc::desc_k_sw128(b_hi + o),
+                                        kIdesc, (kb > 0 || ks > 0) ? 1u : 0u);
+                            tc::mma_f16(dt, tc::desc_k_sw128(a_hi + o), tc::desc_k_sw128(b_lo + o),
+                                        kIdesc, 1u);
+                            tc::mma_f16(dt, tc::desc_k_sw128(a_hi + o), tc::desc_k_sw128(b_hi + o),
+                                        kIdesc, 1u);
                         }
                         tc::mma_commit(&empty_bar[st]);
                     }
@@ -239,6 +249,8 @@ __device__ __forceinline__ void run_pipeline(const typename Mode::Args &a, unsig
                 for (int cc = 0; cc < kN / 32; ++cc) {
                     float v[32];
                     tc::tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + buf * kN + cc * 32, v);
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) v[j] *= kUnscale;
                     const int64_t col0 = (int64_t)ch * kN + cc * 32;
                     const int64_t left = T.nb - col0;
                     epi.chunk(a, T, col0, v, left < 32 ? (int)left : 32);
