@@ -50,6 +50,9 @@ def parse():
     ap.add_argument("--skip-e2e", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="target CPU seconds for the oracle sample")
+    ap.add_argument("--ncu-case", choices=("w8", "fixed"), default=None,
+                    help="run exactly one search (W = the config's W, or fixed probe) and exit: "
+                         "a small, single-call target for an ncu capture")
     return ap.parse_args()
 
 
@@ -416,10 +419,29 @@ def run_sieve(args, cfg, world, rank, local):
     return 0
 
 
+def run_ncu_case(args, cfg):
+    """One search call on the benchmark workload, nothing else on the GPU after it."""
+    import paper_2608_03199_gb300 as sieve
+    dev = torch.device("cuda:0")
+    sieve.lib()
+    wl = synth.make_workload(cfg, device=dev)
+    index = sieve.build_layout(wl["X"], wl["assign"], cfg.nlist, wl["centroids"])
+    W = cfg.W if args.ncu_case == "w8" else cfg.nprobe
+    # host-driven rounds: ncu does not profile kernels inside a CUDA graph with
+    # conditional nodes; the kernels and their arguments are the same
+    out = sieve.search(index, wl["Q"], cfg.tau, cfg.k, cfg.nprobe, W, lookahead=True,
+                       query_ids=wl["qids"], stats=True, loop=1)
+    print(json.dumps({"ncu_case": args.ncu_case, "W": W, "rounds": out[4]["rounds"],
+                      "items": out[4]["items"], "pairs": out[4]["pairs"]}))
+    return 0
+
+
 def main():
     args = parse()
     cfg = synth.CONFIGS[args.config]
     world, rank, local = dist_setup(args.gpus)
+    if args.ncu_case:
+        return run_ncu_case(args, cfg)
     if args.impl == "reference":
         return run_reference(args, cfg, world, rank)
     return run_sieve(args, cfg, world, rank, local)

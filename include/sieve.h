@@ -57,6 +57,12 @@ typedef int32_t sieve_status;
  *   ids          device [n] int64, the external id of each stored row
  *   list_offsets device [nlist+1] int64, nondecreasing, [0] = 0, [nlist] = n
  *   centroids    device [nlist][d] fp32 (unit-norm for cosine ranking)
+ *   tc_rows, tc_row_blocks, tc_centroids  (all nullable) the tensor-core
+ *                layout of the rows and of the centroids, made by
+ *                sieve_build_tc_layout from this view; when present (and
+ *                d <= 256) the tensor-core scan and ranking stream them with
+ *                bulk copies instead of splitting fp32 rows on every pass.
+ *                They must describe the same vectors and centroids.
  * d must be a multiple of 4 and at most 1024; every base pointer 16-byte
  * aligned.  Every row must sit in the partition of its nearest centroid
  * (exact assignment, the precondition of Sec. 4.4); the library does not
@@ -70,6 +76,9 @@ typedef struct {
     const int64_t *ids;
     const int64_t *list_offsets;
     const float *centroids;
+    const void *tc_rows;
+    const int64_t *tc_row_blocks;
+    const void *tc_centroids;
 } sieve_index_view;
 
 /* Search parameters (Sec. 4, Sec. 6.1).
@@ -168,6 +177,23 @@ sieve_status sieve_build_layout(const float *X, const int32_t *assign, int64_t n
                                 int64_t nlist, float *X_sorted, int64_t *ids_sorted,
                                 int64_t *list_offsets, void *ws, size_t ws_bytes,
                                 void *stream);
+
+/* Tensor-core layout of an index: the rows of each partition and the
+ * centroids, pre-split for the fp16 contraction (hi = fp16(256 x),
+ * lo = fp16(256 x - hi)) and stored in blocks of 128 rows in the byte order
+ * of the shared-memory operand tiles (4 bytes per element, each partition
+ * padded to a multiple of 128 rows).  Derived data: it changes no result.
+ *   sieve_tc_layout_size   bytes of tc_rows and of tc_centroids for this view
+ *                          (reads list_offsets from the device: synchronous)
+ *   sieve_build_tc_layout  fills tc_rows (device, rows_bytes), tc_row_blocks
+ *                          (device [nlist+1] int64, block offsets of the
+ *                          partitions) and tc_centroids (device, cent_bytes)
+ *                          from ix->vectors, ix->list_offsets, ix->centroids
+ * Every output 256-byte aligned; asynchronous on `stream`. */
+sieve_status sieve_tc_layout_size(const sieve_index_view *ix, size_t *rows_bytes,
+                                  size_t *cent_bytes);
+sieve_status sieve_build_tc_layout(const sieve_index_view *ix, void *tc_rows,
+                                   int64_t *tc_row_blocks, void *tc_centroids, void *stream);
 
 /* Centroid ranking (Sec. 2.3, Sec. 4.1): for every query, the nprobe
  * centroids with the largest inner product, best first; equal scores rank

@@ -41,7 +41,8 @@ class SieveError(RuntimeError):
 class IndexViewC(C.Structure):
     _fields_ = [("n", C.c_int64), ("nlist", C.c_int64), ("d", C.c_int32), ("reserved0", C.c_int32),
                 ("vectors", C.c_void_p), ("ids", C.c_void_p), ("list_offsets", C.c_void_p),
-                ("centroids", C.c_void_p)]
+                ("centroids", C.c_void_p), ("tc_rows", C.c_void_p), ("tc_row_blocks", C.c_void_p),
+                ("tc_centroids", C.c_void_p)]
 
 
 class ParamsC(C.Structure):
@@ -74,6 +75,10 @@ _SIGNATURES = {
                                        C.c_void_p]),
     "sieve_rank_workspace_size": (C.c_int32, [C.POINTER(IndexViewC), C.c_int64, C.c_int32,
                                               C.POINTER(C.c_size_t)]),
+    "sieve_tc_layout_size": (C.c_int32, [C.POINTER(IndexViewC), C.POINTER(C.c_size_t),
+                                         C.POINTER(C.c_size_t)]),
+    "sieve_build_tc_layout": (C.c_int32, [C.POINTER(IndexViewC), C.c_void_p, C.c_void_p, C.c_void_p,
+                                          C.c_void_p]),
     "sieve_rank_partitions": (C.c_int32, [C.POINTER(IndexViewC), C.c_void_p, C.c_int64, C.c_int32,
                                           C.c_void_p, C.c_void_p, C.c_void_p, C.c_size_t,
                                           C.c_void_p]),
@@ -151,11 +156,17 @@ def _need_cuda(t, dtype, name, ndim=None):
 
 @dataclass
 class Index:
-    """A device-resident IVF index in the layout libsieve reads."""
+    """A device-resident IVF index in the layout libsieve reads.
+
+    ``tc_rows`` / ``tc_row_blocks`` / ``tc_centroids`` optionally hold the
+    tensor-core layout (see :func:`add_tc_layout`)."""
     vectors: torch.Tensor        # [n][d] f32, partition-contiguous
     ids: torch.Tensor            # [n] i64
     list_offsets: torch.Tensor   # [nlist+1] i64
     centroids: torch.Tensor      # [nlist][d] f32
+    tc_rows: torch.Tensor | None = None
+    tc_row_blocks: torch.Tensor | None = None
+    tc_centroids: torch.Tensor | None = None
 
     def view(self) -> IndexViewC:
         v = IndexViewC()
@@ -166,7 +177,14 @@ class Index:
         v.ids = self.ids.data_ptr()
         v.list_offsets = self.list_offsets.data_ptr()
         v.centroids = self.centroids.data_ptr()
+        if self.tc_rows is not None:
+            v.tc_rows = self.tc_rows.data_ptr()
+            v.tc_row_blocks = self.tc_row_blocks.data_ptr()
+            v.tc_centroids = self.tc_centroids.data_ptr()
         return v
+
+    def without_tc_layout(self) -> "Index":
+        return Index(self.vectors, self.ids, self.list_offsets, self.centroids)
 
     @property
     def nlist(self):
@@ -177,8 +195,24 @@ class Index:
         return self.vectors.shape[1]
 
 
-def build_layout(X, assign, nlist, centroids, stream=None) -> Index:
-    """Index from rows X [n][d] and their partitions assign [n] (sieve_build_layout).
+def add_tc_layout(index: Index, stream=None) -> Index:
+    """The same index with its tensor-core layout built (sieve_build_tc_layout)."""
+    base = index.without_tc_layout()
+    v = base.view()
+    rb, cb = C.c_size_t(), C.c_size_t()
+    _check(lib().sieve_tc_layout_size(C.byref(v), C.byref(rb), C.byref(cb)), "sieve_tc_layout_size")
+    dev = index.vectors.device
+    rows = torch.empty(max(rb.value, 256), dtype=torch.uint8, device=dev)
+    blocks = torch.empty(index.nlist + 1, dtype=torch.int64, device=dev)
+    cent = torch.empty(max(cb.value, 256), dtype=torch.uint8, device=dev)
+    _check(lib().sieve_build_tc_layout(C.byref(v), _ptr(rows), _ptr(blocks), _ptr(cent),
+                                       _stream(stream)), "sieve_build_tc_layout")
+    return Index(index.vectors, index.ids, index.list_offsets, index.centroids, rows, blocks, cent)
+
+
+def build_layout(X, assign, nlist, centroids, stream=None, tc_layout=True) -> Index:
+    """Index from rows X [n][d] and their partitions assign [n] (sieve_build_layout),
+    with its tensor-core layout unless ``tc_layout`` is False.
 
     ids of the index are the row numbers of X."""
     _need_cuda(X, torch.float32, "X", 2)
@@ -194,7 +228,8 @@ def build_layout(X, assign, nlist, centroids, stream=None) -> Index:
     off = torch.empty(nlist + 1, dtype=torch.int64, device=X.device)
     _check(L.sieve_build_layout(_ptr(X), _ptr(assign), n, d, nlist, _ptr(Xs), _ptr(ids), _ptr(off),
                                 _ptr(ws), nbytes.value, _stream(stream)), "sieve_build_layout")
-    return Index(Xs, ids, off, centroids.contiguous())
+    index = Index(Xs, ids, off, centroids.contiguous())
+    return add_tc_layout(index, stream) if tc_layout else index
 
 
 def rank_partitions(index: Index, Q, nprobe, return_scores=False, stream=None):

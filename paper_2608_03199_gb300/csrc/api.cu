@@ -167,7 +167,7 @@ cudaError_t launch_search_rank(const SearchArgs &a, int rank_tc, cudaStream_t st
     int32_t *order = const_cast<int32_t *>(a.order);
     if (rank_tc)
         return enqueue_rank_tc(a.Q, a.nq, a.C, a.nlist, a.d, a.nprobe, order, nullptr,
-                               a.rank_scratch, &a.ctl->status, st);
+                               a.rank_scratch, &a.ctl->status, st, a.tc_cent);
     return enqueue_rank(a.Q, a.nq, a.C, a.nlist, a.d, a.nprobe, order, nullptr, st);
 }
 
@@ -309,6 +309,14 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
     a.tc_min = p->scan_path == 1 ? 0 : p->scan_path == 2 ? 1 : (p->k <= kTcMaxK ? 24 : 0);
     a.active = reinterpret_cast<int4 *>(ws + L.active);
     a.rank_scratch = L.rank_scratch ? reinterpret_cast<float *>(ws + L.rank_scratch) : nullptr;
+    a.tc_rows = static_cast<const unsigned char *>(ix->tc_rows);
+    a.tc_row_blocks = ix->tc_row_blocks;
+    a.tc_cent = static_cast<const unsigned char *>(ix->tc_centroids);
+    a.tc_stages = (a.tc_min > 0 && a.tc_rows && a.tc_row_blocks) ? scan_bulk_stages(ix->d, p->k) : 0;
+    if (!a.tc_stages) {
+        a.tc_rows = nullptr;
+        a.tc_row_blocks = nullptr;
+    }
     a.res_cnt = reinterpret_cast<int *>(ws + L.res_cnt);
     a.res_s = reinterpret_cast<float *>(ws + L.res_s);
     a.res_id = reinterpret_cast<long long *>(ws + L.res_id);
@@ -322,8 +330,9 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
     const int rank_tc = with_rank && a.rank_scratch != nullptr;
     const size_t smem = scan_smem_bytes(ix->d, p->k);
     SIEVE_CUDA(prepare_scan_kernel(smem));
-    if (a.tc_min > 0) SIEVE_CUDA(prepare_scan_tc(p->k));
-    if (with_rank) SIEVE_CUDA(rank_tc ? prepare_rank_tc(p->nprobe) : prepare_rank(p->nprobe));
+    if (a.tc_min > 0)
+        SIEVE_CUDA(a.tc_stages ? prepare_scan_bulk(ix->d, p->k, a.tc_stages) : prepare_scan_tc(p->k));
+    if (with_rank) SIEVE_CUDA(rank_tc ? prepare_rank_tc(p->nprobe, ix->d) : prepare_rank(p->nprobe));
     const int blocks = scan_blocks_for(smem);
 
     float ms[SIEVE_NKERNELS] = {0};
@@ -461,6 +470,41 @@ sieve_status sieve_build_layout(const float *X, const int32_t *assign, int64_t n
     return bad ? SIEVE_EINVAL : SIEVE_OK;
 }
 
+sieve_status sieve_tc_layout_size(const sieve_index_view *ix, size_t *rows_bytes,
+                                  size_t *cent_bytes) {
+    if (!rows_bytes || !cent_bytes) return SIEVE_EINVAL;
+    sieve_status rc = check_index(ix, true);
+    if (rc != SIEVE_OK) return rc;
+    std::vector<int64_t> off((size_t)ix->nlist + 1);
+    SIEVE_CUDA(cudaMemcpy(off.data(), ix->list_offsets, off.size() * sizeof(int64_t),
+                          cudaMemcpyDeviceToHost));
+    int64_t blocks = 0;
+    for (int64_t p = 0; p < ix->nlist; ++p) {
+        if (off[p + 1] < off[p]) return SIEVE_EINVAL;
+        blocks += ceil_div(off[p + 1] - off[p], kTcRows);
+    }
+    const int64_t per_block = (int64_t)tc_nkb(ix->d) * kTcBlockBytes;
+    *rows_bytes = (size_t)(blocks * per_block);
+    *cent_bytes = (size_t)(ceil_div(ix->nlist, kTcRows) * per_block);
+    return SIEVE_OK;
+}
+
+sieve_status sieve_build_tc_layout(const sieve_index_view *ix, void *tc_rows,
+                                   int64_t *tc_row_blocks, void *tc_centroids, void *stream) {
+    sieve_status rc = check_index(ix, true);
+    if (rc != SIEVE_OK) return rc;
+    if (!tc_rows || !tc_row_blocks || !tc_centroids) return SIEVE_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(tc_rows) | reinterpret_cast<uintptr_t>(tc_centroids)) & 255u)
+        return SIEVE_EINVAL;
+    if ((rc = check_device()) != SIEVE_OK) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    SIEVE_CUDA(launch_tc_layout_rows(ix->vectors, ix->list_offsets, ix->nlist, ix->d, tc_row_blocks,
+                                     static_cast<unsigned char *>(tc_rows), st));
+    SIEVE_CUDA(launch_tc_layout_matrix(ix->centroids, ix->nlist, ix->d,
+                                       static_cast<unsigned char *>(tc_centroids), st));
+    return SIEVE_OK;
+}
+
 sieve_status sieve_rank_workspace_size(const sieve_index_view *ix, int64_t nq, int32_t nprobe,
                                        size_t *bytes) {
     if (!bytes) return SIEVE_EINVAL;
@@ -485,10 +529,11 @@ sieve_status sieve_rank_partitions(const sieve_index_view *ix, const float *Q, i
         if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) ||
             ws_bytes < rank_tc_scratch_bytes(nq, ix->nlist))
             return SIEVE_EWORKSPACE;
-        SIEVE_CUDA(prepare_rank_tc(nprobe));
+        SIEVE_CUDA(prepare_rank_tc(nprobe, ix->d));
         SIEVE_CUDA(enqueue_rank_tc(Q, nq, ix->centroids, ix->nlist, ix->d, nprobe, order, cscores,
                                    static_cast<float *>(ws), nullptr,
-                                   static_cast<cudaStream_t>(stream)));
+                                   static_cast<cudaStream_t>(stream),
+                                   static_cast<const unsigned char *>(ix->tc_centroids)));
     } else {
         SIEVE_CUDA(prepare_rank(nprobe));
         SIEVE_CUDA(enqueue_rank(Q, nq, ix->centroids, ix->nlist, ix->d, nprobe, order, cscores,

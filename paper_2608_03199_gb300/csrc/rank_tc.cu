@@ -13,6 +13,7 @@
 //              the entries above it plus the lowest-id entries equal to it
 //              are gathered, and a warp bitonic network sorts them by
 //              (score desc, id asc).
+#include "tc_bulk.cuh"
 #include "tc_pipeline.cuh"
 
 namespace sieve {
@@ -26,6 +27,7 @@ struct RankArgs {
     float *scores;   // [nq][ld] score table
     int64_t ld;      // row stride of the table, a multiple of 32
     int *status;     // nullable: where a bounded wait that gives up is reported
+    const unsigned char *tc_cent;   // tensor-core layout of the centroids (bulk path)
 };
 
 __device__ int g_rank_status_sink;
@@ -54,6 +56,9 @@ struct RankMode {
     __device__ static const float *b_row(const Args &a, const Tile &T, int64_t r) {
         return r < T.nb ? a.C + r * a.d : nullptr;
     }
+    __device__ static const unsigned char *b_block(const Args &a, const Tile &, int ch) {
+        return a.tc_cent + (int64_t)ch * ((a.d + 63) / 64) * kTcBlockBytes;
+    }
     struct Epi {
         float *row;
         __device__ void begin(const Args &a, const Tile &T, int slot, unsigned char *) {
@@ -72,6 +77,13 @@ struct RankMode {
 __global__ void __launch_bounds__(tcp::kThreads, 1) k_rank_tc(RankArgs a) {
     extern __shared__ unsigned char smem_raw[];
     tcp::run_pipeline<RankMode>(a, smem_raw);
+}
+
+int rank_bulk_stages(int d) { return tcb::stages_for((int)ceil_div(d, 64), 0, 232448 - 128); }
+
+__global__ void __launch_bounds__(tcb::kThreads, 1) k_rank_bulk(RankArgs a, int stages) {
+    extern __shared__ unsigned char smem_raw[];
+    tcb::run_bulk<RankMode>(a, smem_raw, stages);
 }
 
 // ---------------------------------------------------------------------------
@@ -199,9 +211,13 @@ static cudaError_t set_select_attr(int P) {
                                 kSelectWarps * 2 * P * 4);
 }
 
-cudaError_t prepare_rank_tc(int nprobe) {
+cudaError_t prepare_rank_tc(int nprobe, int d) {
     cudaError_t e = cudaFuncSetAttribute(k_rank_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)tc_smem());
+    const int bulk = rank_bulk_stages(d);
+    if (e == cudaSuccess && bulk)
+        e = cudaFuncSetAttribute(k_rank_bulk, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)tcb::smem_bytes((int)ceil_div(d, 64), bulk, 0));
     const int P = pow2_at_least(nprobe);
     if (e == cudaSuccess) e = set_select_attr<1>(P);
     if (e == cudaSuccess) e = set_select_attr<2>(P);
@@ -215,16 +231,21 @@ cudaError_t prepare_rank_tc(int nprobe) {
 
 cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t nlist, int d,
                             int nprobe, int32_t *order, float *cscores, float *scratch, int *status,
-                            cudaStream_t st) {
+                            cudaStream_t st, const unsigned char *tc_cent) {
+    const int bulk_stages = tc_cent ? rank_bulk_stages(d) : 0;
     const int64_t ld = rank_tc_ld(nlist);
     const int64_t chunk = rank_tc_chunk(nq, nlist);
     const int P = pow2_at_least(nprobe);
     const int kpl = pow2_at_least((int)ceil_div(nlist, 32));
     for (int64_t q0 = 0; q0 < nq; q0 += chunk) {
         const int64_t n = nq - q0 < chunk ? nq - q0 : chunk;
-        RankArgs a{Q + q0 * d, n, C, nlist, d, scratch, ld, status};
+        RankArgs a{Q + q0 * d, n, C, nlist, d, scratch, ld, status, tc_cent};
         const int tiles = (int)ceil_div(n, tcp::kM);
-        k_rank_tc<<<std::min(tiles, num_sms()), tcp::kThreads, tc_smem(), st>>>(a);
+        if (bulk_stages)
+            k_rank_bulk<<<std::min(tiles, num_sms()), tcb::kThreads,
+                          tcb::smem_bytes((int)ceil_div(d, 64), bulk_stages, 0), st>>>(a, bulk_stages);
+        else
+            k_rank_tc<<<std::min(tiles, num_sms()), tcp::kThreads, tc_smem(), st>>>(a);
         const unsigned blocks = (unsigned)ceil_div(n, kSelectWarps);
         const size_t smem = (size_t)kSelectWarps * 2 * P * 4;
         int32_t *o = order + q0 * nprobe;

@@ -9,9 +9,12 @@
 // private top-k in shared memory; after p's last chunk it writes the item's
 // local result and, on a hit at rank j, raises the query's stop line to
 // min(j + W, nprobe) (Sec. 4.3).
+#include "tc_bulk.cuh"
 #include "tc_pipeline.cuh"
 
 namespace sieve {
+
+__device__ __forceinline__ int tc_nkb_dev(int d) { return (d + 63) / 64; }
 
 struct ScanMode {
     using Args = SearchArgs;
@@ -38,6 +41,9 @@ struct ScanMode {
     }
     __device__ static const float *b_row(const Args &a, const Tile &T, int64_t r) {
         return r < T.nb ? a.X + (T.r_begin + r) * a.d : nullptr;
+    }
+    __device__ static const unsigned char *b_block(const Args &a, const Tile &T, int ch) {
+        return a.tc_rows + (a.tc_row_blocks[T.p] + ch) * (int64_t)tc_nkb_dev(a.d) * kTcBlockBytes;
     }
 
     struct Epi {
@@ -116,6 +122,27 @@ size_t scan_tc_smem_bytes(int k) {
 __global__ void __launch_bounds__(tcp::kThreads, 1) k_scan_tc(SearchArgs a) {
     extern __shared__ unsigned char smem_raw[];
     tcp::run_pipeline<ScanMode>(a, smem_raw);
+}
+
+static size_t scan_epi_bytes(int k) { return (size_t)tcp::kM * k * (sizeof(float) + sizeof(long long)); }
+
+int scan_bulk_stages(int d, int k) {
+    return tcb::stages_for((int)ceil_div(d, 64), scan_epi_bytes(k), 232448 - 128);
+}
+
+__global__ void __launch_bounds__(tcb::kThreads, 1) k_scan_bulk(SearchArgs a) {
+    extern __shared__ unsigned char smem_raw[];
+    tcb::run_bulk<ScanMode>(a, smem_raw, a.tc_stages);
+}
+
+cudaError_t prepare_scan_bulk(int d, int k, int stages) {
+    return cudaFuncSetAttribute(k_scan_bulk, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)tcb::smem_bytes((int)ceil_div(d, 64), stages, scan_epi_bytes(k)));
+}
+
+void enqueue_scan_bulk(const SearchArgs &a, cudaStream_t st) {
+    k_scan_bulk<<<num_sms(), tcb::kThreads,
+                  tcb::smem_bytes((int)ceil_div(a.d, 64), a.tc_stages, scan_epi_bytes(a.k)), st>>>(a);
 }
 
 cudaError_t prepare_scan_tc(int k) {

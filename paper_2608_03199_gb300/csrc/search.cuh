@@ -40,6 +40,10 @@ struct SearchArgs {
                                         // tensor cores; 0 = SIMT only
     int4 *active;                       // [nq]: query, first item, items
     float *rank_scratch;                // score table of the tensor-core ranking
+    const unsigned char *tc_rows;       // tensor-core layout of the rows (nullable)
+    const int64_t *tc_row_blocks;       // [nlist+1] block offsets of that layout
+    const unsigned char *tc_cent;       // tensor-core layout of the centroids (nullable)
+    int tc_stages;                      // B stages of the bulk pipeline (0 = not used)
     // per-item local results
     int *res_cnt;                       // [cap]
     float *res_s;                       // [cap][k]
@@ -68,6 +72,10 @@ constexpr int kTcTile = 128;       // items per tensor-core tile
 size_t scan_tc_smem_bytes(int k);
 cudaError_t prepare_scan_tc(int k);
 void enqueue_scan_tc(const SearchArgs &a, cudaStream_t st);
+// the same fed from the tensor-core layout by bulk copies (d <= 256)
+int scan_bulk_stages(int d, int k);              // 0 when it does not apply
+cudaError_t prepare_scan_bulk(int d, int k, int stages);
+void enqueue_scan_bulk(const SearchArgs &a, cudaStream_t st);
 
 // centroid ranking (rank_kernel.cu): prepare_rank once before launches or
 // stream capture, then enqueue_rank (a single kernel launch)
@@ -82,10 +90,20 @@ constexpr int64_t kRankTcMaxNlist = 2048;
 constexpr int64_t kRankScratchBytes = int64_t(512) << 20;
 bool rank_tc_supported(int64_t nlist, int nprobe);
 size_t rank_tc_scratch_bytes(int64_t nq, int64_t nlist);
-cudaError_t prepare_rank_tc(int nprobe);
+cudaError_t prepare_rank_tc(int nprobe, int d);
 cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t nlist, int d,
                             int nprobe, int32_t *order, float *cscores, float *scratch, int *status,
-                            cudaStream_t st);
+                            cudaStream_t st, const unsigned char *tc_cent = nullptr);
+int rank_bulk_stages(int d);                     // 0 when the bulk ranking does not apply
+
+// tensor-core layout of partition rows and centroids (tc_layout.cu)
+constexpr int kTcRows = 128;                   // rows per block
+constexpr int64_t kTcBlockBytes = 32768;       // one K-block (64 elements) of a block: hi + lo fp16
+int tc_nkb(int d);
+cudaError_t launch_tc_layout_rows(const float *X, const int64_t *off, int64_t nparts, int d,
+                                  int64_t *blk_off, unsigned char *out, cudaStream_t st);
+cudaError_t launch_tc_layout_matrix(const float *X, int64_t nrows, int d, unsigned char *out,
+                                    cudaStream_t st);
 
 // partition layout (layout_kernels.cu)
 size_t layout_workspace_bytes(int64_t n, int64_t nlist);

@@ -558,7 +558,12 @@ cudaError_t launch_round(const SearchArgs &a, size_t scan_smem, int scan_blocks,
     k_scatter<<<scatter_blocks, 256, 0, st>>>(a);
     end();
     begin();
-    if (a.tc_min > 0) enqueue_scan_tc(a, st);
+    if (a.tc_min > 0) {
+        if (a.tc_stages)
+            enqueue_scan_bulk(a, st);
+        else
+            enqueue_scan_tc(a, st);
+    }
     end();
     begin();
     k_scan<<<scan_blocks, kThreads, scan_smem, st>>>(a);

@@ -1,0 +1,260 @@
+// tc_bulk.cuh -- the tensor-core contraction fed from the tensor-core layout
+// (tc_layout.cu): S = A * B^T for tiles of 128 A rows (queries) against every
+// block of 128 B rows (a partition's rows, or the centroids), with the same
+// scaled fp16 split and the same per-row epilogues as tc_pipeline.cuh.
+//
+// The B operand arrives pre-split, in tile byte order, so one 32 KB bulk copy
+// per (block, K-block) lands a stage (hi then lo) in shared memory, several
+// stages deep, with no thread touching it.  The tile's 128 A rows are split
+// once per tile into a resident shared-memory copy of all K-blocks (d <= 256),
+// published K-block by K-block so the MMAs start before the whole of A is in.
+//
+// Warp roles (704 threads, one block per SM):
+//   warps 0-15  A converters: per tile, load the 128 A rows (all K-blocks at
+//               once, one float4 per row per thread), wait until the previous
+//               tile's MMAs are done with A ("a_empty"), split and store, and
+//               publish each K-block ("a_full[kb]")
+//   warp 16     lane 0 issues the bulk copies of the B stages ("b_full" with
+//               the transfer byte count; waits on "b_empty")
+//   warp 17     allocates 256 tensor-memory columns (two 128-column
+//               accumulators); lane 0 issues three kind::f16 MMAs per K step
+//   warps 18-21 epilogue: thread i owns tensor-memory lane i = A row i; it
+//               rescales its row of a chunk by 2^-16 and hands it to Mode::Epi
+// Every wait is bounded; giving up sets SIEVE_ETIMEOUT in the mode's status
+// word, all roles leave their loops, the issued MMAs and copies are drained
+// (bounded) and tensor memory is freed.
+#pragma once
+
+#include <cuda_fp16.h>
+
+#include "search.cuh"
+#include "tc_pipeline.cuh"
+#include "tcgen05.cuh"
+
+namespace sieve {
+namespace tcb {
+
+constexpr int kN = 128;                       // B rows per chunk = MMA N = tensor-layout block
+constexpr int kAConvWarps = 16;
+constexpr int kAConvThreads = kAConvWarps * 32;
+constexpr int kProducerWarp = 16;
+constexpr int kMmaWarp = 17;
+constexpr int kThreads = 22 * 32;
+constexpr int kMaxKb = 4;                     // resident A: d <= 256
+constexpr int kMaxStages = 4;
+constexpr uint32_t kKbBytes = 32768;          // one K-block of 128 rows: hi 16 KB + lo 16 KB
+constexpr uint32_t kTmemCols = 2 * kN;
+constexpr uint32_t kWaitPolls = 1u << 24;
+
+// shared memory: 1 KB alignment slack, resident A (nkb K-blocks), the B stages,
+// then the epilogue's bytes
+__host__ __device__ inline size_t smem_bytes(int nkb, int stages, size_t epi_bytes) {
+    return 1024 + (size_t)nkb * kKbBytes + (size_t)stages * kKbBytes + epi_bytes;
+}
+
+// B stages that fit beside A and the epilogue (0 if fewer than two fit)
+inline int stages_for(int nkb, size_t epi_bytes, size_t smem_limit) {
+    if (nkb > kMaxKb) return 0;
+    const size_t base = smem_bytes(nkb, 0, epi_bytes);
+    if (smem_limit < base) return 0;
+    int s = (int)((smem_limit - base) / kKbBytes);
+    if (s > kMaxStages) s = kMaxStages;
+    return s >= 2 ? s : 0;
+}
+
+// Mode provides (in addition to what tc_pipeline.cuh asks): b_block(a, T, ch)
+// = pointer to the tensor-layout bytes of the tile's ch-th block of B rows.
+template <class Mode>
+__device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned char *smem_raw,
+                                         int stages) {
+    constexpr uint32_t kIdesc = tc::idesc_f16(tcp::kM, kN);
+    __shared__ __align__(8) uint64_t a_full[kMaxKb], a_empty, b_full[kMaxStages],
+        b_empty[kMaxStages], dfull_bar[2], dempty_bar[2], drain_bar;
+    __shared__ uint32_t tmem_slot;
+    __shared__ int s_abort;
+
+    unsigned char *base = reinterpret_cast<unsigned char *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int n_tiles = Mode::num_tiles(a);
+    const int d = Mode::d(a);
+    const int nkb = (int)ceil_div(d, 64);
+    unsigned char *A = base;                                   // nkb x 32 KB
+    unsigned char *Bst = base + (size_t)nkb * kKbBytes;        // stages x 32 KB
+    unsigned char *epi_smem = Bst + (size_t)stages * kKbBytes;
+    int *status = Mode::status(a);
+
+    if (threadIdx.x == 0) {
+        for (int kb = 0; kb < kMaxKb; ++kb) tc::mbar_init(&a_full[kb], kAConvThreads);
+        tc::mbar_init(&a_empty, 1);
+        for (int s = 0; s < kMaxStages; ++s) {
+            tc::mbar_init(&b_full[s], 1);
+            tc::mbar_init(&b_empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            tc::mbar_init(&dfull_bar[b], 1);
+            tc::mbar_init(&dempty_bar[b], 4 * 32);
+        }
+        tc::mbar_init(&drain_bar, 1);
+        s_abort = 0;
+        tc::mbar_init_fence();
+    }
+    if (warp == kMmaWarp) tc::tmem_alloc(&tmem_slot, kTmemCols);
+    tc::fence_before_sync();
+    __syncthreads();
+    tc::fence_after_sync();
+    const uint32_t tmem = tmem_slot;
+
+    auto wait = [&](uint64_t *bar, uint32_t parity) -> bool {
+        for (uint32_t it = 0; it < kWaitPolls; ++it) {
+            if (tc::mbar_try_wait(bar, parity)) return true;
+            if ((it & 255u) == 255u && *(volatile int *)&s_abort) return false;
+        }
+        atomicExch(&s_abort, 1);
+        atomicExch(status, SIEVE_ETIMEOUT);
+        return false;
+    };
+
+    if (warp < kAConvWarps) {
+        // ---------------- A converters ----------------
+        const int f = threadIdx.x & 15;                // float4 of a K-block
+        const int r0 = threadIdx.x >> 4;               // rows r0 + 32 i
+        uint32_t u = 0;                                // tiles with B rows seen so far
+        for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) {
+            const typename Mode::Tile T = Mode::tile(a, t);
+            if (T.nb <= 0) continue;
+            float4 x[kMaxKb][4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const float *row = Mode::a_row(a, T, r0 + 32 * i);
+#pragma unroll
+                for (int kb = 0; kb < kMaxKb; ++kb)
+                    x[kb][i] = kb < nkb ? tcp::load_f4(row, kb * 64 + 4 * f, d)
+                                        : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+            if (!wait(&a_empty, (u & 1u) ^ 1u)) break;
+#pragma unroll
+            for (int kb = 0; kb < kMaxKb; ++kb) {
+                if (kb >= nkb) break;
+                unsigned char *blk = A + (size_t)kb * kKbBytes;
+#pragma unroll
+                for (int i = 0; i < 4; ++i) tcp::store_f4(blk, blk + kKbBytes / 2, r0 + 32 * i, f, x[kb][i]);
+                tc::fence_proxy_async_smem();
+                tc::mbar_arrive(&a_full[kb]);
+            }
+            ++u;
+        }
+    } else if (warp == kProducerWarp) {
+        // ---------------- B producer ----------------
+        if (lane == 0) {
+            uint32_t s = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; ok && t < n_tiles; t += gridDim.x) {
+                const typename Mode::Tile T = Mode::tile(a, t);
+                const int nch = (int)ceil_div(T.nb, kN);
+                for (int ch = 0; ok && ch < nch; ++ch) {
+                    const unsigned char *src = Mode::b_block(a, T, ch);
+                    for (int kb = 0; kb < nkb; ++kb) {
+                        const uint32_t st = s % stages, ph = (s / stages) & 1u;
+                        if (!(ok = wait(&b_empty[st], ph ^ 1u))) break;
+                        tc::mbar_arrive_expect_tx(&b_full[st], kKbBytes);
+                        tc::bulk_g2s(Bst + (size_t)st * kKbBytes, src + (size_t)kb * kKbBytes, kKbBytes,
+                                     &b_full[st]);
+                        ++s;
+                    }
+                }
+            }
+            // no copy may still be landing when the block exits: wait (bounded)
+            // for the last copy issued into each stage
+            for (uint32_t j = s > (uint32_t)stages ? s - stages : 0; j < s; ++j)
+                for (uint32_t it = 0; it < kWaitPolls; ++it)
+                    if (tc::mbar_try_wait(&b_full[j % stages], (j / stages) & 1u)) break;
+        }
+        __syncwarp();
+    } else if (warp == kMmaWarp) {
+        // ---------------- MMA issuer ----------------
+        if (lane == 0) {
+            uint32_t s = 0, c = 0, u = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; ok && t < n_tiles; t += gridDim.x) {
+                const typename Mode::Tile T = Mode::tile(a, t);
+                const int nch = (int)ceil_div(T.nb, kN);
+                if (nch == 0) continue;
+                for (int ch = 0; ok && ch < nch; ++ch, ++c) {
+                    const uint32_t buf = c & 1u, dph = (c >> 1) & 1u;
+                    if (!(ok = wait(&dempty_bar[buf], dph ^ 1u))) break;
+                    tc::fence_after_sync();
+                    const uint32_t dt = tmem + buf * kN;
+                    for (int kb = 0; kb < nkb; ++kb, ++s) {
+                        const uint32_t st = s % stages, ph = (s / stages) & 1u;
+                        if (ch == 0 && !(ok = wait(&a_full[kb], u & 1u))) break;
+                        if (!(ok = wait(&b_full[st], ph))) break;
+                        tc::fence_after_sync();
+                        const uint32_t a_hi = tc::smem_u32(A + (size_t)kb * kKbBytes);
+                        const uint32_t a_lo = a_hi + kKbBytes / 2;
+                        const uint32_t b_hi = tc::smem_u32(Bst + (size_t)st * kKbBytes);
+                        const uint32_t b_lo = b_hi + kKbBytes / 2;
+#pragma unroll
+                        for (int ks = 0; ks < 4; ++ks) {   // K = 16 fp16 = 32 bytes per MMA
+                            const uint32_t o = ks * 32;
+                            tc::mma_f16(dt, tc::desc_k_sw128(a_lo + o), tc::desc_k_sw128(b_hi + o), kIdesc,
+                                        (kb > 0 || ks > 0) ? 1u : 0u);
+                            tc::mma_f16(dt, tc::desc_k_sw128(a_hi + o), tc::desc_k_sw128(b_lo + o), kIdesc, 1u);
+                            tc::mma_f16(dt, tc::desc_k_sw128(a_hi + o), tc::desc_k_sw128(b_hi + o), kIdesc, 1u);
+                        }
+                        tc::mma_commit(&b_empty[st]);
+                    }
+                    if (ok) tc::mma_commit(&dfull_bar[buf]);
+                }
+                if (ok) tc::mma_commit(&a_empty);   // A may be overwritten once these are done
+                ++u;
+            }
+            tc::mma_commit(&drain_bar);
+            for (uint32_t it = 0; it < kWaitPolls; ++it)
+                if (tc::mbar_try_wait(&drain_bar, 0u)) break;
+        }
+        __syncwarp();
+    } else {
+        // ---------------- epilogue ----------------
+        const int quarter = warp & 3;
+        const int slot = quarter * 32 + lane;
+        uint32_t c = 0;
+        bool ok = true;
+        typename Mode::Epi epi;
+        for (int t = blockIdx.x; ok && t < n_tiles; t += gridDim.x) {
+            const typename Mode::Tile T = Mode::tile(a, t);
+            const int nch = (int)ceil_div(T.nb, kN);
+            epi.begin(a, T, slot, epi_smem);
+            for (int ch = 0; ch < nch; ++ch, ++c) {
+                const uint32_t buf = c & 1u, dph = (c >> 1) & 1u;
+                ok = __all_sync(0xffffffffu, wait(&dfull_bar[buf], dph));
+                if (!ok) break;
+                tc::fence_after_sync();
+#pragma unroll 1
+                for (int cc = 0; cc < kN / 32; ++cc) {
+                    float v[32];
+                    tc::tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + buf * kN + cc * 32, v);
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) v[j] *= tcp::kUnscale;
+                    const int64_t col0 = (int64_t)ch * kN + cc * 32;
+                    const int64_t left = T.nb - col0;
+                    epi.chunk(a, T, col0, v, left < 32 ? (int)left : 32);
+                }
+                tc::fence_before_sync();
+                tc::mbar_arrive(&dempty_bar[buf]);
+            }
+            if (!ok) break;
+            epi.end(a, T);
+        }
+    }
+
+    tc::fence_before_sync();
+    __syncthreads();
+    if (warp == kMmaWarp) {
+        tc::fence_after_sync();
+        tc::tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+}  // namespace tcb
+}  // namespace sieve

@@ -62,13 +62,14 @@ struct Geometry {
     }
 };
 
-// One unit = 8 consecutive elements of a row = one 16-byte fp16 chunk of the
-// hi and of the lo tile.  Chunk c of row r sits at chunk c ^ (r & 7) (the
-// 128-byte swizzle the descriptors name).
-__device__ __forceinline__ void load_unit(const float *row, int col, int d, float4 &x0, float4 &x1) {
-    const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
-    x0 = (row && col < d) ? __ldg(reinterpret_cast<const float4 *>(row + col)) : z;
-    x1 = (row && col + 4 < d) ? __ldg(reinterpret_cast<const float4 *>(row + col + 4)) : z;
+// A converter thread handles one float4 (4 consecutive elements) of a row at
+// a time: it becomes 8 bytes of fp16 in the hi tile and 8 in the lo tile, one
+// half of a 16-byte chunk.  Chunk c of row r sits at chunk c ^ (r & 7) (the
+// 128-byte swizzle the descriptors name).  Sixteen consecutive threads cover
+// one row's K-block, so a warp reads two rows' 256 contiguous bytes each.
+__device__ __forceinline__ float4 load_f4(const float *row, int col, int d) {
+    return (row && col < d) ? __ldg(reinterpret_cast<const float4 *>(row + col))
+                            : make_float4(0.f, 0.f, 0.f, 0.f);
 }
 
 __device__ __forceinline__ void split2(float a, float b, uint32_t &hi, uint32_t &lo) {
@@ -80,16 +81,16 @@ __device__ __forceinline__ void split2(float a, float b, uint32_t &hi, uint32_t 
     lo = *reinterpret_cast<const uint32_t *>(&l);
 }
 
-__device__ __forceinline__ void store_unit(unsigned char *hi_tile, unsigned char *lo_tile, int row,
-                                           int chunk, const float4 &x0, const float4 &x1) {
-    const uint32_t off = (uint32_t)row * 128u + (uint32_t)((chunk ^ (row & 7)) << 4);
-    uint4 h, l;
-    split2(x0.x, x0.y, h.x, l.x);
-    split2(x0.z, x0.w, h.y, l.y);
-    split2(x1.x, x1.y, h.z, l.z);
-    split2(x1.z, x1.w, h.w, l.w);
-    *reinterpret_cast<uint4 *>(hi_tile + off) = h;
-    *reinterpret_cast<uint4 *>(lo_tile + off) = l;
+// f = index of the float4 within the row's K-block (0..15)
+__device__ __forceinline__ void store_f4(unsigned char *hi_tile, unsigned char *lo_tile, int row,
+                                         int f, const float4 &x) {
+    const uint32_t off =
+        (uint32_t)row * 128u + (uint32_t)((((f >> 1) ^ (row & 7)) << 4) | ((f & 1) << 3));
+    uint2 h, l;
+    split2(x.x, x.y, h.x, l.x);
+    split2(x.z, x.w, h.y, l.y);
+    *reinterpret_cast<uint2 *>(hi_tile + off) = h;
+    *reinterpret_cast<uint2 *>(lo_tile + off) = l;
 }
 
 // Mode provides: kN; Args; Tile; num_tiles(a); tile(a, t) with fields
@@ -102,9 +103,10 @@ __device__ __forceinline__ void run_pipeline(const typename Mode::Args &a, unsig
     constexpr int kN = Mode::kN;
     using G = Geometry<kN>;
     constexpr uint32_t kIdesc = tc::idesc_f16(kM, kN);
-    constexpr int kAUnits = kM * 8 / kConvThreads;       // 2 units of A per converter
-    constexpr int kBUnits = kN * 8 / kConvThreads;       // 4 (N = 256) or 2 (N = 128)
-    static_assert(kAUnits * kConvThreads == kM * 8 && kBUnits * kConvThreads == kN * 8, "");
+    constexpr int kRowsPerPass = kConvThreads / 16;      // 32 rows per pass of all converters
+    constexpr int kAPasses = kM / kRowsPerPass;          // 4
+    constexpr int kBPasses = kN / kRowsPerPass;          // 8 (N = 256) or 4 (N = 128)
+    static_assert(kAPasses * kRowsPerPass == kM && kBPasses * kRowsPerPass == kN, "");
 
     __shared__ __align__(8) uint64_t full_bar[kStages], empty_bar[kStages], dfull_bar[2],
         dempty_bar[2], drain_bar;
@@ -153,34 +155,34 @@ __device__ __forceinline__ void run_pipeline(const typename Mode::Args &a, unsig
 
     if (warp < kConvWarps) {
         // ---------------- converters ----------------
-        const int pt = threadIdx.x;
-        const int arow = pt / (8 / kAUnits), achunk0 = (pt % (8 / kAUnits)) * kAUnits;
-        const int brow_l = pt / (8 / kBUnits), bchunk0 = (pt % (8 / kBUnits)) * kBUnits;
+        const int f = threadIdx.x & 15;          // float4 of the K-block
+        const int r0 = threadIdx.x >> 4;         // first row; rows r0 + 32 i
         uint32_t s = 0;
         for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) {
             const typename Mode::Tile T = Mode::tile(a, t);
             const int nch = (int)ceil_div(T.nb, kN);
-            const float *arow_p = Mode::a_row(a, T, arow);
+            const float *arow_p[kAPasses];
+#pragma unroll
+            for (int i = 0; i < kAPasses; ++i) arow_p[i] = Mode::a_row(a, T, r0 + kRowsPerPass * i);
             for (int ch = 0; ch < nch; ++ch) {
-                const float *brow_p = Mode::b_row(a, T, (int64_t)ch * kN + brow_l);
                 for (int kb = 0; kb < nkb; ++kb, ++s) {
                     const uint32_t st = s & 1u, ph = (s >> 1) & 1u;
-                    float4 bx[kBUnits][2], ax[kAUnits][2];
+                    const int col = kb * kKB + 4 * f;
+                    float4 bx[kBPasses], ax[kAPasses];
 #pragma unroll
-                    for (int u = 0; u < kBUnits; ++u)
-                        load_unit(brow_p, kb * kKB + (bchunk0 + u) * 8, d, bx[u][0], bx[u][1]);
+                    for (int i = 0; i < kBPasses; ++i)
+                        bx[i] = load_f4(Mode::b_row(a, T, (int64_t)ch * kN + r0 + kRowsPerPass * i), col, d);
 #pragma unroll
-                    for (int u = 0; u < kAUnits; ++u)
-                        load_unit(arow_p, kb * kKB + (achunk0 + u) * 8, d, ax[u][0], ax[u][1]);
+                    for (int i = 0; i < kAPasses; ++i) ax[i] = load_f4(arow_p[i], col, d);
                     if (!wait(&empty_bar[st], ph ^ 1u)) goto conv_done;
                     unsigned char *stage = base + st * G::STAGE_BYTES;
 #pragma unroll
-                    for (int u = 0; u < kBUnits; ++u)
-                        store_unit(stage + 2 * A_BYTES, stage + 2 * A_BYTES + G::B_BYTES, brow_l,
-                                   bchunk0 + u, bx[u][0], bx[u][1]);
+                    for (int i = 0; i < kBPasses; ++i)
+                        store_f4(stage + 2 * A_BYTES, stage + 2 * A_BYTES + G::B_BYTES,
+                                 r0 + kRowsPerPass * i, f, bx[i]);
 #pragma unroll
-                    for (int u = 0; u < kAUnits; ++u)
-                        store_unit(stage, stage + A_BYTES, arow, achunk0 + u, ax[u][0], ax[u][1]);
+                    for (int i = 0; i < kAPasses; ++i)
+                        store_f4(stage, stage + A_BYTES, r0 + kRowsPerPass * i, f, ax[i]);
                     tc::fence_proxy_async_smem();
                     tc::mbar_arrive(&full_bar[st]);
                 }

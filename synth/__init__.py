@@ -32,9 +32,14 @@ in for them with the shapes of the evaluated configurations:
 from __future__ import annotations
 
 import math
+import os
 from dataclasses import dataclass, field, replace
 
-import torch
+# deterministic cuBLAS reductions for the k-means matmuls (read when cuBLAS
+# starts, so this must precede the first GPU matmul)
+os.environ.setdefault("CUBLAS_WORKSPACE_CONFIG", ":4096:8")
+
+import torch  # noqa: E402
 
 
 @dataclass(frozen=True)

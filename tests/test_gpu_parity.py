@@ -285,3 +285,79 @@ def test_invalid_arguments_raise(tiny, g_tiny, dev):
     with pytest.raises(sieve.SieveError) as e:
         sieve.search(g_tiny, Q, 0.9, 10, 16, 4, workspace=tiny_ws)
     assert e.value.status == -3
+
+
+# ---------------------------------------------------------------------------
+# tensor-core layout
+
+
+def np_tc_layout(X, off, d):
+    """The tensor-core layout written independently with numpy: blocks of 128
+    rows, per K-block of 64 elements 16 KB hi fp16 + 16 KB lo fp16 with
+    hi = fp16(256 x), lo = fp16(256 x - hi); 16-byte chunk c of row r at
+    chunk c ^ (r & 7); rows past a partition's end are zero."""
+    nkb = (d + 63) // 64
+    parts = []
+    for p in range(len(off) - 1):
+        rows = X[off[p]:off[p + 1]].astype(np.float32)
+        nb = -(-len(rows) // 128)
+        pad = np.zeros((nb * 128, nkb * 64), np.float32)
+        pad[:len(rows), :d] = rows
+        for b in range(nb):
+            for kb in range(nkb):
+                blk = pad[b * 128:(b + 1) * 128, kb * 64:(kb + 1) * 64] * np.float32(256)
+                hi = blk.astype(np.float16)
+                lo = (blk - hi.astype(np.float32)).astype(np.float16)
+                out = []
+                for t in (hi, lo):
+                    tile = np.zeros((128, 8, 8), np.float16)
+                    for c in range(8):
+                        for r in range(128):
+                            tile[r, c ^ (r & 7)] = t[r, c * 8:(c + 1) * 8]
+                    out.append(tile.reshape(-1).view(np.uint8))
+                parts.append(np.concatenate(out))
+    return np.concatenate(parts) if parts else np.zeros(0, np.uint8)
+
+
+def test_tc_layout_bytes(deep, g_deep):
+    assert g_deep.tc_rows is not None
+    off = g_deep.list_offsets.cpu().numpy()
+    X = g_deep.vectors.cpu().numpy()
+    ref = np_tc_layout(X, off, X.shape[1])
+    got = g_deep.tc_rows.cpu().numpy()[:ref.size]
+    assert got.size == ref.size and np.array_equal(got, ref)
+    nb = [-(-(off[p + 1] - off[p]) // 128) for p in range(len(off) - 1)]
+    assert (g_deep.tc_row_blocks.cpu().numpy() == np.concatenate([[0], np.cumsum(nb)])).all()
+    C = g_deep.centroids.cpu().numpy()
+    refc = np_tc_layout(C, np.array([0, C.shape[0]]), C.shape[1])
+    assert np.array_equal(g_deep.tc_centroids.cpu().numpy()[:refc.size], refc)
+
+
+@pytest.mark.parametrize("which", ["tiny", "deep"])
+def test_bulk_path_equals_converter_path(which, tiny, g_tiny, deep, g_deep):
+    """The tensor-core scan fed by bulk copies of the pre-split layout computes
+    the same products in the same order as the one that splits fp32 rows on
+    the fly: identical ids, counts and probes, scores within 1e-6."""
+    w, g = (tiny, g_tiny) if which == "tiny" else (deep, g_deep)
+    c = w["cfg"]
+    a = run(g, w["Q"], w["qids"], c.tau, c.k, c.nprobe, c.W, scan_path="tensor")
+    b = run(g.without_tc_layout(), w["Q"], w["qids"], c.tau, c.k, c.nprobe, c.W, scan_path="tensor")
+    for key in ("ids", "count", "probes"):
+        assert np.array_equal(a[key], b[key]), key
+    valid = np.arange(c.k)[None, :] < a["count"][:, None]
+    assert np.abs(a["scores"] - b["scores"])[valid].max(initial=0) <= 1e-6
+
+
+def test_wide_rows_fall_back_and_match(dev):
+    """d = 320 is beyond the resident-A limit of the bulk pipeline: the search
+    uses the converter pipeline even with a layout present, and matches the
+    oracle."""
+    import synth
+    cfg = synth.scaled("tiny", n=4_000, d=320, ncomp=8, nlist=16, nq=150, dup_frac=0.1,
+                       dup_counts=("uniform", 1, 4), dup_sigma=(0.005, 0.02), tau=0.9,
+                       nprobe=8, W=2, seed=21)
+    w = synth.to_numpy(synth.make_workload(cfg))
+    gidx = gpu_index(w, dev)
+    assert gidx.tc_rows is not None
+    for path in ("tensor", "auto"):
+        check(w, gidx, w["Q"], w["qids"], cfg.tau, cfg.k, cfg.nprobe, cfg.W, 1, scan_path=path)
