@@ -172,16 +172,16 @@ def roofline(prof, cfg, dev):
     launches = max(1, kl[top])
     ms_per_launch = km[top] / launches
     out = {"kernel": f"k_{top}", "launches": kl[top], "ms_per_launch": ms_per_launch}
-    # TF32 dense peak: the measured bf16 cuBLAS peak x the nominal TF32/BF16 ratio (1.1 / 2.25)
-    tf32_tflops = peaks.get("bf16_tflops", 1889.4) * (1.1 / 2.25)
+    # fp16 dense peak: the measured bf16 cuBLAS peak (fp16 and bf16 share the
+    # nominal 2.25 PFLOP/s rate); the burst figure, as the kernel is timed alone
+    f16_tflops = peaks.get("bf16_tflops", 1889.4)
     if top == "scan_tc":
         flops = 2.0 * d * prof["pairs_tc"]
         ach = flops / launches / (ms_per_launch * 1e-3) / 1e12
-        out.update(bound="tensor", achieved=ach, peak=tf32_tflops / 3, unit="TFLOP/s",
-                   frac=ach / (tf32_tflops / 3),
-                   peak_source=(f"3xTF32: three TF32 MMAs per product; TF32 dense peak "
-                                f"{tf32_tflops:.0f} TFLOP/s = measured bf16 "
-                                f"{peaks.get('bf16_tflops', 1889.4):.0f} x 1.1/2.25 (of measured), "
+        out.update(bound="tensor", achieved=ach, peak=f16_tflops / 3, unit="TFLOP/s",
+                   frac=ach / (f16_tflops / 3),
+                   peak_source=(f"fp16 split: three kind::f16 MMAs per product; fp16 dense peak "
+                                f"{f16_tflops:.0f} TFLOP/s = measured bf16 cuBLAS burst (of measured), "
                                 f"so the algorithmic peak is a third of it"),
                    tensor_pipe_tflops=3 * ach)
     elif top == "scan":

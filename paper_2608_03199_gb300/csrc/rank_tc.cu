@@ -64,11 +64,14 @@ struct RankMode {
         __device__ void begin(const Args &a, const Tile &T, int slot, unsigned char *) {
             row = slot < T.ni ? a.scores + (T.q0 + slot) * a.ld : nullptr;
         }
+        // v holds the chunk's raw accumulator values: scores x 2^16
         __device__ void chunk(const Args &a, const Tile &, int64_t col0, const float (&v)[32], int ncol) {
             if (!row || ncol <= 0) return;   // ld is a multiple of 32: whole 32-column groups fit
+            constexpr float kS = 1.f / 65536.f;
             float4 *dst = reinterpret_cast<float4 *>(row + col0);
 #pragma unroll
-            for (int j = 0; j < 8; ++j) dst[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+            for (int j = 0; j < 8; ++j)
+                dst[j] = make_float4(v[4 * j] * kS, v[4 * j + 1] * kS, v[4 * j + 2] * kS, v[4 * j + 3] * kS);
         }
         __device__ void end(const Args &, const Tile &) {}
     };
@@ -217,7 +220,7 @@ cudaError_t prepare_rank_tc(int nprobe, int d) {
     const int bulk = rank_bulk_stages(d);
     if (e == cudaSuccess && bulk)
         e = cudaFuncSetAttribute(k_rank_bulk, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)tcb::smem_bytes((int)ceil_div(d, 64), bulk, 0));
+                                 (int)tcb::smem_bytes(bulk, 0));
     const int P = pow2_at_least(nprobe);
     if (e == cudaSuccess) e = set_select_attr<1>(P);
     if (e == cudaSuccess) e = set_select_attr<2>(P);
@@ -243,7 +246,7 @@ cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t 
         const int tiles = (int)ceil_div(n, tcp::kM);
         if (bulk_stages)
             k_rank_bulk<<<std::min(tiles, num_sms()), tcb::kThreads,
-                          tcb::smem_bytes((int)ceil_div(d, 64), bulk_stages, 0), st>>>(a, bulk_stages);
+                          tcb::smem_bytes(bulk_stages, 0), st>>>(a, bulk_stages);
         else
             k_rank_tc<<<std::min(tiles, num_sms()), tcp::kThreads, tc_smem(), st>>>(a);
         const unsigned blocks = (unsigned)ceil_div(n, kSelectWarps);

@@ -70,27 +70,34 @@ struct ScanMode {
                 if (a.qids) qid = a.qids[q];
             }
         }
+        // one candidate row (s >= tau): self exclusion, then the sorted insert;
+        // kept out of line so the per-chunk loop stays a short run of compares
+        __device__ __noinline__ void take(const Args &a, const Tile &T, int64_t col, float sc) {
+            const long long id = a.ids[T.r_begin + col];
+            if (id == qid) return;
+            const int k = a.k;
+            if (kn == k && !ranks_before(sc, id, KS(k - 1), KI(k - 1))) return;
+            int i = kn < k ? kn++ : k - 1;
+            while (i > 0 && ranks_before(sc, id, KS(i - 1), KI(i - 1))) {
+                KS(i) = KS(i - 1);
+                KI(i) = KI(i - 1);
+                --i;
+            }
+            KS(i) = sc;
+            KI(i) = id;
+        }
+        // v holds the chunk's raw accumulator values: similarities x 2^16
         __device__ void chunk(const Args &a, const Tile &T, int64_t col0, const float (&v)[32],
                               int ncol) {
             if (!valid) return;
-            const int k = a.k;
+            const float tau_raw = a.tau * 65536.f;   // exact: a power-of-two scale
+            unsigned m = 0;
 #pragma unroll
-            for (int j = 0; j < 32; ++j) {
-                if (j < ncol && v[j] >= a.tau) {
-                    const long long id = a.ids[T.r_begin + col0 + j];
-                    if (id == qid) continue;
-                    const float sc = v[j];
-                    if (kn == k && !ranks_before(sc, id, KS(k - 1), KI(k - 1))) continue;
-                    int i = kn < k ? kn++ : k - 1;
-                    while (i > 0 && ranks_before(sc, id, KS(i - 1), KI(i - 1))) {
-                        KS(i) = KS(i - 1);
-                        KI(i) = KI(i - 1);
-                        --i;
-                    }
-                    KS(i) = sc;
-                    KI(i) = id;
-                }
-            }
+            for (int j = 0; j < 32; ++j) m |= (v[j] >= tau_raw && j < ncol) ? (1u << j) : 0u;
+            if (m == 0) return;
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+                if (m & (1u << j)) take(a, T, col0 + j, v[j] * (1.f / 65536.f));
         }
         __device__ void end(const Args &a, const Tile &T) {
             if (valid) {
@@ -137,12 +144,12 @@ __global__ void __launch_bounds__(tcb::kThreads, 1) k_scan_bulk(SearchArgs a) {
 
 cudaError_t prepare_scan_bulk(int d, int k, int stages) {
     return cudaFuncSetAttribute(k_scan_bulk, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)tcb::smem_bytes((int)ceil_div(d, 64), stages, scan_epi_bytes(k)));
+                                (int)tcb::smem_bytes(stages, scan_epi_bytes(k)));
 }
 
 void enqueue_scan_bulk(const SearchArgs &a, cudaStream_t st) {
     k_scan_bulk<<<num_sms(), tcb::kThreads,
-                  tcb::smem_bytes((int)ceil_div(a.d, 64), a.tc_stages, scan_epi_bytes(a.k)), st>>>(a);
+                  tcb::smem_bytes(a.tc_stages, scan_epi_bytes(a.k)), st>>>(a);
 }
 
 cudaError_t prepare_scan_tc(int k) {

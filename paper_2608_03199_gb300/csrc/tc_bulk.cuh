@@ -1,25 +1,30 @@
 // tc_bulk.cuh -- the tensor-core contraction fed from the tensor-core layout
 // (tc_layout.cu): S = A * B^T for tiles of 128 A rows (queries) against every
-// block of 128 B rows (a partition's rows, or the centroids), with the same
-// scaled fp16 split and the same per-row epilogues as tc_pipeline.cuh.
+// block of 128 B rows (a partition's rows, or the centroids), with the scaled
+// fp16 split of tc_pipeline.cuh and the same per-row epilogues.
 //
-// The B operand arrives pre-split, in tile byte order, so one 32 KB bulk copy
-// per (block, K-block) lands a stage (hi then lo) in shared memory, several
-// stages deep, with no thread touching it.  The tile's 128 A rows are split
-// once per tile into a resident shared-memory copy of all K-blocks (d <= 256),
-// published K-block by K-block so the MMAs start before the whole of A is in.
+// The B operand arrives pre-split, in tile byte order: one 32 KB bulk copy per
+// (block, K-block) lands a stage (hi then lo) in shared memory, up to six
+// stages deep, with no thread touching the bytes.  The tile's 128 A rows are
+// split once per tile straight into tensor memory (lane i = A row i, two fp16
+// per 32-bit column, hi and lo of each K-block side by side), so shared memory
+// holds nothing but B stages and the epilogue's lists.
 //
-// Warp roles (704 threads, one block per SM):
-//   warps 0-15  A converters: per tile, load the 128 A rows (all K-blocks at
-//               once, one float4 per row per thread), wait until the previous
-//               tile's MMAs are done with A ("a_empty"), split and store, and
-//               publish each K-block ("a_full[kb]")
-//   warp 16     lane 0 issues the bulk copies of the B stages ("b_full" with
+// Tensor memory (512 columns): two 128-column fp32 accumulators, then the
+// tile's A: 64 columns per K-block of 64 elements (32 hi, 32 lo); d <= 256.
+//
+// Warp roles (448 threads, one block per SM):
+//   warps 0-7   A writers: warp w writes lanes 32 (w % 4) .. +31 for the
+//               K-blocks kb with kb % 2 == w / 4; per tile they wait until the
+//               previous tile's MMAs are done with A ("a_empty"), load their
+//               query row's K-block, split it, store it with tcgen05.st and
+//               publish the K-block ("a_full[kb]")
+//   warp 8      lane 0 issues the bulk copies of the B stages ("b_full" with
 //               the transfer byte count; waits on "b_empty")
-//   warp 17     allocates 256 tensor-memory columns (two 128-column
-//               accumulators); lane 0 issues three kind::f16 MMAs per K step
-//   warps 18-21 epilogue: thread i owns tensor-memory lane i = A row i; it
-//               rescales its row of a chunk by 2^-16 and hands it to Mode::Epi
+//   warp 9      allocates the tensor memory; lane 0 issues three kind::f16
+//               MMAs per K step (A from tensor memory, B from shared memory)
+//   warps 10-13 epilogue: thread i owns tensor-memory lane i = A row i; it
+//               hands its row of a chunk (scores x 2^16) to Mode::Epi
 // Every wait is bounded; giving up sets SIEVE_ETIMEOUT in the mode's status
 // word, all roles leave their loops, the issued MMAs and copies are drained
 // (bounded) and tensor memory is freed.
@@ -35,27 +40,26 @@ namespace sieve {
 namespace tcb {
 
 constexpr int kN = 128;                       // B rows per chunk = MMA N = tensor-layout block
-constexpr int kAConvWarps = 16;
-constexpr int kAConvThreads = kAConvWarps * 32;
-constexpr int kProducerWarp = 16;
-constexpr int kMmaWarp = 17;
-constexpr int kThreads = 22 * 32;
-constexpr int kMaxKb = 4;                     // resident A: d <= 256
-constexpr int kMaxStages = 4;
+constexpr int kAWriterWarps = 8;
+constexpr int kProducerWarp = 8;
+constexpr int kMmaWarp = 9;
+constexpr int kThreads = 14 * 32;
+constexpr int kMaxKb = 4;                     // A in tensor memory: d <= 256
+constexpr int kMaxStages = 6;
 constexpr uint32_t kKbBytes = 32768;          // one K-block of 128 rows: hi 16 KB + lo 16 KB
-constexpr uint32_t kTmemCols = 2 * kN;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kAColumn0 = 2 * kN;        // A after the two accumulators
 constexpr uint32_t kWaitPolls = 1u << 24;
 
-// shared memory: 1 KB alignment slack, resident A (nkb K-blocks), the B stages,
-// then the epilogue's bytes
-__host__ __device__ inline size_t smem_bytes(int nkb, int stages, size_t epi_bytes) {
-    return 1024 + (size_t)nkb * kKbBytes + (size_t)stages * kKbBytes + epi_bytes;
+// shared memory: 1 KB alignment slack, the B stages, the epilogue's bytes
+__host__ __device__ inline size_t smem_bytes(int stages, size_t epi_bytes) {
+    return 1024 + (size_t)stages * kKbBytes + epi_bytes;
 }
 
-// B stages that fit beside A and the epilogue (0 if fewer than two fit)
+// B stages that fit beside the epilogue (0 when the pipeline does not apply)
 inline int stages_for(int nkb, size_t epi_bytes, size_t smem_limit) {
     if (nkb > kMaxKb) return 0;
-    const size_t base = smem_bytes(nkb, 0, epi_bytes);
+    const size_t base = smem_bytes(0, epi_bytes);
     if (smem_limit < base) return 0;
     int s = (int)((smem_limit - base) / kKbBytes);
     if (s > kMaxStages) s = kMaxStages;
@@ -79,13 +83,12 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
     const int n_tiles = Mode::num_tiles(a);
     const int d = Mode::d(a);
     const int nkb = (int)ceil_div(d, 64);
-    unsigned char *A = base;                                   // nkb x 32 KB
-    unsigned char *Bst = base + (size_t)nkb * kKbBytes;        // stages x 32 KB
+    unsigned char *Bst = base;                                 // stages x 32 KB
     unsigned char *epi_smem = Bst + (size_t)stages * kKbBytes;
     int *status = Mode::status(a);
 
     if (threadIdx.x == 0) {
-        for (int kb = 0; kb < kMaxKb; ++kb) tc::mbar_init(&a_full[kb], kAConvThreads);
+        for (int kb = 0; kb < kMaxKb; ++kb) tc::mbar_init(&a_full[kb], 4 * 32);
         tc::mbar_init(&a_empty, 1);
         for (int s = 0; s < kMaxStages; ++s) {
             tc::mbar_init(&b_full[s], 1);
@@ -104,6 +107,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
     __syncthreads();
     tc::fence_after_sync();
     const uint32_t tmem = tmem_slot;
+    const uint32_t tA = tmem + kAColumn0;
 
     auto wait = [&](uint64_t *bar, uint32_t parity) -> bool {
         for (uint32_t it = 0; it < kWaitPolls; ++it) {
@@ -115,31 +119,36 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
         return false;
     };
 
-    if (warp < kAConvWarps) {
-        // ---------------- A converters ----------------
-        const int f = threadIdx.x & 15;                // float4 of a K-block
-        const int r0 = threadIdx.x >> 4;               // rows r0 + 32 i
-        uint32_t u = 0;                                // tiles with B rows seen so far
-        for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) {
+    if (warp < kAWriterWarps) {
+        // ---------------- A writers ----------------
+        const int quarter = warp & 3, group = warp >> 2;
+        const int row = quarter * 32 + lane;
+        const uint32_t lane_bits = (uint32_t)(quarter * 32) << 16;
+        uint32_t u = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; ok && t < n_tiles; t += gridDim.x) {
             const typename Mode::Tile T = Mode::tile(a, t);
             if (T.nb <= 0) continue;
-            float4 x[kMaxKb][4];
+            const float *rp = Mode::a_row(a, T, row);
+            ok = __all_sync(0xffffffffu, wait(&a_empty, (u & 1u) ^ 1u));
+            if (!ok) break;
+            tc::fence_after_sync();
+            for (int kb = group; kb < nkb; kb += 2) {
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const float *row = Mode::a_row(a, T, r0 + 32 * i);
+                for (int half = 0; half < 2; ++half) {     // 32 elements = 16 columns per half
+                    uint32_t hi[16], lo[16];
 #pragma unroll
-                for (int kb = 0; kb < kMaxKb; ++kb)
-                    x[kb][i] = kb < nkb ? tcp::load_f4(row, kb * 64 + 4 * f, d)
-                                        : make_float4(0.f, 0.f, 0.f, 0.f);
-            }
-            if (!wait(&a_empty, (u & 1u) ^ 1u)) break;
-#pragma unroll
-            for (int kb = 0; kb < kMaxKb; ++kb) {
-                if (kb >= nkb) break;
-                unsigned char *blk = A + (size_t)kb * kKbBytes;
-#pragma unroll
-                for (int i = 0; i < 4; ++i) tcp::store_f4(blk, blk + kKbBytes / 2, r0 + 32 * i, f, x[kb][i]);
-                tc::fence_proxy_async_smem();
+                    for (int q4 = 0; q4 < 8; ++q4) {
+                        const float4 x = tcp::load_f4(rp, kb * 64 + half * 32 + 4 * q4, d);
+                        tcp::split2(x.x, x.y, hi[2 * q4], lo[2 * q4]);
+                        tcp::split2(x.z, x.w, hi[2 * q4 + 1], lo[2 * q4 + 1]);
+                    }
+                    const uint32_t col = tA + (uint32_t)kb * 64 + (uint32_t)half * 16;
+                    tc::tmem_st16(col + lane_bits, hi);
+                    tc::tmem_st16(col + 32 + lane_bits, lo);
+                }
+                tc::tmem_st_wait();
+                tc::fence_before_sync();
                 tc::mbar_arrive(&a_full[kb]);
             }
             ++u;
@@ -190,17 +199,19 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                         if (ch == 0 && !(ok = wait(&a_full[kb], u & 1u))) break;
                         if (!(ok = wait(&b_full[st], ph))) break;
                         tc::fence_after_sync();
-                        const uint32_t a_hi = tc::smem_u32(A + (size_t)kb * kKbBytes);
-                        const uint32_t a_lo = a_hi + kKbBytes / 2;
+                        const uint32_t a_hi = tA + (uint32_t)kb * 64, a_lo = a_hi + 32;
                         const uint32_t b_hi = tc::smem_u32(Bst + (size_t)st * kKbBytes);
-                        const uint32_t b_lo = b_hi + kKbBytes / 2;
+                        // a K step moves the descriptors' start address by 32 bytes
+                        // (2 in its 16-byte units; shared addresses stay far below
+                        // the field's 2^14 limit, so no carry)
+                        const uint64_t bh = tc::desc_k_sw128(b_hi), bl = tc::desc_k_sw128(b_hi + kKbBytes / 2);
 #pragma unroll
-                        for (int ks = 0; ks < 4; ++ks) {   // K = 16 fp16 = 32 bytes per MMA
-                            const uint32_t o = ks * 32;
-                            tc::mma_f16(dt, tc::desc_k_sw128(a_lo + o), tc::desc_k_sw128(b_hi + o), kIdesc,
-                                        (kb > 0 || ks > 0) ? 1u : 0u);
-                            tc::mma_f16(dt, tc::desc_k_sw128(a_hi + o), tc::desc_k_sw128(b_lo + o), kIdesc, 1u);
-                            tc::mma_f16(dt, tc::desc_k_sw128(a_hi + o), tc::desc_k_sw128(b_hi + o), kIdesc, 1u);
+                        for (int ks = 0; ks < 4; ++ks) {   // K = 16: 8 columns of A, 32 bytes of B
+                            const uint32_t ao = ks * 8;
+                            const uint64_t bo = 2 * ks;
+                            tc::mma_f16_ta(dt, a_lo + ao, bh + bo, kIdesc, (kb > 0 || ks > 0) ? 1u : 0u);
+                            tc::mma_f16_ta(dt, a_hi + ao, bl + bo, kIdesc, 1u);
+                            tc::mma_f16_ta(dt, a_hi + ao, bh + bo, kIdesc, 1u);
                         }
                         tc::mma_commit(&b_empty[st]);
                     }
@@ -234,8 +245,6 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                 for (int cc = 0; cc < kN / 32; ++cc) {
                     float v[32];
                     tc::tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + buf * kN + cc * 32, v);
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) v[j] *= tcp::kUnscale;
                     const int64_t col0 = (int64_t)ch * kN + cc * 32;
                     const int64_t left = T.nb - col0;
                     epi.chunk(a, T, col0, v, left < 32 ? (int)left : 32);

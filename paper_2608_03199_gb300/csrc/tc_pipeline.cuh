@@ -25,8 +25,9 @@
 //               lane 0 issues the MMAs, commits each stage to its "empty"
 //               barrier and each finished chunk to "dfull"
 //   warps 17-20 epilogue: thread i owns tensor-memory lane i = A row i of the
-//               tile; it reads that row's kN scores of a chunk (Mode::Epi),
-//               then releases the accumulator ("dempty")
+//               tile; it hands that row's kN raw accumulator values of a chunk
+//               (scores x 2^16) to Mode::Epi, then releases the accumulator
+//               ("dempty")
 // Every mbarrier wait is bounded: a wait that gives up marks the block as
 // aborted (SIEVE_ETIMEOUT in the mode's status word), every role leaves its
 // loop, the issued MMAs are drained (bounded) and tensor memory is freed.
@@ -251,8 +252,6 @@ __device__ __forceinline__ void run_pipeline(const typename Mode::Args &a, unsig
                 for (int cc = 0; cc < kN / 32; ++cc) {
                     float v[32];
                     tc::tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + buf * kN + cc * 32, v);
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) v[j] *= kUnscale;
                     const int64_t col0 = (int64_t)ch * kN + cc * 32;
                     const int64_t left = T.nb - col0;
                     epi.chunk(a, T, col0, v, left < 32 ? (int)left : 32);
