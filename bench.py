@@ -50,6 +50,8 @@ def parse():
     ap.add_argument("--skip-e2e", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="target CPU seconds for the oracle sample")
+    ap.add_argument("--scan-path", choices=("auto", "simt", "tensor"), default="auto",
+                    help="which units score the partition groups (sieve_params.scan_path)")
     ap.add_argument("--ncu-case", choices=("w8", "fixed"), default=None,
                     help="run exactly one search (W = the config's W, or fixed probe) and exit: "
                          "a small, single-call target for an ncu capture")
@@ -335,7 +337,8 @@ def run_sieve(args, cfg, world, rank, local):
 
     def step(W):
         return lambda: sieve.search(index, Q, cfg.tau, k, cfg.nprobe, W, lookahead=True,
-                                    query_ids=qids, workspace=ws, out=outs)
+                                    query_ids=qids, workspace=ws, out=outs,
+                                    scan_path=args.scan_path)
 
     clocks = ClockSampler(local)
     clocks.start()
@@ -345,10 +348,10 @@ def run_sieve(args, cfg, world, rank, local):
 
     # one profiled step (host-driven rounds, CUDA events around every launch)
     prof = sieve.search(index, Q, cfg.tau, k, cfg.nprobe, cfg.W, lookahead=True, query_ids=qids,
-                        profile=True, workspace=ws)[4]
+                        profile=True, workspace=ws, scan_path=args.scan_path)[4]
     probes = outs[3]
     sieve.search(index, Q, cfg.tau, k, cfg.nprobe, cfg.W, lookahead=True, query_ids=qids,
-                 workspace=ws, out=outs)
+                 workspace=ws, out=outs, scan_path=args.scan_path)
     mean_probes = float(probes.float().mean().item())
     hit_frac = float((outs[2] > 0).float().mean().item())
 
@@ -365,7 +368,8 @@ def run_sieve(args, cfg, world, rank, local):
 
         def hstep():
             sieve.search_host(index, Qh, cfg.tau, k, cfg.nprobe, cfg.W, lookahead=True,
-                              query_ids_host=qh, workspace=hws, out=houts)
+                              query_ids_host=qh, workspace=hws, out=houts,
+                              scan_path=args.scan_path)
         hsteps = max(3, args.steps // 5)
         for _ in range(2):
             hstep()
@@ -394,6 +398,7 @@ def run_sieve(args, cfg, world, rank, local):
         "dtype": "f32",
         "data": "synthetic",
         "config": {"workload": workload_desc(cfg), "nq_per_gpu": nq, "parallelism": f"query-shard x{world}",
+                   "scan_path": args.scan_path,
                    "l2": "inputs larger than L2 (index 1.02 GB streamed per step)"},
         "fixed_probe": {"value": nq * world / (ms_fixed * 1e-3), "ms_per_step": ms_fixed,
                         "W": cfg.nprobe},

@@ -101,9 +101,9 @@ typedef struct {
  *   scan_path  which units compute similarities; all paths give the same
  *              decisions up to fp32 rounding (see the parity notes):
  *              0 = automatic (ranking on the tensor cores when nlist <= 2048;
- *              partition groups of >= 24 items on the tensor cores when
- *              k <= 16, the rest on FP32 FMA), 1 = FP32 FMA only,
- *              2 = tensor cores for every group (needs k <= 16)
+ *              every partition group on the tensor cores when k <= 16, on
+ *              FP32 FMA otherwise), 1 = FP32 FMA only, 2 = tensor cores
+ *              (needs k <= 16)
  */
 typedef struct {
     float tau;

@@ -341,7 +341,8 @@ def search(index: Index, Q, tau, k, nprobe, W, lookahead=True, query_ids=None, o
 
 
 def search_host(index: Index, Q_host, tau, k, nprobe, W, lookahead=True, query_ids_host=None,
-                max_items_per_round=0, loop=0, workspace=None, out=None, stream=None):
+                max_items_per_round=0, loop=0, scan_path="auto", workspace=None, out=None,
+                stream=None):
     """sieve_search_host: host (CPU, ideally pinned) queries in, host results out.
 
     The call copies the queries to the device, searches, copies the results
@@ -352,7 +353,7 @@ def search_host(index: Index, Q_host, tau, k, nprobe, W, lookahead=True, query_i
         raise TypeError("query_ids_host must be an int64 CPU tensor")
     nq = Q_host.shape[0]
     dev = index.vectors.device
-    p = _params(tau, k, nprobe, W, lookahead, loop, max_items_per_round)
+    p = _params(tau, k, nprobe, W, lookahead, loop, max_items_per_round, 0, scan_path)
     v = index.view()
     nbytes = C.c_size_t()
     _check(lib().sieve_search_workspace_size(C.byref(v), nq, C.byref(p), 1, C.byref(nbytes)),

@@ -306,7 +306,7 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
     a.bucketed = reinterpret_cast<int *>(ws + L.bucketed);
     a.tiles = reinterpret_cast<int4 *>(ws + L.tiles);
     a.tc_tiles = reinterpret_cast<int4 *>(ws + L.tc_tiles);
-    a.tc_min = p->scan_path == 1 ? 0 : p->scan_path == 2 ? 1 : (p->k <= kTcMaxK ? 24 : 0);
+    a.tc_min = p->scan_path == 1 ? 0 : (p->k <= kTcMaxK ? 1 : 0);
     a.active = reinterpret_cast<int4 *>(ws + L.active);
     a.rank_scratch = L.rank_scratch ? reinterpret_cast<float *>(ws + L.rank_scratch) : nullptr;
     a.tc_rows = static_cast<const unsigned char *>(ix->tc_rows);
