@@ -34,6 +34,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 import synth  # noqa: E402
+from paper_2608_03199_gb300 import shard  # noqa: E402
 
 METRIC = ("queries/s at W=8 (tau-filtered top-10) + speedup vs fixed-probe; "
           "% HBM/tensor roofline")
@@ -42,7 +43,7 @@ METRIC = ("queries/s at W=8 (tau-filtered top-10) + speedup vs fixed-probe; "
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--steps", type=int, default=400)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=("sieve", "reference"), default="sieve")
     ap.add_argument("--config", default="1m")
@@ -134,7 +135,8 @@ def measured_peaks():
 
 
 KERNEL_SOURCES = ("common.cuh", "search.cuh", "search_kernels.cu", "rank_kernel.cu",
-                  "scan_tc.cu", "tcgen05.cuh")
+                  "scan_tc.cu", "tcgen05.cuh", "tc_bulk.cuh", "tc_pipeline.cuh", "rank_tc.cu",
+                  "tc_layout.cu")
 
 
 def kernel_source_sha():
@@ -148,9 +150,12 @@ def kernel_source_sha():
     return h.hexdigest()[:16]
 
 
-def committed_traffic(kernel, workload):
+def committed_traffic(kernel, workload, launches):
     """DRAM bytes per launch from the committed ncu summary, if the kernel
-    sources are unchanged since it was taken."""
+    sources are unchanged since it was taken: the capture's bytes over all of
+    one search's launches, averaged over this step's launch count (the same
+    averaging as the achieved rate; launches past the last busy round move
+    no bytes)."""
     try:
         t = json.load(open(os.path.join(ROOT, "profiles", "traffic.json")))
     except Exception:
@@ -158,11 +163,13 @@ def committed_traffic(kernel, workload):
     e = t.get(kernel, {}).get(workload)
     if not e or e.get("source_sha") != kernel_source_sha():
         return None
-    return {"dram_bytes_per_launch": e.get("dram_bytes_per_launch"), "launch": e.get("launch")}
+    return e["dram_bytes_per_search"] / max(1, launches)
 
 
-def roofline(prof, cfg, dev):
-    """Roofline entry for the kernel with the largest share of the step."""
+def roofline(prof, cfg, dev, bulk=True):
+    """Roofline entry for the kernel with the largest share of the step.
+    bulk: the index carries the tensor-core layout, so the tensor-core scan
+    runs as k_scan_bulk (else k_scan_tc)."""
     km, kl = prof["kernel_ms"], prof["kernel_launches"]
     top = max(km, key=lambda k: km[k])
     props = torch.cuda.get_device_properties(dev)
@@ -173,7 +180,8 @@ def roofline(prof, cfg, dev):
     d = cfg.d
     launches = max(1, kl[top])
     ms_per_launch = km[top] / launches
-    out = {"kernel": f"k_{top}", "launches": kl[top], "ms_per_launch": ms_per_launch}
+    name = {"scan_tc": "k_scan_bulk" if bulk else "k_scan_tc"}.get(top, f"k_{top}")
+    out = {"kernel": name, "launches": kl[top], "ms_per_launch": ms_per_launch}
     # fp16 dense peak: the measured bf16 cuBLAS peak (fp16 and bf16 share the
     # nominal 2.25 PFLOP/s rate); the burst figure, as the kernel is timed alone
     f16_tflops = peaks.get("bf16_tflops", 1889.4)
@@ -205,7 +213,7 @@ def roofline(prof, cfg, dev):
                                f"x {clock_mhz:.0f} MHz (measured max clock)")
     else:
         out.update(bound="hbm", achieved=None, peak=hbm, unit="GB/s", frac=None)
-    out["traffic"] = committed_traffic(out["kernel"], cfg.name)
+    out["traffic"] = committed_traffic(out["kernel"], cfg.name, kl[top])
     return out
 
 
@@ -219,15 +227,11 @@ def dist_setup(gpus):
 
 def barrier(world):
     if world > 1:
-        torch.distributed.barrier()
+        shard.barrier()
 
 
 def max_over_ranks(x, world, dev):
-    if world == 1:
-        return x
-    t = torch.tensor([x], dtype=torch.float64, device=dev)
-    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-    return float(t.item())
+    return shard.max_over_ranks(x, device=dev) if world > 1 else x
 
 
 def time_steps(fn, steps, warmup, world, dev):
@@ -396,6 +400,8 @@ def run_sieve(args, cfg, world, rank, local):
         "scaling": "weak",
         "vs_baseline": None,
         "dtype": "f32",
+        "arithmetic": "fp32 inputs; scores from three fp16 tensor-core products per pair "
+                      "(scaled hi/lo split), fp32 accumulation",
         "data": "synthetic",
         "config": {"workload": workload_desc(cfg), "nq_per_gpu": nq, "parallelism": f"query-shard x{world}",
                    "scan_path": args.scan_path,
@@ -405,7 +411,7 @@ def run_sieve(args, cfg, world, rank, local):
         "speedup_vs_fixed": ms_fixed / ms,
         "mean_probes": mean_probes,
         "queries_with_results": hit_frac,
-        "roofline": roofline(prof, cfg, dev),
+        "roofline": roofline(prof, cfg, dev, bulk=index.tc_rows is not None),
         "profile": {"kernel_ms": prof["kernel_ms"], "kernel_launches": prof["kernel_launches"],
                     "rounds": prof["rounds"], "items": prof["items"], "groups": prof["groups"],
                     "mean_group": prof["items"] / max(1, prof["groups"]),
@@ -435,7 +441,7 @@ def run_ncu_case(args, cfg):
     # host-driven rounds: ncu does not profile kernels inside a CUDA graph with
     # conditional nodes; the kernels and their arguments are the same
     out = sieve.search(index, wl["Q"], cfg.tau, cfg.k, cfg.nprobe, W, lookahead=True,
-                       query_ids=wl["qids"], stats=True, loop=1)
+                       query_ids=wl["qids"], stats=True, loop=1, scan_path=args.scan_path)
     print(json.dumps({"ncu_case": args.ncu_case, "W": W, "rounds": out[4]["rounds"],
                       "items": out[4]["items"], "pairs": out[4]["pairs"]}))
     return 0
