@@ -408,6 +408,7 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
         stats->kernel_launches[SIEVE_K_FINALIZE] = 1;
         for (int slot : per_round) stats->kernel_launches[slot] = c.round;
         stats->kernel_launches[SIEVE_K_SCAN_TC] = a.tc_min > 0 ? c.round : 0;
+        if (a.tc_min == 1) stats->kernel_launches[SIEVE_K_SCAN] = 0;
         if (c.status != 0) return c.status;
     }
     return SIEVE_OK;

@@ -32,7 +32,8 @@ struct Ctl {
     int status;        // 0 or a SIEVE_E* code
     int more;          // 1 while another round is needed
     int n_tc_tiles;    // tensor-core scan tiles this round
-    int pad[6];
+    int tc_tile_next;  // tensor-core scan work counter
+    int pad[5];
     unsigned long long tot_items, tot_groups, tot_tiles, tot_rows, tot_pairs;
     unsigned long long tot_rows_tc, tot_pairs_tc;   // the tensor-core share of the two above
 };

@@ -41,6 +41,8 @@ struct RankMode {
         int64_t nb;
     };
     __device__ static int num_tiles(const Args &a) { return (int)ceil_div(a.nq, tcp::kM); }
+    // every tile costs the same: a static stride over the blocks
+    __device__ static int *tile_counter(const Args &) { return nullptr; }
     __device__ static int d(const Args &a) { return a.d; }
     __device__ static int *status(const Args &a) { return a.status ? a.status : &g_rank_status_sink; }
     __device__ static Tile tile(const Args &a, int t) {

@@ -24,6 +24,8 @@ struct ScanMode {
         int64_t r_begin, nb;
     };
     __device__ static int num_tiles(const Args &a) { return a.ctl->n_tc_tiles; }
+    // tiles differ in cost (partition sizes are skewed): blocks draw them dynamically
+    __device__ static int *tile_counter(const Args &a) { return &a.ctl->tc_tile_next; }
     __device__ static int d(const Args &a) { return a.d; }
     __device__ static int *status(const Args &a) { return &a.ctl->status; }
     __device__ static Tile tile(const Args &a, int t) {

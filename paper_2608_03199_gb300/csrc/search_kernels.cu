@@ -214,6 +214,7 @@ __global__ void __launch_bounds__(kBucketThreads) k_bucket(SearchArgs a) {
         ctl->n_tiles = sums[1];
         ctl->n_tc_tiles = sums[2];
         ctl->tile_next = 0;
+        ctl->tc_tile_next = 0;
     }
 }
 
@@ -495,6 +496,7 @@ __global__ void k_round_end(SearchArgs a, cudaGraphConditionalHandle cond, int u
     c->n_tiles = 0;
     c->n_tc_tiles = 0;
     c->tile_next = 0;
+    c->tc_tile_next = 0;
     c->n_deferred = 0;
     c->n_continue = 0;
     if (use_cond) cudaGraphSetConditional(cond, more ? 1u : 0u);
@@ -566,7 +568,8 @@ cudaError_t launch_round(const SearchArgs &a, size_t scan_smem, int scan_blocks,
     }
     end();
     begin();
-    k_scan<<<scan_blocks, kThreads, scan_smem, st>>>(a);
+    if (a.tc_min != 1)   // tc_min == 1 sends every group to the tensor cores
+        k_scan<<<scan_blocks, kThreads, scan_smem, st>>>(a);
     end();
     const int merge_blocks = (int)std::min<int64_t>(ceil_div(a.nq * 32, kMergeThreads), 8 * sms);
     begin();

@@ -15,12 +15,17 @@
 //
 // Warp roles (448 threads, one block per SM):
 //   warps 0-7   A writers: warp w writes lanes 32 (w % 4) .. +31 for the
-//               K-blocks kb with kb % 2 == w / 4; per tile they wait until the
-//               previous tile's MMAs are done with A ("a_empty"), load their
-//               query row's K-block, split it, store it with tcgen05.st and
-//               publish the K-block ("a_full[kb]")
-//   warp 8      lane 0 issues the bulk copies of the B stages ("b_full" with
-//               the transfer byte count; waits on "b_empty")
+//               K-blocks kb with kb % 2 == w / 4.  For each tile they load
+//               their query row early (an L2 prefetch of the whole row, then
+//               the K-block's values into registers), and only then wait until
+//               the previous tile's last MMAs on that K-block are done
+//               ("a_empty[kb]"), split the values, store them with tcgen05.st
+//               and publish the K-block ("a_full[kb]")
+//   warp 8      lane 0 takes the block's next tile (an atomic work counter,
+//               or a static stride when the mode has none) and hands it to the
+//               other roles through a small ring in shared memory; it then
+//               issues the tile's bulk copies of B stages ("b_full" with the
+//               transfer byte count; waits on "b_empty")
 //   warp 9      allocates the tensor memory; lane 0 issues three kind::f16
 //               MMAs per K step (A from tensor memory, B from shared memory)
 //   warps 10-13 epilogue: thread i owns tensor-memory lane i = A row i; it
@@ -50,6 +55,8 @@ constexpr uint32_t kKbBytes = 32768;          // one K-block of 128 rows: hi 16 
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kAColumn0 = 2 * kN;        // A after the two accumulators
 constexpr uint32_t kWaitPolls = 1u << 24;
+constexpr int kRing = 8;                      // tiles handed from the scheduler to the other roles
+constexpr uint32_t kRingReaders = kAWriterWarps + 1 + 4;   // A-writer warps, MMA lane, epilogue warps
 
 // shared memory: 1 KB alignment slack, the B stages, the epilogue's bytes
 __host__ __device__ inline size_t smem_bytes(int stages, size_t epi_bytes) {
@@ -67,13 +74,17 @@ inline int stages_for(int nkb, size_t epi_bytes, size_t smem_limit) {
 }
 
 // Mode provides (in addition to what tc_pipeline.cuh asks): b_block(a, T, ch)
-// = pointer to the tensor-layout bytes of the tile's ch-th block of B rows.
+// = pointer to the tensor-layout bytes of the tile's ch-th block of B rows, and
+// tile_counter(a) = a zeroed global int the blocks draw tiles from (nullptr:
+// block b takes tiles b, b + gridDim.x, ...).
 template <class Mode>
 __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned char *smem_raw,
                                          int stages) {
     constexpr uint32_t kIdesc = tc::idesc_f16(tcp::kM, kN);
-    __shared__ __align__(8) uint64_t a_full[kMaxKb], a_empty, b_full[kMaxStages],
-        b_empty[kMaxStages], dfull_bar[2], dempty_bar[2], drain_bar;
+    __shared__ __align__(8) uint64_t a_full[kMaxKb], a_empty[kMaxKb], b_full[kMaxStages],
+        b_empty[kMaxStages], dfull_bar[2], dempty_bar[2], drain_bar, ring_full[kRing],
+        ring_empty[kRing];
+    __shared__ int ring_tile[kRing];
     __shared__ uint32_t tmem_slot;
     __shared__ int s_abort;
 
@@ -86,10 +97,13 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
     unsigned char *Bst = base;                                 // stages x 32 KB
     unsigned char *epi_smem = Bst + (size_t)stages * kKbBytes;
     int *status = Mode::status(a);
+    int *tile_counter = Mode::tile_counter(a);
 
     if (threadIdx.x == 0) {
-        for (int kb = 0; kb < kMaxKb; ++kb) tc::mbar_init(&a_full[kb], 4 * 32);
-        tc::mbar_init(&a_empty, 1);
+        for (int kb = 0; kb < kMaxKb; ++kb) {
+            tc::mbar_init(&a_full[kb], 4 * 32);
+            tc::mbar_init(&a_empty[kb], 1);
+        }
         for (int s = 0; s < kMaxStages; ++s) {
             tc::mbar_init(&b_full[s], 1);
             tc::mbar_init(&b_empty[s], 1);
@@ -97,6 +111,10 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
         for (int b = 0; b < 2; ++b) {
             tc::mbar_init(&dfull_bar[b], 1);
             tc::mbar_init(&dempty_bar[b], 4 * 32);
+        }
+        for (int r = 0; r < kRing; ++r) {
+            tc::mbar_init(&ring_full[r], 1);
+            tc::mbar_init(&ring_empty[r], kRingReaders);
         }
         tc::mbar_init(&drain_bar, 1);
         s_abort = 0;
@@ -118,6 +136,16 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
         atomicExch(status, SIEVE_ETIMEOUT);
         return false;
     };
+    // the i-th tile of this block from the ring, read by a whole warp (one
+    // arrival per warp); false when the wait gave up.  t < 0 ends the loop.
+    auto ring_take_warp = [&](uint32_t i, int &t) -> bool {
+        const uint32_t slot = i % kRing, ph = (i / kRing) & 1u;
+        if (!__all_sync(0xffffffffu, wait(&ring_full[slot], ph))) return false;
+        t = *(volatile int *)&ring_tile[slot];
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(&ring_empty[slot]);
+        return true;
+    };
 
     if (warp < kAWriterWarps) {
         // ---------------- A writers ----------------
@@ -126,22 +154,27 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
         const uint32_t lane_bits = (uint32_t)(quarter * 32) << 16;
         uint32_t u = 0;
         bool ok = true;
-        for (int t = blockIdx.x; ok && t < n_tiles; t += gridDim.x) {
+        for (uint32_t i = 0; ok; ++i) {
+            int t;
+            if (!ring_take_warp(i, t) || t < 0) break;
             const typename Mode::Tile T = Mode::tile(a, t);
             if (T.nb <= 0) continue;
             const float *rp = Mode::a_row(a, T, row);
-            ok = __all_sync(0xffffffffu, wait(&a_empty, (u & 1u) ^ 1u));
-            if (!ok) break;
-            tc::fence_after_sync();
+            if (rp && group == 0) tc::prefetch_l2(rp, (uint32_t)d * 4u);   // d % 4 == 0
             for (int kb = group; kb < nkb; kb += 2) {
+                float4 x[16];
+#pragma unroll
+                for (int q4 = 0; q4 < 16; ++q4) x[q4] = tcp::load_f4(rp, kb * 64 + 4 * q4, d);
+                if (!(ok = __all_sync(0xffffffffu, wait(&a_empty[kb], (u & 1u) ^ 1u)))) break;
+                tc::fence_after_sync();
 #pragma unroll
                 for (int half = 0; half < 2; ++half) {     // 32 elements = 16 columns per half
                     uint32_t hi[16], lo[16];
 #pragma unroll
                     for (int q4 = 0; q4 < 8; ++q4) {
-                        const float4 x = tcp::load_f4(rp, kb * 64 + half * 32 + 4 * q4, d);
-                        tcp::split2(x.x, x.y, hi[2 * q4], lo[2 * q4]);
-                        tcp::split2(x.z, x.w, hi[2 * q4 + 1], lo[2 * q4 + 1]);
+                        const float4 v = x[half * 8 + q4];
+                        tcp::split2(v.x, v.y, hi[2 * q4], lo[2 * q4]);
+                        tcp::split2(v.z, v.w, hi[2 * q4 + 1], lo[2 * q4 + 1]);
                     }
                     const uint32_t col = tA + (uint32_t)kb * 64 + (uint32_t)half * 16;
                     tc::tmem_st16(col + lane_bits, hi);
@@ -154,18 +187,25 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
             ++u;
         }
     } else if (warp == kProducerWarp) {
-        // ---------------- B producer ----------------
+        // ---------------- tile scheduler + B producer ----------------
         if (lane == 0) {
             uint32_t s = 0;
             bool ok = true;
-            for (int t = blockIdx.x; ok && t < n_tiles; t += gridDim.x) {
+            for (uint32_t i = 0; ok; ++i) {
+                const uint32_t slot = i % kRing, ph = (i / kRing) & 1u;
+                if (!(ok = wait(&ring_empty[slot], ph ^ 1u))) break;
+                int t = tile_counter ? atomicAdd(tile_counter, 1) : (int)(blockIdx.x + i * gridDim.x);
+                if (t >= n_tiles) t = -1;
+                ring_tile[slot] = t;
+                tc::mbar_arrive(&ring_full[slot]);   // release: the tile id is visible with the phase
+                if (t < 0) break;
                 const typename Mode::Tile T = Mode::tile(a, t);
                 const int nch = (int)ceil_div(T.nb, kN);
                 for (int ch = 0; ok && ch < nch; ++ch) {
                     const unsigned char *src = Mode::b_block(a, T, ch);
                     for (int kb = 0; kb < nkb; ++kb) {
-                        const uint32_t st = s % stages, ph = (s / stages) & 1u;
-                        if (!(ok = wait(&b_empty[st], ph ^ 1u))) break;
+                        const uint32_t st = s % stages, sph = (s / stages) & 1u;
+                        if (!(ok = wait(&b_empty[st], sph ^ 1u))) break;
                         tc::mbar_arrive_expect_tx(&b_full[st], kKbBytes);
                         tc::bulk_g2s(Bst + (size_t)st * kKbBytes, src + (size_t)kb * kKbBytes, kKbBytes,
                                      &b_full[st]);
@@ -185,7 +225,12 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
         if (lane == 0) {
             uint32_t s = 0, c = 0, u = 0;
             bool ok = true;
-            for (int t = blockIdx.x; ok && t < n_tiles; t += gridDim.x) {
+            for (uint32_t i = 0; ok; ++i) {
+                const uint32_t slot = i % kRing, rph = (i / kRing) & 1u;
+                if (!(ok = wait(&ring_full[slot], rph))) break;
+                const int t = *(volatile int *)&ring_tile[slot];
+                tc::mbar_arrive(&ring_empty[slot]);
+                if (t < 0) break;
                 const typename Mode::Tile T = Mode::tile(a, t);
                 const int nch = (int)ceil_div(T.nb, kN);
                 if (nch == 0) continue;
@@ -214,10 +259,12 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                             tc::mma_f16_ta(dt, a_hi + ao, bh + bo, kIdesc, 1u);
                         }
                         tc::mma_commit(&b_empty[st]);
+                        // the tile's last reads of this K-block of A: it may be
+                        // overwritten by the next tile once they are done
+                        if (ch == nch - 1) tc::mma_commit(&a_empty[kb]);
                     }
                     if (ok) tc::mma_commit(&dfull_bar[buf]);
                 }
-                if (ok) tc::mma_commit(&a_empty);   // A may be overwritten once these are done
                 ++u;
             }
             tc::mma_commit(&drain_bar);
@@ -232,7 +279,9 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
         uint32_t c = 0;
         bool ok = true;
         typename Mode::Epi epi;
-        for (int t = blockIdx.x; ok && t < n_tiles; t += gridDim.x) {
+        for (uint32_t i = 0; ok; ++i) {
+            int t;
+            if (!ring_take_warp(i, t) || t < 0) break;
             const typename Mode::Tile T = Mode::tile(a, t);
             const int nch = (int)ceil_div(T.nb, kN);
             epi.begin(a, T, slot, epi_smem);
