@@ -92,14 +92,40 @@ __global__ void __launch_bounds__(tcb::kThreads, 1) k_rank_bulk(RankArgs a, int 
 }
 
 // ---------------------------------------------------------------------------
-// selection: monotone map of fp32 to uint32 (larger float -> larger key)
+// selection: monotone map of fp32 to uint32 (larger float -> larger key); -0
+// is mapped as +0 so that equal scores have equal keys
 __device__ __forceinline__ uint32_t order_key(float s) {
-    const uint32_t u = __float_as_uint(s);
+    const uint32_t u = __float_as_uint(s + 0.f);
     return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
 constexpr int kSelectWarps = 4;
+constexpr int kSelectMaxR = 4;   // lane order statistics used for the lower bracket
 
+__device__ __forceinline__ int warp_sum(int x) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+    return x;
+}
+
+template <int KPL>
+__device__ __forceinline__ int count_ge(const uint32_t (&key)[KPL], uint32_t t) {
+    int c = 0;
+#pragma unroll
+    for (int j = 0; j < KPL; ++j) c += key[j] >= t;
+    return warp_sum(c);
+}
+
+// One warp per query.  T* = the nprobe-th largest key.  The search keeps a
+// threshold T <= T* with C = #{keys >= T} >= nprobe and refines T bit by bit
+// (the largest T with at least nprobe keys >= T) until C fits the sort
+// buffer; it starts from the common high bits of a bracket L <= T* <= U
+// (U = the largest key; L = the smallest over lanes of each lane's
+// ceil(nprobe / 32)-th largest key, so at least nprobe keys are >= L).  The
+// C candidates >= T contain the nprobe best, which a bitonic sort by
+// (score desc, id asc) puts first.  When C never fits (many equal scores),
+// the search ends at T = T* and takes the keys > T* plus the lowest-id keys
+// equal to it.  P: a power of two >= nprobe; the buffer holds 2P entries.
 template <int KPL>   // scores per lane: nlist <= 32 * KPL
 __global__ void __launch_bounds__(kSelectWarps * 32) k_select(const float *__restrict__ scores,
                                                               int64_t ld, int64_t nq, int nlist,
@@ -107,9 +133,10 @@ __global__ void __launch_bounds__(kSelectWarps * 32) k_select(const float *__res
                                                               int32_t *__restrict__ order,
                                                               float *__restrict__ cscores) {
     extern __shared__ __align__(16) unsigned char sel_smem[];
+    const int cap = 2 * P;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    float *bs = reinterpret_cast<float *>(sel_smem) + warp * 2 * P;   // P scores, then P ids
-    int *bc = reinterpret_cast<int *>(bs + P);
+    float *bs = reinterpret_cast<float *>(sel_smem) + warp * 2 * cap;   // cap scores, then cap ids
+    int *bc = reinterpret_cast<int *>(bs + cap);
     const int64_t q = (int64_t)blockIdx.x * kSelectWarps + warp;
     if (q >= nq) return;
     const float *row = scores + q * ld;
@@ -121,49 +148,100 @@ __global__ void __launch_bounds__(kSelectWarps * 32) k_select(const float *__res
         s[j] = c < nlist ? row[c] : 0.f;
         key[j] = c < nlist ? order_key(s[j]) : 0u;   // padding ranks below every score
     }
-    // the largest t with at least nprobe keys >= t is the nprobe-th largest key
-    uint32_t T = 0;
-    for (int b = 31; b >= 0; --b) {
-        const uint32_t t = T | (1u << b);
-        int cnt = 0;
+    // bracket: per lane the r largest keys (a small insertion network)
+    const int r = (nprobe + 31) / 32;
+    uint32_t m[kSelectMaxR] = {0u, 0u, 0u, 0u};
+    if (r <= 2) {
 #pragma unroll
-        for (int j = 0; j < KPL; ++j) cnt += key[j] >= t;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, o);
-        if (cnt >= nprobe) T = t;
-    }
-    int gt = 0;
-#pragma unroll
-    for (int j = 0; j < KPL; ++j) gt += key[j] > T;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) gt += __shfl_xor_sync(0xffffffffu, gt, o);
-    const int ties_wanted = nprobe - gt;   // >= 1: equal keys, lowest ids first
-    // gather, in increasing id order (id = 32 j + lane)
-    const unsigned below = (1u << lane) - 1u;
-    int pos = 0, ties_seen = 0;
-#pragma unroll
-    for (int j = 0; j < KPL; ++j) {
-        const bool tie = key[j] == T && j * 32 + lane < nlist;
-        const unsigned tb = __ballot_sync(0xffffffffu, tie);
-        const bool sel = key[j] > T || (tie && ties_seen + __popc(tb & below) < ties_wanted);
-        const unsigned sb = __ballot_sync(0xffffffffu, sel);
-        if (sel) {
-            const int p = pos + __popc(sb & below);
-            bs[p] = s[j];
-            bc[p] = j * 32 + lane;
+        for (int j = 0; j < KPL; ++j) {
+            m[1] = max(m[1], min(m[0], key[j]));
+            m[0] = max(m[0], key[j]);
         }
-        pos += __popc(sb);
-        ties_seen += __popc(tb);
+    } else {
+#pragma unroll
+        for (int j = 0; j < KPL; ++j) {
+            uint32_t x = key[j];
+#pragma unroll
+            for (int i = 0; i < kSelectMaxR; ++i) {
+                const uint32_t hi = max(m[i], x);
+                x = min(m[i], x);
+                m[i] = hi;
+            }
+        }
     }
-    for (int p = nprobe + lane; p < P; p += 32) {   // pad to a power of two
+    uint32_t U = m[0];
+    uint32_t L = r == 1 ? m[0] : r == 2 ? m[1] : r == 3 ? m[2] : r == 4 ? m[3] : 0u;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        U = max(U, __shfl_xor_sync(0xffffffffu, U, o));
+        L = min(L, __shfl_xor_sync(0xffffffffu, L, o));
+    }
+    int b;
+    uint32_t T;
+    if (L == U) {
+        b = -1;
+        T = L;
+    } else {
+        b = 31 - __clz(L ^ U);                                // highest bit where they differ
+        T = b == 31 ? 0u : (L & ~((2u << b) - 1u));           // their common high bits
+    }
+    int C = count_ge(key, T);
+    for (; b >= 0 && C > cap; --b) {
+        const uint32_t t = T | (1u << b);
+        const int cnt = count_ge(key, t);
+        if (cnt >= nprobe) {
+            T = t;
+            C = cnt;
+        }
+    }
+    const unsigned below = (1u << lane) - 1u;
+    int pos = 0;
+    if (C <= cap) {
+        // every key >= T, in increasing id order (id = 32 j + lane)
+#pragma unroll
+        for (int j = 0; j < KPL; ++j) {
+            const bool sel = key[j] >= T && j * 32 + lane < nlist;
+            const unsigned sb = __ballot_sync(0xffffffffu, sel);
+            if (sel) {
+                const int p = pos + __popc(sb & below);
+                bs[p] = s[j];
+                bc[p] = j * 32 + lane;
+            }
+            pos += __popc(sb);
+        }
+    } else {
+        // T == T*: the keys above it, then the lowest-id keys equal to it
+        int gt = 0;
+#pragma unroll
+        for (int j = 0; j < KPL; ++j) gt += key[j] > T;
+        const int ties_wanted = nprobe - warp_sum(gt);   // >= 1
+        int ties_seen = 0;
+#pragma unroll
+        for (int j = 0; j < KPL; ++j) {
+            const bool tie = key[j] == T && j * 32 + lane < nlist;
+            const unsigned tb = __ballot_sync(0xffffffffu, tie);
+            const bool sel = key[j] > T || (tie && ties_seen + __popc(tb & below) < ties_wanted);
+            const unsigned sb = __ballot_sync(0xffffffffu, sel);
+            if (sel) {
+                const int p = pos + __popc(sb & below);
+                bs[p] = s[j];
+                bc[p] = j * 32 + lane;
+            }
+            pos += __popc(sb);
+            ties_seen += __popc(tb);
+        }
+    }
+    int S = 1;   // sort size: a power of two >= pos (pos <= cap)
+    while (S < pos) S <<= 1;
+    for (int p = pos + lane; p < S; p += 32) {
         bs[p] = -__int_as_float(0x7f800000);
         bc[p] = INT32_MAX;
     }
     __syncwarp();
-    // bitonic sort of P entries, first-ranked first
-    for (int k = 2; k <= P; k <<= 1) {
+    // bitonic sort of S entries, first-ranked first
+    for (int k = 2; k <= S; k <<= 1) {
         for (int j = k >> 1; j > 0; j >>= 1) {
-            for (int i = lane; i < P / 2; i += 32) {
+            for (int i = lane; i < S / 2; i += 32) {
                 const int lo = 2 * i - (i & (j - 1));
                 const int hi = lo + j;
                 const bool up = (lo & k) == 0;
@@ -213,7 +291,7 @@ static int pow2_at_least(int x) {
 template <int KPL>
 static cudaError_t set_select_attr(int P) {
     return cudaFuncSetAttribute(k_select<KPL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                kSelectWarps * 2 * P * 4);
+                                kSelectWarps * 2 * (2 * P) * 4);
 }
 
 cudaError_t prepare_rank_tc(int nprobe, int d) {
@@ -252,7 +330,7 @@ cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t 
         else
             k_rank_tc<<<std::min(tiles, num_sms()), tcp::kThreads, tc_smem(), st>>>(a);
         const unsigned blocks = (unsigned)ceil_div(n, kSelectWarps);
-        const size_t smem = (size_t)kSelectWarps * 2 * P * 4;
+        const size_t smem = (size_t)kSelectWarps * 2 * (2 * P) * 4;
         int32_t *o = order + q0 * nprobe;
         float *cs = cscores ? cscores + q0 * nprobe : nullptr;
         switch (kpl) {

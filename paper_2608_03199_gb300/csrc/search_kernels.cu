@@ -148,13 +148,25 @@ __device__ __forceinline__ void count_tiles(int c, int tc_min, int &n_tc, int &n
     }
 }
 
+// Tensor-core tiles are listed longest first (by the partition's 128-row
+// chunks, capped), so the blocks that draw them from the work counter finish
+// together; the tiles of one partition stay adjacent.
+constexpr int kTileClasses = 128;
+__device__ __forceinline__ int tile_class(const SearchArgs &a, int64_t p) {
+    const int64_t ch = ceil_div(a.off[p + 1] - a.off[p], kTcTile);
+    return ch < kTileClasses - 1 ? (int)ch : kTileClasses - 1;
+}
+
 __global__ void __launch_bounds__(kBucketThreads) k_bucket(SearchArgs a) {
     __shared__ int warp_tot[32];
     __shared__ int sums[3];
+    __shared__ int cls[kTileClasses];   // tensor-core tiles per class, then class cursors
     Ctl *ctl = a.ctl;
     const int64_t nl = a.nlist;
     const int per = (int)ceil_div(nl, kBucketThreads);
     const int64_t p0 = (int64_t)threadIdx.x * per;
+    for (int i = threadIdx.x; i < kTileClasses; i += blockDim.x) cls[i] = 0;
+    __syncthreads();
     int my[3] = {0, 0, 0};   // items, SIMT tiles, tensor-core tiles
     int my_groups = 0;
     for (int64_t p = p0; p < p0 + per && p < nl; ++p) {
@@ -165,6 +177,7 @@ __global__ void __launch_bounds__(kBucketThreads) k_bucket(SearchArgs a) {
         my[1] += ns;
         my[2] += ntc;
         my_groups += c > 0;
+        if (ntc) atomicAdd(&cls[tile_class(a, p)], ntc);
     }
     // three exclusive scans over threads
     const unsigned lane = lane_id(), warp = threadIdx.x >> 5;
@@ -190,10 +203,22 @@ __global__ void __launch_bounds__(kBucketThreads) k_bucket(SearchArgs a) {
         ex[v] = (warp > 0 ? warp_tot[warp - 1] : 0) + x - my[v];
         __syncthreads();
     }
-    int ioff = ex[0], soff = ex[1], toff = ex[2];
+    if (threadIdx.x == 0) {   // class cursors: exclusive scan, longest class first
+        int run = 0;
+        for (int i = kTileClasses - 1; i >= 0; --i) {
+            const int v = cls[i];
+            cls[i] = run;
+            run += v;
+        }
+    }
+    __syncthreads();
+    int ioff = ex[0], soff = ex[1];
     for (int64_t p = p0; p < p0 + per && p < nl; ++p) {
         const int c = a.counts[p];
         a.cursor[p] = ioff;
+        int ntc, ns;
+        count_tiles(c, a.tc_min, ntc, ns);
+        int toff = ntc ? atomicAdd(&cls[tile_class(a, p)], ntc) : 0;
         for (int o = 0; o < c; o += kTcTile) {
             const int sz = c - o < kTcTile ? c - o : kTcTile;
             if (a.tc_min > 0 && sz >= a.tc_min) {

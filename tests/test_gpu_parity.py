@@ -88,6 +88,34 @@ def test_rank_parity(tiny, g_tiny, dev):
         assert bad.sum() <= 2
 
 
+@pytest.mark.parametrize("nlist", [1, 33, 64, 100, 1000, 2048])
+def test_rank_selection_exact_ties(nlist, dev):
+    """Scores that are exact in fp32 and fp64 (multiples of 1/64 from
+    coordinates in {-2..2}/8), so equal scores tie exactly: the order must be
+    the (score desc, id asc) sort, for every nprobe shape, including all-equal
+    rows and far more ties than nprobe."""
+    rng = np.random.default_rng(nlist)
+    d = 8
+    C = (rng.integers(-2, 3, size=(nlist, d)) / 8).astype(np.float32)
+    if nlist >= 64:
+        C[nlist // 2:nlist // 2 + 20] = C[3]          # a block of identical centroids
+    Q = (rng.integers(-2, 3, size=(300, d)) / 8).astype(np.float32)
+    Q[0] = 0.0                                        # every score 0: ids in order
+    Cd = torch.from_numpy(C).to(dev)
+    index = sieve.build_layout(Cd.clone(), torch.arange(nlist, dtype=torch.int32, device=dev),
+                               nlist, Cd)
+    Qd = torch.from_numpy(Q).to(dev)
+    ref_sc = Q.astype(np.float64) @ C.astype(np.float64).T
+    for nprobe in sorted({1, 2, 5, max(1, nlist // 2), min(nlist, 64), min(nlist, 512), nlist}):
+        if nprobe > min(nlist, 512):
+            continue
+        order, sc = sieve.rank_partitions(index, Qd, nprobe, return_scores=True)
+        order, sc = order.cpu().numpy(), sc.cpu().numpy()
+        ref = np.stack([np.lexsort((np.arange(nlist), -row))[:nprobe] for row in ref_sc])
+        assert np.array_equal(order, ref), nprobe
+        assert np.array_equal(sc.astype(np.float64), np.take_along_axis(ref_sc, ref, 1))
+
+
 @pytest.mark.parametrize("lookahead", [0, 1])
 def test_search_parity_tiny(tiny, g_tiny, lookahead):
     c = tiny["cfg"]
