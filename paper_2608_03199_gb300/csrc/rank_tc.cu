@@ -76,7 +76,10 @@ struct RankMode {
                 dst[j] = make_float4(v[4 * j] * kS, v[4 * j + 1] * kS, v[4 * j + 2] * kS, v[4 * j + 3] * kS);
         }
         __device__ void end(const Args &, const Tile &) {}
+        __device__ void stage(const Args &, const Tile &, int64_t, int) {}
+        __device__ void use_staged(int) {}
     };
+    static constexpr bool kStage = false;
 };
 
 __global__ void __launch_bounds__(tcp::kThreads, 1) k_rank_tc(RankArgs a) {

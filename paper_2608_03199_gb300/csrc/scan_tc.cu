@@ -16,6 +16,19 @@ namespace sieve {
 
 __device__ __forceinline__ int tc_nkb_dev(int d) { return (d + 63) / 64; }
 
+// v[j] for a j known only at run time, by a tree of selects (no local memory)
+__device__ __forceinline__ float pick32(const float (&v)[32], int j) {
+    float t16[16], t8[8], t4[4];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) t16[i] = (j & 16) ? v[i + 16] : v[i];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) t8[i] = (j & 8) ? t16[i + 8] : t16[i];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) t4[i] = (j & 4) ? t8[i + 4] : t8[i];
+    const float t0 = (j & 2) ? t4[2] : t4[0], t1 = (j & 2) ? t4[3] : t4[1];
+    return (j & 1) ? t1 : t0;
+}
+
 struct ScanMode {
     using Args = SearchArgs;
     static constexpr int kN = 256;
@@ -48,9 +61,15 @@ struct ScanMode {
         return a.tc_rows + (a.tc_row_blocks[T.p] + ch) * (int64_t)tc_nkb_dev(a.d) * kTcBlockBytes;
     }
 
+    // the bulk pipeline stages each chunk's 128 row ids in shared memory
+    static constexpr bool kStage = true;
+    static constexpr int kStageRows = 128;
+
     struct Epi {
         float *ks;
         long long *ki;
+        long long *stage_buf;          // 2 x 128 staged row ids (bulk pipeline)
+        const long long *ids_s;        // the current chunk's staged ids, or nullptr
         int kn, item, q, rank, slot;
         bool valid;
         long long qid;
@@ -61,6 +80,8 @@ struct ScanMode {
             slot = slot_;
             ks = reinterpret_cast<float *>(smem) + slot;
             ki = reinterpret_cast<long long *>(reinterpret_cast<float *>(smem) + tcp::kM * a.k) + slot;
+            stage_buf = reinterpret_cast<long long *>(smem + (size_t)tcp::kM * a.k * 12);
+            ids_s = nullptr;
             kn = 0;
             valid = slot < T.ni;
             item = q = rank = 0;
@@ -72,10 +93,14 @@ struct ScanMode {
                 if (a.qids) qid = a.qids[q];
             }
         }
-        // one candidate row (s >= tau): self exclusion, then the sorted insert;
-        // kept out of line so the per-chunk loop stays a short run of compares
-        __device__ __noinline__ void take(const Args &a, const Tile &T, int64_t col, float sc) {
-            const long long id = a.ids[T.r_begin + col];
+        __device__ void stage(const Args &a, const Tile &T, int64_t col0, int buf) {
+            const int64_t r = col0 + slot;
+            stage_buf[buf * kStageRows + slot] = r < T.nb ? a.ids[T.r_begin + r] : -1;
+        }
+        __device__ void use_staged(int buf) { ids_s = stage_buf + buf * kStageRows; }
+        // one candidate row (s >= tau): self exclusion, then the sorted insert
+        __device__ __forceinline__ void take(const Args &a, const Tile &T, int64_t col, float sc) {
+            const long long id = ids_s ? ids_s[col & (kStageRows - 1)] : a.ids[T.r_begin + col];
             if (id == qid) return;
             const int k = a.k;
             if (kn == k && !ranks_before(sc, id, KS(k - 1), KI(k - 1))) return;
@@ -92,14 +117,30 @@ struct ScanMode {
         __device__ void chunk(const Args &a, const Tile &T, int64_t col0, const float (&v)[32],
                               int ncol) {
             if (!valid) return;
-            const float tau_raw = a.tau * 65536.f;   // exact: a power-of-two scale
+            // a candidate needs s >= tau and, once k are kept, s >= the k-th
+            // kept score (equal scores go on to the id tie-break); scores
+            // here are raw (x 2^16, an exact power-of-two scale)
+            float thr = a.tau * 65536.f;
+            if (kn == a.k) thr = fmaxf(thr, KS(a.k - 1) * 65536.f);
+            // nearly every group has no candidate: one tree of maxima decides
+            float mx[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) mx[j] = fmaxf(v[j], v[j + 16]);
+#pragma unroll
+            for (int w = 8; w > 0; w >>= 1)
+#pragma unroll
+                for (int j = 0; j < w; ++j) mx[j] = fmaxf(mx[j], mx[j + w]);
+            if (!(mx[0] >= thr)) return;
             unsigned m = 0;
 #pragma unroll
-            for (int j = 0; j < 32; ++j) m |= (v[j] >= tau_raw && j < ncol) ? (1u << j) : 0u;
-            if (m == 0) return;
-#pragma unroll
-            for (int j = 0; j < 32; ++j)
-                if (m & (1u << j)) take(a, T, col0 + j, v[j] * (1.f / 65536.f));
+            for (int j = 0; j < 32; ++j) m |= (v[j] >= thr && j < ncol) ? (1u << j) : 0u;
+            // one candidate at a time in a loop that is not unrolled: a single
+            // copy of the insert, the score picked out of the registers
+            while (m) {
+                const int j = __ffs(m) - 1;
+                m &= m - 1u;
+                take(a, T, col0 + j, pick32(v, j) * (1.f / 65536.f));
+            }
         }
         __device__ void end(const Args &a, const Tile &T) {
             if (valid) {
@@ -124,6 +165,8 @@ struct ScanMode {
     };
 };
 
+static_assert(tcb::kN == ScanMode::kStageRows, "a staged chunk is one tensor-layout block");
+
 size_t scan_tc_smem_bytes(int k) {
     return tcp::Geometry<ScanMode::kN>::smem_bytes((size_t)tcp::kM * k * (sizeof(float) + sizeof(long long)));
 }
@@ -133,7 +176,11 @@ __global__ void __launch_bounds__(tcp::kThreads, 1) k_scan_tc(SearchArgs a) {
     tcp::run_pipeline<ScanMode>(a, smem_raw);
 }
 
-static size_t scan_epi_bytes(int k) { return (size_t)tcp::kM * k * (sizeof(float) + sizeof(long long)); }
+// kept lists, then the two staged id buffers
+static size_t scan_epi_bytes(int k) {
+    return (size_t)tcp::kM * k * (sizeof(float) + sizeof(long long)) +
+           2 * ScanMode::kStageRows * sizeof(long long);
+}
 
 int scan_bulk_stages(int d, int k) {
     return tcb::stages_for((int)ceil_div(d, 64), scan_epi_bytes(k), 232448 - 128);

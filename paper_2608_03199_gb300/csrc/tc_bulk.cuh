@@ -73,17 +73,31 @@ inline int stages_for(int nkb, size_t epi_bytes, size_t smem_limit) {
     return s >= 2 ? s : 0;
 }
 
+// one 32-column group of an accumulator row to the mode's epilogue
+template <class Epi, class Args, class Tile>
+__device__ __forceinline__ void hand(Epi &epi, const Args &a, const Tile &T, int64_t col0,
+                                     const uint32_t (&r)[32]) {
+    float v[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+    const int64_t left = T.nb - col0;
+    epi.chunk(a, T, col0, v, left < 32 ? (int)left : 32);
+}
+
 // Mode provides (in addition to what tc_pipeline.cuh asks): b_block(a, T, ch)
-// = pointer to the tensor-layout bytes of the tile's ch-th block of B rows, and
+// = pointer to the tensor-layout bytes of the tile's ch-th block of B rows;
 // tile_counter(a) = a zeroed global int the blocks draw tiles from (nullptr:
-// block b takes tiles b, b + gridDim.x, ...).
+// block b takes tiles b, b + gridDim.x, ...); kStage: when true, before each
+// chunk every epilogue thread calls Epi::stage(a, T, col0, buf) (its share of
+// per-column data into shared-memory buffer buf), the 128 threads meet on an
+// mbarrier, and each calls Epi::use_staged(buf).
 template <class Mode>
 __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned char *smem_raw,
                                          int stages) {
     constexpr uint32_t kIdesc = tc::idesc_f16(tcp::kM, kN);
     __shared__ __align__(8) uint64_t a_full[kMaxKb], a_empty[kMaxKb], b_full[kMaxStages],
         b_empty[kMaxStages], dfull_bar[2], dempty_bar[2], drain_bar, ring_full[kRing],
-        ring_empty[kRing];
+        ring_empty[kRing], staged_bar[2];
     __shared__ int ring_tile[kRing];
     __shared__ uint32_t tmem_slot;
     __shared__ int s_abort;
@@ -111,6 +125,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
         for (int b = 0; b < 2; ++b) {
             tc::mbar_init(&dfull_bar[b], 1);
             tc::mbar_init(&dempty_bar[b], 4 * 32);
+            tc::mbar_init(&staged_bar[b], 4 * 32);
         }
         for (int r = 0; r < kRing; ++r) {
             tc::mbar_init(&ring_full[r], 1);
@@ -287,19 +302,36 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
             epi.begin(a, T, slot, epi_smem);
             for (int ch = 0; ch < nch; ++ch, ++c) {
                 const uint32_t buf = c & 1u, dph = (c >> 1) & 1u;
+                if (Mode::kStage) {   // per-column data of the chunk, shared by the 128 rows
+                    epi.stage(a, T, (int64_t)ch * kN, (int)buf);
+                    tc::mbar_arrive(&staged_bar[buf]);
+                    ok = __all_sync(0xffffffffu, wait(&staged_bar[buf], dph));
+                    if (!ok) break;
+                    epi.use_staged((int)buf);
+                }
                 ok = __all_sync(0xffffffffu, wait(&dfull_bar[buf], dph));
                 if (!ok) break;
                 tc::fence_after_sync();
-#pragma unroll 1
-                for (int cc = 0; cc < kN / 32; ++cc) {
-                    float v[32];
-                    tc::tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + buf * kN + cc * 32, v);
-                    const int64_t col0 = (int64_t)ch * kN + cc * 32;
-                    const int64_t left = T.nb - col0;
-                    epi.chunk(a, T, col0, v, left < 32 ? (int)left : 32);
-                }
+                // four 32-column loads, each issued before the previous group is
+                // handed to the mode; the accumulator is released as soon as
+                // the last load has landed
+                const uint32_t taddr = tmem + ((uint32_t)(quarter * 32) << 16) + buf * kN;
+                const int64_t col0 = (int64_t)ch * kN;
+                uint32_t ra[32], rb[32];
+                tc::tmem_ld32_issue(taddr, ra);
+                tc::tmem_ld_wait(ra);
+                tc::tmem_ld32_issue(taddr + 32, rb);
+                hand(epi, a, T, col0, ra);
+                tc::tmem_ld_wait(rb);
+                tc::tmem_ld32_issue(taddr + 64, ra);
+                hand(epi, a, T, col0 + 32, rb);
+                tc::tmem_ld_wait(ra);
+                tc::tmem_ld32_issue(taddr + 96, rb);
+                hand(epi, a, T, col0 + 64, ra);
+                tc::tmem_ld_wait(rb);
                 tc::fence_before_sync();
                 tc::mbar_arrive(&dempty_bar[buf]);
+                hand(epi, a, T, col0 + 96, rb);
             }
             if (!ok) break;
             epi.end(a, T);
