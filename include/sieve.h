@@ -100,10 +100,10 @@ typedef struct {
  *              stats pointer); 0 = no timing
  *   scan_path  which units compute similarities; all paths give the same
  *              decisions up to fp32 rounding (see the parity notes):
- *              0 = automatic (ranking on the tensor cores when nlist <= 2048;
- *              every partition group on the tensor cores when k <= 16, on
- *              FP32 FMA otherwise), 1 = FP32 FMA only, 2 = tensor cores
- *              (needs k <= 16)
+ *              0 = automatic (ranking on the tensor cores; every partition
+ *              group on the tensor cores when k <= 16, on FP32 FMA
+ *              otherwise), 1 = FP32 FMA only, 2 = tensor cores (needs
+ *              k <= 16)
  */
 typedef struct {
     float tau;
@@ -197,14 +197,16 @@ sieve_status sieve_build_tc_layout(const sieve_index_view *ix, void *tc_rows,
 
 /* Centroid ranking (Sec. 2.3, Sec. 4.1): for every query, the nprobe
  * centroids with the largest inner product, best first; equal scores rank
- * the lower centroid id first.  Scores are fp32-accurate: tensor cores with
- * a 3xTF32 split and a score table in the workspace when nlist <= 2048,
- * FP32 FMA with a fused selection otherwise.
+ * the lower centroid id first.  Scores come from the tensor cores with the
+ * three-product fp16 split (each fp32 value = hi + lo fp16, scaled by 256),
+ * accurate to a few 1e-7 on unit vectors; they go through a score table of at
+ * most 512 MiB per chunk of queries in the workspace, and a warp per
+ * (query, 2,048 centroids) keeps the best nprobe, level by level.
  *   Q        device [nq][d] fp32
  *   order    device [nq][nprobe] int32 out, 0-based centroid ids
  *   cscores  device [nq][nprobe] fp32 out (nullable): the matching scores
- *   ws       workspace of sieve_rank_workspace_size bytes (0 bytes, ws may
- *            be NULL, when nlist > 2048); SIEVE_EWORKSPACE if smaller */
+ *   ws       workspace of sieve_rank_workspace_size bytes; SIEVE_EWORKSPACE
+ *            if smaller */
 sieve_status sieve_rank_workspace_size(const sieve_index_view *ix, int64_t nq, int32_t nprobe,
                                        size_t *bytes);
 sieve_status sieve_rank_partitions(const sieve_index_view *ix, const float *Q, int64_t nq,

@@ -195,6 +195,11 @@ class Index:
         return self.vectors.shape[1]
 
 
+# widest rows the bulk tensor-core pipelines take (their A operand lives in
+# tensor memory: at most four 64-element K-blocks)
+TC_BULK_MAX_D = 256
+
+
 def add_tc_layout(index: Index, stream=None) -> Index:
     """The same index with its tensor-core layout built (sieve_build_tc_layout)."""
     base = index.without_tc_layout()
@@ -210,9 +215,10 @@ def add_tc_layout(index: Index, stream=None) -> Index:
     return Index(index.vectors, index.ids, index.list_offsets, index.centroids, rows, blocks, cent)
 
 
-def build_layout(X, assign, nlist, centroids, stream=None, tc_layout=True) -> Index:
+def build_layout(X, assign, nlist, centroids, stream=None, tc_layout=None) -> Index:
     """Index from rows X [n][d] and their partitions assign [n] (sieve_build_layout),
-    with its tensor-core layout unless ``tc_layout`` is False.
+    with its tensor-core layout when ``tc_layout`` is True, or by default when
+    d <= 256 (the width the bulk tensor-core pipelines take).
 
     ids of the index are the row numbers of X."""
     _need_cuda(X, torch.float32, "X", 2)
@@ -229,6 +235,8 @@ def build_layout(X, assign, nlist, centroids, stream=None, tc_layout=True) -> In
     _check(L.sieve_build_layout(_ptr(X), _ptr(assign), n, d, nlist, _ptr(Xs), _ptr(ids), _ptr(off),
                                 _ptr(ws), nbytes.value, _stream(stream)), "sieve_build_layout")
     index = Index(Xs, ids, off, centroids.contiguous())
+    if tc_layout is None:
+        tc_layout = d <= TC_BULK_MAX_D
     return add_tc_layout(index, stream) if tc_layout else index
 
 

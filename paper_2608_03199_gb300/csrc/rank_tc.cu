@@ -1,22 +1,27 @@
 // rank_tc.cu -- centroid ranking on the tcgen05 tensor cores (Sec. 2.3,
 // Sec. 4.1: P_i = the nprobe centroids with the largest inner product with
-// q_i, best first, equal scores by lower centroid id), for nlist <= 2048.
+// q_i, best first, equal scores by lower centroid id), for any nlist.
 //
-// Two kernels per chunk of queries:
-//   k_rank_tc  the 3xTF32 pipeline of tc_pipeline.cuh: 128 consecutive
-//              queries (A rows) against all centroids (B rows, 128 per
+// Per chunk of queries:
+//   k_rank_bulk / k_rank_tc  the tensor-core contraction (tc_bulk.cuh with the
+//              centroids' tensor-core layout, else the converter pipeline of
+//              tc_pipeline.cuh): a tile is 128 consecutive queries (A rows)
+//              against one range of kRankRange centroids (B rows, 128 per
 //              chunk); each epilogue thread stores its query's scores into a
 //              score table [queries][ld] in the caller's workspace
-//   k_select   one warp per query: the query's scores sit in registers
-//              (nlist / 32 per lane); the exact nprobe-th largest score is
-//              found bit by bit (32 rounds of "how many scores are >= t"),
-//              the entries above it plus the lowest-id entries equal to it
-//              are gathered, and a warp bitonic network sorts them by
-//              (score desc, id asc).
+//   k_select   one warp per (query, segment of at most kSelectSeg entries):
+//              the segment's best min(nprobe, size) entries, sorted by
+//              (score desc, id asc).  With nlist <= kSelectSeg one segment
+//              gives the order directly; otherwise each level keeps the best
+//              nprobe of every segment (the nprobe best of a set lie among the
+//              nprobe best of each of its parts) until one segment is left.
 #include "tc_bulk.cuh"
 #include "tc_pipeline.cuh"
 
 namespace sieve {
+
+constexpr int64_t kRankRange = 2048;   // centroids per tile (a multiple of 128)
+constexpr int kSelectSeg = 2048;       // entries per selecting warp (64 per lane)
 
 struct RankArgs {
     const float *Q;
@@ -28,6 +33,8 @@ struct RankArgs {
     int64_t ld;      // row stride of the table, a multiple of 32
     int *status;     // nullable: where a bounded wait that gives up is reported
     const unsigned char *tc_cent;   // tensor-core layout of the centroids (bulk path)
+    float *gmax;     // nullable: [nq][gld] maxima of each 32-centroid group
+    int64_t gld;
 };
 
 __device__ int g_rank_status_sink;
@@ -36,51 +43,65 @@ struct RankMode {
     using Args = RankArgs;
     static constexpr int kN = 128;
     struct Tile {
-        int64_t q0;
+        int64_t q0;    // first query
         int ni;
-        int64_t nb;
+        int64_t c0;    // first centroid of the tile's range
+        int64_t nb;    // centroids in the range
     };
-    __device__ static int num_tiles(const Args &a) { return (int)ceil_div(a.nq, tcp::kM); }
-    // every tile costs the same: a static stride over the blocks
+    __device__ static int n_ranges(const Args &a) { return (int)ceil_div(a.nlist, kRankRange); }
+    __device__ static int num_tiles(const Args &a) { return (int)ceil_div(a.nq, tcp::kM) * n_ranges(a); }
+    // every tile costs about the same: a static stride over the blocks
     __device__ static int *tile_counter(const Args &) { return nullptr; }
     __device__ static int d(const Args &a) { return a.d; }
     __device__ static int *status(const Args &a) { return a.status ? a.status : &g_rank_status_sink; }
     __device__ static Tile tile(const Args &a, int t) {
+        const int nr = n_ranges(a);
         Tile T;
-        T.q0 = (int64_t)t * tcp::kM;
+        T.q0 = (int64_t)(t / nr) * tcp::kM;
         T.ni = (int)(a.nq - T.q0 < tcp::kM ? a.nq - T.q0 : tcp::kM);
-        T.nb = a.nlist;
+        T.c0 = (int64_t)(t % nr) * kRankRange;
+        T.nb = a.nlist - T.c0 < kRankRange ? a.nlist - T.c0 : kRankRange;
         return T;
     }
     __device__ static const float *a_row(const Args &a, const Tile &T, int i) {
         return i < T.ni ? a.Q + (T.q0 + i) * a.d : nullptr;
     }
     __device__ static const float *b_row(const Args &a, const Tile &T, int64_t r) {
-        return r < T.nb ? a.C + r * a.d : nullptr;
+        return r < T.nb ? a.C + (T.c0 + r) * a.d : nullptr;
     }
-    __device__ static const unsigned char *b_block(const Args &a, const Tile &, int ch) {
-        return a.tc_cent + (int64_t)ch * ((a.d + 63) / 64) * kTcBlockBytes;
+    __device__ static const unsigned char *b_block(const Args &a, const Tile &T, int ch) {
+        return a.tc_cent + (T.c0 / kTcRows + ch) * (int64_t)((a.d + 63) / 64) * kTcBlockBytes;
     }
+    static constexpr bool kStage = false;
     struct Epi {
         float *row;
+        float *grow;   // this query's group maxima from the range start, or nullptr
         __device__ void begin(const Args &a, const Tile &T, int slot, unsigned char *) {
-            row = slot < T.ni ? a.scores + (T.q0 + slot) * a.ld : nullptr;
+            row = slot < T.ni ? a.scores + (T.q0 + slot) * a.ld + T.c0 : nullptr;
+            grow = (slot < T.ni && a.gmax) ? a.gmax + (T.q0 + slot) * a.gld + T.c0 / 32 : nullptr;
         }
         // v holds the chunk's raw accumulator values: scores x 2^16
         __device__ void chunk(const Args &a, const Tile &, int64_t col0, const float (&v)[32], int ncol) {
-            if (!row || ncol <= 0) return;   // ld is a multiple of 32: whole 32-column groups fit
+            // ld and the range start are multiples of 32: whole 32-column groups fit
+            if (!row || ncol <= 0) return;
             constexpr float kS = 1.f / 65536.f;
             float4 *dst = reinterpret_cast<float4 *>(row + col0);
 #pragma unroll
             for (int j = 0; j < 8; ++j)
                 dst[j] = make_float4(v[4 * j] * kS, v[4 * j + 1] * kS, v[4 * j + 2] * kS, v[4 * j + 3] * kS);
+            if (grow) {   // the group's maximum over its real columns only
+                float mx = v[0];
+#pragma unroll
+                for (int j = 1; j < 32; ++j) mx = j < ncol ? fmaxf(mx, v[j]) : mx;
+                grow[col0 / 32] = mx * kS;
+            }
         }
         __device__ void end(const Args &, const Tile &) {}
         __device__ void stage(const Args &, const Tile &, int64_t, int) {}
         __device__ void use_staged(int) {}
     };
-    static constexpr bool kStage = false;
 };
+static_assert(kRankRange % RankMode::kN == 0 && kRankRange % kTcRows == 0, "");
 
 __global__ void __launch_bounds__(tcp::kThreads, 1) k_rank_tc(RankArgs a) {
     extern __shared__ unsigned char smem_raw[];
@@ -102,6 +123,11 @@ __device__ __forceinline__ uint32_t order_key(float s) {
     return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
+// the inverse of order_key
+__device__ __forceinline__ float key_score(uint32_t k) {
+    return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
+}
+
 constexpr int kSelectWarps = 4;
 constexpr int kSelectMaxR = 4;   // lane order statistics used for the lower bracket
 
@@ -119,40 +145,16 @@ __device__ __forceinline__ int count_ge(const uint32_t (&key)[KPL], uint32_t t) 
     return warp_sum(c);
 }
 
-// One warp per query.  T* = the nprobe-th largest key.  The search keeps a
-// threshold T <= T* with C = #{keys >= T} >= nprobe and refines T bit by bit
-// (the largest T with at least nprobe keys >= T) until C fits the sort
-// buffer; it starts from the common high bits of a bracket L <= T* <= U
-// (U = the largest key; L = the smallest over lanes of each lane's
-// ceil(nprobe / 32)-th largest key, so at least nprobe keys are >= L).  The
-// C candidates >= T contain the nprobe best, which a bitonic sort by
-// (score desc, id asc) puts first.  When C never fits (many equal scores),
-// the search ends at T = T* and takes the keys > T* plus the lowest-id keys
-// equal to it.  P: a power of two >= nprobe; the buffer holds 2P entries.
-template <int KPL>   // scores per lane: nlist <= 32 * KPL
-__global__ void __launch_bounds__(kSelectWarps * 32) k_select(const float *__restrict__ scores,
-                                                              int64_t ld, int64_t nq, int nlist,
-                                                              int nprobe, int P,
-                                                              int32_t *__restrict__ order,
-                                                              float *__restrict__ cscores) {
-    extern __shared__ __align__(16) unsigned char sel_smem[];
-    const int cap = 2 * P;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    float *bs = reinterpret_cast<float *>(sel_smem) + warp * 2 * cap;   // cap scores, then cap ids
-    int *bc = reinterpret_cast<int *>(bs + cap);
-    const int64_t q = (int64_t)blockIdx.x * kSelectWarps + warp;
-    if (q >= nq) return;
-    const float *row = scores + q * ld;
-    float s[KPL];
-    uint32_t key[KPL];
-#pragma unroll
-    for (int j = 0; j < KPL; ++j) {
-        const int c = j * 32 + lane;
-        s[j] = c < nlist ? row[c] : 0.f;
-        key[j] = c < nlist ? order_key(s[j]) : 0u;   // padding ranks below every score
-    }
-    // bracket: per lane the r largest keys (a small insertion network)
-    const int r = (nprobe + 31) / 32;
+// A threshold T <= T* (T* = the want-th largest of the warp's keys; keys of
+// padding are 0, below every score) with C = #{keys >= T} >= want, refined
+// bit by bit (the largest T with at least want keys >= T) until C <= cap or
+// T == T*.  The search starts from the common high bits of a bracket
+// L <= T* <= U: U = the largest key, L = the smallest over lanes of each
+// lane's ceil(want / 32)-th largest key (at least want keys are >= L).
+template <int KPL>
+__device__ __forceinline__ void warp_threshold(const uint32_t (&key)[KPL], int want, int cap,
+                                               uint32_t &T, int &C) {
+    const int r = (want + 31) / 32;
     uint32_t m[kSelectMaxR] = {0u, 0u, 0u, 0u};
     if (r <= 2) {
 #pragma unroll
@@ -180,7 +182,6 @@ __global__ void __launch_bounds__(kSelectWarps * 32) k_select(const float *__res
         L = min(L, __shfl_xor_sync(0xffffffffu, L, o));
     }
     int b;
-    uint32_t T;
     if (L == U) {
         b = -1;
         T = L;
@@ -188,47 +189,60 @@ __global__ void __launch_bounds__(kSelectWarps * 32) k_select(const float *__res
         b = 31 - __clz(L ^ U);                                // highest bit where they differ
         T = b == 31 ? 0u : (L & ~((2u << b) - 1u));           // their common high bits
     }
-    int C = count_ge(key, T);
+    C = count_ge(key, T);
     for (; b >= 0 && C > cap; --b) {
         const uint32_t t = T | (1u << b);
-        const int cnt = count_ge(key, t);
-        if (cnt >= nprobe) {
+        const int c = count_ge(key, t);
+        if (c >= want) {
             T = t;
-            C = cnt;
+            C = c;
         }
     }
+}
+
+// The want best of the warp's cnt entries (entry c = key[c / 32] of lane
+// c % 32; its id from id_of(c)), sorted by (score desc, id asc) into bs/bc,
+// given T and C from warp_threshold.  C <= cap: every key >= T is a candidate;
+// otherwise T == T* and the keys > T* plus the first keys equal to it in entry
+// order are taken, which are the lowest ids when entry order is id order among
+// equal scores.  bs/bc hold 2P >= cap entries; returns the count sorted.
+template <int KPL, class IdOf>
+__device__ __forceinline__ void warp_gather_sort(const uint32_t (&key)[KPL], int cnt, int want,
+                                                 uint32_t T, int C, int cap, IdOf id_of,
+                                                 float *bs, int *bc) {
+    const int lane = threadIdx.x & 31;
     const unsigned below = (1u << lane) - 1u;
     int pos = 0;
     if (C <= cap) {
-        // every key >= T, in increasing id order (id = 32 j + lane)
 #pragma unroll
         for (int j = 0; j < KPL; ++j) {
-            const bool sel = key[j] >= T && j * 32 + lane < nlist;
+            const int c = j * 32 + lane;
+            const bool sel = key[j] >= T && c < cnt;
             const unsigned sb = __ballot_sync(0xffffffffu, sel);
             if (sel) {
                 const int p = pos + __popc(sb & below);
-                bs[p] = s[j];
-                bc[p] = j * 32 + lane;
+                bs[p] = key_score(key[j]);
+                bc[p] = id_of(c);
             }
             pos += __popc(sb);
         }
     } else {
-        // T == T*: the keys above it, then the lowest-id keys equal to it
         int gt = 0;
 #pragma unroll
         for (int j = 0; j < KPL; ++j) gt += key[j] > T;
-        const int ties_wanted = nprobe - warp_sum(gt);   // >= 1
+        const int ties_wanted = want - warp_sum(gt);   // >= 1
         int ties_seen = 0;
 #pragma unroll
         for (int j = 0; j < KPL; ++j) {
-            const bool tie = key[j] == T && j * 32 + lane < nlist;
+            const int c = j * 32 + lane;
+            const bool tie = key[j] == T && c < cnt;
             const unsigned tb = __ballot_sync(0xffffffffu, tie);
             const bool sel = key[j] > T || (tie && ties_seen + __popc(tb & below) < ties_wanted);
             const unsigned sb = __ballot_sync(0xffffffffu, sel);
             if (sel) {
                 const int p = pos + __popc(sb & below);
-                bs[p] = s[j];
-                bc[p] = j * 32 + lane;
+                bs[p] = key_score(key[j]);
+                bc[p] = id_of(c);
             }
             pos += __popc(sb);
             ties_seen += __popc(tb);
@@ -260,6 +274,203 @@ __global__ void __launch_bounds__(kSelectWarps * 32) k_select(const float *__res
             __syncwarp();
         }
     }
+}
+
+// One warp per (query, segment).  The segment's entries are positions
+// s*seg .. min(M, (s+1)*seg)-1 of the query's row of `in_s` (ids from `in_id`,
+// or the position itself when in_id is null), in id order among equal scores
+// (a row of centroid scores, or the sorted outputs of consecutive id ranges);
+// want = min(nprobe, entries).  Output: the want best in order at
+// out_id/out_s[q * out_ld + s * nprobe ..], then (-inf, INT32_MAX) padding up
+// to nprobe.  `only` (nullable): queries with only[q] == 0 are skipped.
+// P: a power of two >= nprobe; the sort buffer holds 2P entries.
+template <int KPL>   // entries per lane: seg <= 32 * KPL
+__global__ void __launch_bounds__(kSelectWarps * 32) k_select(
+    const float *__restrict__ in_s, const int32_t *__restrict__ in_id, int64_t in_ld, int64_t nq,
+    int64_t M, int seg, int nseg, int nprobe, int P, int32_t *__restrict__ out_id,
+    float *__restrict__ out_s, int64_t out_ld, const int *__restrict__ only) {
+    extern __shared__ __align__(16) unsigned char sel_smem[];
+    const int cap = 2 * P;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    float *bs = reinterpret_cast<float *>(sel_smem) + warp * 2 * cap;   // cap scores, then cap ids
+    int *bc = reinterpret_cast<int *>(bs + cap);
+    const int64_t w = (int64_t)blockIdx.x * kSelectWarps + warp;
+    if (w >= nq * nseg) return;
+    const int64_t q = w / nseg;
+    if (only && only[q] == 0) return;
+    const int sg = (int)(w % nseg);
+    const int64_t p0 = (int64_t)sg * seg;
+    const int cnt = (int)(M - p0 < seg ? M - p0 : seg);
+    const int want = nprobe < cnt ? nprobe : cnt;
+    const float *row = in_s + q * in_ld + p0;
+    const int32_t *rid = in_id ? in_id + q * in_ld + p0 : nullptr;
+    uint32_t key[KPL];   // the scores themselves are recovered from the keys
+#pragma unroll
+    for (int j = 0; j < KPL; ++j) {
+        const int c = j * 32 + lane;
+        key[j] = c < cnt ? order_key(row[c]) : 0u;   // padding ranks below every score
+    }
+    uint32_t T;
+    int C;
+    warp_threshold(key, want, cap, T, C);
+    warp_gather_sort(key, cnt, want, T, C, cap,
+                     [&](int c) { return rid ? rid[c] : (int)(p0 + c); }, bs, bc);
+    int32_t *oi = out_id + q * out_ld + (int64_t)sg * nprobe;
+    float *os = out_s ? out_s + q * out_ld + (int64_t)sg * nprobe : nullptr;
+    for (int p = lane; p < nprobe; p += 32) {
+        oi[p] = p < want ? bc[p] : INT32_MAX;
+        if (os) os[p] = p < want ? bs[p] : -__int_as_float(0x7f800000);
+    }
+}
+
+// Threshold from group maxima: one warp per query over its ng maxima of
+// 32-centroid groups (ng >= nprobe).  The nprobe-th largest maximum L is a
+// score of nprobe different centroids at least, so at least nprobe scores are
+// >= L and the nprobe best all are.  Writes the order key of L.
+template <int KPL>
+__global__ void __launch_bounds__(kSelectWarps * 32) k_group_threshold(
+    const float *__restrict__ gmax, int64_t gld, int64_t nq, int ng, int nprobe,
+    uint32_t *__restrict__ lkey) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t q = (int64_t)blockIdx.x * kSelectWarps + warp;
+    if (q >= nq) return;
+    const float *row = gmax + q * gld;
+    uint32_t key[KPL];
+#pragma unroll
+    for (int j = 0; j < KPL; ++j) {
+        const int c = j * 32 + lane;
+        key[j] = c < ng ? order_key(row[c]) : 0u;
+    }
+    uint32_t T;
+    int C;
+    warp_threshold(key, nprobe, nprobe, T, C);   // refined to the nprobe-th largest
+    if (lane == 0) lkey[q] = T;
+}
+
+constexpr int kCompactCap = 2048;   // candidates the final warp of a query keeps (64 per lane)
+constexpr int kSegCap = 256;        // candidates one segment may hand on
+
+// One warp per (query, segment of kSelectSeg scores): the scores that reach
+// the query's threshold key, in id order, into the segment's kSegCap slots of
+// cand_k/cand_i [q][nseg * kSegCap]; their number (even past kSegCap) into
+// seg_n[q][nseg].  Lane l reads the segment's 64 scores l*64 .. l*64+63 with
+// 16-byte loads, all issued before any is used.
+__global__ void __launch_bounds__(kSelectWarps * 32) k_compact_seg(
+    const float *__restrict__ scores, int64_t ld, int64_t nq, int64_t nlist, int nseg,
+    const uint32_t *__restrict__ lkey, uint32_t *__restrict__ cand_k, int32_t *__restrict__ cand_i,
+    int *__restrict__ seg_n) {
+    constexpr int kPer = kSelectSeg / 32;   // 64 scores per lane
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t w = (int64_t)blockIdx.x * kSelectWarps + warp;
+    if (w >= nq * nseg) return;
+    const int64_t q = w / nseg;
+    const int sg = (int)(w % nseg);
+    const int64_t c0 = (int64_t)sg * kSelectSeg + lane * kPer;   // this lane's first column
+    const float *row = scores + q * ld;
+    const uint32_t L = lkey[q];
+    float4 v[kPer / 4];
+#pragma unroll
+    for (int i = 0; i < kPer / 4; ++i)   // ld is a multiple of 32: a 4-group below ld is whole
+        v[i] = c0 + 4 * i < ld ? *reinterpret_cast<const float4 *>(row + c0 + 4 * i)
+                               : make_float4(0.f, 0.f, 0.f, 0.f);
+    uint64_t hit = 0;   // bit j: column c0 + j qualifies
+#pragma unroll
+    for (int i = 0; i < kPer / 4; ++i) {
+        const float x[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const int j = 4 * i + e;
+            if (c0 + j < nlist && order_key(x[e]) >= L) hit |= 1ull << j;
+        }
+    }
+    // this lane's place among the segment's candidates: lanes hold consecutive columns
+    const int mine = __popcll(hit);
+    int x = mine;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    int p = x - mine;
+    uint32_t *ok = cand_k + (q * nseg + sg) * kSegCap;
+    int32_t *oi = cand_i + (q * nseg + sg) * kSegCap;
+    while (hit) {
+        const int j = __ffsll((long long)hit) - 1;
+        hit &= hit - 1;
+        if (p < kSegCap) {   // the rare candidate's score again (cached), not a register pick
+            ok[p] = order_key(row[c0 + j]);
+            oi[p] = (int)(c0 + j);
+        }
+        ++p;
+    }
+    if (lane == 31) seg_n[q * nseg + sg] = x;
+}
+
+// One warp per query: its segments' candidates gathered in order (id order),
+// then the nprobe best sorted into order/cscores.  A segment past kSegCap or
+// more than kCompactCap in all (many equal scores): the query is flagged in
+// ovf and left to the level-by-level selection.
+__global__ void __launch_bounds__(kSelectWarps * 32) k_compact_final(
+    const uint32_t *__restrict__ cand_k, const int32_t *__restrict__ cand_i,
+    const int *__restrict__ seg_n, int64_t nq, int nseg, int nprobe, int P,
+    int32_t *__restrict__ order, float *__restrict__ cscores, int *__restrict__ ovf) {
+    extern __shared__ __align__(16) unsigned char sel_smem[];
+    const int cap = 2 * P;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    unsigned char *wbase = sel_smem + (size_t)warp * (kCompactCap * 8 + 2 * cap * 4);
+    uint32_t *ck = reinterpret_cast<uint32_t *>(wbase);              // candidate keys
+    int *ci = reinterpret_cast<int *>(wbase + kCompactCap * 4);      // candidate ids
+    float *bs = reinterpret_cast<float *>(wbase + kCompactCap * 8);  // sort buffer
+    int *bc = reinterpret_cast<int *>(bs + cap);
+    const int64_t q = (int64_t)blockIdx.x * kSelectWarps + warp;
+    if (q >= nq) return;
+    // segment counts and their running offsets, 32 segments at a time
+    int n = 0;
+    bool over = false;
+    for (int s0 = 0; s0 < nseg; s0 += 32) {
+        const int sg = s0 + lane;
+        const int c = sg < nseg ? seg_n[q * nseg + sg] : 0;
+        over |= __any_sync(0xffffffffu, c > kSegCap);
+        int x = c;   // inclusive scan over the lanes
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, x, o);
+            if (lane >= o) x += y;
+        }
+        const int total = __shfl_sync(0xffffffffu, x, 31);
+        if (!over && n + total <= kCompactCap) {
+            // copy each segment's candidates to its place (lanes of the warp in turn)
+            for (int t = 0; t < 32 && s0 + t < nseg; ++t) {
+                const int ct = __shfl_sync(0xffffffffu, c, t);
+                const int at = n + __shfl_sync(0xffffffffu, x, t) - ct;
+                const uint32_t *sk = cand_k + (q * nseg + s0 + t) * kSegCap;
+                const int32_t *si = cand_i + (q * nseg + s0 + t) * kSegCap;
+                for (int i = lane; i < ct; i += 32) {
+                    ck[at + i] = sk[i];
+                    ci[at + i] = si[i];
+                }
+            }
+        }
+        n += total;
+        over |= n > kCompactCap;
+    }
+    if (over) {
+        if (lane == 0) ovf[q] = 1;
+        return;
+    }
+    if (lane == 0) ovf[q] = 0;
+    __syncwarp();
+    uint32_t key[kCompactCap / 32];
+#pragma unroll
+    for (int j = 0; j < kCompactCap / 32; ++j) {
+        const int c = j * 32 + lane;
+        key[j] = c < n ? ck[c] : 0u;
+    }
+    const int want = nprobe;   // n >= nprobe: the threshold is reached by at least nprobe scores
+    uint32_t T;
+    int C;
+    warp_threshold(key, want, cap, T, C);
+    warp_gather_sort(key, n, want, T, C, cap, [&](int c) { return ci[c]; }, bs, bc);
     for (int p = lane; p < nprobe; p += 32) {
         order[q * nprobe + p] = bc[p];
         if (cscores) cscores[q * nprobe + p] = bs[p];
@@ -267,34 +478,66 @@ __global__ void __launch_bounds__(kSelectWarps * 32) k_select(const float *__res
 }
 
 // ---------------------------------------------------------------------------
-bool rank_tc_supported(int64_t nlist, int nprobe) { return nlist <= kRankTcMaxNlist && nprobe <= nlist; }
+bool rank_tc_supported(int64_t nlist, int nprobe) { return nlist >= 1 && nprobe <= nlist; }
 
 int64_t rank_tc_ld(int64_t nlist) { return round_up(nlist, 32); }
 
-int64_t rank_tc_chunk(int64_t nq, int64_t nlist) {
-    const int64_t per_q = rank_tc_ld(nlist) * (int64_t)sizeof(float);
-    int64_t c = kRankScratchBytes / per_q;
+// entries each selection level leaves per query (level 0 = the score row)
+static int64_t level_entries(int64_t M, int nprobe) { return ceil_div(M, kSelectSeg) * nprobe; }
+
+// more centroids than one selecting warp holds: a threshold from the maxima
+// of 32-centroid groups when there are at least nprobe groups (and few enough
+// for one warp), then one compacting pass
+static bool use_group_threshold(int64_t nlist, int nprobe) {
+    const int64_t ng = ceil_div(nlist, 32);
+    return nlist > kSelectSeg && ng >= nprobe && ng <= kCompactCap;
+}
+
+// per query under the group threshold: the group maxima, the segments'
+// candidate slots (keys + ids) and counts, the threshold key, the overflow flag
+static int64_t group_bytes_per_query(int64_t nlist) {
+    const int64_t nseg = ceil_div(nlist, kSelectSeg);
+    return round_up(ceil_div(nlist, 32), 4) * 4 + nseg * kSegCap * 8 + round_up(nseg, 4) * 4 + 8;
+}
+
+// bytes per query: the score row; two candidate buffers (scores + ids) for
+// the levels of a selection over more than kSelectSeg centroids; the group
+// threshold's buffers
+static int64_t rank_bytes_per_query(int64_t nlist, int nprobe) {
+    int64_t b = rank_tc_ld(nlist) * (int64_t)sizeof(float);
+    if (nlist > kSelectSeg) b += 2 * round_up(level_entries(nlist, nprobe), 4) * 8;
+    if (use_group_threshold(nlist, nprobe)) b += group_bytes_per_query(nlist);
+    return b;
+}
+
+int64_t rank_tc_chunk(int64_t nq, int64_t nlist, int nprobe) {
+    int64_t c = kRankScratchBytes / rank_bytes_per_query(nlist, nprobe);
     c = c / tcp::kM * tcp::kM;
     if (c < tcp::kM) c = tcp::kM;
     return nq < c ? nq : c;
 }
 
-size_t rank_tc_scratch_bytes(int64_t nq, int64_t nlist) {
-    return (size_t)(rank_tc_chunk(nq, nlist) * rank_tc_ld(nlist) * (int64_t)sizeof(float));
+size_t rank_tc_scratch_bytes(int64_t nq, int64_t nlist, int nprobe) {
+    return (size_t)(rank_tc_chunk(nq, nlist, nprobe) * rank_bytes_per_query(nlist, nprobe));
 }
 
 static size_t tc_smem() { return tcp::Geometry<RankMode::kN>::smem_bytes(0); }
 
-static int pow2_at_least(int x) {
+static int pow2_at_least(int64_t x) {
     int p = 1;
     while (p < x) p <<= 1;
     return p;
 }
 
+static size_t select_smem(int P) { return (size_t)kSelectWarps * 2 * (2 * P) * 4; }
+static size_t compact_smem(int P) {
+    return (size_t)kSelectWarps * ((size_t)kCompactCap * 8 + 2 * (2 * P) * 4);
+}
+
 template <int KPL>
 static cudaError_t set_select_attr(int P) {
     return cudaFuncSetAttribute(k_select<KPL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                kSelectWarps * 2 * (2 * P) * 4);
+                                (int)select_smem(P));
 }
 
 cudaError_t prepare_rank_tc(int nprobe, int d) {
@@ -312,7 +555,36 @@ cudaError_t prepare_rank_tc(int nprobe, int d) {
     if (e == cudaSuccess) e = set_select_attr<16>(P);
     if (e == cudaSuccess) e = set_select_attr<32>(P);
     if (e == cudaSuccess) e = set_select_attr<64>(P);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_compact_final, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)compact_smem(P));
     return e;
+}
+
+// one selection level: the best nprobe of every segment of at most kSelectSeg
+// entries (nseg = 1: the final order)
+static void launch_select(const float *in_s, const int32_t *in_id, int64_t in_ld, int64_t nq,
+                          int64_t M, int nprobe, int32_t *out_id, float *out_s, int64_t out_ld,
+                          const int *only, cudaStream_t st) {
+    const int seg = M < kSelectSeg ? (int)M : kSelectSeg;
+    const int nseg = (int)ceil_div(M, kSelectSeg);
+    const int P = pow2_at_least(nprobe);
+    const unsigned blocks = (unsigned)ceil_div(nq * nseg, kSelectWarps);
+    const size_t smem = select_smem(P);
+    const int kpl = pow2_at_least(ceil_div(seg, 32));
+#define SIEVE_SELECT(K)                                                                            \
+    k_select<K><<<blocks, kSelectWarps * 32, smem, st>>>(in_s, in_id, in_ld, nq, M, seg, nseg,     \
+                                                        nprobe, P, out_id, out_s, out_ld, only)
+    switch (kpl) {
+        case 1: SIEVE_SELECT(1); break;
+        case 2: SIEVE_SELECT(2); break;
+        case 4: SIEVE_SELECT(4); break;
+        case 8: SIEVE_SELECT(8); break;
+        case 16: SIEVE_SELECT(16); break;
+        case 32: SIEVE_SELECT(32); break;
+        default: SIEVE_SELECT(64); break;
+    }
+#undef SIEVE_SELECT
 }
 
 cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t nlist, int d,
@@ -320,31 +592,74 @@ cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t 
                             cudaStream_t st, const unsigned char *tc_cent) {
     const int bulk_stages = tc_cent ? rank_bulk_stages(d) : 0;
     const int64_t ld = rank_tc_ld(nlist);
-    const int64_t chunk = rank_tc_chunk(nq, nlist);
+    const int64_t chunk = rank_tc_chunk(nq, nlist, nprobe);
+    // after the chunk's score table: two candidate buffers [chunk][lvl_ld]
+    // (scores, then ids) when nlist > kSelectSeg; then the group maxima
+    // [chunk][gld], threshold keys [chunk] and overflow flags [chunk]
+    const int64_t lvl_ld = nlist > kSelectSeg ? round_up(level_entries(nlist, nprobe), 4) : 0;
+    float *cand_s[2] = {scratch + chunk * ld, scratch + chunk * ld + 2 * chunk * lvl_ld};
+    int32_t *cand_id[2] = {reinterpret_cast<int32_t *>(cand_s[0] + chunk * lvl_ld),
+                           reinterpret_cast<int32_t *>(cand_s[1] + chunk * lvl_ld)};
+    const bool grouped = use_group_threshold(nlist, nprobe);
+    const int ng = (int)ceil_div(nlist, 32);
+    const int64_t gld = round_up(ng, 4);
+    const int nseg = (int)ceil_div(nlist, kSelectSeg);
+    float *gmax = scratch + chunk * ld + 4 * chunk * lvl_ld;
+    uint32_t *seg_k = reinterpret_cast<uint32_t *>(gmax + chunk * gld);
+    int32_t *seg_i = reinterpret_cast<int32_t *>(seg_k + chunk * nseg * kSegCap);
+    int *seg_n = seg_i + chunk * nseg * kSegCap;
+    uint32_t *lkey = reinterpret_cast<uint32_t *>(seg_n + chunk * round_up(nseg, 4));
+    int *ovf = reinterpret_cast<int *>(lkey + chunk);
     const int P = pow2_at_least(nprobe);
-    const int kpl = pow2_at_least((int)ceil_div(nlist, 32));
     for (int64_t q0 = 0; q0 < nq; q0 += chunk) {
         const int64_t n = nq - q0 < chunk ? nq - q0 : chunk;
-        RankArgs a{Q + q0 * d, n, C, nlist, d, scratch, ld, status, tc_cent};
-        const int tiles = (int)ceil_div(n, tcp::kM);
+        RankArgs a{Q + q0 * d, n, C, nlist, d, scratch, ld, status, tc_cent,
+                   grouped ? gmax : nullptr, gld};
+        const int tiles = (int)(ceil_div(n, tcp::kM) * ceil_div(nlist, kRankRange));
         if (bulk_stages)
             k_rank_bulk<<<std::min(tiles, num_sms()), tcb::kThreads,
                           tcb::smem_bytes(bulk_stages, 0), st>>>(a, bulk_stages);
         else
             k_rank_tc<<<std::min(tiles, num_sms()), tcp::kThreads, tc_smem(), st>>>(a);
-        const unsigned blocks = (unsigned)ceil_div(n, kSelectWarps);
-        const size_t smem = (size_t)kSelectWarps * 2 * (2 * P) * 4;
         int32_t *o = order + q0 * nprobe;
         float *cs = cscores ? cscores + q0 * nprobe : nullptr;
-        switch (kpl) {
-            case 1: k_select<1><<<blocks, kSelectWarps * 32, smem, st>>>(scratch, ld, n, (int)nlist, nprobe, P, o, cs); break;
-            case 2: k_select<2><<<blocks, kSelectWarps * 32, smem, st>>>(scratch, ld, n, (int)nlist, nprobe, P, o, cs); break;
-            case 4: k_select<4><<<blocks, kSelectWarps * 32, smem, st>>>(scratch, ld, n, (int)nlist, nprobe, P, o, cs); break;
-            case 8: k_select<8><<<blocks, kSelectWarps * 32, smem, st>>>(scratch, ld, n, (int)nlist, nprobe, P, o, cs); break;
-            case 16: k_select<16><<<blocks, kSelectWarps * 32, smem, st>>>(scratch, ld, n, (int)nlist, nprobe, P, o, cs); break;
-            case 32: k_select<32><<<blocks, kSelectWarps * 32, smem, st>>>(scratch, ld, n, (int)nlist, nprobe, P, o, cs); break;
-            default: k_select<64><<<blocks, kSelectWarps * 32, smem, st>>>(scratch, ld, n, (int)nlist, nprobe, P, o, cs); break;
+        const int *only = nullptr;
+        if (grouped) {
+            const unsigned wblocks = (unsigned)ceil_div(n, kSelectWarps);
+            const int kpl = pow2_at_least(ceil_div(ng, 32));
+#define SIEVE_GTHR(K)                                                                              \
+    k_group_threshold<K><<<wblocks, kSelectWarps * 32, 0, st>>>(gmax, gld, n, ng, nprobe, lkey)
+            switch (kpl) {
+                case 1: SIEVE_GTHR(1); break;
+                case 2: SIEVE_GTHR(2); break;
+                case 4: SIEVE_GTHR(4); break;
+                case 8: SIEVE_GTHR(8); break;
+                case 16: SIEVE_GTHR(16); break;
+                case 32: SIEVE_GTHR(32); break;
+                default: SIEVE_GTHR(64); break;
+            }
+#undef SIEVE_GTHR
+            k_compact_seg<<<(unsigned)ceil_div(n * nseg, kSelectWarps), kSelectWarps * 32, 0, st>>>(
+                scratch, ld, n, nlist, nseg, lkey, seg_k, seg_i, seg_n);
+            k_compact_final<<<wblocks, kSelectWarps * 32, compact_smem(P), st>>>(
+                seg_k, seg_i, seg_n, n, nseg, nprobe, P, o, cs, ovf);
+            only = ovf;   // the levels below run only for overflowing queries
         }
+        // levels: the score row, then candidates, until one segment is left
+        const float *in_s = scratch;
+        const int32_t *in_id = nullptr;
+        int64_t in_ld = ld, M = nlist;
+        int buf = 0;
+        while (M > kSelectSeg) {
+            launch_select(in_s, in_id, in_ld, n, M, nprobe, cand_id[buf], cand_s[buf], lvl_ld, only,
+                          st);
+            in_s = cand_s[buf];
+            in_id = cand_id[buf];
+            in_ld = lvl_ld;
+            M = level_entries(M, nprobe);
+            buf ^= 1;
+        }
+        launch_select(in_s, in_id, in_ld, n, M, nprobe, o, cs, nprobe, only, st);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }

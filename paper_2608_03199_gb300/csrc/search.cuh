@@ -83,13 +83,11 @@ cudaError_t prepare_rank(int nprobe);
 cudaError_t enqueue_rank(const float *Q, int64_t nq, const float *C, int64_t nlist, int d,
                          int nprobe, int32_t *order, float *cscores, cudaStream_t st);
 
-// centroid ranking on the tensor cores (rank_tc.cu) for nlist <= kRankTcMaxNlist:
-// a score table of at most kRankScratchBytes per chunk of queries, then a
-// warp-per-query selection
-constexpr int64_t kRankTcMaxNlist = 2048;
-constexpr int64_t kRankScratchBytes = int64_t(512) << 20;
+// centroid ranking on the tensor cores (rank_tc.cu): a score table of at most
+// kRankScratchBytes per chunk of queries, then warp-per-segment selections
+constexpr int64_t kRankScratchBytes = int64_t(2) << 30;
 bool rank_tc_supported(int64_t nlist, int nprobe);
-size_t rank_tc_scratch_bytes(int64_t nq, int64_t nlist);
+size_t rank_tc_scratch_bytes(int64_t nq, int64_t nlist, int nprobe);
 cudaError_t prepare_rank_tc(int nprobe, int d);
 cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t nlist, int d,
                             int nprobe, int32_t *order, float *cscores, float *scratch, int *status,

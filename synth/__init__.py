@@ -74,9 +74,11 @@ CONFIGS = {
     "1m": Workload("1m", 1_000_000, 256, 1024, 1.1, 0.03, ("powerlaw", 2.0, 1000), (0.01, 0.05),
                    1024, 100_000, 0.90, 10, 64, 8, train_cap=256 * 1024, seed=2,
                    sweep_W=(2, 4, 8, 16, 64)),
-    # 10M d=512, 16,384 Zipf components, heavy-tailed duplicates, nlist 16,384,
+    # 10M d=512, 16,384 Zipf components, heavy-tailed duplicates (power-law
+    # alpha 1.5 copy counts up to 1,000: about 23 copies per parent, so 0.2% of
+    # the rows as parents make about 5% of the rows copies), nlist 16,384,
     # 1M queries, tau 0.92, nprobe 128, W 8
-    "10m512": Workload("10m512", 10_000_000, 512, 16384, 1.1, 0.05, ("powerlaw", 1.5, 1000),
+    "10m512": Workload("10m512", 10_000_000, 512, 16384, 1.1, 0.002, ("powerlaw", 1.5, 1000),
                        (0.005, 0.03), 16384, 1_000_000, 0.92, 10, 128, 8,
                        train_cap=256 * 16384, seed=3),
     # 10M d=256, near-uniform density, 0.5% planted duplicates, nlist 8,192,

@@ -27,11 +27,11 @@ def dev():
     return torch.device("cuda:0")
 
 
-def gpu_index(w, dev):
+def gpu_index(w, dev, tc_layout=None):
     X = torch.from_numpy(w["X"]).to(dev)
     assign = torch.from_numpy(w["assign"]).to(dev)
     cent = torch.from_numpy(w["centroids"]).to(dev)
-    return sieve.build_layout(X, assign, cent.shape[0], cent)
+    return sieve.build_layout(X, assign, cent.shape[0], cent, tc_layout=tc_layout)
 
 
 @pytest.fixture(scope="module")
@@ -88,7 +88,7 @@ def test_rank_parity(tiny, g_tiny, dev):
         assert bad.sum() <= 2
 
 
-@pytest.mark.parametrize("nlist", [1, 33, 64, 100, 1000, 2048])
+@pytest.mark.parametrize("nlist", [1, 33, 64, 100, 1000, 2048, 2049, 4100, 9000])
 def test_rank_selection_exact_ties(nlist, dev):
     """Scores that are exact in fp32 and fp64 (multiples of 1/64 from
     coordinates in {-2..2}/8), so equal scores tie exactly: the order must be
@@ -114,6 +114,35 @@ def test_rank_selection_exact_ties(nlist, dev):
         ref = np.stack([np.lexsort((np.arange(nlist), -row))[:nprobe] for row in ref_sc])
         assert np.array_equal(order, ref), nprobe
         assert np.array_equal(sc.astype(np.float64), np.take_along_axis(ref_sc, ref, 1))
+
+
+@pytest.mark.parametrize("nlist,d,nprobe", [(5000, 96, 256), (2500, 36, 100), (16384, 64, 128),
+                                             (9000, 96, 200), (65536, 32, 256)])
+def test_rank_parity_many_centroids(nlist, d, nprobe, dev):
+    """Rankings over more centroids than one selecting warp holds, with d not
+    a multiple of the 64-element K-block, against the fp64 oracle ranking;
+    rank swaps only across score gaps below the tolerance.  Fewer 32-centroid
+    groups than nprobe take the level-by-level selection, the others the
+    group-maximum threshold and one compacting pass."""
+    rng = np.random.default_rng(nlist + d)
+    C = rng.standard_normal((nlist, d)).astype(np.float32)
+    C /= np.linalg.norm(C, axis=1, keepdims=True)
+    Q = (C[rng.integers(0, nlist, 700)] + 0.3 * rng.standard_normal((700, d))).astype(np.float32)
+    Q /= np.linalg.norm(Q, axis=1, keepdims=True)
+    Cd = torch.from_numpy(C).to(dev)
+    index = sieve.build_layout(Cd.clone(), torch.arange(nlist, dtype=torch.int32, device=dev),
+                               nlist, Cd)
+    order, sc = sieve.rank_partitions(index, torch.from_numpy(Q).to(dev), nprobe, return_scores=True)
+    order, sc = order.cpu().numpy(), sc.cpu().numpy()
+    ref, rsc = oracle.rank(Q, C, nprobe + 1, return_scores=True)
+    assert np.abs(sc - rsc[:, :nprobe]).max() <= TOL
+    gaps = (rsc[:, :-1] - rsc[:, 1:]).min(axis=1)
+    bad = (order != ref[:, :nprobe]).any(axis=1)
+    assert (gaps[bad] < TOL).all()
+    assert bad.sum() <= 0.02 * len(Q)
+    # every row is a permutation prefix: distinct ids in range
+    assert ((order >= 0) & (order < nlist)).all()
+    assert all(len(set(r)) == nprobe for r in order[:50])
 
 
 @pytest.mark.parametrize("lookahead", [0, 1])
@@ -385,7 +414,8 @@ def test_wide_rows_fall_back_and_match(dev):
                        dup_counts=("uniform", 1, 4), dup_sigma=(0.005, 0.02), tau=0.9,
                        nprobe=8, W=2, seed=21)
     w = synth.to_numpy(synth.make_workload(cfg))
-    gidx = gpu_index(w, dev)
+    assert gpu_index(w, dev).tc_rows is None   # not built by default past d = 256
+    gidx = gpu_index(w, dev, tc_layout=True)
     assert gidx.tc_rows is not None
     for path in ("tensor", "auto"):
         check(w, gidx, w["Q"], w["qids"], cfg.tau, cfg.k, cfg.nprobe, cfg.W, 1, scan_path=path)
