@@ -166,10 +166,12 @@ def committed_traffic(kernel, workload, launches):
     return e["dram_bytes_per_search"] / max(1, launches)
 
 
-def roofline(prof, cfg, dev, bulk=True):
+def roofline(prof, cfg, dev, bulk=True, rank_on_tensor=True):
     """Roofline entry for the kernel with the largest share of the step.
     bulk: the index carries the tensor-core layout, so the tensor-core scan
-    runs as k_scan_bulk (else k_scan_tc)."""
+    runs as k_scan_bulk (else k_scan_tc) and the ranking as k_rank_bulk;
+    rank_on_tensor: the ranking runs on the tensor cores (every scan path
+    but the FP32 one)."""
     km, kl = prof["kernel_ms"], prof["kernel_launches"]
     top = max(km, key=lambda k: km[k])
     props = torch.cuda.get_device_properties(dev)
@@ -204,6 +206,18 @@ def roofline(prof, cfg, dev, bulk=True):
                                f"x {clock_mhz:.0f} MHz (measured max clock)",
                    hbm_view={"achieved_gbs": bytes_ / launches / (ms_per_launch * 1e-3) / 1e9,
                              "peak_gbs": hbm})
+    elif top == "rank" and rank_on_tensor:
+        # the score contraction of the ranking (tensor cores, three fp16
+        # products per score) plus its selection kernels, timed together
+        name = "k_rank_bulk" if bulk else "k_rank_tc"
+        flops = 2.0 * cfg.nq * cfg.nlist * d
+        ach = flops / (ms_per_launch * 1e-3) / 1e12
+        out.update(kernel=name, bound="tensor", achieved=ach, peak=f16_tflops / 3,
+                   unit="TFLOP/s", frac=ach / (f16_tflops / 3),
+                   peak_source=(f"fp16 split: three kind::f16 MMAs per score; fp16 dense peak "
+                                f"{f16_tflops:.0f} TFLOP/s = measured bf16 cuBLAS burst (of "
+                                f"measured), a third of it; the time includes the selection"),
+                   tensor_pipe_tflops=3 * ach)
     elif top == "rank":
         flops = 2.0 * cfg.nq * cfg.nlist * d
         ach = flops / (ms_per_launch * 1e-3) / 1e12
@@ -411,7 +425,8 @@ def run_sieve(args, cfg, world, rank, local):
         "speedup_vs_fixed": ms_fixed / ms,
         "mean_probes": mean_probes,
         "queries_with_results": hit_frac,
-        "roofline": roofline(prof, cfg, dev, bulk=index.tc_rows is not None),
+        "roofline": roofline(prof, cfg, dev, bulk=index.tc_rows is not None,
+                             rank_on_tensor=args.scan_path != "simt"),
         "profile": {"kernel_ms": prof["kernel_ms"], "kernel_launches": prof["kernel_launches"],
                     "rounds": prof["rounds"], "items": prof["items"], "groups": prof["groups"],
                     "mean_group": prof["items"] / max(1, prof["groups"]),
