@@ -72,7 +72,6 @@ struct RankMode {
     __device__ static const unsigned char *b_block(const Args &a, const Tile &T, int ch) {
         return a.tc_cent + (T.c0 / kTcRows + ch) * (int64_t)((a.d + 63) / 64) * kTcBlockBytes;
     }
-    static constexpr bool kStage = false;
     struct Epi {
         float *row;
         float *grow;   // this query's group maxima from the range start, or nullptr
@@ -97,8 +96,6 @@ struct RankMode {
             }
         }
         __device__ void end(const Args &, const Tile &) {}
-        __device__ void stage(const Args &, const Tile &, int64_t, int) {}
-        __device__ void use_staged(int) {}
     };
 };
 static_assert(kRankRange % RankMode::kN == 0 && kRankRange % kTcRows == 0, "");
@@ -130,6 +127,7 @@ __device__ __forceinline__ float key_score(uint32_t k) {
 
 constexpr int kSelectWarps = 4;
 constexpr int kSelectMaxR = 4;   // lane order statistics used for the lower bracket
+constexpr int kSelectSmallC = 4; // candidate keys per lane of the two-step selection (P <= 64)
 
 __device__ __forceinline__ int warp_sum(int x) {
 #pragma unroll
@@ -313,8 +311,49 @@ __global__ void __launch_bounds__(kSelectWarps * 32) k_select(
     uint32_t T;
     int C;
     warp_threshold(key, want, cap, T, C);
-    warp_gather_sort(key, cnt, want, T, C, cap,
-                     [&](int c) { return rid ? rid[c] : (int)(p0 + c); }, bs, bc);
+    if (C <= cap && cap <= 32 * kSelectSmallC) {
+        // two steps: the C candidates (key >= T) go to shared memory in id
+        // order, come back as kSelectSmallC keys per lane, and a second, cheap
+        // threshold over them leaves exactly want entries to sort
+        const unsigned below = (1u << lane) - 1u;
+        uint32_t *ck = reinterpret_cast<uint32_t *>(bs);
+        int pos = 0;
+#pragma unroll
+        for (int j = 0; j < KPL; ++j) {
+            const int c = j * 32 + lane;
+            const bool sel = key[j] >= T && c < cnt;
+            const unsigned sb = __ballot_sync(0xffffffffu, sel);
+            if (sel) {
+                const int p = pos + __popc(sb & below);
+                ck[p] = key[j];
+                bc[p] = rid ? rid[c] : (int)(p0 + c);
+            }
+            pos += __popc(sb);
+        }
+        __syncwarp();
+        uint32_t k2[kSelectSmallC];
+        int i2[kSelectSmallC];
+#pragma unroll
+        for (int j = 0; j < kSelectSmallC; ++j) {
+            const int c = j * 32 + lane;
+            k2[j] = c < pos ? ck[c] : 0u;
+            i2[j] = c < pos ? bc[c] : 0;
+        }
+        __syncwarp();
+        uint32_t T2;
+        int C2;
+        warp_threshold(k2, want, want, T2, C2);
+        warp_gather_sort(k2, pos, want, T2, C2, want, [&](int c) {
+            // id of candidate c: held by lane c % 32 in slot c / 32 (c is this lane's)
+            int id = i2[0];
+#pragma unroll
+            for (int j = 1; j < kSelectSmallC; ++j) id = (c >> 5) == j ? i2[j] : id;
+            return id;
+        }, bs, bc);
+    } else {
+        warp_gather_sort(key, cnt, want, T, C, cap,
+                         [&](int c) { return rid ? rid[c] : (int)(p0 + c); }, bs, bc);
+    }
     int32_t *oi = out_id + q * out_ld + (int64_t)sg * nprobe;
     float *os = out_s ? out_s + q * out_ld + (int64_t)sg * nprobe : nullptr;
     for (int p = lane; p < nprobe; p += 32) {

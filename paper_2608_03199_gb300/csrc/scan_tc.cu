@@ -61,18 +61,17 @@ struct ScanMode {
         return a.tc_rows + (a.tc_row_blocks[T.p] + ch) * (int64_t)tc_nkb_dev(a.d) * kTcBlockBytes;
     }
 
-    // the bulk pipeline stages each chunk's 128 row ids in shared memory
-    static constexpr bool kStage = true;
-    static constexpr int kStageRows = 128;
-
     struct Epi {
         float *ks;
         long long *ki;
-        long long *stage_buf;          // 2 x 128 staged row ids (bulk pipeline)
-        const long long *ids_s;        // the current chunk's staged ids, or nullptr
         int kn, item, q, rank, slot;
         bool valid;
         long long qid;
+        // the kept list is unordered while the tile runs; once it holds k
+        // entries, (wst_s, wst_id) at wst_pos is the one that ranks last
+        float wst_s;
+        long long wst_id;
+        int wst_pos;
         // entry j of thread slot's list sits at [j * kM + slot] (bank-conflict free)
         __device__ float &KS(int j) const { return ks[j * tcp::kM]; }
         __device__ long long &KI(int j) const { return ki[j * tcp::kM]; }
@@ -80,9 +79,10 @@ struct ScanMode {
             slot = slot_;
             ks = reinterpret_cast<float *>(smem) + slot;
             ki = reinterpret_cast<long long *>(reinterpret_cast<float *>(smem) + tcp::kM * a.k) + slot;
-            stage_buf = reinterpret_cast<long long *>(smem + (size_t)tcp::kM * a.k * 12);
-            ids_s = nullptr;
             kn = 0;
+            wst_s = 0.f;
+            wst_id = 0;
+            wst_pos = 0;
             valid = slot < T.ni;
             item = q = rank = 0;
             qid = (long long)-0x7fffffffffffffffll - 1;
@@ -93,25 +93,37 @@ struct ScanMode {
                 if (a.qids) qid = a.qids[q];
             }
         }
-        __device__ void stage(const Args &a, const Tile &T, int64_t col0, int buf) {
-            const int64_t r = col0 + slot;
-            stage_buf[buf * kStageRows + slot] = r < T.nb ? a.ids[T.r_begin + r] : -1;
-        }
-        __device__ void use_staged(int buf) { ids_s = stage_buf + buf * kStageRows; }
-        // one candidate row (s >= tau): self exclusion, then the sorted insert
-        __device__ __forceinline__ void take(const Args &a, const Tile &T, int64_t col, float sc) {
-            const long long id = ids_s ? ids_s[col & (kStageRows - 1)] : a.ids[T.r_begin + col];
-            if (id == qid) return;
-            const int k = a.k;
-            if (kn == k && !ranks_before(sc, id, KS(k - 1), KI(k - 1))) return;
-            int i = kn < k ? kn++ : k - 1;
-            while (i > 0 && ranks_before(sc, id, KS(i - 1), KI(i - 1))) {
-                KS(i) = KS(i - 1);
-                KI(i) = KI(i - 1);
-                --i;
+        __device__ void find_worst(int k) {
+            wst_pos = 0;
+            wst_s = KS(0);
+            wst_id = KI(0);
+            for (int j = 1; j < k; ++j) {
+                const float s = KS(j);
+                const long long id = KI(j);
+                if (ranks_before(wst_s, wst_id, s, id)) {
+                    wst_pos = j;
+                    wst_s = s;
+                    wst_id = id;
+                }
             }
-            KS(i) = sc;
-            KI(i) = id;
+        }
+        // one candidate row (s >= tau): self exclusion, then into the kept
+        // list (appended while it has room, else in place of its last entry)
+        __device__ __forceinline__ void take(const Args &a, const Tile &T, int64_t col, float sc) {
+            const int k = a.k;
+            if (kn == k && sc < wst_s) return;   // cannot rank before the last kept entry
+            const long long id = a.ids[T.r_begin + col];
+            if (id == qid) return;
+            if (kn < k) {
+                KS(kn) = sc;
+                KI(kn) = id;
+                if (++kn == k) find_worst(k);
+                return;
+            }
+            if (!ranks_before(sc, id, wst_s, wst_id)) return;
+            KS(wst_pos) = sc;
+            KI(wst_pos) = id;
+            find_worst(k);
         }
         // v holds the chunk's raw accumulator values: similarities x 2^16
         __device__ void chunk(const Args &a, const Tile &T, int64_t col0, const float (&v)[32],
@@ -121,7 +133,7 @@ struct ScanMode {
             // kept score (equal scores go on to the id tie-break); scores
             // here are raw (x 2^16, an exact power-of-two scale)
             float thr = a.tau * 65536.f;
-            if (kn == a.k) thr = fmaxf(thr, KS(a.k - 1) * 65536.f);
+            if (kn == a.k) thr = fmaxf(thr, wst_s * 65536.f);
             // nearly every group has no candidate: one tree of maxima decides
             float mx[16];
 #pragma unroll
@@ -145,6 +157,18 @@ struct ScanMode {
         __device__ void end(const Args &a, const Tile &T) {
             if (valid) {
                 const int k = a.k;
+                for (int j = 1; j < kn; ++j) {   // the list in result order (insertion sort)
+                    const float s = KS(j);
+                    const long long id = KI(j);
+                    int i = j;
+                    while (i > 0 && ranks_before(s, id, KS(i - 1), KI(i - 1))) {
+                        KS(i) = KS(i - 1);
+                        KI(i) = KI(i - 1);
+                        --i;
+                    }
+                    KS(i) = s;
+                    KI(i) = id;
+                }
                 for (int j = 0; j < kn; ++j) {
                     a.res_s[(int64_t)item * k + j] = KS(j);
                     a.res_id[(int64_t)item * k + j] = KI(j);
@@ -165,8 +189,6 @@ struct ScanMode {
     };
 };
 
-static_assert(tcb::kN == ScanMode::kStageRows, "a staged chunk is one tensor-layout block");
-
 size_t scan_tc_smem_bytes(int k) {
     return tcp::Geometry<ScanMode::kN>::smem_bytes((size_t)tcp::kM * k * (sizeof(float) + sizeof(long long)));
 }
@@ -176,11 +198,8 @@ __global__ void __launch_bounds__(tcp::kThreads, 1) k_scan_tc(SearchArgs a) {
     tcp::run_pipeline<ScanMode>(a, smem_raw);
 }
 
-// kept lists, then the two staged id buffers
-static size_t scan_epi_bytes(int k) {
-    return (size_t)tcp::kM * k * (sizeof(float) + sizeof(long long)) +
-           2 * ScanMode::kStageRows * sizeof(long long);
-}
+// the kept lists
+static size_t scan_epi_bytes(int k) { return (size_t)tcp::kM * k * (sizeof(float) + sizeof(long long)); }
 
 int scan_bulk_stages(int d, int k) {
     return tcb::stages_for((int)ceil_div(d, 64), scan_epi_bytes(k), 232448 - 128);

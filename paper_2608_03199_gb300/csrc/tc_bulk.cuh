@@ -87,17 +87,14 @@ __device__ __forceinline__ void hand(Epi &epi, const Args &a, const Tile &T, int
 // Mode provides (in addition to what tc_pipeline.cuh asks): b_block(a, T, ch)
 // = pointer to the tensor-layout bytes of the tile's ch-th block of B rows;
 // tile_counter(a) = a zeroed global int the blocks draw tiles from (nullptr:
-// block b takes tiles b, b + gridDim.x, ...); kStage: when true, before each
-// chunk every epilogue thread calls Epi::stage(a, T, col0, buf) (its share of
-// per-column data into shared-memory buffer buf), the 128 threads meet on an
-// mbarrier, and each calls Epi::use_staged(buf).
+// block b takes tiles b, b + gridDim.x, ...).
 template <class Mode>
 __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned char *smem_raw,
                                          int stages) {
     constexpr uint32_t kIdesc = tc::idesc_f16(tcp::kM, kN);
     __shared__ __align__(8) uint64_t a_full[kMaxKb], a_empty[kMaxKb], b_full[kMaxStages],
         b_empty[kMaxStages], dfull_bar[2], dempty_bar[2], drain_bar, ring_full[kRing],
-        ring_empty[kRing], staged_bar[2];
+        ring_empty[kRing];
     __shared__ int ring_tile[kRing];
     __shared__ uint32_t tmem_slot;
     __shared__ int s_abort;
@@ -125,7 +122,6 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
         for (int b = 0; b < 2; ++b) {
             tc::mbar_init(&dfull_bar[b], 1);
             tc::mbar_init(&dempty_bar[b], 4 * 32);
-            tc::mbar_init(&staged_bar[b], 4 * 32);
         }
         for (int r = 0; r < kRing; ++r) {
             tc::mbar_init(&ring_full[r], 1);
@@ -302,35 +298,28 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
             epi.begin(a, T, slot, epi_smem);
             for (int ch = 0; ch < nch; ++ch, ++c) {
                 const uint32_t buf = c & 1u, dph = (c >> 1) & 1u;
-                if (Mode::kStage) {   // per-column data of the chunk, shared by the 128 rows
-                    epi.stage(a, T, (int64_t)ch * kN, (int)buf);
-                    tc::mbar_arrive(&staged_bar[buf]);
-                    ok = __all_sync(0xffffffffu, wait(&staged_bar[buf], dph));
-                    if (!ok) break;
-                    epi.use_staged((int)buf);
-                }
                 ok = __all_sync(0xffffffffu, wait(&dfull_bar[buf], dph));
                 if (!ok) break;
                 tc::fence_after_sync();
-                // four 32-column loads, each issued before the previous group is
-                // handed to the mode; the accumulator is released as soon as
-                // the last load has landed
+                // two pairs of 32-column loads, each pair in flight together;
+                // the accumulator is released as soon as the second pair has
+                // landed, before its columns are handed to the mode
                 const uint32_t taddr = tmem + ((uint32_t)(quarter * 32) << 16) + buf * kN;
                 const int64_t col0 = (int64_t)ch * kN;
                 uint32_t ra[32], rb[32];
                 tc::tmem_ld32_issue(taddr, ra);
-                tc::tmem_ld_wait(ra);
                 tc::tmem_ld32_issue(taddr + 32, rb);
-                hand(epi, a, T, col0, ra);
-                tc::tmem_ld_wait(rb);
-                tc::tmem_ld32_issue(taddr + 64, ra);
-                hand(epi, a, T, col0 + 32, rb);
                 tc::tmem_ld_wait(ra);
+                tc::tmem_ld_wait(rb);
+                hand(epi, a, T, col0, ra);
+                hand(epi, a, T, col0 + 32, rb);
+                tc::tmem_ld32_issue(taddr + 64, ra);
                 tc::tmem_ld32_issue(taddr + 96, rb);
-                hand(epi, a, T, col0 + 64, ra);
+                tc::tmem_ld_wait(ra);
                 tc::tmem_ld_wait(rb);
                 tc::fence_before_sync();
                 tc::mbar_arrive(&dempty_bar[buf]);
+                hand(epi, a, T, col0 + 64, ra);
                 hand(epi, a, T, col0 + 96, rb);
             }
             if (!ok) break;
