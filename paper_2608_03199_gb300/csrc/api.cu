@@ -403,7 +403,8 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
         for (int i = 0; i < SIEVE_NKERNELS; ++i) stats->kernel_ms[i] = ms[i];
         const int per_round[] = {SIEVE_K_ISSUE, SIEVE_K_BUCKET, SIEVE_K_SCATTER, SIEVE_K_SCAN,
                                  SIEVE_K_MERGE, SIEVE_K_ROUND_END};
-        stats->kernel_launches[SIEVE_K_RANK] = with_rank ? 1 : 0;
+        stats->kernel_launches[SIEVE_K_RANK] =
+            !with_rank ? 0 : rank_tc ? rank_tc_launches(a.nq, a.nlist, a.nprobe) : 1;
         stats->kernel_launches[SIEVE_K_INIT] = 1;
         stats->kernel_launches[SIEVE_K_FINALIZE] = 1;
         for (int slot : per_round) stats->kernel_launches[slot] = c.round;

@@ -626,6 +626,14 @@ static void launch_select(const float *in_s, const int32_t *in_id, int64_t in_ld
 #undef SIEVE_SELECT
 }
 
+int rank_tc_launches(int64_t nq, int64_t nlist, int nprobe) {
+    if (nq <= 0) return 0;
+    int per = 2;                                           // contraction + final selection
+    if (use_group_threshold(nlist, nprobe)) per += 3;      // threshold, compaction, gather
+    for (int64_t M = nlist; M > kSelectSeg; M = level_entries(M, nprobe)) ++per;
+    return (int)ceil_div(nq, rank_tc_chunk(nq, nlist, nprobe)) * per;
+}
+
 cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t nlist, int d,
                             int nprobe, int32_t *order, float *cscores, float *scratch, int *status,
                             cudaStream_t st, const unsigned char *tc_cent) {

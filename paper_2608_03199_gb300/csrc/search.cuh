@@ -88,6 +88,7 @@ cudaError_t enqueue_rank(const float *Q, int64_t nq, const float *C, int64_t nli
 constexpr int64_t kRankScratchBytes = int64_t(2) << 30;
 bool rank_tc_supported(int64_t nlist, int nprobe);
 size_t rank_tc_scratch_bytes(int64_t nq, int64_t nlist, int nprobe);
+int rank_tc_launches(int64_t nq, int64_t nlist, int nprobe);   // kernel launches of one ranking
 cudaError_t prepare_rank_tc(int nprobe, int d);
 cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t nlist, int d,
                             int nprobe, int32_t *order, float *cscores, float *scratch, int *status,

@@ -4,7 +4,7 @@
 // fp16 split of tc_pipeline.cuh and the same per-row epilogues.
 //
 // The B operand arrives pre-split, in tile byte order: one 32 KB bulk copy per
-// (block, K-block) lands a stage (hi then lo) in shared memory, up to six
+// (block, K-block) lands a stage (hi then lo) in shared memory, up to five
 // stages deep, with no thread touching the bytes.  The tile's 128 A rows are
 // split once per tile straight into tensor memory (lane i = A row i, two fp16
 // per 32-bit column, hi and lo of each K-block side by side), so shared memory
@@ -50,7 +50,7 @@ constexpr int kProducerWarp = 8;
 constexpr int kMmaWarp = 9;
 constexpr int kThreads = 14 * 32;
 constexpr int kMaxKb = 4;                     // A in tensor memory: d <= 256
-constexpr int kMaxStages = 6;
+constexpr int kMaxStages = 5;                 // timed faster than six: more of the SM memory stays L1
 constexpr uint32_t kKbBytes = 32768;          // one K-block of 128 rows: hi 16 KB + lo 16 KB
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kAColumn0 = 2 * kN;        // A after the two accumulators
