@@ -121,7 +121,7 @@ Layout make_layout(const sieve_index_view *ix, int64_t nq, const sieve_params *p
     L.res_s = take((size_t)cap * p->k * 4);
     L.res_id = take((size_t)cap * p->k * 8);
     L.rank_scratch = (p->scan_path != 1 && rank_tc_supported(ix->nlist, p->nprobe))
-                         ? take(rank_tc_scratch_bytes(nq, ix->nlist, p->nprobe))
+                         ? take(rank_tc_scratch_bytes(nq, ix->nlist, p->nprobe, ix->d))
                          : 0;
     if (host_io) {
         L.h_Q = take((size_t)nq * ix->d * 4);
@@ -404,7 +404,7 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
         const int per_round[] = {SIEVE_K_ISSUE, SIEVE_K_BUCKET, SIEVE_K_SCATTER, SIEVE_K_SCAN,
                                  SIEVE_K_MERGE, SIEVE_K_ROUND_END};
         stats->kernel_launches[SIEVE_K_RANK] =
-            !with_rank ? 0 : rank_tc ? rank_tc_launches(a.nq, a.nlist, a.nprobe) : 1;
+            !with_rank ? 0 : rank_tc ? rank_tc_launches(a.nq, a.nlist, a.nprobe, a.d) : 1;
         stats->kernel_launches[SIEVE_K_INIT] = 1;
         stats->kernel_launches[SIEVE_K_FINALIZE] = 1;
         for (int slot : per_round) stats->kernel_launches[slot] = c.round;
@@ -513,7 +513,7 @@ sieve_status sieve_rank_workspace_size(const sieve_index_view *ix, int64_t nq, i
     sieve_status rc = check_index(ix, true);
     if (rc != SIEVE_OK) return rc;
     if (nprobe < 1 || nprobe > kMaxNprobe || nprobe > ix->nlist || nq < 0) return SIEVE_EINVAL;
-    *bytes = rank_tc_supported(ix->nlist, nprobe) && nq > 0 ? rank_tc_scratch_bytes(nq, ix->nlist, nprobe) : 0;
+    *bytes = rank_tc_supported(ix->nlist, nprobe) && nq > 0 ? rank_tc_scratch_bytes(nq, ix->nlist, nprobe, ix->d) : 0;
     return SIEVE_OK;
 }
 
@@ -529,7 +529,7 @@ sieve_status sieve_rank_partitions(const sieve_index_view *ix, const float *Q, i
     if (nq == 0) return SIEVE_OK;
     if (rank_tc_supported(ix->nlist, nprobe)) {
         if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) ||
-            ws_bytes < rank_tc_scratch_bytes(nq, ix->nlist, nprobe))
+            ws_bytes < rank_tc_scratch_bytes(nq, ix->nlist, nprobe, ix->d))
             return SIEVE_EWORKSPACE;
         SIEVE_CUDA(prepare_rank_tc(nprobe, ix->d));
         SIEVE_CUDA(enqueue_rank_tc(Q, nq, ix->centroids, ix->nlist, ix->d, nprobe, order, cscores,

@@ -23,6 +23,19 @@ namespace sieve {
 constexpr int64_t kRankRange = 2048;   // centroids per tile (a multiple of 128)
 constexpr int kSelectSeg = 2048;       // entries per selecting warp (64 per lane)
 
+// selection: monotone map of fp32 to uint32 (larger float -> larger key); -0
+// is mapped as +0 so that equal scores have equal keys
+__device__ __forceinline__ uint32_t order_key(float s) {
+    const uint32_t u = __float_as_uint(s + 0.f);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+// the inverse of order_key
+__device__ __forceinline__ float key_score(uint32_t k) {
+    return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
+}
+
+
 struct RankArgs {
     const float *Q;
     int64_t nq;
@@ -35,7 +48,17 @@ struct RankArgs {
     const unsigned char *tc_cent;   // tensor-core layout of the centroids (bulk path)
     float *gmax;     // nullable: [nq][gld] maxima of each 32-centroid group
     int64_t gld;
+    int mode;                // kRankTable, kRankMax or kRankKeep
+    const uint32_t *lkey;    // kRankKeep: [nq] threshold keys
+    float *keep_s;           // kRankKeep: [nq][nranges][kRankRange] kept scores, per range
+    int32_t *keep_i;         //            and their centroid ids, in id order
+    int *keep_n;             //            [nq][nranges] how many each range kept
 };
+
+// what the ranking contraction's epilogue does with a query's scores:
+// store them all (and the group maxima when gmax is set), only the maxima of
+// each 32-centroid group, or only the scores that reach the query's threshold
+constexpr int kRankTable = 0, kRankMax = 1, kRankKeep = 2;
 
 __device__ int g_rank_status_sink;
 
@@ -73,29 +96,71 @@ struct RankMode {
         return a.tc_cent + (T.c0 / kTcRows + ch) * (int64_t)((a.d + 63) / 64) * kTcBlockBytes;
     }
     struct Epi {
-        float *row;
-        float *grow;   // this query's group maxima from the range start, or nullptr
+        bool valid;
+        float *row;      // kRankTable: this query's table row from the range start
+        float *grow;     // this query's group maxima from the range start, or nullptr
+        float *ks;       // kRankKeep: this query's kept scores / ids for the range
+        int32_t *ki;
+        int kn;
+        int64_t keep_at; // kRankKeep: index of this (query, range) in keep_n
+        float thr_raw;   // kRankKeep: the threshold score x 2^16
         __device__ void begin(const Args &a, const Tile &T, int slot, unsigned char *) {
-            row = slot < T.ni ? a.scores + (T.q0 + slot) * a.ld + T.c0 : nullptr;
-            grow = (slot < T.ni && a.gmax) ? a.gmax + (T.q0 + slot) * a.gld + T.c0 / 32 : nullptr;
+            valid = slot < T.ni;
+            const int64_t q = T.q0 + slot;
+            row = (valid && a.mode == kRankTable) ? a.scores + q * a.ld + T.c0 : nullptr;
+            grow = (valid && a.gmax) ? a.gmax + q * a.gld + T.c0 / 32 : nullptr;
+            kn = 0;
+            ks = nullptr;
+            ki = nullptr;
+            thr_raw = 0.f;
+            keep_at = 0;
+            if (valid && a.mode == kRankKeep) {
+                keep_at = q * n_ranges(a) + T.c0 / kRankRange;
+                ks = a.keep_s + keep_at * kRankRange;
+                ki = a.keep_i + keep_at * kRankRange;
+                thr_raw = key_score(a.lkey[q]) * 65536.f;   // exact: a power-of-two scale
+            }
         }
         // v holds the chunk's raw accumulator values: scores x 2^16
-        __device__ void chunk(const Args &a, const Tile &, int64_t col0, const float (&v)[32], int ncol) {
-            // ld and the range start are multiples of 32: whole 32-column groups fit
-            if (!row || ncol <= 0) return;
+        __device__ void chunk(const Args &a, const Tile &T, int64_t col0, const float (&v)[32], int ncol) {
+            if (!valid || ncol <= 0) return;
             constexpr float kS = 1.f / 65536.f;
-            float4 *dst = reinterpret_cast<float4 *>(row + col0);
+            if (row) {   // ld and the range start are multiples of 32: whole groups fit
+                float4 *dst = reinterpret_cast<float4 *>(row + col0);
 #pragma unroll
-            for (int j = 0; j < 8; ++j)
-                dst[j] = make_float4(v[4 * j] * kS, v[4 * j + 1] * kS, v[4 * j + 2] * kS, v[4 * j + 3] * kS);
+                for (int j = 0; j < 8; ++j)
+                    dst[j] = make_float4(v[4 * j] * kS, v[4 * j + 1] * kS, v[4 * j + 2] * kS, v[4 * j + 3] * kS);
+            }
             if (grow) {   // the group's maximum over its real columns only
                 float mx = v[0];
 #pragma unroll
                 for (int j = 1; j < 32; ++j) mx = j < ncol ? fmaxf(mx, v[j]) : mx;
                 grow[col0 / 32] = mx * kS;
             }
+            if (ks) {   // the scores that reach the threshold, in id order
+                float mx[16];
+#pragma unroll
+                for (int j = 0; j < 16; ++j) mx[j] = fmaxf(v[j], v[j + 16]);
+#pragma unroll
+                for (int w = 8; w > 0; w >>= 1)
+#pragma unroll
+                    for (int j = 0; j < w; ++j) mx[j] = fmaxf(mx[j], mx[j + w]);
+                if (!(mx[0] >= thr_raw)) return;
+                unsigned m = 0;
+#pragma unroll
+                for (int j = 0; j < 32; ++j) m |= (v[j] >= thr_raw && j < ncol) ? (1u << j) : 0u;
+                while (m) {   // at most kRankRange per range: the slots cannot overflow
+                    const int j = __ffs(m) - 1;
+                    m &= m - 1u;
+                    ks[kn] = pick32(v, j) * kS;
+                    ki[kn] = (int32_t)(T.c0 + col0 + j);
+                    ++kn;
+                }
+            }
         }
-        __device__ void end(const Args &, const Tile &) {}
+        __device__ void end(const Args &a, const Tile &) {
+            if (ks) a.keep_n[keep_at] = kn;
+        }
     };
 };
 static_assert(kRankRange % RankMode::kN == 0 && kRankRange % kTcRows == 0, "");
@@ -112,21 +177,8 @@ __global__ void __launch_bounds__(tcb::kThreads, 1) k_rank_bulk(RankArgs a, int 
     tcb::run_bulk<RankMode>(a, smem_raw, stages);
 }
 
-// ---------------------------------------------------------------------------
-// selection: monotone map of fp32 to uint32 (larger float -> larger key); -0
-// is mapped as +0 so that equal scores have equal keys
-__device__ __forceinline__ uint32_t order_key(float s) {
-    const uint32_t u = __float_as_uint(s + 0.f);
-    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
-}
-
-// the inverse of order_key
-__device__ __forceinline__ float key_score(uint32_t k) {
-    return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
-}
-
 constexpr int kSelectWarps = 4;
-constexpr int kSelectMaxR = 4;   // lane order statistics used for the lower bracket
+constexpr int kSelectMaxR = 8;   // lane order statistics used for the lower bracket
 constexpr int kSelectSmallC = 4; // candidate keys per lane of the two-step selection (P <= 64)
 
 __device__ __forceinline__ int warp_sum(int x) {
@@ -153,14 +205,25 @@ template <int KPL>
 __device__ __forceinline__ void warp_threshold(const uint32_t (&key)[KPL], int want, int cap,
                                                uint32_t &T, int &C) {
     const int r = (want + 31) / 32;
-    uint32_t m[kSelectMaxR] = {0u, 0u, 0u, 0u};
+    uint32_t m[kSelectMaxR] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
     if (r <= 2) {
 #pragma unroll
         for (int j = 0; j < KPL; ++j) {
             m[1] = max(m[1], min(m[0], key[j]));
             m[0] = max(m[0], key[j]);
         }
-    } else {
+    } else if (r <= 4) {
+#pragma unroll
+        for (int j = 0; j < KPL; ++j) {
+            uint32_t x = key[j];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const uint32_t hi = max(m[i], x);
+                x = min(m[i], x);
+                m[i] = hi;
+            }
+        }
+    } else if (r <= kSelectMaxR) {
 #pragma unroll
         for (int j = 0; j < KPL; ++j) {
             uint32_t x = key[j];
@@ -171,9 +234,14 @@ __device__ __forceinline__ void warp_threshold(const uint32_t (&key)[KPL], int w
                 m[i] = hi;
             }
         }
+    } else {   // no lower bracket, but U is still the largest key
+#pragma unroll
+        for (int j = 0; j < KPL; ++j) m[0] = max(m[0], key[j]);
     }
     uint32_t U = m[0];
-    uint32_t L = r == 1 ? m[0] : r == 2 ? m[1] : r == 3 ? m[2] : r == 4 ? m[3] : 0u;
+    uint32_t L = 0u;   // r > kSelectMaxR: no lower bracket
+#pragma unroll
+    for (int i = 0; i < kSelectMaxR; ++i) L = r == i + 1 ? m[i] : L;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
         U = max(U, __shfl_xor_sync(0xffffffffu, U, o));
@@ -211,6 +279,8 @@ __device__ __forceinline__ void warp_gather_sort(const uint32_t (&key)[KPL], int
     const int lane = threadIdx.x & 31;
     const unsigned below = (1u << lane) - 1u;
     int pos = 0;
+    // the buffer holds cap entries: C <= cap, or exactly want <= cap taken
+    // below; the bound on p only keeps a broken invariant from writing past it
     if (C <= cap) {
 #pragma unroll
         for (int j = 0; j < KPL; ++j) {
@@ -219,8 +289,10 @@ __device__ __forceinline__ void warp_gather_sort(const uint32_t (&key)[KPL], int
             const unsigned sb = __ballot_sync(0xffffffffu, sel);
             if (sel) {
                 const int p = pos + __popc(sb & below);
-                bs[p] = key_score(key[j]);
-                bc[p] = id_of(c);
+                if (p < cap) {
+                    bs[p] = key_score(key[j]);
+                    bc[p] = id_of(c);
+                }
             }
             pos += __popc(sb);
         }
@@ -239,13 +311,16 @@ __device__ __forceinline__ void warp_gather_sort(const uint32_t (&key)[KPL], int
             const unsigned sb = __ballot_sync(0xffffffffu, sel);
             if (sel) {
                 const int p = pos + __popc(sb & below);
-                bs[p] = key_score(key[j]);
-                bc[p] = id_of(c);
+                if (p < cap) {
+                    bs[p] = key_score(key[j]);
+                    bc[p] = id_of(c);
+                }
             }
             pos += __popc(sb);
             ties_seen += __popc(tb);
         }
     }
+    if (pos > cap) pos = cap;
     int S = 1;   // sort size: a power of two >= pos (pos <= cap)
     while (S < pos) S <<= 1;
     for (int p = pos + lane; p < S; p += 32) {
@@ -281,12 +356,14 @@ __device__ __forceinline__ void warp_gather_sort(const uint32_t (&key)[KPL], int
 // want = min(nprobe, entries).  Output: the want best in order at
 // out_id/out_s[q * out_ld + s * nprobe ..], then (-inf, INT32_MAX) padding up
 // to nprobe.  `only` (nullable): queries with only[q] == 0 are skipped.
+// `seg_cnt` (nullable): [nq][nseg] entries actually present in each segment.
 // P: a power of two >= nprobe; the sort buffer holds 2P entries.
 template <int KPL>   // entries per lane: seg <= 32 * KPL
 __global__ void __launch_bounds__(kSelectWarps * 32) k_select(
     const float *__restrict__ in_s, const int32_t *__restrict__ in_id, int64_t in_ld, int64_t nq,
     int64_t M, int seg, int nseg, int nprobe, int P, int32_t *__restrict__ out_id,
-    float *__restrict__ out_s, int64_t out_ld, const int *__restrict__ only) {
+    float *__restrict__ out_s, int64_t out_ld, const int *__restrict__ only,
+    const int *__restrict__ seg_cnt) {
     extern __shared__ __align__(16) unsigned char sel_smem[];
     const int cap = 2 * P;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -298,7 +375,8 @@ __global__ void __launch_bounds__(kSelectWarps * 32) k_select(
     if (only && only[q] == 0) return;
     const int sg = (int)(w % nseg);
     const int64_t p0 = (int64_t)sg * seg;
-    const int cnt = (int)(M - p0 < seg ? M - p0 : seg);
+    int cnt = (int)(M - p0 < seg ? M - p0 : seg);
+    if (seg_cnt && seg_cnt[q * nseg + sg] < cnt) cnt = seg_cnt[q * nseg + sg];
     const int want = nprobe < cnt ? nprobe : cnt;
     const float *row = in_s + q * in_ld + p0;
     const int32_t *rid = in_id ? in_id + q * in_ld + p0 : nullptr;
@@ -325,8 +403,10 @@ __global__ void __launch_bounds__(kSelectWarps * 32) k_select(
             const unsigned sb = __ballot_sync(0xffffffffu, sel);
             if (sel) {
                 const int p = pos + __popc(sb & below);
-                ck[p] = key[j];
-                bc[p] = rid ? rid[c] : (int)(p0 + c);
+                if (p < cap) {   // pos <= C <= cap
+                    ck[p] = key[j];
+                    bc[p] = rid ? rid[c] : (int)(p0 + c);
+                }
             }
             pos += __popc(sb);
         }
@@ -391,12 +471,12 @@ constexpr int kSegCap = 256;        // candidates one segment may hand on
 
 // One warp per (query, segment of kSelectSeg scores): the scores that reach
 // the query's threshold key, in id order, into the segment's kSegCap slots of
-// cand_k/cand_i [q][nseg * kSegCap]; their number (even past kSegCap) into
+// cand_s/cand_i [q][nseg * kSegCap]; their number (even past kSegCap) into
 // seg_n[q][nseg].  Lane l reads the segment's 64 scores l*64 .. l*64+63 with
 // 16-byte loads, all issued before any is used.
 __global__ void __launch_bounds__(kSelectWarps * 32) k_compact_seg(
     const float *__restrict__ scores, int64_t ld, int64_t nq, int64_t nlist, int nseg,
-    const uint32_t *__restrict__ lkey, uint32_t *__restrict__ cand_k, int32_t *__restrict__ cand_i,
+    const uint32_t *__restrict__ lkey, float *__restrict__ cand_s, int32_t *__restrict__ cand_i,
     int *__restrict__ seg_n) {
     constexpr int kPer = kSelectSeg / 32;   // 64 scores per lane
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -431,13 +511,13 @@ __global__ void __launch_bounds__(kSelectWarps * 32) k_compact_seg(
         if (lane >= o) x += y;
     }
     int p = x - mine;
-    uint32_t *ok = cand_k + (q * nseg + sg) * kSegCap;
+    float *os = cand_s + (q * nseg + sg) * kSegCap;
     int32_t *oi = cand_i + (q * nseg + sg) * kSegCap;
     while (hit) {
         const int j = __ffsll((long long)hit) - 1;
         hit &= hit - 1;
         if (p < kSegCap) {   // the rare candidate's score again (cached), not a register pick
-            ok[p] = order_key(row[c0 + j]);
+            os[p] = row[c0 + j];
             oi[p] = (int)(c0 + j);
         }
         ++p;
@@ -445,13 +525,31 @@ __global__ void __launch_bounds__(kSelectWarps * 32) k_compact_seg(
     if (lane == 31) seg_n[q * nseg + sg] = x;
 }
 
+// the nprobe best of n candidates (keys ck, ids ci in shared memory, id order;
+// n <= 32 * KPL, n >= nprobe), sorted into bs/bc
+template <int KPL>
+__device__ __forceinline__ void compact_finish(const uint32_t *ck, const int *ci, int n, int nprobe,
+                                               int cap, float *bs, int *bc) {
+    const int lane = threadIdx.x & 31;
+    uint32_t key[KPL];
+#pragma unroll
+    for (int j = 0; j < KPL; ++j) {
+        const int c = j * 32 + lane;
+        key[j] = c < n ? ck[c] : 0u;
+    }
+    uint32_t T;
+    int C;
+    warp_threshold(key, nprobe, cap, T, C);
+    warp_gather_sort(key, n, nprobe, T, C, cap, [&](int c) { return ci[c]; }, bs, bc);
+}
+
 // One warp per query: its segments' candidates gathered in order (id order),
 // then the nprobe best sorted into order/cscores.  A segment past kSegCap or
 // more than kCompactCap in all (many equal scores): the query is flagged in
 // ovf and left to the level-by-level selection.
 __global__ void __launch_bounds__(kSelectWarps * 32) k_compact_final(
-    const uint32_t *__restrict__ cand_k, const int32_t *__restrict__ cand_i,
-    const int *__restrict__ seg_n, int64_t nq, int nseg, int nprobe, int P,
+    const float *__restrict__ cand_s, const int32_t *__restrict__ cand_i,
+    const int *__restrict__ seg_n, int64_t nq, int nseg, int segcap, int nprobe, int P,
     int32_t *__restrict__ order, float *__restrict__ cscores, int *__restrict__ ovf) {
     extern __shared__ __align__(16) unsigned char sel_smem[];
     const int cap = 2 * P;
@@ -469,7 +567,7 @@ __global__ void __launch_bounds__(kSelectWarps * 32) k_compact_final(
     for (int s0 = 0; s0 < nseg; s0 += 32) {
         const int sg = s0 + lane;
         const int c = sg < nseg ? seg_n[q * nseg + sg] : 0;
-        over |= __any_sync(0xffffffffu, c > kSegCap);
+        over |= __any_sync(0xffffffffu, c > segcap);
         int x = c;   // inclusive scan over the lanes
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
@@ -482,10 +580,10 @@ __global__ void __launch_bounds__(kSelectWarps * 32) k_compact_final(
             for (int t = 0; t < 32 && s0 + t < nseg; ++t) {
                 const int ct = __shfl_sync(0xffffffffu, c, t);
                 const int at = n + __shfl_sync(0xffffffffu, x, t) - ct;
-                const uint32_t *sk = cand_k + (q * nseg + s0 + t) * kSegCap;
-                const int32_t *si = cand_i + (q * nseg + s0 + t) * kSegCap;
+                const float *ss = cand_s + (q * nseg + s0 + t) * (int64_t)segcap;
+                const int32_t *si = cand_i + (q * nseg + s0 + t) * (int64_t)segcap;
                 for (int i = lane; i < ct; i += 32) {
-                    ck[at + i] = sk[i];
+                    ck[at + i] = order_key(ss[i]);
                     ci[at + i] = si[i];
                 }
             }
@@ -499,17 +597,15 @@ __global__ void __launch_bounds__(kSelectWarps * 32) k_compact_final(
     }
     if (lane == 0) ovf[q] = 0;
     __syncwarp();
-    uint32_t key[kCompactCap / 32];
-#pragma unroll
-    for (int j = 0; j < kCompactCap / 32; ++j) {
-        const int c = j * 32 + lane;
-        key[j] = c < n ? ck[c] : 0u;
-    }
-    const int want = nprobe;   // n >= nprobe: the threshold is reached by at least nprobe scores
-    uint32_t T;
-    int C;
-    warp_threshold(key, want, cap, T, C);
-    warp_gather_sort(key, n, want, T, C, cap, [&](int c) { return ci[c]; }, bs, bc);
+    // keys per lane sized to the candidates (warp-uniform n)
+    if (n <= 256)
+        compact_finish<8>(ck, ci, n, nprobe, cap, bs, bc);
+    else if (n <= 512)
+        compact_finish<16>(ck, ci, n, nprobe, cap, bs, bc);
+    else if (n <= 1024)
+        compact_finish<32>(ck, ci, n, nprobe, cap, bs, bc);
+    else
+        compact_finish<kCompactCap / 32>(ck, ci, n, nprobe, cap, bs, bc);
     for (int p = lane; p < nprobe; p += 32) {
         order[q * nprobe + p] = bc[p];
         if (cscores) cscores[q * nprobe + p] = bs[p];
@@ -532,32 +628,54 @@ static bool use_group_threshold(int64_t nlist, int nprobe) {
     return nlist > kSelectSeg && ng >= nprobe && ng <= kCompactCap;
 }
 
-// per query under the group threshold: the group maxima, the segments'
-// candidate slots (keys + ids) and counts, the threshold key, the overflow flag
-static int64_t group_bytes_per_query(int64_t nlist) {
-    const int64_t nseg = ceil_div(nlist, kSelectSeg);
-    return round_up(ceil_div(nlist, 32), 4) * 4 + nseg * kSegCap * 8 + round_up(nseg, 4) * 4 + 8;
+// Under the group threshold, narrow rows (d <= 128) skip the score table: one
+// contraction writes only the group maxima, a second keeps only the scores
+// that reach the threshold.  Two passes of 6d fp16 products per score cost
+// less than writing and reading 8 bytes per score when d is this small.
+static bool use_two_pass(int64_t nlist, int nprobe, int d) {
+    return use_group_threshold(nlist, nprobe) && d <= 128;
 }
 
-// bytes per query: the score row; two candidate buffers (scores + ids) for
-// the levels of a selection over more than kSelectSeg centroids; the group
-// threshold's buffers
-static int64_t rank_bytes_per_query(int64_t nlist, int nprobe) {
-    int64_t b = rank_tc_ld(nlist) * (int64_t)sizeof(float);
-    if (nlist > kSelectSeg) b += 2 * round_up(level_entries(nlist, nprobe), 4) * 8;
-    if (use_group_threshold(nlist, nprobe)) b += group_bytes_per_query(nlist);
-    return b;
+// Scratch of one query, in the order enqueue_rank_tc lays it out:
+//   score row (table path only)                      round_up(nlist, 32) f32
+//   two level buffers (scores, then ids)             2 x lvl x 8 B   (nlist > kSelectSeg)
+//   group maxima                                     round_up(ng, 4) f32
+//   candidate slots (scores, then ids)               nseg x cap x 8 B (cap = kSegCap, or
+//                                                    kRankRange on the two-pass path)
+//   candidate counts, threshold key, overflow flag   round_up(nseg, 4) x 4 B + 8 B
+struct RankScratch {
+    int64_t ld, lvl, gld, cap;
+    int nseg;
+    bool table, grouped;
+    int64_t per_query() const {
+        int64_t b = table ? ld * 4 : 0;
+        b += 2 * lvl * 8;
+        if (grouped) b += gld * 4 + (int64_t)nseg * cap * 8 + round_up(nseg, 4) * 4 + 8;
+        return b;
+    }
+};
+
+static RankScratch rank_scratch(int64_t nlist, int nprobe, int d) {
+    RankScratch r;
+    r.ld = rank_tc_ld(nlist);
+    r.lvl = nlist > kSelectSeg ? round_up(level_entries(nlist, nprobe), 4) : 0;
+    r.grouped = use_group_threshold(nlist, nprobe);
+    r.table = !use_two_pass(nlist, nprobe, d);
+    r.gld = round_up(ceil_div(nlist, 32), 4);
+    r.nseg = (int)ceil_div(nlist, kSelectSeg);
+    r.cap = r.table ? kSegCap : kRankRange;
+    return r;
 }
 
-int64_t rank_tc_chunk(int64_t nq, int64_t nlist, int nprobe) {
-    int64_t c = kRankScratchBytes / rank_bytes_per_query(nlist, nprobe);
+int64_t rank_tc_chunk(int64_t nq, int64_t nlist, int nprobe, int d) {
+    int64_t c = kRankScratchBytes / rank_scratch(nlist, nprobe, d).per_query();
     c = c / tcp::kM * tcp::kM;
     if (c < tcp::kM) c = tcp::kM;
     return nq < c ? nq : c;
 }
 
-size_t rank_tc_scratch_bytes(int64_t nq, int64_t nlist, int nprobe) {
-    return (size_t)(rank_tc_chunk(nq, nlist, nprobe) * rank_bytes_per_query(nlist, nprobe));
+size_t rank_tc_scratch_bytes(int64_t nq, int64_t nlist, int nprobe, int d) {
+    return (size_t)(rank_tc_chunk(nq, nlist, nprobe, d) * rank_scratch(nlist, nprobe, d).per_query());
 }
 
 static size_t tc_smem() { return tcp::Geometry<RankMode::kN>::smem_bytes(0); }
@@ -604,7 +722,7 @@ cudaError_t prepare_rank_tc(int nprobe, int d) {
 // entries (nseg = 1: the final order)
 static void launch_select(const float *in_s, const int32_t *in_id, int64_t in_ld, int64_t nq,
                           int64_t M, int nprobe, int32_t *out_id, float *out_s, int64_t out_ld,
-                          const int *only, cudaStream_t st) {
+                          const int *only, const int *seg_cnt, cudaStream_t st) {
     const int seg = M < kSelectSeg ? (int)M : kSelectSeg;
     const int nseg = (int)ceil_div(M, kSelectSeg);
     const int P = pow2_at_least(nprobe);
@@ -613,7 +731,8 @@ static void launch_select(const float *in_s, const int32_t *in_id, int64_t in_ld
     const int kpl = pow2_at_least(ceil_div(seg, 32));
 #define SIEVE_SELECT(K)                                                                            \
     k_select<K><<<blocks, kSelectWarps * 32, smem, st>>>(in_s, in_id, in_ld, nq, M, seg, nseg,     \
-                                                        nprobe, P, out_id, out_s, out_ld, only)
+                                                        nprobe, P, out_id, out_s, out_ld, only, \
+                                                        seg_cnt)
     switch (kpl) {
         case 1: SIEVE_SELECT(1); break;
         case 2: SIEVE_SELECT(2); break;
@@ -626,56 +745,68 @@ static void launch_select(const float *in_s, const int32_t *in_id, int64_t in_ld
 #undef SIEVE_SELECT
 }
 
-int rank_tc_launches(int64_t nq, int64_t nlist, int nprobe) {
+int rank_tc_launches(int64_t nq, int64_t nlist, int nprobe, int d) {
     if (nq <= 0) return 0;
     int per = 2;                                           // contraction + final selection
     if (use_group_threshold(nlist, nprobe)) per += 3;      // threshold, compaction, gather
+    // the two-pass path trades the compaction pass for a second contraction: same count
     for (int64_t M = nlist; M > kSelectSeg; M = level_entries(M, nprobe)) ++per;
-    return (int)ceil_div(nq, rank_tc_chunk(nq, nlist, nprobe)) * per;
+    return (int)ceil_div(nq, rank_tc_chunk(nq, nlist, nprobe, d)) * per;
 }
 
 cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t nlist, int d,
                             int nprobe, int32_t *order, float *cscores, float *scratch, int *status,
                             cudaStream_t st, const unsigned char *tc_cent) {
     const int bulk_stages = tc_cent ? rank_bulk_stages(d) : 0;
-    const int64_t ld = rank_tc_ld(nlist);
-    const int64_t chunk = rank_tc_chunk(nq, nlist, nprobe);
-    // after the chunk's score table: two candidate buffers [chunk][lvl_ld]
-    // (scores, then ids) when nlist > kSelectSeg; then the group maxima
-    // [chunk][gld], threshold keys [chunk] and overflow flags [chunk]
-    const int64_t lvl_ld = nlist > kSelectSeg ? round_up(level_entries(nlist, nprobe), 4) : 0;
-    float *cand_s[2] = {scratch + chunk * ld, scratch + chunk * ld + 2 * chunk * lvl_ld};
-    int32_t *cand_id[2] = {reinterpret_cast<int32_t *>(cand_s[0] + chunk * lvl_ld),
-                           reinterpret_cast<int32_t *>(cand_s[1] + chunk * lvl_ld)};
-    const bool grouped = use_group_threshold(nlist, nprobe);
-    const int ng = (int)ceil_div(nlist, 32);
-    const int64_t gld = round_up(ng, 4);
-    const int nseg = (int)ceil_div(nlist, kSelectSeg);
-    float *gmax = scratch + chunk * ld + 4 * chunk * lvl_ld;
-    uint32_t *seg_k = reinterpret_cast<uint32_t *>(gmax + chunk * gld);
-    int32_t *seg_i = reinterpret_cast<int32_t *>(seg_k + chunk * nseg * kSegCap);
-    int *seg_n = seg_i + chunk * nseg * kSegCap;
-    uint32_t *lkey = reinterpret_cast<uint32_t *>(seg_n + chunk * round_up(nseg, 4));
+    const RankScratch L = rank_scratch(nlist, nprobe, d);
+    const int64_t chunk = rank_tc_chunk(nq, nlist, nprobe, d);
+    // carve the chunk's scratch (RankScratch's order, each part [chunk][...])
+    float *p = scratch;
+    float *table = p;
+    p += L.table ? chunk * L.ld : 0;
+    float *cand_s[2];
+    int32_t *cand_id[2];
+    for (int b = 0; b < 2; ++b) {
+        cand_s[b] = p;
+        cand_id[b] = reinterpret_cast<int32_t *>(p + chunk * L.lvl);
+        p += 2 * chunk * L.lvl;
+    }
+    float *gmax = p;
+    p += chunk * L.gld;
+    float *slot_s = p;
+    int32_t *slot_i = reinterpret_cast<int32_t *>(p + chunk * L.nseg * L.cap);
+    p += 2 * chunk * L.nseg * L.cap;
+    int *slot_n = reinterpret_cast<int *>(p);
+    uint32_t *lkey = reinterpret_cast<uint32_t *>(slot_n + chunk * round_up(L.nseg, 4));
     int *ovf = reinterpret_cast<int *>(lkey + chunk);
+    const int ng = (int)ceil_div(nlist, 32);
     const int P = pow2_at_least(nprobe);
     for (int64_t q0 = 0; q0 < nq; q0 += chunk) {
         const int64_t n = nq - q0 < chunk ? nq - q0 : chunk;
-        RankArgs a{Q + q0 * d, n, C, nlist, d, scratch, ld, status, tc_cent,
-                   grouped ? gmax : nullptr, gld};
         const int tiles = (int)(ceil_div(n, tcp::kM) * ceil_div(nlist, kRankRange));
-        if (bulk_stages)
-            k_rank_bulk<<<std::min(tiles, num_sms()), tcb::kThreads,
-                          tcb::smem_bytes(bulk_stages, 0), st>>>(a, bulk_stages);
-        else
-            k_rank_tc<<<std::min(tiles, num_sms()), tcp::kThreads, tc_smem(), st>>>(a);
+        auto contract = [&](const RankArgs &a) {
+            if (bulk_stages)
+                k_rank_bulk<<<std::min(tiles, num_sms()), tcb::kThreads,
+                              tcb::smem_bytes(bulk_stages, 0), st>>>(a, bulk_stages);
+            else
+                k_rank_tc<<<std::min(tiles, num_sms()), tcp::kThreads, tc_smem(), st>>>(a);
+        };
+        RankArgs a{Q + q0 * d, n, C, nlist, d, table, L.ld, status, tc_cent,
+                   L.grouped ? gmax : nullptr, L.gld, L.table ? kRankTable : kRankMax,
+                   lkey, slot_s, slot_i, slot_n};
+        contract(a);
         int32_t *o = order + q0 * nprobe;
         float *cs = cscores ? cscores + q0 * nprobe : nullptr;
         const int *only = nullptr;
-        if (grouped) {
+        const float *lvl0_s = table;       // what the first selection level reads
+        const int32_t *lvl0_id = nullptr;
+        int64_t lvl0_ld = L.ld;
+        const int *lvl0_cnt = nullptr;
+        if (L.grouped) {
             const unsigned wblocks = (unsigned)ceil_div(n, kSelectWarps);
             const int kpl = pow2_at_least(ceil_div(ng, 32));
 #define SIEVE_GTHR(K)                                                                              \
-    k_group_threshold<K><<<wblocks, kSelectWarps * 32, 0, st>>>(gmax, gld, n, ng, nprobe, lkey)
+    k_group_threshold<K><<<wblocks, kSelectWarps * 32, 0, st>>>(gmax, L.gld, n, ng, nprobe, lkey)
             switch (kpl) {
                 case 1: SIEVE_GTHR(1); break;
                 case 2: SIEVE_GTHR(2); break;
@@ -686,27 +817,44 @@ cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t 
                 default: SIEVE_GTHR(64); break;
             }
 #undef SIEVE_GTHR
-            k_compact_seg<<<(unsigned)ceil_div(n * nseg, kSelectWarps), kSelectWarps * 32, 0, st>>>(
-                scratch, ld, n, nlist, nseg, lkey, seg_k, seg_i, seg_n);
+            if (L.table) {
+                k_compact_seg<<<(unsigned)ceil_div(n * L.nseg, kSelectWarps), kSelectWarps * 32, 0,
+                                st>>>(table, L.ld, n, nlist, L.nseg, lkey, slot_s, slot_i, slot_n);
+            } else {
+                RankArgs keep = a;   // the second contraction keeps what reaches the threshold
+                keep.gmax = nullptr;
+                keep.mode = kRankKeep;
+                contract(keep);
+                // an overflowing query's levels read its kept scores, range by range
+                lvl0_s = slot_s;
+                lvl0_id = slot_i;
+                lvl0_ld = (int64_t)L.nseg * L.cap;
+                lvl0_cnt = slot_n;
+            }
             k_compact_final<<<wblocks, kSelectWarps * 32, compact_smem(P), st>>>(
-                seg_k, seg_i, seg_n, n, nseg, nprobe, P, o, cs, ovf);
+                slot_s, slot_i, slot_n, n, L.nseg, (int)L.cap, nprobe, P, o, cs, ovf);
             only = ovf;   // the levels below run only for overflowing queries
         }
-        // levels: the score row, then candidates, until one segment is left
-        const float *in_s = scratch;
-        const int32_t *in_id = nullptr;
-        int64_t in_ld = ld, M = nlist;
+        // levels until one segment is left (segments of the first level are the
+        // 2,048-centroid ranges, whether read from the table or the kept slots)
+        const float *in_s = lvl0_s;
+        const int32_t *in_id = lvl0_id;
+        int64_t in_ld = lvl0_ld, M = L.table ? nlist : (int64_t)L.nseg * L.cap;
+        const int *in_cnt = lvl0_cnt;
+        int64_t M_left = nlist;
         int buf = 0;
-        while (M > kSelectSeg) {
-            launch_select(in_s, in_id, in_ld, n, M, nprobe, cand_id[buf], cand_s[buf], lvl_ld, only,
-                          st);
+        while (M_left > kSelectSeg) {
+            launch_select(in_s, in_id, in_ld, n, M, nprobe, cand_id[buf], cand_s[buf], L.lvl, only,
+                          in_cnt, st);
             in_s = cand_s[buf];
             in_id = cand_id[buf];
-            in_ld = lvl_ld;
-            M = level_entries(M, nprobe);
+            in_ld = L.lvl;
+            in_cnt = nullptr;
+            M_left = level_entries(M_left, nprobe);
+            M = M_left;
             buf ^= 1;
         }
-        launch_select(in_s, in_id, in_ld, n, M, nprobe, o, cs, nprobe, only, st);
+        launch_select(in_s, in_id, in_ld, n, M, nprobe, o, cs, nprobe, only, in_cnt, st);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }

@@ -16,19 +16,6 @@ namespace sieve {
 
 __device__ __forceinline__ int tc_nkb_dev(int d) { return (d + 63) / 64; }
 
-// v[j] for a j known only at run time, by a tree of selects (no local memory)
-__device__ __forceinline__ float pick32(const float (&v)[32], int j) {
-    float t16[16], t8[8], t4[4];
-#pragma unroll
-    for (int i = 0; i < 16; ++i) t16[i] = (j & 16) ? v[i + 16] : v[i];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) t8[i] = (j & 8) ? t16[i + 8] : t16[i];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) t4[i] = (j & 4) ? t8[i + 4] : t8[i];
-    const float t0 = (j & 2) ? t4[2] : t4[0], t1 = (j & 2) ? t4[3] : t4[1];
-    return (j & 1) ? t1 : t0;
-}
-
 struct ScanMode {
     using Args = SearchArgs;
     static constexpr int kN = 256;

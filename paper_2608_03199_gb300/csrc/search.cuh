@@ -87,8 +87,8 @@ cudaError_t enqueue_rank(const float *Q, int64_t nq, const float *C, int64_t nli
 // kRankScratchBytes per chunk of queries, then warp-per-segment selections
 constexpr int64_t kRankScratchBytes = int64_t(2) << 30;
 bool rank_tc_supported(int64_t nlist, int nprobe);
-size_t rank_tc_scratch_bytes(int64_t nq, int64_t nlist, int nprobe);
-int rank_tc_launches(int64_t nq, int64_t nlist, int nprobe);   // kernel launches of one ranking
+size_t rank_tc_scratch_bytes(int64_t nq, int64_t nlist, int nprobe, int d);
+int rank_tc_launches(int64_t nq, int64_t nlist, int nprobe, int d);   // kernel launches of one ranking
 cudaError_t prepare_rank_tc(int nprobe, int d);
 cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t nlist, int d,
                             int nprobe, int32_t *order, float *cscores, float *scratch, int *status,

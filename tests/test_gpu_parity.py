@@ -117,13 +117,15 @@ def test_rank_selection_exact_ties(nlist, dev):
 
 
 @pytest.mark.parametrize("nlist,d,nprobe", [(5000, 96, 256), (2500, 36, 100), (16384, 64, 128),
-                                             (9000, 96, 200), (65536, 32, 256)])
+                                             (9000, 96, 200), (65536, 32, 256), (8192, 160, 128)])
 def test_rank_parity_many_centroids(nlist, d, nprobe, dev):
     """Rankings over more centroids than one selecting warp holds, with d not
     a multiple of the 64-element K-block, against the fp64 oracle ranking;
     rank swaps only across score gaps below the tolerance.  Fewer 32-centroid
     groups than nprobe take the level-by-level selection, the others the
-    group-maximum threshold and one compacting pass."""
+    group-maximum threshold: with a score table and one compacting pass for
+    d > 128, else with a second contraction that keeps only the scores that
+    reach it."""
     rng = np.random.default_rng(nlist + d)
     C = rng.standard_normal((nlist, d)).astype(np.float32)
     C /= np.linalg.norm(C, axis=1, keepdims=True)
