@@ -66,8 +66,11 @@ def _declare(lib):
     lib.oracle_bruteforce.argtypes = [P, P, I64, I32, P, I64, P, F32, I32, P, P, P, I32]
     lib.oracle_fragility.argtypes = [P, P, P, I64, I32, P, I64, P, I64, P, P, P, F32, I32,
                                      I32, P, P, P, I32]
+    lib.oracle_calibrate.argtypes = [P, P, P, I64, I32, P, I64, P, I64, P, P, I64, F32, I32,
+                                     I32, C.c_double, I64, I64, P, P, P, P, P, P, P, I32]
     for name in ("oracle_rank", "oracle_stop_pattern", "oracle_search", "oracle_hit_matrix",
-                 "oracle_fixed_probe", "oracle_bruteforce", "oracle_fragility"):
+                 "oracle_fixed_probe", "oracle_bruteforce", "oracle_fragility",
+                 "oracle_calibrate"):
         getattr(lib, name).restype = C.c_int
     return lib
 
@@ -239,3 +242,33 @@ def fragility(index, Q, tau, k, nprobe, order, upto, qids=None, threads=None):
                                 float(tau), k, nprobe, _p(tg), _p(kg), _p(cg),
                                 threads or default_threads()), "oracle_fragility")
     return tg, kg, cg
+
+
+def calibrate(index, Q, sample, tau, k, nprobe, eps, min_queries=10_000, fallback=8, qids=None,
+              threads=None):
+    """In-call window calibration (Appendix A, Algorithm 3) on the sample rows
+    `sample` (sorted, distinct indices into Q): dict(ids, scores, count, probes
+    for every query, W = the selected window, hist [nprobe + 1] = H[W] for
+    W = 1..nprobe, Z = sum of the sampled fixed-probe result sizes)."""
+    lib = _load()
+    X, ids, assign, Cent = (_c(index["X"], np.float32), _c(index["ids"], np.int64),
+                            _c(index["assign"], np.int32), _c(index["centroids"], np.float32))
+    Q = _c(Q, np.float32)
+    sample = _c(sample, np.int64)
+    qids = None if qids is None else _c(qids, np.int64)
+    nq, d = Q.shape
+    out_ids = np.empty((nq, k), np.int64)
+    out_sc = np.empty((nq, k), np.float64)
+    cnt = np.empty(nq, np.int32)
+    probes = np.empty(nq, np.int32)
+    W = np.zeros(1, np.int64)
+    hist = np.zeros(nprobe + 1, np.int64)
+    Z = np.zeros(1, np.int64)
+    rc = lib.oracle_calibrate(_p(X), _p(ids), _p(assign), X.shape[0], d, _p(Cent), Cent.shape[0],
+                              _p(Q), nq, _p(qids), _p(sample), len(sample), float(tau), k, nprobe,
+                              float(eps), int(min_queries), int(fallback), _p(out_ids), _p(out_sc),
+                              _p(cnt), _p(probes), _p(W), _p(hist), _p(Z),
+                              threads or default_threads())
+    _check(rc, "oracle_calibrate")
+    return {"ids": out_ids, "scores": out_sc, "count": cnt, "probes": probes, "W": int(W[0]),
+            "hist": hist, "Z": int(Z[0])}

@@ -581,3 +581,174 @@ int oracle_fragility(const float *X, const int64_t *ids, const int32_t *assign, 
     lists_free(&L);
     return 0;
 }
+
+/* ------------------------------------------------------------------------ */
+/* In-call window calibration (Appendix A, Algorithm 3).                      */
+/*                                                                            */
+/* The sample Q_s is given as ns sorted, distinct row indices into Q (the     */
+/* paper draws it uniformly without replacement; here the caller does).      */
+/*  1. nq < min_queries or ns == 0: W* = fallback and every query runs the   */
+/*     W*-rule (the paper's fallback for small calls).                        */
+/*  2. FullProbeByPartition: each sampled query searches all nprobe ranks of */
+/*     its order; L_s = the local result of every rank.                       */
+/*  3. A_fixed = MergeTopK(L_s, k); each neighbour keeps the rank it came    */
+/*     from (every row sits in exactly one partition).                        */
+/*  4. RequiredWindowHistogram: window W reaches rank j iff no run of W      */
+/*     consecutive empty ranks ends before j (the stop rule of Sec. 4.1), so */
+/*     a neighbour found at rank j needs W >= 1 + (longest run of empty      */
+/*     ranks before j); H[W] counts neighbours by that required window.      */
+/*  5. Z = sum |A_fixed(q)|; W* = the smallest W < nprobe with               */
+/*     1 - (H[1] + ... + H[W]) / Z < eps, else nprobe; Z == 0: W* = fallback.*/
+/*  6. Every other query runs the W*-rule (sequential form); the sampled     */
+/*     queries keep A_fixed and report nprobe probes.                         */
+/* hist: [nprobe + 1] (H[0] unused); outputs as oracle_search.                */
+int oracle_calibrate(const float *X, const int64_t *ids, const int32_t *assign, int64_t n,
+                     int32_t d, const float *C, int64_t nlist, const float *Q, int64_t nq,
+                     const int64_t *qids, const int64_t *sample, int64_t ns, float tau, int32_t k,
+                     int32_t nprobe, double eps, int64_t min_queries, int64_t fallback,
+                     int64_t *out_ids, double *out_scores, int32_t *out_count,
+                     int32_t *out_probes, int64_t *W_out, int64_t *hist, int64_t *Z_out,
+                     int32_t nthreads)
+{
+    if (d <= 0 || k < 1 || nprobe < 1 || nprobe > nlist || fallback < 1 || isnan(tau) || ns < 0)
+        return -1;
+    for (int64_t s = 0; s < ns; ++s)
+        if (sample[s] < 0 || sample[s] >= nq || (s > 0 && sample[s] <= sample[s - 1]))
+            return -1;
+    for (int w = 0; w <= nprobe; ++w)
+        hist[w] = 0;
+    *Z_out = 0;
+    if (nq < min_queries || ns == 0) {
+        *W_out = fallback;
+        return oracle_search(X, ids, assign, n, d, C, nlist, Q, nq, qids, NULL, tau, k, nprobe,
+                             fallback, 0, 0, out_ids, out_scores, out_count, out_probes, nthreads);
+    }
+    lists_t L;
+    if (lists_build(&L, assign, n, nlist) != 0) {
+        lists_free(&L);
+        return -2;
+    }
+    index_t ix = {X, ids, &L, d};
+    int64_t Z = 0;
+    int bad = 0;
+    /* steps 2-4 for every sampled query */
+#pragma omp parallel num_threads(nthreads > 0 ? nthreads : 1)
+    {
+        cscore_t *scratch = (cscore_t *)malloc((size_t)nlist * sizeof(cscore_t));
+        int32_t *order = (int32_t *)malloc((size_t)nprobe * sizeof(int32_t));
+        cand_t *store = (cand_t *)malloc((size_t)nprobe * (size_t)k * sizeof(cand_t));
+        int *local_n = (int *)malloc((size_t)nprobe * sizeof(int));
+        cand_t *fin = (cand_t *)malloc((size_t)k * sizeof(cand_t));
+        int64_t *h = (int64_t *)calloc((size_t)nprobe + 1, sizeof(int64_t));
+        int64_t z = 0;
+        if (!scratch || !order || !store || !local_n || !fin || !h) {
+#pragma omp atomic write
+            bad = -2;
+        } else {
+#pragma omp for schedule(dynamic, 4)
+            for (int64_t s = 0; s < ns; ++s) {
+                const int64_t i = sample[s];
+                const float *q = Q + i * (int64_t)d;
+                rank_one(q, C, nlist, d, nprobe, scratch, order, NULL);
+                /* FullProbeByPartition: L_s, rank by rank */
+                query_ctx_t ctx = {&ix, q, qids != NULL, qids ? qids[i] : 0, order, (double)tau,
+                                   k, store, local_n};
+                for (int j = 1; j <= nprobe; ++j)
+                    search_probe(&ctx, j);
+                /* MergeTopK */
+                topk_t final = {k, 0, fin};
+                for (int j = 0; j < nprobe; ++j)
+                    for (int m = 0; m < local_n[j]; ++m)
+                        topk_offer(&final, store[(int64_t)j * k + m].score,
+                                   store[(int64_t)j * k + m].id);
+                /* RequiredWindowHistogram: walk the ranks in order */
+                int run = 0, longest = 0;
+                for (int j = 1; j <= nprobe; ++j) {
+                    for (int m = 0; m < final.n; ++m) {   /* neighbours found at rank j */
+                        int from_j = 0;
+                        for (int t = 0; t < local_n[j - 1]; ++t)
+                            if (store[(int64_t)(j - 1) * k + t].id == fin[m].id)
+                                from_j = 1;
+                        if (from_j)
+                            h[1 + longest]++;
+                    }
+                    run = local_n[j - 1] > 0 ? 0 : run + 1;   /* a hit has a local result */
+                    if (run > longest)
+                        longest = run;
+                }
+                z += final.n;
+                for (int m = 0; m < k; ++m) {
+                    out_ids[i * (int64_t)k + m] = m < final.n ? fin[m].id : -1;
+                    out_scores[i * (int64_t)k + m] = m < final.n ? fin[m].score : -INFINITY;
+                }
+                out_count[i] = final.n;
+                out_probes[i] = nprobe;
+            }
+#pragma omp critical
+            {
+                for (int w = 0; w <= nprobe; ++w)
+                    hist[w] += h[w];
+                Z += z;
+            }
+        }
+        free(scratch); free(order); free(store); free(local_n); free(fin); free(h);
+    }
+    lists_free(&L);
+    if (bad)
+        return bad;
+    /* step 5: the smallest pruned window under the loss target */
+    int64_t Wstar = nprobe;
+    if (Z == 0) {
+        Wstar = fallback;
+    } else {
+        int64_t retained = 0;
+        for (int w = 1; w < nprobe; ++w) {
+            retained += hist[w];
+            double loss = 1.0 - (double)retained / (double)Z;
+            if (loss < eps) {
+                Wstar = w;
+                break;
+            }
+        }
+    }
+    *W_out = Wstar;
+    *Z_out = Z;
+    /* step 6: the rest of the batch under W* */
+    int64_t nr = nq - ns;
+    if (nr == 0)
+        return 0;
+    float *Qr = (float *)malloc((size_t)nr * (size_t)d * sizeof(float));
+    int64_t *qr = qids ? (int64_t *)malloc((size_t)nr * sizeof(int64_t)) : NULL;
+    int64_t *idx = (int64_t *)malloc((size_t)nr * sizeof(int64_t));
+    int64_t *oi = (int64_t *)malloc((size_t)nr * (size_t)k * sizeof(int64_t));
+    double *os = (double *)malloc((size_t)nr * (size_t)k * sizeof(double));
+    int32_t *oc = (int32_t *)malloc((size_t)nr * sizeof(int32_t));
+    int32_t *op = (int32_t *)malloc((size_t)nr * sizeof(int32_t));
+    int rc = -2;
+    if (Qr && (qr || !qids) && idx && oi && os && oc && op) {
+        int64_t r = 0, s = 0;
+        for (int64_t i = 0; i < nq; ++i) {
+            if (s < ns && sample[s] == i) {
+                ++s;
+                continue;
+            }
+            idx[r] = i;
+            memcpy(Qr + r * (int64_t)d, Q + i * (int64_t)d, (size_t)d * sizeof(float));
+            if (qids)
+                qr[r] = qids[i];
+            ++r;
+        }
+        rc = oracle_search(X, ids, assign, n, d, C, nlist, Qr, nr, qr, NULL, tau, k, nprobe, Wstar,
+                           0, 0, oi, os, oc, op, nthreads);
+        if (rc == 0)
+            for (int64_t r2 = 0; r2 < nr; ++r2) {
+                int64_t i = idx[r2];
+                memcpy(out_ids + i * (int64_t)k, oi + r2 * (int64_t)k, (size_t)k * sizeof(int64_t));
+                memcpy(out_scores + i * (int64_t)k, os + r2 * (int64_t)k, (size_t)k * sizeof(double));
+                out_count[i] = oc[r2];
+                out_probes[i] = op[r2];
+            }
+    }
+    free(Qr); free(qr); free(idx); free(oi); free(os); free(oc); free(op);
+    return rc;
+}

@@ -13,6 +13,7 @@ import numpy as np
 import pytest
 
 import oracle
+import test_oracle_calibration as K
 import test_oracle_search as S
 import test_oracle_stopping as T
 
@@ -33,6 +34,10 @@ MUTATIONS = [
      "m + 1 < (local_n[j] > 0 ? local_n[j] : 0)"),
     ("window off by one", "while (searched < nprobe && stale < W)",
      "while (searched < nprobe && stale <= W)"),
+    ("required window one short", "h[1 + longest]++;", "h[longest > 0 ? longest : 1]++;"),
+    ("empty run not reset by a hit", "run = local_n[j - 1] > 0 ? 0 : run + 1;",
+     "run = local_n[j - 1] > 0 ? run : run + 1;"),
+    ("loss target inclusive", "if (loss < eps) {", "if (loss <= eps) {"),
 ]
 
 
@@ -47,6 +52,9 @@ def _pins(tiny, deep):
         lambda: S.test_full_probe_equals_bruteforce(deep),
         lambda: S.test_window_at_least_nprobe_is_fixed_probe(tiny, 16),
         lambda: S.test_probes_follow_hit_pattern(deep),
+        lambda: K.test_calibration_matches_brute_force_loss(deep, 0.05),
+        lambda: K.test_calibration_window_extremes_and_fallbacks(deep),
+        K.test_calibration_histogram_of_gapped_hits,
     ]
 
 
