@@ -285,6 +285,38 @@ sieve_status sieve_search_noalloc(const sieve_index_view *ix, const float *Q, in
                                   int32_t *out_count, int32_t *out_probes, sieve_stats *stats,
                                   void *stream);
 
+/* In-call window calibration (Appendix A, Algorithm 3): the search picks W
+ * itself from a sample of the batch.
+ *   1. If nq < min_queries or ns == 0, W* = fallback_W and every query runs
+ *      with it (the paper's fallback for small calls).
+ *   2. The ns sampled queries (sample: device [ns] int64, strictly increasing
+ *      row indices of Q; the paper draws them uniformly without replacement)
+ *      search all nprobe partitions (fixed probing); their results are final.
+ *   3. Each neighbour kept for a sampled query was found at some rank j; the
+ *      W-rule reaches rank j iff no run of W empty ranks precedes it, so it
+ *      needs W >= 1 + (longest run of empty ranks before j).  H[W] counts the
+ *      neighbours by that required window; Z = their total.
+ *   4. W* = the smallest W < nprobe with 1 - (H[1] + ... + H[W]) / Z < eps,
+ *      else nprobe (full probing); Z == 0: W* = fallback_W.
+ *   5. The other nq - ns queries run the search with W = W*.
+ * p->W is ignored; p->profile must be 0.  Outputs as sieve_search, for every
+ * row of Q (sampled rows report nprobe probes).  W_out (host, required)
+ * receives W*; hist_out (host [nprobe + 1], nullable) receives H (H[0] = 0);
+ * Z_out (host, nullable) receives Z.  The call synchronizes `stream` once,
+ * to read W* back before the second search.  SIEVE_EINVAL if the sample is
+ * not strictly increasing rows of Q.  ws: at least
+ * sieve_calibrated_search_workspace_size bytes, 256-byte aligned. */
+sieve_status sieve_calibrated_search_workspace_size(const sieve_index_view *ix, int64_t nq,
+                                                    int64_t ns, const sieve_params *p,
+                                                    size_t *bytes);
+sieve_status sieve_calibrated_search(const sieve_index_view *ix, const float *Q, int64_t nq,
+                                     const int64_t *query_ids, const sieve_params *p,
+                                     const int64_t *sample, int64_t ns, double eps,
+                                     int64_t min_queries, int32_t fallback_W, int64_t *out_ids,
+                                     float *out_scores, int32_t *out_count, int32_t *out_probes,
+                                     int32_t *W_out, int64_t *hist_out, int64_t *Z_out, void *ws,
+                                     size_t ws_bytes, void *stream);
+
 /* Human-readable name of a status code (static string). */
 const char *sieve_status_str(sieve_status s);
 

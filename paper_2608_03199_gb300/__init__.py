@@ -19,6 +19,7 @@ import ctypes as C
 import threading
 from dataclasses import dataclass
 
+import numpy as np
 import torch
 
 from . import _build
@@ -97,6 +98,16 @@ _SIGNATURES = {
                                          C.c_void_p, C.c_void_p, C.POINTER(ParamsC), C.c_void_p,
                                          C.c_void_p, C.c_void_p, C.c_void_p, C.POINTER(StatsC),
                                          C.c_void_p]),
+    "sieve_calibrated_search_workspace_size": (C.c_int32, [C.POINTER(IndexViewC), C.c_int64,
+                                                           C.c_int64, C.POINTER(ParamsC),
+                                                           C.POINTER(C.c_size_t)]),
+    "sieve_calibrated_search": (C.c_int32, [C.POINTER(IndexViewC), C.c_void_p, C.c_int64,
+                                            C.c_void_p, C.POINTER(ParamsC), C.c_void_p, C.c_int64,
+                                            C.c_double, C.c_int64, C.c_int32, C.c_void_p,
+                                            C.c_void_p, C.c_void_p, C.c_void_p,
+                                            C.POINTER(C.c_int32), C.c_void_p,
+                                            C.POINTER(C.c_int64), C.c_void_p, C.c_size_t,
+                                            C.c_void_p]),
     "sieve_status_str": (C.c_char_p, [C.c_int32]),
     "sieve_last_cuda_error": (C.c_int32, []),
     "sieve_version": (C.c_char_p, []),
@@ -346,6 +357,45 @@ def search(index: Index, Q, tau, k, nprobe, W, lookahead=True, query_ids=None, o
     if stats:
         return ids, scores, count, probes, _stats_dict(st)
     return ids, scores, count, probes
+
+
+def calibrated_search(index: Index, Q, tau, k, nprobe, sample, eps, min_queries=10_000,
+                      fallback_W=8, lookahead=True, query_ids=None, max_items_per_round=0,
+                      scan_path="auto", workspace=None, stream=None):
+    """In-call window calibration (sieve_calibrated_search, Appendix A).
+
+    sample: int64 device tensor of strictly increasing row indices of Q (the
+    queries that are fully probed).  Returns (ids, scores, count, probes,
+    info) with info = dict(W = the selected window, hist = numpy [nprobe + 1]
+    counts of neighbours by required window, Z = their total).  The call
+    synchronizes the stream once."""
+    _need_cuda(Q, torch.float32, "Q", 2)
+    _need_cuda(sample, torch.int64, "sample", 1)
+    if query_ids is not None:
+        _need_cuda(query_ids, torch.int64, "query_ids", 1)
+    nq, ns = Q.shape[0], sample.shape[0]
+    dev = Q.device
+    p = _params(tau, k, nprobe, nprobe, lookahead, 0, max_items_per_round, 0, scan_path)
+    v = index.view()
+    nbytes = C.c_size_t()
+    _check(lib().sieve_calibrated_search_workspace_size(C.byref(v), nq, ns, C.byref(p),
+                                                        C.byref(nbytes)),
+           "sieve_calibrated_search_workspace_size")
+    ws = _workspace(workspace, nbytes.value, dev)
+    ids = torch.empty((nq, k), dtype=torch.int64, device=dev)
+    scores = torch.empty((nq, k), dtype=torch.float32, device=dev)
+    count = torch.empty(nq, dtype=torch.int32, device=dev)
+    probes = torch.empty(nq, dtype=torch.int32, device=dev)
+    W = C.c_int32(0)
+    Z = C.c_int64(0)
+    hist = np.zeros(nprobe + 1, np.int64)
+    _check(lib().sieve_calibrated_search(C.byref(v), _ptr(Q), nq, _ptr(query_ids), C.byref(p),
+                                         _ptr(sample), ns, float(eps), int(min_queries),
+                                         int(fallback_W), _ptr(ids), _ptr(scores), _ptr(count),
+                                         _ptr(probes), C.byref(W),
+                                         hist.ctypes.data_as(C.c_void_p), C.byref(Z), _ptr(ws),
+                                         ws.numel(), _stream(stream)), "sieve_calibrated_search")
+    return ids, scores, count, probes, {"W": W.value, "hist": hist, "Z": Z.value}
 
 
 def search_host(index: Index, Q_host, tau, k, nprobe, W, lookahead=True, query_ids_host=None,

@@ -271,11 +271,17 @@ struct EventSet {
 
 // the device-side search on device buffers (shared by sieve_search and
 // sieve_search_host); arguments already checked
+// optional provenance outputs of a search (window calibration)
+struct SearchExtras {
+    int32_t *out_rank;    // [nq][k]
+    uint32_t *hit_bits;   // [nq][ceil(nprobe / 32)]
+};
+
 sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t nq,
                            const int64_t *qids, const int32_t *order, const sieve_params *p,
                            int64_t *out_ids, float *out_scores, int32_t *out_count,
                            int32_t *out_probes, sieve_stats *stats, unsigned char *ws,
-                           const Layout &L, cudaStream_t st) {
+                           const Layout &L, cudaStream_t st, const SearchExtras *ex = nullptr) {
     SearchArgs a;
     std::memset(&a, 0, sizeof(a));   // padding takes part in the graph-cache key
     a.X = ix->vectors;
@@ -325,6 +331,11 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
     a.out_count = out_count;
     a.out_probes = out_probes;
     a.ctl = reinterpret_cast<Ctl *>(ws + L.ctl);
+    if (ex) {
+        a.out_rank = ex->out_rank;
+        a.hit_bits = ex->hit_bits;
+        a.hit_words = (int)ceil_div(p->nprobe, 32);
+    }
 
     const bool with_rank = order == nullptr;
     const int rank_tc = with_rank && a.rank_scratch != nullptr;
@@ -608,6 +619,156 @@ sieve_status sieve_search_host(const sieve_index_view *ix, const float *Q_host, 
     SIEVE_CUDA(cudaMemcpyAsync(out_count_host, dcnt, (size_t)nq * 4, cudaMemcpyDeviceToHost, st));
     SIEVE_CUDA(cudaMemcpyAsync(out_probes_host, dpr, (size_t)nq * 4, cudaMemcpyDeviceToHost, st));
     SIEVE_CUDA(cudaStreamSynchronize(st));
+    return SIEVE_OK;
+}
+
+// ---------------------------------------------------------------------------
+// In-call window calibration (Appendix A, Algorithm 3).  Scratch, in order:
+// the inner search's workspace (sized for the larger of the two searches, both
+// at W = nprobe, the widest window the calibration can pick), then the sample
+// and remainder buffers below.
+struct CalibLayout {
+    Layout inner;
+    size_t Qs, qs, s_ids, s_sc, s_cnt, s_pr, s_rank, s_hits, rest, Qr, qr, r_ids, r_sc, r_cnt, r_pr,
+        hist, Z, W, bad, total;
+};
+
+static CalibLayout make_calib_layout(const sieve_index_view *ix, int64_t nq, int64_t ns,
+                                     const sieve_params *p) {
+    CalibLayout C{};
+    sieve_params wide = *p;
+    wide.W = p->nprobe;
+    const int64_t nr = nq - ns;
+    const Layout a = make_layout(ix, ns, &wide, false), b = make_layout(ix, nr, &wide, false);
+    C.inner = a.total >= b.total ? a : b;
+    size_t off = C.inner.total;
+    auto take = [&](size_t bytes) {
+        size_t at = off;
+        off += (size_t)round_up((int64_t)std::max<size_t>(bytes, 1), 256);
+        return at;
+    };
+    const int k = p->k, d = ix->d;
+    const int words = (int)ceil_div(p->nprobe, 32);
+    C.Qs = take((size_t)ns * d * 4);
+    C.qs = take((size_t)ns * 8);
+    C.s_ids = take((size_t)ns * k * 8);
+    C.s_sc = take((size_t)ns * k * 4);
+    C.s_cnt = take((size_t)ns * 4);
+    C.s_pr = take((size_t)ns * 4);
+    C.s_rank = take((size_t)ns * k * 4);
+    C.s_hits = take((size_t)ns * words * 4);
+    C.rest = take((size_t)nr * 8);
+    C.Qr = take((size_t)nr * d * 4);
+    C.qr = take((size_t)nr * 8);
+    C.r_ids = take((size_t)nr * k * 8);
+    C.r_sc = take((size_t)nr * k * 4);
+    C.r_cnt = take((size_t)nr * 4);
+    C.r_pr = take((size_t)nr * 4);
+    C.hist = take((size_t)(p->nprobe + 1) * 8);
+    C.Z = take(8);
+    C.W = take(4);
+    C.bad = take(4);
+    C.total = off;
+    return C;
+}
+
+sieve_status sieve_calibrated_search_workspace_size(const sieve_index_view *ix, int64_t nq,
+                                                    int64_t ns, const sieve_params *p,
+                                                    size_t *bytes) {
+    if (!bytes) return SIEVE_EINVAL;
+    sieve_status rc = check_index(ix, true);
+    if (rc != SIEVE_OK) return rc;
+    if ((rc = check_params(ix, p)) != SIEVE_OK) return rc;
+    if (nq < 0 || nq > INT32_MAX / 2 || ns < 0 || ns > nq) return SIEVE_EINVAL;
+    const Layout plain = make_layout(ix, nq, p, false);
+    *bytes = std::max(plain.total, make_calib_layout(ix, nq, ns, p).total);
+    return SIEVE_OK;
+}
+
+sieve_status sieve_calibrated_search(const sieve_index_view *ix, const float *Q, int64_t nq,
+                                     const int64_t *query_ids, const sieve_params *p,
+                                     const int64_t *sample, int64_t ns, double eps,
+                                     int64_t min_queries, int32_t fallback_W, int64_t *out_ids,
+                                     float *out_scores, int32_t *out_count, int32_t *out_probes,
+                                     int32_t *W_out, int64_t *hist_out, int64_t *Z_out, void *ws,
+                                     size_t ws_bytes, void *stream) {
+    sieve_status rc = check_search(ix, Q, nq, nullptr, p, out_ids, out_scores, out_count, out_probes);
+    if (rc != SIEVE_OK) return rc;
+    if (!W_out || ns < 0 || ns > nq || (ns > 0 && !sample) || fallback_W < 1 || !(eps == eps) ||
+        p->profile || (nq > 0 && !aligned16(Q)) || !ix->centroids)
+        return SIEVE_EINVAL;
+    if ((rc = check_device()) != SIEVE_OK) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    unsigned char *w = static_cast<unsigned char *>(ws);
+    if (hist_out)
+        for (int i = 0; i <= p->nprobe; ++i) hist_out[i] = 0;
+    if (Z_out) *Z_out = 0;
+    if (nq == 0) {
+        *W_out = fallback_W;
+        return SIEVE_OK;
+    }
+    if (nq < min_queries || ns == 0) {   // small calls: the fallback window, no sample
+        *W_out = fallback_W;
+        sieve_params q = *p;
+        q.W = fallback_W;
+        const Layout L = make_layout(ix, nq, &q, false);
+        if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < L.total)
+            return SIEVE_EWORKSPACE;
+        return search_device(ix, Q, nq, query_ids, nullptr, &q, out_ids, out_scores, out_count,
+                             out_probes, nullptr, w, L, st);
+    }
+    const CalibLayout C = make_calib_layout(ix, nq, ns, p);
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < C.total)
+        return SIEVE_EWORKSPACE;
+    const int k = p->k, d = ix->d;
+    const int64_t nr = nq - ns;
+    auto F = [&](size_t off) { return reinterpret_cast<float *>(w + off); };
+    auto I64 = [&](size_t off) { return reinterpret_cast<int64_t *>(w + off); };
+    auto I32 = [&](size_t off) { return reinterpret_cast<int32_t *>(w + off); };
+    int *bad_d = I32(C.bad);
+    SIEVE_CUDA(calib_check_sample(sample, ns, nq, bad_d, st));
+    // 1. the sample, fully probed, with each kept result's rank and the hit bits
+    SIEVE_CUDA(calib_gather(Q, query_ids, d, sample, ns, F(C.Qs), I64(C.qs), st));
+    sieve_params full = *p;
+    full.W = p->nprobe;
+    SearchExtras ex{I32(C.s_rank), reinterpret_cast<uint32_t *>(w + C.s_hits)};
+    const Layout Ls = make_layout(ix, ns, &full, false);
+    rc = search_device(ix, F(C.Qs), ns, query_ids ? I64(C.qs) : nullptr, nullptr, &full,
+                       I64(C.s_ids), F(C.s_sc), I32(C.s_cnt), I32(C.s_pr), nullptr, w, Ls, st, &ex);
+    if (rc != SIEVE_OK) return rc;
+    // 2. the histogram of required windows and W*
+    SIEVE_CUDA(calib_pick(reinterpret_cast<const unsigned *>(w + C.s_hits), (int)ceil_div(p->nprobe, 32),
+                          I32(C.s_rank), I32(C.s_cnt), ns, k, p->nprobe, eps, fallback_W,
+                          reinterpret_cast<unsigned long long *>(w + C.hist),
+                          reinterpret_cast<unsigned long long *>(w + C.Z), I32(C.W), st));
+    int32_t w_star = 0, bad = 0;
+    SIEVE_CUDA(cudaMemcpyAsync(&w_star, I32(C.W), 4, cudaMemcpyDeviceToHost, st));
+    SIEVE_CUDA(cudaMemcpyAsync(&bad, bad_d, 4, cudaMemcpyDeviceToHost, st));
+    if (hist_out)
+        SIEVE_CUDA(cudaMemcpyAsync(hist_out, w + C.hist, (size_t)(p->nprobe + 1) * 8,
+                                   cudaMemcpyDeviceToHost, st));
+    if (Z_out) SIEVE_CUDA(cudaMemcpyAsync(Z_out, w + C.Z, 8, cudaMemcpyDeviceToHost, st));
+    SIEVE_CUDA(cudaStreamSynchronize(st));
+    if (bad) return SIEVE_EINVAL;   // the sample was not strictly increasing rows of Q
+    *W_out = w_star;
+    // 3. the rest of the batch under W*, then every row to its place
+    if (nr > 0) {
+        SIEVE_CUDA(calib_complement(sample, ns, nq, I64(C.rest), st));
+        SIEVE_CUDA(calib_gather(Q, query_ids, d, I64(C.rest), nr, F(C.Qr), I64(C.qr), st));
+        sieve_params rest = *p;
+        rest.W = w_star;
+        const Layout Lr = make_layout(ix, nr, &rest, false);
+        rc = search_device(ix, F(C.Qr), nr, query_ids ? I64(C.qr) : nullptr, nullptr, &rest,
+                           I64(C.r_ids), F(C.r_sc), I32(C.r_cnt), I32(C.r_pr), nullptr, w, Lr, st);
+        if (rc != SIEVE_OK) return rc;
+        SIEVE_CUDA(calib_scatter(I64(C.rest), nr, k, reinterpret_cast<const long long *>(I64(C.r_ids)),
+                                 F(C.r_sc), I32(C.r_cnt), I32(C.r_pr),
+                                 reinterpret_cast<long long *>(out_ids), out_scores, out_count,
+                                 out_probes, st));
+    }
+    SIEVE_CUDA(calib_scatter(sample, ns, k, reinterpret_cast<const long long *>(I64(C.s_ids)), F(C.s_sc),
+                             I32(C.s_cnt), I32(C.s_pr), reinterpret_cast<long long *>(out_ids),
+                             out_scores, out_count, out_probes, st));
     return SIEVE_OK;
 }
 

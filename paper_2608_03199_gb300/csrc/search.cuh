@@ -53,6 +53,12 @@ struct SearchArgs {
     float *out_scores;
     int *out_count, *out_probes;
     Ctl *ctl;
+    // optional provenance (window calibration): the 1-based rank each kept
+    // result came from [nq][k], and one bit per rank that held a qualifying
+    // row [nq][hit_words]
+    int *out_rank;
+    unsigned *hit_bits;
+    int hit_words;
 };
 
 size_t scan_smem_bytes(int d, int k);
@@ -94,6 +100,21 @@ cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t 
                             int nprobe, int32_t *order, float *cscores, float *scratch, int *status,
                             cudaStream_t st, const unsigned char *tc_cent = nullptr);
 int rank_bulk_stages(int d);                     // 0 when the bulk ranking does not apply
+
+// in-call window calibration (calibrate.cu)
+cudaError_t calib_gather(const float *Q, const int64_t *qids, int d, const int64_t *idx, int64_t n,
+                         float *Qo, int64_t *qo, cudaStream_t st);
+cudaError_t calib_complement(const int64_t *sample, int64_t ns, int64_t nq, int64_t *rest,
+                             cudaStream_t st);
+cudaError_t calib_check_sample(const int64_t *sample, int64_t ns, int64_t nq, int *bad,
+                               cudaStream_t st);
+cudaError_t calib_pick(const unsigned *hit_bits, int words, const int *out_rank, const int *count,
+                       int64_t ns, int k, int nprobe, double eps, int fallback,
+                       unsigned long long *hist, unsigned long long *Z, int *W_out,
+                       cudaStream_t st);
+cudaError_t calib_scatter(const int64_t *idx, int64_t n, int k, const long long *ids, const float *sc,
+                          const int *cnt, const int *pr, long long *out_ids, float *out_sc,
+                          int *out_cnt, int *out_pr, cudaStream_t st);
 
 // tensor-core layout of partition rows and centroids (tc_layout.cu)
 constexpr int kTcRows = 128;                   // rows per block

@@ -33,7 +33,10 @@ __global__ void k_init(SearchArgs a) {
     for (int64_t i = t0; i < a.nq * a.k; i += stride) {
         a.out_ids[i] = -1;
         a.out_scores[i] = -__int_as_float(0x7f800000);
+        if (a.out_rank) a.out_rank[i] = 0;
     }
+    if (a.hit_bits)
+        for (int64_t i = t0; i < a.nq * a.hit_words; i += stride) a.hit_bits[i] = 0u;
     // the control block was zeroed by a memset before this kernel; a list
     // offset table that is not a partition of [0, n) is reported and the
     // search then issues nothing
@@ -458,12 +461,20 @@ __global__ void __launch_bounds__(kMergeThreads) k_merge(SearchArgs a) {
         int n = a.out_count[q];
         float r0s = ninf, r1s = ninf;
         long long r0i = -1, r1i = -1;
+        int r0r = 0, r1r = 0;   // provenance ranks (kept only when out_rank is set)
         const int64_t ob = (int64_t)q * k;
         if ((int)lane < n) { r0s = a.out_scores[ob + lane]; r0i = a.out_ids[ob + lane]; }
         if ((int)lane + 32 < n) { r1s = a.out_scores[ob + lane + 32]; r1i = a.out_ids[ob + lane + 32]; }
+        if (a.out_rank) {
+            if ((int)lane < n) r0r = a.out_rank[ob + lane];
+            if ((int)lane + 32 < n) r1r = a.out_rank[ob + lane + 32];
+        }
         bool changed = false;
         for (int it = start; it < start + got; ++it) {
             const int c = a.res_cnt[it];
+            const int rk = a.item_rank[it];
+            if (a.hit_bits && c > 0 && lane == 0)   // this query's items: one warp, no race
+                a.hit_bits[(int64_t)q * a.hit_words + (rk - 1) / 32] |= 1u << ((rk - 1) % 32);
             for (int j = 0; j < c; ++j) {
                 const float s = a.res_s[(int64_t)it * k + j];
                 const long long id = a.res_id[(int64_t)it * k + j];
@@ -478,12 +489,15 @@ __global__ void __launch_bounds__(kMergeThreads) k_merge(SearchArgs a) {
                 long long u1i = __shfl_up_sync(0xffffffffu, r1i, 1);
                 float w31s = __shfl_sync(0xffffffffu, r0s, 31);
                 long long w31i = __shfl_sync(0xffffffffu, r0i, 31);
-                if (lane == 0) { u1s = w31s; u1i = w31i; }
+                int u0r = __shfl_up_sync(0xffffffffu, r0r, 1);
+                int u1r = __shfl_up_sync(0xffffffffu, r1r, 1);
+                const int w31r = __shfl_sync(0xffffffffu, r0r, 31);
+                if (lane == 0) { u1s = w31s; u1i = w31i; u1r = w31r; }
                 const int j0 = lane, j1 = lane + 32;
-                if (j0 == pos) { r0s = s; r0i = id; }
-                else if (j0 > pos) { r0s = u0s; r0i = u0i; }
-                if (j1 == pos) { r1s = s; r1i = id; }
-                else if (j1 > pos) { r1s = u1s; r1i = u1i; }
+                if (j0 == pos) { r0s = s; r0i = id; r0r = rk; }
+                else if (j0 > pos) { r0s = u0s; r0i = u0i; r0r = u0r; }
+                if (j1 == pos) { r1s = s; r1i = id; r1r = rk; }
+                else if (j1 > pos) { r1s = u1s; r1i = u1i; r1r = u1r; }
                 n = n < k ? n + 1 : k;
                 changed = true;
             }
@@ -496,6 +510,10 @@ __global__ void __launch_bounds__(kMergeThreads) k_merge(SearchArgs a) {
             if ((int)lane + 32 < k) {
                 a.out_scores[ob + lane + 32] = (int)lane + 32 < n ? r1s : ninf;
                 a.out_ids[ob + lane + 32] = (int)lane + 32 < n ? r1i : -1;
+            }
+            if (a.out_rank) {
+                if ((int)lane < k) a.out_rank[ob + lane] = (int)lane < n ? r0r : 0;
+                if ((int)lane + 32 < k) a.out_rank[ob + lane + 32] = (int)lane + 32 < n ? r1r : 0;
             }
             if (lane == 0) a.out_count[q] = n;
         }
