@@ -49,6 +49,8 @@ def parse():
     ap.add_argument("--config", default="1m")
     ap.add_argument("--skip-cpu-baseline", action="store_true")
     ap.add_argument("--skip-e2e", action="store_true")
+    ap.add_argument("--skip-calibration", action="store_true",
+                    help="skip the in-call window calibration measurement")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="target CPU seconds for the oracle sample")
     ap.add_argument("--scan-path", choices=("auto", "simt", "tensor"), default="auto",
@@ -373,6 +375,35 @@ def run_sieve(args, cfg, world, rank, local):
     mean_probes = float(probes.float().mean().item())
     hit_frac = float((outs[2] > 0).float().mean().item())
 
+    # in-call window calibration (Appendix A): a 2% sample fully probed, a 0.5%
+    # sample-relative loss target, the rest under the selected window
+    calib = None
+    if not args.skip_calibration:
+        g = torch.Generator(device="cpu").manual_seed(12345 + rank)
+        ns = max(1, (cfg.nq * 2 + 99) // 100)
+        sample = torch.sort(torch.randperm(cfg.nq, generator=g)[:ns]).values.to(dev)
+        cws = sieve.Workspace()
+
+        def cstep():
+            return sieve.calibrated_search(index, Q, cfg.tau, k, cfg.nprobe, sample, 0.005,
+                                           query_ids=qids, workspace=cws,
+                                           scan_path=args.scan_path)
+        info = cstep()[4]
+        csteps = max(3, args.steps // 20)
+        torch.cuda.synchronize()
+        barrier(world)
+        t0 = time.perf_counter()
+        for _ in range(csteps):
+            cstep()
+        torch.cuda.synchronize()
+        barrier(world)
+        c_ms = max_over_ranks((time.perf_counter() - t0) / csteps * 1e3, world, dev)
+        calib = {"value": nq * world / (c_ms * 1e-3), "unit": "queries/s", "ms_per_step": c_ms,
+                 "W": info["W"], "sample": ns, "loss_target": 0.005,
+                 "sample_neighbours": info["Z"],
+                 "speedup_vs_fixed": ms_fixed / c_ms,
+                 "timing": "host clock around whole calls (each reads W back once)"}
+
     # end to end through the C ABI with host buffers
     e2e = None
     if not args.skip_e2e:
@@ -423,6 +454,7 @@ def run_sieve(args, cfg, world, rank, local):
         "fixed_probe": {"value": nq * world / (ms_fixed * 1e-3), "ms_per_step": ms_fixed,
                         "W": cfg.nprobe},
         "speedup_vs_fixed": ms_fixed / ms,
+        "calibrated": calib,
         "mean_probes": mean_probes,
         "queries_with_results": hit_frac,
         "roofline": roofline(prof, cfg, dev, bulk=index.tc_rows is not None,
