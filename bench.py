@@ -49,6 +49,9 @@ def parse():
     ap.add_argument("--config", default="1m")
     ap.add_argument("--skip-cpu-baseline", action="store_true")
     ap.add_argument("--skip-e2e", action="store_true")
+    ap.add_argument("--sweep", action="store_true",
+                    help="operating-envelope sweeps (W, lookahead, tau, k, nprobe, batch): one "
+                         "JSON line per setting instead of the benchmark line")
     ap.add_argument("--skip-calibration", action="store_true",
                     help="skip the in-call window calibration measurement")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
@@ -477,6 +480,71 @@ def run_sieve(args, cfg, world, rank, local):
     return 0
 
 
+def run_sweep(args, cfg):
+    """Operating-envelope sweeps on one workload (not the benchmark line): one
+    JSON line per setting with the time per call, queries/s, mean probes and
+    the pooled recall of the kept neighbours against fixed probing (the same
+    index, tau, k and nprobe).  Varied one at a time from the workload's own
+    setting: W with lookahead on and off (serial traversal issues one rank
+    per query per round), tau, k, nprobe, and the batch size."""
+    import paper_2608_03199_gb300 as sieve
+    dev = torch.device("cuda:0")
+    sieve.lib()
+    wl = synth.make_workload(cfg, device=dev)
+    index = sieve.build_layout(wl["X"], wl["assign"], cfg.nlist, wl["centroids"])
+    Q, qids = wl["Q"], wl["qids"]
+    ws = sieve.Workspace()
+
+    def timed(nq, tau, k, nprobe, W, lookahead):
+        run = lambda: sieve.search(index, Q[:nq], tau, k, nprobe, W, lookahead=lookahead,
+                                   query_ids=qids[:nq], workspace=ws)
+        for _ in range(2):
+            out = run()
+        torch.cuda.synchronize()
+        reps = max(3, min(50, int(2e5 // max(nq, 1))))
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            out = run()
+        e1.record()
+        torch.cuda.synchronize()
+        return out, e0.elapsed_time(e1) / reps
+
+    def recall(out, ref):
+        a_ids, a_cnt = out[0].cpu().numpy(), out[2].cpu().numpy()
+        f_ids, f_cnt = ref[0].cpu().numpy(), ref[2].cpu().numpy()
+        kept = sum(len(set(a_ids[i, :a_cnt[i]]) & set(f_ids[i, :f_cnt[i]])) for i in range(len(a_cnt)))
+        tot = int(f_cnt.sum())
+        return kept / tot if tot else 1.0
+
+    settings = []
+    for W in (cfg.sweep_W or (2, 4, 8, 16, cfg.nprobe)):
+        for la in (True, False):
+            settings.append(("W", cfg.nq, cfg.tau, cfg.k, cfg.nprobe, W, la))
+    for tau in (0.85, 0.90, 0.95):
+        settings.append(("tau", cfg.nq, tau, cfg.k, cfg.nprobe, cfg.W, True))
+    for k in (5, 10, 20, 50):
+        settings.append(("k", cfg.nq, cfg.tau, k, cfg.nprobe, cfg.W, True))
+    for nprobe in sorted({16, 32, cfg.nprobe, min(2 * cfg.nprobe, cfg.nlist)}):
+        settings.append(("nprobe", cfg.nq, cfg.tau, cfg.k, nprobe, min(cfg.W, nprobe), True))
+    for nq in sorted({1, 100, 1_000, 10_000, cfg.nq}):
+        if nq <= cfg.nq:
+            settings.append(("batch", nq, cfg.tau, cfg.k, cfg.nprobe, cfg.W, True))
+    fixed_cache = {}
+    for (axis, nq, tau, k, nprobe, W, la) in settings:
+        key = (nq, tau, k, nprobe)
+        if key not in fixed_cache:
+            fixed_cache[key] = timed(nq, tau, k, nprobe, nprobe, True)
+        ref, ms_fixed = fixed_cache[key]
+        out, ms = timed(nq, tau, k, nprobe, W, la)
+        print(json.dumps({"sweep": axis, "nq": nq, "tau": tau, "k": k, "nprobe": nprobe, "W": W,
+                          "lookahead": la, "ms": round(ms, 4), "queries_per_s": round(nq / (ms * 1e-3)),
+                          "fixed_ms": round(ms_fixed, 4), "speedup_vs_fixed": round(ms_fixed / ms, 3),
+                          "mean_probes": round(float(out[3].float().mean()), 3),
+                          "recall_vs_fixed": round(recall(out, ref), 5)}), flush=True)
+    return 0
+
+
 def run_ncu_case(args, cfg):
     """One search call on the benchmark workload, nothing else on the GPU after it."""
     import paper_2608_03199_gb300 as sieve
@@ -500,6 +568,8 @@ def main():
     world, rank, local = dist_setup(args.gpus)
     if args.ncu_case:
         return run_ncu_case(args, cfg)
+    if args.sweep:
+        return run_sweep(args, cfg)
     if args.impl == "reference":
         return run_reference(args, cfg, world, rank)
     return run_sieve(args, cfg, world, rank, local)

@@ -100,10 +100,11 @@ typedef struct {
  *              stats pointer); 0 = no timing
  *   scan_path  which units compute similarities; all paths give the same
  *              decisions up to fp32 rounding (see the parity notes):
- *              0 = automatic (ranking on the tensor cores; every partition
- *              group on the tensor cores when k <= 16, on FP32 FMA
- *              otherwise), 1 = FP32 FMA only, 2 = tensor cores (needs
- *              k <= 16)
+ *              0 = automatic (ranking and every partition group on the
+ *              tensor cores when the epilogue's k-lists fit: any k with
+ *              the tensor-core layout and d <= 256, k <= 22 otherwise; FP32
+ *              FMA beyond), 1 = FP32 FMA only, 2 = tensor cores
+ *              (SIEVE_EINVAL where they do not fit)
  */
 typedef struct {
     float tau;

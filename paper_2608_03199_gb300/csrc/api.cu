@@ -63,7 +63,6 @@ sieve_status check_params(const sieve_index_view *ix, const sieve_params *p) {
     if (p->max_items_per_round < 0) return SIEVE_EINVAL;
     if (p->profile != 0 && p->profile != 1) return SIEVE_EINVAL;
     if (p->scan_path < 0 || p->scan_path > 2) return SIEVE_EINVAL;
-    if (p->scan_path == 2 && p->k > kTcMaxK) return SIEVE_EINVAL;
     return SIEVE_OK;
 }
 
@@ -312,13 +311,19 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
     a.bucketed = reinterpret_cast<int *>(ws + L.bucketed);
     a.tiles = reinterpret_cast<int4 *>(ws + L.tiles);
     a.tc_tiles = reinterpret_cast<int4 *>(ws + L.tc_tiles);
-    a.tc_min = p->scan_path == 1 ? 0 : (p->k <= kTcMaxK ? 1 : 0);
     a.active = reinterpret_cast<int4 *>(ws + L.active);
     a.rank_scratch = L.rank_scratch ? reinterpret_cast<float *>(ws + L.rank_scratch) : nullptr;
     a.tc_rows = static_cast<const unsigned char *>(ix->tc_rows);
     a.tc_row_blocks = ix->tc_row_blocks;
     a.tc_cent = static_cast<const unsigned char *>(ix->tc_centroids);
-    a.tc_stages = (a.tc_min > 0 && a.tc_rows && a.tc_row_blocks) ? scan_bulk_stages(ix->d, p->k) : 0;
+    // the tensor cores take every group when their epilogue's lists fit beside
+    // the pipeline's stages: the bulk pipeline (tensor layout, d <= 256) for
+    // any k <= 64, the converter pipeline for smaller k
+    const int bulk_stages = (a.tc_rows && a.tc_row_blocks) ? scan_bulk_stages(ix->d, p->k) : 0;
+    const bool tc_fits = bulk_stages > 0 || scan_tc_fits(p->k);
+    if (p->scan_path == 2 && !tc_fits) return SIEVE_EINVAL;
+    a.tc_min = (p->scan_path == 1 || !tc_fits) ? 0 : 1;
+    a.tc_stages = a.tc_min > 0 ? bulk_stages : 0;
     if (!a.tc_stages) {
         a.tc_rows = nullptr;
         a.tc_row_blocks = nullptr;

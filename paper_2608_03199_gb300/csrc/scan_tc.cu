@@ -176,6 +176,8 @@ struct ScanMode {
     };
 };
 
+bool scan_tc_fits(int k) { return scan_tc_smem_bytes(k) <= (size_t)(232448 - 128); }
+
 size_t scan_tc_smem_bytes(int k) {
     return tcp::Geometry<ScanMode::kN>::smem_bytes((size_t)tcp::kM * k * (sizeof(float) + sizeof(long long)));
 }

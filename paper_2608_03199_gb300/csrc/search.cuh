@@ -73,9 +73,9 @@ cudaError_t launch_round(const SearchArgs &a, size_t scan_smem, int scan_blocks,
 constexpr int kRoundKernels = 7;   // issue, bucket, scatter, scan_tc, scan, merge, round_end
 
 // tensor-core scan (scan_tc.cu)
-constexpr int kTcMaxK = 16;        // largest k the tensor-core epilogue keeps
 constexpr int kTcTile = 128;       // items per tensor-core tile
 size_t scan_tc_smem_bytes(int k);
+bool scan_tc_fits(int k);          // the converter pipeline's shared memory holds k-lists
 cudaError_t prepare_scan_tc(int k);
 void enqueue_scan_tc(const SearchArgs &a, cudaStream_t st);
 // the same fed from the tensor-core layout by bulk copies (d <= 256)

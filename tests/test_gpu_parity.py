@@ -278,9 +278,20 @@ def test_empty_and_single_query(tiny, g_tiny, dev):
 
 
 @pytest.mark.parametrize("k", [1, 3, 33, 64])
-def test_k_range(deep, g_deep, k):
+@pytest.mark.parametrize("path", ["auto", "simt"])
+def test_k_range(deep, g_deep, k, path):
+    """Large k on the tensor cores (bulk pipeline) and on FP32 FMA."""
     c = deep["cfg"]
-    check(deep, g_deep, deep["Q"], deep["qids"], c.tau, k, c.nprobe, c.W, 1)
+    check(deep, g_deep, deep["Q"], deep["qids"], c.tau, k, c.nprobe, c.W, 1, scan_path=path)
+
+
+def test_k_on_the_converter_pipeline(deep, g_deep):
+    """Without the tensor layout the converter pipeline keeps k-lists up to
+    k = 22 on the tensor cores; larger k falls back to FP32 FMA."""
+    c = deep["cfg"]
+    plain = g_deep.without_tc_layout()
+    for k in (20, 22, 40):
+        check(deep, plain, deep["Q"], deep["qids"], c.tau, k, c.nprobe, c.W, 1)
 
 
 def test_no_query_ids_and_low_tau(deep, g_deep):
@@ -329,8 +340,8 @@ def test_empty_partitions_and_odd_dimension(dev):
 
 def test_invalid_arguments_raise(tiny, g_tiny, dev):
     Q = torch.from_numpy(tiny["Q"][:4]).to(dev)
-    with pytest.raises(sieve.SieveError):
-        sieve.search(g_tiny, Q, 0.9, 17, 16, 4, scan_path="tensor")   # tensor path needs k <= 16
+    with pytest.raises(sieve.SieveError):   # converter pipeline: k-lists up to k = 22 fit
+        sieve.search(g_tiny.without_tc_layout(), Q, 0.9, 23, 16, 4, scan_path="tensor")
     for kw in (dict(k=0), dict(k=65), dict(nprobe=65), dict(W=0)):
         args = dict(tau=0.9, k=10, nprobe=16, W=4)
         args.update(kw)
