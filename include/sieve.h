@@ -318,6 +318,25 @@ sieve_status sieve_calibrated_search(const sieve_index_view *ix, const float *Q,
                                      int32_t *W_out, int64_t *hist_out, int64_t *Z_out, void *ws,
                                      size_t ws_bytes, void *stream);
 
+/* A query batch over nshards independent IVF indexes (the public-100M layout
+ * of Sec. 6.1: coarse shards, each with its own IVF index and centroids;
+ * the ids of all shards are distinct): every shard runs sieve_search on the
+ * whole batch with its own ranking and stopping, with window
+ * W_per_shard[s] (host [nshards], nullable: p->W for every shard), and the
+ * global top-k by (score desc, id asc) merges the shards' results.
+ * out_probes receives the partitions searched over all shards; shard_probes
+ * (device [nq][nshards], nullable) each shard's.  Every shard must have the
+ * same d and satisfy p (nprobe <= its nlist).  ws: at least
+ * sieve_sharded_search_workspace_size bytes, 256-byte aligned. */
+sieve_status sieve_sharded_search_workspace_size(const sieve_index_view *shards, int32_t nshards,
+                                                 int64_t nq, const sieve_params *p,
+                                                 const int32_t *W_per_shard, size_t *bytes);
+sieve_status sieve_sharded_search(const sieve_index_view *shards, int32_t nshards, const float *Q,
+                                  int64_t nq, const int64_t *query_ids, const sieve_params *p,
+                                  const int32_t *W_per_shard, int64_t *out_ids, float *out_scores,
+                                  int32_t *out_count, int32_t *out_probes, int32_t *shard_probes,
+                                  void *ws, size_t ws_bytes, void *stream);
+
 /* Human-readable name of a status code (static string). */
 const char *sieve_status_str(sieve_status s);
 

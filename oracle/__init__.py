@@ -272,3 +272,30 @@ def calibrate(index, Q, sample, tau, k, nprobe, eps, min_queries=10_000, fallbac
     _check(rc, "oracle_calibrate")
     return {"ids": out_ids, "scores": out_sc, "count": cnt, "probes": probes, "W": int(W[0]),
             "hist": hist, "Z": int(Z[0])}
+
+
+def sharded_search(shards, Q, tau, k, nprobe, W, qids=None, threads=None):
+    """A query batch over several independent IVF indexes (the public-100M
+    layout of Sec. 6.1: coarse shards, each with its own IVF index): every
+    shard runs the search on its own (its own ranking and stopping; W is one
+    window or one per shard), then the global top-k by (score desc, id asc)
+    merges the shards' results.  Returns dict(ids, scores, count, probes =
+    partitions searched over all shards, shard_probes [nq][nshards])."""
+    Ws = list(W) if isinstance(W, (list, tuple, np.ndarray)) else [W] * len(shards)
+    parts = [search(sh, Q, tau, k, nprobe, w, qids=qids, threads=threads) for sh, w in zip(shards, Ws)]
+    nq = len(parts[0]["count"])
+    ids = np.concatenate([p["ids"] for p in parts], axis=1)
+    sc = np.concatenate([p["scores"] for p in parts], axis=1)
+    out_ids = np.full((nq, k), -1, np.int64)
+    out_sc = np.full((nq, k), -np.inf)
+    cnt = np.zeros(nq, np.int32)
+    for i in range(nq):
+        valid = ids[i] >= 0
+        order = np.lexsort((ids[i][valid], -sc[i][valid]))[:k]
+        n = len(order)
+        out_ids[i, :n] = ids[i][valid][order]
+        out_sc[i, :n] = sc[i][valid][order]
+        cnt[i] = n
+    shard_probes = np.stack([p["probes"] for p in parts], axis=1)
+    return {"ids": out_ids, "scores": out_sc, "count": cnt,
+            "probes": shard_probes.sum(axis=1).astype(np.int32), "shard_probes": shard_probes}

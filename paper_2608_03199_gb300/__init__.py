@@ -108,6 +108,13 @@ _SIGNATURES = {
                                             C.POINTER(C.c_int32), C.c_void_p,
                                             C.POINTER(C.c_int64), C.c_void_p, C.c_size_t,
                                             C.c_void_p]),
+    "sieve_sharded_search_workspace_size": (C.c_int32, [C.POINTER(IndexViewC), C.c_int32,
+                                                        C.c_int64, C.POINTER(ParamsC),
+                                                        C.c_void_p, C.POINTER(C.c_size_t)]),
+    "sieve_sharded_search": (C.c_int32, [C.POINTER(IndexViewC), C.c_int32, C.c_void_p, C.c_int64,
+                                         C.c_void_p, C.POINTER(ParamsC), C.c_void_p, C.c_void_p,
+                                         C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+                                         C.c_void_p, C.c_size_t, C.c_void_p]),
     "sieve_status_str": (C.c_char_p, [C.c_int32]),
     "sieve_last_cuda_error": (C.c_int32, []),
     "sieve_version": (C.c_char_p, []),
@@ -396,6 +403,38 @@ def calibrated_search(index: Index, Q, tau, k, nprobe, sample, eps, min_queries=
                                          hist.ctypes.data_as(C.c_void_p), C.byref(Z), _ptr(ws),
                                          ws.numel(), _stream(stream)), "sieve_calibrated_search")
     return ids, scores, count, probes, {"W": W.value, "hist": hist, "Z": Z.value}
+
+
+def sharded_search(shards, Q, tau, k, nprobe, W, lookahead=True, query_ids=None,
+                   max_items_per_round=0, scan_path="auto", workspace=None, stream=None):
+    """sieve_sharded_search over a list of Index shards (distinct ids across
+    shards): each shard searches the batch with its own ranking and stopping
+    (W: one window, or one per shard), the global top-k merges them.
+    Returns (ids, scores, count, probes = partitions over all shards,
+    shard_probes [nq][nshards])."""
+    _need_cuda(Q, torch.float32, "Q", 2)
+    if query_ids is not None:
+        _need_cuda(query_ids, torch.int64, "query_ids", 1)
+    nq, ns = Q.shape[0], len(shards)
+    dev = Q.device
+    Ws = list(W) if isinstance(W, (list, tuple)) else [W] * ns
+    p = _params(tau, k, nprobe, max(Ws), lookahead, 0, max_items_per_round, 0, scan_path)
+    views = (IndexViewC * ns)(*[sh.view() for sh in shards])
+    wps = (C.c_int32 * ns)(*[int(min(w, 2**31 - 1)) for w in Ws])
+    nbytes = C.c_size_t()
+    _check(lib().sieve_sharded_search_workspace_size(views, ns, nq, C.byref(p), wps, C.byref(nbytes)),
+           "sieve_sharded_search_workspace_size")
+    ws = _workspace(workspace, nbytes.value, dev)
+    ids = torch.empty((nq, k), dtype=torch.int64, device=dev)
+    scores = torch.empty((nq, k), dtype=torch.float32, device=dev)
+    count = torch.empty(nq, dtype=torch.int32, device=dev)
+    probes = torch.empty(nq, dtype=torch.int32, device=dev)
+    shard_probes = torch.empty((nq, ns), dtype=torch.int32, device=dev)
+    _check(lib().sieve_sharded_search(views, ns, _ptr(Q), nq, _ptr(query_ids), C.byref(p), wps,
+                                      _ptr(ids), _ptr(scores), _ptr(count), _ptr(probes),
+                                      _ptr(shard_probes), _ptr(ws), ws.numel(), _stream(stream)),
+           "sieve_sharded_search")
+    return ids, scores, count, probes, shard_probes
 
 
 def search_host(index: Index, Q_host, tau, k, nprobe, W, lookahead=True, query_ids_host=None,

@@ -777,6 +777,108 @@ sieve_status sieve_calibrated_search(const sieve_index_view *ix, const float *Q,
     return SIEVE_OK;
 }
 
+// ---------------------------------------------------------------------------
+// Sharded search (Sec. 6.1's public-100M layout).  Scratch: the inner
+// search's workspace (the largest any shard needs), then the shards' results.
+struct ShardLayout {
+    Layout inner;
+    size_t ids, sc, cnt, pr, total;
+};
+
+static sieve_status shard_params(const sieve_params *p, const int32_t *W_per_shard, int s,
+                                 sieve_params *out) {
+    *out = *p;
+    if (W_per_shard) out->W = W_per_shard[s];
+    return out->W >= 1 ? SIEVE_OK : SIEVE_EINVAL;
+}
+
+static ShardLayout make_shard_layout(const sieve_index_view *shards, int nshards, int64_t nq,
+                                     const sieve_params *p, const int32_t *W_per_shard) {
+    ShardLayout S{};
+    for (int s = 0; s < nshards; ++s) {
+        sieve_params ps;
+        shard_params(p, W_per_shard, s, &ps);
+        const Layout L = make_layout(&shards[s], nq, &ps, false);
+        if (L.total > S.inner.total) S.inner = L;
+    }
+    size_t off = S.inner.total;
+    auto take = [&](size_t bytes) {
+        size_t at = off;
+        off += (size_t)round_up((int64_t)std::max<size_t>(bytes, 1), 256);
+        return at;
+    };
+    S.ids = take((size_t)nshards * nq * p->k * 8);
+    S.sc = take((size_t)nshards * nq * p->k * 4);
+    S.cnt = take((size_t)nshards * nq * 4);
+    S.pr = take((size_t)nshards * nq * 4);
+    S.total = off;
+    return S;
+}
+
+static sieve_status check_shards(const sieve_index_view *shards, int32_t nshards,
+                                 const sieve_params *p, const int32_t *W_per_shard) {
+    if (!shards || nshards < 1) return SIEVE_EINVAL;
+    for (int s = 0; s < nshards; ++s) {
+        sieve_status rc = check_index(&shards[s], true);
+        if (rc != SIEVE_OK) return rc;
+        if (shards[s].d != shards[0].d) return SIEVE_EINVAL;
+        sieve_params ps;
+        if ((rc = shard_params(p, W_per_shard, s, &ps)) != SIEVE_OK) return rc;
+        if ((rc = check_params(&shards[s], &ps)) != SIEVE_OK) return rc;
+    }
+    return SIEVE_OK;
+}
+
+sieve_status sieve_sharded_search_workspace_size(const sieve_index_view *shards, int32_t nshards,
+                                                 int64_t nq, const sieve_params *p,
+                                                 const int32_t *W_per_shard, size_t *bytes) {
+    if (!bytes || !p) return SIEVE_EINVAL;
+    sieve_status rc = check_shards(shards, nshards, p, W_per_shard);
+    if (rc != SIEVE_OK) return rc;
+    if (nq < 0 || nq > INT32_MAX / 2) return SIEVE_EINVAL;
+    *bytes = make_shard_layout(shards, nshards, nq, p, W_per_shard).total;
+    return SIEVE_OK;
+}
+
+sieve_status sieve_sharded_search(const sieve_index_view *shards, int32_t nshards, const float *Q,
+                                  int64_t nq, const int64_t *query_ids, const sieve_params *p,
+                                  const int32_t *W_per_shard, int64_t *out_ids, float *out_scores,
+                                  int32_t *out_count, int32_t *out_probes, int32_t *shard_probes,
+                                  void *ws, size_t ws_bytes, void *stream) {
+    if (!p) return SIEVE_EINVAL;
+    sieve_status rc = check_shards(shards, nshards, p, W_per_shard);
+    if (rc != SIEVE_OK) return rc;
+    if ((rc = check_search(&shards[0], Q, nq, nullptr, p, out_ids, out_scores, out_count,
+                           out_probes)) != SIEVE_OK)
+        return rc;
+    if (p->profile || (nq > 0 && !aligned16(Q))) return SIEVE_EINVAL;
+    if ((rc = check_device()) != SIEVE_OK) return rc;
+    if (nq == 0) return SIEVE_OK;
+    const ShardLayout S = make_shard_layout(shards, nshards, nq, p, W_per_shard);
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < S.total)
+        return SIEVE_EWORKSPACE;
+    unsigned char *w = static_cast<unsigned char *>(ws);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int k = p->k;
+    int64_t *ids = reinterpret_cast<int64_t *>(w + S.ids);
+    float *sc = reinterpret_cast<float *>(w + S.sc);
+    int32_t *cnt = reinterpret_cast<int32_t *>(w + S.cnt);
+    int32_t *pr = reinterpret_cast<int32_t *>(w + S.pr);
+    for (int s = 0; s < nshards; ++s) {   // each shard ranks and stops on its own
+        sieve_params ps;
+        shard_params(p, W_per_shard, s, &ps);
+        const Layout L = make_layout(&shards[s], nq, &ps, false);
+        rc = search_device(&shards[s], Q, nq, query_ids, nullptr, &ps, ids + (int64_t)s * nq * k,
+                           sc + (int64_t)s * nq * k, cnt + (int64_t)s * nq, pr + (int64_t)s * nq,
+                           nullptr, w, L, st);
+        if (rc != SIEVE_OK) return rc;
+    }
+    SIEVE_CUDA(launch_merge_shards(nshards, nq, k, reinterpret_cast<const long long *>(ids), sc, cnt,
+                                   pr, reinterpret_cast<long long *>(out_ids), out_scores, out_count,
+                                   out_probes, shard_probes, st));
+    return SIEVE_OK;
+}
+
 }  // extern "C"
 
 // ---------------------------------------------------------------------------

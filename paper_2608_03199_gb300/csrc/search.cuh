@@ -116,6 +116,12 @@ cudaError_t calib_scatter(const int64_t *idx, int64_t n, int k, const long long 
                           const int *cnt, const int *pr, long long *out_ids, float *out_sc,
                           int *out_cnt, int *out_pr, cudaStream_t st);
 
+// the global top-k of several shards' results (shard.cu); per-shard arrays
+// are [nshards][nq][k] and [nshards][nq]
+cudaError_t launch_merge_shards(int nshards, int64_t nq, int k, const long long *ids, const float *sc,
+                                const int *cnt, const int *pr, long long *out_ids, float *out_sc,
+                                int *out_cnt, int *out_pr, int *shard_probes, cudaStream_t st);
+
 // tensor-core layout of partition rows and centroids (tc_layout.cu)
 constexpr int kTcRows = 128;                   // rows per block
 constexpr int64_t kTcBlockBytes = 32768;       // one K-block (64 elements) of a block: hi + lo fp16

@@ -232,3 +232,30 @@ def to_numpy(wl: dict) -> dict:
     for key in ("X", "ids", "centroids", "assign", "Q", "qids"):
         out[key] = wl[key].detach().cpu().numpy()
     return out
+
+
+@torch.no_grad()
+def make_sharded_workload(cfg: Workload | str, nshards: int, nlist_per_shard: int, device="cpu"):
+    """The corpus of ``cfg`` split into coarse shards, each with its own IVF
+    index (the public-100M layout of Sec. 6.1: coarse k-means shards, a
+    separately built IVF index per shard): spherical k-means with ``nshards``
+    centroids assigns every row a shard; each shard's rows get their own
+    spherical k-means with ``nlist_per_shard`` centroids and exact assignment.
+    Returns dict(Q, qids, shards = [dict(X, ids, centroids, assign)], cfg);
+    ids are the rows' indices in the unsharded corpus, queries are drawn as in
+    make_workload."""
+    if isinstance(cfg, str):
+        cfg = CONFIGS[cfg]
+    X, g = make_corpus(cfg, device)
+    coarse = replace(cfg, nlist=nshards, train_cap=min(cfg.n, 256 * nshards))
+    _, shard_of = build_index(X, coarse, g)
+    shards = []
+    for s in range(nshards):
+        rows = (shard_of == s).nonzero().flatten()
+        Xs = X[rows].contiguous()
+        scfg = replace(cfg, nlist=min(nlist_per_shard, rows.numel()),
+                       train_cap=min(rows.numel(), 256 * nlist_per_shard))
+        cent, assign = build_index(Xs, scfg, g)
+        shards.append({"X": Xs, "ids": rows.to(torch.int64), "centroids": cent, "assign": assign})
+    qrows = torch.randperm(cfg.n, generator=g, device=device)[:cfg.nq]
+    return {"cfg": cfg, "Q": X[qrows].contiguous(), "qids": qrows.to(torch.int64), "shards": shards}
