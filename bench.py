@@ -52,6 +52,11 @@ def parse():
     ap.add_argument("--sweep", action="store_true",
                     help="operating-envelope sweeps (W, lookahead, tau, k, nprobe, batch): one "
                          "JSON line per setting instead of the benchmark line")
+    ap.add_argument("--shards", type=int, default=0,
+                    help="sharded layout: split the corpus into this many coarse shards, each "
+                         "with its own IVF index (one JSON line instead of the benchmark line)")
+    ap.add_argument("--nlist-per-shard", type=int, default=1500)
+    ap.add_argument("--nprobe", type=int, default=0, help="nprobe per shard (0: the workload's)")
     ap.add_argument("--skip-calibration", action="store_true",
                     help="skip the in-call window calibration measurement")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
@@ -545,6 +550,59 @@ def run_sweep(args, cfg):
     return 0
 
 
+def run_sharded(args, cfg):
+    """The sharded layout of the paper's public-100M workloads (Sec. 6.1): the
+    corpus split into --shards coarse shards, each with its own IVF index of
+    --nlist-per-shard partitions, searched at nprobe per shard with its own
+    stopping, then the global top-k.  One JSON line (not the benchmark line):
+    W = the workload's W against fixed probing on every shard."""
+    import gc
+    import paper_2608_03199_gb300 as sieve
+    dev = torch.device("cuda:0")
+    sieve.lib()
+    nprobe = args.nprobe or cfg.nprobe
+    w = synth.make_sharded_workload(cfg, args.shards, args.nlist_per_shard, device=dev)
+    shards = []
+    for sh in w["shards"]:
+        idx = sieve.build_layout(sh["X"], sh["assign"], sh["centroids"].shape[0], sh["centroids"])
+        shards.append(sieve.Index(idx.vectors, sh["ids"][idx.ids], idx.list_offsets, idx.centroids,
+                                  idx.tc_rows, idx.tc_row_blocks, idx.tc_centroids))
+        sh.clear()
+    Q, qids = w["Q"], w["qids"]
+    del w
+    gc.collect()
+    torch.cuda.empty_cache()
+    ws = sieve.Workspace()
+
+    def timed(W, reps):
+        run = lambda: sieve.sharded_search(shards, Q, cfg.tau, cfg.k, nprobe, W, query_ids=qids,
+                                           workspace=ws)
+        out = run()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            out = run()
+        e1.record()
+        torch.cuda.synchronize()
+        return out, e0.elapsed_time(e1) / reps
+
+    out, ms = timed(cfg.W, max(3, args.steps // 40))
+    fx, ms_fixed = timed(nprobe, 3)
+    a_ids, a_cnt = out[0].cpu().numpy(), out[2].cpu().numpy()
+    f_ids, f_cnt = fx[0].cpu().numpy(), fx[2].cpu().numpy()
+    kept = sum(len(set(a_ids[i, :a_cnt[i]]) & set(f_ids[i, :f_cnt[i]])) for i in range(len(a_cnt)))
+    print(json.dumps({
+        "sharded": True, "workload": workload_desc(cfg), "shards": args.shards,
+        "nlist_per_shard": args.nlist_per_shard, "nprobe_per_shard": nprobe, "W": cfg.W,
+        "nq": cfg.nq, "ms_per_call": ms, "queries_per_s": cfg.nq / (ms * 1e-3),
+        "fixed_ms_per_call": ms_fixed, "speedup_vs_fixed": ms_fixed / ms,
+        "mean_probes_over_shards": float(out[3].float().mean()),
+        "recall_vs_fixed": kept / max(1, int(f_cnt.sum())),
+        "timing": "CUDA events around whole calls (every shard's search and the merge)"}))
+    return 0
+
+
 def run_ncu_case(args, cfg):
     """One search call on the benchmark workload, nothing else on the GPU after it."""
     import paper_2608_03199_gb300 as sieve
@@ -570,6 +628,8 @@ def main():
         return run_ncu_case(args, cfg)
     if args.sweep:
         return run_sweep(args, cfg)
+    if args.shards:
+        return run_sharded(args, cfg)
     if args.impl == "reference":
         return run_reference(args, cfg, world, rank)
     return run_sieve(args, cfg, world, rank, local)
