@@ -337,6 +337,20 @@ sieve_status sieve_sharded_search(const sieve_index_view *shards, int32_t nshard
                                   int32_t *out_count, int32_t *out_probes, int32_t *shard_probes,
                                   void *ws, size_t ws_bytes, void *stream);
 
+/* The global top-k of per-shard results (the merge step of
+ * sieve_sharded_search, for shards searched by separate calls, e.g. each
+ * shard calibrating its own window with sieve_calibrated_search on the same
+ * sample, as Appendix A does for the public-100M shards).  Inputs (device):
+ * ids/scores [nshards][nq][k] sorted by (score desc, id asc) and padded,
+ * count/probes [nshards][nq].  Outputs (device): out_* [nq][k] and [nq]
+ * (probes summed over shards); shard_probes [nq][nshards] (nullable).
+ * Asynchronous on `stream`. */
+sieve_status sieve_merge_shard_results(int32_t nshards, int64_t nq, int32_t k,
+                                       const int64_t *ids, const float *scores,
+                                       const int32_t *count, const int32_t *probes,
+                                       int64_t *out_ids, float *out_scores, int32_t *out_count,
+                                       int32_t *out_probes, int32_t *shard_probes, void *stream);
+
 /* Human-readable name of a status code (static string). */
 const char *sieve_status_str(sieve_status s);
 

@@ -274,15 +274,8 @@ def calibrate(index, Q, sample, tau, k, nprobe, eps, min_queries=10_000, fallbac
             "hist": hist, "Z": int(Z[0])}
 
 
-def sharded_search(shards, Q, tau, k, nprobe, W, qids=None, threads=None):
-    """A query batch over several independent IVF indexes (the public-100M
-    layout of Sec. 6.1: coarse shards, each with its own IVF index): every
-    shard runs the search on its own (its own ranking and stopping; W is one
-    window or one per shard), then the global top-k by (score desc, id asc)
-    merges the shards' results.  Returns dict(ids, scores, count, probes =
-    partitions searched over all shards, shard_probes [nq][nshards])."""
-    Ws = list(W) if isinstance(W, (list, tuple, np.ndarray)) else [W] * len(shards)
-    parts = [search(sh, Q, tau, k, nprobe, w, qids=qids, threads=threads) for sh, w in zip(shards, Ws)]
+def _merge_shards(parts, k):
+    """Global top-k by (score desc, id asc) over per-shard results."""
     nq = len(parts[0]["count"])
     ids = np.concatenate([p["ids"] for p in parts], axis=1)
     sc = np.concatenate([p["scores"] for p in parts], axis=1)
@@ -299,3 +292,26 @@ def sharded_search(shards, Q, tau, k, nprobe, W, qids=None, threads=None):
     shard_probes = np.stack([p["probes"] for p in parts], axis=1)
     return {"ids": out_ids, "scores": out_sc, "count": cnt,
             "probes": shard_probes.sum(axis=1).astype(np.int32), "shard_probes": shard_probes}
+
+
+def sharded_calibrated_search(shards, Q, sample, tau, k, nprobe, eps, min_queries=10_000,
+                              fallback=8, qids=None, threads=None):
+    """Every shard calibrates its own window on the same sample (Appendix A's
+    scale-out evaluation), then the global top-k.  Adds Ws (per shard)."""
+    parts = [calibrate(sh, Q, sample, tau, k, nprobe, eps, min_queries=min_queries,
+                       fallback=fallback, qids=qids, threads=threads) for sh in shards]
+    out = _merge_shards(parts, k)
+    out["Ws"] = [p["W"] for p in parts]
+    return out
+
+
+def sharded_search(shards, Q, tau, k, nprobe, W, qids=None, threads=None):
+    """A query batch over several independent IVF indexes (the public-100M
+    layout of Sec. 6.1: coarse shards, each with its own IVF index): every
+    shard runs the search on its own (its own ranking and stopping; W is one
+    window or one per shard), then the global top-k by (score desc, id asc)
+    merges the shards' results.  Returns dict(ids, scores, count, probes =
+    partitions searched over all shards, shard_probes [nq][nshards])."""
+    Ws = list(W) if isinstance(W, (list, tuple, np.ndarray)) else [W] * len(shards)
+    parts = [search(sh, Q, tau, k, nprobe, w, qids=qids, threads=threads) for sh, w in zip(shards, Ws)]
+    return _merge_shards(parts, k)

@@ -115,6 +115,10 @@ _SIGNATURES = {
                                          C.c_void_p, C.POINTER(ParamsC), C.c_void_p, C.c_void_p,
                                          C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
                                          C.c_void_p, C.c_size_t, C.c_void_p]),
+    "sieve_merge_shard_results": (C.c_int32, [C.c_int32, C.c_int64, C.c_int32, C.c_void_p,
+                                              C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+                                              C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+                                              C.c_void_p]),
     "sieve_status_str": (C.c_char_p, [C.c_int32]),
     "sieve_last_cuda_error": (C.c_int32, []),
     "sieve_version": (C.c_char_p, []),
@@ -435,6 +439,41 @@ def sharded_search(shards, Q, tau, k, nprobe, W, lookahead=True, query_ids=None,
                                       _ptr(shard_probes), _ptr(ws), ws.numel(), _stream(stream)),
            "sieve_sharded_search")
     return ids, scores, count, probes, shard_probes
+
+
+def sharded_calibrated_search(shards, Q, tau, k, nprobe, sample, eps, min_queries=10_000,
+                              fallback_W=8, lookahead=True, query_ids=None, scan_path="auto",
+                              workspace=None, stream=None):
+    """Every shard calibrates its own window on the same sample
+    (sieve_calibrated_search per shard, Appendix A), then the global top-k
+    (sieve_merge_shard_results).  Returns (ids, scores, count, probes,
+    shard_probes, Ws) with Ws the window each shard selected."""
+    nq, ns = Q.shape[0], len(shards)
+    dev = Q.device
+    ids = torch.empty((ns, nq, k), dtype=torch.int64, device=dev)
+    scores = torch.empty((ns, nq, k), dtype=torch.float32, device=dev)
+    count = torch.empty((ns, nq), dtype=torch.int32, device=dev)
+    probes = torch.empty((ns, nq), dtype=torch.int32, device=dev)
+    Ws = []
+    for s, sh in enumerate(shards):
+        out = calibrated_search(sh, Q, tau, k, nprobe, sample, eps, min_queries=min_queries,
+                                fallback_W=fallback_W, lookahead=lookahead, query_ids=query_ids,
+                                scan_path=scan_path, workspace=workspace, stream=stream)
+        ids[s].copy_(out[0])
+        scores[s].copy_(out[1])
+        count[s].copy_(out[2])
+        probes[s].copy_(out[3])
+        Ws.append(out[4]["W"])
+    o_ids = torch.empty((nq, k), dtype=torch.int64, device=dev)
+    o_sc = torch.empty((nq, k), dtype=torch.float32, device=dev)
+    o_cnt = torch.empty(nq, dtype=torch.int32, device=dev)
+    o_pr = torch.empty(nq, dtype=torch.int32, device=dev)
+    o_sp = torch.empty((nq, ns), dtype=torch.int32, device=dev)
+    _check(lib().sieve_merge_shard_results(ns, nq, k, _ptr(ids), _ptr(scores), _ptr(count),
+                                           _ptr(probes), _ptr(o_ids), _ptr(o_sc), _ptr(o_cnt),
+                                           _ptr(o_pr), _ptr(o_sp), _stream(stream)),
+           "sieve_merge_shard_results")
+    return o_ids, o_sc, o_cnt, o_pr, o_sp, Ws
 
 
 def search_host(index: Index, Q_host, tau, k, nprobe, W, lookahead=True, query_ids_host=None,

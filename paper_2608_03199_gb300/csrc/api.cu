@@ -879,6 +879,24 @@ sieve_status sieve_sharded_search(const sieve_index_view *shards, int32_t nshard
     return SIEVE_OK;
 }
 
+sieve_status sieve_merge_shard_results(int32_t nshards, int64_t nq, int32_t k,
+                                       const int64_t *ids, const float *scores,
+                                       const int32_t *count, const int32_t *probes,
+                                       int64_t *out_ids, float *out_scores, int32_t *out_count,
+                                       int32_t *out_probes, int32_t *shard_probes, void *stream) {
+    if (nshards < 1 || nq < 0 || k < 1 || k > kMaxK) return SIEVE_EINVAL;
+    if (nq > 0 && (!ids || !scores || !count || !probes || !out_ids || !out_scores || !out_count ||
+                   !out_probes))
+        return SIEVE_EINVAL;
+    sieve_status rc = check_device();
+    if (rc != SIEVE_OK) return rc;
+    SIEVE_CUDA(launch_merge_shards(nshards, nq, k, reinterpret_cast<const long long *>(ids), scores,
+                                   count, probes, reinterpret_cast<long long *>(out_ids), out_scores,
+                                   out_count, out_probes, shard_probes,
+                                   static_cast<cudaStream_t>(stream)));
+    return SIEVE_OK;
+}
+
 }  // extern "C"
 
 // ---------------------------------------------------------------------------

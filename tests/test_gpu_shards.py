@@ -47,3 +47,21 @@ def test_sharded_search_matches_oracle(sharded, W):
     valid = got[0] >= 0
     assert np.abs(got[1][valid] - ref["scores"][valid]).max(initial=0) <= TOL
     assert np.isneginf(got[1][~valid]).all()
+
+
+def test_per_shard_calibration_matches_oracle(sharded):
+    cfg, host, gshards, Q, qids, dev = sharded
+    sample = np.sort(np.random.default_rng(8).choice(len(Q), 60, replace=False)).astype(np.int64)
+    out = sieve.sharded_calibrated_search(gshards, torch.from_numpy(Q).to(dev), cfg.tau, cfg.k,
+                                          cfg.nprobe, torch.from_numpy(sample).to(dev), 0.02,
+                                          min_queries=0, query_ids=torch.from_numpy(qids).to(dev))
+    torch.cuda.synchronize()
+    ref = oracle.sharded_calibrated_search(host, Q, sample, cfg.tau, cfg.k, cfg.nprobe, 0.02,
+                                           min_queries=0, qids=qids)
+    assert out[5] == ref["Ws"]
+    got = [o.cpu().numpy() for o in out[:5]]
+    assert np.array_equal(got[4], ref["shard_probes"])
+    assert np.array_equal(got[2], ref["count"])
+    assert np.array_equal(got[0], ref["ids"])
+    valid = got[0] >= 0
+    assert np.abs(got[1][valid] - ref["scores"][valid]).max(initial=0) <= TOL

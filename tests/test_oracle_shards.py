@@ -61,3 +61,20 @@ def test_per_shard_windows(sharded):
     # a larger window per shard never keeps fewer results
     b = oracle.sharded_search(shards, Q, cfg.tau, cfg.k, cfg.nprobe, 8, qids=qids)
     assert (b["count"] >= a["count"]).all()
+
+
+def test_per_shard_calibration(sharded):
+    """Each shard calibrates on the same sample: its window equals a separate
+    calibration of that shard alone, and the merge equals the sharded search
+    run with those windows except on the sampled rows (fixed-probe results)."""
+    cfg, shards, Q, qids = sharded
+    sample = np.sort(np.random.default_rng(8).choice(len(Q), 60, replace=False)).astype(np.int64)
+    res = oracle.sharded_calibrated_search(shards, Q, sample, cfg.tau, cfg.k, cfg.nprobe, 0.02,
+                                           min_queries=0, qids=qids)
+    for sh, W in zip(shards, res["Ws"]):
+        assert W == oracle.calibrate(sh, Q, sample, cfg.tau, cfg.k, cfg.nprobe, 0.02,
+                                     min_queries=0, qids=qids)["W"]
+    rest = np.setdiff1d(np.arange(len(Q)), sample)
+    plain = oracle.sharded_search(shards, Q, cfg.tau, cfg.k, cfg.nprobe, res["Ws"], qids=qids)
+    assert np.array_equal(res["ids"][rest], plain["ids"][rest])
+    assert (res["shard_probes"][sample] == cfg.nprobe).all()
