@@ -328,6 +328,44 @@ __device__ __forceinline__ void warp_gather_sort(const uint32_t (&key)[KPL], int
         bc[p] = INT32_MAX;
     }
     __syncwarp();
+    if (S <= 64) {
+        // bitonic sort in registers: entry i = r * 32 + lane in register r;
+        // partners across lanes by shuffles, across registers (j = 32) in place
+        const float ninf = -__int_as_float(0x7f800000);
+        float s0 = lane < S ? bs[lane] : ninf, s1 = lane + 32 < S ? bs[lane + 32] : ninf;
+        int c0 = lane < S ? bc[lane] : INT32_MAX, c1 = lane + 32 < S ? bc[lane + 32] : INT32_MAX;
+        for (int k = 2; k <= S; k <<= 1) {
+            for (int j = k >> 1; j > 0; j >>= 1) {
+                if (j == 32) {   // k == 64: entry lane (kept better) against lane + 32
+                    if (ranks_before(s1, c1, s0, c0)) {
+                        const float ts = s0;
+                        const int tc = c0;
+                        s0 = s1;
+                        c0 = c1;
+                        s1 = ts;
+                        c1 = tc;
+                    }
+                    continue;
+                }
+                const float ps0 = __shfl_xor_sync(0xffffffffu, s0, j);
+                const int pc0 = __shfl_xor_sync(0xffffffffu, c0, j);
+                const float ps1 = __shfl_xor_sync(0xffffffffu, s1, j);
+                const int pc1 = __shfl_xor_sync(0xffffffffu, c1, j);
+                const bool lower = (lane & j) == 0;
+                // the lower entry of a pair keeps the better one when its
+                // block sorts first-ranked first ((i & k) == 0), else the worse
+                const bool take0 = (lower == ((lane & k) == 0)) == ranks_before(ps0, pc0, s0, c0);
+                const bool take1 = (lower == (((lane + 32) & k) == 0)) == ranks_before(ps1, pc1, s1, c1);
+                if (take0) { s0 = ps0; c0 = pc0; }
+                if (take1) { s1 = ps1; c1 = pc1; }
+            }
+        }
+        __syncwarp();
+        if (lane < S) { bs[lane] = s0; bc[lane] = c0; }
+        if (lane + 32 < S) { bs[lane + 32] = s1; bc[lane + 32] = c1; }
+        __syncwarp();
+        return;
+    }
     // bitonic sort of S entries, first-ranked first
     for (int k = 2; k <= S; k <<= 1) {
         for (int j = k >> 1; j > 0; j >>= 1) {
