@@ -44,7 +44,7 @@ def build(force: bool = False) -> str:
             and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
         return _LIB_PATH
     tmp = _LIB_PATH + f".tmp{os.getpid()}"
-    cmd = ["gcc", "-std=c11", "-O2", "-fopenmp", "-fPIC", "-shared",
+    cmd = ["gcc", "-std=c11", "-O2", "-ffp-contract=off", "-fopenmp", "-fPIC", "-shared",
            "-o", tmp, _SRC, "-lm"]
     subprocess.run(cmd, check=True)
     os.replace(tmp, _LIB_PATH)
@@ -66,11 +66,14 @@ def _declare(lib):
     lib.oracle_bruteforce.argtypes = [P, P, I64, I32, P, I64, P, F32, I32, P, P, P, I32]
     lib.oracle_fragility.argtypes = [P, P, P, I64, I32, P, I64, P, I64, P, P, P, F32, I32,
                                      I32, P, P, P, I32]
+    lib.oracle_rq_encode.argtypes = [P, P, I64, I32, P, I64, P, I32, P, P, I32]
+    lib.oracle_rq_search.argtypes = [P, P, P, I64, I32, P, I64, P, P, P, I32, P, I64, P, P, F32,
+                                     I32, I32, I64, I32, U64, P, P, P, P, I32]
     lib.oracle_calibrate.argtypes = [P, P, P, I64, I32, P, I64, P, I64, P, P, I64, F32, I32,
                                      I32, C.c_double, I64, I64, P, P, P, P, P, P, P, I32]
     for name in ("oracle_rank", "oracle_stop_pattern", "oracle_search", "oracle_hit_matrix",
                  "oracle_fixed_probe", "oracle_bruteforce", "oracle_fragility",
-                 "oracle_calibrate"):
+                 "oracle_calibrate", "oracle_rq_encode", "oracle_rq_search"):
         getattr(lib, name).restype = C.c_int
     return lib
 
@@ -315,3 +318,42 @@ def sharded_search(shards, Q, tau, k, nprobe, W, qids=None, threads=None):
     Ws = list(W) if isinstance(W, (list, tuple, np.ndarray)) else [W] * len(shards)
     parts = [search(sh, Q, tau, k, nprobe, w, qids=qids, threads=threads) for sh, w in zip(shards, Ws)]
     return _merge_shards(parts, k)
+
+
+def rq_encode(index, P, bits=7, threads=None):
+    """RaBitQ-style codes of the rows (oracle_rq_encode): codes [n][d] uint8,
+    factors [n] float32, for the rotation P [d][d] (float64, orthogonal)."""
+    lib = _load()
+    X, assign, Cent = (_c(index["X"], np.float32), _c(index["assign"], np.int32),
+                       _c(index["centroids"], np.float32))
+    P = _c(P, np.float64)
+    n, d = X.shape
+    codes = np.empty((n, d), np.uint8)
+    factors = np.empty(n, np.float32)
+    _check(lib.oracle_rq_encode(_p(X), _p(assign), n, d, _p(Cent), Cent.shape[0], _p(P), bits,
+                                _p(codes), _p(factors), threads or default_threads()),
+           "oracle_rq_encode")
+    return codes, factors
+
+
+def rq_search(index, codes, factors, P, Q, tau, k, nprobe, W, bits=7, qids=None, order=None,
+              mode="sequential", seed=0, threads=None):
+    """search() with the quantized local search on the given codes."""
+    lib = _load()
+    X, ids, assign, Cent = (_c(index["X"], np.float32), _c(index["ids"], np.int64),
+                            _c(index["assign"], np.int32), _c(index["centroids"], np.float32))
+    codes, factors, P = _c(codes, np.uint8), _c(factors, np.float32), _c(P, np.float64)
+    Q = _c(Q, np.float32)
+    nq, d = Q.shape
+    qids = None if qids is None else _c(qids, np.int64)
+    order = None if order is None else _c(order, np.int32)
+    out_ids = np.empty((nq, k), np.int64)
+    out_sc = np.empty((nq, k), np.float64)
+    cnt = np.empty(nq, np.int32)
+    probes = np.empty(nq, np.int32)
+    rc = lib.oracle_rq_search(_p(X), _p(ids), _p(assign), X.shape[0], d, _p(Cent), Cent.shape[0],
+                              _p(codes), _p(factors), _p(P), bits, _p(Q), nq, _p(qids), _p(order),
+                              float(tau), k, nprobe, int(W), _MODES[mode], seed, _p(out_ids),
+                              _p(out_sc), _p(cnt), _p(probes), threads or default_threads())
+    _check(rc, "oracle_rq_search")
+    return {"ids": out_ids, "scores": out_sc, "count": cnt, "probes": probes}

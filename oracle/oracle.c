@@ -278,6 +278,11 @@ typedef struct {
     const int64_t *ids;
     const lists_t *L;
     int d;
+    /* quantized local search (NULL codes: exact inner products) */
+    const uint8_t *codes;   /* [n][d] RaBitQ-style codes of the rows */
+    const float *factors;   /* [n] per-row factor f */
+    const float *C;         /* [nlist][d] centroids */
+    double mid;             /* (2^bits - 1) / 2 */
 } index_t;
 
 static int local_search(const index_t *ix, const float *q, int has_qid, int64_t qid, int32_t p,
@@ -299,6 +304,36 @@ static int local_search(const index_t *ix, const float *q, int has_qid, int64_t 
     return hit;
 }
 
+/* The same local search on RaBitQ-style codes (the paper's IVF_RQ7 local  */
+/* search, Sec. 3.1 and Sec. 6.1): the estimate of <q, x> for a row x of    */
+/* partition p with codes u and factor f is                                   */
+/*     <q, c_p> + f * (<u, q'> - mid * sum_i q'_i),   q' = P^T q,             */
+/* the estimator of oracle_rq_encode's header.                                */
+static int rq_local_search(const index_t *ix, const float *q, const double *qrot, double sq,
+                           int has_qid, int64_t qid, int32_t p, double tau, topk_t *local)
+{
+    const int d = ix->d;
+    const double qc = sim64(q, ix->C + (int64_t)p * d, d);
+    int hit = 0;
+    local->n = 0;
+    for (int64_t r = ix->L->start[p]; r < ix->L->start[p + 1]; ++r) {
+        int64_t row = ix->L->rows[r];
+        int64_t id = ix->ids[row];
+        if (has_qid && id == qid)
+            continue;
+        const uint8_t *u = ix->codes + row * (int64_t)d;
+        double dot = 0.0;
+        for (int t = 0; t < d; ++t)
+            dot += (double)u[t] * qrot[t];
+        double s = qc + (double)ix->factors[row] * (dot - ix->mid * sq);
+        if (s >= tau) {
+            hit = 1;
+            topk_offer(local, s, id);
+        }
+    }
+    return hit;
+}
+
 /* per-query state for one search (the "results" of Table 2 kept per rank) */
 typedef struct {
     const index_t *ix;
@@ -310,13 +345,19 @@ typedef struct {
     int k;
     cand_t *local_store;  /* [nprobe][k] */
     int *local_n;         /* [nprobe] entries kept per rank, -1 = not searched */
+    const double *qrot;   /* quantized search: P^T q, and its coordinate sum */
+    double sq;
 } query_ctx_t;
 
 static int search_probe(void *vctx, int rank)
 {
     query_ctx_t *c = (query_ctx_t *)vctx;
     topk_t local = {c->k, 0, c->local_store + (int64_t)(rank - 1) * c->k};
-    int hit = local_search(c->ix, c->q, c->has_qid, c->qid, c->order[rank - 1], c->tau, &local);
+    int hit = c->ix->codes
+                  ? rq_local_search(c->ix, c->q, c->qrot, c->sq, c->has_qid, c->qid,
+                                    c->order[rank - 1], c->tau, &local)
+                  : local_search(c->ix, c->q, c->has_qid, c->qid, c->order[rank - 1], c->tau,
+                                 &local);
     c->local_n[rank - 1] = local.n;
     return hit;
 }
@@ -333,11 +374,52 @@ static int search_probe(void *vctx, int rank)
  * Returns 0, or <0 on bad arguments; returns -3 if the lookahead form ever
  * searched a rank twice or skipped a rank below its stop line.
  */
+typedef struct {
+    const uint8_t *codes;
+    const float *factors;
+    const double *P;   /* [d][d] rotation */
+    int bits;
+} rq_in_t;
+
+static int search_impl(const float *X, const int64_t *ids, const int32_t *assign, int64_t n,
+                       int32_t d, const float *C, int64_t nlist, const float *Q, int64_t nq,
+                       const int64_t *qids, const int32_t *order_in, float tau, int32_t k,
+                       int32_t nprobe, int64_t W, int32_t mode, uint64_t seed, int64_t *out_ids,
+                       double *out_scores, int32_t *out_count, int32_t *out_probes,
+                       int32_t nthreads, const rq_in_t *rq);
+
 int oracle_search(const float *X, const int64_t *ids, const int32_t *assign, int64_t n, int32_t d,
                   const float *C, int64_t nlist, const float *Q, int64_t nq, const int64_t *qids,
                   const int32_t *order_in, float tau, int32_t k, int32_t nprobe, int64_t W,
                   int32_t mode, uint64_t seed, int64_t *out_ids, double *out_scores,
                   int32_t *out_count, int32_t *out_probes, int32_t nthreads)
+{
+    return search_impl(X, ids, assign, n, d, C, nlist, Q, nq, qids, order_in, tau, k, nprobe, W,
+                       mode, seed, out_ids, out_scores, out_count, out_probes, nthreads, NULL);
+}
+
+/* oracle_search with the quantized local search of rq_local_search: codes
+ * [n][d], factors [n] as made by oracle_rq_encode with the same rotation P. */
+int oracle_rq_search(const float *X, const int64_t *ids, const int32_t *assign, int64_t n,
+                     int32_t d, const float *C, int64_t nlist, const uint8_t *codes,
+                     const float *factors, const double *P, int32_t bits, const float *Q,
+                     int64_t nq, const int64_t *qids, const int32_t *order_in, float tau, int32_t k,
+                     int32_t nprobe, int64_t W, int32_t mode, uint64_t seed, int64_t *out_ids,
+                     double *out_scores, int32_t *out_count, int32_t *out_probes, int32_t nthreads)
+{
+    if (!codes || !factors || !P || bits < 1 || bits > 8)
+        return -1;
+    rq_in_t rq = {codes, factors, P, bits};
+    return search_impl(X, ids, assign, n, d, C, nlist, Q, nq, qids, order_in, tau, k, nprobe, W,
+                       mode, seed, out_ids, out_scores, out_count, out_probes, nthreads, &rq);
+}
+
+static int search_impl(const float *X, const int64_t *ids, const int32_t *assign, int64_t n,
+                       int32_t d, const float *C, int64_t nlist, const float *Q, int64_t nq,
+                       const int64_t *qids, const int32_t *order_in, float tau, int32_t k,
+                       int32_t nprobe, int64_t W, int32_t mode, uint64_t seed, int64_t *out_ids,
+                       double *out_scores, int32_t *out_count, int32_t *out_probes,
+                       int32_t nthreads, const rq_in_t *rq)
 {
     if (d <= 0 || k < 1 || nprobe < 1 || nprobe > nlist || W < 1 || isnan(tau))
         return -1;
@@ -346,7 +428,12 @@ int oracle_search(const float *X, const int64_t *ids, const int32_t *assign, int
         lists_free(&L);
         return -2;
     }
-    index_t ix = {X, ids, &L, d};
+    index_t ix = {X, ids, &L, d, NULL, NULL, C, 0.0};
+    if (rq) {
+        ix.codes = rq->codes;
+        ix.factors = rq->factors;
+        ix.mid = ((double)(1 << rq->bits) - 1.0) / 2.0;
+    }
     int bad = 0;
 #pragma omp parallel num_threads(nthreads > 0 ? nthreads : 1)
     {
@@ -357,7 +444,8 @@ int oracle_search(const float *X, const int64_t *ids, const int32_t *assign, int
         int *pending = (int *)malloc((size_t)(nprobe + 1) * sizeof(int));
         int *visits = (int *)malloc((size_t)(nprobe + 1) * sizeof(int));
         cand_t *fin = (cand_t *)malloc((size_t)k * sizeof(cand_t));
-        if (!scratch || !order || !store || !local_n || !pending || !visits || !fin) {
+        double *qrot = (double *)malloc((size_t)d * sizeof(double));
+        if (!scratch || !order || !store || !local_n || !pending || !visits || !fin || !qrot) {
 #pragma omp atomic write
             bad = -2;
         } else {
@@ -371,8 +459,18 @@ int oracle_search(const float *X, const int64_t *ids, const int32_t *assign, int
                     rank_one(q, C, nlist, d, nprobe, scratch, order, NULL);
                 for (int j = 0; j < nprobe; ++j)
                     local_n[j] = -1;
+                double sq = 0.0;
+                if (rq) {   /* q' = P^T q and its coordinate sum */
+                    for (int t = 0; t < d; ++t) {
+                        double acc = 0.0;
+                        for (int j = 0; j < d; ++j)
+                            acc += rq->P[(int64_t)j * d + t] * (double)q[j];
+                        qrot[t] = acc;
+                        sq += acc;
+                    }
+                }
                 query_ctx_t ctx = {&ix, q, qids != NULL, qids ? qids[i] : 0, P, (double)tau,
-                                   k, store, local_n};
+                                   k, store, local_n, qrot, sq};
                 int probes;
                 if (mode == 0) {
                     probes = stop_sequential(nprobe, W, search_probe, &ctx);
@@ -401,7 +499,7 @@ int oracle_search(const float *X, const int64_t *ids, const int32_t *assign, int
             }
         }
         free(scratch); free(order); free(store); free(local_n);
-        free(pending); free(visits); free(fin);
+        free(pending); free(visits); free(fin); free(qrot);
     }
     lists_free(&L);
     return bad;
@@ -423,7 +521,7 @@ int oracle_hit_matrix(const float *X, const int64_t *ids, const int32_t *assign,
         lists_free(&L);
         return -2;
     }
-    index_t ix = {X, ids, &L, d};
+    index_t ix = {X, ids, &L, d, NULL, NULL, NULL, 0.0};
 #pragma omp parallel for schedule(dynamic, 4) num_threads(nthreads > 0 ? nthreads : 1)
     for (int64_t i = 0; i < nq; ++i) {
         cand_t one;
@@ -628,7 +726,7 @@ int oracle_calibrate(const float *X, const int64_t *ids, const int32_t *assign, 
         lists_free(&L);
         return -2;
     }
-    index_t ix = {X, ids, &L, d};
+    index_t ix = {X, ids, &L, d, NULL, NULL, C, 0.0};
     int64_t Z = 0;
     int bad = 0;
     /* steps 2-4 for every sampled query */
@@ -751,4 +849,85 @@ int oracle_calibrate(const float *X, const int64_t *ids, const int32_t *assign, 
     }
     free(Qr); free(qr); free(idx); free(oi); free(os); free(oc); free(op);
     return rc;
+}
+
+
+/* ------------------------------------------------------------------------ */
+/* RaBitQ-style codes of the rows (the paper's IVF_RQ7, Sec. 3.1: RaBitQ     */
+/* configured with 7 bits), given a d x d orthogonal rotation P (row-major). */
+/* For a row x of partition p, with r = x - c_p:                             */
+/*   o  = r / |r|,  o' = P^T o   (o'_i = sum_j P[j][i] o_j)                   */
+/*   D  = 2 max_i |o'_i| / (2^bits - 1),  mid = (2^bits - 1) / 2             */
+/*   u_i = rint(o'_i / D + mid) clamped to [0, 2^bits - 1]  (the codes)      */
+/*   f  = |r| / <u - mid, o'>  (stored as fp32)                               */
+/* and the estimate of <q, x> is <q, c_p> + f (<u, q'> - mid sum_i q'_i),    */
+/* q' = P^T q: RaBitQ's estimator <o', q'> ~ <o_bar, q'> / <o_bar, o'> with   */
+/* o_bar the normalised code vector, scaled back by |r| and shifted by the   */
+/* centroid term.  A row equal to its centroid gets codes rint(mid), f = 0.  */
+/* Every sum runs in fp64 in index order with fused multiply-adds, so an     */
+/* implementation that does the same gets the same codes and factors.        */
+int oracle_rq_encode(const float *X, const int32_t *assign, int64_t n, int32_t d, const float *C,
+                     int64_t nlist, const double *P, int32_t bits, uint8_t *codes, float *factors,
+                     int32_t nthreads)
+{
+    if (d <= 0 || bits < 1 || bits > 8 || !P)
+        return -1;
+    const double top = (double)((1 << bits) - 1), mid = top / 2.0;
+    int bad = 0;
+#pragma omp parallel num_threads(nthreads > 0 ? nthreads : 1)
+    {
+        double *o = (double *)malloc((size_t)d * sizeof(double));
+        double *rot = (double *)malloc((size_t)d * sizeof(double));
+        if (!o || !rot) {
+#pragma omp atomic write
+            bad = -2;
+        } else {
+#pragma omp for schedule(static)
+            for (int64_t i = 0; i < n; ++i) {
+                const int32_t p = assign[i];
+                uint8_t *u = codes + i * (int64_t)d;
+                if (p < 0 || p >= nlist) {
+#pragma omp atomic write
+                    bad = -1;
+                    continue;
+                }
+                const float *x = X + i * (int64_t)d, *c = C + (int64_t)p * d;
+                double nn = 0.0;
+                for (int j = 0; j < d; ++j) {
+                    o[j] = (double)x[j] - (double)c[j];
+                    nn = fma(o[j], o[j], nn);
+                }
+                const double norm = sqrt(nn);
+                if (norm == 0.0) {
+                    for (int t = 0; t < d; ++t)
+                        u[t] = (uint8_t)rint(mid);
+                    factors[i] = 0.0f;
+                    continue;
+                }
+                for (int j = 0; j < d; ++j)
+                    o[j] = o[j] / norm;
+                double mx = 0.0;
+                for (int t = 0; t < d; ++t) {
+                    double acc = 0.0;
+                    for (int j = 0; j < d; ++j)
+                        acc = fma(P[(int64_t)j * d + t], o[j], acc);
+                    rot[t] = acc;
+                    if (fabs(acc) > mx)
+                        mx = fabs(acc);
+                }
+                const double delta = 2.0 * mx / top;
+                double dot = 0.0;
+                for (int t = 0; t < d; ++t) {
+                    double v = rint(rot[t] / delta + mid);
+                    v = v < 0.0 ? 0.0 : (v > top ? top : v);
+                    u[t] = (uint8_t)v;
+                    dot = fma(v - mid, rot[t], dot);
+                }
+                factors[i] = (float)(norm / dot);
+            }
+        }
+        free(o);
+        free(rot);
+    }
+    return bad;
 }

@@ -259,3 +259,15 @@ def make_sharded_workload(cfg: Workload | str, nshards: int, nlist_per_shard: in
         shards.append({"X": Xs, "ids": rows.to(torch.int64), "centroids": cent, "assign": assign})
     qrows = torch.randperm(cfg.n, generator=g, device=device)[:cfg.nq]
     return {"cfg": cfg, "Q": X[qrows].contiguous(), "qids": qrows.to(torch.int64), "shards": shards}
+
+
+def make_rotation(d: int, seed: int = 7):
+    """A seeded random orthogonal d x d matrix (float64, numpy): the rotation
+    the quantized local search draws (QR of a Gaussian matrix, signs fixed so
+    that R has a positive diagonal)."""
+    import numpy as np
+    g = torch.Generator(device="cpu").manual_seed(seed)
+    A = torch.randn(d, d, generator=g, dtype=torch.float64)
+    Qm, R = torch.linalg.qr(A)
+    Qm = Qm * torch.sign(torch.diagonal(R)).unsqueeze(0)
+    return np.ascontiguousarray(Qm.numpy())

@@ -14,21 +14,24 @@ import pytest
 
 import oracle
 import test_oracle_calibration as K
+import test_oracle_rq as R
 import test_oracle_search as S
 import test_oracle_stopping as T
 
 SRC = os.path.join(os.path.dirname(oracle.__file__), "oracle.c")
 
 MUTATIONS = [
-    ("tau test strict", "if (s >= tau) {", "if (s > tau) {"),
+    ("tau test strict", "ix->d);\n        if (s >= tau) {", "ix->d);\n        if (s > tau) {"),
     ("hit does not reset the run", "if (f(ctx, searched))\n            stale = 0;",
      "if (f(ctx, searched))\n            stale = stale;"),
     ("id tie-break reversed", "(sa == sb && ia < ib)", "(sa == sb && ia > ib)"),
     ("stop line one short", "int64_t reach = (int64_t)j + W;", "int64_t reach = (int64_t)j + W - 1;"),
-    ("first coordinate dropped", "for (int t = 0; t < d; ++t)", "for (int t = 1; t < d; ++t)"),
+    ("first coordinate dropped", "for (int t = 0; t < d; ++t)\n        acc += (double)a[t]",
+     "for (int t = 1; t < d; ++t)\n        acc += (double)a[t]"),
     ("centroid order reversed", "if (x->score > y->score) return -1;",
      "if (x->score > y->score) return 1;"),
-    ("self not excluded", "if (has_qid && id == qid)\n            continue;", ""),
+    ("self not excluded", "if (has_qid && id == qid)\n            continue;\n        double s = sim64",
+     "double s = sim64"),
     ("initial stop line 1", "int64_t s = W < nprobe ? W : nprobe;", "int64_t s = 1;"),
     ("merge drops last local entry", "m < (local_n[j] > 0 ? local_n[j] : 0)",
      "m + 1 < (local_n[j] > 0 ? local_n[j] : 0)"),
@@ -38,6 +41,16 @@ MUTATIONS = [
     ("empty run not reset by a hit", "run = local_n[j - 1] > 0 ? 0 : run + 1;",
      "run = local_n[j - 1] > 0 ? run : run + 1;"),
     ("loss target inclusive", "if (loss < eps) {", "if (loss <= eps) {"),
+    ("quantized estimate without the centroid term",
+     "double s = qc + (double)ix->factors[row] * (dot - ix->mid * sq);",
+     "double s = (double)ix->factors[row] * (dot - ix->mid * sq);"),
+    ("quantized estimate with the code offset added", "(dot - ix->mid * sq)", "(dot + ix->mid * sq)"),
+    ("codes from the untransposed rotation", "acc = fma(P[(int64_t)j * d + t], o[j], acc);",
+     "acc = fma(P[(int64_t)t * d + j], o[j], acc);"),
+    ("code step half as wide", "const double delta = 2.0 * mx / top;",
+     "const double delta = mx / top;"),
+    ("query rotated by the untransposed matrix", "acc += rq->P[(int64_t)j * d + t] * (double)q[j];",
+     "acc += rq->P[(int64_t)t * d + j] * (double)q[j];"),
 ]
 
 
@@ -55,6 +68,10 @@ def _pins(tiny, deep):
         lambda: K.test_calibration_matches_brute_force_loss(deep, 0.05),
         lambda: K.test_calibration_window_extremes_and_fallbacks(deep),
         K.test_calibration_histogram_of_gapped_hits,
+        R.test_grid_aligned_rows_are_estimated_exactly,
+        lambda: R.test_estimator_error_shrinks_with_bits_and_is_unbiased(tiny),
+        lambda: R.test_quantized_search_approaches_exact(deep),
+        lambda: R.test_rows_at_their_centroid_and_bounds(tiny),
     ]
 
 
@@ -65,7 +82,8 @@ def test_planted_mistake_is_caught(tmp_path, tiny, deep, name, old, new):
     mutated = tmp_path / "oracle_mut.c"
     mutated.write_text(src.replace(old, new))
     lib = tmp_path / "liboracle_mut.so"
-    subprocess.run(["gcc", "-std=c11", "-O2", "-fopenmp", "-fPIC", "-shared", "-o", str(lib),
+    subprocess.run(["gcc", "-std=c11", "-O2", "-ffp-contract=off", "-fopenmp", "-fPIC", "-shared",
+                    "-o", str(lib),
                     str(mutated), "-lm"], check=True)
     oracle.use_library(str(lib))
     failed = []
