@@ -63,7 +63,9 @@ def parse():
                     help="target CPU seconds for the oracle sample")
     ap.add_argument("--scan-path", choices=("auto", "simt", "tensor"), default="auto",
                     help="which units score the partition groups (sieve_params.scan_path)")
-    ap.add_argument("--ncu-case", choices=("w8", "fixed"), default=None,
+    ap.add_argument("--rq", action="store_true",
+                    help="the quantized local search (RaBitQ-style 7-bit codes) on the workload")
+    ap.add_argument("--ncu-case", choices=("w8", "fixed", "rqw8"), default=None,
                     help="run exactly one search (W = the config's W, or fixed probe) and exit: "
                          "a small, single-call target for an ncu capture")
     return ap.parse_args()
@@ -146,7 +148,7 @@ def measured_peaks():
 
 KERNEL_SOURCES = ("common.cuh", "search.cuh", "search_kernels.cu", "rank_kernel.cu",
                   "scan_tc.cu", "tcgen05.cuh", "tc_bulk.cuh", "tc_pipeline.cuh", "rank_tc.cu",
-                  "tc_layout.cu")
+                  "tc_layout.cu", "rq.cu")
 
 
 def kernel_source_sha():
@@ -176,7 +178,7 @@ def committed_traffic(kernel, workload, launches):
     return e["dram_bytes_per_search"] / max(1, launches)
 
 
-def roofline(prof, cfg, dev, bulk=True, rank_on_tensor=True):
+def roofline(prof, cfg, dev, bulk=True, rank_on_tensor=True, rq=False):
     """Roofline entry for the kernel with the largest share of the step.
     bulk: the index carries the tensor-core layout, so the tensor-core scan
     runs as k_scan_bulk (else k_scan_tc) and the ranking as k_rank_bulk;
@@ -192,12 +194,21 @@ def roofline(prof, cfg, dev, bulk=True, rank_on_tensor=True):
     d = cfg.d
     launches = max(1, kl[top])
     ms_per_launch = km[top] / launches
-    name = {"scan_tc": "k_scan_bulk" if bulk else "k_scan_tc"}.get(top, f"k_{top}")
+    name = {"scan_tc": "k_scan_rq" if rq else "k_scan_bulk" if bulk else "k_scan_tc"}.get(top, f"k_{top}")
     out = {"kernel": name, "launches": kl[top], "ms_per_launch": ms_per_launch}
     # fp16 dense peak: the measured bf16 cuBLAS peak (fp16 and bf16 share the
     # nominal 2.25 PFLOP/s rate); the burst figure, as the kernel is timed alone
     f16_tflops = peaks.get("bf16_tflops", 1889.4)
-    if top == "scan_tc":
+    if top == "scan_tc" and rq:
+        flops = 2.0 * d * prof["pairs_tc"]
+        ach = flops / launches / (ms_per_launch * 1e-3) / 1e12
+        out.update(bound="tensor", achieved=ach, peak=f16_tflops / 2, unit="TFLOP/s",
+                   frac=ach / (f16_tflops / 2),
+                   peak_source=(f"codes exact in fp16, queries split: two kind::f16 MMAs per "
+                                f"estimate; fp16 dense peak {f16_tflops:.0f} TFLOP/s = measured "
+                                f"bf16 cuBLAS burst (of measured), so the algorithmic peak is half"),
+                   tensor_pipe_tflops=2 * ach)
+    elif top == "scan_tc":
         flops = 2.0 * d * prof["pairs_tc"]
         ach = flops / launches / (ms_per_launch * 1e-3) / 1e12
         out.update(bound="tensor", achieved=ach, peak=f16_tflops / 3, unit="TFLOP/s",
@@ -625,6 +636,99 @@ def run_sharded(args, cfg):
     return 0
 
 
+def run_rq(args, cfg):
+    """The quantized local search (RaBitQ-style codes, the paper's IVF_RQ7)
+    on one workload: index build times, the search at the workload's W and
+    at fixed probing, the kept neighbours against the exact search, the
+    roofline of the scan over codes and the oracle's quantized search on a
+    bounded query sample.  One JSON line."""
+    import paper_2608_03199_gb300 as sieve
+    dev = torch.device("cuda:0")
+    sieve.lib()
+    wl = synth.make_workload(cfg, device=dev)
+    index = sieve.build_layout(wl["X"], wl["assign"], cfg.nlist, wl["centroids"])
+    Q, qids = wl["Q"], wl["qids"]
+    P_host = synth.make_rotation(cfg.d, seed=1234)
+    P = torch.from_numpy(P_host).to(dev)
+    torch.cuda.synchronize()
+    e0, e1, e2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+    e0.record()
+    codes, factors = sieve.rq_encode(index, P, 7)
+    e1.record()
+    rqi = sieve.build_rq_layout(index, P, 7, codes=codes, factors=factors)
+    e2.record()
+    torch.cuda.synchronize()
+    enc_ms, lay_ms = e0.elapsed_time(e1), e1.elapsed_time(e2)
+    ws = sieve.Workspace()
+    nq, k = cfg.nq, cfg.k
+    outs = (torch.empty((nq, k), dtype=torch.int64, device=dev),
+            torch.empty((nq, k), dtype=torch.float32, device=dev),
+            torch.empty(nq, dtype=torch.int32, device=dev),
+            torch.empty(nq, dtype=torch.int32, device=dev))
+
+    def step(W):
+        return lambda: sieve.rq_search(index, rqi, Q, cfg.tau, k, cfg.nprobe, W, query_ids=qids,
+                                       workspace=ws, out=outs)
+    clocks = ClockSampler(0)
+    clocks.start()
+    ms = time_steps(step(cfg.W), args.steps, args.warmup, 1, dev)
+    clock_rec = clocks.stop()
+    ms_fixed = time_steps(step(cfg.nprobe), max(3, args.steps // 5), 2, 1, dev)
+    prof = sieve.rq_search(index, rqi, Q, cfg.tau, k, cfg.nprobe, cfg.W, query_ids=qids,
+                           profile=True, workspace=ws)[4]
+    step(cfg.W)()
+    rq_ids = outs[0].cpu().numpy()
+    rq_cnt = outs[2].cpu().numpy()
+    mean_probes = float(outs[3].float().mean().item())
+    ex = sieve.search(index, Q, cfg.tau, k, cfg.nprobe, cfg.W, lookahead=True, query_ids=qids)
+    ex_ids, ex_cnt = ex[0].cpu().numpy(), ex[2].cpu().numpy()
+    kept = sum(len(set(rq_ids[i, :rq_cnt[i]]) & set(ex_ids[i, :ex_cnt[i]])) for i in range(nq))
+    line = {
+        "metric": METRIC + " (quantized local search)",
+        "value": nq / (ms * 1e-3), "unit": "queries/s", "n_gpus": 1, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "u8 codes (fp16 u - mid on the tensor cores), f32 queries",
+        "data": "synthetic",
+        "config": {"workload": workload_desc(cfg), "bits": 7, "rotation": "seeded Haar (QR)",
+                   "l2": "inputs larger than L2 (codes 0.51 GB streamed per step)"},
+        "index_build_ms": {"encode": enc_ms, "layout": lay_ms},
+        "fixed_probe": {"value": nq / (ms_fixed * 1e-3), "ms_per_step": ms_fixed, "W": cfg.nprobe},
+        "speedup_vs_fixed": ms_fixed / ms,
+        "mean_probes": mean_probes,
+        "kept_vs_exact": {"common": kept, "exact": int(ex_cnt.sum()), "quantized": int(rq_cnt.sum())},
+        "roofline": roofline(prof, cfg, dev, bulk=True, rq=True),
+        "profile": {"kernel_ms": prof["kernel_ms"], "kernel_launches": prof["kernel_launches"],
+                    "rounds": prof["rounds"], "items": prof["items"], "pairs": prof["pairs"]},
+        "gpu_launches": args.steps * int(sum(prof["kernel_launches"].values())),
+        "clocks": clock_rec,
+    }
+    if not args.skip_cpu_baseline:
+        import oracle
+        w = host_arrays(wl)
+        idx = {kk: w[kk] for kk in ("X", "ids", "assign", "centroids")}
+        threads = oracle.default_threads()
+        t0 = time.perf_counter()
+        hc, hf = oracle.rq_encode(idx, P_host, 7, threads=threads)
+        enc_s = time.perf_counter() - t0
+        probe = min(nq, 64)
+        t0 = time.perf_counter()
+        oracle.rq_search(idx, hc, hf, P_host, w["Q"][:probe], cfg.tau, k, cfg.nprobe, cfg.W,
+                         qids=w["qids"][:probe], threads=threads)
+        per_q = (time.perf_counter() - t0) / probe
+        sample = int(min(nq, max(probe, args.cpu_seconds / max(per_q, 1e-9))))
+        t0 = time.perf_counter()
+        oracle.rq_search(idx, hc, hf, P_host, w["Q"][:sample], cfg.tau, k, cfg.nprobe, cfg.W,
+                         qids=w["qids"][:sample], threads=threads)
+        dt = time.perf_counter() - t0
+        line["cpu_baseline"] = {"value": sample / dt, "unit": "queries/s", "cores": threads,
+                                "kind": "oracle",
+                                "sample": f"first {sample:,} of the {nq:,} queries, W={cfg.W}, "
+                                          f"{dt:.1f} s on {threads} host threads (encoding the "
+                                          f"index took {enc_s:.1f} s more)"}
+    print(json.dumps(line))
+    return 0
+
+
 def run_ncu_case(args, cfg):
     """One search call on the benchmark workload, nothing else on the GPU after it."""
     import paper_2608_03199_gb300 as sieve
@@ -632,11 +736,17 @@ def run_ncu_case(args, cfg):
     sieve.lib()
     wl = synth.make_workload(cfg, device=dev)
     index = sieve.build_layout(wl["X"], wl["assign"], cfg.nlist, wl["centroids"])
-    W = cfg.W if args.ncu_case == "w8" else cfg.nprobe
+    W = cfg.nprobe if args.ncu_case == "fixed" else cfg.W
     # host-driven rounds: ncu does not profile kernels inside a CUDA graph with
     # conditional nodes; the kernels and their arguments are the same
-    out = sieve.search(index, wl["Q"], cfg.tau, cfg.k, cfg.nprobe, W, lookahead=True,
-                       query_ids=wl["qids"], stats=True, loop=1, scan_path=args.scan_path)
+    if args.ncu_case == "rqw8":
+        P = torch.from_numpy(synth.make_rotation(cfg.d, seed=1234)).to(dev)
+        rqi = sieve.build_rq_layout(index, P, 7)
+        out = sieve.rq_search(index, rqi, wl["Q"], cfg.tau, cfg.k, cfg.nprobe, W,
+                              query_ids=wl["qids"], stats=True, loop=1)
+    else:
+        out = sieve.search(index, wl["Q"], cfg.tau, cfg.k, cfg.nprobe, W, lookahead=True,
+                           query_ids=wl["qids"], stats=True, loop=1, scan_path=args.scan_path)
     print(json.dumps({"ncu_case": args.ncu_case, "W": W, "rounds": out[4]["rounds"],
                       "items": out[4]["items"], "pairs": out[4]["pairs"]}))
     return 0
@@ -650,6 +760,8 @@ def main():
         return run_ncu_case(args, cfg)
     if args.sweep:
         return run_sweep(args, cfg)
+    if args.rq:
+        return run_rq(args, cfg)
     if args.shards:
         return run_sharded(args, cfg)
     if args.impl == "reference":

@@ -122,7 +122,8 @@ typedef struct {
  * centroid ranking, state initialisation, the issuer, the ready-queue
  * bucketing, the scatter into partition groups, the grouped scan with its
  * fused epilogue on FP32 FMA, the per-query merge, the end-of-round step,
- * finalisation, and the grouped scan on the tensor cores. */
+ * finalisation, the grouped scan on the tensor cores, and the query rotation
+ * of the quantized search (sieve_rq_search). */
 enum {
     SIEVE_K_RANK = 0,
     SIEVE_K_INIT,
@@ -134,6 +135,7 @@ enum {
     SIEVE_K_ROUND_END,
     SIEVE_K_FINALIZE,
     SIEVE_K_SCAN_TC,
+    SIEVE_K_RQ_ROTATE,
     SIEVE_NKERNELS
 };
 
@@ -350,6 +352,80 @@ sieve_status sieve_merge_shard_results(int32_t nshards, int64_t nq, int32_t k,
                                        const int32_t *count, const int32_t *probes,
                                        int64_t *out_ids, float *out_scores, int32_t *out_count,
                                        int32_t *out_probes, int32_t *shard_probes, void *stream);
+
+/* ---------------------------------------------------------------------
+ * Quantized local search over RaBitQ-style codes (the paper's IVF_RQ7
+ * index: RaBitQ configured with 7 bits, Sec. 3.1; the local search of
+ * Sec. 6.1).  For a row x of partition p, with r = x - c_p and a d x d
+ * orthogonal rotation P (row-major, fp64):
+ *   o = r / |r|,  o' = P^T o,  D = 2 max_i |o'_i| / (2^bits - 1),
+ *   mid = (2^bits - 1) / 2,
+ *   u_i = rint(o'_i / D + mid) clamped to [0, 2^bits - 1]   (the codes)
+ *   f   = |r| / <u - mid, o'>                                 (the factor)
+ * and the search replaces sim(q, x) by the estimate
+ *   <q, c_p> + f <u - mid, q'>,   q' = P^T q,
+ * RaBitQ's estimator <o', q'> ~ <o_bar, q'> / <o_bar, o'> (o_bar the
+ * normalised code vector) scaled by |r| and shifted by the centroid term.
+ * Everything else (ranking, tau, the W-rule, rounds, MergeTopK) is
+ * sieve_search's.  These calls need d <= 256 and bits in 1..8.
+ * ------------------------------------------------------------------- */
+
+/* Codes and factors of the index's rows (in the view's row order), each
+ * row against the centroid of the partition that holds it.
+ *   P        device [d][d] fp64, orthogonal (not checked)
+ *   codes    device [n][d] uint8 out;  factors device [n] fp32 out
+ * Every sum runs in fp64 in index order with fused multiply-adds; divisions
+ * and square roots are correctly rounded, so the codes are a deterministic
+ * function of the rows.  A row equal to its centroid gets codes rint(mid)
+ * and factor 0.  Asynchronous on `stream`. */
+sieve_status sieve_rq_encode(const sieve_index_view *ix, const double *P, int32_t bits,
+                             uint8_t *codes, float *factors, void *stream);
+
+/* The scan's layout of the codes (derived data, as sieve_build_tc_layout):
+ *   rq_rows        per block of 128 rows of a partition and K-block of 64
+ *                  elements, 16 KB of fp16 (u - mid) in the byte order of the
+ *                  shared-memory operand tile (2 bytes per element)
+ *   rq_row_blocks  device [nlist+1] int64, block offsets of the partitions
+ *   rq_factors     device [blocks * 128] fp32: the factors in the same block
+ *                  order, 0 on the padding rows
+ *   rq_rotation    the tensor-core layout of P^T (P rounded to fp32), used to
+ *                  rotate the queries
+ * sieve_rq_layout_size reads list_offsets from the device (synchronous);
+ * sieve_build_rq_layout is asynchronous on `stream`.  Outputs 256-byte
+ * aligned; codes / factors as made by sieve_rq_encode with the same P. */
+sieve_status sieve_rq_layout_size(const sieve_index_view *ix, size_t *rows_bytes,
+                                  size_t *factors_bytes, size_t *rotation_bytes);
+sieve_status sieve_build_rq_layout(const sieve_index_view *ix, const uint8_t *codes,
+                                   const float *factors, int32_t bits, const double *P,
+                                   void *rq_rows, int64_t *rq_row_blocks, float *rq_factors,
+                                   void *rq_rotation, void *stream);
+
+/* The quantized index beside an index view (borrowed, read-only). */
+typedef struct {
+    int32_t bits;
+    int32_t reserved0;
+    const void *rq_rows;
+    const int64_t *rq_row_blocks;
+    const float *rq_factors;
+    const void *rq_rotation;
+} sieve_rq_view;
+
+/* sieve_search with the quantized local search: a row qualifies iff its
+ * estimate >= tau, and results carry estimates as scores.  The centroid
+ * term <q, c_p> is the ranking's score of p: with order == NULL the call
+ * ranks (and keeps the scores in the workspace); with a precomputed order,
+ * cscores (device [nq][nprobe] fp32, the scores sieve_rank_partitions
+ * returns beside it) is required.  Every group runs on the tensor cores
+ * (scan_path 1 is SIEVE_EINVAL); ix->tc_rows is not used.  Profiling reports
+ * the query rotation under SIEVE_K_RQ_ROTATE.  ws: at least
+ * sieve_rq_search_workspace_size bytes, 256-byte aligned. */
+sieve_status sieve_rq_search_workspace_size(const sieve_index_view *ix, int64_t nq,
+                                            const sieve_params *p, size_t *bytes);
+sieve_status sieve_rq_search(const sieve_index_view *ix, const sieve_rq_view *rq, const float *Q,
+                             int64_t nq, const int64_t *query_ids, const int32_t *order,
+                             const float *cscores, const sieve_params *p, int64_t *out_ids,
+                             float *out_scores, int32_t *out_count, int32_t *out_probes,
+                             sieve_stats *stats, void *ws, size_t ws_bytes, void *stream);
 
 /* Human-readable name of a status code (static string). */
 const char *sieve_status_str(sieve_status s);

@@ -67,13 +67,16 @@ def _declare(lib):
     lib.oracle_fragility.argtypes = [P, P, P, I64, I32, P, I64, P, I64, P, P, P, F32, I32,
                                      I32, P, P, P, I32]
     lib.oracle_rq_encode.argtypes = [P, P, I64, I32, P, I64, P, I32, P, P, I32]
+    lib.oracle_rq_fragility.argtypes = [P, P, P, I64, I32, P, I64, P, P, P, I32, P, I64, P, P, P,
+                                        F32, I32, I32, P, P, P, I32]
     lib.oracle_rq_search.argtypes = [P, P, P, I64, I32, P, I64, P, P, P, I32, P, I64, P, P, F32,
                                      I32, I32, I64, I32, U64, P, P, P, P, I32]
     lib.oracle_calibrate.argtypes = [P, P, P, I64, I32, P, I64, P, I64, P, P, I64, F32, I32,
                                      I32, C.c_double, I64, I64, P, P, P, P, P, P, P, I32]
     for name in ("oracle_rank", "oracle_stop_pattern", "oracle_search", "oracle_hit_matrix",
                  "oracle_fixed_probe", "oracle_bruteforce", "oracle_fragility",
-                 "oracle_calibrate", "oracle_rq_encode", "oracle_rq_search"):
+                 "oracle_calibrate", "oracle_rq_encode", "oracle_rq_search",
+                 "oracle_rq_fragility"):
         getattr(lib, name).restype = C.c_int
     return lib
 
@@ -227,8 +230,10 @@ def bruteforce(X, ids, Q, tau, k, qids=None, threads=None):
     return {"ids": out_ids, "scores": out_sc, "count": cnt}
 
 
-def fragility(index, Q, tau, k, nprobe, order, upto, qids=None, threads=None):
-    """Per-query (tau_gap, kth_gap, cen_gap); see oracle_fragility in oracle.c."""
+def fragility(index, Q, tau, k, nprobe, order, upto, qids=None, threads=None, rq=None):
+    """Per-query (tau_gap, kth_gap, cen_gap); see oracle_fragility in oracle.c.
+    rq = (codes, factors, P, bits): the gaps of the quantized estimates
+    (oracle_rq_fragility)."""
     lib = _load()
     X, ids, assign, Cent = (_c(index["X"], np.float32), _c(index["ids"], np.int64),
                             _c(index["assign"], np.int32), _c(index["centroids"], np.float32))
@@ -240,10 +245,19 @@ def fragility(index, Q, tau, k, nprobe, order, upto, qids=None, threads=None):
     tg = np.empty(nq, np.float64)
     kg = np.empty(nq, np.float64)
     cg = np.empty(nq, np.float64)
-    _check(lib.oracle_fragility(_p(X), _p(ids), _p(assign), X.shape[0], d, _p(Cent),
-                                Cent.shape[0], _p(Q), nq, _p(qids), _p(order), _p(upto),
-                                float(tau), k, nprobe, _p(tg), _p(kg), _p(cg),
-                                threads or default_threads()), "oracle_fragility")
+    if rq is None:
+        _check(lib.oracle_fragility(_p(X), _p(ids), _p(assign), X.shape[0], d, _p(Cent),
+                                    Cent.shape[0], _p(Q), nq, _p(qids), _p(order), _p(upto),
+                                    float(tau), k, nprobe, _p(tg), _p(kg), _p(cg),
+                                    threads or default_threads()), "oracle_fragility")
+    else:
+        codes, factors, P, bits = rq
+        codes, factors, P = _c(codes, np.uint8), _c(factors, np.float32), _c(P, np.float64)
+        _check(lib.oracle_rq_fragility(_p(X), _p(ids), _p(assign), X.shape[0], d, _p(Cent),
+                                       Cent.shape[0], _p(codes), _p(factors), _p(P), int(bits),
+                                       _p(Q), nq, _p(qids), _p(order), _p(upto), float(tau), k,
+                                       nprobe, _p(tg), _p(kg), _p(cg),
+                                       threads or default_threads()), "oracle_rq_fragility")
     return tg, kg, cg
 
 

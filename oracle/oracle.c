@@ -309,6 +309,31 @@ static int local_search(const index_t *ix, const float *q, int has_qid, int64_t 
 /* partition p with codes u and factor f is                                   */
 /*     <q, c_p> + f * (<u, q'> - mid * sum_i q'_i),   q' = P^T q,             */
 /* the estimator of oracle_rq_encode's header.                                */
+/* the estimate for one row, given qc = <q, c_p> */
+static double rq_estimate(const index_t *ix, const double *qrot, double sq, double qc, int64_t row)
+{
+    const int d = ix->d;
+    const uint8_t *u = ix->codes + row * (int64_t)d;
+    double dot = 0.0;
+    for (int t = 0; t < d; ++t)
+        dot += (double)u[t] * qrot[t];
+    return qc + (double)ix->factors[row] * (dot - ix->mid * sq);
+}
+
+/* q' = P^T q and the sum of its coordinates */
+static double rq_rotate_query(const double *P, const float *q, int d, double *qrot)
+{
+    double sq = 0.0;
+    for (int t = 0; t < d; ++t) {
+        double acc = 0.0;
+        for (int j = 0; j < d; ++j)
+            acc += P[(int64_t)j * d + t] * (double)q[j];
+        qrot[t] = acc;
+        sq += acc;
+    }
+    return sq;
+}
+
 static int rq_local_search(const index_t *ix, const float *q, const double *qrot, double sq,
                            int has_qid, int64_t qid, int32_t p, double tau, topk_t *local)
 {
@@ -321,11 +346,7 @@ static int rq_local_search(const index_t *ix, const float *q, const double *qrot
         int64_t id = ix->ids[row];
         if (has_qid && id == qid)
             continue;
-        const uint8_t *u = ix->codes + row * (int64_t)d;
-        double dot = 0.0;
-        for (int t = 0; t < d; ++t)
-            dot += (double)u[t] * qrot[t];
-        double s = qc + (double)ix->factors[row] * (dot - ix->mid * sq);
+        double s = rq_estimate(ix, qrot, sq, qc, row);
         if (s >= tau) {
             hit = 1;
             topk_offer(local, s, id);
@@ -460,15 +481,8 @@ static int search_impl(const float *X, const int64_t *ids, const int32_t *assign
                 for (int j = 0; j < nprobe; ++j)
                     local_n[j] = -1;
                 double sq = 0.0;
-                if (rq) {   /* q' = P^T q and its coordinate sum */
-                    for (int t = 0; t < d; ++t) {
-                        double acc = 0.0;
-                        for (int j = 0; j < d; ++j)
-                            acc += rq->P[(int64_t)j * d + t] * (double)q[j];
-                        qrot[t] = acc;
-                        sq += acc;
-                    }
-                }
+                if (rq)   /* q' = P^T q and its coordinate sum */
+                    sq = rq_rotate_query(rq->P, q, d, qrot);
                 query_ctx_t ctx = {&ix, q, qids != NULL, qids ? qids[i] : 0, P, (double)tau,
                                    k, store, local_n, qrot, sq};
                 int probes;
@@ -623,11 +637,11 @@ int oracle_bruteforce(const float *X, const int64_t *ids, int64_t n, int32_t d, 
 /*                 (+inf when fewer than k+1 qualify)                         */
 /*   cen_gap[i]  = min gap between consecutive fp64 centroid scores among     */
 /*                 ranks 1..min(nprobe+1, nlist)                              */
-int oracle_fragility(const float *X, const int64_t *ids, const int32_t *assign, int64_t n,
-                     int32_t d, const float *C, int64_t nlist, const float *Q, int64_t nq,
-                     const int64_t *qids, const int32_t *order, const int32_t *upto, float tau,
-                     int32_t k, int32_t nprobe, double *tau_gap, double *kth_gap,
-                     double *cen_gap, int32_t nthreads)
+static int fragility_impl(const float *X, const int64_t *ids, const int32_t *assign, int64_t n,
+                          int32_t d, const float *C, int64_t nlist, const float *Q, int64_t nq,
+                          const int64_t *qids, const int32_t *order, const int32_t *upto,
+                          float tau, int32_t k, int32_t nprobe, double *tau_gap, double *kth_gap,
+                          double *cen_gap, int32_t nthreads, const rq_in_t *rq)
 {
     if (d <= 0 || k < 1 || nprobe < 1 || nprobe > nlist)
         return -1;
@@ -636,25 +650,35 @@ int oracle_fragility(const float *X, const int64_t *ids, const int32_t *assign, 
         lists_free(&L);
         return -2;
     }
+    index_t ix = {X, ids, &L, d, NULL, NULL, C, 0.0};
+    if (rq) {
+        ix.codes = rq->codes;
+        ix.factors = rq->factors;
+        ix.mid = ((double)(1 << rq->bits) - 1.0) / 2.0;
+    }
 #pragma omp parallel num_threads(nthreads > 0 ? nthreads : 1)
     {
         cand_t *fin = (cand_t *)malloc((size_t)(k + 1) * sizeof(cand_t));
         cscore_t *scratch = (cscore_t *)malloc((size_t)nlist * sizeof(cscore_t));
         int32_t *ord = (int32_t *)malloc((size_t)nprobe * sizeof(int32_t));
         double *cs = (double *)malloc((size_t)nlist * sizeof(double));
+        double *qrot = (double *)malloc((size_t)d * sizeof(double));
 #pragma omp for schedule(dynamic, 4)
         for (int64_t i = 0; i < nq; ++i) {
             const float *q = Q + i * (int64_t)d;
             topk_t t = {k + 1, 0, fin};
             double tg = INFINITY;
             int lim = upto[i] < nprobe ? upto[i] : nprobe;
+            const double sq = rq ? rq_rotate_query(rq->P, q, d, qrot) : 0.0;
             for (int j = 0; j < lim; ++j) {
                 int32_t p = order[i * (int64_t)nprobe + j];
+                const double qc = rq ? sim64(q, C + (int64_t)p * d, d) : 0.0;
                 for (int64_t r = L.start[p]; r < L.start[p + 1]; ++r) {
                     int64_t row = L.rows[r];
                     if (qids && ids[row] == qids[i])
                         continue;
-                    double s = sim64(q, X + row * (int64_t)d, d);
+                    double s = rq ? rq_estimate(&ix, qrot, sq, qc, row)
+                                  : sim64(q, X + row * (int64_t)d, d);
                     double g = fabs(s - (double)tau);
                     if (g < tg)
                         tg = g;
@@ -674,10 +698,36 @@ int oracle_fragility(const float *X, const int64_t *ids, const int32_t *assign, 
             }
             cen_gap[i] = cg;
         }
-        free(fin); free(scratch); free(ord); free(cs);
+        free(fin); free(scratch); free(ord); free(cs); free(qrot);
     }
     lists_free(&L);
     return 0;
+}
+
+int oracle_fragility(const float *X, const int64_t *ids, const int32_t *assign, int64_t n,
+                     int32_t d, const float *C, int64_t nlist, const float *Q, int64_t nq,
+                     const int64_t *qids, const int32_t *order, const int32_t *upto, float tau,
+                     int32_t k, int32_t nprobe, double *tau_gap, double *kth_gap,
+                     double *cen_gap, int32_t nthreads)
+{
+    return fragility_impl(X, ids, assign, n, d, C, nlist, Q, nq, qids, order, upto, tau, k, nprobe,
+                          tau_gap, kth_gap, cen_gap, nthreads, NULL);
+}
+
+/* oracle_fragility with the quantized estimates (codes and factors as for
+ * oracle_rq_search): the gaps of the estimates the quantized search decides on */
+int oracle_rq_fragility(const float *X, const int64_t *ids, const int32_t *assign, int64_t n,
+                        int32_t d, const float *C, int64_t nlist, const uint8_t *codes,
+                        const float *factors, const double *P, int32_t bits, const float *Q,
+                        int64_t nq, const int64_t *qids, const int32_t *order, const int32_t *upto,
+                        float tau, int32_t k, int32_t nprobe, double *tau_gap, double *kth_gap,
+                        double *cen_gap, int32_t nthreads)
+{
+    if (!codes || !factors || !P || bits < 1 || bits > 8)
+        return -1;
+    rq_in_t rq = {codes, factors, P, bits};
+    return fragility_impl(X, ids, assign, n, d, C, nlist, Q, nq, qids, order, upto, tau, k, nprobe,
+                          tau_gap, kth_gap, cen_gap, nthreads, &rq);
 }
 
 /* ------------------------------------------------------------------------ */

@@ -12,6 +12,8 @@ Entry points (same names as the C ABI):
 * :func:`rank_partitions`   -- per-query top-nprobe centroid order
 * :func:`search`            -- SieveIVF search on device tensors
 * :func:`search_host`       -- the same with host queries and host results
+* :func:`rq_encode`, :func:`build_rq_layout`, :func:`rq_search` -- the local
+  search over RaBitQ-style codes (the paper's IVF_RQ7 index)
 """
 from __future__ import annotations
 
@@ -57,11 +59,17 @@ class StatsC(C.Structure):
                 ("tiles", C.c_int64), ("rows_read", C.c_int64), ("pairs", C.c_int64),
                 ("rows_read_tc", C.c_int64), ("pairs_tc", C.c_int64),
                 ("status", C.c_int32), ("reserved0", C.c_int32),
-                ("kernel_ms", C.c_float * 10), ("kernel_launches", C.c_int32 * 10)]
+                ("kernel_ms", C.c_float * 11), ("kernel_launches", C.c_int32 * 11)]
+
+
+class RqViewC(C.Structure):
+    _fields_ = [("bits", C.c_int32), ("reserved0", C.c_int32), ("rq_rows", C.c_void_p),
+                ("rq_row_blocks", C.c_void_p), ("rq_factors", C.c_void_p),
+                ("rq_rotation", C.c_void_p)]
 
 
 KERNELS = ("rank", "init", "issue", "bucket", "scatter", "scan", "merge", "round_end", "finalize",
-           "scan_tc")
+           "scan_tc", "rq_rotate")
 SCAN_PATHS = {"auto": 0, "simt": 1, "tensor": 2}
 
 
@@ -119,6 +127,20 @@ _SIGNATURES = {
                                               C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
                                               C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
                                               C.c_void_p]),
+    "sieve_rq_encode": (C.c_int32, [C.POINTER(IndexViewC), C.c_void_p, C.c_int32, C.c_void_p,
+                                    C.c_void_p, C.c_void_p]),
+    "sieve_rq_layout_size": (C.c_int32, [C.POINTER(IndexViewC), C.POINTER(C.c_size_t),
+                                         C.POINTER(C.c_size_t), C.POINTER(C.c_size_t)]),
+    "sieve_build_rq_layout": (C.c_int32, [C.POINTER(IndexViewC), C.c_void_p, C.c_void_p,
+                                          C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p,
+                                          C.c_void_p, C.c_void_p, C.c_void_p]),
+    "sieve_rq_search_workspace_size": (C.c_int32, [C.POINTER(IndexViewC), C.c_int64,
+                                                   C.POINTER(ParamsC), C.POINTER(C.c_size_t)]),
+    "sieve_rq_search": (C.c_int32, [C.POINTER(IndexViewC), C.POINTER(RqViewC), C.c_void_p,
+                                    C.c_int64, C.c_void_p, C.c_void_p, C.c_void_p,
+                                    C.POINTER(ParamsC), C.c_void_p, C.c_void_p, C.c_void_p,
+                                    C.c_void_p, C.POINTER(StatsC), C.c_void_p, C.c_size_t,
+                                    C.c_void_p]),
     "sieve_status_str": (C.c_char_p, [C.c_int32]),
     "sieve_last_cuda_error": (C.c_int32, []),
     "sieve_version": (C.c_char_p, []),
@@ -365,6 +387,106 @@ def search(index: Index, Q, tau, k, nprobe, W, lookahead=True, query_ids=None, o
                               _ptr(ids), _ptr(scores), _ptr(count), _ptr(probes),
                               C.byref(st) if st is not None else None, _ptr(ws), ws.numel(),
                               _stream(stream)), "sieve_search")
+    if stats:
+        return ids, scores, count, probes, _stats_dict(st)
+    return ids, scores, count, probes
+
+
+@dataclass
+class RQIndex:
+    """RaBitQ-style codes of an index (the paper's IVF_RQ7: RaBitQ with 7
+    bits) in the layout the quantized scan reads.  ``codes`` [n][d] u8 and
+    ``factors`` [n] f32 are in the index's row order; the rest is their scan
+    layout (:func:`build_rq_layout`)."""
+    bits: int
+    codes: torch.Tensor
+    factors: torch.Tensor
+    rows: torch.Tensor            # fp16 (u - mid) tiles, 16 KB per block K-block
+    row_blocks: torch.Tensor      # [nlist+1] i64
+    block_factors: torch.Tensor   # [blocks * 128] f32
+    rotation: torch.Tensor        # tensor-core layout of P^T
+
+    def view(self) -> RqViewC:
+        v = RqViewC()
+        v.bits = self.bits
+        v.rq_rows = self.rows.data_ptr()
+        v.rq_row_blocks = self.row_blocks.data_ptr()
+        v.rq_factors = self.block_factors.data_ptr()
+        v.rq_rotation = self.rotation.data_ptr()
+        return v
+
+
+def rq_encode(index: Index, P, bits=7, stream=None):
+    """Codes [n][d] u8 and factors [n] f32 of the index's rows for the
+    orthogonal rotation P [d][d] (float64, device) (sieve_rq_encode)."""
+    _need_cuda(P, torch.float64, "P", 2)
+    n, d = index.vectors.shape
+    dev = index.vectors.device
+    codes = torch.empty((n, d), dtype=torch.uint8, device=dev)
+    factors = torch.empty(n, dtype=torch.float32, device=dev)
+    v = index.view()
+    _check(lib().sieve_rq_encode(C.byref(v), _ptr(P), int(bits), _ptr(codes), _ptr(factors),
+                                 _stream(stream)), "sieve_rq_encode")
+    return codes, factors
+
+
+def build_rq_layout(index: Index, P, bits=7, codes=None, factors=None, stream=None) -> RQIndex:
+    """The quantized index: codes (encoded here unless given) and their scan
+    layout (sieve_build_rq_layout)."""
+    _need_cuda(P, torch.float64, "P", 2)
+    if codes is None or factors is None:
+        codes, factors = rq_encode(index, P, bits, stream)
+    _need_cuda(codes, torch.uint8, "codes", 2)
+    _need_cuda(factors, torch.float32, "factors", 1)
+    v = index.view()
+    rb, fb, ob = C.c_size_t(), C.c_size_t(), C.c_size_t()
+    _check(lib().sieve_rq_layout_size(C.byref(v), C.byref(rb), C.byref(fb), C.byref(ob)),
+           "sieve_rq_layout_size")
+    dev = index.vectors.device
+    rows = torch.empty(max(rb.value, 256), dtype=torch.uint8, device=dev)
+    blocks = torch.empty(index.nlist + 1, dtype=torch.int64, device=dev)
+    bfac = torch.empty(max(fb.value // 4, 64), dtype=torch.float32, device=dev)
+    rot = torch.empty(max(ob.value, 256), dtype=torch.uint8, device=dev)
+    _check(lib().sieve_build_rq_layout(C.byref(v), _ptr(codes), _ptr(factors), int(bits), _ptr(P),
+                                       _ptr(rows), _ptr(blocks), _ptr(bfac), _ptr(rot),
+                                       _stream(stream)), "sieve_build_rq_layout")
+    return RQIndex(int(bits), codes, factors, rows, blocks, bfac, rot)
+
+
+def rq_search(index: Index, rq: RQIndex, Q, tau, k, nprobe, W, lookahead=True, query_ids=None,
+              order=None, cscores=None, max_items_per_round=0, loop=0, stats=False,
+              profile=False, workspace=None, out=None, stream=None):
+    """search() with the quantized local search over rq's codes
+    (sieve_rq_search): a row qualifies iff its estimate <q, c_p> +
+    f <u - mid, P^T q> >= tau.  A precomputed ``order`` needs its ``cscores``."""
+    stats = stats or profile
+    _need_cuda(Q, torch.float32, "Q", 2)
+    if query_ids is not None:
+        _need_cuda(query_ids, torch.int64, "query_ids", 1)
+    if order is not None:
+        _need_cuda(order, torch.int32, "order", 2)
+    if cscores is not None:
+        _need_cuda(cscores, torch.float32, "cscores", 2)
+    nq = Q.shape[0]
+    dev = Q.device
+    p = _params(tau, k, nprobe, W, lookahead, loop, max_items_per_round, profile, "auto")
+    v = index.view()
+    rv = rq.view()
+    nbytes = C.c_size_t()
+    _check(lib().sieve_rq_search_workspace_size(C.byref(v), nq, C.byref(p), C.byref(nbytes)),
+           "sieve_rq_search_workspace_size")
+    ws = _workspace(workspace, nbytes.value, dev)
+    if out is None:
+        out = (torch.empty((nq, k), dtype=torch.int64, device=dev),
+               torch.empty((nq, k), dtype=torch.float32, device=dev),
+               torch.empty(nq, dtype=torch.int32, device=dev),
+               torch.empty(nq, dtype=torch.int32, device=dev))
+    ids, scores, count, probes = out
+    st = StatsC() if stats else None
+    _check(lib().sieve_rq_search(C.byref(v), C.byref(rv), _ptr(Q), nq, _ptr(query_ids), _ptr(order),
+                                 _ptr(cscores), C.byref(p), _ptr(ids), _ptr(scores), _ptr(count),
+                                 _ptr(probes), C.byref(st) if st is not None else None, _ptr(ws),
+                                 ws.numel(), _stream(stream)), "sieve_rq_search")
     if stats:
         return ids, scores, count, probes, _stats_dict(st)
     return ids, scores, count, probes

@@ -84,11 +84,13 @@ struct Layout {
     size_t ctl, order, S, E, counts, cursor, item_q, item_rank, item_p, bucketed, tiles, tc_tiles,
         active, res_cnt, res_s, res_id, rank_scratch;
     size_t h_Q, h_qids, h_ids, h_scores, h_count, h_probes;
+    size_t qrot, cscores;   // quantized search: rotated queries, centroid scores
     size_t total;
     int64_t cap, max_tiles;
 };
 
-Layout make_layout(const sieve_index_view *ix, int64_t nq, const sieve_params *p, bool host_io) {
+Layout make_layout(const sieve_index_view *ix, int64_t nq, const sieve_params *p, bool host_io,
+                   bool rq = false) {
     Layout L{};
     size_t off = 0;
     auto take = [&](size_t bytes) {
@@ -130,6 +132,10 @@ Layout make_layout(const sieve_index_view *ix, int64_t nq, const sieve_params *p
         L.h_count = take((size_t)nq * 4);
         L.h_probes = take((size_t)nq * 4);
     }
+    if (rq) {
+        L.qrot = take((size_t)nq * ix->d * 4);
+        L.cscores = take((size_t)nq * p->nprobe * 4);
+    }
     L.total = off;
     return L;
 }
@@ -165,9 +171,15 @@ constexpr size_t kGraphCacheMax = 8;
 cudaError_t launch_search_rank(const SearchArgs &a, int rank_tc, cudaStream_t st) {
     int32_t *order = const_cast<int32_t *>(a.order);
     if (rank_tc)
-        return enqueue_rank_tc(a.Q, a.nq, a.C, a.nlist, a.d, a.nprobe, order, nullptr,
+        return enqueue_rank_tc(a.Q, a.nq, a.C, a.nlist, a.d, a.nprobe, order, a.cscores,
                                a.rank_scratch, &a.ctl->status, st, a.tc_cent);
-    return enqueue_rank(a.Q, a.nq, a.C, a.nlist, a.d, a.nprobe, order, nullptr, st);
+    return enqueue_rank(a.Q, a.nq, a.C, a.nlist, a.d, a.nprobe, order, a.cscores, st);
+}
+
+// quantized search: q' = P^T q for the batch, after init (which clears the
+// status word the rotation's bounded waits report to)
+cudaError_t launch_search_rotate(const SearchArgs &a, cudaStream_t st) {
+    return launch_rq_rotate(a.Q, a.nq, a.d, a.rq_rot, const_cast<float *>(a.Qrot), &a.ctl->status, st);
 }
 
 sieve_status build_graph(const GraphKey &key, cudaGraph_t *g_out, cudaGraphExec_t *exec_out) {
@@ -183,6 +195,7 @@ sieve_status build_graph(const GraphKey &key, cudaGraph_t *g_out, cudaGraphExec_
         // outer graph: [rank] -> init -> WHILE(rounds) -> finalize
         if ((e = cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal)) != cudaSuccess) break;
         e = launch_init(a, cs);
+        if (e == cudaSuccess && a.rq) e = launch_search_rotate(a, cs);
         if (e == cudaSuccess && key.with_rank) e = launch_search_rank(a, key.rank_tc, cs);
         cudaStreamCaptureStatus cst;
         cudaGraph_t cg = nullptr;
@@ -276,11 +289,20 @@ struct SearchExtras {
     uint32_t *hit_bits;   // [nq][ceil(nprobe / 32)]
 };
 
+// quantized local search (sieve_rq_search): the code layout, the rotation's
+// layout, and centroid scores given with a precomputed order (else nullptr:
+// the ranking writes them into the workspace)
+struct RqInputs {
+    const sieve_rq_view *v;
+    const float *cscores;
+};
+
 sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t nq,
                            const int64_t *qids, const int32_t *order, const sieve_params *p,
                            int64_t *out_ids, float *out_scores, int32_t *out_count,
                            int32_t *out_probes, sieve_stats *stats, unsigned char *ws,
-                           const Layout &L, cudaStream_t st, const SearchExtras *ex = nullptr) {
+                           const Layout &L, cudaStream_t st, const SearchExtras *ex = nullptr,
+                           const RqInputs *rq = nullptr) {
     SearchArgs a;
     std::memset(&a, 0, sizeof(a));   // padding takes part in the graph-cache key
     a.X = ix->vectors;
@@ -328,6 +350,21 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
         a.tc_rows = nullptr;
         a.tc_row_blocks = nullptr;
     }
+    if (rq) {   // every group on the tensor cores, over the codes
+        const int rq_stages = scan_rq_stages(ix->d, p->k);
+        if (rq_stages == 0 || p->scan_path == 1) return SIEVE_EINVAL;
+        a.rq = 1;
+        a.tc_min = 1;
+        a.tc_stages = rq_stages;
+        a.tc_rows = nullptr;
+        a.tc_row_blocks = nullptr;
+        a.rq_rows = static_cast<const unsigned char *>(rq->v->rq_rows);
+        a.rq_row_blocks = rq->v->rq_row_blocks;
+        a.rq_fac = rq->v->rq_factors;
+        a.rq_rot = static_cast<const unsigned char *>(rq->v->rq_rotation);
+        a.Qrot = reinterpret_cast<const float *>(ws + L.qrot);
+        a.cscores = rq->cscores ? const_cast<float *>(rq->cscores) : reinterpret_cast<float *>(ws + L.cscores);
+    }
     a.res_cnt = reinterpret_cast<int *>(ws + L.res_cnt);
     a.res_s = reinterpret_cast<float *>(ws + L.res_s);
     a.res_id = reinterpret_cast<long long *>(ws + L.res_id);
@@ -346,8 +383,12 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
     const int rank_tc = with_rank && a.rank_scratch != nullptr;
     const size_t smem = scan_smem_bytes(ix->d, p->k);
     SIEVE_CUDA(prepare_scan_kernel(smem));
-    if (a.tc_min > 0)
+    if (a.rq) {
+        SIEVE_CUDA(prepare_scan_rq(ix->d, p->k, a.tc_stages));
+        SIEVE_CUDA(prepare_rq_rotate(ix->d));
+    } else if (a.tc_min > 0) {
         SIEVE_CUDA(a.tc_stages ? prepare_scan_bulk(ix->d, p->k, a.tc_stages) : prepare_scan_tc(p->k));
+    }
     if (with_rank) SIEVE_CUDA(rank_tc ? prepare_rank_tc(p->nprobe, ix->d) : prepare_rank(p->nprobe));
     const int blocks = scan_blocks_for(smem);
 
@@ -381,6 +422,7 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
             return e;
         };
         SIEVE_CUDA(timed(SIEVE_K_INIT, [&] { return launch_init(a, st); }));
+        if (a.rq) SIEVE_CUDA(timed(SIEVE_K_RQ_ROTATE, [&] { return launch_search_rotate(a, st); }));
         if (with_rank)
             SIEVE_CUDA(timed(SIEVE_K_RANK, [&] { return launch_search_rank(a, rank_tc, st); }));
         for (;;) {
@@ -425,6 +467,7 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
         stats->kernel_launches[SIEVE_K_FINALIZE] = 1;
         for (int slot : per_round) stats->kernel_launches[slot] = c.round;
         stats->kernel_launches[SIEVE_K_SCAN_TC] = a.tc_min > 0 ? c.round : 0;
+        stats->kernel_launches[SIEVE_K_RQ_ROTATE] = a.rq ? 1 : 0;
         if (a.tc_min == 1) stats->kernel_launches[SIEVE_K_SCAN] = 0;
         if (c.status != 0) return c.status;
     }
@@ -589,6 +632,103 @@ sieve_status sieve_search(const sieve_index_view *ix, const float *Q, int64_t nq
     return search_device(ix, Q, nq, query_ids, order, p, out_ids, out_scores, out_count,
                          out_probes, stats, static_cast<unsigned char *>(ws), L,
                          static_cast<cudaStream_t>(stream));
+}
+
+// ---------------------------------------------------------------------------
+// Quantized local search over RaBitQ-style codes (Sec. 3.1, Sec. 6.1).
+static sieve_status check_rq_index(const sieve_index_view *ix, int32_t bits) {
+    sieve_status rc = check_index(ix, true);
+    if (rc != SIEVE_OK) return rc;
+    if (ix->d > kRqMaxD || bits < 1 || bits > 8) return SIEVE_EINVAL;
+    return SIEVE_OK;
+}
+
+sieve_status sieve_rq_encode(const sieve_index_view *ix, const double *P, int32_t bits,
+                             uint8_t *codes, float *factors, void *stream) {
+    sieve_status rc = check_rq_index(ix, bits);
+    if (rc != SIEVE_OK) return rc;
+    if (!P || (ix->n > 0 && (!codes || !factors))) return SIEVE_EINVAL;
+    if ((rc = check_device()) != SIEVE_OK) return rc;
+    SIEVE_CUDA(launch_rq_encode(ix->vectors, ix->list_offsets, ix->nlist, ix->n, ix->d, ix->centroids, P,
+                                bits, codes, factors, static_cast<cudaStream_t>(stream)));
+    return SIEVE_OK;
+}
+
+sieve_status sieve_rq_layout_size(const sieve_index_view *ix, size_t *rows_bytes,
+                                  size_t *factors_bytes, size_t *rotation_bytes) {
+    if (!rows_bytes || !factors_bytes || !rotation_bytes) return SIEVE_EINVAL;
+    sieve_status rc = check_rq_index(ix, 7);
+    if (rc != SIEVE_OK) return rc;
+    std::vector<int64_t> off((size_t)ix->nlist + 1);
+    SIEVE_CUDA(cudaMemcpy(off.data(), ix->list_offsets, off.size() * sizeof(int64_t),
+                          cudaMemcpyDeviceToHost));
+    int64_t blocks = 0;
+    for (int64_t p = 0; p < ix->nlist; ++p) {
+        if (off[p + 1] < off[p]) return SIEVE_EINVAL;
+        blocks += ceil_div(off[p + 1] - off[p], kTcRows);
+    }
+    *rows_bytes = rq_rows_bytes(blocks, ix->d);
+    *factors_bytes = (size_t)blocks * kTcRows * sizeof(float);
+    *rotation_bytes = (size_t)(ceil_div(ix->d, kTcRows) * (int64_t)tc_nkb(ix->d) * kTcBlockBytes);
+    return SIEVE_OK;
+}
+
+sieve_status sieve_build_rq_layout(const sieve_index_view *ix, const uint8_t *codes,
+                                   const float *factors, int32_t bits, const double *P,
+                                   void *rq_rows, int64_t *rq_row_blocks, float *rq_factors,
+                                   void *rq_rotation, void *stream) {
+    sieve_status rc = check_rq_index(ix, bits);
+    if (rc != SIEVE_OK) return rc;
+    if (!P || !rq_rows || !rq_row_blocks || !rq_factors || !rq_rotation) return SIEVE_EINVAL;
+    if (ix->n > 0 && (!codes || !factors)) return SIEVE_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(rq_rows) | reinterpret_cast<uintptr_t>(rq_rotation) |
+         reinterpret_cast<uintptr_t>(rq_factors)) & 255u)
+        return SIEVE_EINVAL;
+    if ((rc = check_device()) != SIEVE_OK) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    SIEVE_CUDA(launch_rq_layout(codes, factors, ix->list_offsets, ix->nlist, ix->d, bits, rq_row_blocks,
+                                static_cast<unsigned char *>(rq_rows), rq_factors, st));
+    SIEVE_CUDA(launch_rq_rotation_layout(P, ix->d, static_cast<unsigned char *>(rq_rotation), st));
+    return SIEVE_OK;
+}
+
+sieve_status sieve_rq_search_workspace_size(const sieve_index_view *ix, int64_t nq,
+                                            const sieve_params *p, size_t *bytes) {
+    if (!bytes) return SIEVE_EINVAL;
+    sieve_status rc = check_rq_index(ix, 7);
+    if (rc != SIEVE_OK) return rc;
+    if ((rc = check_params(ix, p)) != SIEVE_OK) return rc;
+    if (nq < 0 || nq > INT32_MAX / 2) return SIEVE_EINVAL;
+    *bytes = make_layout(ix, nq, p, false, true).total;
+    return SIEVE_OK;
+}
+
+sieve_status sieve_rq_search(const sieve_index_view *ix, const sieve_rq_view *rq, const float *Q,
+                             int64_t nq, const int64_t *query_ids, const int32_t *order,
+                             const float *cscores, const sieve_params *p, int64_t *out_ids,
+                             float *out_scores, int32_t *out_count, int32_t *out_probes,
+                             sieve_stats *stats, void *ws, size_t ws_bytes, void *stream) {
+    sieve_status rc = check_search(ix, Q, nq, order, p, out_ids, out_scores, out_count, out_probes);
+    if (rc != SIEVE_OK) return rc;
+    if (!rq || (rc = check_rq_index(ix, rq->bits)) != SIEVE_OK) return SIEVE_EINVAL;
+    if (!rq->rq_rows || !rq->rq_row_blocks || !rq->rq_factors || !rq->rq_rotation) return SIEVE_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(rq->rq_rows) | reinterpret_cast<uintptr_t>(rq->rq_rotation) |
+         reinterpret_cast<uintptr_t>(rq->rq_factors)) & 15u)
+        return SIEVE_EINVAL;
+    if (order && !cscores) return SIEVE_EINVAL;
+    if (p->scan_path == 1 || scan_rq_stages(ix->d, p->k) == 0) return SIEVE_EINVAL;
+    if (nq > 0 && !aligned16(Q)) return SIEVE_EINVAL;
+    if (p->profile && !stats) return SIEVE_EINVAL;
+    if ((rc = check_device()) != SIEVE_OK) return rc;
+    if (stats) std::memset(stats, 0, sizeof(*stats));
+    if (nq == 0) return SIEVE_OK;
+    const Layout L = make_layout(ix, nq, p, false, true);
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < L.total)
+        return SIEVE_EWORKSPACE;
+    const RqInputs in{rq, order ? cscores : nullptr};
+    return search_device(ix, Q, nq, query_ids, order, p, out_ids, out_scores, out_count, out_probes,
+                         stats, static_cast<unsigned char *>(ws), L, static_cast<cudaStream_t>(stream),
+                         nullptr, &in);
 }
 
 sieve_status sieve_search_host(const sieve_index_view *ix, const float *Q_host, int64_t nq,

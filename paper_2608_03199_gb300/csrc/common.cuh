@@ -10,6 +10,7 @@ namespace sieve {
 
 constexpr int kMaxK = 64;        // results per query
 constexpr int kMaxD = 1024;      // vector dimension
+constexpr int kRqMaxD = 256;     // quantized search: the query tile's split lives in tensor memory
 constexpr int kMaxNprobe = 512;  // partitions per query
 
 // SIMT contraction tile: QT queries x RT rows per thread block of 128 threads;

@@ -16,12 +16,17 @@ namespace sieve {
 
 __device__ __forceinline__ int tc_nkb_dev(int d) { return (d + 63) / 64; }
 
-struct ScanMode {
+// kRQ = false: exact inner products (B = the rows' hi / lo split);
+// kRQ = true: RaBitQ-style estimates from the code layout (B = u - mid)
+template <bool kRQ>
+struct ScanModeT {
     using Args = SearchArgs;
     static constexpr int kN = 256;
+    static constexpr bool kBHasLo = !kRQ;
     struct Tile {
         int p, ib, ni;
         int64_t r_begin, nb;
+        const float *fac;   // kRQ: the factors of p's rows (block order)
     };
     __device__ static int num_tiles(const Args &a) { return a.ctl->n_tc_tiles; }
     // tiles differ in cost (partition sizes are skewed): blocks draw them dynamically
@@ -36,15 +41,18 @@ struct ScanMode {
         T.ni = x.z;
         T.r_begin = a.off[T.p];
         T.nb = a.off[T.p + 1] - T.r_begin;
+        T.fac = kRQ ? a.rq_fac + a.rq_row_blocks[T.p] * kTcRows : nullptr;
         return T;
     }
     __device__ static const float *a_row(const Args &a, const Tile &T, int i) {
-        return i < T.ni ? a.Q + (int64_t)a.item_q[a.bucketed[T.ib + i]] * a.d : nullptr;
+        const float *Qa = kRQ ? a.Qrot : a.Q;
+        return i < T.ni ? Qa + (int64_t)a.item_q[a.bucketed[T.ib + i]] * a.d : nullptr;
     }
     __device__ static const float *b_row(const Args &a, const Tile &T, int64_t r) {
         return r < T.nb ? a.X + (T.r_begin + r) * a.d : nullptr;
     }
     __device__ static const unsigned char *b_block(const Args &a, const Tile &T, int ch) {
+        if (kRQ) return a.rq_rows + (a.rq_row_blocks[T.p] + ch) * (int64_t)tc_nkb_dev(a.d) * tcb::kKbBytesHi;
         return a.tc_rows + (a.tc_row_blocks[T.p] + ch) * (int64_t)tc_nkb_dev(a.d) * kTcBlockBytes;
     }
 
@@ -52,6 +60,7 @@ struct ScanMode {
         float *ks;
         long long *ki;
         int kn, item, q, rank, slot;
+        float qc;   // kRQ: <q, c_p>, the centroid score of the item's rank
         bool valid;
         long long qid;
         // the kept list is unordered while the tile runs; once it holds k
@@ -73,11 +82,13 @@ struct ScanMode {
             valid = slot < T.ni;
             item = q = rank = 0;
             qid = (long long)-0x7fffffffffffffffll - 1;
+            qc = 0.f;
             if (valid) {
                 item = a.bucketed[T.ib + slot];
                 q = a.item_q[item];
                 rank = a.item_rank[item];
                 if (a.qids) qid = a.qids[q];
+                if (kRQ) qc = a.cscores[(int64_t)q * a.nprobe + rank - 1];
             }
         }
         __device__ void find_worst(int k) {
@@ -112,19 +123,17 @@ struct ScanMode {
             KI(wst_pos) = id;
             find_worst(k);
         }
-        // v holds the chunk's raw accumulator values: similarities x 2^16
-        __device__ void chunk(const Args &a, const Tile &T, int64_t col0, const float (&v)[32],
-                              int ncol) {
-            if (!valid) return;
+        // e holds 32 scores x `scale` (an exact power of two): the candidates
+        __device__ __forceinline__ void select(const Args &a, const Tile &T, int64_t col0,
+                                               const float (&e)[32], int ncol, float scale) {
             // a candidate needs s >= tau and, once k are kept, s >= the k-th
-            // kept score (equal scores go on to the id tie-break); scores
-            // here are raw (x 2^16, an exact power-of-two scale)
-            float thr = a.tau * 65536.f;
-            if (kn == a.k) thr = fmaxf(thr, wst_s * 65536.f);
+            // kept score (equal scores go on to the id tie-break)
+            float thr = a.tau * scale;
+            if (kn == a.k) thr = fmaxf(thr, wst_s * scale);
             // nearly every group has no candidate: one tree of maxima decides
             float mx[16];
 #pragma unroll
-            for (int j = 0; j < 16; ++j) mx[j] = fmaxf(v[j], v[j + 16]);
+            for (int j = 0; j < 16; ++j) mx[j] = fmaxf(e[j], e[j + 16]);
 #pragma unroll
             for (int w = 8; w > 0; w >>= 1)
 #pragma unroll
@@ -132,13 +141,46 @@ struct ScanMode {
             if (!(mx[0] >= thr)) return;
             unsigned m = 0;
 #pragma unroll
-            for (int j = 0; j < 32; ++j) m |= (v[j] >= thr && j < ncol) ? (1u << j) : 0u;
+            for (int j = 0; j < 32; ++j) m |= (e[j] >= thr && j < ncol) ? (1u << j) : 0u;
             // one candidate at a time in a loop that is not unrolled: a single
             // copy of the insert, the score picked out of the registers
+            const float inv = 1.f / scale;
             while (m) {
                 const int j = __ffs(m) - 1;
                 m &= m - 1u;
-                take(a, T, col0 + j, pick32(v, j) * (1.f / 65536.f));
+                take(a, T, col0 + j, pick32(e, j) * inv);
+            }
+        }
+        // v holds the chunk's raw accumulator values: exact, similarities x
+        // 2^16; kRQ, <u - mid, q'> x 2^8 (the codes are not scaled)
+        __device__ void chunk(const Args &a, const Tile &T, int64_t col0, const float (&v)[32],
+                              int ncol) {
+            if (!valid || ncol <= 0) return;
+            if constexpr (kRQ) {
+                // the estimates qc + f <u - mid, q'> against the threshold,
+                // straight into a mask (no array of estimates stays live); the
+                // factor array covers whole blocks (0 on padding rows), so the
+                // 32 loads stay inside it
+                float thr = a.tau;
+                if (kn == a.k) thr = fmaxf(thr, wst_s);
+                const float4 *f4 = reinterpret_cast<const float4 *>(T.fac + col0);
+                unsigned m = 0;
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    const float4 f = __ldg(f4 + j);
+                    m |= (fmaf(f.x, v[4 * j] * (1.f / 256.f), qc) >= thr) ? 1u << (4 * j) : 0u;
+                    m |= (fmaf(f.y, v[4 * j + 1] * (1.f / 256.f), qc) >= thr) ? 2u << (4 * j) : 0u;
+                    m |= (fmaf(f.z, v[4 * j + 2] * (1.f / 256.f), qc) >= thr) ? 4u << (4 * j) : 0u;
+                    m |= (fmaf(f.w, v[4 * j + 3] * (1.f / 256.f), qc) >= thr) ? 8u << (4 * j) : 0u;
+                }
+                if (ncol < 32) m &= (1u << ncol) - 1u;
+                while (m) {   // the rare candidates: the estimate again, the same arithmetic
+                    const int j = __ffs(m) - 1;
+                    m &= m - 1u;
+                    take(a, T, col0 + j, fmaf(T.fac[col0 + j], pick32(v, j) * (1.f / 256.f), qc));
+                }
+            } else {
+                select(a, T, col0, v, ncol, 65536.f);
             }
         }
         __device__ void end(const Args &a, const Tile &T) {
@@ -176,6 +218,9 @@ struct ScanMode {
     };
 };
 
+using ScanMode = ScanModeT<false>;
+using ScanModeRQ = ScanModeT<true>;
+
 bool scan_tc_fits(int k) { return scan_tc_smem_bytes(k) <= (size_t)(232448 - 128); }
 
 size_t scan_tc_smem_bytes(int k) {
@@ -207,6 +252,27 @@ cudaError_t prepare_scan_bulk(int d, int k, int stages) {
 void enqueue_scan_bulk(const SearchArgs &a, cudaStream_t st) {
     k_scan_bulk<<<num_sms(), tcb::kThreads,
                   tcb::smem_bytes(a.tc_stages, scan_epi_bytes(a.k)), st>>>(a);
+}
+
+// the scan over codes: 16 KB stages, up to eight
+int scan_rq_stages(int d, int k) {
+    return tcb::stages_for((int)ceil_div(d, 64), scan_epi_bytes(k), 232448 - 128, tcb::kKbBytesHi,
+                           tcb::kMaxStages);
+}
+
+__global__ void __launch_bounds__(tcb::kThreads, 1) k_scan_rq(SearchArgs a) {
+    extern __shared__ unsigned char smem_raw[];
+    tcb::run_bulk<ScanModeRQ>(a, smem_raw, a.tc_stages);
+}
+
+cudaError_t prepare_scan_rq(int d, int k, int stages) {
+    return cudaFuncSetAttribute(k_scan_rq, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)tcb::smem_bytes(stages, scan_epi_bytes(k), tcb::kKbBytesHi));
+}
+
+void enqueue_scan_rq(const SearchArgs &a, cudaStream_t st) {
+    k_scan_rq<<<num_sms(), tcb::kThreads, tcb::smem_bytes(a.tc_stages, scan_epi_bytes(a.k), tcb::kKbBytesHi),
+                st>>>(a);
 }
 
 cudaError_t prepare_scan_tc(int k) {

@@ -59,6 +59,16 @@ struct SearchArgs {
     int *out_rank;
     unsigned *hit_bits;
     int hit_words;
+    // quantized local search over RaBitQ-style codes (rq = 1): the estimate
+    // of <q, x> for row x of partition p is cscores(q, rank of p) + f_x
+    // <u_x - mid, q'>; rq = 0: exact inner products
+    int rq;
+    const float *Qrot;                  // [nq][d] rotated queries q' = P^T q
+    float *cscores;                     // [nq][nprobe] centroid scores of the ranking
+    const unsigned char *rq_rows;       // code layout: fp16 (u - mid), 16 KB per block K-block
+    const int64_t *rq_row_blocks;       // [nlist+1] block offsets of that layout
+    const float *rq_fac;                // [blocks * 128] factors f in block order
+    const unsigned char *rq_rot;        // tensor-core layout of P^T (the query rotation)
 };
 
 size_t scan_smem_bytes(int d, int k);
@@ -130,6 +140,28 @@ cudaError_t launch_tc_layout_rows(const float *X, const int64_t *off, int64_t np
                                   int64_t *blk_off, unsigned char *out, cudaStream_t st);
 cudaError_t launch_tc_layout_matrix(const float *X, int64_t nrows, int d, unsigned char *out,
                                     cudaStream_t st);
+// block offsets of the partitions: blk_off[p] = sum over p' < p of ceil(rows / 128)
+cudaError_t launch_tc_block_scan(const int64_t *off, int64_t nparts, int64_t *blk_off, cudaStream_t st);
+
+// RaBitQ-style codes (rq.cu): codes and factors of partition-contiguous rows,
+// the scan's code layout (16 KB per block K-block, factors in block order),
+// and the query rotation q' = P^T q on the tensor cores
+int rq_nkb(int d);
+size_t rq_rows_bytes(int64_t nblocks, int d);
+cudaError_t launch_rq_encode(const float *X, const int64_t *off, int64_t nlist, int64_t n, int d,
+                             const float *C, const double *P, int bits, uint8_t *codes, float *factors,
+                             cudaStream_t st);
+cudaError_t launch_rq_layout(const uint8_t *codes, const float *factors, const int64_t *off,
+                             int64_t nparts, int d, int bits, int64_t *blk_off, unsigned char *out,
+                             float *fac_out, cudaStream_t st);
+cudaError_t launch_rq_rotation_layout(const double *P, int d, unsigned char *out, cudaStream_t st);
+cudaError_t prepare_rq_rotate(int d);
+cudaError_t launch_rq_rotate(const float *Q, int64_t nq, int d, const unsigned char *rot, float *Qrot,
+                             int *status, cudaStream_t st);
+// the tensor-core scan over codes (scan_tc.cu)
+int scan_rq_stages(int d, int k);                // 0 when it does not apply
+cudaError_t prepare_scan_rq(int d, int k, int stages);
+void enqueue_scan_rq(const SearchArgs &a, cudaStream_t st);
 
 // partition layout (layout_kernels.cu)
 size_t layout_workspace_bytes(int64_t n, int64_t nlist);

@@ -604,7 +604,9 @@ cudaError_t launch_round(const SearchArgs &a, size_t scan_smem, int scan_blocks,
     end();
     begin();
     if (a.tc_min > 0) {
-        if (a.tc_stages)
+        if (a.rq)
+            enqueue_scan_rq(a, st);
+        else if (a.tc_stages)
             enqueue_scan_bulk(a, st);
         else
             enqueue_scan_tc(a, st);

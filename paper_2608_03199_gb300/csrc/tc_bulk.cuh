@@ -50,7 +50,9 @@ constexpr int kProducerWarp = 8;
 constexpr int kMmaWarp = 9;
 constexpr int kThreads = 14 * 32;
 constexpr int kMaxKb = 4;                     // A in tensor memory: d <= 256
-constexpr int kMaxStages = 5;                 // timed faster than six: more of the SM memory stays L1
+constexpr int kMaxStages = 8;                 // barrier slots for B stages
+constexpr int kStages32 = 5;                  // 32 KB stages: five timed faster than six (more
+                                              // of the SM memory stays L1)
 constexpr uint32_t kKbBytes = 32768;          // one K-block of 128 rows: hi 16 KB + lo 16 KB
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kAColumn0 = 2 * kN;        // A after the two accumulators
@@ -58,20 +60,33 @@ constexpr uint32_t kWaitPolls = 1u << 24;
 constexpr int kRing = 8;                      // tiles handed from the scheduler to the other roles
 constexpr uint32_t kRingReaders = kAWriterWarps + 1 + 4;   // A-writer warps, MMA lane, epilogue warps
 
+constexpr uint32_t kKbBytesHi = 16384;        // one K-block of 128 rows with no lo part (codes)
+
 // shared memory: 1 KB alignment slack, the B stages, the epilogue's bytes
-__host__ __device__ inline size_t smem_bytes(int stages, size_t epi_bytes) {
-    return 1024 + (size_t)stages * kKbBytes + epi_bytes;
+__host__ __device__ inline size_t smem_bytes(int stages, size_t epi_bytes,
+                                             uint32_t stage_bytes = kKbBytes) {
+    return 1024 + (size_t)stages * stage_bytes + epi_bytes;
 }
 
 // B stages that fit beside the epilogue (0 when the pipeline does not apply)
-inline int stages_for(int nkb, size_t epi_bytes, size_t smem_limit) {
+inline int stages_for(int nkb, size_t epi_bytes, size_t smem_limit, uint32_t stage_bytes = kKbBytes,
+                      int max_stages = kStages32) {
     if (nkb > kMaxKb) return 0;
-    const size_t base = smem_bytes(0, epi_bytes);
+    const size_t base = smem_bytes(0, epi_bytes, stage_bytes);
     if (smem_limit < base) return 0;
-    int s = (int)((smem_limit - base) / kKbBytes);
+    int s = (int)((smem_limit - base) / stage_bytes);
+    if (s > max_stages) s = max_stages;
     if (s > kMaxStages) s = kMaxStages;
     return s >= 2 ? s : 0;
 }
+
+// Modes whose B operand has a lo part (a split fp32 value: three products
+// per K step) and modes whose B is exact in fp16 (integer codes: B = hi only,
+// two products, half the stage)
+template <class Mode, class = void>
+struct b_has_lo { static constexpr bool value = true; };
+template <class Mode>
+struct b_has_lo<Mode, decltype((void)Mode::kBHasLo)> { static constexpr bool value = Mode::kBHasLo; };
 
 // one 32-column group of an accumulator row to the mode's epilogue
 template <class Epi, class Args, class Tile>
@@ -92,6 +107,8 @@ template <class Mode>
 __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned char *smem_raw,
                                          int stages) {
     constexpr uint32_t kIdesc = tc::idesc_f16(tcp::kM, kN);
+    constexpr bool kLo = b_has_lo<Mode>::value;
+    constexpr uint32_t kStage = kLo ? kKbBytes : kKbBytesHi;   // bytes of one B stage
     __shared__ __align__(8) uint64_t a_full[kMaxKb], a_empty[kMaxKb], b_full[kMaxStages],
         b_empty[kMaxStages], dfull_bar[2], dempty_bar[2], drain_bar, ring_full[kRing],
         ring_empty[kRing];
@@ -105,8 +122,8 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
     const int n_tiles = Mode::num_tiles(a);
     const int d = Mode::d(a);
     const int nkb = (int)ceil_div(d, 64);
-    unsigned char *Bst = base;                                 // stages x 32 KB
-    unsigned char *epi_smem = Bst + (size_t)stages * kKbBytes;
+    unsigned char *Bst = base;                                 // stages x kStage
+    unsigned char *epi_smem = Bst + (size_t)stages * kStage;
     int *status = Mode::status(a);
     int *tile_counter = Mode::tile_counter(a);
 
@@ -217,8 +234,8 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                     for (int kb = 0; kb < nkb; ++kb) {
                         const uint32_t st = s % stages, sph = (s / stages) & 1u;
                         if (!(ok = wait(&b_empty[st], sph ^ 1u))) break;
-                        tc::mbar_arrive_expect_tx(&b_full[st], kKbBytes);
-                        tc::bulk_g2s(Bst + (size_t)st * kKbBytes, src + (size_t)kb * kKbBytes, kKbBytes,
+                        tc::mbar_arrive_expect_tx(&b_full[st], kStage);
+                        tc::bulk_g2s(Bst + (size_t)st * kStage, src + (size_t)kb * kStage, kStage,
                                      &b_full[st]);
                         ++s;
                     }
@@ -256,18 +273,29 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                         if (!(ok = wait(&b_full[st], ph))) break;
                         tc::fence_after_sync();
                         const uint32_t a_hi = tA + (uint32_t)kb * 64, a_lo = a_hi + 32;
-                        const uint32_t b_hi = tc::smem_u32(Bst + (size_t)st * kKbBytes);
+                        const uint32_t b_hi = tc::smem_u32(Bst + (size_t)st * kStage);
                         // a K step moves the descriptors' start address by 32 bytes
                         // (2 in its 16-byte units; shared addresses stay far below
                         // the field's 2^14 limit, so no carry)
-                        const uint64_t bh = tc::desc_k_sw128(b_hi), bl = tc::desc_k_sw128(b_hi + kKbBytes / 2);
+                        const uint64_t bh = tc::desc_k_sw128(b_hi);
+                        if constexpr (kLo) {
+                            const uint64_t bl = tc::desc_k_sw128(b_hi + kKbBytes / 2);
 #pragma unroll
-                        for (int ks = 0; ks < 4; ++ks) {   // K = 16: 8 columns of A, 32 bytes of B
-                            const uint32_t ao = ks * 8;
-                            const uint64_t bo = 2 * ks;
-                            tc::mma_f16_ta(dt, a_lo + ao, bh + bo, kIdesc, (kb > 0 || ks > 0) ? 1u : 0u);
-                            tc::mma_f16_ta(dt, a_hi + ao, bl + bo, kIdesc, 1u);
-                            tc::mma_f16_ta(dt, a_hi + ao, bh + bo, kIdesc, 1u);
+                            for (int ks = 0; ks < 4; ++ks) {   // K = 16: 8 columns of A, 32 bytes of B
+                                const uint32_t ao = ks * 8;
+                                const uint64_t bo = 2 * ks;
+                                tc::mma_f16_ta(dt, a_lo + ao, bh + bo, kIdesc, (kb > 0 || ks > 0) ? 1u : 0u);
+                                tc::mma_f16_ta(dt, a_hi + ao, bl + bo, kIdesc, 1u);
+                                tc::mma_f16_ta(dt, a_hi + ao, bh + bo, kIdesc, 1u);
+                            }
+                        } else {   // B exact in fp16: hi and lo of A against it
+#pragma unroll
+                            for (int ks = 0; ks < 4; ++ks) {
+                                const uint32_t ao = ks * 8;
+                                const uint64_t bo = 2 * ks;
+                                tc::mma_f16_ta(dt, a_lo + ao, bh + bo, kIdesc, (kb > 0 || ks > 0) ? 1u : 0u);
+                                tc::mma_f16_ta(dt, a_hi + ao, bh + bo, kIdesc, 1u);
+                            }
                         }
                         tc::mma_commit(&b_empty[st]);
                         // the tile's last reads of this K-block of A: it may be

@@ -101,6 +101,11 @@ __global__ void k_tc_fill(const float *X, const int64_t *off, int64_t nparts, in
 
 int tc_nkb(int d) { return (int)ceil_div(d, 64); }
 
+cudaError_t launch_tc_block_scan(const int64_t *off, int64_t nparts, int64_t *blk_off, cudaStream_t st) {
+    k_tc_block_scan<<<1, 1024, 0, st>>>(off, nparts, blk_off);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_tc_layout_rows(const float *X, const int64_t *off, int64_t nparts, int d,
                                   int64_t *blk_off, unsigned char *out, cudaStream_t st) {
     k_tc_block_scan<<<1, 1024, 0, st>>>(off, nparts, blk_off);

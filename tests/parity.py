@@ -15,8 +15,10 @@ import oracle
 TOL = 1e-5
 
 
-def compare(gpu, ref, index, Q, qids, tau, k, nprobe, order, threads=None):
-    """gpu/ref: dicts with ids, scores, count, probes (numpy). Returns a report."""
+def compare(gpu, ref, index, Q, qids, tau, k, nprobe, order, threads=None, rq=None):
+    """gpu/ref: dicts with ids, scores, count, probes (numpy). Returns a report.
+    rq = (codes, factors, P, bits) for the quantized search: its decisions
+    are on the estimates, so their gaps decide what may differ."""
     g_ids, g_sc, g_cnt, g_pr = (np.asarray(gpu[x]) for x in ("ids", "scores", "count", "probes"))
     r_ids, r_sc, r_cnt, r_pr = ref["ids"], ref["scores"], ref["count"], ref["probes"]
     nq = len(r_pr)
@@ -26,7 +28,8 @@ def compare(gpu, ref, index, Q, qids, tau, k, nprobe, order, threads=None):
     if len(bad):
         upto = np.maximum(g_pr, r_pr).astype(np.int32)
         tg, kg, cg = oracle.fragility(index, Q[bad], tau, k, nprobe, order[bad], upto[bad],
-                                      qids=None if qids is None else qids[bad], threads=threads)
+                                      qids=None if qids is None else qids[bad], threads=threads,
+                                      rq=rq)
         allowed[bad] = (tg < TOL) | (kg < TOL) | (cg < TOL)
     unexplained = np.flatnonzero(~same & ~allowed)
     # scores of the matching queries

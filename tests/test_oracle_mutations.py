@@ -42,15 +42,15 @@ MUTATIONS = [
      "run = local_n[j - 1] > 0 ? run : run + 1;"),
     ("loss target inclusive", "if (loss < eps) {", "if (loss <= eps) {"),
     ("quantized estimate without the centroid term",
-     "double s = qc + (double)ix->factors[row] * (dot - ix->mid * sq);",
-     "double s = (double)ix->factors[row] * (dot - ix->mid * sq);"),
+     "return qc + (double)ix->factors[row] * (dot - ix->mid * sq);",
+     "return (double)ix->factors[row] * (dot - ix->mid * sq);"),
     ("quantized estimate with the code offset added", "(dot - ix->mid * sq)", "(dot + ix->mid * sq)"),
     ("codes from the untransposed rotation", "acc = fma(P[(int64_t)j * d + t], o[j], acc);",
      "acc = fma(P[(int64_t)t * d + j], o[j], acc);"),
     ("code step half as wide", "const double delta = 2.0 * mx / top;",
      "const double delta = mx / top;"),
-    ("query rotated by the untransposed matrix", "acc += rq->P[(int64_t)j * d + t] * (double)q[j];",
-     "acc += rq->P[(int64_t)t * d + j] * (double)q[j];"),
+    ("query rotated by the untransposed matrix", "acc += P[(int64_t)j * d + t] * (double)q[j];",
+     "acc += P[(int64_t)t * d + j] * (double)q[j];"),
 ]
 
 

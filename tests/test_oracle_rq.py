@@ -97,3 +97,30 @@ def test_rows_at_their_centroid_and_bounds(tiny):
     codes, f = oracle.rq_encode(idx2, synth.make_rotation(d, seed=4), 7)
     assert (codes[:3] == 64).all() and (f[:3] == 0).all()
     assert codes.max() <= 127 and np.isfinite(f).all() and (f[3:] > 0).all()
+
+
+def test_quantized_fragility_measures_the_estimates(deep):
+    """oracle_rq_fragility (the parity tests' allowance for the quantized
+    search) reports the distance of the nearest estimate from tau over the
+    searched partitions, and the centroid gaps of the exact ranking."""
+    w, c = deep, deep["cfg"]
+    idx = index_of(w)
+    d = idx["X"].shape[1]
+    P = synth.make_rotation(d, seed=6)
+    codes, f = oracle.rq_encode(idx, P, 7)
+    Q = w["Q"][:25]
+    qids = w["qids"][:25]
+    order = oracle.rank(Q, idx["centroids"], c.nprobe)
+    upto = np.full(len(Q), 5, np.int32)
+    tg, kg, cg = oracle.fragility(idx, Q, c.tau, c.k, c.nprobe, order, upto, qids=qids,
+                                  rq=(codes, f, P, 7))
+    tg0, _, cg0 = oracle.fragility(idx, Q, c.tau, c.k, c.nprobe, order, upto, qids=qids)
+    assert np.array_equal(cg, cg0)
+    mid = 63.5
+    C = idx["centroids"].astype(np.float64)
+    for i, q in enumerate(Q.astype(np.float64)):
+        qr = P.T @ q
+        rows = np.flatnonzero(np.isin(idx["assign"], order[i, :5]) & (idx["ids"] != qids[i]))
+        est = C[idx["assign"][rows]] @ q + f[rows].astype(np.float64) * (codes[rows] @ qr - mid * qr.sum())
+        assert abs(tg[i] - np.abs(est - np.float64(np.float32(c.tau))).min()) < 1e-9
+    assert not np.array_equal(tg, tg0)   # the estimates, not the exact similarities
