@@ -386,8 +386,9 @@ sieve_status sieve_rq_encode(const sieve_index_view *ix, const double *P, int32_
  *                  elements, 16 KB of fp16 (u - mid) in the byte order of the
  *                  shared-memory operand tile (2 bytes per element)
  *   rq_row_blocks  device [nlist+1] int64, block offsets of the partitions
- *   rq_factors     device [blocks * 128] fp32: the factors in the same block
- *                  order, 0 on the padding rows
+ *   rq_factors     device [blocks * 128] fp32: the factors x 2^-8 (an exact
+ *                  power-of-two scale, the scale of the scan's query split) in
+ *                  the same block order, 0 on the padding rows
  *   rq_rotation    the tensor-core layout of P^T (P rounded to fp32), used to
  *                  rotate the queries
  * sieve_rq_layout_size reads list_offsets from the device (synchronous);

@@ -158,6 +158,8 @@ struct RankMode {
                 }
             }
         }
+        __device__ void prefetch(const Args &, const Tile &, int) {}
+        __device__ void start(const Args &, const Tile &, int) {}
         __device__ void end(const Args &a, const Tile &) {
             if (ks) a.keep_n[keep_at] = kn;
         }

@@ -15,8 +15,8 @@
 //   k_rq_fill      the code layout the tensor-core scan streams: per block of
 //                  128 rows and K-block of 64 elements, 16 KB of fp16 (u - mid)
 //                  (half-integers, exact in fp16) in the swizzled byte order of
-//                  the shared-memory operand tile; and the factors in the same
-//                  block order, 0 on padding rows.
+//                  the shared-memory operand tile; and the factors x 2^-8 in
+//                  the same block order, 0 on padding rows.
 //   k_rq_rotate    q' = P^T q for a query batch on the tensor cores: the bulk
 //                  pipeline with the columns of P as B rows (the three-product
 //                  fp16 split of fp32), written out as fp32 rows.
@@ -160,7 +160,9 @@ __global__ void k_rq_fill(const uint8_t *__restrict__ codes, const float *__rest
         }
         unsigned char *dst = out + bk * (int64_t)tcb::kKbBytesHi + (int64_t)r * 128 + ((c ^ (r & 7)) << 4);
         *reinterpret_cast<uint4 *>(dst) = make_uint4(h[0], h[1], h[2], h[3]);
-        if (kb == 0 && c == 0) fac_out[blk * kTcRows + r] = valid ? factors[row] : 0.f;
+        // the factors scaled by 2^-8 (exact): the scan's accumulator holds
+        // <u - mid, q'> x 2^8, so f x 2^-8 turns it into f <u - mid, q'>
+        if (kb == 0 && c == 0) fac_out[blk * kTcRows + r] = valid ? factors[row] * (1.f / 256.f) : 0.f;
     }
 }
 
@@ -247,6 +249,8 @@ struct RotMode {
                         make_float4(v[4 * j] * tcp::kUnscale, v[4 * j + 1] * tcp::kUnscale,
                                     v[4 * j + 2] * tcp::kUnscale, v[4 * j + 3] * tcp::kUnscale);
         }
+        __device__ void prefetch(const Args &, const Tile &, int) {}
+        __device__ void start(const Args &, const Tile &, int) {}
         __device__ void end(const Args &, const Tile &) {}
     };
 };

@@ -26,7 +26,8 @@ struct ScanModeT {
     struct Tile {
         int p, ib, ni;
         int64_t r_begin, nb;
-        const float *fac;   // kRQ: the factors of p's rows (block order)
+        int64_t blk0;       // p's first block in the bulk layout (codes for kRQ)
+        const float *fac;   // kRQ: the factors x 2^-8 of p's rows (block order)
     };
     __device__ static int num_tiles(const Args &a) { return a.ctl->n_tc_tiles; }
     // tiles differ in cost (partition sizes are skewed): blocks draw them dynamically
@@ -41,7 +42,8 @@ struct ScanModeT {
         T.ni = x.z;
         T.r_begin = a.off[T.p];
         T.nb = a.off[T.p + 1] - T.r_begin;
-        T.fac = kRQ ? a.rq_fac + a.rq_row_blocks[T.p] * kTcRows : nullptr;
+        T.blk0 = kRQ ? a.rq_row_blocks[T.p] : (a.tc_row_blocks ? a.tc_row_blocks[T.p] : 0);
+        T.fac = kRQ ? a.rq_fac + T.blk0 * kTcRows : nullptr;
         return T;
     }
     __device__ static const float *a_row(const Args &a, const Tile &T, int i) {
@@ -52,8 +54,8 @@ struct ScanModeT {
         return r < T.nb ? a.X + (T.r_begin + r) * a.d : nullptr;
     }
     __device__ static const unsigned char *b_block(const Args &a, const Tile &T, int ch) {
-        if (kRQ) return a.rq_rows + (a.rq_row_blocks[T.p] + ch) * (int64_t)tc_nkb_dev(a.d) * tcb::kKbBytesHi;
-        return a.tc_rows + (a.tc_row_blocks[T.p] + ch) * (int64_t)tc_nkb_dev(a.d) * kTcBlockBytes;
+        if (kRQ) return a.rq_rows + (T.blk0 + ch) * (int64_t)tc_nkb_dev(a.d) * tcb::kKbBytesHi;
+        return a.tc_rows + (T.blk0 + ch) * (int64_t)tc_nkb_dev(a.d) * kTcBlockBytes;
     }
 
     struct Epi {
@@ -61,6 +63,7 @@ struct ScanModeT {
         long long *ki;
         int kn, item, q, rank, slot;
         float qc;   // kRQ: <q, c_p>, the centroid score of the item's rank
+        float *fs;  // kRQ: this warp's copy of the chunk's 128 factors (shared memory)
         bool valid;
         long long qid;
         // the kept list is unordered while the tile runs; once it holds k
@@ -83,6 +86,7 @@ struct ScanModeT {
             item = q = rank = 0;
             qid = (long long)-0x7fffffffffffffffll - 1;
             qc = 0.f;
+            fs = reinterpret_cast<float *>(smem + (size_t)tcp::kM * a.k * 12) + (slot >> 5) * 128;
             if (valid) {
                 item = a.bucketed[T.ib + slot];
                 q = a.item_q[item];
@@ -151,33 +155,49 @@ struct ScanModeT {
                 take(a, T, col0 + j, pick32(e, j) * inv);
             }
         }
+        // kRQ: the chunk's factors into this warp's shared copy, one coalesced
+        // 512-byte asynchronous copy per warp issued before the accumulator wait
+        __device__ __forceinline__ void prefetch(const Args &, const Tile &T, int ch) {
+            if constexpr (kRQ) {
+                __syncwarp();   // every lane is done with the previous chunk's copy
+                const float *src = T.fac + (int64_t)ch * tcb::kN + 4 * (slot & 31);
+                const uint32_t dst = tc::smem_u32(fs + 4 * (slot & 31));
+                asm volatile("cp.async.ca.shared.global [%0], [%1], 16;\n" ::"r"(dst), "l"(src) : "memory");
+            }
+        }
+        __device__ __forceinline__ void start(const Args &, const Tile &, int) {
+            if constexpr (kRQ) {
+                asm volatile("cp.async.wait_all;\n" ::: "memory");
+                __syncwarp();
+            }
+        }
         // v holds the chunk's raw accumulator values: exact, similarities x
         // 2^16; kRQ, <u - mid, q'> x 2^8 (the codes are not scaled)
         __device__ void chunk(const Args &a, const Tile &T, int64_t col0, const float (&v)[32],
                               int ncol) {
             if (!valid || ncol <= 0) return;
             if constexpr (kRQ) {
-                // the estimates qc + f <u - mid, q'> against the threshold,
-                // straight into a mask (no array of estimates stays live); the
-                // factor array covers whole blocks (0 on padding rows), so the
-                // 32 loads stay inside it
+                // the estimates qc + f <u - mid, q'> (the factor copy holds
+                // f x 2^-8, the scale of the accumulator: one fma each) against
+                // the threshold, straight into a mask; the rare candidates
+                // compute theirs again, with the same arithmetic
+                const float4 *f4 = reinterpret_cast<const float4 *>(fs + (col0 & (tcb::kN - 1)));
                 float thr = a.tau;
                 if (kn == a.k) thr = fmaxf(thr, wst_s);
-                const float4 *f4 = reinterpret_cast<const float4 *>(T.fac + col0);
                 unsigned m = 0;
 #pragma unroll
                 for (int j = 0; j < 8; ++j) {
-                    const float4 f = __ldg(f4 + j);
-                    m |= (fmaf(f.x, v[4 * j] * (1.f / 256.f), qc) >= thr) ? 1u << (4 * j) : 0u;
-                    m |= (fmaf(f.y, v[4 * j + 1] * (1.f / 256.f), qc) >= thr) ? 2u << (4 * j) : 0u;
-                    m |= (fmaf(f.z, v[4 * j + 2] * (1.f / 256.f), qc) >= thr) ? 4u << (4 * j) : 0u;
-                    m |= (fmaf(f.w, v[4 * j + 3] * (1.f / 256.f), qc) >= thr) ? 8u << (4 * j) : 0u;
+                    const float4 f = f4[j];
+                    m |= (fmaf(f.x, v[4 * j], qc) >= thr) ? 1u << (4 * j) : 0u;
+                    m |= (fmaf(f.y, v[4 * j + 1], qc) >= thr) ? 2u << (4 * j) : 0u;
+                    m |= (fmaf(f.z, v[4 * j + 2], qc) >= thr) ? 4u << (4 * j) : 0u;
+                    m |= (fmaf(f.w, v[4 * j + 3], qc) >= thr) ? 8u << (4 * j) : 0u;
                 }
                 if (ncol < 32) m &= (1u << ncol) - 1u;
-                while (m) {   // the rare candidates: the estimate again, the same arithmetic
+                while (m) {
                     const int j = __ffs(m) - 1;
                     m &= m - 1u;
-                    take(a, T, col0 + j, fmaf(T.fac[col0 + j], pick32(v, j) * (1.f / 256.f), qc));
+                    take(a, T, col0 + j, fmaf(fs[(col0 & (tcb::kN - 1)) + j], pick32(v, j), qc));
                 }
             } else {
                 select(a, T, col0, v, ncol, 65536.f);
@@ -254,10 +274,12 @@ void enqueue_scan_bulk(const SearchArgs &a, cudaStream_t st) {
                   tcb::smem_bytes(a.tc_stages, scan_epi_bytes(a.k)), st>>>(a);
 }
 
-// the scan over codes: 16 KB stages, up to eight
+// the scan over codes: stages of two 16 KB K-blocks; the epilogue's bytes add
+// one 512-byte factor copy per epilogue warp
+static size_t scan_rq_epi_bytes(int k) { return scan_epi_bytes(k) + 4 * 512; }
+
 int scan_rq_stages(int d, int k) {
-    return tcb::stages_for((int)ceil_div(d, 64), scan_epi_bytes(k), 232448 - 128, tcb::kKbBytesHi,
-                           tcb::kMaxStages);
+    return tcb::stages_for((int)ceil_div(d, 64), scan_rq_epi_bytes(k), 232448 - 128, tcb::kStageBytesHi);
 }
 
 __global__ void __launch_bounds__(tcb::kThreads, 1) k_scan_rq(SearchArgs a) {
@@ -267,11 +289,11 @@ __global__ void __launch_bounds__(tcb::kThreads, 1) k_scan_rq(SearchArgs a) {
 
 cudaError_t prepare_scan_rq(int d, int k, int stages) {
     return cudaFuncSetAttribute(k_scan_rq, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)tcb::smem_bytes(stages, scan_epi_bytes(k), tcb::kKbBytesHi));
+                                (int)tcb::smem_bytes(stages, scan_rq_epi_bytes(k), tcb::kStageBytesHi));
 }
 
 void enqueue_scan_rq(const SearchArgs &a, cudaStream_t st) {
-    k_scan_rq<<<num_sms(), tcb::kThreads, tcb::smem_bytes(a.tc_stages, scan_epi_bytes(a.k), tcb::kKbBytesHi),
+    k_scan_rq<<<num_sms(), tcb::kThreads, tcb::smem_bytes(a.tc_stages, scan_rq_epi_bytes(a.k), tcb::kStageBytesHi),
                 st>>>(a);
 }
 

@@ -5,7 +5,8 @@
 //
 // The B operand arrives pre-split, in tile byte order: one 32 KB bulk copy per
 // (block, K-block) lands a stage (hi then lo) in shared memory, up to five
-// stages deep, with no thread touching the bytes.  The tile's 128 A rows are
+// stages deep, with no thread touching the bytes.  B operands that are exact
+// in fp16 (codes) have no lo part: 16 KB per K-block, two K-blocks per stage.  The tile's 128 A rows are
 // split once per tile straight into tensor memory (lane i = A row i, two fp16
 // per 32-bit column, hi and lo of each K-block side by side), so shared memory
 // holds nothing but B stages and the epilogue's lists.
@@ -61,6 +62,9 @@ constexpr int kRing = 8;                      // tiles handed from the scheduler
 constexpr uint32_t kRingReaders = kAWriterWarps + 1 + 4;   // A-writer warps, MMA lane, epilogue warps
 
 constexpr uint32_t kKbBytesHi = 16384;        // one K-block of 128 rows with no lo part (codes)
+constexpr int kKbPerStageHi = 2;              // codes: two K-blocks per stage (one copy, one
+                                              // commit for 16 MMAs instead of 8)
+constexpr uint32_t kStageBytesHi = kKbPerStageHi * kKbBytesHi;
 
 // shared memory: 1 KB alignment slack, the B stages, the epilogue's bytes
 __host__ __device__ inline size_t smem_bytes(int stages, size_t epi_bytes,
@@ -99,7 +103,9 @@ __device__ __forceinline__ void hand(Epi &epi, const Args &a, const Tile &T, int
     epi.chunk(a, T, col0, v, left < 32 ? (int)left : 32);
 }
 
-// Mode provides (in addition to what tc_pipeline.cuh asks): b_block(a, T, ch)
+// Mode provides (in addition to what tc_pipeline.cuh asks): Epi::prefetch(a,
+// T, ch) and Epi::start(a, T, ch), called by every epilogue lane of a warp
+// before and after the wait for chunk ch's accumulator; b_block(a, T, ch)
 // = pointer to the tensor-layout bytes of the tile's ch-th block of B rows;
 // tile_counter(a) = a zeroed global int the blocks draw tiles from (nullptr:
 // block b takes tiles b, b + gridDim.x, ...).
@@ -108,7 +114,9 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                                          int stages) {
     constexpr uint32_t kIdesc = tc::idesc_f16(tcp::kM, kN);
     constexpr bool kLo = b_has_lo<Mode>::value;
-    constexpr uint32_t kStage = kLo ? kKbBytes : kKbBytesHi;   // bytes of one B stage
+    constexpr uint32_t kKbB = kLo ? kKbBytes : kKbBytesHi;     // bytes of one K-block of B
+    constexpr int kKs = kLo ? 1 : kKbPerStageHi;              // K-blocks per B stage
+    constexpr uint32_t kStage = kKs * kKbB;                    // bytes of one B stage
     __shared__ __align__(8) uint64_t a_full[kMaxKb], a_empty[kMaxKb], b_full[kMaxStages],
         b_empty[kMaxStages], dfull_bar[2], dempty_bar[2], drain_bar, ring_full[kRing],
         ring_empty[kRing];
@@ -230,12 +238,14 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                 const typename Mode::Tile T = Mode::tile(a, t);
                 const int nch = (int)ceil_div(T.nb, kN);
                 for (int ch = 0; ok && ch < nch; ++ch) {
+                    // a block's K-blocks are contiguous: a stage is one copy
                     const unsigned char *src = Mode::b_block(a, T, ch);
-                    for (int kb = 0; kb < nkb; ++kb) {
+                    for (int kb = 0; kb < nkb; kb += kKs) {
                         const uint32_t st = s % stages, sph = (s / stages) & 1u;
+                        const uint32_t bytes = (uint32_t)(nkb - kb < kKs ? nkb - kb : kKs) * kKbB;
                         if (!(ok = wait(&b_empty[st], sph ^ 1u))) break;
-                        tc::mbar_arrive_expect_tx(&b_full[st], kStage);
-                        tc::bulk_g2s(Bst + (size_t)st * kStage, src + (size_t)kb * kStage, kStage,
+                        tc::mbar_arrive_expect_tx(&b_full[st], bytes);
+                        tc::bulk_g2s(Bst + (size_t)st * kStage, src + (size_t)kb * kKbB, bytes,
                                      &b_full[st]);
                         ++s;
                     }
@@ -267,40 +277,46 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                     if (!(ok = wait(&dempty_bar[buf], dph ^ 1u))) break;
                     tc::fence_after_sync();
                     const uint32_t dt = tmem + buf * kN;
-                    for (int kb = 0; kb < nkb; ++kb, ++s) {
+                    for (int kb0 = 0; kb0 < nkb; kb0 += kKs, ++s) {
                         const uint32_t st = s % stages, ph = (s / stages) & 1u;
-                        if (ch == 0 && !(ok = wait(&a_full[kb], u & 1u))) break;
-                        if (!(ok = wait(&b_full[st], ph))) break;
+                        const int kb1 = nkb - kb0 < kKs ? nkb : kb0 + kKs;   // this stage's K-blocks
+                        if (ch == 0)
+                            for (int kb = kb0; ok && kb < kb1; ++kb) ok = wait(&a_full[kb], u & 1u);
+                        if (!ok || !(ok = wait(&b_full[st], ph))) break;
                         tc::fence_after_sync();
-                        const uint32_t a_hi = tA + (uint32_t)kb * 64, a_lo = a_hi + 32;
-                        const uint32_t b_hi = tc::smem_u32(Bst + (size_t)st * kStage);
-                        // a K step moves the descriptors' start address by 32 bytes
-                        // (2 in its 16-byte units; shared addresses stay far below
-                        // the field's 2^14 limit, so no carry)
-                        const uint64_t bh = tc::desc_k_sw128(b_hi);
-                        if constexpr (kLo) {
-                            const uint64_t bl = tc::desc_k_sw128(b_hi + kKbBytes / 2);
+                        for (int kb = kb0; kb < kb1; ++kb) {
+                            const uint32_t a_hi = tA + (uint32_t)kb * 64, a_lo = a_hi + 32;
+                            const uint32_t b_hi = tc::smem_u32(Bst + (size_t)st * kStage) +
+                                                  (uint32_t)(kb - kb0) * kKbB;
+                            // a K step moves the descriptors' start address by 32 bytes
+                            // (2 in its 16-byte units; shared addresses stay far below
+                            // the field's 2^14 limit, so no carry)
+                            const uint64_t bh = tc::desc_k_sw128(b_hi);
+                            if constexpr (kLo) {
+                                const uint64_t bl = tc::desc_k_sw128(b_hi + kKbBytes / 2);
 #pragma unroll
-                            for (int ks = 0; ks < 4; ++ks) {   // K = 16: 8 columns of A, 32 bytes of B
-                                const uint32_t ao = ks * 8;
-                                const uint64_t bo = 2 * ks;
-                                tc::mma_f16_ta(dt, a_lo + ao, bh + bo, kIdesc, (kb > 0 || ks > 0) ? 1u : 0u);
-                                tc::mma_f16_ta(dt, a_hi + ao, bl + bo, kIdesc, 1u);
-                                tc::mma_f16_ta(dt, a_hi + ao, bh + bo, kIdesc, 1u);
-                            }
-                        } else {   // B exact in fp16: hi and lo of A against it
+                                for (int ks = 0; ks < 4; ++ks) {   // K = 16: 8 columns of A, 32 bytes of B
+                                    const uint32_t ao = ks * 8;
+                                    const uint64_t bo = 2 * ks;
+                                    tc::mma_f16_ta(dt, a_lo + ao, bh + bo, kIdesc, (kb > 0 || ks > 0) ? 1u : 0u);
+                                    tc::mma_f16_ta(dt, a_hi + ao, bl + bo, kIdesc, 1u);
+                                    tc::mma_f16_ta(dt, a_hi + ao, bh + bo, kIdesc, 1u);
+                                }
+                            } else {   // B exact in fp16: hi and lo of A against it
 #pragma unroll
-                            for (int ks = 0; ks < 4; ++ks) {
-                                const uint32_t ao = ks * 8;
-                                const uint64_t bo = 2 * ks;
-                                tc::mma_f16_ta(dt, a_lo + ao, bh + bo, kIdesc, (kb > 0 || ks > 0) ? 1u : 0u);
-                                tc::mma_f16_ta(dt, a_hi + ao, bh + bo, kIdesc, 1u);
+                                for (int ks = 0; ks < 4; ++ks) {
+                                    const uint32_t ao = ks * 8;
+                                    const uint64_t bo = 2 * ks;
+                                    tc::mma_f16_ta(dt, a_lo + ao, bh + bo, kIdesc, (kb > 0 || ks > 0) ? 1u : 0u);
+                                    tc::mma_f16_ta(dt, a_hi + ao, bh + bo, kIdesc, 1u);
+                                }
                             }
                         }
                         tc::mma_commit(&b_empty[st]);
-                        // the tile's last reads of this K-block of A: it may be
+                        // the tile's last reads of these K-blocks of A: they may be
                         // overwritten by the next tile once they are done
-                        if (ch == nch - 1) tc::mma_commit(&a_empty[kb]);
+                        if (ch == nch - 1)
+                            for (int kb = kb0; kb < kb1; ++kb) tc::mma_commit(&a_empty[kb]);
                     }
                     if (ok) tc::mma_commit(&dfull_bar[buf]);
                 }
@@ -326,8 +342,10 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
             epi.begin(a, T, slot, epi_smem);
             for (int ch = 0; ch < nch; ++ch, ++c) {
                 const uint32_t buf = c & 1u, dph = (c >> 1) & 1u;
+                epi.prefetch(a, T, ch);   // per-chunk loads, in flight during the wait
                 ok = __all_sync(0xffffffffu, wait(&dfull_bar[buf], dph));
                 if (!ok) break;
+                epi.start(a, T, ch);
                 tc::fence_after_sync();
                 // two pairs of 32-column loads, each pair in flight together;
                 // the accumulator is released as soon as the second pair has
