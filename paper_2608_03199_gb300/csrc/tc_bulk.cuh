@@ -3,10 +3,10 @@
 // block of 128 B rows (a partition's rows, or the centroids), with the scaled
 // fp16 split of tc_pipeline.cuh and the same per-row epilogues.
 //
-// The B operand arrives pre-split, in tile byte order: one 32 KB bulk copy per
-// (block, K-block) lands a stage (hi then lo) in shared memory, up to five
-// stages deep, with no thread touching the bytes.  B operands that are exact
-// in fp16 (codes) have no lo part: 16 KB per K-block, two K-blocks per stage.  The tile's 128 A rows are
+// The B operand arrives pre-split, in tile byte order: a block's K-blocks (32 KB
+// each: hi then lo) are contiguous, and one bulk copy lands two of them as a
+// stage in shared memory, a few stages deep, with no thread touching the bytes.
+// B operands that are exact in fp16 (codes) have no lo part: 16 KB per K-block.  The tile's 128 A rows are
 // split once per tile straight into tensor memory (lane i = A row i, two fp16
 // per 32-bit column, hi and lo of each K-block side by side), so shared memory
 // holds nothing but B stages and the epilogue's lists.
@@ -52,8 +52,7 @@ constexpr int kMmaWarp = 9;
 constexpr int kThreads = 14 * 32;
 constexpr int kMaxKb = 4;                     // A in tensor memory: d <= 256
 constexpr int kMaxStages = 8;                 // barrier slots for B stages
-constexpr int kStages32 = 5;                  // 32 KB stages: five timed faster than six (more
-                                              // of the SM memory stays L1)
+constexpr int kStagesMax = 5;                 // stages beyond five did not time faster
 constexpr uint32_t kKbBytes = 32768;          // one K-block of 128 rows: hi 16 KB + lo 16 KB
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kAColumn0 = 2 * kN;        // A after the two accumulators
@@ -62,19 +61,21 @@ constexpr int kRing = 8;                      // tiles handed from the scheduler
 constexpr uint32_t kRingReaders = kAWriterWarps + 1 + 4;   // A-writer warps, MMA lane, epilogue warps
 
 constexpr uint32_t kKbBytesHi = 16384;        // one K-block of 128 rows with no lo part (codes)
-constexpr int kKbPerStageHi = 2;              // codes: two K-blocks per stage (one copy, one
-                                              // commit for 16 MMAs instead of 8)
-constexpr uint32_t kStageBytesHi = kKbPerStageHi * kKbBytesHi;
+constexpr int kKbPerStage = 2;                // two K-blocks per B stage: one copy and one
+                                              // commit per 24 (or 16) MMAs; timed 8-10%
+                                              // faster than one K-block per stage
+constexpr uint32_t kStageBytes = kKbPerStage * kKbBytes;       // 64 KB
+constexpr uint32_t kStageBytesHi = kKbPerStage * kKbBytesHi;   // 32 KB
 
 // shared memory: 1 KB alignment slack, the B stages, the epilogue's bytes
 __host__ __device__ inline size_t smem_bytes(int stages, size_t epi_bytes,
-                                             uint32_t stage_bytes = kKbBytes) {
+                                             uint32_t stage_bytes = kStageBytes) {
     return 1024 + (size_t)stages * stage_bytes + epi_bytes;
 }
 
 // B stages that fit beside the epilogue (0 when the pipeline does not apply)
-inline int stages_for(int nkb, size_t epi_bytes, size_t smem_limit, uint32_t stage_bytes = kKbBytes,
-                      int max_stages = kStages32) {
+inline int stages_for(int nkb, size_t epi_bytes, size_t smem_limit, uint32_t stage_bytes = kStageBytes,
+                      int max_stages = kStagesMax) {
     if (nkb > kMaxKb) return 0;
     const size_t base = smem_bytes(0, epi_bytes, stage_bytes);
     if (smem_limit < base) return 0;
@@ -115,7 +116,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
     constexpr uint32_t kIdesc = tc::idesc_f16(tcp::kM, kN);
     constexpr bool kLo = b_has_lo<Mode>::value;
     constexpr uint32_t kKbB = kLo ? kKbBytes : kKbBytesHi;     // bytes of one K-block of B
-    constexpr int kKs = kLo ? 1 : kKbPerStageHi;              // K-blocks per B stage
+    constexpr int kKs = kKbPerStage;                          // K-blocks per B stage
     constexpr uint32_t kStage = kKs * kKbB;                    // bytes of one B stage
     __shared__ __align__(8) uint64_t a_full[kMaxKb], a_empty[kMaxKb], b_full[kMaxStages],
         b_empty[kMaxStages], dfull_bar[2], dempty_bar[2], drain_bar, ring_full[kRing],
