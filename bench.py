@@ -146,16 +146,17 @@ def measured_peaks():
         return {}
 
 
-KERNEL_SOURCES = ("common.cuh", "search.cuh", "search_kernels.cu", "rank_kernel.cu",
-                  "scan_tc.cu", "tcgen05.cuh", "tc_bulk.cuh", "tc_pipeline.cuh", "rank_tc.cu",
-                  "tc_layout.cu", "rq.cu")
+# the sources that define each profiled kernel and the layout it streams
+_SCAN_SOURCES = ("common.cuh", "search.cuh", "scan_tc.cu", "tcgen05.cuh", "tc_bulk.cuh",
+                 "tc_pipeline.cuh", "tc_layout.cu", "rq.cu")
+KERNEL_SOURCES = {"k_scan_bulk": _SCAN_SOURCES, "k_scan_rq": _SCAN_SOURCES}
 
 
-def kernel_source_sha():
-    """Hash of the files that define the search kernels (not the host API)."""
+def kernel_source_sha(kernel):
+    """Hash of the files that define one kernel (not the host API)."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2608_03199_gb300", "csrc")
-    for f in KERNEL_SOURCES:
+    for f in KERNEL_SOURCES.get(kernel, ()):
         p = os.path.join(csrc, f)
         if os.path.exists(p):
             h.update(open(p, "rb").read())
@@ -173,7 +174,7 @@ def committed_traffic(kernel, workload, launches):
     except Exception:
         return None
     e = t.get(kernel, {}).get(workload)
-    if not e or e.get("source_sha") != kernel_source_sha():
+    if not e or e.get("source_sha") != kernel_source_sha(kernel):
         return None
     return e["dram_bytes_per_search"] / max(1, launches)
 

@@ -183,11 +183,8 @@ constexpr int kSelectWarps = 4;
 constexpr int kSelectMaxR = 8;   // lane order statistics used for the lower bracket
 constexpr int kSelectSmallC = 4; // candidate keys per lane of the two-step selection (P <= 64)
 
-__device__ __forceinline__ int warp_sum(int x) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-    return x;
-}
+// warp-wide reductions in one instruction (redux.sync), not a chain of shuffles
+__device__ __forceinline__ int warp_sum(int x) { return __reduce_add_sync(0xffffffffu, x); }
 
 template <int KPL>
 __device__ __forceinline__ int count_ge(const uint32_t (&key)[KPL], uint32_t t) {
@@ -244,11 +241,8 @@ __device__ __forceinline__ void warp_threshold(const uint32_t (&key)[KPL], int w
     uint32_t L = 0u;   // r > kSelectMaxR: no lower bracket
 #pragma unroll
     for (int i = 0; i < kSelectMaxR; ++i) L = r == i + 1 ? m[i] : L;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        U = max(U, __shfl_xor_sync(0xffffffffu, U, o));
-        L = min(L, __shfl_xor_sync(0xffffffffu, L, o));
-    }
+    U = __reduce_max_sync(0xffffffffu, U);
+    L = __reduce_min_sync(0xffffffffu, L);
     int b;
     if (L == U) {
         b = -1;
@@ -398,8 +392,11 @@ __device__ __forceinline__ void warp_gather_sort(const uint32_t (&key)[KPL], int
 // to nprobe.  `only` (nullable): queries with only[q] == 0 are skipped.
 // `seg_cnt` (nullable): [nq][nseg] entries actually present in each segment.
 // P: a power of two >= nprobe; the sort buffer holds 2P entries.
+// Eight blocks per SM (64 registers) where the keys fit: the selection is a chain
+// of dependent warp reductions, so it needs the warps to hide their latency
+// (timed 25% faster than 120 registers at four blocks).
 template <int KPL>   // entries per lane: seg <= 32 * KPL
-__global__ void __launch_bounds__(kSelectWarps * 32) k_select(
+__global__ void __launch_bounds__(kSelectWarps * 32, KPL >= 64 ? 4 : 8) k_select(
     const float *__restrict__ in_s, const int32_t *__restrict__ in_id, int64_t in_ld, int64_t nq,
     int64_t M, int seg, int nseg, int nprobe, int P, int32_t *__restrict__ out_id,
     float *__restrict__ out_s, int64_t out_ld, const int *__restrict__ only,
