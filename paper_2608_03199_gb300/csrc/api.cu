@@ -83,7 +83,7 @@ int64_t items_cap(int64_t nq, const sieve_params *p) {
 struct Layout {
     size_t ctl, order, S, E, counts, cursor, item_q, item_rank, item_p, bucketed, tiles, tc_tiles,
         active, res_cnt, res_s, res_id, rank_scratch;
-    size_t h_Q, h_qids, h_ids, h_scores, h_count, h_probes;
+    size_t h_Q, h_qids, h_ids, h_scores, h_count, h_probes, h_status;
     size_t qrot, cscores;   // quantized search: rotated queries, centroid scores
     size_t total;
     int64_t cap, max_tiles;
@@ -131,6 +131,7 @@ Layout make_layout(const sieve_index_view *ix, int64_t nq, const sieve_params *p
         L.h_scores = take((size_t)nq * p->k * 4);
         L.h_count = take((size_t)nq * 4);
         L.h_probes = take((size_t)nq * 4);
+        L.h_status = take(sizeof(int));
     }
     if (rq) {
         L.qrot = take((size_t)nq * ix->d * 4);
@@ -280,6 +281,40 @@ struct EventSet {
             if (x) cudaEventDestroy(x);
     }
 };
+
+// sieve_search_host's copy stream and events, one set per device and host
+// thread (created on first use, kept for the thread's life)
+constexpr int kHostChunks = 4;
+struct CopyLane {
+    bool ok = false;
+    cudaError_t err = cudaSuccess;
+    int device = -1;
+    cudaStream_t stream = nullptr;
+    cudaEvent_t start = nullptr, landed[kHostChunks] = {};
+};
+
+CopyLane &copy_lane() {
+    thread_local std::vector<CopyLane> lanes;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    static CopyLane failed;
+    if (e != cudaSuccess) {
+        failed.err = e;
+        return failed;
+    }
+    for (auto &l : lanes)
+        if (l.device == dev) return l;
+    CopyLane l;
+    l.device = dev;
+    e = cudaStreamCreateWithFlags(&l.stream, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&l.start, cudaEventDisableTiming);
+    for (int i = 0; e == cudaSuccess && i < kHostChunks; ++i)
+        e = cudaEventCreateWithFlags(&l.landed[i], cudaEventDisableTiming);
+    l.ok = e == cudaSuccess;
+    l.err = e;
+    lanes.push_back(l);
+    return lanes.back();
+}
 
 // the device-side search on device buffers (shared by sieve_search and
 // sieve_search_host); arguments already checked
@@ -754,17 +789,64 @@ sieve_status sieve_search_host(const sieve_index_view *ix, const float *Q_host, 
     float *dsc = reinterpret_cast<float *>(w + L.h_scores);
     int32_t *dcnt = reinterpret_cast<int32_t *>(w + L.h_count);
     int32_t *dpr = reinterpret_cast<int32_t *>(w + L.h_probes);
-    SIEVE_CUDA(cudaMemcpyAsync(dQ, Q_host, (size_t)nq * ix->d * 4, cudaMemcpyHostToDevice, st));
-    if (dqids)
+    int *dstatus = reinterpret_cast<int *>(w + L.h_status);
+    int32_t *dorder = reinterpret_cast<int32_t *>(w + L.order);
+    // The queries go to the device in chunks on a copy stream, and each
+    // chunk's centroid ranking starts as soon as it has landed, so the copy
+    // overlaps the ranking; the search then runs with the order it made.
+    // Chunks are multiples of 128 x (SMs) queries: whole waves of ranking tiles.
+    // (With profile = 1 the ranking stays inside the search, where it is timed.)
+    CopyLane &cl = copy_lane();
+    if (!cl.ok) return cuda_fail(cl.err);
+    const int64_t wave = (int64_t)128 * num_sms();
+    const int64_t chunk = round_up(ceil_div(nq, kHostChunks), wave);
+    const int nchunks = p->profile ? 0 : (int)std::min<int64_t>(kHostChunks, ceil_div(nq, chunk));
+    const bool rank_tc = p->scan_path != 1 && L.rank_scratch != 0;
+    SIEVE_CUDA(rank_tc ? prepare_rank_tc(p->nprobe, ix->d) : prepare_rank(p->nprobe));
+    SIEVE_CUDA(cudaMemsetAsync(dstatus, 0, sizeof(int), st));
+    SIEVE_CUDA(cudaEventRecord(cl.start, st));             // earlier work on the staging
+    SIEVE_CUDA(cudaStreamWaitEvent(cl.stream, cl.start, 0));
+    // the ids first: a copy queued behind the chunks on the same copy engine
+    // would hold the first chunk's ranking back until every chunk had landed
+    if (dqids && nchunks)
+        SIEVE_CUDA(cudaMemcpyAsync(dqids, query_ids_host, (size_t)nq * 8, cudaMemcpyHostToDevice,
+                                   cl.stream));
+    for (int c = 0; c < nchunks; ++c) {
+        const int64_t q0 = c * chunk, n = std::min<int64_t>(chunk, nq - q0);
+        SIEVE_CUDA(cudaMemcpyAsync(dQ + q0 * ix->d, Q_host + q0 * ix->d, (size_t)n * ix->d * 4,
+                                   cudaMemcpyHostToDevice, cl.stream));
+        SIEVE_CUDA(cudaEventRecord(cl.landed[c], cl.stream));
+    }
+    if (p->profile)
+        SIEVE_CUDA(cudaMemcpyAsync(dQ, Q_host, (size_t)nq * ix->d * 4, cudaMemcpyHostToDevice, st));
+    if (dqids && !nchunks)
         SIEVE_CUDA(cudaMemcpyAsync(dqids, query_ids_host, (size_t)nq * 8, cudaMemcpyHostToDevice, st));
-    rc = search_device(ix, dQ, nq, dqids, nullptr, p, dids, dsc, dcnt, dpr, stats, w, L, st);
+    int rank_launches = 0;
+    for (int c = 0; c < nchunks; ++c) {
+        const int64_t q0 = c * chunk, n = std::min<int64_t>(chunk, nq - q0);
+        SIEVE_CUDA(cudaStreamWaitEvent(st, cl.landed[c], 0));
+        if (rank_tc)
+            SIEVE_CUDA(enqueue_rank_tc(dQ + q0 * ix->d, n, ix->centroids, ix->nlist, ix->d, p->nprobe,
+                                       dorder + q0 * p->nprobe, nullptr,
+                                       reinterpret_cast<float *>(w + L.rank_scratch), dstatus, st,
+                                       static_cast<const unsigned char *>(ix->tc_centroids)));
+        else
+            SIEVE_CUDA(enqueue_rank(dQ + q0 * ix->d, n, ix->centroids, ix->nlist, ix->d, p->nprobe,
+                                    dorder + q0 * p->nprobe, nullptr, st));
+        rank_launches += rank_tc ? rank_tc_launches(n, ix->nlist, p->nprobe, ix->d) : 1;
+    }
+    rc = search_device(ix, dQ, nq, dqids, nchunks ? dorder : nullptr, p, dids, dsc, dcnt, dpr, stats,
+                       w, L, st);
     if (rc != SIEVE_OK) return rc;
     SIEVE_CUDA(cudaMemcpyAsync(out_ids_host, dids, (size_t)nq * p->k * 8, cudaMemcpyDeviceToHost, st));
     SIEVE_CUDA(cudaMemcpyAsync(out_scores_host, dsc, (size_t)nq * p->k * 4, cudaMemcpyDeviceToHost, st));
     SIEVE_CUDA(cudaMemcpyAsync(out_count_host, dcnt, (size_t)nq * 4, cudaMemcpyDeviceToHost, st));
     SIEVE_CUDA(cudaMemcpyAsync(out_probes_host, dpr, (size_t)nq * 4, cudaMemcpyDeviceToHost, st));
+    int rank_status = 0;
+    SIEVE_CUDA(cudaMemcpyAsync(&rank_status, dstatus, sizeof(int), cudaMemcpyDeviceToHost, st));
     SIEVE_CUDA(cudaStreamSynchronize(st));
-    return SIEVE_OK;
+    if (stats && nchunks > 0) stats->kernel_launches[SIEVE_K_RANK] = rank_launches;   // ran here
+    return rank_status != 0 ? rank_status : SIEVE_OK;
 }
 
 // ---------------------------------------------------------------------------

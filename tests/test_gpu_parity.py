@@ -13,6 +13,7 @@ import torch
 
 import oracle
 import paper_2608_03199_gb300 as sieve
+import synth
 from conftest import index_of
 from parity import TOL, assert_parity, compare
 
@@ -250,6 +251,25 @@ def test_given_order_and_host_variant(tiny, g_tiny, dev):
     for a, b, h in zip(base, given, host):
         assert torch.equal(a.cpu(), b.cpu())
         assert torch.equal(a.cpu(), h)
+
+
+def test_host_variant_uploads_in_chunks(dev):
+    """50K queries: sieve_search_host uploads them in three chunks, ranking each
+    as it lands (the copy overlaps the ranking); the results are the device
+    call's, bit for bit, on the tensor and the FP32 ranking."""
+    cfg = synth.scaled("tiny", n=60_000, nq=50_000, nlist=96, ncomp=96, seed=23)
+    w = synth.to_numpy(synth.make_workload(cfg, device="cpu"))
+    index = sieve.build_layout(torch.from_numpy(w["X"]).to(dev), torch.from_numpy(w["assign"]).to(dev),
+                               cfg.nlist, torch.from_numpy(w["centroids"]).to(dev))
+    Q = torch.from_numpy(w["Q"])
+    qids = torch.from_numpy(w["qids"])
+    for path in ("auto", "simt"):
+        base = sieve.search(index, Q.to(dev), cfg.tau, cfg.k, cfg.nprobe, cfg.W,
+                            query_ids=qids.to(dev), scan_path=path)
+        host = sieve.search_host(index, Q.pin_memory(), cfg.tau, cfg.k, cfg.nprobe, cfg.W,
+                                 query_ids_host=qids, scan_path=path)
+        for a, h in zip(base, host):
+            assert torch.equal(a.cpu(), h), path
 
 
 def test_stats_account_for_the_work(deep, g_deep):
