@@ -250,7 +250,13 @@ sieve_status sieve_search(const sieve_index_view *ix, const float *Q, int64_t nq
  * query_ids) to device staging inside the workspace, searches, copies the
  * results back and synchronizes `stream` before returning.  Pointers as in
  * sieve_search but host-side; workspace from
- * sieve_search_workspace_size(..., host_io = 1, ...). */
+ * sieve_search_workspace_size(..., host_io = 1, ...).  The queries go up in
+ * up to four chunks on a copy stream that the library creates once per device
+ * and host thread (with its events), and each chunk's centroid ranking runs on
+ * `stream` as soon as the chunk has landed, so the upload overlaps the
+ * ranking (with profile = 1 the upload is one copy and the ranking runs
+ * inside the search).  Q_host should be page-locked for the copies to be
+ * asynchronous. */
 sieve_status sieve_search_host(const sieve_index_view *ix, const float *Q_host, int64_t nq,
                                const int64_t *query_ids_host, const sieve_params *p,
                                int64_t *out_ids_host, float *out_scores_host,
