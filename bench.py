@@ -185,7 +185,13 @@ def roofline(prof, cfg, dev, bulk=True, rank_on_tensor=True, rq=False):
     runs as k_scan_bulk (else k_scan_tc) and the ranking as k_rank_bulk;
     rank_on_tensor: the ranking runs on the tensor cores (every scan path
     but the FP32 one)."""
-    km, kl = prof["kernel_ms"], prof["kernel_launches"]
+    km, kl = dict(prof["kernel_ms"]), dict(prof["kernel_launches"])
+    # the ranking's contraction is timed on its own ("rank_mma", a part of
+    # "rank"); the rest of "rank" is its selection
+    if km.get("rank_mma", 0) > 0:
+        km["rank_select"] = km["rank"] - km["rank_mma"]
+        kl["rank_select"] = kl["rank"] - kl["rank_mma"]
+        del km["rank"], kl["rank"]
     top = max(km, key=lambda k: km[k])
     props = torch.cuda.get_device_properties(dev)
     peaks = measured_peaks()
@@ -228,21 +234,41 @@ def roofline(prof, cfg, dev, bulk=True, rank_on_tensor=True, rq=False):
                                f"x {clock_mhz:.0f} MHz (measured max clock)",
                    hbm_view={"achieved_gbs": bytes_ / launches / (ms_per_launch * 1e-3) / 1e9,
                              "peak_gbs": hbm})
-    elif top == "rank" and rank_on_tensor:
-        # the score contraction of the ranking (tensor cores, three fp16
-        # products per score) plus its selection kernels, timed together
+    elif top == "rank_mma":
+        # the score contraction of the ranking alone (tensor cores, three fp16
+        # products per score); its algorithmic work is every query-centroid
+        # score once, spread over its launches (a maxima pass and a keeping
+        # pass each compute every score when the ranking has no score table)
         name = "k_rank_bulk" if bulk else "k_rank_tc"
         flops = 2.0 * cfg.nq * cfg.nlist * d
-        ach = flops / (ms_per_launch * 1e-3) / 1e12
+        ach = flops / launches / (ms_per_launch * 1e-3) / 1e12
+        ng = -(-cfg.nlist // 32)   # 32-centroid groups
+        # no score table (d <= 128 under the group threshold): two passes
+        passes = 2 if (d <= 128 and cfg.nlist > 2048 and cfg.nprobe <= ng <= 2048) else 1
         out.update(kernel=name, bound="tensor", achieved=ach, peak=f16_tflops / 3,
                    unit="TFLOP/s", frac=ach / (f16_tflops / 3),
                    peak_source=(f"fp16 split: three kind::f16 MMAs per score; fp16 dense peak "
                                 f"{f16_tflops:.0f} TFLOP/s = measured bf16 cuBLAS burst (of "
-                                f"measured), a third of it; the time includes the selection"),
+                                f"measured), a third of it"),
+                   passes=passes, tensor_pipe_tflops=3 * passes * ach,
+                   rank_select_ms=km.get("rank_select"))
+    elif top == "rank_select":
+        out.update(kernel="ranking selection (k_select / k_compact_final)", bound="alu",
+                   achieved=None, peak=None, unit=None, frac=None)
+    elif top == "rank" and rank_on_tensor:
+        name = "k_rank_bulk" if bulk else "k_rank_tc"
+        flops = 2.0 * cfg.nq * cfg.nlist * d
+        ach = flops / (km[top] * 1e-3) / 1e12
+        out.update(kernel=name + " + selection", bound="tensor", achieved=ach, peak=f16_tflops / 3,
+                   unit="TFLOP/s", frac=ach / (f16_tflops / 3),
+                   peak_source=(f"fp16 split: three kind::f16 MMAs per score; fp16 dense peak "
+                                f"{f16_tflops:.0f} TFLOP/s = measured bf16 cuBLAS burst (of "
+                                f"measured), a third of it; the time is every launch of the "
+                                f"ranking, selection included"),
                    tensor_pipe_tflops=3 * ach)
     elif top == "rank":
         flops = 2.0 * cfg.nq * cfg.nlist * d
-        ach = flops / (ms_per_launch * 1e-3) / 1e12
+        ach = flops / (km[top] * 1e-3) / 1e12
         out.update(bound="alu", achieved=ach, peak=fp32_tflops, unit="TFLOP/s",
                    frac=ach / fp32_tflops,
                    peak_source=f"FP32 FMA: {props.multi_processor_count} SMs x 128 lanes x 2 "
@@ -484,7 +510,8 @@ def run_sieve(args, cfg, world, rank, local):
                     "mean_group": prof["items"] / max(1, prof["groups"]),
                     "pairs": prof["pairs"], "rows_read": prof["rows_read"],
                     "pairs_tc": prof["pairs_tc"], "rows_read_tc": prof["rows_read_tc"]},
-        "gpu_launches": args.steps * int(sum(prof["kernel_launches"].values())),
+        "gpu_launches": args.steps * int(sum(v for k, v in prof["kernel_launches"].items()
+                                             if k != "rank_mma")),
         "clocks": clock_rec,
         "e2e": e2e,
     }
@@ -700,7 +727,8 @@ def run_rq(args, cfg):
         "roofline": roofline(prof, cfg, dev, bulk=True, rq=True),
         "profile": {"kernel_ms": prof["kernel_ms"], "kernel_launches": prof["kernel_launches"],
                     "rounds": prof["rounds"], "items": prof["items"], "pairs": prof["pairs"]},
-        "gpu_launches": args.steps * int(sum(prof["kernel_launches"].values())),
+        "gpu_launches": args.steps * int(sum(v for k, v in prof["kernel_launches"].items()
+                                             if k != "rank_mma")),
         "clocks": clock_rec,
     }
     if not args.skip_cpu_baseline:

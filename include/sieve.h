@@ -122,8 +122,10 @@ typedef struct {
  * centroid ranking, state initialisation, the issuer, the ready-queue
  * bucketing, the scatter into partition groups, the grouped scan with its
  * fused epilogue on FP32 FMA, the per-query merge, the end-of-round step,
- * finalisation, the grouped scan on the tensor cores, and the query rotation
- * of the quantized search (sieve_rq_search). */
+ * finalisation, the grouped scan on the tensor cores, the query rotation
+ * of the quantized search (sieve_rq_search), and the score contraction of
+ * the tensor-core ranking alone (its launches are also counted, and its time
+ * included, under SIEVE_K_RANK). */
 enum {
     SIEVE_K_RANK = 0,
     SIEVE_K_INIT,
@@ -136,6 +138,7 @@ enum {
     SIEVE_K_FINALIZE,
     SIEVE_K_SCAN_TC,
     SIEVE_K_RQ_ROTATE,
+    SIEVE_K_RANK_MMA,
     SIEVE_NKERNELS
 };
 

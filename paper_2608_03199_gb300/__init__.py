@@ -59,7 +59,7 @@ class StatsC(C.Structure):
                 ("tiles", C.c_int64), ("rows_read", C.c_int64), ("pairs", C.c_int64),
                 ("rows_read_tc", C.c_int64), ("pairs_tc", C.c_int64),
                 ("status", C.c_int32), ("reserved0", C.c_int32),
-                ("kernel_ms", C.c_float * 11), ("kernel_launches", C.c_int32 * 11)]
+                ("kernel_ms", C.c_float * 12), ("kernel_launches", C.c_int32 * 12)]
 
 
 class RqViewC(C.Structure):
@@ -69,7 +69,7 @@ class RqViewC(C.Structure):
 
 
 KERNELS = ("rank", "init", "issue", "bucket", "scatter", "scan", "merge", "round_end", "finalize",
-           "scan_tc", "rq_rotate")
+           "scan_tc", "rq_rotate", "rank_mma")
 SCAN_PATHS = {"auto": 0, "simt": 1, "tensor": 2}
 
 

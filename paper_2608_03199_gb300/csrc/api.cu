@@ -169,11 +169,13 @@ constexpr size_t kGraphCacheMax = 8;
 
 // the centroid ranking of a search: the tensor-core kernel when it applies,
 // reporting a bounded wait that gives up in the search's status word
-cudaError_t launch_search_rank(const SearchArgs &a, int rank_tc, cudaStream_t st) {
+// (mma_ms, nullable: the contraction's own time is added there; the call syncs)
+cudaError_t launch_search_rank(const SearchArgs &a, int rank_tc, cudaStream_t st,
+                               float *mma_ms = nullptr) {
     int32_t *order = const_cast<int32_t *>(a.order);
     if (rank_tc)
         return enqueue_rank_tc(a.Q, a.nq, a.C, a.nlist, a.d, a.nprobe, order, a.cscores,
-                               a.rank_scratch, &a.ctl->status, st, a.tc_cent);
+                               a.rank_scratch, &a.ctl->status, st, a.tc_cent, mma_ms);
     return enqueue_rank(a.Q, a.nq, a.C, a.nlist, a.d, a.nprobe, order, a.cscores, st);
 }
 
@@ -459,7 +461,9 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
         SIEVE_CUDA(timed(SIEVE_K_INIT, [&] { return launch_init(a, st); }));
         if (a.rq) SIEVE_CUDA(timed(SIEVE_K_RQ_ROTATE, [&] { return launch_search_rotate(a, st); }));
         if (with_rank)
-            SIEVE_CUDA(timed(SIEVE_K_RANK, [&] { return launch_search_rank(a, rank_tc, st); }));
+            SIEVE_CUDA(timed(SIEVE_K_RANK, [&] {
+                return launch_search_rank(a, rank_tc, st, p->profile ? &ms[SIEVE_K_RANK_MMA] : nullptr);
+            }));
         for (;;) {
             SIEVE_CUDA(launch_round(a, smem, blocks, 0, 0, st, p->profile ? ev.e : nullptr));
             int more = 0;
@@ -503,6 +507,8 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
         for (int slot : per_round) stats->kernel_launches[slot] = c.round;
         stats->kernel_launches[SIEVE_K_SCAN_TC] = a.tc_min > 0 ? c.round : 0;
         stats->kernel_launches[SIEVE_K_RQ_ROTATE] = a.rq ? 1 : 0;
+        stats->kernel_launches[SIEVE_K_RANK_MMA] =
+            with_rank && rank_tc ? rank_tc_mma_launches(a.nq, a.nlist, a.nprobe, a.d) : 0;
         if (a.tc_min == 1) stats->kernel_launches[SIEVE_K_SCAN] = 0;
         if (c.status != 0) return c.status;
     }
@@ -821,7 +827,7 @@ sieve_status sieve_search_host(const sieve_index_view *ix, const float *Q_host, 
         SIEVE_CUDA(cudaMemcpyAsync(dQ, Q_host, (size_t)nq * ix->d * 4, cudaMemcpyHostToDevice, st));
     if (dqids && !nchunks)
         SIEVE_CUDA(cudaMemcpyAsync(dqids, query_ids_host, (size_t)nq * 8, cudaMemcpyHostToDevice, st));
-    int rank_launches = 0;
+    int rank_launches = 0, mma_launches = 0;
     for (int c = 0; c < nchunks; ++c) {
         const int64_t q0 = c * chunk, n = std::min<int64_t>(chunk, nq - q0);
         SIEVE_CUDA(cudaStreamWaitEvent(st, cl.landed[c], 0));
@@ -834,6 +840,7 @@ sieve_status sieve_search_host(const sieve_index_view *ix, const float *Q_host, 
             SIEVE_CUDA(enqueue_rank(dQ + q0 * ix->d, n, ix->centroids, ix->nlist, ix->d, p->nprobe,
                                     dorder + q0 * p->nprobe, nullptr, st));
         rank_launches += rank_tc ? rank_tc_launches(n, ix->nlist, p->nprobe, ix->d) : 1;
+        mma_launches += rank_tc ? rank_tc_mma_launches(n, ix->nlist, p->nprobe, ix->d) : 0;
     }
     rc = search_device(ix, dQ, nq, dqids, nchunks ? dorder : nullptr, p, dids, dsc, dcnt, dpr, stats,
                        w, L, st);
@@ -845,7 +852,10 @@ sieve_status sieve_search_host(const sieve_index_view *ix, const float *Q_host, 
     int rank_status = 0;
     SIEVE_CUDA(cudaMemcpyAsync(&rank_status, dstatus, sizeof(int), cudaMemcpyDeviceToHost, st));
     SIEVE_CUDA(cudaStreamSynchronize(st));
-    if (stats && nchunks > 0) stats->kernel_launches[SIEVE_K_RANK] = rank_launches;   // ran here
+    if (stats && nchunks > 0) {   // ran here
+        stats->kernel_launches[SIEVE_K_RANK] = rank_launches;
+        stats->kernel_launches[SIEVE_K_RANK_MMA] = mma_launches;
+    }
     return rank_status != 0 ? rank_status : SIEVE_OK;
 }
 

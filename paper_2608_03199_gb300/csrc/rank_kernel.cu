@@ -91,10 +91,28 @@ __device__ __forceinline__ void warp_merge_list(float *Ls, int *Lc, int *n_ptr, 
     __syncwarp();
 }
 
+// QT query rows of Q given by row index (rows >= nrows and columns >= d are
+// zero-filled): DK columns from c0 into Xs[QT][LDX], like stage_rows
+__device__ __forceinline__ void stage_query_rows(float *Xs, const float *__restrict__ Q,
+                                                 const int64_t *qrow, int nrows, int d, int c0) {
+    constexpr int kVec = DK / 4;
+    for (int idx = threadIdx.x; idx < QT * kVec; idx += kThreads) {
+        const int r = idx / kVec, v = idx % kVec;
+        const int col = c0 + 4 * v;
+        const bool ok = r < nrows && col < d;
+        const float *src = ok ? Q + qrow[r] * (int64_t)d + col : Q;
+        cp_async16(Xs + r * LDX + 4 * v, src, ok ? 16 : 0);
+    }
+}
+
+// qlist (nullable): rank only the queries qlist[0 .. *qlist_n - 1] (rows of Q
+// and of order/cscores); block b takes list entries b*QT .. b*QT+QT-1
 __global__ void __launch_bounds__(kThreads) k_rank(const float *__restrict__ Q, int64_t nq,
                                                    const float *__restrict__ C, int64_t nlist,
                                                    int d, int nprobe, int32_t *__restrict__ order,
-                                                   float *__restrict__ cscores) {
+                                                   float *__restrict__ cscores,
+                                                   const int *__restrict__ qlist,
+                                                   const int *__restrict__ qlist_n) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     __shared__ int list_n[QT];
     float *Qst = reinterpret_cast<float *>(smem_raw);
@@ -108,16 +126,22 @@ __global__ void __launch_bounds__(kThreads) k_rank(const float *__restrict__ Q, 
                   (threadIdx.x >> 5) * (2 * nprobe);
     int *oc_w = reinterpret_cast<int *>(os_w + nprobe);
 
+    __shared__ int64_t qrow[QT];   // the block's queries (rows of Q and of order)
     const int tid = threadIdx.x, tq = tid & 7, tr = tid >> 3;
     const unsigned lane = lane_id(), warp = tid >> 5;
     const int64_t q0 = (int64_t)blockIdx.x * QT;
-    const int nqb = (int)(nq - q0 < QT ? nq - q0 : QT);
-    const float *Qb = Q + q0 * d;
-    if (tid < QT) list_n[tid] = 0;
+    const int64_t nsel = qlist ? (int64_t)*qlist_n : nq;
+    if (q0 >= nsel) return;
+    const int nqb = (int)(nsel - q0 < QT ? nsel - q0 : QT);
+    if (tid < QT) {
+        list_n[tid] = 0;
+        qrow[tid] = tid < nqb ? (qlist ? (int64_t)qlist[q0 + tid] : q0 + tid) : 0;
+    }
+    __syncthreads();
 
     const int nch = (int)ceil_div(d, DK);
     const int64_t nsteps = ceil_div(nlist, RT) * nch;
-    stage_rows<QT>(Qst, Qb, nqb, d, 0, 0);
+    stage_query_rows(Qst, Q, qrow, nqb, d, 0);
     stage_rows<RT>(Cst, C, nlist, d, 0, 0);
     cp_async_commit();
     float acc[4][4];
@@ -127,7 +151,7 @@ __global__ void __launch_bounds__(kThreads) k_rank(const float *__restrict__ Q, 
         if (s + 1 < nsteps) {
             const int64_t s1 = s + 1;
             const int b1 = (int)(s1 & 1);
-            stage_rows<QT>(Qst + b1 * QT * LDX, Qb, nqb, d, 0, (int)(s1 % nch) * DK);
+            stage_query_rows(Qst + b1 * QT * LDX, Q, qrow, nqb, d, (int)(s1 % nch) * DK);
             stage_rows<RT>(Cst + b1 * RT * LDX, C, nlist, d, (s1 / nch) * RT, (int)(s1 % nch) * DK);
             cp_async_commit();
             cp_async_wait<1>();
@@ -199,8 +223,8 @@ __global__ void __launch_bounds__(kThreads) k_rank(const float *__restrict__ Q, 
     }
     for (int i = warp; i < nqb; i += kThreads / 32) {
         for (int j = lane; j < nprobe; j += 32) {
-            order[(q0 + i) * nprobe + j] = lc[i * nprobe + j];
-            if (cscores) cscores[(q0 + i) * nprobe + j] = ls[i * nprobe + j];
+            order[qrow[i] * nprobe + j] = lc[i * nprobe + j];
+            if (cscores) cscores[qrow[i] * nprobe + j] = ls[i * nprobe + j];
         }
     }
 }
@@ -211,11 +235,12 @@ cudaError_t prepare_rank(int nprobe) {
 }
 
 cudaError_t enqueue_rank(const float *Q, int64_t nq, const float *C, int64_t nlist, int d,
-                         int nprobe, int32_t *order, float *cscores, cudaStream_t st) {
+                         int nprobe, int32_t *order, float *cscores, cudaStream_t st,
+                         const int *qlist, const int *qlist_n) {
     if (nq == 0) return cudaSuccess;
     const int64_t blocks = ceil_div(nq, QT);
     k_rank<<<(unsigned)blocks, kThreads, rank_smem_bytes(nprobe), st>>>(Q, nq, C, nlist, d, nprobe,
-                                                                       order, cscores);
+                                                                       order, cscores, qlist, qlist_n);
     return cudaGetLastError();
 }
 

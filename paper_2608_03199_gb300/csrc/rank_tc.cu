@@ -7,14 +7,26 @@
 //              centroids' tensor-core layout, else the converter pipeline of
 //              tc_pipeline.cuh): a tile is 128 consecutive queries (A rows)
 //              against one range of kRankRange centroids (B rows, 128 per
-//              chunk); each epilogue thread stores its query's scores into a
-//              score table [queries][ld] in the caller's workspace
+//              chunk); each epilogue thread owns one query's scores and stores
+//              them into a score table, or only the maxima of 32-centroid
+//              groups, or only the scores that reach the query's threshold
 //   k_select   one warp per (query, segment of at most kSelectSeg entries):
 //              the segment's best min(nprobe, size) entries, sorted by
-//              (score desc, id asc).  With nlist <= kSelectSeg one segment
-//              gives the order directly; otherwise each level keeps the best
-//              nprobe of every segment (the nprobe best of a set lie among the
-//              nprobe best of each of its parts) until one segment is left.
+//              (score desc, id asc): a threshold refined bit by bit over the
+//              keys in registers picks exactly that many, and a bitonic
+//              network in registers sorts them.  With nlist <= kSelectSeg one
+//              segment gives the order directly.
+// More centroids: the nprobe-th largest of the 32-centroid group maxima is a
+// threshold that at least nprobe scores reach (k_group_threshold); the scores
+// that reach it are compacted per 2,048-centroid range (from the table by
+// k_compact_seg, or kept by a second contraction when d <= 128) and one warp
+// per query selects and sorts the nprobe best of them (k_compact_final).  A
+// query whose candidates overflow their slots is listed and finished exactly:
+// by levels of k_select over its table row (the nprobe best of a set lie among
+// the nprobe best of each of its parts), or by the FP32 ranking of
+// rank_kernel.cu when there is no table.
+#include <vector>
+
 #include "tc_bulk.cuh"
 #include "tc_pipeline.cuh"
 
@@ -50,9 +62,10 @@ struct RankArgs {
     int64_t gld;
     int mode;                // kRankTable, kRankMax or kRankKeep
     const uint32_t *lkey;    // kRankKeep: [nq] threshold keys
-    float *keep_s;           // kRankKeep: [nq][nranges][kRankRange] kept scores, per range
+    float *keep_s;           // kRankKeep: [nq][nranges][keep_cap] kept scores, per range
     int32_t *keep_i;         //            and their centroid ids, in id order
-    int *keep_n;             //            [nq][nranges] how many each range kept
+    int *keep_n;             //            [nq][nranges] how many each range had (even past keep_cap)
+    int keep_cap;            //            slots per range
 };
 
 // what the ranking contraction's epilogue does with a query's scores:
@@ -116,8 +129,8 @@ struct RankMode {
             keep_at = 0;
             if (valid && a.mode == kRankKeep) {
                 keep_at = q * n_ranges(a) + T.c0 / kRankRange;
-                ks = a.keep_s + keep_at * kRankRange;
-                ki = a.keep_i + keep_at * kRankRange;
+                ks = a.keep_s + keep_at * a.keep_cap;
+                ki = a.keep_i + keep_at * a.keep_cap;
                 thr_raw = key_score(a.lkey[q]) * 65536.f;   // exact: a power-of-two scale
             }
         }
@@ -138,22 +151,20 @@ struct RankMode {
                 grow[col0 / 32] = mx * kS;
             }
             if (ks) {   // the scores that reach the threshold, in id order
-                float mx[16];
-#pragma unroll
-                for (int j = 0; j < 16; ++j) mx[j] = fmaxf(v[j], v[j + 16]);
-#pragma unroll
-                for (int w = 8; w > 0; w >>= 1)
-#pragma unroll
-                    for (int j = 0; j < w; ++j) mx[j] = fmaxf(mx[j], mx[j + w]);
-                if (!(mx[0] >= thr_raw)) return;
+                // (a mask straight from the compares: some lane of a warp
+                // nearly always has a candidate in a group, so a maximum
+                // test first would not let the warp skip the group)
                 unsigned m = 0;
 #pragma unroll
-                for (int j = 0; j < 32; ++j) m |= (v[j] >= thr_raw && j < ncol) ? (1u << j) : 0u;
-                while (m) {   // at most kRankRange per range: the slots cannot overflow
+                for (int j = 0; j < 32; ++j) m |= v[j] >= thr_raw ? (1u << j) : 0u;
+                if (ncol < 32) m &= (1u << ncol) - 1u;
+                while (m) {   // counted past keep_cap: an overflow is seen, not lost
                     const int j = __ffs(m) - 1;
                     m &= m - 1u;
-                    ks[kn] = pick32(v, j) * kS;
-                    ki[kn] = (int32_t)(T.c0 + col0 + j);
+                    if (kn < a.keep_cap) {
+                        ks[kn] = pick32(v, j) * kS;
+                        ki[kn] = (int32_t)(T.c0 + col0 + j);
+                    }
                     ++kn;
                 }
             }
@@ -181,7 +192,8 @@ __global__ void __launch_bounds__(tcb::kThreads, 1) k_rank_bulk(RankArgs a, int 
 
 constexpr int kSelectWarps = 4;
 constexpr int kSelectMaxR = 8;   // lane order statistics used for the lower bracket
-constexpr int kSelectSmallC = 4; // candidate keys per lane of the two-step selection (P <= 64)
+constexpr int kStage2 = 16;      // keys per lane of the second selection step (512 entries)
+constexpr int kGroupMax = 2048;  // group maxima one threshold warp holds (64 per lane)
 
 // warp-wide reductions in one instruction (redux.sync), not a chain of shuffles
 __device__ __forceinline__ int warp_sum(int x) { return __reduce_add_sync(0xffffffffu, x); }
@@ -194,15 +206,13 @@ __device__ __forceinline__ int count_ge(const uint32_t (&key)[KPL], uint32_t t) 
     return warp_sum(c);
 }
 
-// A threshold T <= T* (T* = the want-th largest of the warp's keys; keys of
-// padding are 0, below every score) with C = #{keys >= T} >= want, refined
-// bit by bit (the largest T with at least want keys >= T) until C <= cap or
-// T == T*.  The search starts from the common high bits of a bracket
-// L <= T* <= U: U = the largest key, L = the smallest over lanes of each
-// lane's ceil(want / 32)-th largest key (at least want keys are >= L).
+// A bracket L <= T* <= U of the want-th largest of the warp's keys (keys of
+// padding are 0, below every score): U = the largest key, L = the smallest over
+// lanes of each lane's ceil(want / 32)-th largest key, so at least want keys
+// are >= L.  L = 0 when that rank is past kSelectMaxR.
 template <int KPL>
-__device__ __forceinline__ void warp_threshold(const uint32_t (&key)[KPL], int want, int cap,
-                                               uint32_t &T, int &C) {
+__device__ __forceinline__ void warp_bracket(const uint32_t (&key)[KPL], int want, uint32_t &L,
+                                             uint32_t &U) {
     const int r = (want + 31) / 32;
     uint32_t m[kSelectMaxR] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
     if (r <= 2) {
@@ -237,12 +247,22 @@ __device__ __forceinline__ void warp_threshold(const uint32_t (&key)[KPL], int w
 #pragma unroll
         for (int j = 0; j < KPL; ++j) m[0] = max(m[0], key[j]);
     }
-    uint32_t U = m[0];
-    uint32_t L = 0u;   // r > kSelectMaxR: no lower bracket
+    L = 0u;
 #pragma unroll
     for (int i = 0; i < kSelectMaxR; ++i) L = r == i + 1 ? m[i] : L;
-    U = __reduce_max_sync(0xffffffffu, U);
+    U = __reduce_max_sync(0xffffffffu, m[0]);
     L = __reduce_min_sync(0xffffffffu, L);
+}
+
+// A threshold T <= T* (T* = the want-th largest of the warp's keys) with C =
+// #{keys >= T} >= want, refined bit by bit (the largest T with at least want
+// keys >= T) until C <= cap or T == T*.  The search starts from the common
+// high bits of the bracket L, U.
+template <int KPL>
+__device__ __forceinline__ void warp_threshold(const uint32_t (&key)[KPL], int want, int cap,
+                                               uint32_t &T, int &C) {
+    uint32_t L, U;
+    warp_bracket(key, want, L, U);
     int b;
     if (L == U) {
         b = -1;
@@ -262,220 +282,244 @@ __device__ __forceinline__ void warp_threshold(const uint32_t (&key)[KPL], int w
     }
 }
 
-// The want best of the warp's cnt entries (entry c = key[c / 32] of lane
-// c % 32; its id from id_of(c)), sorted by (score desc, id asc) into bs/bc,
-// given T and C from warp_threshold.  C <= cap: every key >= T is a candidate;
-// otherwise T == T* and the keys > T* plus the first keys equal to it in entry
-// order are taken, which are the lowest ids when entry order is id order among
-// equal scores.  bs/bc hold 2P >= cap entries; returns the count sorted.
-template <int KPL, class IdOf>
-__device__ __forceinline__ void warp_gather_sort(const uint32_t (&key)[KPL], int cnt, int want,
-                                                 uint32_t T, int C, int cap, IdOf id_of,
-                                                 float *bs, int *bc) {
+// Bitonic sort of the warp's R * 32 entries (entry i = r * 32 + lane in
+// register r), first-ranked first by (score desc, id asc).  Partners within a
+// register are exchanged by shuffles, partners across registers in place.
+// Entries are distinct except identical padding, so both sides of a pair
+// take the same decision.
+template <int R>
+__device__ __forceinline__ void warp_sort_regs(float (&s)[R], int (&c)[R]) {
     const int lane = threadIdx.x & 31;
-    const unsigned below = (1u << lane) - 1u;
-    int pos = 0;
-    // the buffer holds cap entries: C <= cap, or exactly want <= cap taken
-    // below; the bound on p only keeps a broken invariant from writing past it
-    if (C <= cap) {
 #pragma unroll
-        for (int j = 0; j < KPL; ++j) {
-            const int c = j * 32 + lane;
-            const bool sel = key[j] >= T && c < cnt;
-            const unsigned sb = __ballot_sync(0xffffffffu, sel);
-            if (sel) {
-                const int p = pos + __popc(sb & below);
-                if (p < cap) {
-                    bs[p] = key_score(key[j]);
-                    bc[p] = id_of(c);
-                }
-            }
-            pos += __popc(sb);
-        }
-    } else {
-        int gt = 0;
+    for (int k = 2; k <= 32 * R; k <<= 1) {
 #pragma unroll
-        for (int j = 0; j < KPL; ++j) gt += key[j] > T;
-        const int ties_wanted = want - warp_sum(gt);   // >= 1
-        int ties_seen = 0;
-#pragma unroll
-        for (int j = 0; j < KPL; ++j) {
-            const int c = j * 32 + lane;
-            const bool tie = key[j] == T && c < cnt;
-            const unsigned tb = __ballot_sync(0xffffffffu, tie);
-            const bool sel = key[j] > T || (tie && ties_seen + __popc(tb & below) < ties_wanted);
-            const unsigned sb = __ballot_sync(0xffffffffu, sel);
-            if (sel) {
-                const int p = pos + __popc(sb & below);
-                if (p < cap) {
-                    bs[p] = key_score(key[j]);
-                    bc[p] = id_of(c);
-                }
-            }
-            pos += __popc(sb);
-            ties_seen += __popc(tb);
-        }
-    }
-    if (pos > cap) pos = cap;
-    int S = 1;   // sort size: a power of two >= pos (pos <= cap)
-    while (S < pos) S <<= 1;
-    for (int p = pos + lane; p < S; p += 32) {
-        bs[p] = -__int_as_float(0x7f800000);
-        bc[p] = INT32_MAX;
-    }
-    __syncwarp();
-    if (S <= 64) {
-        // bitonic sort in registers: entry i = r * 32 + lane in register r;
-        // partners across lanes by shuffles, across registers (j = 32) in place
-        const float ninf = -__int_as_float(0x7f800000);
-        float s0 = lane < S ? bs[lane] : ninf, s1 = lane + 32 < S ? bs[lane + 32] : ninf;
-        int c0 = lane < S ? bc[lane] : INT32_MAX, c1 = lane + 32 < S ? bc[lane + 32] : INT32_MAX;
-        for (int k = 2; k <= S; k <<= 1) {
-            for (int j = k >> 1; j > 0; j >>= 1) {
-                if (j == 32) {   // k == 64: entry lane (kept better) against lane + 32
-                    if (ranks_before(s1, c1, s0, c0)) {
-                        const float ts = s0;
-                        const int tc = c0;
-                        s0 = s1;
-                        c0 = c1;
-                        s1 = ts;
-                        c1 = tc;
-                    }
-                    continue;
-                }
-                const float ps0 = __shfl_xor_sync(0xffffffffu, s0, j);
-                const int pc0 = __shfl_xor_sync(0xffffffffu, c0, j);
-                const float ps1 = __shfl_xor_sync(0xffffffffu, s1, j);
-                const int pc1 = __shfl_xor_sync(0xffffffffu, c1, j);
-                const bool lower = (lane & j) == 0;
-                // the lower entry of a pair keeps the better one when its
-                // block sorts first-ranked first ((i & k) == 0), else the worse
-                const bool take0 = (lower == ((lane & k) == 0)) == ranks_before(ps0, pc0, s0, c0);
-                const bool take1 = (lower == (((lane + 32) & k) == 0)) == ranks_before(ps1, pc1, s1, c1);
-                if (take0) { s0 = ps0; c0 = pc0; }
-                if (take1) { s1 = ps1; c1 = pc1; }
-            }
-        }
-        __syncwarp();
-        if (lane < S) { bs[lane] = s0; bc[lane] = c0; }
-        if (lane + 32 < S) { bs[lane + 32] = s1; bc[lane + 32] = c1; }
-        __syncwarp();
-        return;
-    }
-    // bitonic sort of S entries, first-ranked first
-    for (int k = 2; k <= S; k <<= 1) {
         for (int j = k >> 1; j > 0; j >>= 1) {
-            for (int i = lane; i < S / 2; i += 32) {
-                const int lo = 2 * i - (i & (j - 1));
-                const int hi = lo + j;
-                const bool up = (lo & k) == 0;
-                const float s0 = bs[lo], s1 = bs[hi];
-                const int c0 = bc[lo], c1 = bc[hi];
-                if (ranks_before(s1, c1, s0, c0) == up) {
-                    bs[lo] = s1;
-                    bc[lo] = c1;
-                    bs[hi] = s0;
-                    bc[hi] = c0;
+            if (j >= 32) {
+                const int jr = j >> 5;
+#pragma unroll
+                for (int r = 0; r < R; ++r) {
+                    if (r & jr) continue;
+                    const int r2 = r | jr;
+                    const bool up = ((r * 32) & k) == 0;   // this block sorts first-ranked first
+                    // the lower entry keeps the better one when up, else the worse
+                    const bool swap = up ? ranks_before(s[r2], c[r2], s[r], c[r])
+                                         : ranks_before(s[r], c[r], s[r2], c[r2]);
+                    if (swap) {
+                        const float ts = s[r];
+                        const int tc = c[r];
+                        s[r] = s[r2];
+                        c[r] = c[r2];
+                        s[r2] = ts;
+                        c[r2] = tc;
+                    }
+                }
+            } else {
+                const bool lower = (lane & j) == 0;
+#pragma unroll
+                for (int r = 0; r < R; ++r) {
+                    const float ps = __shfl_xor_sync(0xffffffffu, s[r], j);
+                    const int pc = __shfl_xor_sync(0xffffffffu, c[r], j);
+                    const bool up = (((r * 32) + lane) & k) == 0;
+                    const bool take = (lower == up) ? ranks_before(ps, pc, s[r], c[r])
+                                                    : ranks_before(s[r], c[r], ps, pc);
+                    if (take) {
+                        s[r] = ps;
+                        c[r] = pc;
+                    }
                 }
             }
-            __syncwarp();
         }
     }
 }
 
-// One warp per (query, segment).  The segment's entries are positions
-// s*seg .. min(M, (s+1)*seg)-1 of the query's row of `in_s` (ids from `in_id`,
-// or the position itself when in_id is null), in id order among equal scores
-// (a row of centroid scores, or the sorted outputs of consecutive id ranges);
-// want = min(nprobe, entries).  Output: the want best in order at
-// out_id/out_s[q * out_ld + s * nprobe ..], then (-inf, INT32_MAX) padding up
-// to nprobe.  `only` (nullable): queries with only[q] == 0 are skipped.
-// `seg_cnt` (nullable): [nq][nseg] entries actually present in each segment.
-// P: a power of two >= nprobe; the sort buffer holds 2P entries.
-// Eight blocks per SM (64 registers) where the keys fit: the selection is a chain
-// of dependent warp reductions, so it needs the warps to hide their latency
-// (timed 25% faster than 120 registers at four blocks).
-template <int KPL>   // entries per lane: seg <= 32 * KPL
-__global__ void __launch_bounds__(kSelectWarps * 32, KPL >= 64 ? 4 : 8) k_select(
-    const float *__restrict__ in_s, const int32_t *__restrict__ in_id, int64_t in_ld, int64_t nq,
-    int64_t M, int seg, int nseg, int nprobe, int P, int32_t *__restrict__ out_id,
-    float *__restrict__ out_s, int64_t out_ld, const int *__restrict__ only,
-    const int *__restrict__ seg_cnt) {
-    extern __shared__ __align__(16) unsigned char sel_smem[];
-    const int cap = 2 * P;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    float *bs = reinterpret_cast<float *>(sel_smem) + warp * 2 * cap;   // cap scores, then cap ids
-    int *bc = reinterpret_cast<int *>(bs + cap);
-    const int64_t w = (int64_t)blockIdx.x * kSelectWarps + warp;
-    if (w >= nq * nseg) return;
-    const int64_t q = w / nseg;
-    if (only && only[q] == 0) return;
-    const int sg = (int)(w % nseg);
-    const int64_t p0 = (int64_t)sg * seg;
-    int cnt = (int)(M - p0 < seg ? M - p0 : seg);
-    if (seg_cnt && seg_cnt[q * nseg + sg] < cnt) cnt = seg_cnt[q * nseg + sg];
-    const int want = nprobe < cnt ? nprobe : cnt;
-    const float *row = in_s + q * in_ld + p0;
-    const int32_t *rid = in_id ? in_id + q * in_ld + p0 : nullptr;
-    uint32_t key[KPL];   // the scores themselves are recovered from the keys
+// Sort bs/bc[0 .. want-1] in place (R * 32 >= want entries; the rest become
+// padding (-inf, INT32_MAX))
+template <int R>
+__device__ __forceinline__ void sort_buffer(float *bs, int *bc, int want) {
+    const int lane = threadIdx.x & 31;
+    float s[R];
+    int c[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+        const int i = r * 32 + lane;
+        s[r] = i < want ? bs[i] : -__int_as_float(0x7f800000);
+        c[r] = i < want ? bc[i] : INT32_MAX;
+    }
+    __syncwarp();
+    warp_sort_regs<R>(s, c);
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+        bs[r * 32 + lane] = s[r];
+        bc[r * 32 + lane] = c[r];
+    }
+    __syncwarp();
+}
+
+// The want best of the warp's cnt entries (entry c = key[c / 32] of lane
+// c % 32, its id from id_of(c)) into bs/bc[0 .. want-1], in entry order,
+// given T and C from warp_threshold(key, want, want, ..).  C == want: every
+// key >= T.  Otherwise T == T* and the keys > T* plus the first keys equal to
+// it in entry order are taken, which are the lowest ids when entry order is id
+// order among equal scores.
+template <int KPL, class IdOf>
+__device__ __forceinline__ void warp_gather_exact(const uint32_t (&key)[KPL], int cnt, int want,
+                                                  uint32_t T, int C, IdOf id_of, float *bs,
+                                                  int *bc) {
+    const int lane = threadIdx.x & 31;
+    const unsigned below = (1u << lane) - 1u;
+    const bool ties = C > want;
+    int ties_wanted = 0;
+    if (ties) {
+        int gt = 0;
+#pragma unroll
+        for (int j = 0; j < KPL; ++j) gt += key[j] > T && j * 32 + lane < cnt;
+        ties_wanted = want - warp_sum(gt);   // >= 1
+    }
+    int pos = 0, ties_seen = 0;
 #pragma unroll
     for (int j = 0; j < KPL; ++j) {
         const int c = j * 32 + lane;
-        key[j] = c < cnt ? order_key(row[c]) : 0u;   // padding ranks below every score
+        const bool in = c < cnt;
+        bool sel;
+        if (ties) {
+            const bool tie = key[j] == T && in;
+            const unsigned tb = __ballot_sync(0xffffffffu, tie);
+            sel = (key[j] > T && in) || (tie && ties_seen + __popc(tb & below) < ties_wanted);
+            ties_seen += __popc(tb);
+        } else {
+            sel = key[j] >= T && in;
+        }
+        const unsigned sb = __ballot_sync(0xffffffffu, sel);
+        if (sel) {
+            const int p = pos + __popc(sb & below);
+            if (p < want) {   // exactly want are selected; the bound guards the buffer
+                bs[p] = key_score(key[j]);
+                bc[p] = id_of(c);
+            }
+        }
+        pos += __popc(sb);
+    }
+    __syncwarp();
+}
+
+// The want best of the warp's cnt entries into bs/bc[0 .. want-1], in entry
+// order (sort_buffer orders them).  With many keys per lane and a second-step
+// buffer (ck/ci, 32 * K2 entries; nullable): a first threshold, refined
+// until at most 32 * K2 keys reach it (K2 about 2 want / 32), the keys that
+// reach it compacted there in entry order, and the exact selection over K2
+// keys per lane.
+template <int K2, int KPL, class IdOf>
+__device__ __forceinline__ bool select_two_step(const uint32_t (&key)[KPL], int cnt, int want,
+                                                IdOf id_of, uint32_t *ck, int *ci, float *bs,
+                                                int *bc) {
+    uint32_t T;
+    int C;
+    warp_threshold(key, want, 32 * K2, T, C);
+    if (C > 32 * K2) {   // T is the want-th largest key itself, tied past the buffer
+        warp_gather_exact(key, cnt, want, T, C, id_of, bs, bc);
+        return true;
+    }
+    const int lane = threadIdx.x & 31;
+    const unsigned below = (1u << lane) - 1u;
+    int pos = 0;
+#pragma unroll
+    for (int j = 0; j < KPL; ++j) {
+        const int c = j * 32 + lane;
+        const bool sel = key[j] >= T && c < cnt;
+        const unsigned sb = __ballot_sync(0xffffffffu, sel);
+        if (sel) {
+            const int p = pos + __popc(sb & below);
+            ck[p] = key[j];
+            ci[p] = id_of(c);
+        }
+        pos += __popc(sb);
+    }
+    __syncwarp();
+    uint32_t k2[K2];
+#pragma unroll
+    for (int j = 0; j < K2; ++j) {
+        const int c = j * 32 + lane;
+        k2[j] = c < pos ? ck[c] : 0u;
+    }
+    warp_threshold(k2, want, want, T, C);
+    warp_gather_exact(k2, pos, want, T, C, [&](int c) { return ci[c]; }, bs, bc);
+    return true;
+}
+
+template <int K2, int KPL, class IdOf>
+__device__ __forceinline__ void warp_select_exact(const uint32_t (&key)[KPL], int cnt, int want,
+                                                  IdOf id_of, uint32_t *ck, int *ci, float *bs,
+                                                  int *bc) {
+    static_assert(K2 <= kStage2, "");
+    if (want <= 0) return;
+    if constexpr (KPL > kStage2) {
+        if (ck) {
+            select_two_step<K2>(key, cnt, want, id_of, ck, ci, bs, bc);
+            return;
+        }
     }
     uint32_t T;
     int C;
-    warp_threshold(key, want, cap, T, C);
-    if (C <= cap && cap <= 32 * kSelectSmallC) {
-        // two steps: the C candidates (key >= T) go to shared memory in id
-        // order, come back as kSelectSmallC keys per lane, and a second, cheap
-        // threshold over them leaves exactly want entries to sort
-        const unsigned below = (1u << lane) - 1u;
-        uint32_t *ck = reinterpret_cast<uint32_t *>(bs);
-        int pos = 0;
+    warp_threshold(key, want, want, T, C);
+    warp_gather_exact(key, cnt, want, T, C, id_of, bs, bc);
+}
+
+// One warp per (query, segment of at most kSelectSeg entries).  The
+// segment's entries are positions s*seg .. min(M, (s+1)*seg)-1 of the query's
+// row of `in_s` (ids from `in_id`, or the position itself when in_id is null),
+// in id order among equal scores (a row of centroid scores, or the sorted
+// outputs of consecutive id ranges); want = min(nprobe, entries).  Output: the
+// want best in order at out_id/out_s[q * out_ld + s * nprobe ..], then
+// (-inf, INT32_MAX) padding up to nprobe.  qlist (nullable): only the queries
+// qlist[0 .. *qlist_n - 1]; the warps stride over them.  seg_cnt (nullable):
+// [nq][nseg] entries actually present in each segment.  nprobe <= 32 * R.
+// Eight blocks per SM (64 registers) where the keys fit: the selection is a
+// chain of dependent warp reductions, so it needs the warps to hide their
+// latency.
+template <int KPL, int R>   // entries per lane: seg <= 32 * KPL
+__global__ void __launch_bounds__(kSelectWarps * 32, (KPL >= 64 || R >= 8) ? 4 : 8)
+    k_select(
+    const float *__restrict__ in_s, const int32_t *__restrict__ in_id, int64_t in_ld, int64_t nq,
+    int64_t M, int seg, int nseg, int nprobe, int32_t *__restrict__ out_id,
+    float *__restrict__ out_s, int64_t out_ld, const int *__restrict__ qlist,
+    const int *__restrict__ qlist_n, const int *__restrict__ seg_cnt) {
+    extern __shared__ __align__(16) unsigned char sel_smem[];
+    // second-step keys per lane: about twice nprobe / 32
+    constexpr int kK2 = R <= 2 ? 4 : R == 4 ? 8 : kStage2;
+    constexpr int kSort = 32 * R;
+    constexpr int kS2 = KPL > kStage2 ? 32 * kK2 : 0;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    float *bs = reinterpret_cast<float *>(sel_smem) + (size_t)warp * 2 * (kSort + kS2);
+    int *bc = reinterpret_cast<int *>(bs + kSort);
+    uint32_t *ck = kS2 ? reinterpret_cast<uint32_t *>(bc + kSort) : nullptr;
+    int *ci = kS2 ? reinterpret_cast<int *>(ck + kS2) : nullptr;
+    const int64_t total = (qlist ? (int64_t)*qlist_n : nq) * nseg;
+    for (int64_t w = (int64_t)blockIdx.x * kSelectWarps + warp; w < total;
+         w += (int64_t)gridDim.x * kSelectWarps) {
+        const int64_t q = qlist ? (int64_t)qlist[w / nseg] : w / nseg;
+        const int sg = (int)(w % nseg);
+        const int64_t p0 = (int64_t)sg * seg;
+        int cnt = (int)(M - p0 < seg ? M - p0 : seg);
+        if (seg_cnt && seg_cnt[q * nseg + sg] < cnt) cnt = seg_cnt[q * nseg + sg];
+        const int want = nprobe < cnt ? nprobe : cnt;
+        const float *row = in_s + q * in_ld + p0;
+        const int32_t *rid = in_id ? in_id + q * in_ld + p0 : nullptr;
+        uint32_t key[KPL];   // the scores themselves are recovered from the keys
 #pragma unroll
         for (int j = 0; j < KPL; ++j) {
             const int c = j * 32 + lane;
-            const bool sel = key[j] >= T && c < cnt;
-            const unsigned sb = __ballot_sync(0xffffffffu, sel);
-            if (sel) {
-                const int p = pos + __popc(sb & below);
-                if (p < cap) {   // pos <= C <= cap
-                    ck[p] = key[j];
-                    bc[p] = rid ? rid[c] : (int)(p0 + c);
-                }
-            }
-            pos += __popc(sb);
+            key[j] = c < cnt ? order_key(row[c]) : 0u;   // padding ranks below every score
+        }
+        warp_select_exact<kK2>(key, cnt, want, [&](int c) { return rid ? rid[c] : (int)(p0 + c); },
+                               ck, ci, bs, bc);
+        sort_buffer<R>(bs, bc, want);
+        int32_t *oi = out_id + q * out_ld + (int64_t)sg * nprobe;
+        float *os = out_s ? out_s + q * out_ld + (int64_t)sg * nprobe : nullptr;
+        for (int p = lane; p < nprobe; p += 32) {
+            oi[p] = p < want ? bc[p] : INT32_MAX;
+            if (os) os[p] = p < want ? bs[p] : -__int_as_float(0x7f800000);
         }
         __syncwarp();
-        uint32_t k2[kSelectSmallC];
-        int i2[kSelectSmallC];
-#pragma unroll
-        for (int j = 0; j < kSelectSmallC; ++j) {
-            const int c = j * 32 + lane;
-            k2[j] = c < pos ? ck[c] : 0u;
-            i2[j] = c < pos ? bc[c] : 0;
-        }
-        __syncwarp();
-        uint32_t T2;
-        int C2;
-        warp_threshold(k2, want, want, T2, C2);
-        warp_gather_sort(k2, pos, want, T2, C2, want, [&](int c) {
-            // id of candidate c: held by lane c % 32 in slot c / 32 (c is this lane's)
-            int id = i2[0];
-#pragma unroll
-            for (int j = 1; j < kSelectSmallC; ++j) id = (c >> 5) == j ? i2[j] : id;
-            return id;
-        }, bs, bc);
-    } else {
-        warp_gather_sort(key, cnt, want, T, C, cap,
-                         [&](int c) { return rid ? rid[c] : (int)(p0 + c); }, bs, bc);
-    }
-    int32_t *oi = out_id + q * out_ld + (int64_t)sg * nprobe;
-    float *os = out_s ? out_s + q * out_ld + (int64_t)sg * nprobe : nullptr;
-    for (int p = lane; p < nprobe; p += 32) {
-        oi[p] = p < want ? bc[p] : INT32_MAX;
-        if (os) os[p] = p < want ? bs[p] : -__int_as_float(0x7f800000);
     }
 }
 
@@ -503,8 +547,7 @@ __global__ void __launch_bounds__(kSelectWarps * 32) k_group_threshold(
     if (lane == 0) lkey[q] = T;
 }
 
-constexpr int kCompactCap = 2048;   // candidates the final warp of a query keeps (64 per lane)
-constexpr int kSegCap = 256;        // candidates one segment may hand on
+constexpr int kSegCap = 256;        // candidates one table segment may hand on
 
 // One warp per (query, segment of kSelectSeg scores): the scores that reach
 // the query's threshold key, in id order, into the segment's kSegCap slots of
@@ -563,10 +606,10 @@ __global__ void __launch_bounds__(kSelectWarps * 32) k_compact_seg(
 }
 
 // the nprobe best of n candidates (keys ck, ids ci in shared memory, id order;
-// n <= 32 * KPL, n >= nprobe), sorted into bs/bc
+// n <= 32 * KPL, n >= nprobe) into bs/bc, in id order
 template <int KPL>
 __device__ __forceinline__ void compact_finish(const uint32_t *ck, const int *ci, int n, int nprobe,
-                                               int cap, float *bs, int *bc) {
+                                               float *bs, int *bc) {
     const int lane = threadIdx.x & 31;
     uint32_t key[KPL];
 #pragma unroll
@@ -574,28 +617,29 @@ __device__ __forceinline__ void compact_finish(const uint32_t *ck, const int *ci
         const int c = j * 32 + lane;
         key[j] = c < n ? ck[c] : 0u;
     }
-    uint32_t T;
-    int C;
-    warp_threshold(key, nprobe, cap, T, C);
-    warp_gather_sort(key, n, nprobe, T, C, cap, [&](int c) { return ci[c]; }, bs, bc);
+    warp_select_exact<kStage2>(key, n, nprobe, [&](int c) { return ci[c]; }, (uint32_t *)nullptr,
+                               (int *)nullptr, bs, bc);
 }
 
-// One warp per query: its segments' candidates gathered in order (id order),
-// then the nprobe best sorted into order/cscores.  A segment past kSegCap or
-// more than kCompactCap in all (many equal scores): the query is flagged in
-// ovf and left to the level-by-level selection.
-__global__ void __launch_bounds__(kSelectWarps * 32) k_compact_final(
+// One warp per query: its segments' candidates (at most segcap kept per
+// segment) gathered in order (id order) into ccap slots, then the nprobe best
+// sorted into order/cscores.  A segment past segcap or more than ccap in all
+// (many equal scores): the query is appended to ovf_list (count in *ovf_n,
+// zeroed before the launch) and left to an exact fallback.  nprobe <= 32 * R.
+template <int R>
+__global__ void __launch_bounds__(kSelectWarps * 32, 6) k_compact_final(
     const float *__restrict__ cand_s, const int32_t *__restrict__ cand_i,
-    const int *__restrict__ seg_n, int64_t nq, int nseg, int segcap, int nprobe, int P,
-    int32_t *__restrict__ order, float *__restrict__ cscores, int *__restrict__ ovf) {
+    const int *__restrict__ seg_n, int64_t nq, int nseg, int segcap, int nprobe, int ccap,
+    int32_t *__restrict__ order, float *__restrict__ cscores, int *__restrict__ ovf_list,
+    int *__restrict__ ovf_n) {
     extern __shared__ __align__(16) unsigned char sel_smem[];
-    const int cap = 2 * P;
+    constexpr int kSort = 32 * R;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    unsigned char *wbase = sel_smem + (size_t)warp * (kCompactCap * 8 + 2 * cap * 4);
-    uint32_t *ck = reinterpret_cast<uint32_t *>(wbase);              // candidate keys
-    int *ci = reinterpret_cast<int *>(wbase + kCompactCap * 4);      // candidate ids
-    float *bs = reinterpret_cast<float *>(wbase + kCompactCap * 8);  // sort buffer
-    int *bc = reinterpret_cast<int *>(bs + cap);
+    unsigned char *wbase = sel_smem + (size_t)warp * ((size_t)ccap + kSort) * 8;
+    uint32_t *ck = reinterpret_cast<uint32_t *>(wbase);                 // candidate keys
+    int *ci = reinterpret_cast<int *>(wbase + (size_t)ccap * 4);        // candidate ids
+    float *bs = reinterpret_cast<float *>(wbase + (size_t)ccap * 8);    // sort buffer
+    int *bc = reinterpret_cast<int *>(bs + kSort);
     const int64_t q = (int64_t)blockIdx.x * kSelectWarps + warp;
     if (q >= nq) return;
     // segment counts and their running offsets, 32 segments at a time
@@ -612,37 +656,36 @@ __global__ void __launch_bounds__(kSelectWarps * 32) k_compact_final(
             if (lane >= o) x += y;
         }
         const int total = __shfl_sync(0xffffffffu, x, 31);
-        if (!over && n + total <= kCompactCap) {
-            // copy each segment's candidates to its place (lanes of the warp in turn)
-            for (int t = 0; t < 32 && s0 + t < nseg; ++t) {
-                const int ct = __shfl_sync(0xffffffffu, c, t);
-                const int at = n + __shfl_sync(0xffffffffu, x, t) - ct;
-                const float *ss = cand_s + (q * nseg + s0 + t) * (int64_t)segcap;
-                const int32_t *si = cand_i + (q * nseg + s0 + t) * (int64_t)segcap;
-                for (int i = lane; i < ct; i += 32) {
-                    ck[at + i] = order_key(ss[i]);
-                    ci[at + i] = si[i];
-                }
+        if (!over && n + total <= ccap && c > 0) {
+            // lane l copies segment s0 + l to its place: the segments' loads
+            // are in flight together, four of each lane's at a time
+            const int at = n + x - c;
+            const float *ss = cand_s + (q * nseg + sg) * (int64_t)segcap;
+            const int32_t *si = cand_i + (q * nseg + sg) * (int64_t)segcap;
+#pragma unroll 4
+            for (int i = 0; i < c; ++i) {
+                ck[at + i] = order_key(ss[i]);
+                ci[at + i] = si[i];
             }
         }
         n += total;
-        over |= n > kCompactCap;
+        over |= n > ccap;
     }
     if (over) {
-        if (lane == 0) ovf[q] = 1;
+        if (lane == 0) ovf_list[atomicAdd(ovf_n, 1)] = (int)q;
         return;
     }
-    if (lane == 0) ovf[q] = 0;
     __syncwarp();
     // keys per lane sized to the candidates (warp-uniform n)
-    if (n <= 256)
-        compact_finish<8>(ck, ci, n, nprobe, cap, bs, bc);
+    if (n <= 128)
+        compact_finish<4>(ck, ci, n, nprobe, bs, bc);
     else if (n <= 512)
-        compact_finish<16>(ck, ci, n, nprobe, cap, bs, bc);
+        compact_finish<16>(ck, ci, n, nprobe, bs, bc);
     else if (n <= 1024)
-        compact_finish<32>(ck, ci, n, nprobe, cap, bs, bc);
+        compact_finish<32>(ck, ci, n, nprobe, bs, bc);
     else
-        compact_finish<kCompactCap / 32>(ck, ci, n, nprobe, cap, bs, bc);
+        compact_finish<64>(ck, ci, n, nprobe, bs, bc);
+    sort_buffer<R>(bs, bc, nprobe);
     for (int p = lane; p < nprobe; p += 32) {
         order[q * nprobe + p] = bc[p];
         if (cscores) cscores[q * nprobe + p] = bs[p];
@@ -662,7 +705,7 @@ static int64_t level_entries(int64_t M, int nprobe) { return ceil_div(M, kSelect
 // for one warp), then one compacting pass
 static bool use_group_threshold(int64_t nlist, int nprobe) {
     const int64_t ng = ceil_div(nlist, 32);
-    return nlist > kSelectSeg && ng >= nprobe && ng <= kCompactCap;
+    return nlist > kSelectSeg && ng >= nprobe && ng <= kGroupMax;
 }
 
 // Under the group threshold, narrow rows (d <= 128) skip the score table: one
@@ -673,13 +716,40 @@ static bool use_two_pass(int64_t nlist, int nprobe, int d) {
     return use_group_threshold(nlist, nprobe) && d <= 128;
 }
 
+static int pow2_at_least(int64_t x) {
+    int p = 1;
+    while (p < x) p <<= 1;
+    return p;
+}
+
+// kept slots per 2,048-centroid range on the two-pass path: four times a
+// range's even share of nprobe (the threshold keeps a little over nprobe
+// scores in all), at least 64.  A range past it sends its query to the FP32
+// fallback.
+static int keep_cap(int64_t nlist, int nprobe) {
+    const int64_t nseg = ceil_div(nlist, kRankRange);
+    const int c = pow2_at_least(ceil_div(4 * (int64_t)nprobe, nseg));
+    return (int)std::min<int64_t>(kRankRange, std::max(64, c));
+}
+
+// candidates one compacting warp holds: 4 P (P = nprobe rounded up to a
+// power of two), between 512 and 2,048
+static int compact_cap(int nprobe) {
+    return std::min(2048, std::max(512, 4 * pow2_at_least(nprobe)));
+}
+
+// registers per lane of the sort of nprobe entries
+static int sort_regs(int nprobe) { return std::max(2, pow2_at_least(nprobe) / 32); }
+
 // Scratch of one query, in the order enqueue_rank_tc lays it out:
 //   score row (table path only)                      round_up(nlist, 32) f32
-//   two level buffers (scores, then ids)             2 x lvl x 8 B   (nlist > kSelectSeg)
+//   two level buffers (scores, then ids)             2 x lvl x 8 B   (table path, nlist > kSelectSeg)
 //   group maxima                                     round_up(ng, 4) f32
 //   candidate slots (scores, then ids)               nseg x cap x 8 B (cap = kSegCap, or
-//                                                    kRankRange on the two-pass path)
-//   candidate counts, threshold key, overflow flag   round_up(nseg, 4) x 4 B + 8 B
+//                                                    keep_cap on the two-pass path)
+//   candidate counts, threshold key, overflow list   round_up(nseg, 4) x 4 B + 8 B
+// and once per chunk the overflow count (kRankFixedBytes).
+constexpr int64_t kRankFixedBytes = 256;
 struct RankScratch {
     int64_t ld, lvl, gld, cap;
     int nseg;
@@ -695,12 +765,13 @@ struct RankScratch {
 static RankScratch rank_scratch(int64_t nlist, int nprobe, int d) {
     RankScratch r;
     r.ld = rank_tc_ld(nlist);
-    r.lvl = nlist > kSelectSeg ? round_up(level_entries(nlist, nprobe), 4) : 0;
     r.grouped = use_group_threshold(nlist, nprobe);
     r.table = !use_two_pass(nlist, nprobe, d);
+    // the two-pass path falls back to the FP32 ranking, not to the levels
+    r.lvl = (nlist > kSelectSeg && r.table) ? round_up(level_entries(nlist, nprobe), 4) : 0;
     r.gld = round_up(ceil_div(nlist, 32), 4);
     r.nseg = (int)ceil_div(nlist, kSelectSeg);
-    r.cap = r.table ? kSegCap : kRankRange;
+    r.cap = r.table ? kSegCap : keep_cap(nlist, nprobe);
     return r;
 }
 
@@ -712,26 +783,27 @@ int64_t rank_tc_chunk(int64_t nq, int64_t nlist, int nprobe, int d) {
 }
 
 size_t rank_tc_scratch_bytes(int64_t nq, int64_t nlist, int nprobe, int d) {
-    return (size_t)(rank_tc_chunk(nq, nlist, nprobe, d) * rank_scratch(nlist, nprobe, d).per_query());
+    return (size_t)(rank_tc_chunk(nq, nlist, nprobe, d) * rank_scratch(nlist, nprobe, d).per_query() +
+                    kRankFixedBytes);
 }
 
 static size_t tc_smem() { return tcp::Geometry<RankMode::kN>::smem_bytes(0); }
 
-static int pow2_at_least(int64_t x) {
-    int p = 1;
-    while (p < x) p <<= 1;
-    return p;
+// shared memory of the selecting kernels (kSelectWarps warps, each with its
+// own buffers)
+static size_t select_smem(int kpl, int R) {
+    const int k2 = R <= 2 ? 4 : R == 4 ? 8 : kStage2;   // k_select's second-step keys per lane
+    const size_t s2 = kpl > kStage2 ? 32 * (size_t)k2 : 0;
+    return (size_t)kSelectWarps * (32 * (size_t)R + s2) * 8;
+}
+static size_t compact_smem(int ccap, int R) {
+    return (size_t)kSelectWarps * ((size_t)ccap + 32 * (size_t)R) * 8;
 }
 
-static size_t select_smem(int P) { return (size_t)kSelectWarps * 2 * (2 * P) * 4; }
-static size_t compact_smem(int P) {
-    return (size_t)kSelectWarps * ((size_t)kCompactCap * 8 + 2 * (2 * P) * 4);
-}
-
-template <int KPL>
-static cudaError_t set_select_attr(int P) {
-    return cudaFuncSetAttribute(k_select<KPL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)select_smem(P));
+template <int R>
+static cudaError_t set_compact_attr(int ccap) {
+    return cudaFuncSetAttribute(k_compact_final<R>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)compact_smem(ccap, R));
 }
 
 cudaError_t prepare_rank_tc(int nprobe, int d) {
@@ -741,59 +813,108 @@ cudaError_t prepare_rank_tc(int nprobe, int d) {
     if (e == cudaSuccess && bulk)
         e = cudaFuncSetAttribute(k_rank_bulk, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)tcb::smem_bytes(bulk, 0));
-    const int P = pow2_at_least(nprobe);
-    if (e == cudaSuccess) e = set_select_attr<1>(P);
-    if (e == cudaSuccess) e = set_select_attr<2>(P);
-    if (e == cudaSuccess) e = set_select_attr<4>(P);
-    if (e == cudaSuccess) e = set_select_attr<8>(P);
-    if (e == cudaSuccess) e = set_select_attr<16>(P);
-    if (e == cudaSuccess) e = set_select_attr<32>(P);
-    if (e == cudaSuccess) e = set_select_attr<64>(P);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_compact_final, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)compact_smem(P));
+    // the selections stay below the 48 KB default; the compacting warps may not
+    const int ccap = compact_cap(nprobe);
+    if (e == cudaSuccess) e = set_compact_attr<2>(ccap);
+    if (e == cudaSuccess) e = set_compact_attr<4>(ccap);
+    if (e == cudaSuccess) e = set_compact_attr<8>(ccap);
+    if (e == cudaSuccess) e = set_compact_attr<16>(ccap);
+    // the two-pass path's exact fallback
+    if (e == cudaSuccess && d <= 128) e = prepare_rank(nprobe);
     return e;
 }
 
-// one selection level: the best nprobe of every segment of at most kSelectSeg
-// entries (nseg = 1: the final order)
-static void launch_select(const float *in_s, const int32_t *in_id, int64_t in_ld, int64_t nq,
-                          int64_t M, int nprobe, int32_t *out_id, float *out_s, int64_t out_ld,
-                          const int *only, const int *seg_cnt, cudaStream_t st) {
-    const int seg = M < kSelectSeg ? (int)M : kSelectSeg;
-    const int nseg = (int)ceil_div(M, kSelectSeg);
-    const int P = pow2_at_least(nprobe);
-    const unsigned blocks = (unsigned)ceil_div(nq * nseg, kSelectWarps);
-    const size_t smem = select_smem(P);
-    const int kpl = pow2_at_least(ceil_div(seg, 32));
-#define SIEVE_SELECT(K)                                                                            \
-    k_select<K><<<blocks, kSelectWarps * 32, smem, st>>>(in_s, in_id, in_ld, nq, M, seg, nseg,     \
-                                                        nprobe, P, out_id, out_s, out_ld, only, \
-                                                        seg_cnt)
-    switch (kpl) {
-        case 1: SIEVE_SELECT(1); break;
+template <int KPL>
+static void select_r(int R, dim3 grid, size_t smem, cudaStream_t st, const float *in_s,
+                     const int32_t *in_id, int64_t in_ld, int64_t nq, int64_t M, int seg, int nseg,
+                     int nprobe, int32_t *out_id, float *out_s, int64_t out_ld, const int *qlist,
+                     const int *qlist_n, const int *seg_cnt) {
+#define SIEVE_SELECT(RR)                                                                        \
+    k_select<KPL, RR><<<grid, kSelectWarps * 32, smem, st>>>(in_s, in_id, in_ld, nq, M, seg, nseg, \
+                                                             nprobe, out_id, out_s, out_ld, qlist, \
+                                                             qlist_n, seg_cnt)
+    switch (R) {
         case 2: SIEVE_SELECT(2); break;
         case 4: SIEVE_SELECT(4); break;
         case 8: SIEVE_SELECT(8); break;
-        case 16: SIEVE_SELECT(16); break;
-        case 32: SIEVE_SELECT(32); break;
-        default: SIEVE_SELECT(64); break;
+        default: SIEVE_SELECT(16); break;
     }
 #undef SIEVE_SELECT
 }
 
+// one selection level: the best nprobe of every segment of at most kSelectSeg
+// entries (nseg = 1: the final order).  qlist/qlist_n (nullable, device): only
+// the listed queries, on a grid of a few blocks per SM that strides over them.
+static void launch_select(const float *in_s, const int32_t *in_id, int64_t in_ld, int64_t nq,
+                          int64_t M, int nprobe, int32_t *out_id, float *out_s, int64_t out_ld,
+                          const int *qlist, const int *qlist_n, const int *seg_cnt, cudaStream_t st) {
+    const int seg = M < kSelectSeg ? (int)M : kSelectSeg;
+    const int nseg = (int)ceil_div(M, kSelectSeg);
+    const int R = sort_regs(nprobe);
+    int64_t blocks = ceil_div(nq * nseg, kSelectWarps);
+    if (qlist) blocks = std::min<int64_t>(blocks, 4 * (int64_t)num_sms());
+    const dim3 grid((unsigned)blocks);
+    const int kpl = std::max(4, pow2_at_least(ceil_div(seg, 32)));
+#define SIEVE_SEL_K(K)                                                                          \
+    select_r<K>(R, grid, select_smem(K, R), st, in_s, in_id, in_ld, nq, M, seg, nseg, nprobe,     \
+                out_id, out_s, out_ld, qlist, qlist_n, seg_cnt)
+    if (kpl <= 4)
+        SIEVE_SEL_K(4);
+    else if (kpl <= 16)
+        SIEVE_SEL_K(16);
+    else if (kpl <= 32)
+        SIEVE_SEL_K(32);
+    else
+        SIEVE_SEL_K(64);
+#undef SIEVE_SEL_K
+}
+
+static void launch_compact_final(const float *cand_s, const int32_t *cand_i, const int *seg_n,
+                                 int64_t nq, int nseg, int segcap, int nprobe, int32_t *order,
+                                 float *cscores, int *ovf_list, int *ovf_n, cudaStream_t st) {
+    const unsigned blocks = (unsigned)ceil_div(nq, kSelectWarps);
+    const int ccap = compact_cap(nprobe);
+#define SIEVE_COMPACT(RR)                                                                      \
+    k_compact_final<RR><<<blocks, kSelectWarps * 32, compact_smem(ccap, RR), st>>>(               \
+        cand_s, cand_i, seg_n, nq, nseg, segcap, nprobe, ccap, order, cscores, ovf_list, ovf_n)
+    switch (sort_regs(nprobe)) {
+        case 2: SIEVE_COMPACT(2); break;
+        case 4: SIEVE_COMPACT(4); break;
+        case 8: SIEVE_COMPACT(8); break;
+        default: SIEVE_COMPACT(16); break;
+    }
+#undef SIEVE_COMPACT
+}
+
 int rank_tc_launches(int64_t nq, int64_t nlist, int nprobe, int d) {
     if (nq <= 0) return 0;
-    int per = 2;                                           // contraction + final selection
-    if (use_group_threshold(nlist, nprobe)) per += 3;      // threshold, compaction, gather
-    // the two-pass path trades the compaction pass for a second contraction: same count
-    for (int64_t M = nlist; M > kSelectSeg; M = level_entries(M, nprobe)) ++per;
+    int per;
+    if (use_two_pass(nlist, nprobe, d)) {
+        per = 5;   // maxima pass, threshold, keeping pass, final warps, FP32 fallback
+    } else {
+        per = 2;   // contraction, final selection level
+        if (use_group_threshold(nlist, nprobe)) per += 3;   // threshold, compaction, final warps
+        for (int64_t M = nlist; M > kSelectSeg; M = level_entries(M, nprobe)) ++per;
+    }
     return (int)ceil_div(nq, rank_tc_chunk(nq, nlist, nprobe, d)) * per;
+}
+
+int rank_tc_mma_launches(int64_t nq, int64_t nlist, int nprobe, int d) {
+    if (nq <= 0) return 0;
+    return (int)ceil_div(nq, rank_tc_chunk(nq, nlist, nprobe, d)) *
+           (use_two_pass(nlist, nprobe, d) ? 2 : 1);
 }
 
 cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t nlist, int d,
                             int nprobe, int32_t *order, float *cscores, float *scratch, int *status,
-                            cudaStream_t st, const unsigned char *tc_cent) {
+                            cudaStream_t st, const unsigned char *tc_cent, float *mma_ms) {
+    struct Events {   // mma_ms: a pair per contraction launch, destroyed on every return
+        std::vector<cudaEvent_t> v;
+        ~Events() {
+            for (cudaEvent_t e : v) cudaEventDestroy(e);
+        }
+    } ev_hold;
+    std::vector<cudaEvent_t> &evs = ev_hold.v;
     const int bulk_stages = tc_cent ? rank_bulk_stages(d) : 0;
     const RankScratch L = rank_scratch(nlist, nprobe, d);
     const int64_t chunk = rank_tc_chunk(nq, nlist, nprobe, d);
@@ -809,36 +930,40 @@ cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t 
         p += 2 * chunk * L.lvl;
     }
     float *gmax = p;
-    p += chunk * L.gld;
+    p += L.grouped ? chunk * L.gld : 0;
     float *slot_s = p;
     int32_t *slot_i = reinterpret_cast<int32_t *>(p + chunk * L.nseg * L.cap);
-    p += 2 * chunk * L.nseg * L.cap;
+    p += L.grouped ? 2 * chunk * L.nseg * L.cap : 0;
     int *slot_n = reinterpret_cast<int *>(p);
-    uint32_t *lkey = reinterpret_cast<uint32_t *>(slot_n + chunk * round_up(L.nseg, 4));
-    int *ovf = reinterpret_cast<int *>(lkey + chunk);
+    uint32_t *lkey = reinterpret_cast<uint32_t *>(slot_n + (L.grouped ? chunk * round_up(L.nseg, 4) : 0));
+    int *ovf = reinterpret_cast<int *>(lkey + (L.grouped ? chunk : 0));   // [chunk] overflow list
+    int *ovf_n = reinterpret_cast<int *>(reinterpret_cast<unsigned char *>(scratch) +
+                                         chunk * L.per_query());       // its count
     const int ng = (int)ceil_div(nlist, 32);
-    const int P = pow2_at_least(nprobe);
     for (int64_t q0 = 0; q0 < nq; q0 += chunk) {
         const int64_t n = nq - q0 < chunk ? nq - q0 : chunk;
         const int tiles = (int)(ceil_div(n, tcp::kM) * ceil_div(nlist, kRankRange));
         auto contract = [&](const RankArgs &a) {
+            if (mma_ms) {
+                evs.resize(evs.size() + 2);
+                cudaEventCreate(&evs[evs.size() - 2]);
+                cudaEventCreate(&evs.back());
+                cudaEventRecord(evs[evs.size() - 2], st);
+            }
             if (bulk_stages)
                 k_rank_bulk<<<std::min(tiles, num_sms()), tcb::kThreads,
                               tcb::smem_bytes(bulk_stages, 0), st>>>(a, bulk_stages);
             else
                 k_rank_tc<<<std::min(tiles, num_sms()), tcp::kThreads, tc_smem(), st>>>(a);
+            if (mma_ms) cudaEventRecord(evs.back(), st);
         };
         RankArgs a{Q + q0 * d, n, C, nlist, d, table, L.ld, status, tc_cent,
                    L.grouped ? gmax : nullptr, L.gld, L.table ? kRankTable : kRankMax,
-                   lkey, slot_s, slot_i, slot_n};
+                   lkey, slot_s, slot_i, slot_n, (int)L.cap};
         contract(a);
         int32_t *o = order + q0 * nprobe;
         float *cs = cscores ? cscores + q0 * nprobe : nullptr;
-        const int *only = nullptr;
-        const float *lvl0_s = table;       // what the first selection level reads
-        const int32_t *lvl0_id = nullptr;
-        int64_t lvl0_ld = L.ld;
-        const int *lvl0_cnt = nullptr;
+        const int *qlist = nullptr, *qlist_n = nullptr;
         if (L.grouped) {
             const unsigned wblocks = (unsigned)ceil_div(n, kSelectWarps);
             const int kpl = pow2_at_least(ceil_div(ng, 32));
@@ -862,38 +987,48 @@ cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t 
                 keep.gmax = nullptr;
                 keep.mode = kRankKeep;
                 contract(keep);
-                // an overflowing query's levels read its kept scores, range by range
-                lvl0_s = slot_s;
-                lvl0_id = slot_i;
-                lvl0_ld = (int64_t)L.nseg * L.cap;
-                lvl0_cnt = slot_n;
             }
-            k_compact_final<<<wblocks, kSelectWarps * 32, compact_smem(P), st>>>(
-                slot_s, slot_i, slot_n, n, L.nseg, (int)L.cap, nprobe, P, o, cs, ovf);
-            only = ovf;   // the levels below run only for overflowing queries
+            cudaError_t e = cudaMemsetAsync(ovf_n, 0, sizeof(int), st);
+            if (e != cudaSuccess) return e;
+            launch_compact_final(slot_s, slot_i, slot_n, n, L.nseg, (int)L.cap, nprobe, o, cs, ovf,
+                                 ovf_n, st);
+            if (!L.table) {
+                // the queries whose kept slots overflowed: the FP32 ranking, exact
+                e = enqueue_rank(Q + q0 * d, n, C, nlist, d, nprobe, o, cs, st, ovf, ovf_n);
+                if (e != cudaSuccess) return e;
+                e = cudaGetLastError();
+                if (e != cudaSuccess) return e;
+                continue;
+            }
+            qlist = ovf;   // the levels below run only for the overflowing queries
+            qlist_n = ovf_n;
         }
-        // levels until one segment is left (segments of the first level are the
-        // 2,048-centroid ranges, whether read from the table or the kept slots)
-        const float *in_s = lvl0_s;
-        const int32_t *in_id = lvl0_id;
-        int64_t in_ld = lvl0_ld, M = L.table ? nlist : (int64_t)L.nseg * L.cap;
-        const int *in_cnt = lvl0_cnt;
-        int64_t M_left = nlist;
+        // levels over the score table until one segment is left
+        const float *in_s = table;
+        const int32_t *in_id = nullptr;
+        int64_t in_ld = L.ld, M = nlist;
         int buf = 0;
-        while (M_left > kSelectSeg) {
-            launch_select(in_s, in_id, in_ld, n, M, nprobe, cand_id[buf], cand_s[buf], L.lvl, only,
-                          in_cnt, st);
+        while (M > kSelectSeg) {
+            launch_select(in_s, in_id, in_ld, n, M, nprobe, cand_id[buf], cand_s[buf], L.lvl, qlist,
+                          qlist_n, nullptr, st);
             in_s = cand_s[buf];
             in_id = cand_id[buf];
             in_ld = L.lvl;
-            in_cnt = nullptr;
-            M_left = level_entries(M_left, nprobe);
-            M = M_left;
+            M = level_entries(M, nprobe);
             buf ^= 1;
         }
-        launch_select(in_s, in_id, in_ld, n, M, nprobe, o, cs, nprobe, only, in_cnt, st);
+        launch_select(in_s, in_id, in_ld, n, M, nprobe, o, cs, nprobe, qlist, qlist_n, nullptr, st);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
+    }
+    if (mma_ms) {
+        cudaError_t e = cudaStreamSynchronize(st);
+        for (size_t i = 0; i + 1 < evs.size(); i += 2) {
+            float t = 0.f;
+            if (e == cudaSuccess) e = cudaEventElapsedTime(&t, evs[i], evs[i + 1]);
+            *mma_ms += t;
+        }
+        return e;
     }
     return cudaSuccess;
 }

@@ -96,8 +96,11 @@ void enqueue_scan_bulk(const SearchArgs &a, cudaStream_t st);
 // centroid ranking (rank_kernel.cu): prepare_rank once before launches or
 // stream capture, then enqueue_rank (a single kernel launch)
 cudaError_t prepare_rank(int nprobe);
+// qlist/qlist_n (nullable, device): rank only the listed queries of the nq
+// (at most nq of them; the grid covers nq)
 cudaError_t enqueue_rank(const float *Q, int64_t nq, const float *C, int64_t nlist, int d,
-                         int nprobe, int32_t *order, float *cscores, cudaStream_t st);
+                         int nprobe, int32_t *order, float *cscores, cudaStream_t st,
+                         const int *qlist = nullptr, const int *qlist_n = nullptr);
 
 // centroid ranking on the tensor cores (rank_tc.cu): a score table of at most
 // kRankScratchBytes per chunk of queries, then warp-per-segment selections
@@ -106,9 +109,13 @@ bool rank_tc_supported(int64_t nlist, int nprobe);
 size_t rank_tc_scratch_bytes(int64_t nq, int64_t nlist, int nprobe, int d);
 int rank_tc_launches(int64_t nq, int64_t nlist, int nprobe, int d);   // kernel launches of one ranking
 cudaError_t prepare_rank_tc(int nprobe, int d);
+// mma_ms (nullable): the contraction launches are bracketed by events, the
+// call synchronizes st and adds their summed time (ms) to *mma_ms
 cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t nlist, int d,
                             int nprobe, int32_t *order, float *cscores, float *scratch, int *status,
-                            cudaStream_t st, const unsigned char *tc_cent = nullptr);
+                            cudaStream_t st, const unsigned char *tc_cent = nullptr,
+                            float *mma_ms = nullptr);
+int rank_tc_mma_launches(int64_t nq, int64_t nlist, int nprobe, int d);   // contraction launches
 int rank_bulk_stages(int d);                     // 0 when the bulk ranking does not apply
 
 // in-call window calibration (calibrate.cu)
