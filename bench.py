@@ -333,6 +333,47 @@ def cpu_baseline(w, cfg, target_s):
                       f"{dt:.1f} s on {threads} host threads"}
 
 
+def bruteforce_recall(X, ids, Q, qids, tau, k, results, sample=1000, seed=777):
+    """Pooled filtered top-k recall against exhaustive search, the paper's
+    quality measure (Sec. 6.1): on a seeded sample of the queries, the number
+    of exact filtered top-k neighbours (score >= tau, the query's own row
+    excluded) that a result set holds, over the number of exact neighbours.
+    The exact sets come from fp32 inner products of each sampled query with
+    every row (a plain matmul: it evaluates the outputs, it is not the
+    search).  results: {name: (ids [nq][k] i64, count [nq] i32)} on the
+    device."""
+    nq = Q.shape[0]
+    g = torch.Generator(device="cpu").manual_seed(seed)
+    pick = torch.sort(torch.randperm(nq, generator=g)[:min(sample, nq)]).values.to(Q.device)
+    chunk = max(1, int(2 ** 28 // max(1, X.shape[0])))       # <= 1 GiB of scores at a time
+    tf32 = torch.backends.cuda.matmul.allow_tf32
+    torch.backends.cuda.matmul.allow_tf32 = False
+    hits = {name: 0 for name in results}
+    total = 0
+    try:
+        for lo in range(0, pick.numel(), chunk):
+            p = pick[lo:lo + chunk]
+            S = Q[p] @ X.T
+            S[ids[None, :] == qids[p][:, None]] = float("-inf")
+            S[S < tau] = float("-inf")
+            val, pos = torch.topk(S, k, dim=1)
+            valid = val > float("-inf")
+            gt = torch.where(valid, ids[pos], torch.full_like(pos, -2))
+            total += int(valid.sum().item())
+            for name, (r_ids, r_cnt) in results.items():
+                r = r_ids[p]
+                r = torch.where(torch.arange(k, device=r.device)[None, :] < r_cnt[p][:, None].long(),
+                                r, torch.full_like(r, -3))
+                hits[name] += int((r[:, :, None] == gt[:, None, :]).any(-1).sum().item())
+            del S
+    finally:
+        torch.backends.cuda.matmul.allow_tf32 = tf32
+    out = {name: (h / total if total else 1.0) for name, h in hits.items()}
+    out.update(sample_queries=int(pick.numel()), exact_neighbours=total,
+               ground_truth="fp32 inner products with every row, score >= tau, own row excluded")
+    return out
+
+
 def host_arrays(wl):
     return {k: wl[k].detach().cpu().numpy() for k in ("X", "ids", "assign", "centroids", "Q", "qids")}
 
@@ -420,6 +461,13 @@ def run_sieve(args, cfg, world, rank, local):
                  workspace=ws, out=outs, scan_path=args.scan_path)
     mean_probes = float(probes.float().mean().item())
     hit_frac = float((outs[2] > 0).float().mean().item())
+    # quality context: pooled filtered top-k recall of W = 8 and of fixed
+    # probing against exhaustive search on a query sample
+    fixed = sieve.search(index, Q, cfg.tau, k, cfg.nprobe, cfg.nprobe, lookahead=True,
+                         query_ids=qids, workspace=ws, scan_path=args.scan_path)
+    recall_bf = bruteforce_recall(wl["X"], wl["ids"], Q, qids, cfg.tau, k,
+                                  {f"W{cfg.W}": (outs[0], outs[2]), "fixed_probe": (fixed[0], fixed[2])})
+    del fixed
 
     # in-call window calibration (Appendix A): a 2% sample fully probed, a 0.5%
     # sample-relative loss target, the rest under the selected window
@@ -503,6 +551,7 @@ def run_sieve(args, cfg, world, rank, local):
         "calibrated": calib,
         "mean_probes": mean_probes,
         "queries_with_results": hit_frac,
+        "recall_vs_bruteforce": recall_bf,
         "roofline": roofline(prof, cfg, dev, bulk=index.tc_rows is not None,
                              rank_on_tensor=args.scan_path != "simt"),
         "profile": {"kernel_ms": prof["kernel_ms"], "kernel_launches": prof["kernel_launches"],

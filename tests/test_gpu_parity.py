@@ -435,7 +435,7 @@ def test_bulk_path_equals_converter_path(which, tiny, g_tiny, deep, g_deep):
     for key in ("ids", "count", "probes"):
         assert np.array_equal(a[key], b[key]), key
     valid = np.arange(c.k)[None, :] < a["count"][:, None]
-    assert np.abs(a["scores"] - b["scores"])[valid].max(initial=0) <= 1e-6
+    assert np.abs(a["scores"][valid] - b["scores"][valid]).max(initial=0) <= 1e-6
 
 
 def test_wide_rows_fall_back_and_match(dev):
