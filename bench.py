@@ -61,8 +61,11 @@ def parse():
                     help="skip the in-call window calibration measurement")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="target CPU seconds for the oracle sample")
-    ap.add_argument("--scan-path", choices=("auto", "simt", "tensor"), default="auto",
-                    help="which units score the partition groups (sieve_params.scan_path)")
+    ap.add_argument("--scan-path", choices=("auto", "simt", "tensor", "screen"), default="auto",
+                    help="which units score the partition groups (sieve_params.scan_path: "
+                         "tensor = three fp16 products per pair, screen = one product per pair "
+                         "and an fp32 rescore of the candidates, auto = the screen from a "
+                         "window of 16 up)")
     ap.add_argument("--rq", action="store_true",
                     help="the quantized local search (RaBitQ-style 7-bit codes) on the workload")
     ap.add_argument("--ncu-case", choices=("w8", "fixed", "rqw8"), default=None,
@@ -149,7 +152,8 @@ def measured_peaks():
 # the sources that define each profiled kernel and the layout it streams
 _SCAN_SOURCES = ("common.cuh", "search.cuh", "scan_tc.cu", "tcgen05.cuh", "tc_bulk.cuh",
                  "tc_pipeline.cuh", "tc_layout.cu", "rq.cu")
-KERNEL_SOURCES = {"k_scan_bulk": _SCAN_SOURCES, "k_scan_rq": _SCAN_SOURCES}
+KERNEL_SOURCES = {"k_scan_bulk": _SCAN_SOURCES, "k_scan_rq": _SCAN_SOURCES,
+                  "k_scan_screen": _SCAN_SOURCES}
 
 
 def kernel_source_sha(kernel):
@@ -179,10 +183,18 @@ def committed_traffic(kernel, workload, launches):
     return e["dram_bytes_per_search"] / max(1, launches)
 
 
-def roofline(prof, cfg, dev, bulk=True, rank_on_tensor=True, rq=False):
+def uses_screen(args, cfg, W, bulk):
+    """Whether the bulk scan screens (sieve_params.scan_path; the automatic
+    path screens from a window of 16 up)."""
+    return bulk and (args.scan_path == "screen" or
+                     (args.scan_path == "auto" and min(W, cfg.nprobe) >= 16))
+
+
+def roofline(prof, cfg, dev, bulk=True, rank_on_tensor=True, rq=False, screen=False):
     """Roofline entry for the kernel with the largest share of the step.
     bulk: the index carries the tensor-core layout, so the tensor-core scan
     runs as k_scan_bulk (else k_scan_tc) and the ranking as k_rank_bulk;
+    screen: the bulk scan screens with one product per pair (k_scan_screen);
     rank_on_tensor: the ranking runs on the tensor cores (every scan path
     but the FP32 one)."""
     km, kl = dict(prof["kernel_ms"]), dict(prof["kernel_launches"])
@@ -201,7 +213,8 @@ def roofline(prof, cfg, dev, bulk=True, rank_on_tensor=True, rq=False):
     d = cfg.d
     launches = max(1, kl[top])
     ms_per_launch = km[top] / launches
-    name = {"scan_tc": "k_scan_rq" if rq else "k_scan_bulk" if bulk else "k_scan_tc"}.get(top, f"k_{top}")
+    name = {"scan_tc": "k_scan_rq" if rq else ("k_scan_screen" if screen else "k_scan_bulk") if bulk
+            else "k_scan_tc"}.get(top, f"k_{top}")
     out = {"kernel": name, "launches": kl[top], "ms_per_launch": ms_per_launch}
     # fp16 dense peak: the measured bf16 cuBLAS peak (fp16 and bf16 share the
     # nominal 2.25 PFLOP/s rate); the burst figure, as the kernel is timed alone
@@ -215,6 +228,17 @@ def roofline(prof, cfg, dev, bulk=True, rank_on_tensor=True, rq=False):
                                 f"estimate; fp16 dense peak {f16_tflops:.0f} TFLOP/s = measured "
                                 f"bf16 cuBLAS burst (of measured), so the algorithmic peak is half"),
                    tensor_pipe_tflops=2 * ach)
+    elif top == "scan_tc" and screen and bulk:
+        flops = 2.0 * d * prof["pairs_tc"]
+        ach = flops / launches / (ms_per_launch * 1e-3) / 1e12
+        out.update(bound="tensor", achieved=ach, peak=f16_tflops, unit="TFLOP/s",
+                   frac=ach / f16_tflops,
+                   peak_source=(f"screen: one kind::f16 MMA per product (hi halves), the rare "
+                                f"candidates rescored in FP32; fp16 dense peak {f16_tflops:.0f} "
+                                f"TFLOP/s = measured bf16 cuBLAS burst (of measured)"),
+                   tensor_pipe_tflops=ach,
+                   l2_stream_gbs=2.0 * d * prof["rows_read_tc"] / launches
+                   / (ms_per_launch * 1e-3) / 1e9)
     elif top == "scan_tc":
         flops = 2.0 * d * prof["pairs_tc"]
         ach = flops / launches / (ms_per_launch * 1e-3) / 1e12
@@ -546,14 +570,17 @@ def run_sieve(args, cfg, world, rank, local):
                    "scan_path": args.scan_path,
                    "l2": "inputs larger than L2 (index 1.02 GB streamed per step)"},
         "fixed_probe": {"value": nq * world / (ms_fixed * 1e-3), "ms_per_step": ms_fixed,
-                        "W": cfg.nprobe},
+                        "W": cfg.nprobe,
+                        "scan": "screen" if uses_screen(args, cfg, cfg.nprobe, index.tc_rows is not None)
+                        else "three products"},
         "speedup_vs_fixed": ms_fixed / ms,
         "calibrated": calib,
         "mean_probes": mean_probes,
         "queries_with_results": hit_frac,
         "recall_vs_bruteforce": recall_bf,
         "roofline": roofline(prof, cfg, dev, bulk=index.tc_rows is not None,
-                             rank_on_tensor=args.scan_path != "simt"),
+                             rank_on_tensor=args.scan_path != "simt",
+                             screen=uses_screen(args, cfg, cfg.W, index.tc_rows is not None)),
         "profile": {"kernel_ms": prof["kernel_ms"], "kernel_launches": prof["kernel_launches"],
                     "rounds": prof["rounds"], "items": prof["items"], "groups": prof["groups"],
                     "mean_group": prof["items"] / max(1, prof["groups"]),

@@ -103,8 +103,17 @@ typedef struct {
  *              0 = automatic (ranking and every partition group on the
  *              tensor cores when the epilogue's k-lists fit: any k with
  *              the tensor-core layout and d <= 256, k <= 22 otherwise; FP32
- *              FMA beyond), 1 = FP32 FMA only, 2 = tensor cores
- *              (SIEVE_EINVAL where they do not fit)
+ *              FMA beyond; with the tensor-core layout the screen below
+ *              when min(W, nprobe) >= 16, three products per pair under it),
+ *              1 = FP32 FMA only, 2 = tensor cores, three products per pair
+ *              (SIEVE_EINVAL where they do not fit), 3 = as 2, but with the
+ *              tensor-core layout every pair is screened.
+ *              The screen: one fp16 product of the hi halves per (query, row) pair, whose
+ *              error is bounded by (2^-10 + 2^-12 + d 2^-22) |q| |x| +
+ *              2^-26 sqrt(d) (|q| + |x|) (|x| the largest row norm of the
+ *              row's 128-row block); only rows whose screened score reaches
+ *              the threshold minus that bound are scored again, in fp32 FMA,
+ *              and that score decides and is returned.
  */
 typedef struct {
     float tau;
@@ -188,7 +197,9 @@ sieve_status sieve_build_layout(const float *X, const int32_t *assign, int64_t n
  * centroids, pre-split for the fp16 contraction (hi = fp16(256 x),
  * lo = fp16(256 x - hi)) and stored in blocks of 128 rows in the byte order
  * of the shared-memory operand tiles (4 bytes per element, each partition
- * padded to a multiple of 128 rows).  Derived data: it changes no result.
+ * padded to a multiple of 128 rows), followed by one fp32 per block of rows:
+ * the largest Euclidean norm of its rows (the screening scan's error bound
+ * uses it).  Derived data: it changes no result.
  *   sieve_tc_layout_size   bytes of tc_rows and of tc_centroids for this view
  *                          (reads list_offsets from the device: synchronous)
  *   sieve_build_tc_layout  fills tc_rows (device, rows_bytes), tc_row_blocks

@@ -70,7 +70,7 @@ class RqViewC(C.Structure):
 
 KERNELS = ("rank", "init", "issue", "bucket", "scatter", "scan", "merge", "round_end", "finalize",
            "scan_tc", "rq_rotate", "rank_mma")
-SCAN_PATHS = {"auto": 0, "simt": 1, "tensor": 2}
+SCAN_PATHS = {"auto": 0, "simt": 1, "tensor": 2, "screen": 3}
 
 
 _lib = None

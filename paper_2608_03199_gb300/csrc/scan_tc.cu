@@ -17,12 +17,15 @@ namespace sieve {
 __device__ __forceinline__ int tc_nkb_dev(int d) { return (d + 63) / 64; }
 
 // kRQ = false: exact inner products (B = the rows' hi / lo split);
-// kRQ = true: RaBitQ-style estimates from the code layout (B = u - mid)
-template <bool kRQ>
+// kRQ = true: RaBitQ-style estimates from the code layout (B = u - mid).
+// kScreen (exact only): one product of the hi halves per pair screens every
+// row, and the rows that may reach the threshold are scored again exactly
+template <bool kRQ, bool kScreen = false>
 struct ScanModeT {
     using Args = SearchArgs;
     static constexpr int kN = 256;
     static constexpr bool kBHasLo = !kRQ;
+    static constexpr int kProducts = kScreen ? 1 : (kRQ ? 2 : 3);
     struct Tile {
         int p, ib, ni;
         int64_t r_begin, nb;
@@ -64,6 +67,12 @@ struct ScanModeT {
         int kn, item, q, rank, slot;
         float qc;   // kRQ: <q, c_p>, the centroid score of the item's rank
         float *fs;  // kRQ: this warp's copy of the chunk's 128 factors (shared memory)
+        // kScreen: |q| of the item's query, the error-bound coefficients, the
+        // largest row norm of each of the tile's 128-row blocks and that of
+        // the current chunk (loaded before its accumulator wait)
+        float qn, m_rel, m_abs, xn;
+        const float *bn;
+        long long *ids_s;   // kScreen: this warp's copy of the chunk's 128 row ids
         bool valid;
         long long qid;
         // the kept list is unordered while the tile runs; once it holds k
@@ -87,12 +96,31 @@ struct ScanModeT {
             qid = (long long)-0x7fffffffffffffffll - 1;
             qc = 0.f;
             fs = reinterpret_cast<float *>(smem + (size_t)tcp::kM * a.k * 12) + (slot >> 5) * 128;
+            ids_s = reinterpret_cast<long long *>(smem + (size_t)tcp::kM * a.k * 12) + (slot >> 5) * 128;
             if (valid) {
                 item = a.bucketed[T.ib + slot];
                 q = a.item_q[item];
                 rank = a.item_rank[item];
                 if (a.qids) qid = a.qids[q];
                 if (kRQ) qc = a.cscores[(int64_t)q * a.nprobe + rank - 1];
+            }
+            if constexpr (kScreen) {
+                // the block norms follow the layout's blocks
+                const int nkb = tc_nkb_dev(a.d);
+                bn = reinterpret_cast<const float *>(
+                         a.tc_rows + a.tc_row_blocks[a.nlist] * (int64_t)nkb * kTcBlockBytes) + T.blk0;
+                // one product of the hi halves h(256 q), h(256 x) (fp16, round to
+                // nearest: |256 q - h| <= 2^-11 |256 q| + 2^-25) differs from
+                // <q, x> by at most 2^-10 (1 + 2^-11) sum |q_i x_i| + 2^-33 sqrt(d)
+                // (|q| + |x|) (1 + 2^-11), and its fp32 accumulation of d exact
+                // products by at most d 2^-24 sum |q_i x_i| (to nearest); the
+                // margin takes 2^-10 + 2^-12 + d 2^-22 times |q| |x| (Cauchy-
+                // Schwarz, with room for the norms' own rounding and an
+                // accumulator that truncates) plus 2^-26 sqrt(d) (|q| + |x|)
+                m_rel = 0.0009765625f + 0.000244140625f + (float)a.d * 2.384185791015625e-7f;
+                m_abs = 1.4901161193847656e-8f * sqrtf((float)a.d);
+                qn = valid ? a.qnorm[q] : 0.f;
+                xn = 0.f;
             }
         }
         __device__ void find_worst(int k) {
@@ -112,10 +140,13 @@ struct ScanModeT {
         // one candidate row (s >= tau): self exclusion, then into the kept
         // list (appended while it has room, else in place of its last entry)
         __device__ __forceinline__ void take(const Args &a, const Tile &T, int64_t col, float sc) {
-            const int k = a.k;
-            if (kn == k && sc < wst_s) return;   // cannot rank before the last kept entry
+            if (a.k == kn && sc < wst_s) return;   // cannot rank before the last kept entry
             const long long id = a.ids[T.r_begin + col];
             if (id == qid) return;
+            insert(a, sc, id);
+        }
+        __device__ __forceinline__ void insert(const Args &a, float sc, long long id) {
+            const int k = a.k;
             if (kn < k) {
                 KS(kn) = sc;
                 KI(kn) = id;
@@ -155,9 +186,111 @@ struct ScanModeT {
                 take(a, T, col0 + j, pick32(e, j) * inv);
             }
         }
+        // kScreen: v holds one-product scores x 2^16.  A row whose exact score
+        // reaches the threshold (tau, or the last kept entry once k are kept)
+        // has a screened score of at least the threshold minus the margin;
+        // such rows, other than the query's own, are scored again by the
+        // whole warp in fp32, one at a time, and only that score decides.
+        // Every lane of the warp takes part (ncol is the same for all).
+        __device__ __forceinline__ void screen(const Args &a, const Tile &T, int64_t col0,
+                                               const float (&v)[32], int ncol) {
+            if (ncol <= 0) return;
+            float thr = a.tau;
+            if (kn == a.k) thr = fmaxf(thr, wst_s);
+            const float cut = (thr - (m_rel * qn * xn + m_abs * (qn + xn))) * 65536.f;
+            float mx[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) mx[j] = fmaxf(v[j], v[j + 16]);
+#pragma unroll
+            for (int w = 8; w > 0; w >>= 1)
+#pragma unroll
+                for (int j = 0; j < w; ++j) mx[j] = fmaxf(mx[j], mx[j + w]);
+            const bool any = valid && mx[0] >= cut;
+            if (!__any_sync(0xffffffffu, any)) return;
+            unsigned m = 0;
+            if (any) {
+#pragma unroll
+                for (int j = 0; j < 32; ++j) m |= (v[j] >= cut && j < ncol) ? (1u << j) : 0u;
+                // the query's own row leaves here (ids from the warp's copy)
+                const long long *cid = ids_s + (col0 & (tcb::kN - 1));
+                for (unsigned mm = m; mm; mm &= mm - 1u) {
+                    const int j = __ffs(mm) - 1;
+                    if (cid[j] == qid) m &= ~(1u << j);
+                }
+            }
+            // up to four candidates at a time, one from each of the first four
+            // lanes that have one, each scored by eight lanes (lane-strided
+            // fused multiply-adds, all loads in flight, then a butterfly sum
+            // over the eight)
+            const int lane = (int)(threadIdx.x & 31u), sub = lane >> 3;
+            for (;;) {
+                unsigned lanes = __ballot_sync(0xffffffffu, m != 0u);
+                if (!lanes) break;
+                int own = -1;   // which of the batch's pairs this lane owns
+                int Lg = 0, jg = 0, npick = 0;
+#pragma unroll
+                for (int g = 0; g < 4; ++g) {
+                    if (!lanes) break;
+                    const int L = __ffs(lanes) - 1;
+                    lanes &= lanes - 1u;
+                    const int j = __ffs(__shfl_sync(0xffffffffu, m, L)) - 1;
+                    if (lane == L) own = g;
+                    if (sub == g) {
+                        Lg = L;
+                        jg = j;
+                    }
+                    ++npick;
+                }
+                const int qL = __shfl_sync(0xffffffffu, q, Lg);
+                float acc = 0.f;
+                if (sub < npick) {   // d <= 256: at most 8 float4 of each row per lane, all in flight
+                    const float *u = a.Q + (int64_t)qL * a.d;
+                    const float *w = a.X + (T.r_begin + col0 + jg) * a.d;
+                    float4 x[8], y[8];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        const int c = 4 * (lane & 7) + 32 * i;
+                        x[i] = c < a.d ? __ldg(reinterpret_cast<const float4 *>(u + c)) : make_float4(0.f, 0.f, 0.f, 0.f);
+                        y[i] = c < a.d ? __ldg(reinterpret_cast<const float4 *>(w + c)) : make_float4(0.f, 0.f, 0.f, 0.f);
+                    }
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        acc = fmaf(x[i].x, y[i].x, acc);
+                        acc = fmaf(x[i].y, y[i].y, acc);
+                        acc = fmaf(x[i].z, y[i].z, acc);
+                        acc = fmaf(x[i].w, y[i].w, acc);
+                    }
+                }
+#pragma unroll
+                for (int o = 4; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+                // lane L of pair g reads the sum of sub-group g
+                const float sc = __shfl_sync(0xffffffffu, acc, own >= 0 ? 8 * own : 0);
+                if (own >= 0) {
+                    const int j = __ffs(m) - 1;
+                    m &= m - 1u;
+                    if (sc >= a.tau && !(kn == a.k && sc < wst_s))
+                        insert(a, sc, ids_s[(col0 & (tcb::kN - 1)) + j]);
+                }
+            }
+        }
         // kRQ: the chunk's factors into this warp's shared copy, one coalesced
         // 512-byte asynchronous copy per warp issued before the accumulator wait
-        __device__ __forceinline__ void prefetch(const Args &, const Tile &T, int ch) {
+        __device__ __forceinline__ void prefetch(const Args &a, const Tile &T, int ch) {
+            if constexpr (kScreen) {
+                // the chunk's block norm and its row ids (8-byte asynchronous
+                // copies into this warp's shared copy), in flight during the
+                // accumulator wait; every lane is done with the previous copy
+                __syncwarp();
+                xn = bn[ch];
+                const int64_t r0 = T.r_begin + (int64_t)ch * tcb::kN;
+                const int64_t left = T.nb - (int64_t)ch * tcb::kN;
+                const int nrow = left < tcb::kN ? (int)left : tcb::kN;
+                for (int j = slot & 31; j < nrow; j += 32) {
+                    const uint32_t dst = tc::smem_u32(ids_s + j);
+                    asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(dst), "l"(a.ids + r0 + j)
+                                 : "memory");
+                }
+            }
             if constexpr (kRQ) {
                 __syncwarp();   // every lane is done with the previous chunk's copy
                 const float *src = T.fac + (int64_t)ch * tcb::kN + 4 * (slot & 31);
@@ -166,7 +299,7 @@ struct ScanModeT {
             }
         }
         __device__ __forceinline__ void start(const Args &, const Tile &, int) {
-            if constexpr (kRQ) {
+            if constexpr (kRQ || kScreen) {
                 asm volatile("cp.async.wait_all;\n" ::: "memory");
                 __syncwarp();
             }
@@ -175,6 +308,10 @@ struct ScanModeT {
         // 2^16; kRQ, <u - mid, q'> x 2^8 (the codes are not scaled)
         __device__ void chunk(const Args &a, const Tile &T, int64_t col0, const float (&v)[32],
                               int ncol) {
+            if constexpr (kScreen) {
+                screen(a, T, col0, v, ncol);
+                return;
+            }
             if (!valid || ncol <= 0) return;
             if constexpr (kRQ) {
                 // the estimates qc + f <u - mid, q'> (the factor copy holds
@@ -240,6 +377,7 @@ struct ScanModeT {
 
 using ScanMode = ScanModeT<false>;
 using ScanModeRQ = ScanModeT<true>;
+using ScanModeScreen = ScanModeT<false, true>;
 
 bool scan_tc_fits(int k) { return scan_tc_smem_bytes(k) <= (size_t)(232448 - 128); }
 
@@ -269,9 +407,33 @@ cudaError_t prepare_scan_bulk(int d, int k, int stages) {
                                 (int)tcb::smem_bytes(stages, scan_epi_bytes(k)));
 }
 
+// the screening scan: stages of two 16 KB K-blocks (the hi halves); the
+// epilogue's bytes add one 1 KB copy of a chunk's row ids per epilogue warp
+constexpr int kScreenStagesMax = 6;
+static size_t scan_screen_epi_bytes(int k) { return scan_epi_bytes(k) + 4 * 1024; }
+
+int scan_screen_stages(int d, int k) {
+    return tcb::stages_for((int)ceil_div(d, 64), scan_screen_epi_bytes(k), 232448 - 128,
+                           tcb::kStageBytesHi, kScreenStagesMax);
+}
+
+__global__ void __launch_bounds__(tcb::kThreads, 1) k_scan_screen(SearchArgs a) {
+    extern __shared__ unsigned char smem_raw[];
+    tcb::run_bulk<ScanModeScreen>(a, smem_raw, a.tc_stages);
+}
+
+cudaError_t prepare_scan_screen(int d, int k, int stages) {
+    return cudaFuncSetAttribute(k_scan_screen, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)tcb::smem_bytes(stages, scan_screen_epi_bytes(k), tcb::kStageBytesHi));
+}
+
 void enqueue_scan_bulk(const SearchArgs &a, cudaStream_t st) {
-    k_scan_bulk<<<num_sms(), tcb::kThreads,
-                  tcb::smem_bytes(a.tc_stages, scan_epi_bytes(a.k)), st>>>(a);
+    if (a.tc_screen)
+        k_scan_screen<<<num_sms(), tcb::kThreads,
+                        tcb::smem_bytes(a.tc_stages, scan_screen_epi_bytes(a.k), tcb::kStageBytesHi), st>>>(a);
+    else
+        k_scan_bulk<<<num_sms(), tcb::kThreads,
+                      tcb::smem_bytes(a.tc_stages, scan_epi_bytes(a.k)), st>>>(a);
 }
 
 // the scan over codes: stages of two 16 KB K-blocks; the epilogue's bytes add

@@ -44,6 +44,10 @@ struct SearchArgs {
     const int64_t *tc_row_blocks;       // [nlist+1] block offsets of that layout
     const unsigned char *tc_cent;       // tensor-core layout of the centroids (nullable)
     int tc_stages;                      // B stages of the bulk pipeline (0 = not used)
+    int tc_screen;                      // 1: the bulk scan screens with one product per
+                                        // pair and rescores candidates in FP32; 0: three
+                                        // products per pair
+    float *qnorm;                       // [nq] Euclidean norms of the queries (screening)
     // per-item local results
     int *res_cnt;                       // [cap]
     float *res_s;                       // [cap][k]
@@ -91,7 +95,10 @@ void enqueue_scan_tc(const SearchArgs &a, cudaStream_t st);
 // the same fed from the tensor-core layout by bulk copies (d <= 256)
 int scan_bulk_stages(int d, int k);              // 0 when it does not apply
 cudaError_t prepare_scan_bulk(int d, int k, int stages);
-void enqueue_scan_bulk(const SearchArgs &a, cudaStream_t st);
+// the screening variant (a.tc_screen = 1): hi halves of B only, one product
+int scan_screen_stages(int d, int k);            // 0 when it does not apply
+cudaError_t prepare_scan_screen(int d, int k, int stages);
+void enqueue_scan_bulk(const SearchArgs &a, cudaStream_t st);   // either variant
 
 // centroid ranking (rank_kernel.cu): prepare_rank once before launches or
 // stream capture, then enqueue_rank (a single kernel launch)
@@ -143,6 +150,7 @@ cudaError_t launch_merge_shards(int nshards, int64_t nq, int k, const long long 
 constexpr int kTcRows = 128;                   // rows per block
 constexpr int64_t kTcBlockBytes = 32768;       // one K-block (64 elements) of a block: hi + lo fp16
 int tc_nkb(int d);
+size_t tc_norms_bytes(int64_t nblocks);        // the per-block row norms after the blocks
 cudaError_t launch_tc_layout_rows(const float *X, const int64_t *off, int64_t nparts, int d,
                                   int64_t *blk_off, unsigned char *out, cudaStream_t st);
 cudaError_t launch_tc_layout_matrix(const float *X, int64_t nrows, int d, unsigned char *out,

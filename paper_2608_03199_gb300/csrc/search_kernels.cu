@@ -48,6 +48,24 @@ __global__ void k_init(SearchArgs a) {
     }
 }
 
+// the queries' Euclidean norms for the screening scan's error bound: a warp
+// per query, lane-strided fp32 sums of squares and a butterfly sum
+__global__ void k_qnorm(SearchArgs a) {
+    const int lane = (int)lane_id();
+    const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
+    for (int64_t q = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; q < a.nq; q += warps) {
+        const float *row = a.Q + q * a.d;
+        float ss = 0.f;
+        for (int c = 4 * lane; c < a.d; c += 128) {
+            const float4 x = __ldg(reinterpret_cast<const float4 *>(row + c));
+            ss = fmaf(x.x, x.x, fmaf(x.y, x.y, fmaf(x.z, x.z, fmaf(x.w, x.w, ss))));
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+        if (lane == 0) a.qnorm[q] = sqrtf(ss);
+    }
+}
+
 __global__ void k_finalize(SearchArgs a) {
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < a.nq; q += stride)
@@ -569,6 +587,8 @@ cudaError_t launch_init(const SearchArgs &a, cudaStream_t st) {
     cudaError_t e = cudaMemsetAsync(a.ctl, 0, sizeof(Ctl), st);
     if (e != cudaSuccess) return e;
     k_init<<<blocks, 256, 0, st>>>(a);
+    if (a.tc_screen && a.nq > 0)
+        k_qnorm<<<(int)std::min<int64_t>(ceil_div(a.nq, 8), 16 * num_sms()), 256, 0, st>>>(a);
     return cudaGetLastError();
 }
 

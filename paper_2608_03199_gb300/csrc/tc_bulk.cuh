@@ -13,6 +13,9 @@
 //
 // Tensor memory (512 columns): two 128-column fp32 accumulators, then the
 // tile's A: 64 columns per K-block of 64 elements (32 hi, 32 lo); d <= 256.
+// A screening mode (one product per K step, hi halves only) copies just the
+// hi half of each K-block of B and keeps only A's hi columns (32 per
+// K-block), so three accumulators fit.
 //
 // Warp roles (448 threads, one block per SM):
 //   warps 0-7   A writers: warp w writes lanes 32 (w % 4) .. +31 for the
@@ -27,8 +30,9 @@
 //               other roles through a small ring in shared memory; it then
 //               issues the tile's bulk copies of B stages ("b_full" with the
 //               transfer byte count; waits on "b_empty")
-//   warp 9      allocates the tensor memory; lane 0 issues three kind::f16
-//               MMAs per K step (A from tensor memory, B from shared memory)
+//   warp 9      allocates the tensor memory; lane 0 issues the mode's one to
+//               three kind::f16 MMAs per K step (A from tensor memory, B from
+//               shared memory)
 //   warps 10-13 epilogue: thread i owns tensor-memory lane i = A row i; it
 //               hands its row of a chunk (scores x 2^16) to Mode::Epi
 // Every wait is bounded; giving up sets SIEVE_ETIMEOUT in the mode's status
@@ -55,7 +59,7 @@ constexpr int kMaxStages = 8;                 // barrier slots for B stages
 constexpr int kStagesMax = 5;                 // stages beyond five did not time faster
 constexpr uint32_t kKbBytes = 32768;          // one K-block of 128 rows: hi 16 KB + lo 16 KB
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kAColumn0 = 2 * kN;        // A after the two accumulators
+constexpr int kMaxAcc = 3;                    // accumulator slots (barriers)
 constexpr uint32_t kWaitPolls = 1u << 24;
 constexpr int kRing = 8;                      // tiles handed from the scheduler to the other roles
 constexpr uint32_t kRingReaders = kAWriterWarps + 1 + 4;   // A-writer warps, MMA lane, epilogue warps
@@ -93,6 +97,14 @@ struct b_has_lo { static constexpr bool value = true; };
 template <class Mode>
 struct b_has_lo<Mode, decltype((void)Mode::kBHasLo)> { static constexpr bool value = Mode::kBHasLo; };
 
+// products per K step: 3 (lo_a hi_b + hi_a lo_b + hi_a hi_b), 2 (B exact in
+// fp16: lo_a b + hi_a b) or 1 (a screen: hi_a hi_b, the hi halves of a split
+// B copied alone)
+template <class Mode, class = void>
+struct mma_products { static constexpr int value = b_has_lo<Mode>::value ? 3 : 2; };
+template <class Mode>
+struct mma_products<Mode, decltype((void)Mode::kProducts)> { static constexpr int value = Mode::kProducts; };
+
 // one 32-column group of an accumulator row to the mode's epilogue
 template <class Epi, class Args, class Tile>
 __device__ __forceinline__ void hand(Epi &epi, const Args &a, const Tile &T, int64_t col0,
@@ -114,12 +126,21 @@ template <class Mode>
 __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned char *smem_raw,
                                          int stages) {
     constexpr uint32_t kIdesc = tc::idesc_f16(tcp::kM, kN);
-    constexpr bool kLo = b_has_lo<Mode>::value;
+    constexpr int kProd = mma_products<Mode>::value;
+    constexpr bool kLo = kProd == 3;                          // B's lo half in the stage
     constexpr uint32_t kKbB = kLo ? kKbBytes : kKbBytesHi;     // bytes of one K-block of B
+    // bytes of one K-block of B in global memory: a screen copies the hi half
+    // of each K-block of the split layout, one copy per K-block
+    constexpr uint32_t kSrcKb = b_has_lo<Mode>::value ? kKbBytes : kKbBytesHi;
+    // accumulators and A's tensor-memory columns per K-block: with hi and lo
+    // of A (64 columns per K-block) two 128-column accumulators fit beside it;
+    // a screen keeps only A's hi half (32 columns), which leaves room for three
+    constexpr uint32_t kAcc = kProd == 1 ? 3 : 2;
+    constexpr uint32_t kAKb = kProd == 1 ? 32 : 64;
     constexpr int kKs = kKbPerStage;                          // K-blocks per B stage
     constexpr uint32_t kStage = kKs * kKbB;                    // bytes of one B stage
     __shared__ __align__(8) uint64_t a_full[kMaxKb], a_empty[kMaxKb], b_full[kMaxStages],
-        b_empty[kMaxStages], dfull_bar[2], dempty_bar[2], drain_bar, ring_full[kRing],
+        b_empty[kMaxStages], dfull_bar[kMaxAcc], dempty_bar[kMaxAcc], drain_bar, ring_full[kRing],
         ring_empty[kRing];
     __shared__ int ring_tile[kRing];
     __shared__ uint32_t tmem_slot;
@@ -145,7 +166,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
             tc::mbar_init(&b_full[s], 1);
             tc::mbar_init(&b_empty[s], 1);
         }
-        for (int b = 0; b < 2; ++b) {
+        for (uint32_t b = 0; b < kAcc; ++b) {
             tc::mbar_init(&dfull_bar[b], 1);
             tc::mbar_init(&dempty_bar[b], 4 * 32);
         }
@@ -162,7 +183,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
     __syncthreads();
     tc::fence_after_sync();
     const uint32_t tmem = tmem_slot;
-    const uint32_t tA = tmem + kAColumn0;
+    const uint32_t tA = tmem + kAcc * kN;                      // A after the accumulators
 
     auto wait = [&](uint64_t *bar, uint32_t parity) -> bool {
         for (uint32_t it = 0; it < kWaitPolls; ++it) {
@@ -213,9 +234,9 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                         tcp::split2(v.x, v.y, hi[2 * q4], lo[2 * q4]);
                         tcp::split2(v.z, v.w, hi[2 * q4 + 1], lo[2 * q4 + 1]);
                     }
-                    const uint32_t col = tA + (uint32_t)kb * 64 + (uint32_t)half * 16;
+                    const uint32_t col = tA + (uint32_t)kb * kAKb + (uint32_t)half * 16;
                     tc::tmem_st16(col + lane_bits, hi);
-                    tc::tmem_st16(col + 32 + lane_bits, lo);
+                    if constexpr (kProd > 1) tc::tmem_st16(col + 32 + lane_bits, lo);
                 }
                 tc::tmem_st_wait();
                 tc::fence_before_sync();
@@ -246,8 +267,14 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                         const uint32_t bytes = (uint32_t)(nkb - kb < kKs ? nkb - kb : kKs) * kKbB;
                         if (!(ok = wait(&b_empty[st], sph ^ 1u))) break;
                         tc::mbar_arrive_expect_tx(&b_full[st], bytes);
-                        tc::bulk_g2s(Bst + (size_t)st * kStage, src + (size_t)kb * kKbB, bytes,
-                                     &b_full[st]);
+                        if constexpr (kSrcKb == kKbB) {
+                            tc::bulk_g2s(Bst + (size_t)st * kStage, src + (size_t)kb * kKbB, bytes,
+                                         &b_full[st]);
+                        } else {   // the hi halves of this stage's K-blocks
+                            for (uint32_t j = 0; j * kKbB < bytes; ++j)
+                                tc::bulk_g2s(Bst + (size_t)st * kStage + j * kKbB,
+                                             src + ((size_t)kb + j) * kSrcKb, kKbB, &b_full[st]);
+                        }
                         ++s;
                     }
                 }
@@ -274,7 +301,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                 const int nch = (int)ceil_div(T.nb, kN);
                 if (nch == 0) continue;
                 for (int ch = 0; ok && ch < nch; ++ch, ++c) {
-                    const uint32_t buf = c & 1u, dph = (c >> 1) & 1u;
+                    const uint32_t buf = c % kAcc, dph = (c / kAcc) & 1u;
                     if (!(ok = wait(&dempty_bar[buf], dph ^ 1u))) break;
                     tc::fence_after_sync();
                     const uint32_t dt = tmem + buf * kN;
@@ -286,7 +313,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                         if (!ok || !(ok = wait(&b_full[st], ph))) break;
                         tc::fence_after_sync();
                         for (int kb = kb0; kb < kb1; ++kb) {
-                            const uint32_t a_hi = tA + (uint32_t)kb * 64, a_lo = a_hi + 32;
+                            const uint32_t a_hi = tA + (uint32_t)kb * kAKb, a_lo = a_hi + 32;
                             const uint32_t b_hi = tc::smem_u32(Bst + (size_t)st * kStage) +
                                                   (uint32_t)(kb - kb0) * kKbB;
                             // a K step moves the descriptors' start address by 32 bytes
@@ -303,7 +330,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                                     tc::mma_f16_ta(dt, a_hi + ao, bl + bo, kIdesc, 1u);
                                     tc::mma_f16_ta(dt, a_hi + ao, bh + bo, kIdesc, 1u);
                                 }
-                            } else {   // B exact in fp16: hi and lo of A against it
+                            } else if constexpr (kProd == 2) {   // B exact in fp16: hi and lo of A against it
 #pragma unroll
                                 for (int ks = 0; ks < 4; ++ks) {
                                     const uint32_t ao = ks * 8;
@@ -311,6 +338,11 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                                     tc::mma_f16_ta(dt, a_lo + ao, bh + bo, kIdesc, (kb > 0 || ks > 0) ? 1u : 0u);
                                     tc::mma_f16_ta(dt, a_hi + ao, bh + bo, kIdesc, 1u);
                                 }
+                            } else {   // a screen: the hi halves alone
+#pragma unroll
+                                for (int ks = 0; ks < 4; ++ks)
+                                    tc::mma_f16_ta(dt, a_hi + ks * 8, bh + 2 * ks, kIdesc,
+                                                   (kb > 0 || ks > 0) ? 1u : 0u);
                             }
                         }
                         tc::mma_commit(&b_empty[st]);
@@ -342,7 +374,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
             const int nch = (int)ceil_div(T.nb, kN);
             epi.begin(a, T, slot, epi_smem);
             for (int ch = 0; ch < nch; ++ch, ++c) {
-                const uint32_t buf = c & 1u, dph = (c >> 1) & 1u;
+                const uint32_t buf = c % kAcc, dph = (c / kAcc) & 1u;
                 epi.prefetch(a, T, ch);   // per-chunk loads, in flight during the wait
                 ok = __all_sync(0xffffffffu, wait(&dfull_bar[buf], dph));
                 if (!ok) break;

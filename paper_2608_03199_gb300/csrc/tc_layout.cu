@@ -10,6 +10,9 @@
 // each a 128-row x 128-byte tile whose 16-byte chunk c of row r sits at
 // chunk c ^ (r & 7).  Block b, K-block kb of the matrix starts at byte
 // (b * nkb + kb) * 32768.  Partition p owns blocks blk_off[p] .. blk_off[p+1]-1.
+// The row layout ends with one fp32 per block, the largest Euclidean norm of
+// its rows: the screening scan bounds the error of its one-product scores
+// with it.
 #include <cuda_fp16.h>
 
 #include "search.cuh"
@@ -99,7 +102,41 @@ __global__ void k_tc_fill(const float *X, const int64_t *off, int64_t nparts, in
     }
 }
 
+// a warp per block of partition rows: the largest norm of the block's rows,
+// stored after the blocks (fp32 sums of squares; the screening bound leaves
+// room for their rounding)
+__global__ void k_tc_norms(const float *X, const int64_t *off, int64_t nparts, const int64_t *blk_off,
+                           int d, int nkb, unsigned char *out) {
+    const int64_t nblocks = blk_off[nparts];
+    float *norms = reinterpret_cast<float *>(out + nblocks * nkb * kTcBlockBytes);
+    const int lane = (int)lane_id();
+    const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
+    for (int64_t blk = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; blk < nblocks; blk += warps) {
+        int64_t lo_p = 0, hi_p = nparts;    // partition: blk_off[p] <= blk < blk_off[p + 1]
+        while (hi_p - lo_p > 1) {
+            const int64_t mid = (lo_p + hi_p) >> 1;
+            if (blk_off[mid] <= blk) lo_p = mid; else hi_p = mid;
+        }
+        const int64_t r0 = off[lo_p] + (blk - blk_off[lo_p]) * kTcRows;
+        const int64_t r1 = r0 + kTcRows < off[lo_p + 1] ? r0 + kTcRows : off[lo_p + 1];
+        float best = 0.f;
+        for (int64_t r = r0; r < r1; ++r) {
+            float ss = 0.f;
+            for (int c = 4 * lane; c < d; c += 128) {
+                const float4 x = __ldg(reinterpret_cast<const float4 *>(X + r * d + c));
+                ss = fmaf(x.x, x.x, fmaf(x.y, x.y, fmaf(x.z, x.z, fmaf(x.w, x.w, ss))));
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+            best = fmaxf(best, sqrtf(ss));
+        }
+        if (lane == 0) norms[blk] = best;
+    }
+}
+
 int tc_nkb(int d) { return (int)ceil_div(d, 64); }
+
+size_t tc_norms_bytes(int64_t nblocks) { return (size_t)round_up(nblocks * 4, 256); }
 
 cudaError_t launch_tc_block_scan(const int64_t *off, int64_t nparts, int64_t *blk_off, cudaStream_t st) {
     k_tc_block_scan<<<1, 1024, 0, st>>>(off, nparts, blk_off);
@@ -110,6 +147,7 @@ cudaError_t launch_tc_layout_rows(const float *X, const int64_t *off, int64_t np
                                   int64_t *blk_off, unsigned char *out, cudaStream_t st) {
     k_tc_block_scan<<<1, 1024, 0, st>>>(off, nparts, blk_off);
     k_tc_fill<<<16 * num_sms(), 256, 0, st>>>(X, off, nparts, 0, blk_off, d, tc_nkb(d), out);
+    k_tc_norms<<<8 * num_sms(), 256, 0, st>>>(X, off, nparts, blk_off, d, tc_nkb(d), out);
     return cudaGetLastError();
 }
 
