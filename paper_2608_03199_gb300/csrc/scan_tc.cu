@@ -3,8 +3,8 @@
 // within-partition search of Sec. 4.1 and Sec. 5, for large groups).
 //
 // A tile is (partition p, up to 128 items of p's group): the items' queries
-// are the A rows, p's rows are the B rows, streamed 256 at a time through the
-// 3xTF32 pipeline of tc_pipeline.cuh.  Epilogue thread i (the tile's i-th
+// are the A rows, p's rows are the B rows, streamed in chunks through the
+// fp16-split pipelines (tc_bulk.cuh, tc_pipeline.cuh).  Epilogue thread i (the tile's i-th
 // item) keeps the rows with s >= tau, other than the query itself, in a
 // private top-k in shared memory; after p's last chunk it writes the item's
 // local result and, on a hit at rank j, raises the query's stop line to

@@ -1,7 +1,7 @@
 // tcgen05.cuh -- thin wrappers over the sm_100-family tensor-core PTX used by
-// the 3xTF32 scan: tensor-memory allocation, shared-memory matrix
-// descriptors, kind::tf32 MMA, commit to an mbarrier, tensor-memory loads,
-// and bounded mbarrier waits.
+// the tensor-core pipelines: tensor-memory allocation, shared-memory matrix
+// descriptors, kind::f16 MMA, commit to an mbarrier, tensor-memory loads and
+// stores, bulk copies and bounded mbarrier waits.
 #pragma once
 
 #include <stdint.h>
@@ -29,14 +29,6 @@ __device__ __forceinline__ uint64_t desc_k_sw128(uint32_t saddr) {
     return d;
 }
 
-// Instruction descriptor of kind::tf32 with fp32 accumulation, both
-// operands K-major: D format f32 (bits 4-5 = 1), A and B format tf32
-// (bits 7-9 and 10-12 = 2), N >> 3 in bits 17-22, M >> 4 in bits 24-28.
-__host__ __device__ constexpr uint32_t idesc_tf32(int M, int N) {
-    return (1u << 4) | (2u << 7) | (2u << 10) | ((uint32_t)(N >> 3) << 17) |
-           ((uint32_t)(M >> 4) << 24);
-}
-
 // Instruction descriptor of kind::f16 with fp16 A and B, fp32 accumulation,
 // both operands K-major: D format f32 (bits 4-5 = 1), A and B format f16
 // (bits 7-9 and 10-12 = 0), N >> 3 in bits 17-22, M >> 4 in bits 24-28.
@@ -55,15 +47,6 @@ __device__ __forceinline__ void tmem_alloc(uint32_t *slot_smem, uint32_t ncols) 
 __device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
                  : "memory");
-}
-
-__device__ __forceinline__ void mma_tf32(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
-                                         uint32_t idesc, uint32_t accumulate) {
-    asm volatile(
-        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
-        : "memory");
 }
 
 // kind::f16 MMA with A in tensor memory: lane i holds row i of A, each 32-bit
@@ -206,12 +189,6 @@ __device__ __forceinline__ void bulk_g2s(void *smem_dst, const void *gmem_src, u
 // memory to be brought into L2; no completion to wait for
 __device__ __forceinline__ void prefetch_l2(const void *gmem, uint32_t bytes) {
     asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(gmem), "r"(bytes) : "memory");
-}
-
-__device__ __forceinline__ uint32_t to_tf32(float x) {
-    uint32_t r;
-    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
-    return r;
 }
 
 }  // namespace tc

@@ -190,8 +190,9 @@ def test_schedule_changes_nothing(deep, g_deep, path):
 
 @pytest.mark.parametrize("path", ["simt", "tensor", "auto"])
 def test_scan_paths_parity(tiny, g_tiny, deep, g_deep, path):
-    """Both contraction paths (FP32 FMA, tensor-core 3xTF32) and the automatic
-    split meet the parity bar, on groups of every size."""
+    """Both contraction paths (FP32 FMA, the tensor-core fp16 split) and the
+    automatic choice meet the parity bar, on groups of every size (the
+    automatic path screens at W = infinity)."""
     c = tiny["cfg"]
     for la in (0, 1):
         check(tiny, g_tiny, tiny["Q"], tiny["qids"], c.tau, c.k, c.nprobe, c.W, la, scan_path=path)
@@ -201,9 +202,9 @@ def test_scan_paths_parity(tiny, g_tiny, deep, g_deep, path):
 
 
 def test_tensor_path_scores_match_fp64(tiny, g_tiny, dev):
-    """Every returned similarity of the 3xTF32 path is within 1e-6 of the fp64
-    inner product of the same pair (the split's error bound, well inside the
-    1e-5 tolerance)."""
+    """Every returned similarity of the three-product fp16 split is within 1e-6
+    of the fp64 inner product of the same pair (the split's error bound, well
+    inside the 1e-5 tolerance)."""
     c = tiny["cfg"]
     got = run(g_tiny, tiny["Q"], tiny["qids"], 0.5, 16, c.nprobe, BIG_W, lookahead=1,
               scan_path="tensor")
