@@ -57,3 +57,19 @@ def test_host_only_calls_without_gpu():
     v.d = 62
     assert lib.sieve_search_workspace_size(ctypes.byref(v), 100, ctypes.byref(p), 0,
                                            ctypes.byref(n)) == -1
+
+
+def test_scan_path_values_without_gpu():
+    """scan_path 0..3 (automatic, FP32 FMA, three fp16 products, the screen)
+    are accepted; anything else is SIEVE_EINVAL before any device work."""
+    lib = sieve.lib()
+    n = ctypes.c_size_t()
+    v = sieve.IndexViewC(n=1000, nlist=16, d=64, vectors=16, ids=16, list_offsets=16, centroids=16)
+    for path in ("auto", "simt", "tensor", "screen", 0, 1, 2, 3):
+        p = sieve._params(0.9, 10, 8, 4, True, 0, 0, scan_path=path)
+        assert lib.sieve_search_workspace_size(ctypes.byref(v), 100, ctypes.byref(p), 0,
+                                               ctypes.byref(n)) == 0
+    for path in (-1, 4):
+        p = sieve._params(0.9, 10, 8, 4, True, 0, 0, scan_path=path)
+        assert lib.sieve_search_workspace_size(ctypes.byref(v), 100, ctypes.byref(p), 0,
+                                               ctypes.byref(n)) == -1
