@@ -352,9 +352,21 @@ def cpu_baseline(w, cfg, target_s):
     oracle.search(idx, w["Q"][:sample], cfg.tau, cfg.k, cfg.nprobe, cfg.W,
                   qids=w["qids"][:sample], threads=threads)
     dt = time.perf_counter() - t0
+    # fixed probing (W = nprobe) on a smaller sample: a third of the time budget
+    t0 = time.perf_counter()
+    oracle.search(idx, w["Q"][:probe], cfg.tau, cfg.k, cfg.nprobe, cfg.nprobe,
+                  qids=w["qids"][:probe], threads=threads)
+    per_q = (time.perf_counter() - t0) / probe
+    fsample = int(min(cfg.nq, max(probe, target_s / 3 / max(per_q, 1e-9))))
+    t0 = time.perf_counter()
+    oracle.search(idx, w["Q"][:fsample], cfg.tau, cfg.k, cfg.nprobe, cfg.nprobe,
+                  qids=w["qids"][:fsample], threads=threads)
+    fdt = time.perf_counter() - t0
     return {"value": sample / dt, "unit": "queries/s", "cores": threads, "kind": "oracle",
             "sample": f"first {sample:,} of the {cfg.nq:,} queries, W={cfg.W}, "
-                      f"{dt:.1f} s on {threads} host threads"}
+                      f"{dt:.1f} s on {threads} host threads",
+            "fixed_probe": {"value": fsample / fdt, "unit": "queries/s",
+                            "sample": f"first {fsample:,} queries, W={cfg.nprobe}, {fdt:.1f} s"}}
 
 
 def bruteforce_recall(X, ids, Q, qids, tau, k, results, sample=1000, seed=777):

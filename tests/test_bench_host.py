@@ -41,3 +41,15 @@ def test_automatic_scan_rule():
     assert bench.uses_screen(types.SimpleNamespace(scan_path="screen"), cfg, 8, True)
     assert not bench.uses_screen(types.SimpleNamespace(scan_path="tensor"), cfg, 64, True)
     assert not bench.uses_screen(auto, types.SimpleNamespace(nprobe=12), 64, True)
+
+
+def test_cpu_baseline_times_both_modes():
+    """The oracle's CPU timing (the bench's cpu_baseline leg) on the tiny
+    workload: the W = 8-style window and fixed probing, each on a bounded
+    sample, with the thread count reported."""
+    wl = synth.make_workload("tiny", device="cpu")
+    cfg = wl["cfg"]
+    out = bench.cpu_baseline(bench.host_arrays(wl), cfg, 0.5)
+    assert out["kind"] == "oracle" and out["cores"] >= 1 and out["value"] > 0
+    assert out["fixed_probe"]["value"] > 0
+    assert f"W={cfg.nprobe}" in out["fixed_probe"]["sample"]
