@@ -4,9 +4,13 @@
 A step is one ``sieve_search`` call over one batch of queries: centroid
 ranking, then device-resident rounds of issue / bucketing / grouped scan with
 the fused tau, top-k and stop-line epilogue / merge until every query has
-stopped.  The workload is the 1M x 256 configuration (1,024 partitions,
-100K database-drawn queries, tau 0.90, k 10, nprobe 64, W 8, lookahead on),
-synthetic and seeded (``synth``), with the index resident in HBM.
+stopped.  The default workload is the largest single-GPU configuration, the
+100M x 96 corpus (65,536 partitions, 1M database-drawn queries, tau 0.90,
+k 10, nprobe 256, W 8 against fixed probing, lookahead on), synthetic and
+seeded (``synth``), with the index resident in HBM; ``--config`` picks
+another (tiny, 1m, 10m512, 10m256, 100m) and ``--all-configs`` runs every
+configuration in its own process and prints one line per configuration plus
+a summary line.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl sieve|reference]
 
@@ -46,7 +50,10 @@ def parse():
     ap.add_argument("--steps", type=int, default=400)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=("sieve", "reference"), default="sieve")
-    ap.add_argument("--config", default="1m")
+    ap.add_argument("--config", default="100m")
+    ap.add_argument("--all-configs", action="store_true",
+                    help="every configuration, each in its own process (a line per "
+                         "configuration, then a summary line with a per_config dict)")
     ap.add_argument("--skip-cpu-baseline", action="store_true")
     ap.add_argument("--skip-e2e", action="store_true")
     ap.add_argument("--sweep", action="store_true",
@@ -337,8 +344,57 @@ def time_steps(fn, steps, warmup, world, dev):
     return max_over_ranks(ms, world, dev)
 
 
-def cpu_baseline(w, cfg, target_s):
-    """The oracle (fp64, OpenMP over queries) on a bounded query sample."""
+def cpu_model():
+    """The host CPU's model name (lscpu, else /proc/cpuinfo), for the record."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    try:
+        for line in open("/proc/cpuinfo"):
+            if line.lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    import platform
+    return platform.processor() or platform.machine()
+
+
+PARITY_TOL = 1e-5   # scores; and how close to a rounding flip a divergence may sit
+
+
+def parity_sample(oracle, idx, Q, qids, cfg, W, ref, got):
+    """GPU results of the first queries against the oracle's on the same
+    queries: ids, counts and probes identical, or the query differs where
+    the oracle's fragility tags put a decision within 1e-5 of a flip (a
+    similarity that close to tau, a k-th / (k+1)-th gap or two centroid
+    scores that close: allowed, counted); scores within 1e-5."""
+    g_ids, g_sc, g_cnt, g_pr = got
+    same = ((g_pr == ref["probes"]) & (g_cnt == ref["count"]) & (g_ids == ref["ids"]).all(axis=1))
+    bad = np.flatnonzero(~same)
+    allowed = np.zeros(len(same), bool)
+    if len(bad):
+        order = oracle.rank(Q[bad], idx["centroids"], cfg.nprobe)
+        upto = np.maximum(g_pr[bad], ref["probes"][bad]).astype(np.int32)
+        tg, kg, cg = oracle.fragility(idx, Q[bad], cfg.tau, cfg.k, cfg.nprobe, order, upto,
+                                      qids=qids[bad])
+        allowed[bad] = (tg < PARITY_TOL) | (kg < PARITY_TOL) | (cg < PARITY_TOL)
+    valid = np.arange(cfg.k)[None, :] < ref["count"][:, None]
+    with np.errstate(invalid="ignore"):
+        err = np.where(valid & same[:, None], np.abs(g_sc.astype(np.float64) - ref["scores"]), 0.0)
+    return {"queries": int(len(same)), "W": W, "exact": int(same.sum()),
+            "allowed": int(allowed.sum()), "unexplained": int((~same & ~allowed).sum()),
+            "max_score_err": float(err.max()) if err.size else 0.0}
+
+
+def cpu_baseline(w, cfg, target_s, gpu_w=None, gpu_fixed=None):
+    """The oracle (fp64, OpenMP over queries) on a bounded query sample, timed
+    at the workload's W and at fixed probing.  gpu_w / gpu_fixed (host numpy
+    (ids, scores, count, probes) of every query, nullable): the GPU's results
+    of the same calls, compared with the oracle's on the timed samples."""
     import oracle
     idx = {k: w[k] for k in ("X", "ids", "assign", "centroids")}
     threads = oracle.default_threads()
@@ -349,8 +405,8 @@ def cpu_baseline(w, cfg, target_s):
     per_q = (time.perf_counter() - t0) / probe
     sample = int(min(cfg.nq, max(probe, target_s / max(per_q, 1e-9))))
     t0 = time.perf_counter()
-    oracle.search(idx, w["Q"][:sample], cfg.tau, cfg.k, cfg.nprobe, cfg.W,
-                  qids=w["qids"][:sample], threads=threads)
+    ref = oracle.search(idx, w["Q"][:sample], cfg.tau, cfg.k, cfg.nprobe, cfg.W,
+                        qids=w["qids"][:sample], threads=threads)
     dt = time.perf_counter() - t0
     # fixed probing (W = nprobe) on a smaller sample: a third of the time budget
     t0 = time.perf_counter()
@@ -359,14 +415,24 @@ def cpu_baseline(w, cfg, target_s):
     per_q = (time.perf_counter() - t0) / probe
     fsample = int(min(cfg.nq, max(probe, target_s / 3 / max(per_q, 1e-9))))
     t0 = time.perf_counter()
-    oracle.search(idx, w["Q"][:fsample], cfg.tau, cfg.k, cfg.nprobe, cfg.nprobe,
-                  qids=w["qids"][:fsample], threads=threads)
+    fref = oracle.search(idx, w["Q"][:fsample], cfg.tau, cfg.k, cfg.nprobe, cfg.nprobe,
+                         qids=w["qids"][:fsample], threads=threads)
     fdt = time.perf_counter() - t0
-    return {"value": sample / dt, "unit": "queries/s", "cores": threads, "kind": "oracle",
-            "sample": f"first {sample:,} of the {cfg.nq:,} queries, W={cfg.W}, "
-                      f"{dt:.1f} s on {threads} host threads",
-            "fixed_probe": {"value": fsample / fdt, "unit": "queries/s",
-                            "sample": f"first {fsample:,} queries, W={cfg.nprobe}, {fdt:.1f} s"}}
+    out = {"value": sample / dt, "unit": "queries/s", "cores": threads, "kind": "oracle",
+           "cpu_model": cpu_model(),
+           "sample": f"first {sample:,} of the {cfg.nq:,} queries, W={cfg.W}, "
+                     f"{dt:.1f} s on {threads} host threads",
+           "fixed_probe": {"value": fsample / fdt, "unit": "queries/s",
+                           "sample": f"first {fsample:,} queries, W={cfg.nprobe}, {fdt:.1f} s"}}
+    parity = {}
+    if gpu_w is not None:
+        parity[f"W{cfg.W}"] = parity_sample(oracle, idx, w["Q"][:sample], w["qids"][:sample], cfg,
+                                            cfg.W, ref, tuple(a[:sample] for a in gpu_w))
+    if gpu_fixed is not None:
+        parity["fixed_probe"] = parity_sample(oracle, idx, w["Q"][:fsample], w["qids"][:fsample],
+                                              cfg, cfg.nprobe, fref,
+                                              tuple(a[:fsample] for a in gpu_fixed))
+    return out, parity
 
 
 def bruteforce_recall(X, ids, Q, qids, tau, k, results, sample=1000, seed=777):
@@ -503,6 +569,11 @@ def run_sieve(args, cfg, world, rank, local):
                          query_ids=qids, workspace=ws, scan_path=args.scan_path)
     recall_bf = bruteforce_recall(wl["X"], wl["ids"], Q, qids, cfg.tau, k,
                                   {f"W{cfg.W}": (outs[0], outs[2]), "fixed_probe": (fixed[0], fixed[2])})
+    # host copies of both result sets, for the oracle comparison of the
+    # cpu_baseline leg (the first queries are the oracle's sample)
+    keep = min(nq, 200_000)
+    gpu_w = tuple(t[:keep].cpu().numpy() for t in outs)
+    gpu_fixed = tuple(t[:keep].cpu().numpy() for t in fixed)
     del fixed
 
     # in-call window calibration (Appendix A): a 2% sample fully probed, a 0.5%
@@ -580,7 +651,8 @@ def run_sieve(args, cfg, world, rank, local):
         "data": "synthetic",
         "config": {"workload": workload_desc(cfg), "nq_per_gpu": nq, "parallelism": f"query-shard x{world}",
                    "scan_path": args.scan_path,
-                   "l2": "inputs larger than L2 (index 1.02 GB streamed per step)"},
+                   "l2": f"inputs larger than L2 (index {cfg.n * cfg.d * 4 / 1e9:.2f} GB "
+                         f"streamed per step)"},
         "fixed_probe": {"value": nq * world / (ms_fixed * 1e-3), "ms_per_step": ms_fixed,
                         "W": cfg.nprobe,
                         "scan": "screen" if uses_screen(args, cfg, cfg.nprobe, index.tc_rows is not None)
@@ -604,7 +676,8 @@ def run_sieve(args, cfg, world, rank, local):
         "e2e": e2e,
     }
     if rank == 0 and world == 1 and not args.skip_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(host_arrays(wl), cfg, args.cpu_seconds)
+        line["cpu_baseline"], line["parity"] = cpu_baseline(host_arrays(wl), cfg, args.cpu_seconds,
+                                                            gpu_w, gpu_fixed)
     if rank == 0:
         print(json.dumps(line))
     if world > 1:
@@ -846,6 +919,41 @@ def run_rq(args, cfg):
     return 0
 
 
+ALL_CONFIGS = ("tiny", "1m", "10m256", "10m512", "100m")
+
+
+def run_all_configs(args):
+    """Every configuration in its own process (the index and its layouts of
+    one configuration leave the device before the next is built): each
+    prints its own benchmark line, then one summary line with per_config."""
+    per = {}
+    for name in ALL_CONFIGS:
+        cmd = [sys.executable, os.path.abspath(__file__), "--config", name, "--steps",
+               str(args.steps), "--warmup", str(args.warmup), "--cpu-seconds", str(args.cpu_seconds),
+               "--scan-path", args.scan_path, "--skip-calibration"]
+        if args.skip_e2e:
+            cmd.append("--skip-e2e")
+        if args.skip_cpu_baseline:
+            cmd.append("--skip-cpu-baseline")
+        r = subprocess.run(cmd, capture_output=True, text=True)
+        lines = [x for x in r.stdout.splitlines() if x.startswith("{")]
+        if r.returncode != 0 or not lines:
+            per[name] = {"error": f"rc={r.returncode}: {r.stderr.strip().splitlines()[-1:]}"}
+            continue
+        print(lines[-1], flush=True)
+        b = json.loads(lines[-1])
+        roof = b.get("roofline") or {}
+        per[name] = {"value": b["value"], "ms_per_step": b["ms_per_step"],
+                     "fixed_probe_value": b["fixed_probe"]["value"],
+                     "speedup_vs_fixed": b["speedup_vs_fixed"], "mean_probes": b["mean_probes"],
+                     "top_kernel": roof.get("kernel"), "frac": roof.get("frac"),
+                     "roofline_unit": roof.get("unit"), "parity": b.get("parity"),
+                     "clocks": b.get("clocks")}
+    print(json.dumps({"all_configs": True, "metric": METRIC, "unit": "queries/s",
+                      "steps": args.steps, "warmup": args.warmup, "per_config": per}))
+    return 0 if all("error" not in v for v in per.values()) else 1
+
+
 def run_ncu_case(args, cfg):
     """One search call on the benchmark workload, nothing else on the GPU after it."""
     import paper_2608_03199_gb300 as sieve
@@ -873,6 +981,8 @@ def main():
     args = parse()
     cfg = synth.CONFIGS[args.config]
     world, rank, local = dist_setup(args.gpus)
+    if args.all_configs:
+        return run_all_configs(args)
     if args.ncu_case:
         return run_ncu_case(args, cfg)
     if args.sweep:

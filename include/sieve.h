@@ -252,13 +252,24 @@ sieve_status sieve_search_workspace_size(const sieve_index_view *ix, int64_t nq,
  *   stats      host (nullable): counters; non-NULL synchronizes `stream`
  * nq = 0 is valid and does nothing.  A list_offsets table that is not a
  * partition of [0, n), or an order entry outside [0, nlist), is detected on
- * the device: nothing past it is searched and, with stats, the call returns
- * SIEVE_EINVAL (without stats the outputs are then undefined). */
+ * the device: nothing past it is searched and the outputs are undefined.
+ * Such a device-side error (SIEVE_EINVAL, or SIEVE_ETIMEOUT / SIEVE_ELIMIT)
+ * lands in the status word of the workspace's control block.  The call
+ * returns it when it synchronizes anyway: with stats, or with host-driven
+ * rounds (p->loop = 1).  Otherwise the call returns as soon as the work is
+ * enqueued, and sieve_search_status reads the word afterwards. */
 sieve_status sieve_search(const sieve_index_view *ix, const float *Q, int64_t nq,
                           const int64_t *query_ids, const int32_t *order,
                           const sieve_params *p, int64_t *out_ids, float *out_scores,
                           int32_t *out_count, int32_t *out_probes, sieve_stats *stats,
                           void *ws, size_t ws_bytes, void *stream);
+
+/* The device status word of the last search enqueued with workspace ws
+ * (sieve_search, or sieve_rq_search, whose workspaces start with the same
+ * control block): 0, or the SIEVE_E* code the device recorded.  Copies the
+ * word to *status (host) on `stream` and synchronizes `stream`, so call it
+ * on the search's stream.  SIEVE_EINVAL for a null or misaligned ws. */
+sieve_status sieve_search_status(const void *ws, size_t ws_bytes, int32_t *status, void *stream);
 
 /* sieve_search with the queries and results in HOST memory: copies Q (and
  * query_ids) to device staging inside the workspace, searches, copies the
@@ -270,7 +281,9 @@ sieve_status sieve_search(const sieve_index_view *ix, const float *Q, int64_t nq
  * `stream` as soon as the chunk has landed, so the upload overlaps the
  * ranking (with profile = 1 the upload is one copy and the ranking runs
  * inside the search).  Q_host should be page-locked for the copies to be
- * asynchronous. */
+ * asynchronous.
+ * As the call synchronizes, it returns a device-side error (see
+ * sieve_search) with or without stats. */
 sieve_status sieve_search_host(const sieve_index_view *ix, const float *Q_host, int64_t nq,
                                const int64_t *query_ids_host, const sieve_params *p,
                                int64_t *out_ids_host, float *out_scores_host,
@@ -292,9 +305,16 @@ sieve_status sieve_search_host(const sieve_index_view *ix, const float *Q_host, 
  *   - A call whose scratch need (sieve_search_workspace_size with
  *     host_io = 0) exceeds SIEVE_NOALLOC_SCRATCH_BYTES returns
  *     SIEVE_ESCRATCH and touches nothing.
- *   - The first call on a device looks up the array's device address on that
- *     device (cudaGetSymbolAddress); make that first call before any stream
- *     capture begins.
+ *   - Every call looks the array's device address up on the current device
+ *     (cudaGetSymbolAddress; the address is not cached, so it stays valid
+ *     across a cudaDeviceReset).  Under CUDA's lazy module loading the first
+ *     call on a device is the one that loads the library's device code and
+ *     so commits the array: that call can fail with an out-of-memory
+ *     SIEVE_ECUDA.  A caller that must not fail later makes one small call
+ *     at start-up, before any stream capture begins.
+ *   - The rounds are host-driven and synchronize `stream`, so a device-side
+ *     error (SIEVE_EINVAL for an order entry outside [0, nlist),
+ *     SIEVE_ETIMEOUT, SIEVE_ELIMIT) is returned with or without stats.
  *   - Every call on a device uses the same array and leaves its contents
  *     behind; each call initialises what it reads.  Calls that can overlap
  *     on the GPU (other host threads, other streams) race on the array and

@@ -98,6 +98,7 @@ _SIGNATURES = {
                                  C.c_void_p, C.POINTER(ParamsC), C.c_void_p, C.c_void_p,
                                  C.c_void_p, C.c_void_p, C.POINTER(StatsC), C.c_void_p,
                                  C.c_size_t, C.c_void_p]),
+    "sieve_search_status": (C.c_int32, [C.c_void_p, C.c_size_t, C.POINTER(C.c_int32), C.c_void_p]),
     "sieve_search_host": (C.c_int32, [C.POINTER(IndexViewC), C.c_void_p, C.c_int64, C.c_void_p,
                                       C.POINTER(ParamsC), C.c_void_p, C.c_void_p, C.c_void_p,
                                       C.c_void_p, C.POINTER(StatsC), C.c_void_p, C.c_size_t,
@@ -356,12 +357,15 @@ def _stats_dict(st):
 
 def search(index: Index, Q, tau, k, nprobe, W, lookahead=True, query_ids=None, order=None,
            max_items_per_round=0, loop=0, stats=False, profile=False, scan_path="auto",
-           workspace=None, out=None, stream=None):
+           workspace=None, out=None, stream=None, check=False):
     """SieveIVF search on device tensors (sieve_search).
 
     Returns (ids [nq][k] i64, scores [nq][k] f32, count [nq] i32, probes [nq] i32),
     plus a dict of counters when ``stats`` or ``profile`` (both synchronize the
-    stream; ``profile`` also times every kernel launch with CUDA events)."""
+    stream; ``profile`` also times every kernel launch with CUDA events).
+    ``check``: read the device status word after the call
+    (sieve_search_status, which synchronizes the stream) and raise on a
+    device-side error; stats and host-driven rounds check it anyway."""
     stats = stats or profile
     _need_cuda(Q, torch.float32, "Q", 2)
     if query_ids is not None:
@@ -387,9 +391,23 @@ def search(index: Index, Q, tau, k, nprobe, W, lookahead=True, query_ids=None, o
                               _ptr(ids), _ptr(scores), _ptr(count), _ptr(probes),
                               C.byref(st) if st is not None else None, _ptr(ws), ws.numel(),
                               _stream(stream)), "sieve_search")
+    if check and nq > 0:
+        _check(search_status(ws, stream), "sieve_search (device status)")
     if stats:
         return ids, scores, count, probes, _stats_dict(st)
     return ids, scores, count, probes
+
+
+def search_status(ws, stream=None) -> int:
+    """The device status word of the last search that used the workspace
+    tensor ``ws`` (sieve_search_status; synchronizes the stream): 0 or a
+    negative SIEVE_E* code."""
+    if isinstance(ws, Workspace):
+        ws = ws.buf
+    v = C.c_int32(0)
+    _check(lib().sieve_search_status(_ptr(ws), ws.numel(), C.byref(v), _stream(stream)),
+           "sieve_search_status")
+    return int(v.value)
 
 
 @dataclass

@@ -1,6 +1,7 @@
 // api.cu -- the C ABI of libsieve (declared in include/sieve.h): argument
 // checks, workspace layout, the device-resident round loop as a CUDA graph
 // with a WHILE conditional node, and the host-buffer variant.
+#include <cstddef>
 #include <cstring>
 #include <mutex>
 #include <vector>
@@ -449,6 +450,7 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
     const int blocks = scan_blocks_for(smem);
 
     float ms[SIEVE_NKERNELS] = {0};
+    int host_status = 0;   // host-driven rounds: the status word, read with every round's flag
     if (p->loop == 0 && !p->profile) {
         GraphKey key;
         std::memset(&key, 0, sizeof(key));
@@ -485,9 +487,13 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
             }));
         for (;;) {
             SIEVE_CUDA(launch_round(a, smem, blocks, 0, 0, st, p->profile ? ev.e : nullptr));
-            int more = 0;
-            SIEVE_CUDA(cudaMemcpyAsync(&more, &a.ctl->more, sizeof(int), cudaMemcpyDeviceToHost, st));
+            // the status word and the loop flag are adjacent in the control block
+            static_assert(offsetof(Ctl, more) == offsetof(Ctl, status) + sizeof(int), "");
+            int word[2] = {0, 0};
+            SIEVE_CUDA(cudaMemcpyAsync(word, &a.ctl->status, sizeof(word), cudaMemcpyDeviceToHost, st));
             SIEVE_CUDA(cudaStreamSynchronize(st));
+            host_status = word[0];
+            const int more = word[1];
             if (p->profile) {
                 const int slot[kRoundKernels] = {SIEVE_K_ISSUE, SIEVE_K_BUCKET, SIEVE_K_SCATTER,
                                                  SIEVE_K_SCAN_TC, SIEVE_K_SCAN, SIEVE_K_MERGE,
@@ -531,7 +537,9 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
         if (a.tc_min == 1) stats->kernel_launches[SIEVE_K_SCAN] = 0;
         if (c.status != 0) return c.status;
     }
-    return SIEVE_OK;
+    // host-driven rounds synchronize every round anyway: a device error is
+    // returned even without stats (in graph mode sieve_search_status reads it)
+    return host_status != 0 ? host_status : SIEVE_OK;
 }
 
 sieve_status check_search(const sieve_index_view *ix, const float *Q, int64_t nq,
@@ -692,6 +700,19 @@ sieve_status sieve_search(const sieve_index_view *ix, const float *Q, int64_t nq
     return search_device(ix, Q, nq, query_ids, order, p, out_ids, out_scores, out_count,
                          out_probes, stats, static_cast<unsigned char *>(ws), L,
                          static_cast<cudaStream_t>(stream));
+}
+
+sieve_status sieve_search_status(const void *ws, size_t ws_bytes, int32_t *status, void *stream) {
+    if (!ws || !status || (reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < sizeof(Ctl))
+        return SIEVE_EINVAL;
+    // the control block opens every search layout (make_layout's first part)
+    const Ctl *ctl = static_cast<const Ctl *>(ws);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    int32_t v = 0;
+    SIEVE_CUDA(cudaMemcpyAsync(&v, &ctl->status, sizeof(v), cudaMemcpyDeviceToHost, st));
+    SIEVE_CUDA(cudaStreamSynchronize(st));
+    *status = v;
+    return SIEVE_OK;
 }
 
 // ---------------------------------------------------------------------------
@@ -868,14 +889,16 @@ sieve_status sieve_search_host(const sieve_index_view *ix, const float *Q_host, 
     SIEVE_CUDA(cudaMemcpyAsync(out_scores_host, dsc, (size_t)nq * p->k * 4, cudaMemcpyDeviceToHost, st));
     SIEVE_CUDA(cudaMemcpyAsync(out_count_host, dcnt, (size_t)nq * 4, cudaMemcpyDeviceToHost, st));
     SIEVE_CUDA(cudaMemcpyAsync(out_probes_host, dpr, (size_t)nq * 4, cudaMemcpyDeviceToHost, st));
-    int rank_status = 0;
+    int rank_status = 0, search_status = 0;
     SIEVE_CUDA(cudaMemcpyAsync(&rank_status, dstatus, sizeof(int), cudaMemcpyDeviceToHost, st));
+    SIEVE_CUDA(cudaMemcpyAsync(&search_status, &reinterpret_cast<const Ctl *>(w + L.ctl)->status,
+                               sizeof(int), cudaMemcpyDeviceToHost, st));
     SIEVE_CUDA(cudaStreamSynchronize(st));
     if (stats && nchunks > 0) {   // ran here
         stats->kernel_launches[SIEVE_K_RANK] = rank_launches;
         stats->kernel_launches[SIEVE_K_RANK_MMA] = mma_launches;
     }
-    return rank_status != 0 ? rank_status : SIEVE_OK;
+    return rank_status != 0 ? rank_status : search_status != 0 ? search_status : SIEVE_OK;
 }
 
 // ---------------------------------------------------------------------------
@@ -1160,28 +1183,21 @@ sieve_status sieve_merge_shard_results(int32_t nshards, int64_t nq, int32_t k,
 namespace {
 
 constexpr size_t kNoallocScratchBytes = size_t(64) << 20;   // SIEVE_NOALLOC_SCRATCH_BYTES
-constexpr int kNoallocMaxDevices = 64;
+static_assert(kNoallocScratchBytes == SIEVE_NOALLOC_SCRATCH_BYTES,
+              "the header's scratch size and the array's must agree");
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocScratchBytes];
 
-std::mutex g_noalloc_mu;
-void *g_noalloc_ptr[kNoallocMaxDevices] = {};
-
-// Device address of the scratch array on the current device.  Host code only
-// sees a host-side stand-in under the array's name, so the address is asked
-// of the runtime once per device (with that device current) and kept.
+// Device address of the scratch array on the current device.  In host code
+// the array's name is only a host-side stand-in, so the address is asked of
+// the runtime, with the device current, on every call: a lookup in the
+// loaded module, no allocation.  Nothing is cached, so a context that was
+// destroyed and created again (cudaDeviceReset) gets the new address.
 sieve_status noalloc_scratch(void **out) {
-    int dev = 0;
-    SIEVE_CUDA(cudaGetDevice(&dev));
-    if (dev < 0 || dev >= kNoallocMaxDevices) return SIEVE_EUNSUPPORTED;
-    std::lock_guard<std::mutex> lk(g_noalloc_mu);
-    if (!g_noalloc_ptr[dev]) {
-        void *p = nullptr;
-        cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-        if (e != cudaSuccess || !p) return cuda_fail(e != cudaSuccess ? e : cudaErrorInvalidSymbol);
-        g_noalloc_ptr[dev] = p;
-    }
-    *out = g_noalloc_ptr[dev];
+    void *p = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess || !p) return cuda_fail(e != cudaSuccess ? e : cudaErrorInvalidSymbol);
+    *out = p;
     return SIEVE_OK;
 }
 

@@ -13,6 +13,29 @@ def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU (runs through the C ABI)")
 
 
+def pytest_terminal_summary(terminalreporter):
+    """The divergence count of every parity comparison of the session: queries
+    identical to the oracle, queries that differ where the oracle's fragility
+    tags put a decision within 1e-5 of a rounding flip (allowed), and
+    queries that differ without one (unexplained, which fail their test)."""
+    parity = sys.modules.get("parity")
+    reports = getattr(parity, "REPORTS", None)
+    if not reports:
+        return
+    tr = terminalreporter
+    tr.section("parity against the oracle")
+    tot = [0, 0, 0, 0]
+    worst = 0.0
+    for label, nq, exact, allowed, unexplained, err in reports:
+        tr.write_line(f"{label}: {nq} queries, {exact} exact, {allowed} allowed, "
+                      f"{unexplained} unexplained, max score err {err:.2e}")
+        for i, v in enumerate((nq, exact, allowed, unexplained)):
+            tot[i] += v
+        worst = max(worst, err)
+    tr.write_line(f"total: {len(reports)} comparisons, {tot[0]} queries, {tot[1]} exact, "
+                  f"{tot[2]} allowed, {tot[3]} unexplained, max score err {worst:.2e}")
+
+
 @pytest.fixture(scope="session")
 def tiny():
     """The tiny workload (20K x 64, nlist 64, 1K queries), host numpy arrays."""

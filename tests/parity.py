@@ -8,11 +8,24 @@ a k-th / (k+1)-th result gap below TOL, or two centroid scores closer than TOL
 counted and reported; every other query must match exactly, with result
 scores within TOL (absolute).
 """
+import os
+
 import numpy as np
 
 import oracle
 
 TOL = 1e-5
+
+# every report checked in this process: (label, queries, exact, allowed,
+# unexplained, max score error); the test session prints them at its end
+REPORTS = []
+
+
+def summary(rep):
+    """One line: how many queries matched exactly, how many differed with a
+    fragility tag (allowed), how many differed without one."""
+    return (f"{rep['queries']} queries: {rep['exact']} exact, {rep['allowed']} allowed (tagged), "
+            f"{len(rep['unexplained'])} unexplained, max score err {rep['max_score_err']:.2e}")
 
 
 def compare(gpu, ref, index, Q, qids, tau, k, nprobe, order, threads=None, rq=None):
@@ -47,7 +60,11 @@ def compare(gpu, ref, index, Q, qids, tau, k, nprobe, order, threads=None, rq=No
     }
 
 
-def assert_parity(rep, max_allowed_frac=0.01):
+def assert_parity(rep, max_allowed_frac=0.01, label=None):
+    label = label or os.environ.get("PYTEST_CURRENT_TEST", "").split(" ")[0] or "parity"
+    REPORTS.append((label, rep["queries"], rep["exact"], rep["allowed"], len(rep["unexplained"]),
+                    rep["max_score_err"]))
+    print(f"parity {label}: {summary(rep)}")
     assert len(rep["unexplained"]) == 0, f"unexplained mismatches at queries {rep['unexplained'][:20]}"
     assert rep["max_score_err"] <= TOL, rep
     assert rep["pad_ok"], rep

@@ -57,6 +57,12 @@ def test_host_only_calls_without_gpu():
     v.d = 62
     assert lib.sieve_search_workspace_size(ctypes.byref(v), 100, ctypes.byref(p), 0,
                                            ctypes.byref(n)) == -1
+    # the status query rejects a missing or misaligned workspace before any copy
+    st = ctypes.c_int32(5)
+    assert lib.sieve_search_status(None, 1 << 20, ctypes.byref(st), None) == -1
+    assert lib.sieve_search_status(ctypes.c_void_p(16), 1 << 20, ctypes.byref(st), None) == -1
+    assert lib.sieve_search_status(ctypes.c_void_p(256), 1 << 20, None, None) == -1
+    assert st.value == 5
 
 
 def test_scan_path_values_without_gpu():

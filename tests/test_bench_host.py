@@ -49,7 +49,35 @@ def test_cpu_baseline_times_both_modes():
     sample, with the thread count reported."""
     wl = synth.make_workload("tiny", device="cpu")
     cfg = wl["cfg"]
-    out = bench.cpu_baseline(bench.host_arrays(wl), cfg, 0.5)
+    out, parity = bench.cpu_baseline(bench.host_arrays(wl), cfg, 0.5)
     assert out["kind"] == "oracle" and out["cores"] >= 1 and out["value"] > 0
     assert out["fixed_probe"]["value"] > 0
     assert f"W={cfg.nprobe}" in out["fixed_probe"]["sample"]
+    assert isinstance(out["cpu_model"], str) and out["cpu_model"]
+    assert parity == {}
+
+
+def test_parity_sample_counts_divergences():
+    """The bench's parity record: the oracle's own results compare as all
+    exact; a planted wrong id and a wrong probe count on two queries are
+    counted as unexplained (their decisions sit far from any flip)."""
+    wl = synth.make_workload("tiny", device="cpu")
+    cfg = wl["cfg"]
+    w = bench.host_arrays(wl)
+    idx = {k: w[k] for k in ("X", "ids", "assign", "centroids")}
+    ref = oracle.search(idx, w["Q"], cfg.tau, cfg.k, cfg.nprobe, cfg.W, qids=w["qids"])
+    got = [ref["ids"].copy(), ref["scores"].astype(np.float32), ref["count"].copy(),
+           ref["probes"].copy()]
+    rep = bench.parity_sample(oracle, idx, w["Q"], w["qids"], cfg, cfg.W, ref, tuple(got))
+    assert rep["queries"] == len(w["Q"]) and rep["exact"] == rep["queries"]
+    assert rep["allowed"] == 0 and rep["unexplained"] == 0 and rep["max_score_err"] < 1e-7
+    # two planted mistakes: a query's probe count off by one, another's first id
+    tg, kg, cg = oracle.fragility(idx, w["Q"], cfg.tau, cfg.k, cfg.nprobe,
+                                  oracle.rank(w["Q"], w["centroids"], cfg.nprobe),
+                                  ref["probes"] + 1, qids=w["qids"])
+    far = np.flatnonzero((tg > 1e-3) & (kg > 1e-3) & (cg > 1e-3) & (ref["count"] > 0))
+    a, b = far[0], far[1]
+    got[3][a] += 1
+    got[0][b, 0] = 10**9
+    rep = bench.parity_sample(oracle, idx, w["Q"], w["qids"], cfg, cfg.W, ref, tuple(got))
+    assert rep["exact"] == rep["queries"] - 2 and rep["unexplained"] == 2

@@ -453,3 +453,30 @@ def test_wide_rows_fall_back_and_match(dev):
     assert gidx.tc_rows is not None
     for path in ("tensor", "auto"):
         check(w, gidx, w["Q"], w["qids"], cfg.tau, cfg.k, cfg.nprobe, cfg.W, 1, scan_path=path)
+
+
+def test_device_error_reported_without_stats(tiny, g_tiny, dev):
+    """An order entry outside [0, nlist) is caught on the device.  In graph
+    mode without stats the call returns at once; sieve_search_status then
+    reads SIEVE_EINVAL from the workspace, and search(check=True) raises.
+    Host-driven rounds return it directly.  A correct call on the same
+    workspace afterwards reports 0."""
+    c = tiny["cfg"]
+    Q = torch.from_numpy(tiny["Q"][:200]).to(dev)
+    qids = torch.from_numpy(tiny["qids"][:200]).to(dev)
+    order = sieve.rank_partitions(g_tiny, Q, c.nprobe)
+    bad = order.clone()
+    bad[7, 3] = -1
+    ws = sieve.Workspace()
+    sieve.search(g_tiny, Q, c.tau, c.k, c.nprobe, c.W, query_ids=qids, order=bad, workspace=ws)
+    assert sieve.search_status(ws) == -1
+    with pytest.raises(sieve.SieveError) as ei:
+        sieve.search(g_tiny, Q, c.tau, c.k, c.nprobe, c.W, query_ids=qids, order=bad,
+                     workspace=ws, check=True)
+    assert ei.value.status == -1
+    with pytest.raises(sieve.SieveError):
+        sieve.search(g_tiny, Q, c.tau, c.k, c.nprobe, c.W, query_ids=qids, order=bad,
+                     workspace=ws, loop=1)
+    sieve.search(g_tiny, Q, c.tau, c.k, c.nprobe, c.W, query_ids=qids, order=order, workspace=ws,
+                 check=True)
+    assert sieve.search_status(ws) == 0

@@ -14,6 +14,7 @@ import pytest
 
 import oracle
 import test_oracle_calibration as K
+import test_oracle_fragility as F
 import test_oracle_rq as R
 import test_oracle_search as S
 import test_oracle_stopping as T
@@ -51,6 +52,17 @@ MUTATIONS = [
      "const double delta = mx / top;"),
     ("query rotated by the untransposed matrix", "acc += P[(int64_t)j * d + t] * (double)q[j];",
      "acc += P[(int64_t)t * d + j] * (double)q[j];"),
+    # the divergence tagger: which mismatches the parity tests excuse
+    ("k-th gap taken one rank early",
+     "kth_gap[i] = (t.n > k) ? fin[k - 1].score - fin[k].score : INFINITY;",
+     "kth_gap[i] = (t.n > k) ? fin[k > 1 ? k - 2 : 0].score - fin[k - 1].score : INFINITY;"),
+    ("centroid gap over nprobe ranks, not nprobe + 1",
+     "int64_t top = (int64_t)nprobe + 1 < nlist ? (int64_t)nprobe + 1 : nlist;",
+     "int64_t top = (int64_t)nprobe < nlist ? (int64_t)nprobe : nlist;"),
+    ("tau gap counts the query's own row",
+     "if (qids && ids[row] == qids[i])\n                        continue;\n"
+     "                    double s = rq ? rq_estimate",
+     "double s = rq ? rq_estimate"),
 ]
 
 
@@ -72,6 +84,12 @@ def _pins(tiny, deep):
         lambda: R.test_estimator_error_shrinks_with_bits_and_is_unbiased(tiny),
         lambda: R.test_quantized_search_approaches_exact(deep),
         lambda: R.test_rows_at_their_centroid_and_bounds(tiny),
+        lambda: F.test_hand_built_gaps(F.hand_index()),
+        lambda: F.test_upto_below_nprobe_limits_the_rows(F.hand_index()),
+        lambda: F.test_fewer_than_k_plus_one_qualifiers_give_infinity(F.hand_index()),
+        F.test_exact_ties_give_zero_gaps,
+        lambda: F.test_nlist_at_most_nprobe_plus_one(F.hand_index()),
+        lambda: F.test_tags_equal_numpy_restatement(deep, 3),
     ]
 
 
