@@ -197,6 +197,20 @@ def uses_screen(args, cfg, W, bulk):
                      (args.scan_path == "auto" and min(W, cfg.nprobe) >= 16))
 
 
+def rank_passes(cfg, bulk):
+    """(contraction passes of the tensor-core ranking, products per score of
+    the first pass): more than 2,048 centroids with 2 nprobe to 2,048 groups of
+    64 (or 32) take a first pass of group maxima, on the screen (one product)
+    with the tensor-core layout (d <= 256), else with three products."""
+    if cfg.nlist <= 2048:
+        return 1, 0
+    for g in (64, 32):
+        ng = -(-cfg.nlist // g)
+        if 2 * cfg.nprobe <= ng <= 2048:
+            return 2, (1 if bulk and cfg.d <= 256 else 3)
+    return 1, 0
+
+
 def roofline(prof, cfg, dev, bulk=True, rank_on_tensor=True, rq=False, screen=False):
     """Roofline entry for the kernel with the largest share of the step.
     bulk: the index carries the tensor-core layout, so the tensor-core scan
@@ -266,22 +280,27 @@ def roofline(prof, cfg, dev, bulk=True, rank_on_tensor=True, rq=False, screen=Fa
                    hbm_view={"achieved_gbs": bytes_ / launches / (ms_per_launch * 1e-3) / 1e9,
                              "peak_gbs": hbm})
     elif top == "rank_mma":
-        # the score contraction of the ranking alone (tensor cores, three fp16
-        # products per score); its algorithmic work is every query-centroid
-        # score once, spread over its launches (a maxima pass and a keeping
-        # pass each compute every score when the ranking has no score table)
-        name = "k_rank_bulk" if bulk else "k_rank_tc"
+        # the score contraction of the ranking (tensor cores, three fp16
+        # products per score in the pass that keeps candidates); its
+        # algorithmic work is every query-centroid score once, spread over
+        # all its launches: with many centroids a first pass of group maxima
+        # (one product per score, on the screen, with the tensor-core layout)
+        # sets each query's starting threshold
+        passes, first_products = rank_passes(cfg, bulk)
+        name = "k_rank_bulk" + (" + k_rank_screen" if passes == 2 and bulk else "") if bulk \
+            else "k_rank_tc"
         flops = 2.0 * cfg.nq * cfg.nlist * d
         ach = flops / launches / (ms_per_launch * 1e-3) / 1e12
-        ng = -(-cfg.nlist // 32)   # 32-centroid groups
-        # no score table (d <= 128 under the group threshold): two passes
-        passes = 2 if (d <= 128 and cfg.nlist > 2048 and cfg.nprobe <= ng <= 2048) else 1
+        # K steps of 16 issued (the zero padding of the last K-block is skipped)
+        d_mma = 16 * -(-d // 16)
         out.update(kernel=name, bound="tensor", achieved=ach, peak=f16_tflops / 3,
                    unit="TFLOP/s", frac=ach / (f16_tflops / 3),
                    peak_source=(f"fp16 split: three kind::f16 MMAs per score; fp16 dense peak "
                                 f"{f16_tflops:.0f} TFLOP/s = measured bf16 cuBLAS burst (of "
-                                f"measured), a third of it"),
-                   passes=passes, tensor_pipe_tflops=3 * passes * ach,
+                                f"measured), a third of it; achieved = every score once over "
+                                f"the summed time of all contraction launches"),
+                   passes=passes,
+                   tensor_pipe_tflops=(3 + first_products) * ach * d_mma / d,
                    rank_select_ms=km.get("rank_select"))
     elif top == "rank_select":
         out.update(kernel="ranking selection (k_select / k_compact_final)", bound="alu",

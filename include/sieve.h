@@ -216,9 +216,12 @@ sieve_status sieve_build_tc_layout(const sieve_index_view *ix, void *tc_rows,
  * centroids with the largest inner product, best first; equal scores rank
  * the lower centroid id first.  Scores come from the tensor cores with the
  * three-product fp16 split (each fp32 value = hi + lo fp16, scaled by 256),
- * accurate to a few 1e-7 on unit vectors; they go through a score table of at
- * most 512 MiB per chunk of queries in the workspace, and a warp per
- * (query, 2,048 centroids) keeps the best nprobe, level by level.
+ * accurate to a few 1e-7 on unit vectors.  One contraction pass: the
+ * epilogue keeps, per query, a running threshold (a histogram of the scores
+ * it has kept) and appends only scores that reach it to a candidate list in
+ * the workspace; a warp per query then takes the exact nprobe best of its
+ * list.  A list that overflows (many equal scores) sends its query to an
+ * exact FP32 ranking.
  *   Q        device [nq][d] fp32
  *   order    device [nq][nprobe] int32 out, 0-based centroid ids
  *   cscores  device [nq][nprobe] fp32 out (nullable): the matching scores

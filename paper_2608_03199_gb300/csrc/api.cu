@@ -526,14 +526,19 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
         const int per_round[] = {SIEVE_K_ISSUE, SIEVE_K_BUCKET, SIEVE_K_SCATTER, SIEVE_K_SCAN,
                                  SIEVE_K_MERGE, SIEVE_K_ROUND_END};
         stats->kernel_launches[SIEVE_K_RANK] =
-            !with_rank ? 0 : rank_tc ? rank_tc_launches(a.nq, a.nlist, a.nprobe, a.d) : 1;
+            !with_rank ? 0
+            : rank_tc ? rank_tc_launches(a.nq, a.nlist, a.nprobe, a.d, 0,
+                                         a.tc_cent && rank_bulk_stages(a.d) > 0)
+                      : 1;
         stats->kernel_launches[SIEVE_K_INIT] = a.tc_screen ? 2 : 1;   // + the query norms
         stats->kernel_launches[SIEVE_K_FINALIZE] = 1;
         for (int slot : per_round) stats->kernel_launches[slot] = c.round;
         stats->kernel_launches[SIEVE_K_SCAN_TC] = a.tc_min > 0 ? c.round : 0;
         stats->kernel_launches[SIEVE_K_RQ_ROTATE] = a.rq ? 1 : 0;
         stats->kernel_launches[SIEVE_K_RANK_MMA] =
-            with_rank && rank_tc ? rank_tc_mma_launches(a.nq, a.nlist, a.nprobe, a.d) : 0;
+            with_rank && rank_tc ? rank_tc_mma_launches(a.nq, a.nlist, a.nprobe, a.d, 0,
+                                                         a.tc_cent && rank_bulk_stages(a.d) > 0)
+                                  : 0;
         if (a.tc_min == 1) stats->kernel_launches[SIEVE_K_SCAN] = 0;
         if (c.status != 0) return c.status;
     }
@@ -875,12 +880,14 @@ sieve_status sieve_search_host(const sieve_index_view *ix, const float *Q_host, 
             SIEVE_CUDA(enqueue_rank_tc(dQ + q0 * ix->d, n, ix->centroids, ix->nlist, ix->d, p->nprobe,
                                        dorder + q0 * p->nprobe, nullptr,
                                        reinterpret_cast<float *>(w + L.rank_scratch), dstatus, st,
-                                       static_cast<const unsigned char *>(ix->tc_centroids)));
+                                       static_cast<const unsigned char *>(ix->tc_centroids),
+                                       nullptr, nq));
         else
             SIEVE_CUDA(enqueue_rank(dQ + q0 * ix->d, n, ix->centroids, ix->nlist, ix->d, p->nprobe,
                                     dorder + q0 * p->nprobe, nullptr, st));
-        rank_launches += rank_tc ? rank_tc_launches(n, ix->nlist, p->nprobe, ix->d) : 1;
-        mma_launches += rank_tc ? rank_tc_mma_launches(n, ix->nlist, p->nprobe, ix->d) : 0;
+        const bool bulk = ix->tc_centroids && rank_bulk_stages(ix->d) > 0;
+        rank_launches += rank_tc ? rank_tc_launches(n, ix->nlist, p->nprobe, ix->d, nq, bulk) : 1;
+        mma_launches += rank_tc ? rank_tc_mma_launches(n, ix->nlist, p->nprobe, ix->d, nq, bulk) : 0;
     }
     rc = search_device(ix, dQ, nq, dqids, nchunks ? dorder : nullptr, p, dids, dsc, dcnt, dpr, stats,
                        w, L, st);

@@ -1,39 +1,32 @@
 // rank_tc.cu -- centroid ranking on the tcgen05 tensor cores (Sec. 2.3,
 // Sec. 4.1: P_i = the nprobe centroids with the largest inner product with
-// q_i, best first, equal scores by lower centroid id), for any nlist.
+// q_i, best first, equal scores by lower centroid id), for any nlist, in one
+// contraction pass: no score table, no second pass.
 //
-// Per chunk of queries:
 //   k_rank_bulk / k_rank_tc  the tensor-core contraction (tc_bulk.cuh with the
 //              centroids' tensor-core layout, else the converter pipeline of
-//              tc_pipeline.cuh): a tile is 128 consecutive queries (A rows)
-//              against one range of kRankRange centroids (B rows, 128 per
-//              chunk); each epilogue thread owns one query's scores and stores
-//              them into a score table, or only the maxima of 32-centroid
-//              groups, or only the scores that reach the query's threshold
-//   k_select   one warp per (query, segment of at most kSelectSeg entries):
-//              the segment's best min(nprobe, size) entries, sorted by
-//              (score desc, id asc): a threshold refined bit by bit over the
-//              keys in registers picks exactly that many, and a bitonic
-//              network in registers sorts them.  With nlist <= kSelectSeg one
-//              segment gives the order directly.
-// More centroids: the nprobe-th largest of the 32-centroid group maxima is a
-// threshold that at least nprobe scores reach (k_group_threshold); the scores
-// that reach it are compacted per 2,048-centroid range (from the table by
-// k_compact_seg, or kept by a second contraction when d <= 128) and one warp
-// per query selects and sorts the nprobe best of them (k_compact_final).  A
-// query whose candidates overflow their slots is listed and finished exactly:
-// by levels of k_select over its table row (the nprobe best of a set lie among
-// the nprobe best of each of its parts), or by the FP32 ranking of
-// rank_kernel.cu when there is no table.
+//              tc_pipeline.cuh).  A tile is 128 consecutive queries (A rows)
+//              against one range of centroids (B rows, 128 per chunk, in
+//              increasing id order).  Each epilogue thread owns one query and
+//              streams its scores: a 256-bin histogram of the scores it has
+//              kept (shared memory) gives a running threshold -- the lower edge
+//              of the highest bin such that at least nprobe kept scores lie in
+//              it or above -- and a score is appended to the query's candidate
+//              list only when it reaches that threshold.  A score below it has
+//              nprobe larger ones already, so it cannot be among the nprobe best.
+//   k_rank_final  one warp per query: the candidates of its ranges that reach
+//              their final thresholds, the exact nprobe best of them by (score
+//              desc, id asc), sorted.  The lists are in id order, so among equal
+//              scores the first taken are the lowest ids.
+// A query whose list overflowed (many equal scores, or an adversarial order)
+// is finished by the exact FP32 ranking of rank_kernel.cu.
+#include <cmath>
 #include <vector>
 
 #include "tc_bulk.cuh"
 #include "tc_pipeline.cuh"
 
 namespace sieve {
-
-constexpr int64_t kRankRange = 2048;   // centroids per tile (a multiple of 128)
-constexpr int kSelectSeg = 2048;       // entries per selecting warp (64 per lane)
 
 // selection: monotone map of fp32 to uint32 (larger float -> larger key); -0
 // is mapped as +0 so that equal scores have equal keys
@@ -47,6 +40,28 @@ __device__ __forceinline__ float key_score(uint32_t k) {
     return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
 }
 
+// Running-threshold histogram: 256 bins of width 1/128 over scores in
+// [-1, 1); scores outside fall into the end bins.  In raw accumulator units
+// (scores x 2^16) a bin is 512 wide, so bin and edge are exact.
+constexpr int kRankBins = 256;
+constexpr int kRankBinStride = 260;   // bytes per query: 4-byte words offset by one bank per slot
+constexpr size_t kRankEpiBytes = (size_t)tcp::kM * kRankBinStride;
+
+__device__ __forceinline__ int rank_bin(float raw) {
+    const float t = fminf(fmaxf(raw * (1.f / 512.f), -129.f), 128.f);
+    const int b = __float2int_rd(t) + kRankBins / 2;
+    return b < 0 ? 0 : (b > kRankBins - 1 ? kRankBins - 1 : b);
+}
+
+// lower edge of a bin in raw units; bin 0 takes everything
+__device__ __forceinline__ float rank_edge_raw(int b) {
+    return b == 0 ? -__int_as_float(0x7f800000) : (float)(b - kRankBins / 2) * 512.f;
+}
+
+// What the ranking contraction's epilogue does with a query's scores.
+constexpr int kRankGroupMax = 0;   // the maximum of each group of `group` centroids
+constexpr int kRankStream = 1;     // the scores that reach the running threshold
+constexpr int kRankDense = 2;      // every score (ids implicit: the list position)
 
 struct RankArgs {
     const float *Q;
@@ -54,28 +69,26 @@ struct RankArgs {
     const float *C;
     int64_t nlist;
     int d;
-    float *scores;   // [nq][ld] score table
-    int64_t ld;      // row stride of the table, a multiple of 32
     int *status;     // nullable: where a bounded wait that gives up is reported
     const unsigned char *tc_cent;   // tensor-core layout of the centroids (bulk path)
-    float *gmax;     // nullable: [nq][gld] maxima of each 32-centroid group
+    int nprobe;
+    int nranges;     // centroid ranges per query tile
+    int64_t range_len;   // centroids per range, a multiple of 128
+    int cap;         // list slots per (query, range)
+    float *list_s;   // [nq][nranges][cap] candidate scores, in id order
+    int32_t *list_i; //                    and their centroid ids (not kRankDense)
+    int *list_n;     // [nq][nranges] candidates offered (above cap: the list overflowed)
+    float *list_edge;   // [nq][nranges] the final threshold score (-inf: none)
+    const float *init_edge;   // kRankStream, nullable: [nq] starting threshold (score units)
+    float *gmax;     // kRankGroupMax: [nq][gld] group maxima (score units)
     int64_t gld;
-    int mode;                // kRankTable, kRankMax or kRankKeep
-    const uint32_t *lkey;    // kRankKeep: [nq] threshold keys
-    float *keep_s;           // kRankKeep: [nq][nranges][keep_cap] kept scores, per range
-    int32_t *keep_i;         //            and their centroid ids, in id order
-    int *keep_n;             //            [nq][nranges] how many each range had (even past keep_cap)
-    int keep_cap;            //            slots per range
+    int group;       // kRankGroupMax: centroids per group, 32 or 64
 };
-
-// what the ranking contraction's epilogue does with a query's scores:
-// store them all (and the group maxima when gmax is set), only the maxima of
-// each 32-centroid group, or only the scores that reach the query's threshold
-constexpr int kRankTable = 0, kRankMax = 1, kRankKeep = 2;
 
 __device__ int g_rank_status_sink;
 
-struct RankMode {
+template <int kMode>
+struct RankModeT {
     using Args = RankArgs;
     static constexpr int kN = 128;
     struct Tile {
@@ -84,19 +97,17 @@ struct RankMode {
         int64_t c0;    // first centroid of the tile's range
         int64_t nb;    // centroids in the range
     };
-    __device__ static int n_ranges(const Args &a) { return (int)ceil_div(a.nlist, kRankRange); }
-    __device__ static int num_tiles(const Args &a) { return (int)ceil_div(a.nq, tcp::kM) * n_ranges(a); }
+    __device__ static int num_tiles(const Args &a) { return (int)ceil_div(a.nq, tcp::kM) * a.nranges; }
     // every tile costs about the same: a static stride over the blocks
     __device__ static int *tile_counter(const Args &) { return nullptr; }
     __device__ static int d(const Args &a) { return a.d; }
     __device__ static int *status(const Args &a) { return a.status ? a.status : &g_rank_status_sink; }
     __device__ static Tile tile(const Args &a, int t) {
-        const int nr = n_ranges(a);
         Tile T;
-        T.q0 = (int64_t)(t / nr) * tcp::kM;
+        T.q0 = (int64_t)(t / a.nranges) * tcp::kM;
         T.ni = (int)(a.nq - T.q0 < tcp::kM ? a.nq - T.q0 : tcp::kM);
-        T.c0 = (int64_t)(t % nr) * kRankRange;
-        T.nb = a.nlist - T.c0 < kRankRange ? a.nlist - T.c0 : kRankRange;
+        T.c0 = (int64_t)(t % a.nranges) * a.range_len;
+        T.nb = a.nlist - T.c0 < a.range_len ? a.nlist - T.c0 : a.range_len;
         return T;
     }
     __device__ static const float *a_row(const Args &a, const Tile &T, int i) {
@@ -110,90 +121,176 @@ struct RankMode {
     }
     struct Epi {
         bool valid;
-        float *row;      // kRankTable: this query's table row from the range start
-        float *grow;     // this query's group maxima from the range start, or nullptr
-        float *ks;       // kRankKeep: this query's kept scores / ids for the range
-        int32_t *ki;
-        int kn;
-        int64_t keep_at; // kRankKeep: index of this (query, range) in keep_n
-        float thr_raw;   // kRankKeep: the threshold score x 2^16
-        __device__ void begin(const Args &a, const Tile &T, int slot, unsigned char *) {
+        float *ls;         // this (query, range)'s list
+        int32_t *li;
+        float *gm;         // kRankGroupMax: this query's group maxima
+        float gacc;        // kRankGroupMax: the running maximum of a 64-centroid group
+        int64_t at;        // index of this (query, range)
+        int n;             // candidates offered so far
+        int bin;           // histogram bin: scores below its lower edge are rejected
+        int above;         // kept scores in bins above it (saturated counts)
+        float init;        // the starting threshold, raw units
+        float edge;        // the threshold in force: max(init, lower edge of bin), raw units
+        unsigned char *h;  // this query's bin counts, saturating at 255
+        __device__ void begin(const Args &a, const Tile &T, int slot, unsigned char *smem) {
             valid = slot < T.ni;
             const int64_t q = T.q0 + slot;
-            row = (valid && a.mode == kRankTable) ? a.scores + q * a.ld + T.c0 : nullptr;
-            grow = (valid && a.gmax) ? a.gmax + q * a.gld + T.c0 / 32 : nullptr;
-            kn = 0;
-            ks = nullptr;
-            ki = nullptr;
-            thr_raw = 0.f;
-            keep_at = 0;
-            if (valid && a.mode == kRankKeep) {
-                keep_at = q * n_ranges(a) + T.c0 / kRankRange;
-                ks = a.keep_s + keep_at * a.keep_cap;
-                ki = a.keep_i + keep_at * a.keep_cap;
-                thr_raw = key_score(a.lkey[q]) * 65536.f;   // exact: a power-of-two scale
+            at = q * a.nranges + T.c0 / a.range_len;
+            n = 0;
+            bin = 0;
+            above = 0;
+            gacc = -__int_as_float(0x7f800000);
+            h = smem + (size_t)slot * kRankBinStride;
+            if constexpr (kMode == kRankStream) {
+                uint32_t *hw = reinterpret_cast<uint32_t *>(h);
+#pragma unroll
+                for (int i = 0; i < kRankBins / 4; ++i) hw[i] = 0u;
             }
+            init = (valid && a.init_edge) ? a.init_edge[q] * 65536.f : rank_edge_raw(0);
+            edge = init;
+            ls = valid ? a.list_s + at * a.cap : nullptr;
+            li = (valid && a.list_i) ? a.list_i + at * a.cap : nullptr;
+            gm = (valid && kMode == kRankGroupMax) ? a.gmax + q * a.gld + T.c0 / a.group : nullptr;
         }
-        // v holds the chunk's raw accumulator values: scores x 2^16
+        // v holds the chunk's raw accumulator values: scores x 2^16, for
+        // centroids T.c0 + col0 + j, j < ncol (warp-uniform)
         __device__ void chunk(const Args &a, const Tile &T, int64_t col0, const float (&v)[32], int ncol) {
-            if (!valid || ncol <= 0) return;
             constexpr float kS = 1.f / 65536.f;
-            if (row) {   // ld and the range start are multiples of 32: whole groups fit
-                float4 *dst = reinterpret_cast<float4 *>(row + col0);
+            if (ncol <= 0) return;   // a group past the range's end (warp-uniform)
+            if constexpr (kMode == kRankDense) {   // the range's scores in order; ids implicit
+                if (!valid) return;
+                float *dst = ls + col0;
+                if (ncol == 32) {   // cap and the range start are multiples of 32
 #pragma unroll
-                for (int j = 0; j < 8; ++j)
-                    dst[j] = make_float4(v[4 * j] * kS, v[4 * j + 1] * kS, v[4 * j + 2] * kS, v[4 * j + 3] * kS);
-            }
-            if (grow) {   // the group's maximum over its real columns only
-                float mx = v[0];
+                    for (int j = 0; j < 8; ++j)
+                        reinterpret_cast<float4 *>(dst)[j] = make_float4(
+                            v[4 * j] * kS, v[4 * j + 1] * kS, v[4 * j + 2] * kS, v[4 * j + 3] * kS);
+                } else {
 #pragma unroll
-                for (int j = 1; j < 32; ++j) mx = j < ncol ? fmaxf(mx, v[j]) : mx;
-                grow[col0 / 32] = mx * kS;
+                    for (int j = 0; j < 32; ++j)
+                        if (j < ncol) dst[j] = v[j] * kS;
+                }
+                n += ncol;
+                return;
             }
-            if (ks) {   // the scores that reach the threshold, in id order
-                // (a mask straight from the compares: some lane of a warp
-                // nearly always has a candidate in a group, so a maximum
-                // test first would not let the warp skip the group)
+            if (kMode == kRankStream && a.init_edge) {
+                // a starting threshold from the first pass: it already keeps
+                // only a little over nprobe scores, so no running histogram.
+                // The mask comes straight from the compares (some lane of a
+                // warp nearly always has a candidate in a group, so a maximum
+                // test first would not let the warp skip it)
                 unsigned m = 0;
+                if (valid) {
 #pragma unroll
-                for (int j = 0; j < 32; ++j) m |= v[j] >= thr_raw ? (1u << j) : 0u;
-                if (ncol < 32) m &= (1u << ncol) - 1u;
-                while (m) {   // counted past keep_cap: an overflow is seen, not lost
+                    for (int j = 0; j < 32; ++j) m |= v[j] >= edge ? (1u << j) : 0u;
+                    if (ncol < 32) m &= (1u << ncol) - 1u;
+                }
+                const int32_t id0 = (int32_t)(T.c0 + col0);
+                while (m) {
                     const int j = __ffs(m) - 1;
                     m &= m - 1u;
-                    if (kn < a.keep_cap) {
-                        ks[kn] = pick32(v, j) * kS;
-                        ki[kn] = (int32_t)(T.c0 + col0 + j);
+                    if (n < a.cap) {
+                        ls[n] = pick32(v, j) * kS;
+                        li[n] = id0 + j;
                     }
-                    ++kn;
+                    ++n;   // counted past cap: an overflow is seen, not lost
+                }
+                return;
+            }
+            float mx = v[0];
+            if (ncol == 32) {
+#pragma unroll
+                for (int j = 1; j < 32; ++j) mx = fmaxf(mx, v[j]);
+            } else {
+#pragma unroll
+                for (int j = 1; j < 32; ++j) mx = j < ncol ? fmaxf(mx, v[j]) : mx;
+            }
+            if constexpr (kMode == kRankGroupMax) {
+                if (!valid) return;
+                if (a.group == 32) {
+                    gm[col0 / 32] = mx * kS;
+                } else {   // 64: two consecutive 32-column groups (col0 = 0, 32, 64, 96 in turn)
+                    gacc = (col0 & 32) ? fmaxf(gacc, mx) : mx;
+                    if ((col0 & 32) || ncol < 32 || col0 + 32 >= T.nb) gm[col0 / 64] = gacc * kS;
+                }
+                return;
+            }
+            const bool any = valid && mx >= edge;
+            if (!__any_sync(0xffffffffu, any)) return;   // the common case: the group is rejected
+            unsigned m = 0;
+            if (any) {
+#pragma unroll
+                for (int j = 0; j < 32; ++j) m |= v[j] >= edge ? (1u << j) : 0u;
+                if (ncol < 32) m &= (1u << ncol) - 1u;
+            }
+            const int32_t id0 = (int32_t)(T.c0 + col0);
+            while (m) {
+                const int j = __ffs(m) - 1;
+                m &= m - 1u;
+                const float x = pick32(v, j);
+                if (!(x >= edge)) continue;   // the threshold rose within this group
+                if (n < a.cap) {
+                    ls[n] = x * kS;
+                    li[n] = id0 + j;
+                }
+                ++n;   // counted past cap: an overflow is seen, not lost
+                const int b = rank_bin(x);   // >= bin, since x reaches the bin's edge
+                if (h[b] < 255) {            // a saturated bin stops counting (conservative)
+                    ++h[b];
+                    if (b > bin && ++above >= a.nprobe) {
+                        // nprobe kept scores lie above the threshold bin: raise it
+                        while (above >= a.nprobe && bin < kRankBins - 1) {
+                            ++bin;
+                            above -= h[bin];
+                        }
+                        edge = fmaxf(init, rank_edge_raw(bin));
+                    }
                 }
             }
         }
         __device__ void prefetch(const Args &, const Tile &, int) {}
         __device__ void start(const Args &, const Tile &, int) {}
         __device__ void end(const Args &a, const Tile &) {
-            if (ks) a.keep_n[keep_at] = kn;
+            if (!valid || kMode == kRankGroupMax) return;
+            a.list_n[at] = n;
+            a.list_edge[at] = edge * (1.f / 65536.f);   // exact (-inf stays -inf)
         }
     };
 };
-static_assert(kRankRange % RankMode::kN == 0 && kRankRange % kTcRows == 0, "");
+// the first pass on the bulk pipeline: one fp16 product per score (hi halves
+// of A and B), whose error the threshold allows for
+struct RankScreenMode : RankModeT<kRankGroupMax> {
+    static constexpr int kProducts = 1;
+};
+static_assert(kTcRows == RankModeT<kRankStream>::kN, "");
 
+template <int kMode>
 __global__ void __launch_bounds__(tcp::kThreads, 1) k_rank_tc(RankArgs a) {
     extern __shared__ unsigned char smem_raw[];
-    tcp::run_pipeline<RankMode>(a, smem_raw);
+    tcp::run_pipeline<RankModeT<kMode>>(a, smem_raw);
 }
 
-int rank_bulk_stages(int d) { return tcb::stages_for((int)ceil_div(d, 64), 0, 232448 - 128); }
+int rank_bulk_stages(int d) {
+    return tcb::stages_for((int)ceil_div(d, 64), kRankEpiBytes, 232448 - 128);
+}
 
+template <int kMode>
 __global__ void __launch_bounds__(tcb::kThreads, 1) k_rank_bulk(RankArgs a, int stages) {
     extern __shared__ unsigned char smem_raw[];
-    tcb::run_bulk<RankMode>(a, smem_raw, stages);
+    tcb::run_bulk<RankModeT<kMode>>(a, smem_raw, stages);
 }
 
-constexpr int kSelectWarps = 4;
+int rank_screen_stages(int d) {
+    return tcb::stages_for((int)ceil_div(d, 64), kRankEpiBytes, 232448 - 128, tcb::kStageBytesHi);
+}
+
+__global__ void __launch_bounds__(tcb::kThreads, 1) k_rank_screen(RankArgs a, int stages) {
+    extern __shared__ unsigned char smem_raw[];
+    tcb::run_bulk<RankScreenMode>(a, smem_raw, stages);
+}
+
+constexpr int kSelectWarps = 4;  // warps (queries) per block of the final selection
 constexpr int kSelectMaxR = 8;   // lane order statistics used for the lower bracket
-constexpr int kStage2 = 16;      // keys per lane of the second selection step (512 entries)
-constexpr int kGroupMax = 2048;  // group maxima one threshold warp holds (64 per lane)
 
 // warp-wide reductions in one instruction (redux.sync), not a chain of shuffles
 __device__ __forceinline__ int warp_sum(int x) { return __reduce_add_sync(0xffffffffu, x); }
@@ -402,22 +499,41 @@ __device__ __forceinline__ void warp_gather_exact(const uint32_t (&key)[KPL], in
     __syncwarp();
 }
 
-// The want best of the warp's cnt entries into bs/bc[0 .. want-1], in entry
-// order (sort_buffer orders them).  With many keys per lane and a second-step
-// buffer (ck/ci, 32 * K2 entries; nullable): a first threshold, refined
-// until at most 32 * K2 keys reach it (K2 about 2 want / 32), the keys that
-// reach it compacted there in entry order, and the exact selection over K2
-// keys per lane.
+// the want best of n candidates (keys ck, ids ci in shared memory, id order;
+// n <= 32 * KPL, want <= n) into bs/bc, in id order
+template <int KPL>
+__device__ __forceinline__ void select_candidates(const uint32_t *ck, const int *ci, int n, int want,
+                                                  float *bs, int *bc) {
+    const int lane = threadIdx.x & 31;
+    uint32_t key[KPL];
+#pragma unroll
+    for (int j = 0; j < KPL; ++j) {
+        const int c = j * 32 + lane;
+        key[j] = c < n ? ck[c] : 0u;
+    }
+    uint32_t T;
+    int C;
+    warp_threshold(key, want, want, T, C);
+    warp_gather_exact(key, n, want, T, C, [&](int c) { return ci[c]; }, bs, bc);
+}
+
+// The want best of the warp's cnt entries (KPL keys per lane, entry c =
+// key[c / 32] of lane c % 32, its id id_of(c)) into bs/bc in entry order, in
+// two steps: a first threshold refined until at most 32 * K2 keys reach it
+// (K2 about 2 want / 32), those keys compacted in entry order into ck/ci, and
+// the exact selection over K2 keys per lane.  A first threshold still
+// reached by more than 32 * K2 keys is the want-th largest key itself, tied:
+// the exact gather over all keys takes it from there.
 template <int K2, int KPL, class IdOf>
-__device__ __forceinline__ bool select_two_step(const uint32_t (&key)[KPL], int cnt, int want,
+__device__ __forceinline__ void select_two_step(const uint32_t (&key)[KPL], int cnt, int want,
                                                 IdOf id_of, uint32_t *ck, int *ci, float *bs,
                                                 int *bc) {
     uint32_t T;
     int C;
     warp_threshold(key, want, 32 * K2, T, C);
-    if (C > 32 * K2) {   // T is the want-th largest key itself, tied past the buffer
+    if (C > 32 * K2) {
         warp_gather_exact(key, cnt, want, T, C, id_of, bs, bc);
-        return true;
+        return;
     }
     const int lane = threadIdx.x & 31;
     const unsigned below = (1u << lane) - 1u;
@@ -443,94 +559,166 @@ __device__ __forceinline__ bool select_two_step(const uint32_t (&key)[KPL], int 
     }
     warp_threshold(k2, want, want, T, C);
     warp_gather_exact(k2, pos, want, T, C, [&](int c) { return ci[c]; }, bs, bc);
-    return true;
 }
 
-template <int K2, int KPL, class IdOf>
-__device__ __forceinline__ void warp_select_exact(const uint32_t (&key)[KPL], int cnt, int want,
-                                                  IdOf id_of, uint32_t *ck, int *ci, float *bs,
-                                                  int *bc) {
-    static_assert(K2 <= kStage2, "");
-    if (want <= 0) return;
-    if constexpr (KPL > kStage2) {
-        if (ck) {
-            select_two_step<K2>(key, cnt, want, id_of, ck, ci, bs, bc);
-            return;
-        }
-    }
-    uint32_t T;
-    int C;
-    warp_threshold(key, want, want, T, C);
-    warp_gather_exact(key, cnt, want, T, C, id_of, bs, bc);
-}
+constexpr int kDenseK2Max = 16;   // second-step keys per lane of the dense selection
 
-// One warp per (query, segment of at most kSelectSeg entries).  The
-// segment's entries are positions s*seg .. min(M, (s+1)*seg)-1 of the query's
-// row of `in_s` (ids from `in_id`, or the position itself when in_id is null),
-// in id order among equal scores (a row of centroid scores, or the sorted
-// outputs of consecutive id ranges); want = min(nprobe, entries).  Output: the
-// want best in order at out_id/out_s[q * out_ld + s * nprobe ..], then
-// (-inf, INT32_MAX) padding up to nprobe.  qlist (nullable): only the queries
-// qlist[0 .. *qlist_n - 1]; the warps stride over them.  seg_cnt (nullable):
-// [nq][nseg] entries actually present in each segment.  nprobe <= 32 * R.
-// Eight blocks per SM (64 registers) where the keys fit: the selection is a
-// chain of dependent warp reductions, so it needs the warps to hide their
-// latency.
-template <int KPL, int R>   // entries per lane: seg <= 32 * KPL
-__global__ void __launch_bounds__(kSelectWarps * 32, (KPL >= 64 || R >= 8) ? 4 : 8)
-    k_select(
-    const float *__restrict__ in_s, const int32_t *__restrict__ in_id, int64_t in_ld, int64_t nq,
-    int64_t M, int seg, int nseg, int nprobe, int32_t *__restrict__ out_id,
-    float *__restrict__ out_s, int64_t out_ld, const int *__restrict__ qlist,
-    const int *__restrict__ qlist_n, const int *__restrict__ seg_cnt) {
+// One warp per query of a dense single-range ranking (every score of the
+// query in its list, ids = positions): the keys straight from the list into
+// registers (KPL per lane), the nprobe best (two steps when KPL > 16), sorted.
+template <int KPL, int R>
+__global__ void __launch_bounds__(kSelectWarps * 32, (KPL >= 64 || R >= 8) ? 4 : 8) k_rank_dense_final(
+    const float *__restrict__ list_s, const int *__restrict__ list_n, int64_t nq, int cap,
+    int nprobe, int32_t *__restrict__ order, float *__restrict__ cscores) {
     extern __shared__ __align__(16) unsigned char sel_smem[];
-    // second-step keys per lane: about twice nprobe / 32
-    constexpr int kK2 = R <= 2 ? 4 : R == 4 ? 8 : kStage2;
+    constexpr int kK2 = R <= 2 ? 4 : R == 4 ? 8 : kDenseK2Max;   // about twice nprobe / 32
     constexpr int kSort = 32 * R;
-    constexpr int kS2 = KPL > kStage2 ? 32 * kK2 : 0;
+    constexpr int kS2 = KPL > kDenseK2Max ? 32 * kK2 : 0;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     float *bs = reinterpret_cast<float *>(sel_smem) + (size_t)warp * 2 * (kSort + kS2);
     int *bc = reinterpret_cast<int *>(bs + kSort);
-    uint32_t *ck = kS2 ? reinterpret_cast<uint32_t *>(bc + kSort) : nullptr;
-    int *ci = kS2 ? reinterpret_cast<int *>(ck + kS2) : nullptr;
-    const int64_t total = (qlist ? (int64_t)*qlist_n : nq) * nseg;
-    for (int64_t w = (int64_t)blockIdx.x * kSelectWarps + warp; w < total;
-         w += (int64_t)gridDim.x * kSelectWarps) {
-        const int64_t q = qlist ? (int64_t)qlist[w / nseg] : w / nseg;
-        const int sg = (int)(w % nseg);
-        const int64_t p0 = (int64_t)sg * seg;
-        int cnt = (int)(M - p0 < seg ? M - p0 : seg);
-        if (seg_cnt && seg_cnt[q * nseg + sg] < cnt) cnt = seg_cnt[q * nseg + sg];
-        const int want = nprobe < cnt ? nprobe : cnt;
-        const float *row = in_s + q * in_ld + p0;
-        const int32_t *rid = in_id ? in_id + q * in_ld + p0 : nullptr;
-        uint32_t key[KPL];   // the scores themselves are recovered from the keys
+    uint32_t *ck = reinterpret_cast<uint32_t *>(bc + kSort);
+    int *ci = reinterpret_cast<int *>(ck + kS2);
+    const int64_t q = (int64_t)blockIdx.x * kSelectWarps + warp;
+    if (q >= nq) return;
+    const float *row = list_s + q * cap;
+    const int cnt = list_n[q];
+    const int want = nprobe < cnt ? nprobe : cnt;
+    uint32_t key[KPL];
 #pragma unroll
-        for (int j = 0; j < KPL; ++j) {
-            const int c = j * 32 + lane;
-            key[j] = c < cnt ? order_key(row[c]) : 0u;   // padding ranks below every score
-        }
-        warp_select_exact<kK2>(key, cnt, want, [&](int c) { return rid ? rid[c] : (int)(p0 + c); },
-                               ck, ci, bs, bc);
-        sort_buffer<R>(bs, bc, want);
-        int32_t *oi = out_id + q * out_ld + (int64_t)sg * nprobe;
-        float *os = out_s ? out_s + q * out_ld + (int64_t)sg * nprobe : nullptr;
-        for (int p = lane; p < nprobe; p += 32) {
-            oi[p] = p < want ? bc[p] : INT32_MAX;
-            if (os) os[p] = p < want ? bs[p] : -__int_as_float(0x7f800000);
-        }
-        __syncwarp();
+    for (int j = 0; j < KPL; ++j) {
+        const int c = j * 32 + lane;
+        key[j] = c < cnt ? order_key(row[c]) : 0u;   // padding ranks below every score
+    }
+    auto id_of = [](int c) { return c; };
+    if constexpr (KPL > kDenseK2Max) {
+        select_two_step<kK2>(key, cnt, want, id_of, ck, ci, bs, bc);
+    } else {
+        uint32_t T;
+        int C;
+        warp_threshold(key, want, want, T, C);
+        warp_gather_exact(key, cnt, want, T, C, id_of, bs, bc);
+    }
+    sort_buffer<R>(bs, bc, want);
+    for (int p = lane; p < nprobe; p += 32) {
+        order[q * nprobe + p] = p < want ? bc[p] : INT32_MAX;
+        if (cscores) cscores[q * nprobe + p] = p < want ? bs[p] : -__int_as_float(0x7f800000);
     }
 }
 
-// Threshold from group maxima: one warp per query over its ng maxima of
-// 32-centroid groups (ng >= nprobe).  The nprobe-th largest maximum L is a
-// score of nprobe different centroids at least, so at least nprobe scores are
-// >= L and the nprobe best all are.  Writes the order key of L.
+static size_t dense_smem(int kpl, int R) {
+    const int k2 = R <= 2 ? 4 : R == 4 ? 8 : kDenseK2Max;
+    return (size_t)kSelectWarps * 2 * (32 * (size_t)R + (kpl > kDenseK2Max ? 32 * (size_t)k2 : 0)) * 4;
+}
+
+// One warp per query: the candidates of its ranges that reach their final
+// thresholds, gathered in order (id order) into ccap slots, then the nprobe
+// best sorted into order/cscores.  Dense lists (list_i null) hold every score
+// of their range, the id being the range start plus the position.  A list past cap, more than ccap
+// candidates, or fewer than nprobe (NaN scores): the query is appended to
+// ovf_list (count in *ovf_n, zeroed before the launch) for the exact FP32
+// ranking.  nprobe <= 32 * R.
+template <int R, int KMAX>   // KMAX: keys per lane of the largest candidate set (ccap / 32)
+__global__ void __launch_bounds__(kSelectWarps * 32, KMAX <= 16 ? 8 : 4) k_rank_final(
+    const float *__restrict__ list_s, const int32_t *__restrict__ list_i,
+    const int *__restrict__ list_n, const float *__restrict__ list_edge, int64_t nq, int nranges,
+    int64_t range_len, int cap, int nprobe, int ccap, int32_t *__restrict__ order,
+    float *__restrict__ cscores, int *__restrict__ ovf_list, int *__restrict__ ovf_n) {
+    extern __shared__ __align__(16) unsigned char sel_smem[];
+    constexpr int kSort = 32 * R;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    unsigned char *wbase = sel_smem + (size_t)warp * ((size_t)ccap + kSort) * 8;
+    uint32_t *ck = reinterpret_cast<uint32_t *>(wbase);                 // candidate keys
+    int *ci = reinterpret_cast<int *>(wbase + (size_t)ccap * 4);        // candidate ids
+    float *bs = reinterpret_cast<float *>(wbase + (size_t)ccap * 8);    // sort buffer
+    int *bc = reinterpret_cast<int *>(bs + kSort);
+    const int64_t q = (int64_t)blockIdx.x * kSelectWarps + warp;
+    if (q >= nq) return;
+    const unsigned below = (1u << lane) - 1u;
+    int n = 0;
+    bool over = false;
+    for (int r = 0; r < nranges && !over; ++r) {
+        const int64_t at = q * nranges + r;
+        const int cnt = list_n[at];
+        if (cnt > cap) {
+            over = true;
+            break;
+        }
+        const float e = list_edge[at];
+        const float *s = list_s + at * cap;
+        const int32_t *id = list_i ? list_i + at * cap : nullptr;   // null: dense, id = position
+        const int32_t id0 = (int32_t)(r * range_len);
+        for (int i0 = 0; i0 < cnt; i0 += 32) {
+            const int i = i0 + lane;
+            const float x = i < cnt ? s[i] : 0.f;
+            const bool keep = i < cnt && x >= e;
+            const unsigned bal = __ballot_sync(0xffffffffu, keep);
+            const int p = n + __popc(bal & below);
+            if (keep && p < ccap) {
+                ck[p] = order_key(x);
+                ci[p] = id ? id[i] : id0 + i;
+            }
+            n += __popc(bal);
+        }
+        over = n > ccap;
+    }
+    if (over || n < nprobe) {
+        if (lane == 0) ovf_list[atomicAdd(ovf_n, 1)] = (int)q;
+        return;
+    }
+    __syncwarp();
+    // keys per lane sized to the candidates (warp-uniform n <= ccap <= 32 KMAX)
+    if (n <= 128 || KMAX <= 4)
+        select_candidates<4>(ck, ci, n, nprobe, bs, bc);
+    else if (n <= 512 || KMAX <= 16)
+        select_candidates<(KMAX < 16 ? KMAX : 16)>(ck, ci, n, nprobe, bs, bc);
+    else if (n <= 1024 || KMAX <= 32)
+        select_candidates<(KMAX < 32 ? KMAX : 32)>(ck, ci, n, nprobe, bs, bc);
+    else
+        select_candidates<KMAX>(ck, ci, n, nprobe, bs, bc);
+    sort_buffer<R>(bs, bc, nprobe);
+    for (int p = lane; p < nprobe; p += 32) {
+        order[q * nprobe + p] = bc[p];
+        if (cscores) cscores[q * nprobe + p] = bs[p];
+    }
+}
+
+// The largest centroid norm (one float, zeroed before the launch; norms are
+// non-negative, so their bit patterns order like the floats)
+__global__ void k_cnorm_max(const float *__restrict__ C, int64_t nlist, int d,
+                            unsigned *__restrict__ out) {
+    const int lane = threadIdx.x & 31;
+    float best = 0.f;
+    const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
+    for (int64_t c = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; c < nlist; c += warps) {
+        float ss = 0.f;
+        for (int t = lane; t < d; t += 32) ss = fmaf(C[c * d + t], C[c * d + t], ss);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+        best = fmaxf(best, sqrtf(ss));
+    }
+    if (lane == 0) atomicMax(out, __float_as_uint(best));
+}
+
+// One warp per query: T = a key reached by at least nprobe of its ng group
+// maxima (warp_threshold; each maximum is a different centroid's score), so
+// at least nprobe centroids score >= T in the first pass.  The second pass
+// keeps every score >= T - margin, margin = the first pass's error bound plus
+// the second's (slack = 0 when both passes compute identical scores):
+//   screen (one fp16 product of the hi halves, fp32 sums, as in the screening
+//   scan): (2^-10 + 2^-12 + d 2^-22) |q| |c| + 2^-26 sqrt(d) (|q| + |c|);
+//   three products: (2^-20 + d 2^-22) |q| |c| + 2^-26 sqrt(d) (|q| + |c|)
+//   (the dropped lo*lo term and the rounding of the lo halves, 3 2^-22 of each
+//   |q_i c_i|, and the fp32 sums of 3d products);
+// |c| = the largest centroid norm.  Every centroid among the nprobe best of
+// the second pass then scores >= T - margin: the nprobe centroids with a
+// first-pass score >= T score at least T - margin there.  Writes the
+// starting threshold (score units) of each query.
 template <int KPL>
-__global__ void __launch_bounds__(kSelectWarps * 32) k_group_threshold(
+__global__ void __launch_bounds__(kSelectWarps * 32) k_rank_threshold(
     const float *__restrict__ gmax, int64_t gld, int64_t nq, int ng, int nprobe,
-    uint32_t *__restrict__ lkey) {
+    const float *__restrict__ Q, int d, const unsigned *__restrict__ cmax_bits, int screen,
+    float *__restrict__ init_edge) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t q = (int64_t)blockIdx.x * kSelectWarps + warp;
     if (q >= nq) return;
@@ -543,178 +731,25 @@ __global__ void __launch_bounds__(kSelectWarps * 32) k_group_threshold(
     }
     uint32_t T;
     int C;
-    warp_threshold(key, nprobe, nprobe, T, C);   // refined to the nprobe-th largest
-    if (lane == 0) lkey[q] = T;
-}
-
-constexpr int kSegCap = 256;        // candidates one table segment may hand on
-
-// One warp per (query, segment of kSelectSeg scores): the scores that reach
-// the query's threshold key, in id order, into the segment's kSegCap slots of
-// cand_s/cand_i [q][nseg * kSegCap]; their number (even past kSegCap) into
-// seg_n[q][nseg].  Lane l reads the segment's 64 scores l*64 .. l*64+63 with
-// 16-byte loads, all issued before any is used.
-__global__ void __launch_bounds__(kSelectWarps * 32) k_compact_seg(
-    const float *__restrict__ scores, int64_t ld, int64_t nq, int64_t nlist, int nseg,
-    const uint32_t *__restrict__ lkey, float *__restrict__ cand_s, int32_t *__restrict__ cand_i,
-    int *__restrict__ seg_n) {
-    constexpr int kPer = kSelectSeg / 32;   // 64 scores per lane
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int64_t w = (int64_t)blockIdx.x * kSelectWarps + warp;
-    if (w >= nq * nseg) return;
-    const int64_t q = w / nseg;
-    const int sg = (int)(w % nseg);
-    const int64_t c0 = (int64_t)sg * kSelectSeg + lane * kPer;   // this lane's first column
-    const float *row = scores + q * ld;
-    const uint32_t L = lkey[q];
-    float4 v[kPer / 4];
+    warp_threshold(key, nprobe, nprobe, T, C);
+    float ss = 0.f;
+    for (int t = lane; t < d; t += 32) ss = fmaf(Q[q * d + t], Q[q * d + t], ss);
 #pragma unroll
-    for (int i = 0; i < kPer / 4; ++i)   // ld is a multiple of 32: a 4-group below ld is whole
-        v[i] = c0 + 4 * i < ld ? *reinterpret_cast<const float4 *>(row + c0 + 4 * i)
-                               : make_float4(0.f, 0.f, 0.f, 0.f);
-    uint64_t hit = 0;   // bit j: column c0 + j qualifies
-#pragma unroll
-    for (int i = 0; i < kPer / 4; ++i) {
-        const float x[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            const int j = 4 * i + e;
-            if (c0 + j < nlist && order_key(x[e]) >= L) hit |= 1ull << j;
-        }
-    }
-    // this lane's place among the segment's candidates: lanes hold consecutive columns
-    const int mine = __popcll(hit);
-    int x = mine;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_up_sync(0xffffffffu, x, o);
-        if (lane >= o) x += y;
-    }
-    int p = x - mine;
-    float *os = cand_s + (q * nseg + sg) * kSegCap;
-    int32_t *oi = cand_i + (q * nseg + sg) * kSegCap;
-    while (hit) {
-        const int j = __ffsll((long long)hit) - 1;
-        hit &= hit - 1;
-        if (p < kSegCap) {   // the rare candidate's score again (cached), not a register pick
-            os[p] = row[c0 + j];
-            oi[p] = (int)(c0 + j);
-        }
-        ++p;
-    }
-    if (lane == 31) seg_n[q * nseg + sg] = x;
-}
-
-// the nprobe best of n candidates (keys ck, ids ci in shared memory, id order;
-// n <= 32 * KPL, n >= nprobe) into bs/bc, in id order
-template <int KPL>
-__device__ __forceinline__ void compact_finish(const uint32_t *ck, const int *ci, int n, int nprobe,
-                                               float *bs, int *bc) {
-    const int lane = threadIdx.x & 31;
-    uint32_t key[KPL];
-#pragma unroll
-    for (int j = 0; j < KPL; ++j) {
-        const int c = j * 32 + lane;
-        key[j] = c < n ? ck[c] : 0u;
-    }
-    warp_select_exact<kStage2>(key, n, nprobe, [&](int c) { return ci[c]; }, (uint32_t *)nullptr,
-                               (int *)nullptr, bs, bc);
-}
-
-// One warp per query: its segments' candidates (at most segcap kept per
-// segment) gathered in order (id order) into ccap slots, then the nprobe best
-// sorted into order/cscores.  A segment past segcap or more than ccap in all
-// (many equal scores): the query is appended to ovf_list (count in *ovf_n,
-// zeroed before the launch) and left to an exact fallback.  nprobe <= 32 * R.
-template <int R>
-__global__ void __launch_bounds__(kSelectWarps * 32, 6) k_compact_final(
-    const float *__restrict__ cand_s, const int32_t *__restrict__ cand_i,
-    const int *__restrict__ seg_n, int64_t nq, int nseg, int segcap, int nprobe, int ccap,
-    int32_t *__restrict__ order, float *__restrict__ cscores, int *__restrict__ ovf_list,
-    int *__restrict__ ovf_n) {
-    extern __shared__ __align__(16) unsigned char sel_smem[];
-    constexpr int kSort = 32 * R;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    unsigned char *wbase = sel_smem + (size_t)warp * ((size_t)ccap + kSort) * 8;
-    uint32_t *ck = reinterpret_cast<uint32_t *>(wbase);                 // candidate keys
-    int *ci = reinterpret_cast<int *>(wbase + (size_t)ccap * 4);        // candidate ids
-    float *bs = reinterpret_cast<float *>(wbase + (size_t)ccap * 8);    // sort buffer
-    int *bc = reinterpret_cast<int *>(bs + kSort);
-    const int64_t q = (int64_t)blockIdx.x * kSelectWarps + warp;
-    if (q >= nq) return;
-    // segment counts and their running offsets, 32 segments at a time
-    int n = 0;
-    bool over = false;
-    for (int s0 = 0; s0 < nseg; s0 += 32) {
-        const int sg = s0 + lane;
-        const int c = sg < nseg ? seg_n[q * nseg + sg] : 0;
-        over |= __any_sync(0xffffffffu, c > segcap);
-        int x = c;   // inclusive scan over the lanes
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int y = __shfl_up_sync(0xffffffffu, x, o);
-            if (lane >= o) x += y;
-        }
-        const int total = __shfl_sync(0xffffffffu, x, 31);
-        if (!over && n + total <= ccap && c > 0) {
-            // lane l copies segment s0 + l to its place: the segments' loads
-            // are in flight together, four of each lane's at a time
-            const int at = n + x - c;
-            const float *ss = cand_s + (q * nseg + sg) * (int64_t)segcap;
-            const int32_t *si = cand_i + (q * nseg + sg) * (int64_t)segcap;
-#pragma unroll 4
-            for (int i = 0; i < c; ++i) {
-                ck[at + i] = order_key(ss[i]);
-                ci[at + i] = si[i];
-            }
-        }
-        n += total;
-        over |= n > ccap;
-    }
-    if (over) {
-        if (lane == 0) ovf_list[atomicAdd(ovf_n, 1)] = (int)q;
-        return;
-    }
-    __syncwarp();
-    // keys per lane sized to the candidates (warp-uniform n)
-    if (n <= 128)
-        compact_finish<4>(ck, ci, n, nprobe, bs, bc);
-    else if (n <= 512)
-        compact_finish<16>(ck, ci, n, nprobe, bs, bc);
-    else if (n <= 1024)
-        compact_finish<32>(ck, ci, n, nprobe, bs, bc);
-    else
-        compact_finish<64>(ck, ci, n, nprobe, bs, bc);
-    sort_buffer<R>(bs, bc, nprobe);
-    for (int p = lane; p < nprobe; p += 32) {
-        order[q * nprobe + p] = bc[p];
-        if (cscores) cscores[q * nprobe + p] = bs[p];
-    }
+    for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+    // the norms and the margin rounded upward, so the margin is never short
+    const float qn = __fsqrt_ru(ss) * (1.f + 0x1p-20f);
+    const float cn = __uint_as_float(*cmax_bits) * (1.f + 0x1p-20f);
+    const float rd = __fsqrt_ru((float)d);
+    const float three = (0x1p-20f + (float)d * 0x1p-22f) * qn * cn + 0x1p-26f * rd * (qn + cn);
+    const float scr = screen ? (0x1p-10f + 0x1p-12f + (float)d * 0x1p-22f) * qn * cn +
+                                   0x1p-26f * rd * (qn + cn)
+                             : 0.f;
+    const float margin = screen ? (scr + three) * (1.f + 0x1p-16f) : 0.f;
+    if (lane == 0) init_edge[q] = __fsub_rd(key_score(T), margin);
 }
 
 // ---------------------------------------------------------------------------
 bool rank_tc_supported(int64_t nlist, int nprobe) { return nlist >= 1 && nprobe <= nlist; }
-
-int64_t rank_tc_ld(int64_t nlist) { return round_up(nlist, 32); }
-
-// entries each selection level leaves per query (level 0 = the score row)
-static int64_t level_entries(int64_t M, int nprobe) { return ceil_div(M, kSelectSeg) * nprobe; }
-
-// more centroids than one selecting warp holds: a threshold from the maxima
-// of 32-centroid groups when there are at least nprobe groups (and few enough
-// for one warp), then one compacting pass
-static bool use_group_threshold(int64_t nlist, int nprobe) {
-    const int64_t ng = ceil_div(nlist, 32);
-    return nlist > kSelectSeg && ng >= nprobe && ng <= kGroupMax;
-}
-
-// Under the group threshold, narrow rows (d <= 128) skip the score table: one
-// contraction writes only the group maxima, a second keeps only the scores
-// that reach the threshold.  Two passes of 6d fp16 products per score cost
-// less than writing and reading 8 bytes per score when d is this small.
-static bool use_two_pass(int64_t nlist, int nprobe, int d) {
-    return use_group_threshold(nlist, nprobe) && d <= 128;
-}
 
 static int pow2_at_least(int64_t x) {
     int p = 1;
@@ -722,192 +757,228 @@ static int pow2_at_least(int64_t x) {
     return p;
 }
 
-// kept slots per 2,048-centroid range on the two-pass path: four times a
-// range's even share of nprobe (the threshold keeps a little over nprobe
-// scores in all), at least 64.  A range past it sends its query to the FP32
-// fallback.
-static int keep_cap(int64_t nlist, int nprobe) {
-    const int64_t nseg = ceil_div(nlist, kRankRange);
-    const int c = pow2_at_least(ceil_div(4 * (int64_t)nprobe, nseg));
-    return (int)std::min<int64_t>(kRankRange, std::max(64, c));
-}
-
-// candidates one compacting warp holds: 4 P (P = nprobe rounded up to a
-// power of two), between 512 and 2,048
-static int compact_cap(int nprobe) {
-    return std::min(2048, std::max(512, 4 * pow2_at_least(nprobe)));
-}
-
 // registers per lane of the sort of nprobe entries
 static int sort_regs(int nprobe) { return std::max(2, pow2_at_least(nprobe) / 32); }
 
-// Scratch of one query, in the order enqueue_rank_tc lays it out:
-//   score row (table path only)                      round_up(nlist, 32) f32
-//   two level buffers (scores, then ids)             2 x lvl x 8 B   (table path, nlist > kSelectSeg)
-//   group maxima                                     round_up(ng, 4) f32
-//   candidate slots (scores, then ids)               nseg x cap x 8 B (cap = kSegCap, or
-//                                                    keep_cap on the two-pass path)
-//   candidate counts, threshold key, overflow list   round_up(nseg, 4) x 4 B + 8 B
-// and once per chunk the overflow count (kRankFixedBytes).
-constexpr int64_t kRankFixedBytes = 256;
-struct RankScratch {
-    int64_t ld, lvl, gld, cap;
-    int nseg;
-    bool table, grouped;
+constexpr int kFinalCapMax = 2048;   // candidates one final-selection warp holds (64 per lane)
+constexpr int kMaxGroups = 2048;     // group maxima one threshold warp holds (64 per lane)
+
+// How one ranking call is cut up.
+//  kind: nlist <= 2,048: one pass keeping every score (dense lists, ids
+//    implicit).  Else, when there are at least 2 nprobe groups of 64 (or 32)
+//    centroids and at most 2,048 of them: two passes -- group maxima (on the
+//    screen when the bulk pipeline applies), a per-query threshold, and the
+//    streaming pass from that threshold.  Else the streaming pass alone.
+//  ranges: enough (query tile, range) tiles for about four waves of the
+//    persistent contraction; the streaming pass alone takes at most
+//    2,048 / 2P ranges (each keeps P plus a bin's width of candidates);
+//  cap: list slots per (query, range): the whole range (dense); 2P, at least
+//    256 (two passes: the threshold keeps a little over P per query in all);
+//    with the running threshold alone, a random order offers about
+//    P (1 + ln(len / P)) scores (the expected number of times a new score
+//    enters the running best P, standard deviation near sqrt(P ln(len / P))),
+//    and the cap is 1.25 times that plus 64, at most 8,192;
+//  chunk: queries per pass, so that their scratch fits kRankScratchBytes.
+struct RankPlan {
+    int mode;        // the final pass: kRankDense or kRankStream
+    int group;       // centroids per group of the first pass; 0 = no first pass
+    bool screen;     // the first pass screens (bulk pipeline)
+    int nranges;
+    int64_t range_len;
+    int cap;
+    int ng;          // groups of the first pass
+    int64_t gld;
+    int ccap;        // final-selection slots
+    int64_t chunk;
     int64_t per_query() const {
-        int64_t b = table ? ld * 4 : 0;
-        b += 2 * lvl * 8;
-        if (grouped) b += gld * 4 + (int64_t)nseg * cap * 8 + round_up(nseg, 4) * 4 + 8;
-        return b;
+        const int64_t entry = mode == kRankDense ? 4 : 8;
+        return (int64_t)nranges * ((int64_t)cap * entry + 8) + 4 + (group ? gld * 4 + 4 : 0);
     }
 };
+constexpr int64_t kRankFixedBytes = 256;   // the overflow count and the largest centroid norm
 
-static RankScratch rank_scratch(int64_t nlist, int nprobe, int d) {
-    RankScratch r;
-    r.ld = rank_tc_ld(nlist);
-    r.grouped = use_group_threshold(nlist, nprobe);
-    r.table = !use_two_pass(nlist, nprobe, d);
-    // the two-pass path falls back to the FP32 ranking, not to the levels
-    r.lvl = (nlist > kSelectSeg && r.table) ? round_up(level_entries(nlist, nprobe), 4) : 0;
-    r.gld = round_up(ceil_div(nlist, 32), 4);
-    r.nseg = (int)ceil_div(nlist, kSelectSeg);
-    r.cap = r.table ? kSegCap : keep_cap(nlist, nprobe);
-    return r;
-}
-
-int64_t rank_tc_chunk(int64_t nq, int64_t nlist, int nprobe, int d) {
-    int64_t c = kRankScratchBytes / rank_scratch(nlist, nprobe, d).per_query();
-    c = c / tcp::kM * tcp::kM;
-    if (c < tcp::kM) c = tcp::kM;
-    return nq < c ? nq : c;
+static RankPlan rank_plan(int64_t nq, int64_t nlist, int nprobe, int d, bool bulk) {
+    RankPlan L{};
+    const int P = pow2_at_least(nprobe);
+    L.group = 0;
+    if (nlist <= kFinalCapMax) {
+        L.mode = kRankDense;
+    } else {
+        L.mode = kRankStream;
+        for (int g : {64, 32}) {
+            const int64_t ng = ceil_div(nlist, g);
+            if (ng >= 2 * (int64_t)nprobe && ng <= kMaxGroups) {
+                L.group = g;
+                break;
+            }
+        }
+    }
+    L.screen = L.group && bulk && rank_screen_stages(d) > 0;
+    const int64_t qtiles = std::max<int64_t>(1, ceil_div(nq, tcp::kM));
+    const int64_t want = ceil_div(4 * (int64_t)num_sms(), qtiles);
+    int64_t most = ceil_div(nlist, RankModeT<kRankStream>::kN);
+    if (L.mode == kRankStream && !L.group) most = std::min<int64_t>(most, std::max(1, kFinalCapMax / (2 * P)));
+    const int64_t r = std::max<int64_t>(1, std::min(want, most));
+    L.range_len = round_up(ceil_div(nlist, r), RankModeT<kRankStream>::kN);
+    L.nranges = (int)ceil_div(nlist, L.range_len);
+    if (L.mode == kRankDense) {
+        L.cap = (int)round_up(L.range_len, 32);
+    } else if (L.group) {
+        L.cap = std::max(256, 2 * P);
+    } else {
+        const double offered = P * (1.0 + std::log(std::max(1.0, (double)L.range_len / P)));
+        L.cap = (int)std::min<int64_t>(8192, round_up((int64_t)std::ceil(1.25 * offered) + 64, 64));
+    }
+    L.cap = (int)std::min<int64_t>(L.cap, round_up(L.range_len, 32));
+    L.ng = L.group ? (int)ceil_div(nlist, L.group) : 0;
+    L.gld = L.group ? round_up(L.ng, 4) : 0;
+    L.ccap = (int)std::min<int64_t>(kFinalCapMax, round_up((int64_t)L.nranges * L.cap, 32));
+    int64_t c = (kRankScratchBytes - kRankFixedBytes) / L.per_query();
+    c = std::max<int64_t>(tcp::kM, c / tcp::kM * tcp::kM);
+    L.chunk = std::min(nq, c);
+    return L;
 }
 
 size_t rank_tc_scratch_bytes(int64_t nq, int64_t nlist, int nprobe, int d) {
-    return (size_t)(rank_tc_chunk(nq, nlist, nprobe, d) * rank_scratch(nlist, nprobe, d).per_query() +
-                    kRankFixedBytes);
+    if (nq <= 0) return kRankFixedBytes;
+    // the bulk pipeline's plan needs at least the converter's scratch: size for the larger
+    const RankPlan a = rank_plan(nq, nlist, nprobe, d, true), b = rank_plan(nq, nlist, nprobe, d, false);
+    return (size_t)(std::max(a.chunk * a.per_query(), b.chunk * b.per_query()) + kRankFixedBytes);
 }
 
-static size_t tc_smem() { return tcp::Geometry<RankMode::kN>::smem_bytes(0); }
+static size_t tc_smem() { return tcp::Geometry<RankModeT<kRankStream>::kN>::smem_bytes(kRankEpiBytes); }
 
-// shared memory of the selecting kernels (kSelectWarps warps, each with its
-// own buffers)
-static size_t select_smem(int kpl, int R) {
-    const int k2 = R <= 2 ? 4 : R == 4 ? 8 : kStage2;   // k_select's second-step keys per lane
-    const size_t s2 = kpl > kStage2 ? 32 * (size_t)k2 : 0;
-    return (size_t)kSelectWarps * (32 * (size_t)R + s2) * 8;
-}
-static size_t compact_smem(int ccap, int R) {
+static size_t final_smem(int ccap, int R) {
     return (size_t)kSelectWarps * ((size_t)ccap + 32 * (size_t)R) * 8;
 }
 
 template <int R>
-static cudaError_t set_compact_attr(int ccap) {
-    return cudaFuncSetAttribute(k_compact_final<R>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)compact_smem(ccap, R));
-}
-
-cudaError_t prepare_rank_tc(int nprobe, int d) {
-    cudaError_t e = cudaFuncSetAttribute(k_rank_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)tc_smem());
-    const int bulk = rank_bulk_stages(d);
-    if (e == cudaSuccess && bulk)
-        e = cudaFuncSetAttribute(k_rank_bulk, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)tcb::smem_bytes(bulk, 0));
-    // the selections stay below the 48 KB default; the compacting warps may not
-    const int ccap = compact_cap(nprobe);
-    if (e == cudaSuccess) e = set_compact_attr<2>(ccap);
-    if (e == cudaSuccess) e = set_compact_attr<4>(ccap);
-    if (e == cudaSuccess) e = set_compact_attr<8>(ccap);
-    if (e == cudaSuccess) e = set_compact_attr<16>(ccap);
-    // the two-pass path's exact fallback
-    if (e == cudaSuccess && d <= 128) e = prepare_rank(nprobe);
+static cudaError_t set_final_attr() {
+    cudaError_t e = cudaSuccess;
+    for (auto f : {k_rank_final<R, 4>, k_rank_final<R, 16>, k_rank_final<R, 32>, k_rank_final<R, 64>})
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)final_smem(kFinalCapMax, R));
     return e;
 }
 
-template <int KPL>
-static void select_r(int R, dim3 grid, size_t smem, cudaStream_t st, const float *in_s,
-                     const int32_t *in_id, int64_t in_ld, int64_t nq, int64_t M, int seg, int nseg,
-                     int nprobe, int32_t *out_id, float *out_s, int64_t out_ld, const int *qlist,
-                     const int *qlist_n, const int *seg_cnt) {
-#define SIEVE_SELECT(RR)                                                                        \
-    k_select<KPL, RR><<<grid, kSelectWarps * 32, smem, st>>>(in_s, in_id, in_ld, nq, M, seg, nseg, \
-                                                             nprobe, out_id, out_s, out_ld, qlist, \
-                                                             qlist_n, seg_cnt)
-    switch (R) {
-        case 2: SIEVE_SELECT(2); break;
-        case 4: SIEVE_SELECT(4); break;
-        case 8: SIEVE_SELECT(8); break;
-        default: SIEVE_SELECT(16); break;
+cudaError_t prepare_rank_tc(int nprobe, int d) {
+    cudaError_t e = cudaSuccess;
+    for (auto f : {k_rank_tc<kRankGroupMax>, k_rank_tc<kRankStream>, k_rank_tc<kRankDense>})
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc_smem());
+    const int bulk = rank_bulk_stages(d);
+    for (auto f : {k_rank_bulk<kRankGroupMax>, k_rank_bulk<kRankStream>, k_rank_bulk<kRankDense>})
+        if (e == cudaSuccess && bulk)
+            e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)tcb::smem_bytes(bulk, kRankEpiBytes));
+    const int scr = rank_screen_stages(d);
+    if (e == cudaSuccess && scr)
+        e = cudaFuncSetAttribute(k_rank_screen, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)tcb::smem_bytes(scr, kRankEpiBytes, tcb::kStageBytesHi));
+    if (e == cudaSuccess) e = set_final_attr<2>();
+    if (e == cudaSuccess) e = set_final_attr<4>();
+    if (e == cudaSuccess) e = set_final_attr<8>();
+    if (e == cudaSuccess) e = set_final_attr<16>();
+    // the exact fallback for overflowing lists
+    if (e == cudaSuccess) e = prepare_rank(nprobe);
+    return e;
+}
+
+static void launch_final(const RankArgs &a, const RankPlan &L, int64_t n, int32_t *order,
+                         float *cscores, int *ovf, int *ovf_n, cudaStream_t st) {
+    const unsigned blocks = (unsigned)ceil_div(n, kSelectWarps);
+    if (L.mode == kRankDense && L.nranges == 1) {   // every score of a query in one list
+        const int kpl = std::max(4, pow2_at_least(ceil_div(L.cap, 32)));
+#define SIEVE_DENSE(KK, RR)                                                                      \
+    k_rank_dense_final<KK, RR><<<blocks, kSelectWarps * 32, dense_smem(KK, RR), st>>>(              \
+        a.list_s, a.list_n, n, a.cap, a.nprobe, order, cscores)
+#define SIEVE_DENSE_R(KK)                   \
+    switch (sort_regs(a.nprobe)) {          \
+        case 2: SIEVE_DENSE(KK, 2); break;  \
+        case 4: SIEVE_DENSE(KK, 4); break;  \
+        case 8: SIEVE_DENSE(KK, 8); break;  \
+        default: SIEVE_DENSE(KK, 16); break; \
     }
-#undef SIEVE_SELECT
-}
-
-// one selection level: the best nprobe of every segment of at most kSelectSeg
-// entries (nseg = 1: the final order).  qlist/qlist_n (nullable, device): only
-// the listed queries, on a grid of a few blocks per SM that strides over them.
-static void launch_select(const float *in_s, const int32_t *in_id, int64_t in_ld, int64_t nq,
-                          int64_t M, int nprobe, int32_t *out_id, float *out_s, int64_t out_ld,
-                          const int *qlist, const int *qlist_n, const int *seg_cnt, cudaStream_t st) {
-    const int seg = M < kSelectSeg ? (int)M : kSelectSeg;
-    const int nseg = (int)ceil_div(M, kSelectSeg);
-    const int R = sort_regs(nprobe);
-    int64_t blocks = ceil_div(nq * nseg, kSelectWarps);
-    if (qlist) blocks = std::min<int64_t>(blocks, 4 * (int64_t)num_sms());
-    const dim3 grid((unsigned)blocks);
-    const int kpl = std::max(4, pow2_at_least(ceil_div(seg, 32)));
-#define SIEVE_SEL_K(K)                                                                          \
-    select_r<K>(R, grid, select_smem(K, R), st, in_s, in_id, in_ld, nq, M, seg, nseg, nprobe,     \
-                out_id, out_s, out_ld, qlist, qlist_n, seg_cnt)
-    if (kpl <= 4)
-        SIEVE_SEL_K(4);
-    else if (kpl <= 16)
-        SIEVE_SEL_K(16);
-    else if (kpl <= 32)
-        SIEVE_SEL_K(32);
-    else
-        SIEVE_SEL_K(64);
-#undef SIEVE_SEL_K
-}
-
-static void launch_compact_final(const float *cand_s, const int32_t *cand_i, const int *seg_n,
-                                 int64_t nq, int nseg, int segcap, int nprobe, int32_t *order,
-                                 float *cscores, int *ovf_list, int *ovf_n, cudaStream_t st) {
-    const unsigned blocks = (unsigned)ceil_div(nq, kSelectWarps);
-    const int ccap = compact_cap(nprobe);
-#define SIEVE_COMPACT(RR)                                                                      \
-    k_compact_final<RR><<<blocks, kSelectWarps * 32, compact_smem(ccap, RR), st>>>(               \
-        cand_s, cand_i, seg_n, nq, nseg, segcap, nprobe, ccap, order, cscores, ovf_list, ovf_n)
-    switch (sort_regs(nprobe)) {
-        case 2: SIEVE_COMPACT(2); break;
-        case 4: SIEVE_COMPACT(4); break;
-        case 8: SIEVE_COMPACT(8); break;
-        default: SIEVE_COMPACT(16); break;
+        switch (kpl) {
+            case 4: SIEVE_DENSE_R(4); break;
+            case 8: SIEVE_DENSE_R(8); break;
+            case 16: SIEVE_DENSE_R(16); break;
+            case 32: SIEVE_DENSE_R(32); break;
+            default: SIEVE_DENSE_R(64); break;
+        }
+#undef SIEVE_DENSE_R
+#undef SIEVE_DENSE
+        return;
     }
-#undef SIEVE_COMPACT
+    const int kmax = L.ccap <= 128 ? 4 : L.ccap <= 512 ? 16 : L.ccap <= 1024 ? 32 : 64;
+#define SIEVE_FINAL(RR, KK)                                                                      \
+    k_rank_final<RR, KK><<<blocks, kSelectWarps * 32, final_smem(L.ccap, RR), st>>>(                \
+        a.list_s, a.list_i, a.list_n, a.list_edge, n, a.nranges, a.range_len, a.cap, a.nprobe,    \
+        L.ccap, order, cscores, ovf, ovf_n)
+#define SIEVE_FINAL_R(RR)                   \
+    switch (kmax) {                         \
+        case 4: SIEVE_FINAL(RR, 4); break;   \
+        case 16: SIEVE_FINAL(RR, 16); break; \
+        case 32: SIEVE_FINAL(RR, 32); break; \
+        default: SIEVE_FINAL(RR, 64); break; \
+    }
+    switch (sort_regs(a.nprobe)) {
+        case 2: SIEVE_FINAL_R(2); break;
+        case 4: SIEVE_FINAL_R(4); break;
+        case 8: SIEVE_FINAL_R(8); break;
+        default: SIEVE_FINAL_R(16); break;
+    }
+#undef SIEVE_FINAL_R
+#undef SIEVE_FINAL
 }
 
-int rank_tc_launches(int64_t nq, int64_t nlist, int nprobe, int d) {
+static void launch_threshold(const RankPlan &L, const float *gmax, int64_t n, int nprobe,
+                             const float *Q, int d, const unsigned *cmax, float *init_edge,
+                             cudaStream_t st) {
+    const unsigned blocks = (unsigned)ceil_div(n, kSelectWarps);
+    const int kpl = std::max(1, pow2_at_least(ceil_div(L.ng, 32)));
+#define SIEVE_THR(K)                                                                             \
+    k_rank_threshold<K><<<blocks, kSelectWarps * 32, 0, st>>>(gmax, L.gld, n, L.ng, nprobe, Q, d, \
+                                                              cmax, L.screen ? 1 : 0, init_edge)
+    switch (kpl) {
+        case 1: SIEVE_THR(1); break;
+        case 2: SIEVE_THR(2); break;
+        case 4: SIEVE_THR(4); break;
+        case 8: SIEVE_THR(8); break;
+        case 16: SIEVE_THR(16); break;
+        case 32: SIEVE_THR(32); break;
+        default: SIEVE_THR(64); break;
+    }
+#undef SIEVE_THR
+}
+
+// per chunk of queries: [the first pass and the threshold,] the final pass,
+// the final selection and the FP32 fallback; once per call the largest
+// centroid norm (the screen's bound)
+int rank_tc_launches(int64_t nq, int64_t nlist, int nprobe, int d, int64_t plan_nq,
+                     bool bulk) {
     if (nq <= 0) return 0;
-    int per;
-    if (use_two_pass(nlist, nprobe, d)) {
-        per = 5;   // maxima pass, threshold, keeping pass, final warps, FP32 fallback
-    } else {
-        per = 2;   // contraction, final selection level
-        if (use_group_threshold(nlist, nprobe)) per += 3;   // threshold, compaction, final warps
-        for (int64_t M = nlist; M > kSelectSeg; M = level_entries(M, nprobe)) ++per;
-    }
-    return (int)ceil_div(nq, rank_tc_chunk(nq, nlist, nprobe, d)) * per;
+    const RankPlan L = rank_plan(std::max(nq, plan_nq), nlist, nprobe, d, bulk);
+    const int chunks = (int)ceil_div(nq, L.chunk);
+    return chunks * (L.group ? 5 : 3) + (L.screen ? 1 : 0);
 }
 
-int rank_tc_mma_launches(int64_t nq, int64_t nlist, int nprobe, int d) {
+int rank_tc_mma_launches(int64_t nq, int64_t nlist, int nprobe, int d, int64_t plan_nq,
+                         bool bulk) {
     if (nq <= 0) return 0;
-    return (int)ceil_div(nq, rank_tc_chunk(nq, nlist, nprobe, d)) *
-           (use_two_pass(nlist, nprobe, d) ? 2 : 1);
+    const RankPlan L = rank_plan(std::max(nq, plan_nq), nlist, nprobe, d, bulk);
+    return (int)ceil_div(nq, L.chunk) * (L.group ? 2 : 1);
 }
 
 cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t nlist, int d,
                             int nprobe, int32_t *order, float *cscores, float *scratch, int *status,
-                            cudaStream_t st, const unsigned char *tc_cent, float *mma_ms) {
+                            cudaStream_t st, const unsigned char *tc_cent, float *mma_ms,
+                            int64_t plan_nq) {
+    if (nq <= 0) return cudaSuccess;
+    // the layout of the scratch follows the batch it was sized for; a part of
+    // that batch uses the same layout, so it never needs more
+    if (plan_nq < nq) plan_nq = nq;
     struct Events {   // mma_ms: a pair per contraction launch, destroyed on every return
         std::vector<cudaEvent_t> v;
         ~Events() {
@@ -916,109 +987,75 @@ cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t 
     } ev_hold;
     std::vector<cudaEvent_t> &evs = ev_hold.v;
     const int bulk_stages = tc_cent ? rank_bulk_stages(d) : 0;
-    const RankScratch L = rank_scratch(nlist, nprobe, d);
-    const int64_t chunk = rank_tc_chunk(nq, nlist, nprobe, d);
-    // carve the chunk's scratch (RankScratch's order, each part [chunk][...])
-    float *p = scratch;
-    float *table = p;
-    p += L.table ? chunk * L.ld : 0;
-    float *cand_s[2];
-    int32_t *cand_id[2];
-    for (int b = 0; b < 2; ++b) {
-        cand_s[b] = p;
-        cand_id[b] = reinterpret_cast<int32_t *>(p + chunk * L.lvl);
-        p += 2 * chunk * L.lvl;
+    const RankPlan L = rank_plan(plan_nq, nlist, nprobe, d, bulk_stages > 0);
+    const int screen_stages = L.screen ? rank_screen_stages(d) : 0;
+    // the chunk's scratch: lists (scores, ids), counts, final thresholds,
+    // overflow list, group maxima, starting thresholds; then the fixed part
+    const int64_t slots = L.chunk * L.nranges;
+    float *list_s = scratch;
+    int32_t *list_i = L.mode == kRankDense ? nullptr : reinterpret_cast<int32_t *>(list_s + slots * L.cap);
+    int *list_n = reinterpret_cast<int *>(list_s + slots * L.cap * (L.mode == kRankDense ? 1 : 2));
+    float *list_edge = reinterpret_cast<float *>(list_n + slots);
+    int *ovf = reinterpret_cast<int *>(list_edge + slots);
+    float *gmax = reinterpret_cast<float *>(ovf + L.chunk);
+    float *init_edge = gmax + (L.group ? L.chunk * L.gld : 0);
+    unsigned char *fixed = reinterpret_cast<unsigned char *>(scratch) + L.chunk * L.per_query();
+    int *ovf_n = reinterpret_cast<int *>(fixed);
+    unsigned *cmax = reinterpret_cast<unsigned *>(fixed + 4);
+    auto contract = [&](int mode, const RankArgs &a, int tiles, bool scr) {
+        if (mma_ms) {
+            evs.resize(evs.size() + 2);
+            cudaEventCreate(&evs[evs.size() - 2]);
+            cudaEventCreate(&evs.back());
+            cudaEventRecord(evs[evs.size() - 2], st);
+        }
+        const unsigned grid = (unsigned)std::min(tiles, num_sms());
+        const size_t bsm = tcb::smem_bytes(bulk_stages, kRankEpiBytes);
+        if (scr)
+            k_rank_screen<<<grid, tcb::kThreads,
+                            tcb::smem_bytes(screen_stages, kRankEpiBytes, tcb::kStageBytesHi), st>>>(
+                a, screen_stages);
+        else if (bulk_stages && mode == kRankGroupMax)
+            k_rank_bulk<kRankGroupMax><<<grid, tcb::kThreads, bsm, st>>>(a, bulk_stages);
+        else if (bulk_stages && mode == kRankStream)
+            k_rank_bulk<kRankStream><<<grid, tcb::kThreads, bsm, st>>>(a, bulk_stages);
+        else if (bulk_stages)
+            k_rank_bulk<kRankDense><<<grid, tcb::kThreads, bsm, st>>>(a, bulk_stages);
+        else if (mode == kRankGroupMax)
+            k_rank_tc<kRankGroupMax><<<grid, tcp::kThreads, tc_smem(), st>>>(a);
+        else if (mode == kRankStream)
+            k_rank_tc<kRankStream><<<grid, tcp::kThreads, tc_smem(), st>>>(a);
+        else
+            k_rank_tc<kRankDense><<<grid, tcp::kThreads, tc_smem(), st>>>(a);
+        if (mma_ms) cudaEventRecord(evs.back(), st);
+    };
+    if (L.screen) {
+        cudaError_t e = cudaMemsetAsync(cmax, 0, sizeof(unsigned), st);
+        if (e != cudaSuccess) return e;
+        const unsigned blocks = (unsigned)std::min<int64_t>(ceil_div(nlist, 8), 4 * (int64_t)num_sms());
+        k_cnorm_max<<<blocks, 256, 0, st>>>(C, nlist, d, cmax);
     }
-    float *gmax = p;
-    p += L.grouped ? chunk * L.gld : 0;
-    float *slot_s = p;
-    int32_t *slot_i = reinterpret_cast<int32_t *>(p + chunk * L.nseg * L.cap);
-    p += L.grouped ? 2 * chunk * L.nseg * L.cap : 0;
-    int *slot_n = reinterpret_cast<int *>(p);
-    uint32_t *lkey = reinterpret_cast<uint32_t *>(slot_n + (L.grouped ? chunk * round_up(L.nseg, 4) : 0));
-    int *ovf = reinterpret_cast<int *>(lkey + (L.grouped ? chunk : 0));   // [chunk] overflow list
-    int *ovf_n = reinterpret_cast<int *>(reinterpret_cast<unsigned char *>(scratch) +
-                                         chunk * L.per_query());       // its count
-    const int ng = (int)ceil_div(nlist, 32);
-    for (int64_t q0 = 0; q0 < nq; q0 += chunk) {
-        const int64_t n = nq - q0 < chunk ? nq - q0 : chunk;
-        const int tiles = (int)(ceil_div(n, tcp::kM) * ceil_div(nlist, kRankRange));
-        auto contract = [&](const RankArgs &a) {
-            if (mma_ms) {
-                evs.resize(evs.size() + 2);
-                cudaEventCreate(&evs[evs.size() - 2]);
-                cudaEventCreate(&evs.back());
-                cudaEventRecord(evs[evs.size() - 2], st);
-            }
-            if (bulk_stages)
-                k_rank_bulk<<<std::min(tiles, num_sms()), tcb::kThreads,
-                              tcb::smem_bytes(bulk_stages, 0), st>>>(a, bulk_stages);
-            else
-                k_rank_tc<<<std::min(tiles, num_sms()), tcp::kThreads, tc_smem(), st>>>(a);
-            if (mma_ms) cudaEventRecord(evs.back(), st);
-        };
-        RankArgs a{Q + q0 * d, n, C, nlist, d, table, L.ld, status, tc_cent,
-                   L.grouped ? gmax : nullptr, L.gld, L.table ? kRankTable : kRankMax,
-                   lkey, slot_s, slot_i, slot_n, (int)L.cap};
-        contract(a);
+    for (int64_t q0 = 0; q0 < nq; q0 += L.chunk) {
+        const int64_t n = nq - q0 < L.chunk ? nq - q0 : L.chunk;
+        const int tiles = (int)(ceil_div(n, tcp::kM) * L.nranges);
+        RankArgs a{Q + q0 * d, n, C, nlist, d, status, tc_cent, nprobe, L.nranges,
+                   L.range_len, L.cap, list_s, list_i, list_n, list_edge, nullptr, gmax, L.gld,
+                   L.group};
+        if (L.group) {   // the first pass: group maxima, then each query's starting threshold
+            contract(kRankGroupMax, a, tiles, L.screen);
+            launch_threshold(L, gmax, n, nprobe, Q + q0 * d, d, cmax, init_edge, st);
+            a.init_edge = init_edge;
+        }
+        contract(L.mode, a, tiles, false);
+        cudaError_t e = cudaMemsetAsync(ovf_n, 0, sizeof(int), st);
+        if (e != cudaSuccess) return e;
         int32_t *o = order + q0 * nprobe;
         float *cs = cscores ? cscores + q0 * nprobe : nullptr;
-        const int *qlist = nullptr, *qlist_n = nullptr;
-        if (L.grouped) {
-            const unsigned wblocks = (unsigned)ceil_div(n, kSelectWarps);
-            const int kpl = pow2_at_least(ceil_div(ng, 32));
-#define SIEVE_GTHR(K)                                                                              \
-    k_group_threshold<K><<<wblocks, kSelectWarps * 32, 0, st>>>(gmax, L.gld, n, ng, nprobe, lkey)
-            switch (kpl) {
-                case 1: SIEVE_GTHR(1); break;
-                case 2: SIEVE_GTHR(2); break;
-                case 4: SIEVE_GTHR(4); break;
-                case 8: SIEVE_GTHR(8); break;
-                case 16: SIEVE_GTHR(16); break;
-                case 32: SIEVE_GTHR(32); break;
-                default: SIEVE_GTHR(64); break;
-            }
-#undef SIEVE_GTHR
-            if (L.table) {
-                k_compact_seg<<<(unsigned)ceil_div(n * L.nseg, kSelectWarps), kSelectWarps * 32, 0,
-                                st>>>(table, L.ld, n, nlist, L.nseg, lkey, slot_s, slot_i, slot_n);
-            } else {
-                RankArgs keep = a;   // the second contraction keeps what reaches the threshold
-                keep.gmax = nullptr;
-                keep.mode = kRankKeep;
-                contract(keep);
-            }
-            cudaError_t e = cudaMemsetAsync(ovf_n, 0, sizeof(int), st);
-            if (e != cudaSuccess) return e;
-            launch_compact_final(slot_s, slot_i, slot_n, n, L.nseg, (int)L.cap, nprobe, o, cs, ovf,
-                                 ovf_n, st);
-            if (!L.table) {
-                // the queries whose kept slots overflowed: the FP32 ranking, exact
-                e = enqueue_rank(Q + q0 * d, n, C, nlist, d, nprobe, o, cs, st, ovf, ovf_n);
-                if (e != cudaSuccess) return e;
-                e = cudaGetLastError();
-                if (e != cudaSuccess) return e;
-                continue;
-            }
-            qlist = ovf;   // the levels below run only for the overflowing queries
-            qlist_n = ovf_n;
-        }
-        // levels over the score table until one segment is left
-        const float *in_s = table;
-        const int32_t *in_id = nullptr;
-        int64_t in_ld = L.ld, M = nlist;
-        int buf = 0;
-        while (M > kSelectSeg) {
-            launch_select(in_s, in_id, in_ld, n, M, nprobe, cand_id[buf], cand_s[buf], L.lvl, qlist,
-                          qlist_n, nullptr, st);
-            in_s = cand_s[buf];
-            in_id = cand_id[buf];
-            in_ld = L.lvl;
-            M = level_entries(M, nprobe);
-            buf ^= 1;
-        }
-        launch_select(in_s, in_id, in_ld, n, M, nprobe, o, cs, nprobe, qlist, qlist_n, nullptr, st);
-        cudaError_t e = cudaGetLastError();
+        launch_final(a, L, n, o, cs, ovf, ovf_n, st);
+        // the queries whose lists overflowed: the FP32 ranking, exact
+        e = enqueue_rank(Q + q0 * d, n, C, nlist, d, nprobe, o, cs, st, ovf, ovf_n);
+        if (e != cudaSuccess) return e;
+        e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
     if (mma_ms) {

@@ -39,7 +39,7 @@ struct SearchArgs {
     int tc_min;                         // groups chunks of >= tc_min items go to the
                                         // tensor cores; 0 = SIMT only
     int4 *active;                       // [nq]: query, first item, items
-    float *rank_scratch;                // score table of the tensor-core ranking
+    float *rank_scratch;                // candidate lists of the tensor-core ranking
     const unsigned char *tc_rows;       // tensor-core layout of the rows (nullable)
     const int64_t *tc_row_blocks;       // [nlist+1] block offsets of that layout
     const unsigned char *tc_cent;       // tensor-core layout of the centroids (nullable)
@@ -109,20 +109,27 @@ cudaError_t enqueue_rank(const float *Q, int64_t nq, const float *C, int64_t nli
                          int nprobe, int32_t *order, float *cscores, cudaStream_t st,
                          const int *qlist = nullptr, const int *qlist_n = nullptr);
 
-// centroid ranking on the tensor cores (rank_tc.cu): a score table of at most
-// kRankScratchBytes per chunk of queries, then warp-per-segment selections
-constexpr int64_t kRankScratchBytes = int64_t(2) << 30;
+// centroid ranking on the tensor cores (rank_tc.cu): one contraction pass with
+// a streaming threshold per query, candidate lists of at most
+// kRankScratchBytes per chunk of queries, then a warp-per-query selection
+constexpr int64_t kRankScratchBytes = int64_t(4) << 30;
 bool rank_tc_supported(int64_t nlist, int nprobe);
 size_t rank_tc_scratch_bytes(int64_t nq, int64_t nlist, int nprobe, int d);
-int rank_tc_launches(int64_t nq, int64_t nlist, int nprobe, int d);   // kernel launches of one ranking
+// kernel launches of one ranking (plan_nq as for enqueue_rank_tc; bulk: the
+// centroids' tensor-core layout is given and rank_bulk_stages(d) > 0)
+int rank_tc_launches(int64_t nq, int64_t nlist, int nprobe, int d, int64_t plan_nq, bool bulk);
 cudaError_t prepare_rank_tc(int nprobe, int d);
 // mma_ms (nullable): the contraction launches are bracketed by events, the
-// call synchronizes st and adds their summed time (ms) to *mma_ms
+// call synchronizes st and adds their summed time (ms) to *mma_ms.
+// plan_nq: the query count scratch was sized for (rank_tc_scratch_bytes), when
+// these nq queries are a part of that batch; 0 = nq
 cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t nlist, int d,
                             int nprobe, int32_t *order, float *cscores, float *scratch, int *status,
                             cudaStream_t st, const unsigned char *tc_cent = nullptr,
-                            float *mma_ms = nullptr);
-int rank_tc_mma_launches(int64_t nq, int64_t nlist, int nprobe, int d);   // contraction launches
+                            float *mma_ms = nullptr, int64_t plan_nq = 0);
+int rank_tc_mma_launches(int64_t nq, int64_t nlist, int nprobe, int d, int64_t plan_nq,
+                         bool bulk);   // contraction launches
+int rank_screen_stages(int d);                   // 0 when the screening first pass does not apply
 int rank_bulk_stages(int d);                     // 0 when the bulk ranking does not apply
 
 // in-call window calibration (calibrate.cu)

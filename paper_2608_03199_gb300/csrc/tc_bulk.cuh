@@ -11,8 +11,10 @@
 // per 32-bit column, hi and lo of each K-block side by side), so shared memory
 // holds nothing but B stages and the epilogue's lists.
 //
-// Tensor memory (512 columns): two 128-column fp32 accumulators, then the
-// tile's A: 64 columns per K-block of 64 elements (32 hi, 32 lo); d <= 256.
+// Tensor memory (512 columns): two 128-column fp32 accumulators (three when
+// d <= 128), then the tile's A: 64 columns per K-block of 64 elements (32 hi,
+// 32 lo); d <= 256.  K steps of 16 that lie wholly in the zero padding of the
+// last K-block are not issued (d = 96: six of eight).
 // A screening mode (one product per K step, hi halves only) copies just the
 // hi half of each K-block of B and keeps only A's hi columns (32 per
 // K-block), so three accumulators fit.
@@ -132,10 +134,8 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
     // bytes of one K-block of B in global memory: a screen copies the hi half
     // of each K-block of the split layout, one copy per K-block
     constexpr uint32_t kSrcKb = b_has_lo<Mode>::value ? kKbBytes : kKbBytesHi;
-    // accumulators and A's tensor-memory columns per K-block: with hi and lo
-    // of A (64 columns per K-block) two 128-column accumulators fit beside it;
-    // a screen keeps only A's hi half (32 columns), which leaves room for three
-    constexpr uint32_t kAcc = kProd == 1 ? 3 : 2;
+    // A's tensor-memory columns per K-block: hi and lo (64), or a screen's hi
+    // half alone (32)
     constexpr uint32_t kAKb = kProd == 1 ? 32 : 64;
     constexpr int kKs = kKbPerStage;                          // K-blocks per B stage
     constexpr uint32_t kStage = kKs * kKbB;                    // bytes of one B stage
@@ -152,6 +152,9 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
     const int n_tiles = Mode::num_tiles(a);
     const int d = Mode::d(a);
     const int nkb = (int)ceil_div(d, 64);
+    // 128-column accumulators beside A: three when A takes at most 128
+    // columns (a screen, or d <= 128), two otherwise (512 columns in all)
+    const uint32_t nacc = (kProd == 1 || nkb <= 2) ? 3u : 2u;
     unsigned char *Bst = base;                                 // stages x kStage
     unsigned char *epi_smem = Bst + (size_t)stages * kStage;
     int *status = Mode::status(a);
@@ -166,7 +169,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
             tc::mbar_init(&b_full[s], 1);
             tc::mbar_init(&b_empty[s], 1);
         }
-        for (uint32_t b = 0; b < kAcc; ++b) {
+        for (uint32_t b = 0; b < (uint32_t)kMaxAcc; ++b) {
             tc::mbar_init(&dfull_bar[b], 1);
             tc::mbar_init(&dempty_bar[b], 4 * 32);
         }
@@ -183,7 +186,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
     __syncthreads();
     tc::fence_after_sync();
     const uint32_t tmem = tmem_slot;
-    const uint32_t tA = tmem + kAcc * kN;                      // A after the accumulators
+    const uint32_t tA = tmem + nacc * kN;                      // A after the accumulators
 
     auto wait = [&](uint64_t *bar, uint32_t parity) -> bool {
         for (uint32_t it = 0; it < kWaitPolls; ++it) {
@@ -301,7 +304,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                 const int nch = (int)ceil_div(T.nb, kN);
                 if (nch == 0) continue;
                 for (int ch = 0; ok && ch < nch; ++ch, ++c) {
-                    const uint32_t buf = c % kAcc, dph = (c / kAcc) & 1u;
+                    const uint32_t buf = c % nacc, dph = (c / nacc) & 1u;
                     if (!(ok = wait(&dempty_bar[buf], dph ^ 1u))) break;
                     tc::fence_after_sync();
                     const uint32_t dt = tmem + buf * kN;
@@ -313,6 +316,9 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                         if (!ok || !(ok = wait(&b_full[st], ph))) break;
                         tc::fence_after_sync();
                         for (int kb = kb0; kb < kb1; ++kb) {
+                            // K steps of 16 that hold any of the d elements: the
+                            // rest of the last K-block is zero padding
+                            const int kst = d - kb * 64 >= 64 ? 4 : (d - kb * 64 + 15) / 16;
                             const uint32_t a_hi = tA + (uint32_t)kb * kAKb, a_lo = a_hi + 32;
                             const uint32_t b_hi = tc::smem_u32(Bst + (size_t)st * kStage) +
                                                   (uint32_t)(kb - kb0) * kKbB;
@@ -324,6 +330,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                                 const uint64_t bl = tc::desc_k_sw128(b_hi + kKbBytes / 2);
 #pragma unroll
                                 for (int ks = 0; ks < 4; ++ks) {   // K = 16: 8 columns of A, 32 bytes of B
+                                    if (ks >= kst) break;
                                     const uint32_t ao = ks * 8;
                                     const uint64_t bo = 2 * ks;
                                     tc::mma_f16_ta(dt, a_lo + ao, bh + bo, kIdesc, (kb > 0 || ks > 0) ? 1u : 0u);
@@ -333,6 +340,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                             } else if constexpr (kProd == 2) {   // B exact in fp16: hi and lo of A against it
 #pragma unroll
                                 for (int ks = 0; ks < 4; ++ks) {
+                                    if (ks >= kst) break;
                                     const uint32_t ao = ks * 8;
                                     const uint64_t bo = 2 * ks;
                                     tc::mma_f16_ta(dt, a_lo + ao, bh + bo, kIdesc, (kb > 0 || ks > 0) ? 1u : 0u);
@@ -341,8 +349,9 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                             } else {   // a screen: the hi halves alone
 #pragma unroll
                                 for (int ks = 0; ks < 4; ++ks)
-                                    tc::mma_f16_ta(dt, a_hi + ks * 8, bh + 2 * ks, kIdesc,
-                                                   (kb > 0 || ks > 0) ? 1u : 0u);
+                                    if (ks < kst)
+                                        tc::mma_f16_ta(dt, a_hi + ks * 8, bh + 2 * ks, kIdesc,
+                                                       (kb > 0 || ks > 0) ? 1u : 0u);
                             }
                         }
                         tc::mma_commit(&b_empty[st]);
@@ -374,7 +383,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
             const int nch = (int)ceil_div(T.nb, kN);
             epi.begin(a, T, slot, epi_smem);
             for (int ch = 0; ch < nch; ++ch, ++c) {
-                const uint32_t buf = c % kAcc, dph = (c / kAcc) & 1u;
+                const uint32_t buf = c % nacc, dph = (c / nacc) & 1u;
                 epi.prefetch(a, T, ch);   // per-chunk loads, in flight during the wait
                 ok = __all_sync(0xffffffffu, wait(&dfull_bar[buf], dph));
                 if (!ok) break;

@@ -210,8 +210,11 @@ __device__ __forceinline__ void run_pipeline(const typename Mode::Args &a, unsig
                         const uint32_t sa = tc::smem_u32(base + st * G::STAGE_BYTES);
                         const uint32_t a_hi = sa, a_lo = sa + A_BYTES;
                         const uint32_t b_hi = sa + 2 * A_BYTES, b_lo = b_hi + G::B_BYTES;
+                        // K steps holding any of the d elements (the rest is zero padding)
+                        const int kst = d - kb * kKB >= kKB ? kKB / 16 : (d - kb * kKB + 15) / 16;
 #pragma unroll
                         for (int ks = 0; ks < kKB / 16; ++ks) {   // K = 16 fp16 = 32 bytes per MMA
+                            if (ks >= kst) break;
                             const uint32_t o = ks * 32;
                             tc::mma_f16(dt, tc::desc_k_sw128(a_lo + o), tc::desc_k_sw128(b_hi + o),
                                         kIdesc, (kb > 0 || ks > 0) ? 1u : 0u);
