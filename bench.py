@@ -190,24 +190,25 @@ def committed_traffic(kernel, workload, launches):
     return e["dram_bytes_per_search"] / max(1, launches)
 
 
-def uses_screen(args, cfg, W, bulk):
+def uses_screen(args, cfg, W, bulk, tau=None):
     """Whether the bulk scan screens (sieve_params.scan_path; the automatic
-    path screens from a window of 16 up)."""
+    path screens from a window of 16 up when tau >= 0.85)."""
+    tau = cfg.tau if tau is None else tau
     return bulk and (args.scan_path == "screen" or
-                     (args.scan_path == "auto" and min(W, cfg.nprobe) >= 16))
+                     (args.scan_path == "auto" and min(W, cfg.nprobe) >= 16 and tau >= 0.85))
 
 
 def rank_passes(cfg, bulk):
     """(contraction passes of the tensor-core ranking, products per score of
-    the first pass): more than 2,048 centroids with 2 nprobe to 2,048 groups of
-    64 (or 32) take a first pass of group maxima, on the screen (one product)
-    with the tensor-core layout (d <= 256), else with three products."""
-    if cfg.nlist <= 2048:
+    the first pass): with the tensor-core layout (d <= 256), more than 2,048
+    centroids and 2 nprobe to 2,048 groups of 64 (or 32), a first pass of
+    group maxima on the screen (one product per score); else one pass."""
+    if cfg.nlist <= 2048 or not bulk or cfg.d > 256:
         return 1, 0
     for g in (64, 32):
         ng = -(-cfg.nlist // g)
         if 2 * cfg.nprobe <= ng <= 2048:
-            return 2, (1 if bulk and cfg.d <= 256 else 3)
+            return 2, 1
     return 1, 0
 
 
@@ -417,22 +418,31 @@ def cpu_baseline(w, cfg, target_s, gpu_w=None, gpu_fixed=None):
     import oracle
     idx = {k: w[k] for k in ("X", "ids", "assign", "centroids")}
     threads = oracle.default_threads()
-    probe = min(cfg.nq, 64)
-    t0 = time.perf_counter()
-    oracle.search(idx, w["Q"][:probe], cfg.tau, cfg.k, cfg.nprobe, cfg.W, qids=w["qids"][:probe],
-                  threads=threads)
-    per_q = (time.perf_counter() - t0) / probe
-    sample = int(min(cfg.nq, max(probe, target_s / max(per_q, 1e-9))))
+
+    def sized(W, budget, least):
+        """Queries that fill the budget: two probe calls separate a call's
+        fixed cost (the oracle builds its partition lists from the rows) from
+        the cost per query."""
+        lo = min(cfg.nq, 64)
+        hi = min(cfg.nq, 4 * lo)
+        ts = []
+        for m in (lo, hi):
+            t0 = time.perf_counter()
+            oracle.search(idx, w["Q"][:m], cfg.tau, cfg.k, cfg.nprobe, W, qids=w["qids"][:m],
+                          threads=threads)
+            ts.append(time.perf_counter() - t0)
+        per_q = max((ts[1] - ts[0]) / max(1, hi - lo), ts[1] / hi * 0.05, 1e-9)
+        fixed = max(0.0, ts[0] - lo * per_q)
+        return int(min(cfg.nq, max(least, (budget - fixed) / per_q)))
+
+    # at the workload's window: at least 10,000 queries (the whole batch when smaller)
+    sample = sized(cfg.W, target_s, min(cfg.nq, 10_000))
     t0 = time.perf_counter()
     ref = oracle.search(idx, w["Q"][:sample], cfg.tau, cfg.k, cfg.nprobe, cfg.W,
                         qids=w["qids"][:sample], threads=threads)
     dt = time.perf_counter() - t0
     # fixed probing (W = nprobe) on a smaller sample: a third of the time budget
-    t0 = time.perf_counter()
-    oracle.search(idx, w["Q"][:probe], cfg.tau, cfg.k, cfg.nprobe, cfg.nprobe,
-                  qids=w["qids"][:probe], threads=threads)
-    per_q = (time.perf_counter() - t0) / probe
-    fsample = int(min(cfg.nq, max(probe, target_s / 3 / max(per_q, 1e-9))))
+    fsample = sized(cfg.nprobe, target_s / 3, min(cfg.nq, 64))
     t0 = time.perf_counter()
     fref = oracle.search(idx, w["Q"][:fsample], cfg.tau, cfg.k, cfg.nprobe, cfg.nprobe,
                          qids=w["qids"][:fsample], threads=threads)
@@ -709,8 +719,9 @@ def run_sweep(args, cfg):
     JSON line per setting with the time per call, queries/s, mean probes and
     the pooled recall of the kept neighbours against fixed probing (the same
     index, tau, k and nprobe).  Varied one at a time from the workload's own
-    setting: W with lookahead on and off (serial traversal issues one rank
-    per query per round), tau, k, nprobe, and the batch size."""
+    setting: W under the three schedules of the execution ablation (serial
+    traversal, continuous batching, continuous batching with lookahead), tau
+    from 0.10 to 0.95, k, nprobe, and the batch size."""
     import paper_2608_03199_gb300 as sieve
     dev = torch.device("cuda:0")
     sieve.lib()
@@ -719,13 +730,15 @@ def run_sweep(args, cfg):
     Q, qids = wl["Q"], wl["qids"]
     ws = sieve.Workspace()
 
-    def timed(nq, tau, k, nprobe, W, lookahead):
+    def timed(nq, tau, k, nprobe, W, lookahead, serial=False):
         run = lambda: sieve.search(index, Q[:nq], tau, k, nprobe, W, lookahead=lookahead,
-                                   query_ids=qids[:nq], workspace=ws)
+                                   query_ids=qids[:nq], workspace=ws, serial=serial)
         for _ in range(2):
             out = run()
         torch.cuda.synchronize()
         reps = max(3, min(50, int(2e5 // max(nq, 1))))
+        if serial:
+            reps = 3
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record()
         for _ in range(reps):
@@ -742,10 +755,14 @@ def run_sweep(args, cfg):
         return kept / tot if tot else 1.0
 
     settings = []
+    # the execution ablation of Sec. 6.3: serial traversal (every (query, rank)
+    # its own partition call), continuous batching (one rank per query per
+    # round, regrouped by partition), and continuous batching with lookahead
     for W in (cfg.sweep_W or (2, 4, 8, 16, cfg.nprobe)):
-        for la in (True, False):
-            settings.append(("W", cfg.nq, cfg.tau, cfg.k, cfg.nprobe, W, la))
-    for tau in (0.85, 0.90, 0.95):
+        for la, ser in ((False, True), (False, False), (True, False)):
+            settings.append(("W", cfg.nq, cfg.tau, cfg.k, cfg.nprobe, W, la, ser))
+    # threshold selectivity (Sec. 6.4): loose thresholds make most probes hit
+    for tau in (0.10, 0.30, 0.50, 0.70, 0.85, 0.90, 0.95):
         settings.append(("tau", cfg.nq, tau, cfg.k, cfg.nprobe, cfg.W, True))
     for k in (5, 10, 20, 50):
         settings.append(("k", cfg.nq, cfg.tau, k, cfg.nprobe, cfg.W, True))
@@ -755,14 +772,19 @@ def run_sweep(args, cfg):
         if nq <= cfg.nq:
             settings.append(("batch", nq, cfg.tau, cfg.k, cfg.nprobe, cfg.W, True))
     fixed_cache = {}
-    for (axis, nq, tau, k, nprobe, W, la) in settings:
+    for setting in settings:
+        axis, nq, tau, k, nprobe, W, la = setting[:7]
+        ser = setting[7] if len(setting) > 7 else False
         key = (nq, tau, k, nprobe)
         if key not in fixed_cache:
             fixed_cache[key] = timed(nq, tau, k, nprobe, nprobe, True)
         ref, ms_fixed = fixed_cache[key]
-        out, ms = timed(nq, tau, k, nprobe, W, la)
+        out, ms = timed(nq, tau, k, nprobe, W, la, ser)
+        schedule = ("serial traversal" if ser else
+                    "continuous batching + lookahead" if la else "continuous batching")
         print(json.dumps({"sweep": axis, "nq": nq, "tau": tau, "k": k, "nprobe": nprobe, "W": W,
-                          "lookahead": la, "ms": round(ms, 4), "queries_per_s": round(nq / (ms * 1e-3)),
+                          "lookahead": la, "schedule": schedule, "ms": round(ms, 4),
+                          "queries_per_s": round(nq / (ms * 1e-3)),
                           "fixed_ms": round(ms_fixed, 4), "speedup_vs_fixed": round(ms_fixed / ms, 3),
                           "mean_probes": round(float(out[3].float().mean()), 3),
                           "recall_vs_fixed": round(recall(out, ref), 5)}), flush=True)

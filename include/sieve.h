@@ -88,6 +88,20 @@ typedef struct {
  *   W          consecutive-empty window, >= 1; W >= nprobe is fixed probing
  *   lookahead  0 = continuous batching (one rank per query per round,
  *              Algorithm 1), 1 = issue every committed rank (Algorithm 2)
+ *   serial     0 = regroup the ready items by partition every round, up to
+ *              128 items per tile (continuous batching, Sec. 4.2); 1 = the
+ *              serial traversal of the execution ablation (Sec. 6.3): every
+ *              (query, rank) item is its own partition call, one query
+ *              against the partition's rows, with the same stopping rule and
+ *              the same results; a baseline for measurement
+ *   wait_limit iteration limit of one device wait: the tensor-core scan
+ *              epilogue's wait for an accumulator (a wait with no
+ *              asynchronous work of its own outstanding); 0 = the default,
+ *              2^24 polls.  A testing aid for the bounded waits: a wait that
+ *              gives up records SIEVE_ETIMEOUT in the call's status word,
+ *              the kernel lets every copy and MMA it issued land (those
+ *              waits keep their full limit), frees its tensor memory and
+ *              returns; the search stops and reports SIEVE_ETIMEOUT.
  *   max_items_per_round  cap on (query, rank) items issued in one round;
  *              0 = automatic.  Only splits work into more rounds: the result
  *              does not depend on it (Sec. 4.2).
@@ -104,7 +118,8 @@ typedef struct {
  *              tensor cores when the epilogue's k-lists fit: any k with
  *              the tensor-core layout and d <= 256, k <= 22 otherwise; FP32
  *              FMA beyond; with the tensor-core layout the screen below
- *              when min(W, nprobe) >= 16, three products per pair under it),
+ *              when min(W, nprobe) >= 16 and tau >= 0.85, three products
+ *              per pair otherwise),
  *              1 = FP32 FMA only, 2 = tensor cores, three products per pair
  *              (SIEVE_EINVAL where they do not fit), 3 = as 2, but with the
  *              tensor-core layout every pair is screened.
@@ -124,6 +139,8 @@ typedef struct {
     int32_t loop;
     int32_t profile;
     int32_t scan_path;
+    int32_t serial;
+    int32_t wait_limit;
     int64_t max_items_per_round;
 } sieve_params;
 

@@ -51,7 +51,8 @@ class IndexViewC(C.Structure):
 class ParamsC(C.Structure):
     _fields_ = [("tau", C.c_float), ("k", C.c_int32), ("nprobe", C.c_int32), ("W", C.c_int32),
                 ("lookahead", C.c_int32), ("loop", C.c_int32), ("profile", C.c_int32),
-                ("scan_path", C.c_int32), ("max_items_per_round", C.c_int64)]
+                ("scan_path", C.c_int32), ("serial", C.c_int32), ("wait_limit", C.c_int32),
+                ("max_items_per_round", C.c_int64)]
 
 
 class StatsC(C.Structure):
@@ -301,8 +302,11 @@ def rank_partitions(index: Index, Q, nprobe, return_scores=False, stream=None):
     return (order, sc) if return_scores else order
 
 
-def _params(tau, k, nprobe, W, lookahead, loop, max_items_per_round, profile=0, scan_path="auto"):
+def _params(tau, k, nprobe, W, lookahead, loop, max_items_per_round, profile=0, scan_path="auto",
+            serial=False, wait_limit=0):
     p = ParamsC()
+    p.serial = 1 if serial else 0
+    p.wait_limit = int(wait_limit)
     p.profile = int(profile)
     p.scan_path = SCAN_PATHS[scan_path] if isinstance(scan_path, str) else int(scan_path)
     p.tau = float(tau)
@@ -357,7 +361,7 @@ def _stats_dict(st):
 
 def search(index: Index, Q, tau, k, nprobe, W, lookahead=True, query_ids=None, order=None,
            max_items_per_round=0, loop=0, stats=False, profile=False, scan_path="auto",
-           workspace=None, out=None, stream=None, check=False):
+           workspace=None, out=None, stream=None, check=False, serial=False, wait_limit=0):
     """SieveIVF search on device tensors (sieve_search).
 
     Returns (ids [nq][k] i64, scores [nq][k] f32, count [nq] i32, probes [nq] i32),
@@ -365,7 +369,9 @@ def search(index: Index, Q, tau, k, nprobe, W, lookahead=True, query_ids=None, o
     stream; ``profile`` also times every kernel launch with CUDA events).
     ``check``: read the device status word after the call
     (sieve_search_status, which synchronizes the stream) and raise on a
-    device-side error; stats and host-driven rounds check it anyway."""
+    device-side error; stats and host-driven rounds check it anyway.
+    ``serial``: the serial traversal (every (query, rank) item its own
+    partition call; the same results)."""
     stats = stats or profile
     _need_cuda(Q, torch.float32, "Q", 2)
     if query_ids is not None:
@@ -374,7 +380,8 @@ def search(index: Index, Q, tau, k, nprobe, W, lookahead=True, query_ids=None, o
         _need_cuda(order, torch.int32, "order", 2)
     nq = Q.shape[0]
     dev = Q.device
-    p = _params(tau, k, nprobe, W, lookahead, loop, max_items_per_round, profile, scan_path)
+    p = _params(tau, k, nprobe, W, lookahead, loop, max_items_per_round, profile, scan_path, serial,
+                wait_limit)
     v = index.view()
     nbytes = C.c_size_t()
     _check(lib().sieve_search_workspace_size(C.byref(v), nq, C.byref(p), 0, C.byref(nbytes)),

@@ -64,10 +64,14 @@ sieve_status check_params(const sieve_index_view *ix, const sieve_params *p) {
     if (p->max_items_per_round < 0) return SIEVE_EINVAL;
     if (p->profile != 0 && p->profile != 1) return SIEVE_EINVAL;
     if (p->scan_path < 0 || p->scan_path > 3) return SIEVE_EINVAL;
+    if (p->serial != 0 && p->serial != 1) return SIEVE_EINVAL;
+    if (p->wait_limit < 0) return SIEVE_EINVAL;
     return SIEVE_OK;
 }
 
-constexpr int kScreenMinWindow = 16;   // automatic scan path: the screen from this window up
+constexpr int kScreenMinWindow = 16;   // automatic scan path: the screen from this window up ...
+constexpr float kScreenMinTau = 0.85f; // ... and this threshold up (below it nearly every row
+                                       // of a probed partition needs its fp32 rescore)
 constexpr int64_t kAutoCapMax = int64_t(1) << 24;
 constexpr int64_t kCapMax = int64_t(1) << 30;
 
@@ -103,8 +107,10 @@ Layout make_layout(const sieve_index_view *ix, int64_t nq, const sieve_params *p
     const int64_t cap = items_cap(nq, p);
     // SIMT tiles: at most one per QT items plus one per partial chunk; tensor-core
     // tiles: at most one per kTcTile items plus one per partition
-    const int64_t max_tiles = ceil_div(cap, QT) + ceil_div(cap, kTcTile) + ix->nlist + 1;
-    const int64_t max_tc_tiles = ceil_div(cap, kTcTile) + ix->nlist + 1;
+    // (serial traversal: one tile per item)
+    const int64_t max_tiles = p->serial ? cap + 1
+                                        : ceil_div(cap, QT) + ceil_div(cap, kTcTile) + ix->nlist + 1;
+    const int64_t max_tc_tiles = p->serial ? cap + 1 : ceil_div(cap, kTcTile) + ix->nlist + 1;
     L.cap = cap;
     L.max_tiles = max_tiles;
     L.ctl = take(sizeof(Ctl));
@@ -361,6 +367,8 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
     a.nprobe = p->nprobe;
     a.W = p->W;
     a.lookahead = p->lookahead;
+    a.serial = p->serial;
+    a.wait_limit = p->wait_limit;
     a.cap = L.cap;
     a.max_rounds = (int)std::min<int64_t>(INT32_MAX, p->nprobe + ceil_div(nq * p->nprobe, L.cap) + 2);
     a.S = reinterpret_cast<int *>(ws + L.S);
@@ -390,7 +398,8 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
     // the screen.
     const bool with_layout = a.tc_rows && a.tc_row_blocks;
     const bool screen = with_layout && (p->scan_path == 3 ||
-                                        (p->scan_path == 0 && std::min(p->W, p->nprobe) >= kScreenMinWindow));
+                                        (p->scan_path == 0 && std::min(p->W, p->nprobe) >= kScreenMinWindow &&
+                                         p->tau >= kScreenMinTau));
     const int bulk_stages = !with_layout ? 0
                             : screen    ? scan_screen_stages(ix->d, p->k)
                                         : scan_bulk_stages(ix->d, p->k);

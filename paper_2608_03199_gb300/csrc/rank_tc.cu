@@ -765,10 +765,10 @@ constexpr int kMaxGroups = 2048;     // group maxima one threshold warp holds (6
 
 // How one ranking call is cut up.
 //  kind: nlist <= 2,048: one pass keeping every score (dense lists, ids
-//    implicit).  Else, when there are at least 2 nprobe groups of 64 (or 32)
-//    centroids and at most 2,048 of them: two passes -- group maxima (on the
-//    screen when the bulk pipeline applies), a per-query threshold, and the
-//    streaming pass from that threshold.  Else the streaming pass alone.
+//    implicit).  Else, on the bulk pipeline with at least 2 nprobe groups of
+//    64 (or 32) centroids and at most 2,048 of them: two passes -- group
+//    maxima on the screen, a per-query threshold, and the streaming pass
+//    from that threshold.  Else the streaming pass alone.
 //  ranges: enough (query tile, range) tiles for about four waves of the
 //    persistent contraction; the streaming pass alone takes at most
 //    2,048 / 2P ranges (each keeps P plus a bin's width of candidates);
@@ -805,7 +805,11 @@ static RankPlan rank_plan(int64_t nq, int64_t nlist, int nprobe, int d, bool bul
         L.mode = kRankDense;
     } else {
         L.mode = kRankStream;
+        // a first pass pays off on the screen (a third of the products and
+        // half the operand bytes); without the bulk pipeline it would cost a
+        // full second contraction
         for (int g : {64, 32}) {
+            if (!bulk || rank_screen_stages(d) == 0) break;
             const int64_t ng = ceil_div(nlist, g);
             if (ng >= 2 * (int64_t)nprobe && ng <= kMaxGroups) {
                 L.group = g;

@@ -37,6 +37,7 @@ struct ScanModeT {
     __device__ static int *tile_counter(const Args &a) { return &a.ctl->tc_tile_next; }
     __device__ static int d(const Args &a) { return a.d; }
     __device__ static int *status(const Args &a) { return &a.ctl->status; }
+    __device__ static uint32_t epi_wait_polls(const Args &a) { return (uint32_t)a.wait_limit; }
     __device__ static Tile tile(const Args &a, int t) {
         const int4 x = a.tc_tiles[t];
         Tile T;
@@ -374,6 +375,8 @@ struct ScanModeT {
         }
     };
 };
+static_assert(tcb::has_epi_wait<ScanModeT<false>>::value && tcb::has_epi_wait<ScanModeT<false, true>>::value,
+              "the scan's epilogue wait takes the search's wait_limit");
 
 using ScanMode = ScanModeT<false>;
 using ScanModeRQ = ScanModeT<true>;

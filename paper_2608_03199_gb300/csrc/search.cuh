@@ -25,6 +25,8 @@ struct SearchArgs {
     // parameters
     float tau;
     int k, nprobe, W, lookahead;
+    int serial;                // 1: every (query, rank) item is its own tile (serial traversal)
+    int wait_limit;            // polls of the tensor-core scan epilogue's accumulator wait (0: default)
     int64_t cap;               // items per round
     int max_rounds;
     // per-query state: stop line S (Sec. 4.3) and enqueue cursor E (first

@@ -157,9 +157,14 @@ constexpr int kBucketThreads = 1024;
 // A group of c items is cut into chunks of up to kTcTile; a chunk with at
 // least tc_min items is one tensor-core tile, a smaller one is cut into SIMT
 // tiles of up to QT items.
-__device__ __forceinline__ void count_tiles(int c, int tc_min, int &n_tc, int &n_simt) {
+__device__ __forceinline__ void count_tiles(int c, int tc_min, int serial, int &n_tc, int &n_simt) {
     n_tc = 0;
     n_simt = 0;
+    if (serial) {   // serial traversal: one tile per item, no regrouping across queries
+        if (tc_min > 0) n_tc = c;
+        else n_simt = c;
+        return;
+    }
     for (int o = 0; o < c; o += kTcTile) {
         const int sz = c - o < kTcTile ? c - o : kTcTile;
         if (tc_min > 0 && sz >= tc_min)
@@ -193,7 +198,7 @@ __global__ void __launch_bounds__(kBucketThreads) k_bucket(SearchArgs a) {
     for (int64_t p = p0; p < p0 + per && p < nl; ++p) {
         const int c = a.counts[p];
         int ntc, ns;
-        count_tiles(c, a.tc_min, ntc, ns);
+        count_tiles(c, a.tc_min, a.serial, ntc, ns);
         my[0] += c;
         my[1] += ns;
         my[2] += ntc;
@@ -238,8 +243,19 @@ __global__ void __launch_bounds__(kBucketThreads) k_bucket(SearchArgs a) {
         const int c = a.counts[p];
         a.cursor[p] = ioff;
         int ntc, ns;
-        count_tiles(c, a.tc_min, ntc, ns);
+        count_tiles(c, a.tc_min, a.serial, ntc, ns);
         int toff = ntc ? atomicAdd(&cls[tile_class(a, p)], ntc) : 0;
+        if (a.serial) {   // one tile per item
+            for (int o = 0; o < c; ++o) {
+                if (a.tc_min > 0)
+                    a.tc_tiles[toff++] = make_int4((int)p, ioff + o, 1, 0);
+                else
+                    a.tiles[soff++] = make_int4((int)p, ioff + o, 1, 0);
+            }
+            ioff += c;
+            a.counts[p] = 0;
+            continue;
+        }
         for (int o = 0; o < c; o += kTcTile) {
             const int sz = c - o < kTcTile ? c - o : kTcTile;
             if (a.tc_min > 0 && sz >= a.tc_min) {

@@ -107,6 +107,25 @@ struct mma_products { static constexpr int value = b_has_lo<Mode>::value ? 3 : 2
 template <class Mode>
 struct mma_products<Mode, decltype((void)Mode::kProducts)> { static constexpr int value = Mode::kProducts; };
 
+// polls of the epilogue's accumulator wait: the mode's epi_wait_polls(a) if
+// it has one (a testing aid that lets that wait give up early; 0 = default),
+// else kWaitPolls.  No other wait takes it: every drain keeps the full limit.
+template <class Mode, class = void>
+struct has_epi_wait { static constexpr bool value = false; };
+template <class Mode>
+struct has_epi_wait<Mode, decltype((void)Mode::epi_wait_polls(*(const typename Mode::Args *)nullptr))> {
+    static constexpr bool value = true;
+};
+template <class Mode>
+__device__ __forceinline__ uint32_t epi_wait_polls(const typename Mode::Args &a) {
+    if constexpr (has_epi_wait<Mode>::value) {
+        const uint32_t n = Mode::epi_wait_polls(a);
+        return n ? n : kWaitPolls;
+    } else {
+        return kWaitPolls;
+    }
+}
+
 // one 32-column group of an accumulator row to the mode's epilogue
 template <class Epi, class Args, class Tile>
 __device__ __forceinline__ void hand(Epi &epi, const Args &a, const Tile &T, int64_t col0,
@@ -188,15 +207,20 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
     const uint32_t tmem = tmem_slot;
     const uint32_t tA = tmem + nacc * kN;                      // A after the accumulators
 
-    auto wait = [&](uint64_t *bar, uint32_t parity) -> bool {
-        for (uint32_t it = 0; it < kWaitPolls; ++it) {
-            if (tc::mbar_try_wait(bar, parity)) return true;
+    auto wait_n = [&](uint64_t *bar, uint32_t parity, uint32_t polls) -> bool {
+        // a shortened limit polls without blocking (try_wait may suspend the
+        // thread for a hardware-chosen time, which would stretch the limit)
+        const bool quick = polls < kWaitPolls;
+        for (uint32_t it = 0; it < polls; ++it) {
+            if (quick ? tc::mbar_test_wait(bar, parity) : tc::mbar_try_wait(bar, parity)) return true;
             if ((it & 255u) == 255u && *(volatile int *)&s_abort) return false;
         }
         atomicExch(&s_abort, 1);
         atomicExch(status, SIEVE_ETIMEOUT);
         return false;
     };
+    auto wait = [&](uint64_t *bar, uint32_t parity) -> bool { return wait_n(bar, parity, kWaitPolls); };
+    const uint32_t epi_wait = epi_wait_polls<Mode>(a);
     // the i-th tile of this block from the ring, read by a whole warp (one
     // arrival per warp); false when the wait gave up.  t < 0 ends the loop.
     auto ring_take_warp = [&](uint32_t i, int &t) -> bool {
@@ -385,7 +409,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
             for (int ch = 0; ch < nch; ++ch, ++c) {
                 const uint32_t buf = c % nacc, dph = (c / nacc) & 1u;
                 epi.prefetch(a, T, ch);   // per-chunk loads, in flight during the wait
-                ok = __all_sync(0xffffffffu, wait(&dfull_bar[buf], dph));
+                ok = __all_sync(0xffffffffu, wait_n(&dfull_bar[buf], dph, epi_wait));
                 if (!ok) break;
                 epi.start(a, T, ch);
                 tc::fence_after_sync();

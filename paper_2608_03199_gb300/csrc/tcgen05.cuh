@@ -154,6 +154,18 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *mbar, uint32_t parity) {
     return ok != 0;
 }
 
+// Whether the phase of the given parity has completed, without blocking
+__device__ __forceinline__ bool mbar_test_wait(uint64_t *mbar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tmbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(mbar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
 // Wait until the phase of the given parity has completed, giving up after
 // `limit` polls (each try_wait itself blocks for a bounded, hardware-chosen
 // time).  Returns false on giving up.

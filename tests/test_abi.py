@@ -75,6 +75,17 @@ def test_scan_path_values_without_gpu():
         p = sieve._params(0.9, 10, 8, 4, True, 0, 0, scan_path=path)
         assert lib.sieve_search_workspace_size(ctypes.byref(v), 100, ctypes.byref(p), 0,
                                                ctypes.byref(n)) == 0
+    for serial in (0, 1):
+        p = sieve._params(0.9, 10, 8, 4, True, 0, 0, serial=serial)
+        assert lib.sieve_search_workspace_size(ctypes.byref(v), 100, ctypes.byref(p), 0,
+                                               ctypes.byref(n)) == 0
+    p = sieve._params(0.9, 10, 8, 4, True, 0, 0)
+    p.serial = 2
+    assert lib.sieve_search_workspace_size(ctypes.byref(v), 100, ctypes.byref(p), 0,
+                                           ctypes.byref(n)) == -1
+    p.serial, p.wait_limit = 0, -1
+    assert lib.sieve_search_workspace_size(ctypes.byref(v), 100, ctypes.byref(p), 0,
+                                           ctypes.byref(n)) == -1
     for path in (-1, 4):
         p = sieve._params(0.9, 10, 8, 4, True, 0, 0, scan_path=path)
         assert lib.sieve_search_workspace_size(ctypes.byref(v), 100, ctypes.byref(p), 0,

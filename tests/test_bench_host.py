@@ -32,7 +32,7 @@ def test_bruteforce_recall_against_the_oracle():
 
 
 def test_automatic_scan_rule():
-    cfg = types.SimpleNamespace(nprobe=64)
+    cfg = types.SimpleNamespace(nprobe=64, tau=0.9)
     auto = types.SimpleNamespace(scan_path="auto")
     assert not bench.uses_screen(auto, cfg, 8, True)
     assert bench.uses_screen(auto, cfg, 16, True)
@@ -40,7 +40,8 @@ def test_automatic_scan_rule():
     assert not bench.uses_screen(auto, cfg, 64, False)          # no tensor layout
     assert bench.uses_screen(types.SimpleNamespace(scan_path="screen"), cfg, 8, True)
     assert not bench.uses_screen(types.SimpleNamespace(scan_path="tensor"), cfg, 64, True)
-    assert not bench.uses_screen(auto, types.SimpleNamespace(nprobe=12), 64, True)
+    assert not bench.uses_screen(auto, types.SimpleNamespace(nprobe=12, tau=0.9), 64, True)
+    assert not bench.uses_screen(auto, cfg, 64, True, tau=0.5)       # loose threshold
 
 
 def test_cpu_baseline_times_both_modes():

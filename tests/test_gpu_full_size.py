@@ -82,3 +82,27 @@ def test_full_size_schedule_invariance_and_fixed_probe(full):
     rep = compare({k: v[sample] for k, v in fx.items()}, ref, idx, Q, qids, cfg.tau, cfg.k,
                   cfg.nprobe, order)
     assert_parity(rep)
+
+
+@pytest.mark.parametrize("W,tau", [(2, None), (4, None), (16, None), (8, 0.3)])
+def test_full_size_other_windows_and_loose_tau(full, W, tau):
+    """The whole 100K-query batch at other windows (W = 16 takes the screening
+    scan on the automatic path) and at tau = 0.3, where most probes hit and
+    the epilogue keeps the most candidates (the loose end of Sec. 6.4); the
+    oracle recomputes 600 sampled queries."""
+    cfg, wl, index, h = full
+    tau = cfg.tau if tau is None else tau
+    got = _np(sieve.search(index, wl["Q"], tau, cfg.k, cfg.nprobe, W, lookahead=True,
+                           query_ids=wl["qids"]))
+    assert ((got["probes"] >= min(W, cfg.nprobe)) & (got["probes"] <= cfg.nprobe)).all()
+    rng = np.random.default_rng(100 + W)
+    sample = np.sort(rng.choice(cfg.nq, 600, replace=False))
+    idx = {k: h[k] for k in ("X", "ids", "assign", "centroids")}
+    Q, qids = h["Q"][sample], h["qids"][sample]
+    ref = oracle.search(idx, Q, tau, cfg.k, cfg.nprobe, W, qids=qids)
+    order = oracle.rank(Q, h["centroids"], cfg.nprobe)
+    rep = compare({k: v[sample] for k, v in got.items()}, ref, idx, Q, qids, tau, cfg.k,
+                  cfg.nprobe, order)
+    assert_parity(rep)
+    if tau < 0.5:   # loose threshold: nearly every query fills its k results
+        assert (got["count"] == cfg.k).mean() > 0.9

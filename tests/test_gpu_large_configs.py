@@ -62,3 +62,36 @@ def test_large_config_sampled_parity(name, sample):
     rep = compare({k: v[pick] for k, v in got.items()}, ref, idx, Q, qids, cfg.tau, cfg.k,
                   cfg.nprobe, order)
     assert_parity(rep, max_allowed_frac=0.02)
+
+
+def test_10m256_windows_and_lookahead():
+    """The 10M x 256 workload (near-uniform density, few duplicates: most
+    queries find no tau-neighbour and stop at W) at W = 4 and 16, lookahead on
+    and off: outputs identical across the schedules, and the oracle agrees on
+    300 sampled queries for each window."""
+    assert torch.cuda.is_available()
+    dev = torch.device("cuda:0")
+    cfg = synth.CONFIGS["10m256"]
+    wl = synth.make_workload(cfg, device=dev)
+    index = sieve.build_layout(wl["X"], wl["assign"], cfg.nlist, wl["centroids"])
+    rng = np.random.default_rng(77)
+    pick = np.sort(rng.choice(cfg.nq, 300, replace=False))
+    pick_d = torch.from_numpy(pick).to(dev)
+    Q = wl["Q"][pick_d].cpu().numpy()
+    qids = wl["qids"][pick_d].cpu().numpy()
+    idx = {"X": wl["X"].cpu().numpy(), "ids": wl["ids"].cpu().numpy(),
+           "assign": wl["assign"].cpu().numpy(), "centroids": wl["centroids"].cpu().numpy()}
+    order = oracle.rank(Q, idx["centroids"], cfg.nprobe)
+    for W in (4, 16):
+        runs = []
+        for la in (True, False):
+            out = sieve.search(index, wl["Q"], cfg.tau, cfg.k, cfg.nprobe, W, lookahead=la,
+                               query_ids=wl["qids"])
+            runs.append({"ids": out[0].cpu().numpy(), "scores": out[1].cpu().numpy(),
+                         "count": out[2].cpu().numpy(), "probes": out[3].cpu().numpy()})
+        for key in runs[0]:
+            assert np.array_equal(runs[0][key], runs[1][key]), (W, key)
+        ref = oracle.search(idx, Q, cfg.tau, cfg.k, cfg.nprobe, W, qids=qids)
+        rep = compare({k: v[pick] for k, v in runs[0].items()}, ref, idx, Q, qids, cfg.tau,
+                      cfg.k, cfg.nprobe, order)
+        assert_parity(rep, max_allowed_frac=0.02)

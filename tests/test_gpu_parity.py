@@ -175,7 +175,10 @@ def test_schedule_changes_nothing(deep, g_deep, path):
     base = run(g_deep, Q, qids, c.tau, c.k, c.nprobe, c.W, lookahead=1, scan_path=path)
     variants = [dict(lookahead=0), dict(lookahead=1, max_items_per_round=4096),
                 dict(lookahead=1, max_items_per_round=7), dict(lookahead=0, loop=1),
-                dict(lookahead=1, loop=1, max_items_per_round=100)]
+                dict(lookahead=1, loop=1, max_items_per_round=100),
+                # the serial traversal (Sec. 6.3): every item its own partition call
+                dict(lookahead=0, serial=True), dict(lookahead=1, serial=True),
+                dict(lookahead=1, serial=True, loop=1, max_items_per_round=100)]
     for kw in variants:
         got = run(g_deep, Q, qids, c.tau, c.k, c.nprobe, c.W, scan_path=path, **kw)
         for key in ("ids", "scores", "count", "probes"):
@@ -186,6 +189,10 @@ def test_schedule_changes_nothing(deep, g_deep, path):
     for key in ("ids", "scores", "count", "probes"):
         assert np.array_equal(one[key], base[key][sub]), key
     assert one["stats"]["rounds"] >= one["probes"].sum()
+    # serial traversal: as many tiles as items, one query per partition call
+    ser = run(g_deep, Q, qids, c.tau, c.k, c.nprobe, c.W, lookahead=0, serial=True, stats=True,
+              scan_path=path)
+    assert ser["stats"]["tiles"] == ser["stats"]["items"] == base["probes"].sum()
 
 
 @pytest.mark.parametrize("path", ["simt", "tensor", "auto"])
