@@ -75,9 +75,12 @@ def parse():
                          "window of 16 up)")
     ap.add_argument("--rq", action="store_true",
                     help="the quantized local search (RaBitQ-style 7-bit codes) on the workload")
-    ap.add_argument("--ncu-case", choices=("w8", "fixed", "rqw8"), default=None,
+    ap.add_argument("--ncu-case", choices=("w8", "fixed", "rqw8", "rank"), default=None,
                     help="run exactly one search (W = the config's W, or fixed probe) and exit: "
-                         "a small, single-call target for an ncu capture")
+                         "a small, single-call target for an ncu capture; 'rank': one centroid "
+                         "ranking of --ncu-queries queries against seeded centroids of the "
+                         "config's nlist x d (under 1 GB on the device)")
+    ap.add_argument("--ncu-queries", type=int, default=20_000)
     return ap.parse_args()
 
 
@@ -159,8 +162,10 @@ def measured_peaks():
 # the sources that define each profiled kernel and the layout it streams
 _SCAN_SOURCES = ("common.cuh", "search.cuh", "scan_tc.cu", "tcgen05.cuh", "tc_bulk.cuh",
                  "tc_pipeline.cuh", "tc_layout.cu", "rq.cu")
+_RANK_SOURCES = ("common.cuh", "search.cuh", "rank_tc.cu", "tcgen05.cuh", "tc_bulk.cuh",
+                 "tc_pipeline.cuh", "tc_layout.cu")
 KERNEL_SOURCES = {"k_scan_bulk": _SCAN_SOURCES, "k_scan_rq": _SCAN_SOURCES,
-                  "k_scan_screen": _SCAN_SOURCES}
+                  "k_scan_screen": _SCAN_SOURCES, "k_rank_bulk + k_rank_screen": _RANK_SOURCES}
 
 
 def kernel_source_sha(kernel):
@@ -185,7 +190,7 @@ def committed_traffic(kernel, workload, launches):
     except Exception:
         return None
     e = t.get(kernel, {}).get(workload)
-    if not e or e.get("source_sha") != kernel_source_sha(kernel):
+    if not e or e.get("source_sha") != kernel_source_sha(kernel) or "dram_bytes_per_search" not in e:
         return None
     return e["dram_bytes_per_search"] / max(1, launches)
 
@@ -1000,6 +1005,22 @@ def run_ncu_case(args, cfg):
     import paper_2608_03199_gb300 as sieve
     dev = torch.device("cuda:0")
     sieve.lib()
+    if args.ncu_case == "rank":
+        # the ranking alone, on its own shape: unit centroids of the config's
+        # nlist x d, queries near seeded centroids
+        g = torch.Generator(device=dev).manual_seed(cfg.seed)
+        C = torch.randn(cfg.nlist, cfg.d, device=dev, generator=g)
+        C /= C.norm(dim=1, keepdim=True)
+        Q = C[torch.randint(0, cfg.nlist, (args.ncu_queries,), device=dev, generator=g)]
+        Q = Q + 0.1 * torch.randn(Q.shape, device=dev, generator=g)
+        Q /= Q.norm(dim=1, keepdim=True)
+        index = sieve.build_layout(C.clone(), torch.arange(cfg.nlist, dtype=torch.int32, device=dev),
+                                   cfg.nlist, C)
+        order = sieve.rank_partitions(index, Q, cfg.nprobe)
+        torch.cuda.synchronize()
+        print(json.dumps({"ncu_case": "rank", "nq": args.ncu_queries, "nlist": cfg.nlist, "d": cfg.d,
+                          "nprobe": cfg.nprobe, "first": int(order[0, 0])}))
+        return 0
     wl = synth.make_workload(cfg, device=dev)
     index = sieve.build_layout(wl["X"], wl["assign"], cfg.nlist, wl["centroids"])
     W = cfg.nprobe if args.ncu_case == "fixed" else cfg.W
