@@ -1,23 +1,33 @@
 // rank_tc.cu -- centroid ranking on the tcgen05 tensor cores (Sec. 2.3,
 // Sec. 4.1: P_i = the nprobe centroids with the largest inner product with
-// q_i, best first, equal scores by lower centroid id), for any nlist, in one
-// contraction pass: no score table, no second pass.
+// q_i, best first, equal scores by lower centroid id), for any nlist, with no
+// score table and one exact contraction pass.
 //
-//   k_rank_bulk / k_rank_tc  the tensor-core contraction (tc_bulk.cuh with the
+//   k_rank_screen  (nlist > 2,048, bulk pipeline) the first pass: one fp16
+//              product of the hi halves per score; the epilogue writes the
+//              maximum of each group of 64 (or 32) centroids.  Tiles of two
+//              sub-tiles of 128 queries share every B stage.
+//   k_rank_threshold  one warp per query: the nprobe-th largest group maximum
+//              less the proven error bounds of both passes, a starting
+//              threshold that at least nprobe centroids reach.
+//   k_rank_bulk / k_rank_tc  the exact contraction (tc_bulk.cuh with the
 //              centroids' tensor-core layout, else the converter pipeline of
-//              tc_pipeline.cuh).  A tile is 128 consecutive queries (A rows)
-//              against one range of centroids (B rows, 128 per chunk, in
-//              increasing id order).  Each epilogue thread owns one query and
-//              streams its scores: a 256-bin histogram of the scores it has
-//              kept (shared memory) gives a running threshold -- the lower edge
-//              of the highest bin such that at least nprobe kept scores lie in
-//              it or above -- and a score is appended to the query's candidate
-//              list only when it reaches that threshold.  A score below it has
-//              nprobe larger ones already, so it cannot be among the nprobe best.
-//   k_rank_final  one warp per query: the candidates of its ranges that reach
-//              their final thresholds, the exact nprobe best of them by (score
-//              desc, id asc), sorted.  The lists are in id order, so among equal
-//              scores the first taken are the lowest ids.
+//              tc_pipeline.cuh) against one range of centroids (B rows, 128
+//              per chunk, in increasing id order).  Each epilogue thread owns
+//              one query and appends the scores that reach its threshold to
+//              the query's list: the starting threshold of the first pass
+//              (two sub-tiles per tile where A fits tensor memory twice), or,
+//              without a first pass, a running threshold from a 256-bin
+//              histogram of the scores it has kept (shared memory) -- the
+//              lower edge of the highest bin such that at least nprobe kept
+//              scores lie in it or above.  A score below either threshold has
+//              nprobe larger ones, so it cannot be among the nprobe best.  Up
+//              to 2,048 centroids every score is kept (ids implicit).
+//   k_rank_final / k_rank_dense_final  one warp per query: the candidates of
+//              its ranges that reach their final thresholds, the exact nprobe
+//              best of them by (score desc, id asc), sorted.  The lists are in
+//              id order, so among equal scores the first taken are the lowest
+//              ids.
 // A query whose list overflowed (many equal scores, or an adversarial order)
 // is finished by the exact FP32 ranking of rank_kernel.cu.
 #include <cmath>
@@ -62,6 +72,7 @@ __device__ __forceinline__ float rank_edge_raw(int b) {
 constexpr int kRankGroupMax = 0;   // the maximum of each group of `group` centroids
 constexpr int kRankStream = 1;     // the scores that reach the running threshold
 constexpr int kRankDense = 2;      // every score (ids implicit: the list position)
+constexpr int kRankStreamInit = 3; // the scores that reach a given starting threshold (no histogram)
 
 struct RankArgs {
     const float *Q;
@@ -87,25 +98,31 @@ struct RankArgs {
 
 __device__ int g_rank_status_sink;
 
-template <int kMode>
+// kSubT sub-tiles of 128 queries per tile (tc_bulk.cuh); two only in modes
+// that keep nothing in shared memory
+template <int kMode, int kSubT = 1>
 struct RankModeT {
     using Args = RankArgs;
     static constexpr int kN = 128;
+    static constexpr int kSub = kSubT;
+    static constexpr int kRows = kSubT * tcp::kM;   // queries per tile
+    static_assert(kSubT == 1 || kMode == kRankGroupMax || kMode == kRankStreamInit,
+                  "two sub-tiles: no shared-memory state");
     struct Tile {
         int64_t q0;    // first query
         int ni;
         int64_t c0;    // first centroid of the tile's range
         int64_t nb;    // centroids in the range
     };
-    __device__ static int num_tiles(const Args &a) { return (int)ceil_div(a.nq, tcp::kM) * a.nranges; }
+    __device__ static int num_tiles(const Args &a) { return (int)ceil_div(a.nq, kRows) * a.nranges; }
     // every tile costs about the same: a static stride over the blocks
     __device__ static int *tile_counter(const Args &) { return nullptr; }
     __device__ static int d(const Args &a) { return a.d; }
     __device__ static int *status(const Args &a) { return a.status ? a.status : &g_rank_status_sink; }
     __device__ static Tile tile(const Args &a, int t) {
         Tile T;
-        T.q0 = (int64_t)(t / a.nranges) * tcp::kM;
-        T.ni = (int)(a.nq - T.q0 < tcp::kM ? a.nq - T.q0 : tcp::kM);
+        T.q0 = (int64_t)(t / a.nranges) * kRows;
+        T.ni = (int)(a.nq - T.q0 < kRows ? a.nq - T.q0 : kRows);
         T.c0 = (int64_t)(t % a.nranges) * a.range_len;
         T.nb = a.nlist - T.c0 < a.range_len ? a.nlist - T.c0 : a.range_len;
         return T;
@@ -140,7 +157,7 @@ struct RankModeT {
             bin = 0;
             above = 0;
             gacc = -__int_as_float(0x7f800000);
-            h = smem + (size_t)slot * kRankBinStride;
+            h = kMode == kRankStream ? smem + (size_t)slot * kRankBinStride : nullptr;
             if constexpr (kMode == kRankStream) {
                 uint32_t *hw = reinterpret_cast<uint32_t *>(h);
 #pragma unroll
@@ -173,7 +190,7 @@ struct RankModeT {
                 n += ncol;
                 return;
             }
-            if (kMode == kRankStream && a.init_edge) {
+            if constexpr (kMode == kRankStreamInit) {
                 // a starting threshold from the first pass: it already keeps
                 // only a little over nprobe scores, so no running histogram.
                 // The mask comes straight from the compares (some lane of a
@@ -251,15 +268,16 @@ struct RankModeT {
         __device__ void prefetch(const Args &, const Tile &, int) {}
         __device__ void start(const Args &, const Tile &, int) {}
         __device__ void end(const Args &a, const Tile &) {
-            if (!valid || kMode == kRankGroupMax) return;
+            if (!valid || kMode == kRankGroupMax || !a.list_n) return;
             a.list_n[at] = n;
             a.list_edge[at] = edge * (1.f / 65536.f);   // exact (-inf stays -inf)
         }
     };
 };
 // the first pass on the bulk pipeline: one fp16 product per score (hi halves
-// of A and B), whose error the threshold allows for
-struct RankScreenMode : RankModeT<kRankGroupMax> {
+// of A and B), whose error the threshold allows for; two sub-tiles of 128
+// queries share every B stage
+struct RankScreenMode : RankModeT<kRankGroupMax, 2> {
     static constexpr int kProducts = 1;
 };
 static_assert(kTcRows == RankModeT<kRankStream>::kN, "");
@@ -274,14 +292,33 @@ int rank_bulk_stages(int d) {
     return tcb::stages_for((int)ceil_div(d, 64), kRankEpiBytes, 232448 - 128);
 }
 
-template <int kMode>
+// every pair's screened score (one fp16 product of the hi halves) in a dense
+// row per query: a diagnostic of the first pass's arithmetic
+struct RankScreenDenseMode : RankModeT<kRankDense> {
+    static constexpr int kProducts = 1;
+};
+
+__global__ void __launch_bounds__(tcb::kThreads, 1) k_rank_screen_dense(RankArgs a, int stages) {
+    extern __shared__ unsigned char smem_raw[];
+    tcb::run_bulk<RankScreenDenseMode>(a, smem_raw, stages);
+}
+
+template <int kMode, int kSub = 1>
 __global__ void __launch_bounds__(tcb::kThreads, 1) k_rank_bulk(RankArgs a, int stages) {
     extern __shared__ unsigned char smem_raw[];
-    tcb::run_bulk<RankModeT<kMode>>(a, smem_raw, stages);
+    tcb::run_bulk<RankModeT<kMode, kSub>>(a, smem_raw, stages);
+}
+
+// the streaming pass from a starting threshold with two sub-tiles: A of both
+// (hi and lo) must leave two accumulators of tensor memory, d <= 128
+int rank_pair_stages(int d) {
+    const int nkb = (int)ceil_div(d, 64);
+    return tcb::sub_fits(nkb, 3, 2) ? tcb::stages_for(nkb, 0, 232448 - 128) : 0;
 }
 
 int rank_screen_stages(int d) {
-    return tcb::stages_for((int)ceil_div(d, 64), kRankEpiBytes, 232448 - 128, tcb::kStageBytesHi);
+    const int nkb = (int)ceil_div(d, 64);
+    return tcb::sub_fits(nkb, 1, 2) ? tcb::stages_for(nkb, 0, 232448 - 128, tcb::kStageBytesHi) : 0;
 }
 
 __global__ void __launch_bounds__(tcb::kThreads, 1) k_rank_screen(RankArgs a, int stages) {
@@ -749,6 +786,34 @@ __global__ void __launch_bounds__(kSelectWarps * 32) k_rank_threshold(
 }
 
 // ---------------------------------------------------------------------------
+cudaError_t enqueue_screen_scores(const float *Q, int64_t nq, int64_t nlist, int d,
+                                  const unsigned char *tc_cent, float *out, int64_t ld,
+                                  int *status, cudaStream_t st) {
+    if (nq <= 0) return cudaSuccess;
+    const int nkb = (int)ceil_div(d, 64);
+    const int stages = tcb::stages_for(nkb, 0, 232448 - 128, tcb::kStageBytesHi);
+    if (stages == 0) return cudaErrorInvalidValue;
+    const size_t smem = tcb::smem_bytes(stages, 0, tcb::kStageBytesHi);
+    cudaError_t e = cudaFuncSetAttribute(k_rank_screen_dense, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+    RankArgs a{};
+    a.Q = Q;
+    a.nq = nq;
+    a.nlist = nlist;
+    a.d = d;
+    a.status = status;
+    a.tc_cent = tc_cent;
+    a.nprobe = 1;
+    a.nranges = 1;
+    a.range_len = round_up(nlist, (int64_t)kTcRows);
+    a.cap = (int)ld;
+    a.list_s = out;
+    const int tiles = (int)ceil_div(nq, tcp::kM);
+    k_rank_screen_dense<<<(unsigned)std::min(tiles, num_sms()), tcb::kThreads, smem, st>>>(a, stages);
+    return cudaGetLastError();
+}
+
 bool rank_tc_supported(int64_t nlist, int nprobe) { return nlist >= 1 && nprobe <= nlist; }
 
 static int pow2_at_least(int64_t x) {
@@ -872,14 +937,19 @@ cudaError_t prepare_rank_tc(int nprobe, int d) {
         if (e == cudaSuccess)
             e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc_smem());
     const int bulk = rank_bulk_stages(d);
-    for (auto f : {k_rank_bulk<kRankGroupMax>, k_rank_bulk<kRankStream>, k_rank_bulk<kRankDense>})
+    for (auto f : {k_rank_bulk<kRankGroupMax>, k_rank_bulk<kRankStream>, k_rank_bulk<kRankDense>,
+                   k_rank_bulk<kRankStreamInit>})
         if (e == cudaSuccess && bulk)
             e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      (int)tcb::smem_bytes(bulk, kRankEpiBytes));
+    const int pair = rank_pair_stages(d);
+    if (e == cudaSuccess && pair)
+        e = cudaFuncSetAttribute(k_rank_bulk<kRankStreamInit, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)tcb::smem_bytes(pair, 0));
     const int scr = rank_screen_stages(d);
     if (e == cudaSuccess && scr)
         e = cudaFuncSetAttribute(k_rank_screen, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)tcb::smem_bytes(scr, kRankEpiBytes, tcb::kStageBytesHi));
+                                 (int)tcb::smem_bytes(scr, 0, tcb::kStageBytesHi));
     if (e == cudaSuccess) e = set_final_attr<2>();
     if (e == cudaSuccess) e = set_final_attr<4>();
     if (e == cudaSuccess) e = set_final_attr<8>();
@@ -993,6 +1063,7 @@ cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t 
     const int bulk_stages = tc_cent ? rank_bulk_stages(d) : 0;
     const RankPlan L = rank_plan(plan_nq, nlist, nprobe, d, bulk_stages > 0);
     const int screen_stages = L.screen ? rank_screen_stages(d) : 0;
+    const int pair_stages = bulk_stages && L.group ? rank_pair_stages(d) : 0;
     // the chunk's scratch: lists (scores, ids), counts, final thresholds,
     // overflow list, group maxima, starting thresholds; then the fixed part
     const int64_t slots = L.chunk * L.nranges;
@@ -1006,19 +1077,27 @@ cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t 
     unsigned char *fixed = reinterpret_cast<unsigned char *>(scratch) + L.chunk * L.per_query();
     int *ovf_n = reinterpret_cast<int *>(fixed);
     unsigned *cmax = reinterpret_cast<unsigned *>(fixed + 4);
-    auto contract = [&](int mode, const RankArgs &a, int tiles, bool scr) {
+    auto contract = [&](int mode, const RankArgs &a, int64_t n, bool scr) {
         if (mma_ms) {
             evs.resize(evs.size() + 2);
             cudaEventCreate(&evs[evs.size() - 2]);
             cudaEventCreate(&evs.back());
             cudaEventRecord(evs[evs.size() - 2], st);
         }
+        // tiles of 128 queries, or of two sub-tiles of 128 (the screen, and the
+        // streaming pass from a starting threshold where A fits twice)
+        const bool two = scr || (mode == kRankStreamInit && pair_stages);
+        const int tiles = (int)(ceil_div(n, (two ? 2 : 1) * tcp::kM) * L.nranges);
         const unsigned grid = (unsigned)std::min(tiles, num_sms());
         const size_t bsm = tcb::smem_bytes(bulk_stages, kRankEpiBytes);
         if (scr)
-            k_rank_screen<<<grid, tcb::kThreads,
-                            tcb::smem_bytes(screen_stages, kRankEpiBytes, tcb::kStageBytesHi), st>>>(
-                a, screen_stages);
+            k_rank_screen<<<grid, tcb::kThreads, tcb::smem_bytes(screen_stages, 0, tcb::kStageBytesHi),
+                            st>>>(a, screen_stages);
+        else if (mode == kRankStreamInit && pair_stages)
+            k_rank_bulk<kRankStreamInit, 2><<<grid, tcb::kThreads, tcb::smem_bytes(pair_stages, 0), st>>>(
+                a, pair_stages);
+        else if (mode == kRankStreamInit)
+            k_rank_bulk<kRankStreamInit><<<grid, tcb::kThreads, bsm, st>>>(a, bulk_stages);
         else if (bulk_stages && mode == kRankGroupMax)
             k_rank_bulk<kRankGroupMax><<<grid, tcb::kThreads, bsm, st>>>(a, bulk_stages);
         else if (bulk_stages && mode == kRankStream)
@@ -1041,16 +1120,15 @@ cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t 
     }
     for (int64_t q0 = 0; q0 < nq; q0 += L.chunk) {
         const int64_t n = nq - q0 < L.chunk ? nq - q0 : L.chunk;
-        const int tiles = (int)(ceil_div(n, tcp::kM) * L.nranges);
         RankArgs a{Q + q0 * d, n, C, nlist, d, status, tc_cent, nprobe, L.nranges,
                    L.range_len, L.cap, list_s, list_i, list_n, list_edge, nullptr, gmax, L.gld,
                    L.group};
         if (L.group) {   // the first pass: group maxima, then each query's starting threshold
-            contract(kRankGroupMax, a, tiles, L.screen);
+            contract(kRankGroupMax, a, n, L.screen);
             launch_threshold(L, gmax, n, nprobe, Q + q0 * d, d, cmax, init_edge, st);
             a.init_edge = init_edge;
         }
-        contract(L.mode, a, tiles, false);
+        contract(L.group ? kRankStreamInit : L.mode, a, n, false);
         cudaError_t e = cudaMemsetAsync(ovf_n, 0, sizeof(int), st);
         if (e != cudaSuccess) return e;
         int32_t *o = order + q0 * nprobe;

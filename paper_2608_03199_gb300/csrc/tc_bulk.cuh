@@ -37,6 +37,18 @@
 //               shared memory)
 //   warps 10-13 epilogue: thread i owns tensor-memory lane i = A row i; it
 //               hands its row of a chunk (scores x 2^16) to Mode::Epi
+//
+// Two sub-tiles (a mode with kSub = 2): a tile is 256 A rows, two sets of 128
+// in tensor memory side by side, and every B stage feeds the MMAs of both, so
+// each byte of B streamed into shared memory does twice the work.  Where the
+// A rows are few per tile and many B chunks follow (the centroid ranking),
+// writing A is rare and the epilogue is the busy role: warps 0-3 write A
+// (every K-block of both sub-tiles), warp 4 is the producer, warp 5 the MMA
+// issuer and warps 6-13 the epilogue, 6-9 on sub-tile 0 and 10-13 on
+// sub-tile 1 (warp w reads tensor-memory lanes 32 (w % 4) .. +31).  Each
+// sub-tile has its own accumulator, handed to its epilogue as soon as its
+// MMAs of the chunk are issued, so one sub-tile's epilogue runs while the
+// other's MMAs do.
 // Every wait is bounded; giving up sets SIEVE_ETIMEOUT in the mode's status
 // word, all roles leave their loops, the issued MMAs and copies are drained
 // (bounded) and tensor memory is freed.
@@ -107,6 +119,31 @@ struct mma_products { static constexpr int value = b_has_lo<Mode>::value ? 3 : 2
 template <class Mode>
 struct mma_products<Mode, decltype((void)Mode::kProducts)> { static constexpr int value = Mode::kProducts; };
 
+// sub-tiles of 128 A rows per tile: Mode::kSub if given (1 or 2), else 1
+template <class Mode, class = void>
+struct sub_tiles { static constexpr int value = 1; };
+template <class Mode>
+struct sub_tiles<Mode, decltype((void)Mode::kSub)> { static constexpr int value = Mode::kSub; };
+
+// tensor-memory columns of one sub-tile's A: 64 per K-block (hi and lo), 32
+// for a screen (hi alone)
+__host__ __device__ constexpr uint32_t a_cols(int nkb, int products) {
+    return (uint32_t)nkb * (products == 1 ? 32u : 64u);
+}
+
+// 128-column accumulators beside A: one sub-tile takes three when its A
+// takes at most 128 columns, else two; two sub-tiles take two, accumulator j
+// always sub-tile j's, so that each accumulator's barriers have one reader
+// group and phases cannot be skipped
+__host__ __device__ constexpr uint32_t acc_slots(int nkb, int products, int sub) {
+    return sub == 1 ? ((products == 1 || nkb <= 2) ? 3u : 2u) : 2u;
+}
+
+// whether a pipeline of sub sub-tiles fits tensor memory at this d
+__host__ __device__ constexpr bool sub_fits(int nkb, int products, int sub) {
+    return nkb <= kMaxKb && (uint32_t)sub * a_cols(nkb, products) + 2u * kN <= kTmemCols;
+}
+
 // polls of the epilogue's accumulator wait: the mode's epi_wait_polls(a) if
 // it has one (a testing aid that lets that wait give up early; 0 = default),
 // else kWaitPolls.  No other wait takes it: every drain keeps the full limit.
@@ -158,6 +195,14 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
     constexpr uint32_t kAKb = kProd == 1 ? 32 : 64;
     constexpr int kKs = kKbPerStage;                          // K-blocks per B stage
     constexpr uint32_t kStage = kKs * kKbB;                    // bytes of one B stage
+    constexpr int kSub = sub_tiles<Mode>::value;
+    static_assert(kSub == 1 || kSub == 2, "one or two sub-tiles");
+    // warp roles: A writers, producer, MMA issuer, epilogue (4 warps per sub-tile)
+    constexpr int kAW = kSub == 1 ? kAWriterWarps : 4;
+    constexpr int kAWGroups = kAW / 4;                         // K-block classes of A writers
+    constexpr int kProdW = kAW, kMmaW = kAW + 1, kEpiW0 = kAW + 2;
+    static_assert(kEpiW0 + 4 * kSub == kThreads / 32, "every warp has a role");
+    static_assert(kAW + 1 + 4 * kSub == (int)kRingReaders, "ring readers");
     __shared__ __align__(8) uint64_t a_full[kMaxKb], a_empty[kMaxKb], b_full[kMaxStages],
         b_empty[kMaxStages], dfull_bar[kMaxAcc], dempty_bar[kMaxAcc], drain_bar, ring_full[kRing],
         ring_empty[kRing];
@@ -171,12 +216,17 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
     const int n_tiles = Mode::num_tiles(a);
     const int d = Mode::d(a);
     const int nkb = (int)ceil_div(d, 64);
-    // 128-column accumulators beside A: three when A takes at most 128
-    // columns (a screen, or d <= 128), two otherwise (512 columns in all)
-    const uint32_t nacc = (kProd == 1 || nkb <= 2) ? 3u : 2u;
+    int *status = Mode::status(a);
+    // a d whose A does not fit tensor memory (the host never launches one):
+    // report it and leave before any barrier or tensor memory is set up
+    if (!sub_fits(nkb, kProd, kSub)) {
+        if (threadIdx.x == 0) atomicExch(status, SIEVE_EINVAL);
+        return;
+    }
+    const uint32_t nacc = acc_slots(nkb, kProd, kSub);
+    const uint32_t aTile = a_cols(nkb, kProd);                 // A columns of one sub-tile
     unsigned char *Bst = base;                                 // stages x kStage
     unsigned char *epi_smem = Bst + (size_t)stages * kStage;
-    int *status = Mode::status(a);
     int *tile_counter = Mode::tile_counter(a);
 
     if (threadIdx.x == 0) {
@@ -200,7 +250,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
         s_abort = 0;
         tc::mbar_init_fence();
     }
-    if (warp == kMmaWarp) tc::tmem_alloc(&tmem_slot, kTmemCols);
+    if (warp == kMmaW) tc::tmem_alloc(&tmem_slot, kTmemCols);
     tc::fence_before_sync();
     __syncthreads();
     tc::fence_after_sync();
@@ -232,7 +282,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
         return true;
     };
 
-    if (warp < kAWriterWarps) {
+    if (warp < kAW) {
         // ---------------- A writers ----------------
         const int quarter = warp & 3, group = warp >> 2;
         const int row = quarter * 32 + lane;
@@ -244,34 +294,44 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
             if (!ring_take_warp(i, t) || t < 0) break;
             const typename Mode::Tile T = Mode::tile(a, t);
             if (T.nb <= 0) continue;
-            const float *rp = Mode::a_row(a, T, row);
-            if (rp && group == 0) tc::prefetch_l2(rp, (uint32_t)d * 4u);   // d % 4 == 0
-            for (int kb = group; kb < nkb; kb += 2) {
-                float4 x[16];
-#pragma unroll
-                for (int q4 = 0; q4 < 16; ++q4) x[q4] = tcp::load_f4(rp, kb * 64 + 4 * q4, d);
-                if (!(ok = __all_sync(0xffffffffu, wait(&a_empty[kb], (u & 1u) ^ 1u)))) break;
-                tc::fence_after_sync();
-#pragma unroll
-                for (int half = 0; half < 2; ++half) {     // 32 elements = 16 columns per half
-                    uint32_t hi[16], lo[16];
-#pragma unroll
-                    for (int q4 = 0; q4 < 8; ++q4) {
-                        const float4 v = x[half * 8 + q4];
-                        tcp::split2(v.x, v.y, hi[2 * q4], lo[2 * q4]);
-                        tcp::split2(v.z, v.w, hi[2 * q4 + 1], lo[2 * q4 + 1]);
-                    }
-                    const uint32_t col = tA + (uint32_t)kb * kAKb + (uint32_t)half * 16;
-                    tc::tmem_st16(col + lane_bits, hi);
-                    if constexpr (kProd > 1) tc::tmem_st16(col + 32 + lane_bits, lo);
+            if (group == 0)
+                for (int h = 0; h < kSub; ++h) {
+                    const float *rp = Mode::a_row(a, T, row + h * tcp::kM);
+                    if (rp) tc::prefetch_l2(rp, (uint32_t)d * 4u);   // d % 4 == 0
                 }
+            for (int kb = group; ok && kb < nkb; kb += kAWGroups) {
+#pragma unroll 1
+                for (int h = 0; h < kSub; ++h) {
+                    const float *rp = Mode::a_row(a, T, row + h * tcp::kM);
+                    float4 x[16];
+#pragma unroll
+                    for (int q4 = 0; q4 < 16; ++q4) x[q4] = tcp::load_f4(rp, kb * 64 + 4 * q4, d);
+                    if (h == 0) {
+                        if (!(ok = __all_sync(0xffffffffu, wait(&a_empty[kb], (u & 1u) ^ 1u)))) break;
+                        tc::fence_after_sync();
+                    }
+#pragma unroll
+                    for (int half = 0; half < 2; ++half) {     // 32 elements = 16 columns per half
+                        uint32_t hi[16], lo[16];
+#pragma unroll
+                        for (int q4 = 0; q4 < 8; ++q4) {
+                            const float4 v = x[half * 8 + q4];
+                            tcp::split2(v.x, v.y, hi[2 * q4], lo[2 * q4]);
+                            tcp::split2(v.z, v.w, hi[2 * q4 + 1], lo[2 * q4 + 1]);
+                        }
+                        const uint32_t col = tA + (uint32_t)h * aTile + (uint32_t)kb * kAKb + (uint32_t)half * 16;
+                        tc::tmem_st16(col + lane_bits, hi);
+                        if constexpr (kProd > 1) tc::tmem_st16(col + 32 + lane_bits, lo);
+                    }
+                }
+                if (!ok) break;
                 tc::tmem_st_wait();
                 tc::fence_before_sync();
                 tc::mbar_arrive(&a_full[kb]);
             }
             ++u;
         }
-    } else if (warp == kProducerWarp) {
+    } else if (warp == kProdW) {
         // ---------------- tile scheduler + B producer ----------------
         if (lane == 0) {
             uint32_t s = 0;
@@ -313,10 +373,10 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                     if (tc::mbar_try_wait(&b_full[j % stages], (j / stages) & 1u)) break;
         }
         __syncwarp();
-    } else if (warp == kMmaWarp) {
+    } else if (warp == kMmaW) {
         // ---------------- MMA issuer ----------------
         if (lane == 0) {
-            uint32_t s = 0, c = 0, u = 0;
+            uint32_t s = 0, c = 0, u = 0;   // c: accumulator uses, kSub per chunk
             bool ok = true;
             for (uint32_t i = 0; ok; ++i) {
                 const uint32_t slot = i % kRing, rph = (i / kRing) & 1u;
@@ -327,64 +387,78 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                 const typename Mode::Tile T = Mode::tile(a, t);
                 const int nch = (int)ceil_div(T.nb, kN);
                 if (nch == 0) continue;
-                for (int ch = 0; ok && ch < nch; ++ch, ++c) {
-                    const uint32_t buf = c % nacc, dph = (c / nacc) & 1u;
-                    if (!(ok = wait(&dempty_bar[buf], dph ^ 1u))) break;
-                    tc::fence_after_sync();
-                    const uint32_t dt = tmem + buf * kN;
+                for (int ch = 0; ok && ch < nch; ++ch, c += kSub) {
+                    if constexpr (kSub == 1) {   // the chunk's accumulator
+                        if (!(ok = wait(&dempty_bar[c % nacc], ((c / nacc) & 1u) ^ 1u))) break;
+                        tc::fence_after_sync();
+                    }
                     for (int kb0 = 0; kb0 < nkb; kb0 += kKs, ++s) {
                         const uint32_t st = s % stages, ph = (s / stages) & 1u;
                         const int kb1 = nkb - kb0 < kKs ? nkb : kb0 + kKs;   // this stage's K-blocks
+                        const bool last = kb1 == nkb;                       // the chunk's last stage
                         if (ch == 0)
                             for (int kb = kb0; ok && kb < kb1; ++kb) ok = wait(&a_full[kb], u & 1u);
                         if (!ok || !(ok = wait(&b_full[st], ph))) break;
                         tc::fence_after_sync();
-                        for (int kb = kb0; kb < kb1; ++kb) {
-                            // K steps of 16 that hold any of the d elements: the
-                            // rest of the last K-block is zero padding
-                            const int kst = d - kb * 64 >= 64 ? 4 : (d - kb * 64 + 15) / 16;
-                            const uint32_t a_hi = tA + (uint32_t)kb * kAKb, a_lo = a_hi + 32;
-                            const uint32_t b_hi = tc::smem_u32(Bst + (size_t)st * kStage) +
-                                                  (uint32_t)(kb - kb0) * kKbB;
-                            // a K step moves the descriptors' start address by 32 bytes
-                            // (2 in its 16-byte units; shared addresses stay far below
-                            // the field's 2^14 limit, so no carry)
-                            const uint64_t bh = tc::desc_k_sw128(b_hi);
-                            if constexpr (kLo) {
-                                const uint64_t bl = tc::desc_k_sw128(b_hi + kKbBytes / 2);
-#pragma unroll
-                                for (int ks = 0; ks < 4; ++ks) {   // K = 16: 8 columns of A, 32 bytes of B
-                                    if (ks >= kst) break;
-                                    const uint32_t ao = ks * 8;
-                                    const uint64_t bo = 2 * ks;
-                                    tc::mma_f16_ta(dt, a_lo + ao, bh + bo, kIdesc, (kb > 0 || ks > 0) ? 1u : 0u);
-                                    tc::mma_f16_ta(dt, a_hi + ao, bl + bo, kIdesc, 1u);
-                                    tc::mma_f16_ta(dt, a_hi + ao, bh + bo, kIdesc, 1u);
-                                }
-                            } else if constexpr (kProd == 2) {   // B exact in fp16: hi and lo of A against it
-#pragma unroll
-                                for (int ks = 0; ks < 4; ++ks) {
-                                    if (ks >= kst) break;
-                                    const uint32_t ao = ks * 8;
-                                    const uint64_t bo = 2 * ks;
-                                    tc::mma_f16_ta(dt, a_lo + ao, bh + bo, kIdesc, (kb > 0 || ks > 0) ? 1u : 0u);
-                                    tc::mma_f16_ta(dt, a_hi + ao, bh + bo, kIdesc, 1u);
-                                }
-                            } else {   // a screen: the hi halves alone
-#pragma unroll
-                                for (int ks = 0; ks < 4; ++ks)
-                                    if (ks < kst)
-                                        tc::mma_f16_ta(dt, a_hi + ks * 8, bh + 2 * ks, kIdesc,
-                                                       (kb > 0 || ks > 0) ? 1u : 0u);
+#pragma unroll 1
+                        for (int h = 0; ok && h < kSub; ++h) {
+                            if (kSub > 1 && kb0 == 0) {   // sub-tile h's accumulator, just before its MMAs
+                                if (!(ok = wait(&dempty_bar[(c + h) % nacc], (((c + h) / nacc) & 1u) ^ 1u))) break;
+                                tc::fence_after_sync();
                             }
+                            const uint32_t dt = tmem + ((c + h) % nacc) * kN;
+                            for (int kb = kb0; kb < kb1; ++kb) {
+                                // K steps of 16 that hold any of the d elements: the
+                                // rest of the last K-block is zero padding
+                                const int kst = d - kb * 64 >= 64 ? 4 : (d - kb * 64 + 15) / 16;
+                                const uint32_t a_hi = tA + (uint32_t)h * aTile + (uint32_t)kb * kAKb,
+                                               a_lo = a_hi + 32;
+                                const uint32_t b_hi = tc::smem_u32(Bst + (size_t)st * kStage) +
+                                                      (uint32_t)(kb - kb0) * kKbB;
+                                // a K step moves the descriptors' start address by 32 bytes
+                                // (2 in its 16-byte units; shared addresses stay far below
+                                // the field's 2^14 limit, so no carry)
+                                const uint64_t bh = tc::desc_k_sw128(b_hi);
+                                if constexpr (kLo) {
+                                    const uint64_t bl = tc::desc_k_sw128(b_hi + kKbBytes / 2);
+#pragma unroll
+                                    for (int ks = 0; ks < 4; ++ks) {   // K = 16: 8 columns of A, 32 bytes of B
+                                        if (ks >= kst) break;
+                                        const uint32_t ao = ks * 8;
+                                        const uint64_t bo = 2 * ks;
+                                        tc::mma_f16_ta(dt, a_lo + ao, bh + bo, kIdesc, (kb > 0 || ks > 0) ? 1u : 0u);
+                                        tc::mma_f16_ta(dt, a_hi + ao, bl + bo, kIdesc, 1u);
+                                        tc::mma_f16_ta(dt, a_hi + ao, bh + bo, kIdesc, 1u);
+                                    }
+                                } else if constexpr (kProd == 2) {   // B exact in fp16: hi and lo of A against it
+#pragma unroll
+                                    for (int ks = 0; ks < 4; ++ks) {
+                                        if (ks >= kst) break;
+                                        const uint32_t ao = ks * 8;
+                                        const uint64_t bo = 2 * ks;
+                                        tc::mma_f16_ta(dt, a_lo + ao, bh + bo, kIdesc, (kb > 0 || ks > 0) ? 1u : 0u);
+                                        tc::mma_f16_ta(dt, a_hi + ao, bh + bo, kIdesc, 1u);
+                                    }
+                                } else {   // a screen: the hi halves alone
+#pragma unroll
+                                    for (int ks = 0; ks < 4; ++ks)
+                                        if (ks < kst)
+                                            tc::mma_f16_ta(dt, a_hi + ks * 8, bh + 2 * ks, kIdesc,
+                                                           (kb > 0 || ks > 0) ? 1u : 0u);
+                                }
+                            }
+                            // with two sub-tiles, the first sub-tile's accumulator is
+                            // handed over before the second's MMAs are issued
+                            if (kSub > 1 && last && h + 1 < kSub) tc::mma_commit(&dfull_bar[(c + h) % nacc]);
                         }
+                        if (!ok) break;
                         tc::mma_commit(&b_empty[st]);
                         // the tile's last reads of these K-blocks of A: they may be
                         // overwritten by the next tile once they are done
                         if (ch == nch - 1)
                             for (int kb = kb0; kb < kb1; ++kb) tc::mma_commit(&a_empty[kb]);
                     }
-                    if (ok) tc::mma_commit(&dfull_bar[buf]);
+                    if (ok) tc::mma_commit(&dfull_bar[(c + kSub - 1) % nacc]);
                 }
                 ++u;
             }
@@ -395,9 +469,10 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
         __syncwarp();
     } else {
         // ---------------- epilogue ----------------
-        const int quarter = warp & 3;
-        const int slot = quarter * 32 + lane;
-        uint32_t c = 0;
+        const int quarter = warp & 3;                      // the lanes this warp may read
+        const int h = (warp - kEpiW0) >> 2;                // its sub-tile
+        const int slot = h * tcp::kM + quarter * 32 + lane;
+        uint32_t c = h;
         bool ok = true;
         typename Mode::Epi epi;
         for (uint32_t i = 0; ok; ++i) {
@@ -406,7 +481,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
             const typename Mode::Tile T = Mode::tile(a, t);
             const int nch = (int)ceil_div(T.nb, kN);
             epi.begin(a, T, slot, epi_smem);
-            for (int ch = 0; ch < nch; ++ch, ++c) {
+            for (int ch = 0; ch < nch; ++ch, c += kSub) {
                 const uint32_t buf = c % nacc, dph = (c / nacc) & 1u;
                 epi.prefetch(a, T, ch);   // per-chunk loads, in flight during the wait
                 ok = __all_sync(0xffffffffu, wait_n(&dfull_bar[buf], dph, epi_wait));
@@ -441,7 +516,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
 
     tc::fence_before_sync();
     __syncthreads();
-    if (warp == kMmaWarp) {
+    if (warp == kMmaW) {
         tc::fence_after_sync();
         tc::tmem_dealloc(tmem, kTmemCols);
     }
