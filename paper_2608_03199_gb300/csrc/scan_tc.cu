@@ -16,6 +16,12 @@ namespace sieve {
 
 __device__ __forceinline__ int tc_nkb_dev(int d) { return (d + 63) / 64; }
 
+// epilogue shared memory beyond the kept lists (bulk pipeline): per epilogue
+// warp one 512-byte copy of a chunk's factors (the scan over codes) and two
+// 1 KB buffers of row ids
+constexpr size_t kEpiFacBytes = 4 * 512;
+constexpr size_t kEpiIdsBytes = 4 * 2 * 1024;
+
 // kRQ = false: exact inner products (B = the rows' hi / lo split);
 // kRQ = true: RaBitQ-style estimates from the code layout (B = u - mid).
 // kScreen (exact only): one product of the hi halves per pair screens every
@@ -71,9 +77,14 @@ struct ScanModeT {
         // kScreen: |q| of the item's query, the error-bound coefficients, the
         // largest row norm of each of the tile's 128-row blocks and that of
         // the current chunk (loaded before its accumulator wait)
-        float qn, m_rel, m_abs, xn;
+        float qn, m_rel, m_abs, xn, xn_next;
         const float *bn;
-        long long *ids_s;   // kScreen: this warp's copy of the chunk's 128 row ids
+        // bulk pipeline: this warp's two buffers of 128 row ids, filled by
+        // asynchronous copies one chunk ahead; buffer ids_ch % 2 holds the
+        // current chunk's (ids_ch < 0 on the converter pipeline, which reads
+        // ids from global memory)
+        long long *ids_b;
+        int ids_ch;
         bool valid;
         long long qid;
         // the kept list is unordered while the tile runs; once it holds k
@@ -97,7 +108,9 @@ struct ScanModeT {
             qid = (long long)-0x7fffffffffffffffll - 1;
             qc = 0.f;
             fs = reinterpret_cast<float *>(smem + (size_t)tcp::kM * a.k * 12) + (slot >> 5) * 128;
-            ids_s = reinterpret_cast<long long *>(smem + (size_t)tcp::kM * a.k * 12) + (slot >> 5) * 128;
+            ids_b = reinterpret_cast<long long *>(smem + (size_t)tcp::kM * a.k * 12 + kEpiFacBytes) +
+                    (slot >> 5) * 2 * tcb::kN;
+            ids_ch = -1;
             if (valid) {
                 item = a.bucketed[T.ib + slot];
                 q = a.item_q[item];
@@ -121,7 +134,7 @@ struct ScanModeT {
                 m_rel = 0.0009765625f + 0.000244140625f + (float)a.d * 2.384185791015625e-7f;
                 m_abs = 1.4901161193847656e-8f * sqrtf((float)a.d);
                 qn = valid ? a.qnorm[q] : 0.f;
-                xn = 0.f;
+                xn = xn_next = 0.f;
             }
         }
         __device__ void find_worst(int k) {
@@ -142,7 +155,8 @@ struct ScanModeT {
         // list (appended while it has room, else in place of its last entry)
         __device__ __forceinline__ void take(const Args &a, const Tile &T, int64_t col, float sc) {
             if (a.k == kn && sc < wst_s) return;   // cannot rank before the last kept entry
-            const long long id = a.ids[T.r_begin + col];
+            const long long id = ids_ch >= 0 ? ids_b[(ids_ch & 1) * tcb::kN + (col & (tcb::kN - 1))]
+                                             : a.ids[T.r_begin + col];
             if (id == qid) return;
             insert(a, sc, id);
         }
@@ -213,7 +227,7 @@ struct ScanModeT {
 #pragma unroll
                 for (int j = 0; j < 32; ++j) m |= (v[j] >= cut && j < ncol) ? (1u << j) : 0u;
                 // the query's own row leaves here (ids from the warp's copy)
-                const long long *cid = ids_s + (col0 & (tcb::kN - 1));
+                const long long *cid = ids_b + (ids_ch & 1) * tcb::kN + (col0 & (tcb::kN - 1));
                 for (unsigned mm = m; mm; mm &= mm - 1u) {
                     const int j = __ffs(mm) - 1;
                     if (cid[j] == qid) m &= ~(1u << j);
@@ -270,40 +284,55 @@ struct ScanModeT {
                     const int j = __ffs(m) - 1;
                     m &= m - 1u;
                     if (sc >= a.tau && !(kn == a.k && sc < wst_s))
-                        insert(a, sc, ids_s[(col0 & (tcb::kN - 1)) + j]);
+                        insert(a, sc, ids_b[(ids_ch & 1) * tcb::kN + (col0 & (tcb::kN - 1)) + j]);
                 }
             }
         }
-        // kRQ: the chunk's factors into this warp's shared copy, one coalesced
-        // 512-byte asynchronous copy per warp issued before the accumulator wait
+        // the row ids of chunk c into buffer c % 2 of this warp (8-byte
+        // asynchronous copies, one group)
+        __device__ __forceinline__ void copy_ids(const Args &a, const Tile &T, int c) {
+            const int64_t r0 = T.r_begin + (int64_t)c * tcb::kN;
+            const int64_t left = T.nb - (int64_t)c * tcb::kN;
+            const int nrow = left < tcb::kN ? (int)left : tcb::kN;
+            long long *dst = ids_b + (c & 1) * tcb::kN;
+            for (int j = slot & 31; j < nrow; j += 32)
+                asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(tc::smem_u32(dst + j)),
+                             "l"(a.ids + r0 + j)
+                             : "memory");
+            asm volatile("cp.async.commit_group;\n" ::: "memory");
+        }
+        // Before chunk ch's accumulator wait (bulk pipeline): copies in flight
+        // for it -- kRQ, the chunk's factors into this warp's shared copy (one
+        // coalesced 512-byte copy per warp); the row ids one chunk ahead (both
+        // of the first two chunks at ch = 0), so their latency hides behind a
+        // chunk; kScreen, the block norm of the next chunk into a register.
+        // Every lane of the warp is done with the buffers being refilled (the
+        // chunk before last).
         __device__ __forceinline__ void prefetch(const Args &a, const Tile &T, int ch) {
-            if constexpr (kScreen) {
-                // the chunk's block norm and its row ids (8-byte asynchronous
-                // copies into this warp's shared copy), in flight during the
-                // accumulator wait; every lane is done with the previous copy
-                __syncwarp();
-                xn = bn[ch];
-                const int64_t r0 = T.r_begin + (int64_t)ch * tcb::kN;
-                const int64_t left = T.nb - (int64_t)ch * tcb::kN;
-                const int nrow = left < tcb::kN ? (int)left : tcb::kN;
-                for (int j = slot & 31; j < nrow; j += 32) {
-                    const uint32_t dst = tc::smem_u32(ids_s + j);
-                    asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(dst), "l"(a.ids + r0 + j)
-                                 : "memory");
-                }
-            }
+            const int nch = (int)ceil_div(T.nb, tcb::kN);
+            __syncwarp();
+            if (ch == 0) copy_ids(a, T, 0);
             if constexpr (kRQ) {
-                __syncwarp();   // every lane is done with the previous chunk's copy
                 const float *src = T.fac + (int64_t)ch * tcb::kN + 4 * (slot & 31);
                 const uint32_t dst = tc::smem_u32(fs + 4 * (slot & 31));
                 asm volatile("cp.async.ca.shared.global [%0], [%1], 16;\n" ::"r"(dst), "l"(src) : "memory");
+                asm volatile("cp.async.commit_group;\n" ::: "memory");
+            }
+            if (ch + 1 < nch) copy_ids(a, T, ch + 1);
+            if constexpr (kScreen) {
+                xn = ch == 0 ? bn[0] : xn_next;
+                xn_next = ch + 1 < nch ? bn[ch + 1] : 0.f;
             }
         }
-        __device__ __forceinline__ void start(const Args &, const Tile &, int) {
-            if constexpr (kRQ || kScreen) {
-                asm volatile("cp.async.wait_all;\n" ::: "memory");
-                __syncwarp();
-            }
+        // after the accumulator wait: every group but the next chunk's ids
+        // has landed
+        __device__ __forceinline__ void start(const Args &, const Tile &T, int ch) {
+            if (ch + 1 < (int)ceil_div(T.nb, tcb::kN))
+                asm volatile("cp.async.wait_group 1;\n" ::: "memory");
+            else
+                asm volatile("cp.async.wait_group 0;\n" ::: "memory");
+            __syncwarp();
+            ids_ch = ch;
         }
         // v holds the chunk's raw accumulator values: exact, similarities x
         // 2^16; kRQ, <u - mid, q'> x 2^8 (the codes are not scaled)
@@ -393,8 +422,11 @@ __global__ void __launch_bounds__(tcp::kThreads, 1) k_scan_tc(SearchArgs a) {
     tcp::run_pipeline<ScanMode>(a, smem_raw);
 }
 
-// the kept lists
-static size_t scan_epi_bytes(int k) { return (size_t)tcp::kM * k * (sizeof(float) + sizeof(long long)); }
+// the kept lists, the factor copies (the scan over codes) and the row-id
+// buffers (two per epilogue warp)
+static size_t scan_epi_bytes(int k) {
+    return (size_t)tcp::kM * k * (sizeof(float) + sizeof(long long)) + kEpiFacBytes + kEpiIdsBytes;
+}
 
 int scan_bulk_stages(int d, int k) {
     return tcb::stages_for((int)ceil_div(d, 64), scan_epi_bytes(k), 232448 - 128);
@@ -410,10 +442,9 @@ cudaError_t prepare_scan_bulk(int d, int k, int stages) {
                                 (int)tcb::smem_bytes(stages, scan_epi_bytes(k)));
 }
 
-// the screening scan: stages of two 16 KB K-blocks (the hi halves); the
-// epilogue's bytes add one 1 KB copy of a chunk's row ids per epilogue warp
+// the screening scan: stages of two 16 KB K-blocks (the hi halves)
 constexpr int kScreenStagesMax = 6;
-static size_t scan_screen_epi_bytes(int k) { return scan_epi_bytes(k) + 4 * 1024; }
+static size_t scan_screen_epi_bytes(int k) { return scan_epi_bytes(k); }
 
 int scan_screen_stages(int d, int k) {
     return tcb::stages_for((int)ceil_div(d, 64), scan_screen_epi_bytes(k), 232448 - 128,
@@ -439,9 +470,8 @@ void enqueue_scan_bulk(const SearchArgs &a, cudaStream_t st) {
                       tcb::smem_bytes(a.tc_stages, scan_epi_bytes(a.k)), st>>>(a);
 }
 
-// the scan over codes: stages of two 16 KB K-blocks; the epilogue's bytes add
-// one 512-byte factor copy per epilogue warp
-static size_t scan_rq_epi_bytes(int k) { return scan_epi_bytes(k) + 4 * 512; }
+// the scan over codes: stages of two 16 KB K-blocks
+static size_t scan_rq_epi_bytes(int k) { return scan_epi_bytes(k); }
 
 int scan_rq_stages(int d, int k) {
     return tcb::stages_for((int)ceil_div(d, 64), scan_rq_epi_bytes(k), 232448 - 128, tcb::kStageBytesHi);

@@ -335,16 +335,26 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
         // ---------------- tile scheduler + B producer ----------------
         if (lane == 0) {
             uint32_t s = 0;
-            bool ok = true;
-            for (uint32_t i = 0; ok; ++i) {
+            // the block's i-th tile into ring slot i % kRing (t < 0: no more)
+            auto publish = [&](uint32_t i, int &t) -> bool {
                 const uint32_t slot = i % kRing, ph = (i / kRing) & 1u;
-                if (!(ok = wait(&ring_empty[slot], ph ^ 1u))) break;
-                int t = tile_counter ? atomicAdd(tile_counter, 1) : (int)(blockIdx.x + i * gridDim.x);
+                if (!wait(&ring_empty[slot], ph ^ 1u)) return false;
+                t = tile_counter ? atomicAdd(tile_counter, 1) : (int)(blockIdx.x + i * gridDim.x);
                 if (t >= n_tiles) t = -1;
                 ring_tile[slot] = t;
                 tc::mbar_arrive(&ring_full[slot]);   // release: the tile id is visible with the phase
-                if (t < 0) break;
-                const typename Mode::Tile T = Mode::tile(a, t);
+                return true;
+            };
+            int cur = -1;
+            bool ok = publish(0, cur);
+            for (uint32_t i = 0; ok && cur >= 0; ++i) {
+                // the next tile is published before this one's copies are
+                // issued: the A writers gather its rows while this tile's MMAs
+                // run, instead of after its last copy
+                int nxt = -1;
+                if (!(ok = publish(i + 1, nxt))) break;
+                const typename Mode::Tile T = Mode::tile(a, cur);
+                cur = nxt;
                 const int nch = (int)ceil_div(T.nb, kN);
                 for (int ch = 0; ok && ch < nch; ++ch) {
                     // a block's K-blocks are contiguous: a stage is one copy
