@@ -250,6 +250,21 @@ sieve_status sieve_rank_partitions(const sieve_index_view *ix, const float *Q, i
                                    int32_t nprobe, int32_t *order, float *cscores, void *ws,
                                    size_t ws_bytes, void *stream);
 
+/* The ranking's first-pass score of every (query, centroid) pair: one fp16
+ * product of the hi halves of the scaled split (hi = fp16(256 x)), summed in
+ * fp32 on the tensor cores -- the screen that bounds the exact scores before
+ * the exact pass (the paper has no counterpart: its ranking is exact; this
+ * is a diagnostic of this library's arithmetic, used to measure how much of
+ * the proven error bound the hardware uses).
+ *   ix   needs centroids, tc_centroids and d <= 256
+ *   Q    device [nq][d] fp32, 16-byte aligned
+ *   out  device [nq][ld] fp32, 16-byte aligned, ld >= nlist and a multiple
+ *        of 32; out[q][c] for c < nlist (the rest of a row is not written)
+ * Enqueued on `stream`; no workspace, nothing allocated.  SIEVE_EINVAL for a
+ * missing layout, d > 256 or a bad ld. */
+sieve_status sieve_screen_scores(const sieve_index_view *ix, const float *Q, int64_t nq,
+                                 float *out, int64_t ld, void *stream);
+
 /* Workspace bytes sieve_search needs for nq queries with these parameters.
  * host_io = 1 sizes it for sieve_search_host (adds device staging for the
  * queries and results). */

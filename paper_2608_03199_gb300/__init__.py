@@ -92,6 +92,8 @@ _SIGNATURES = {
     "sieve_rank_partitions": (C.c_int32, [C.POINTER(IndexViewC), C.c_void_p, C.c_int64, C.c_int32,
                                           C.c_void_p, C.c_void_p, C.c_void_p, C.c_size_t,
                                           C.c_void_p]),
+    "sieve_screen_scores": (C.c_int32, [C.POINTER(IndexViewC), C.c_void_p, C.c_int64, C.c_void_p,
+                                        C.c_int64, C.c_void_p]),
     "sieve_search_workspace_size": (C.c_int32, [C.POINTER(IndexViewC), C.c_int64,
                                                 C.POINTER(ParamsC), C.c_int32,
                                                 C.POINTER(C.c_size_t)]),
@@ -300,6 +302,21 @@ def rank_partitions(index: Index, Q, nprobe, return_scores=False, stream=None):
     _check(lib().sieve_rank_partitions(C.byref(v), _ptr(Q), nq, nprobe, _ptr(order), _ptr(sc),
                                        _ptr(ws), ws.numel(), _stream(stream)), "sieve_rank_partitions")
     return (order, sc) if return_scores else order
+
+
+def screen_scores(index: Index, Q, stream=None):
+    """fp32 [nq][nlist]: the ranking's first-pass (screen) score of every
+    (query, centroid) pair, one fp16 product of the hi halves summed on the
+    tensor cores (sieve_screen_scores); needs the centroids' tensor layout."""
+    _need_cuda(Q, torch.float32, "Q", 2)
+    nq = Q.shape[0]
+    nlist = index.centroids.shape[0]
+    ld = (nlist + 31) // 32 * 32
+    out = torch.empty((nq, ld), dtype=torch.float32, device=Q.device)
+    v = index.view()
+    _check(lib().sieve_screen_scores(C.byref(v), _ptr(Q), nq, _ptr(out), ld, _stream(stream)),
+           "sieve_screen_scores")
+    return out[:, :nlist]
 
 
 def _params(tau, k, nprobe, W, lookahead, loop, max_items_per_round, profile=0, scan_path="auto",

@@ -685,6 +685,22 @@ sieve_status sieve_rank_partitions(const sieve_index_view *ix, const float *Q, i
     return SIEVE_OK;
 }
 
+sieve_status sieve_screen_scores(const sieve_index_view *ix, const float *Q, int64_t nq,
+                                 float *out, int64_t ld, void *stream) {
+    sieve_status rc = check_index(ix, true);
+    if (rc != SIEVE_OK) return rc;
+    if (!ix->tc_centroids || ix->d > 256) return SIEVE_EINVAL;
+    if (nq < 0 || nq > INT32_MAX / 2) return SIEVE_EINVAL;
+    if (ld < ix->nlist || ld % 32 != 0 || ld > INT32_MAX) return SIEVE_EINVAL;
+    if (nq > 0 && (!Q || !out || !aligned16(Q) || !aligned16(out))) return SIEVE_EINVAL;
+    if ((rc = check_device()) != SIEVE_OK) return rc;
+    if (nq == 0) return SIEVE_OK;
+    SIEVE_CUDA(enqueue_screen_scores(Q, nq, ix->nlist, ix->d,
+                                     static_cast<const unsigned char *>(ix->tc_centroids), out, ld,
+                                     nullptr, static_cast<cudaStream_t>(stream)));
+    return SIEVE_OK;
+}
+
 sieve_status sieve_search_workspace_size(const sieve_index_view *ix, int64_t nq,
                                          const sieve_params *p, int32_t host_io, size_t *bytes) {
     if (!bytes) return SIEVE_EINVAL;

@@ -216,8 +216,7 @@ struct RankModeT {
             }
             float mx = v[0];
             if (ncol == 32) {
-#pragma unroll
-                for (int j = 1; j < 32; ++j) mx = fmaxf(mx, v[j]);
+                mx = max_of_32(v);
             } else {
 #pragma unroll
                 for (int j = 1; j < 32; ++j) mx = j < ncol ? fmaxf(mx, v[j]) : mx;
@@ -491,7 +490,8 @@ __device__ __forceinline__ void sort_buffer(float *bs, int *bc, int want) {
 
 // The want best of the warp's cnt entries (entry c = key[c / 32] of lane
 // c % 32, its id from id_of(c)) into bs/bc[0 .. want-1], in entry order,
-// given T and C from warp_threshold(key, want, want, ..).  C == want: every
+// given T and C from warp_threshold(key, want, want, ..); id_of(j, c) is the
+// id of entry c = j * 32 + lane.  C == want: every
 // key >= T.  Otherwise T == T* and the keys > T* plus the first keys equal to
 // it in entry order are taken, which are the lowest ids when entry order is id
 // order among equal scores.
@@ -528,7 +528,7 @@ __device__ __forceinline__ void warp_gather_exact(const uint32_t (&key)[KPL], in
             const int p = pos + __popc(sb & below);
             if (p < want) {   // exactly want are selected; the bound guards the buffer
                 bs[p] = key_score(key[j]);
-                bc[p] = id_of(c);
+                bc[p] = id_of(j, c);
             }
         }
         pos += __popc(sb);
@@ -551,7 +551,7 @@ __device__ __forceinline__ void select_candidates(const uint32_t *ck, const int 
     uint32_t T;
     int C;
     warp_threshold(key, want, want, T, C);
-    warp_gather_exact(key, n, want, T, C, [&](int c) { return ci[c]; }, bs, bc);
+    warp_gather_exact(key, n, want, T, C, [&](int, int c) { return ci[c]; }, bs, bc);
 }
 
 // The want best of the warp's cnt entries (KPL keys per lane, entry c =
@@ -583,7 +583,7 @@ __device__ __forceinline__ void select_two_step(const uint32_t (&key)[KPL], int 
         if (sel) {
             const int p = pos + __popc(sb & below);
             ck[p] = key[j];
-            ci[p] = id_of(c);
+            ci[p] = id_of(j, c);
         }
         pos += __popc(sb);
     }
@@ -595,7 +595,7 @@ __device__ __forceinline__ void select_two_step(const uint32_t (&key)[KPL], int 
         k2[j] = c < pos ? ck[c] : 0u;
     }
     warp_threshold(k2, want, want, T, C);
-    warp_gather_exact(k2, pos, want, T, C, [&](int c) { return ci[c]; }, bs, bc);
+    warp_gather_exact(k2, pos, want, T, C, [&](int, int c) { return ci[c]; }, bs, bc);
 }
 
 constexpr int kDenseK2Max = 16;   // second-step keys per lane of the dense selection
@@ -627,7 +627,7 @@ __global__ void __launch_bounds__(kSelectWarps * 32, (KPL >= 64 || R >= 8) ? 4 :
         const int c = j * 32 + lane;
         key[j] = c < cnt ? order_key(row[c]) : 0u;   // padding ranks below every score
     }
-    auto id_of = [](int c) { return c; };
+    auto id_of = [](int, int c) { return c; };
     if constexpr (KPL > kDenseK2Max) {
         select_two_step<kK2>(key, cnt, want, id_of, ck, ci, bs, bc);
     } else {

@@ -132,6 +132,11 @@ cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t 
 int rank_tc_mma_launches(int64_t nq, int64_t nlist, int nprobe, int d, int64_t plan_nq,
                          bool bulk);   // contraction launches
 int rank_screen_stages(int d);                   // 0 when the screening first pass does not apply
+// the first pass's one-product score of every (query, centroid) pair into
+// out[q * ld + c] (ld a multiple of 32, out 16-byte aligned, d <= 256)
+cudaError_t enqueue_screen_scores(const float *Q, int64_t nq, int64_t nlist, int d,
+                                  const unsigned char *tc_cent, float *out, int64_t ld,
+                                  int *status, cudaStream_t st);
 int rank_bulk_stages(int d);                     // 0 when the bulk ranking does not apply
 
 // in-call window calibration (calibrate.cu)
