@@ -63,6 +63,25 @@ __device__ __forceinline__ float pick32(const float (&v)[32], int j) {
     return (j & 1) ? t1 : t0;
 }
 
+// max(a, b, c) in one instruction (the three-input form of max.f32 on
+// sm_100-family GPUs); a NaN input is ignored as by fmaxf
+__device__ __forceinline__ float fmax3f(float a, float b, float c) {
+    float r;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+    return r;
+}
+
+// the largest of 32 values: a tree of three-input maxima (16 instructions)
+__device__ __forceinline__ float max_of_32(const float (&v)[32]) {
+    float t[11];
+#pragma unroll
+    for (int i = 0; i < 10; ++i) t[i] = fmax3f(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
+    t[10] = fmaxf(v[30], v[31]);
+    const float u0 = fmax3f(t[0], t[1], t[2]), u1 = fmax3f(t[3], t[4], t[5]),
+                u2 = fmax3f(t[6], t[7], t[8]), u3 = fmaxf(t[9], t[10]);
+    return fmaxf(fmax3f(u0, u1, u2), u3);
+}
+
 // 16-byte global->shared async copy; src_bytes = 0 zero-fills the destination.
 __device__ __forceinline__ void cp_async16(void *smem_dst, const void *gmem_src, int src_bytes) {
     unsigned dst = static_cast<unsigned>(__cvta_generic_to_shared(smem_dst));

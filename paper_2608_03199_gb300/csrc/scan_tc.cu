@@ -181,14 +181,7 @@ struct ScanModeT {
             float thr = a.tau * scale;
             if (kn == a.k) thr = fmaxf(thr, wst_s * scale);
             // nearly every group has no candidate: one tree of maxima decides
-            float mx[16];
-#pragma unroll
-            for (int j = 0; j < 16; ++j) mx[j] = fmaxf(e[j], e[j + 16]);
-#pragma unroll
-            for (int w = 8; w > 0; w >>= 1)
-#pragma unroll
-                for (int j = 0; j < w; ++j) mx[j] = fmaxf(mx[j], mx[j + w]);
-            if (!(mx[0] >= thr)) return;
+            if (!(max_of_32(e) >= thr)) return;
             unsigned m = 0;
 #pragma unroll
             for (int j = 0; j < 32; ++j) m |= (e[j] >= thr && j < ncol) ? (1u << j) : 0u;
@@ -213,14 +206,7 @@ struct ScanModeT {
             float thr = a.tau;
             if (kn == a.k) thr = fmaxf(thr, wst_s);
             const float cut = (thr - (m_rel * qn * xn + m_abs * (qn + xn))) * 65536.f;
-            float mx[16];
-#pragma unroll
-            for (int j = 0; j < 16; ++j) mx[j] = fmaxf(v[j], v[j + 16]);
-#pragma unroll
-            for (int w = 8; w > 0; w >>= 1)
-#pragma unroll
-                for (int j = 0; j < w; ++j) mx[j] = fmaxf(mx[j], mx[j + w]);
-            const bool any = valid && mx[0] >= cut;
+            const bool any = valid && max_of_32(v) >= cut;
             if (!__any_sync(0xffffffffu, any)) return;
             unsigned m = 0;
             if (any) {

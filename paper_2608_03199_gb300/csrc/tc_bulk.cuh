@@ -174,6 +174,57 @@ __device__ __forceinline__ void hand(Epi &epi, const Args &a, const Tile &T, int
     epi.chunk(a, T, col0, v, left < 32 ? (int)left : 32);
 }
 
+// The MMAs of one B stage for one sub-tile, fully unrolled: K1 K steps of 16
+// in the stage's first K-block and K2 in its second (0: none).  a0 = the
+// sub-tile's A columns of that first K-block (hi; lo 32 columns on), b0 = the
+// shared-memory descriptor of the stage's first K-block; a K step moves A by
+// 8 columns and B's start address by 32 bytes (2 in the descriptor's 16-byte
+// units; shared addresses stay below the field's 2^14 limit, so no carry).
+// acc_first: whether the first MMA accumulates (0 at a chunk's first K step).
+// One straight run of MMAs with their operands a constant off two bases: the
+// single issuing thread keeps up with the tensor pipe.
+template <int kProd, int K1, int K2>
+__device__ __forceinline__ void issue_stage(uint32_t dt, uint32_t a0, uint64_t b0, uint32_t acc_first,
+                                            uint32_t idesc) {
+    constexpr uint32_t kAKbT = kProd == 1 ? 32 : 64;                       // A columns per K-block
+    constexpr uint64_t kKbDesc = (kProd == 3 ? kKbBytes : kKbBytesHi) >> 4;  // B K-block in 16-byte units
+    constexpr uint64_t kLoDesc = (kKbBytes / 2) >> 4;                        // hi to lo of a split K-block
+#pragma unroll
+    for (int j = 0; j < K1 + K2; ++j) {
+        const int kb = j < K1 ? 0 : 1, ks = j < K1 ? j : j - K1;
+        const uint32_t a = a0 + (uint32_t)kb * kAKbT + (uint32_t)ks * 8u;
+        const uint64_t bh = b0 + (uint64_t)kb * kKbDesc + 2u * (uint64_t)ks;
+        const uint32_t acc = j == 0 ? acc_first : 1u;
+        if constexpr (kProd == 3) {        // lo_a hi_b + hi_a lo_b + hi_a hi_b
+            tc::mma_f16_ta(dt, a + 32u, bh, idesc, acc);
+            tc::mma_f16_ta(dt, a, bh + kLoDesc, idesc, 1u);
+            tc::mma_f16_ta(dt, a, bh, idesc, 1u);
+        } else if constexpr (kProd == 2) { // B exact in fp16: lo_a b + hi_a b
+            tc::mma_f16_ta(dt, a + 32u, bh, idesc, acc);
+            tc::mma_f16_ta(dt, a, bh, idesc, 1u);
+        } else {                           // a screen: hi_a hi_b
+            tc::mma_f16_ta(dt, a, bh, idesc, acc);
+        }
+    }
+}
+
+// issue_stage for a run-time K-step pattern: a stage's first K-block has k1
+// steps (1..4) and its second k2 (0..4, only after a full first block)
+template <int kProd>
+__device__ __forceinline__ void issue_stage_rt(int k1, int k2, uint32_t dt, uint32_t a0, uint64_t b0,
+                                               uint32_t acc_first, uint32_t idesc) {
+    switch (k1 * 8 + k2) {
+        case 4 * 8 + 4: issue_stage<kProd, 4, 4>(dt, a0, b0, acc_first, idesc); break;
+        case 4 * 8 + 3: issue_stage<kProd, 4, 3>(dt, a0, b0, acc_first, idesc); break;
+        case 4 * 8 + 2: issue_stage<kProd, 4, 2>(dt, a0, b0, acc_first, idesc); break;
+        case 4 * 8 + 1: issue_stage<kProd, 4, 1>(dt, a0, b0, acc_first, idesc); break;
+        case 4 * 8 + 0: issue_stage<kProd, 4, 0>(dt, a0, b0, acc_first, idesc); break;
+        case 3 * 8 + 0: issue_stage<kProd, 3, 0>(dt, a0, b0, acc_first, idesc); break;
+        case 2 * 8 + 0: issue_stage<kProd, 2, 0>(dt, a0, b0, acc_first, idesc); break;
+        default: issue_stage<kProd, 1, 0>(dt, a0, b0, acc_first, idesc); break;
+    }
+}
+
 // Mode provides (in addition to what tc_pipeline.cuh asks): Epi::prefetch(a,
 // T, ch) and Epi::start(a, T, ch), called by every epilogue lane of a warp
 // before and after the wait for chunk ch's accumulator; b_block(a, T, ch)
@@ -258,6 +309,10 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
     const uint32_t tA = tmem + nacc * kN;                      // A after the accumulators
 
     auto wait_n = [&](uint64_t *bar, uint32_t parity, uint32_t polls) -> bool {
+        // a phase that has completed already is seen by a non-blocking test:
+        // a (blocking) try_wait costs about 200 cycles of the waiting thread
+        // even then, which the single MMA-issuing thread cannot afford
+        if (tc::mbar_test_wait(bar, parity)) return true;
         // a shortened limit polls without blocking (try_wait may suspend the
         // thread for a hardware-chosen time, which would stretch the limit)
         const bool quick = polls < kWaitPolls;
@@ -388,6 +443,10 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
         if (lane == 0) {
             uint32_t s = 0, c = 0, u = 0;   // c: accumulator uses, kSub per chunk
             bool ok = true;
+            // the descriptor of stage 0's first K-block; stage st is st * kStage
+            // bytes on (the start-address field does not carry: shared
+            // addresses stay below 2^18)
+            const uint64_t b_desc0 = tc::desc_k_sw128(tc::smem_u32(Bst));
             for (uint32_t i = 0; ok; ++i) {
                 const uint32_t slot = i % kRing, rph = (i / kRing) & 1u;
                 if (!(ok = wait(&ring_full[slot], rph))) break;
@@ -410,6 +469,11 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                             for (int kb = kb0; ok && kb < kb1; ++kb) ok = wait(&a_full[kb], u & 1u);
                         if (!ok || !(ok = wait(&b_full[st], ph))) break;
                         tc::fence_after_sync();
+                        // K steps of 16 that hold any of the d elements (the rest of
+                        // the last K-block is zero padding), per K-block of the stage
+                        const int k1 = d - kb0 * 64 >= 64 ? 4 : (d - kb0 * 64 + 15) / 16;
+                        const int k2 = kb1 - kb0 < 2 ? 0 : d - (kb0 + 1) * 64 >= 64 ? 4 : (d - (kb0 + 1) * 64 + 15) / 16;
+                        const uint64_t b_stage = b_desc0 + (uint64_t)st * (kStage >> 4);
 #pragma unroll 1
                         for (int h = 0; ok && h < kSub; ++h) {
                             if (kSub > 1 && kb0 == 0) {   // sub-tile h's accumulator, just before its MMAs
@@ -417,46 +481,8 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                                 tc::fence_after_sync();
                             }
                             const uint32_t dt = tmem + ((c + h) % nacc) * kN;
-                            for (int kb = kb0; kb < kb1; ++kb) {
-                                // K steps of 16 that hold any of the d elements: the
-                                // rest of the last K-block is zero padding
-                                const int kst = d - kb * 64 >= 64 ? 4 : (d - kb * 64 + 15) / 16;
-                                const uint32_t a_hi = tA + (uint32_t)h * aTile + (uint32_t)kb * kAKb,
-                                               a_lo = a_hi + 32;
-                                const uint32_t b_hi = tc::smem_u32(Bst + (size_t)st * kStage) +
-                                                      (uint32_t)(kb - kb0) * kKbB;
-                                // a K step moves the descriptors' start address by 32 bytes
-                                // (2 in its 16-byte units; shared addresses stay far below
-                                // the field's 2^14 limit, so no carry)
-                                const uint64_t bh = tc::desc_k_sw128(b_hi);
-                                if constexpr (kLo) {
-                                    const uint64_t bl = tc::desc_k_sw128(b_hi + kKbBytes / 2);
-#pragma unroll
-                                    for (int ks = 0; ks < 4; ++ks) {   // K = 16: 8 columns of A, 32 bytes of B
-                                        if (ks >= kst) break;
-                                        const uint32_t ao = ks * 8;
-                                        const uint64_t bo = 2 * ks;
-                                        tc::mma_f16_ta(dt, a_lo + ao, bh + bo, kIdesc, (kb > 0 || ks > 0) ? 1u : 0u);
-                                        tc::mma_f16_ta(dt, a_hi + ao, bl + bo, kIdesc, 1u);
-                                        tc::mma_f16_ta(dt, a_hi + ao, bh + bo, kIdesc, 1u);
-                                    }
-                                } else if constexpr (kProd == 2) {   // B exact in fp16: hi and lo of A against it
-#pragma unroll
-                                    for (int ks = 0; ks < 4; ++ks) {
-                                        if (ks >= kst) break;
-                                        const uint32_t ao = ks * 8;
-                                        const uint64_t bo = 2 * ks;
-                                        tc::mma_f16_ta(dt, a_lo + ao, bh + bo, kIdesc, (kb > 0 || ks > 0) ? 1u : 0u);
-                                        tc::mma_f16_ta(dt, a_hi + ao, bh + bo, kIdesc, 1u);
-                                    }
-                                } else {   // a screen: the hi halves alone
-#pragma unroll
-                                    for (int ks = 0; ks < 4; ++ks)
-                                        if (ks < kst)
-                                            tc::mma_f16_ta(dt, a_hi + ks * 8, bh + 2 * ks, kIdesc,
-                                                           (kb > 0 || ks > 0) ? 1u : 0u);
-                                }
-                            }
+                            issue_stage_rt<kProd>(k1, k2, dt, tA + (uint32_t)h * aTile + (uint32_t)kb0 * kAKb,
+                                                  b_stage, kb0 > 0 ? 1u : 0u, kIdesc);
                             // with two sub-tiles, the first sub-tile's accumulator is
                             // handed over before the second's MMAs are issued
                             if (kSub > 1 && last && h + 1 < kSub) tc::mma_commit(&dfull_bar[(c + h) % nacc]);

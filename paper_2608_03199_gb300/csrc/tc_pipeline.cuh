@@ -145,6 +145,9 @@ __device__ __forceinline__ void run_pipeline(const typename Mode::Args &a, unsig
 
     // bounded wait; gives up early once another role has aborted
     auto wait = [&](uint64_t *bar, uint32_t parity) -> bool {
+        // a completed phase is seen by a non-blocking test (a blocking
+        // try_wait costs about 200 cycles even then)
+        if (tc::mbar_test_wait(bar, parity)) return true;
         for (uint32_t it = 0; it < kWaitPolls; ++it) {
             if (tc::mbar_try_wait(bar, parity)) return true;
             if ((it & 255u) == 255u && *(volatile int *)&s_abort) return false;

@@ -171,6 +171,7 @@ __device__ __forceinline__ bool mbar_test_wait(uint64_t *mbar, uint32_t parity) 
 // time).  Returns false on giving up.
 __device__ __forceinline__ bool mbar_wait_bounded(uint64_t *mbar, uint32_t parity,
                                                   uint32_t limit) {
+    if (mbar_test_wait(mbar, parity)) return true;   // done already: no blocking try_wait
     for (uint32_t it = 0; it < limit; ++it)
         if (mbar_try_wait(mbar, parity)) return true;
     return false;
