@@ -71,8 +71,8 @@ def parse():
     ap.add_argument("--scan-path", choices=("auto", "simt", "tensor", "screen"), default="auto",
                     help="which units score the partition groups (sieve_params.scan_path: "
                          "tensor = three fp16 products per pair, screen = one product per pair "
-                         "and an fp32 rescore of the candidates, auto = the screen from a "
-                         "window of 16 up)")
+                         "and an fp32 rescore of the candidates, auto = the screen from "
+                         "tau 0.85 up, at a window of 16 or d >= 192)")
     ap.add_argument("--rq", action="store_true",
                     help="the quantized local search (RaBitQ-style 7-bit codes) on the workload")
     ap.add_argument("--ncu-case", choices=("w8", "fixed", "rqw8", "rank"), default=None,
@@ -197,10 +197,10 @@ def committed_traffic(kernel, workload, launches):
 
 def uses_screen(args, cfg, W, bulk, tau=None):
     """Whether the bulk scan screens (sieve_params.scan_path; the automatic
-    path screens from a window of 16 up when tau >= 0.85)."""
+    path screens when tau >= 0.85, from a window of 16 up or at d >= 192)."""
     tau = cfg.tau if tau is None else tau
     return bulk and (args.scan_path == "screen" or
-                     (args.scan_path == "auto" and min(W, cfg.nprobe) >= 16 and tau >= 0.85))
+                     (args.scan_path == "auto" and (min(W, cfg.nprobe) >= 16 or cfg.d >= 192) and tau >= 0.85))
 
 
 def rank_passes(cfg, bulk):

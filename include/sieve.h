@@ -118,8 +118,8 @@ typedef struct {
  *              tensor cores when the epilogue's k-lists fit: any k with
  *              the tensor-core layout and d <= 256, k <= 22 otherwise; FP32
  *              FMA beyond; with the tensor-core layout the screen below
- *              when min(W, nprobe) >= 16 and tau >= 0.85, three products
- *              per pair otherwise),
+ *              when tau >= 0.85 and min(W, nprobe) >= 16 or d >= 192,
+ *              three products per pair otherwise),
  *              1 = FP32 FMA only, 2 = tensor cores, three products per pair
  *              (SIEVE_EINVAL where they do not fit), 3 = as 2, but with the
  *              tensor-core layout every pair is screened.

@@ -69,7 +69,8 @@ sieve_status check_params(const sieve_index_view *ix, const sieve_params *p) {
     return SIEVE_OK;
 }
 
-constexpr int kScreenMinWindow = 16;   // automatic scan path: the screen from this window up ...
+constexpr int kScreenMinWindow = 16;   // automatic scan path: the screen from this window up
+constexpr int kScreenMinD = 192;       // ... or at any window from this d up ...
 constexpr float kScreenMinTau = 0.85f; // ... and this threshold up (below it nearly every row
                                        // of a probed partition needs its fp32 rescore)
 constexpr int64_t kAutoCapMax = int64_t(1) << 24;
@@ -394,11 +395,14 @@ sieve_status search_device(const sieve_index_view *ix, const float *Q, int64_t n
     // The screen pays per candidate (an fp32 rescore) and saves per pair, so
     // it wins when a round scans many partitions per qualifying row: on the
     // 1M x 256 workload a window of 64 ran 25% faster, one of 8 the same.
-    // Automatic: the screen from a window of 16 up; 2 = three products, 3 =
-    // the screen.
+    // At small d the three-product scan is bound by its per-chunk overheads
+    // rather than the tensor pipe, and screening saves nothing (100M x 96,
+    // W = 8: the same time); from d = 192 a window of 8 ran 3% (1M x 256) and
+    // 10% (10M x 256) faster screened.  Automatic: the screen from tau 0.85
+    // up, at a window of 16 or d >= 192; 2 = three products, 3 = the screen.
     const bool with_layout = a.tc_rows && a.tc_row_blocks;
     const bool screen = with_layout && (p->scan_path == 3 ||
-                                        (p->scan_path == 0 && std::min(p->W, p->nprobe) >= kScreenMinWindow &&
+                                        (p->scan_path == 0 && (std::min(p->W, p->nprobe) >= kScreenMinWindow || ix->d >= kScreenMinD) &&
                                          p->tau >= kScreenMinTau));
     const int bulk_stages = !with_layout ? 0
                             : screen    ? scan_screen_stages(ix->d, p->k)

@@ -32,7 +32,7 @@ def test_bruteforce_recall_against_the_oracle():
 
 
 def test_automatic_scan_rule():
-    cfg = types.SimpleNamespace(nprobe=64, tau=0.9)
+    cfg = types.SimpleNamespace(nprobe=64, tau=0.9, d=96)
     auto = types.SimpleNamespace(scan_path="auto")
     assert not bench.uses_screen(auto, cfg, 8, True)
     assert bench.uses_screen(auto, cfg, 16, True)
@@ -40,8 +40,12 @@ def test_automatic_scan_rule():
     assert not bench.uses_screen(auto, cfg, 64, False)          # no tensor layout
     assert bench.uses_screen(types.SimpleNamespace(scan_path="screen"), cfg, 8, True)
     assert not bench.uses_screen(types.SimpleNamespace(scan_path="tensor"), cfg, 64, True)
-    assert not bench.uses_screen(auto, types.SimpleNamespace(nprobe=12, tau=0.9), 64, True)
+    assert not bench.uses_screen(auto, types.SimpleNamespace(nprobe=12, tau=0.9, d=96), 64, True)
     assert not bench.uses_screen(auto, cfg, 64, True, tau=0.5)       # loose threshold
+    wide = types.SimpleNamespace(nprobe=64, tau=0.9, d=256)         # d >= 192: at any window
+    assert bench.uses_screen(auto, wide, 8, True)
+    assert bench.uses_screen(auto, wide, 2, True)
+    assert not bench.uses_screen(auto, wide, 8, True, tau=0.5)
 
 
 def test_cpu_baseline_times_both_modes():

@@ -1,5 +1,5 @@
 """The screening scan (scan_path "screen", and the automatic path from a
-window of 16 up, with the tensor-core layout): one fp16 product of the hi
+window of 16 up or at d >= 192, from tau 0.85 up, with the tensor-core layout): one fp16 product of the hi
 halves per (query, row) pair bounds every score, and only the rows whose
 bound reaches the threshold are scored again in fp32.
 
