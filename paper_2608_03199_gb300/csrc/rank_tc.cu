@@ -279,6 +279,12 @@ struct RankModeT {
 struct RankScreenMode : RankModeT<kRankGroupMax, 2> {
     static constexpr int kProducts = 1;
 };
+// d <= 128: chunks of 192 centroids (MMA N = 192), two sub-tiles' A and two
+// 192-column accumulators filling tensor memory; a third fewer MMA
+// instructions per score than 128-centroid chunks
+struct RankScreen192Mode : RankScreenMode {
+    static constexpr int kNB = 192;
+};
 static_assert(kTcRows == RankModeT<kRankStream>::kN, "");
 
 template <int kMode>
@@ -315,14 +321,25 @@ int rank_pair_stages(int d) {
     return tcb::sub_fits(nkb, 3, 2) ? tcb::stages_for(nkb, 0, 232448 - 128) : 0;
 }
 
+// whether the screen takes 192-centroid chunks (d <= 128), and its B stage bytes
+static bool screen_wide(int d) { return ceil_div(d, 64) <= 2; }
+static uint32_t screen_stage_bytes(int d) {
+    return screen_wide(d) ? tcb::kStageBytesHi / tcb::kN * 192 : tcb::kStageBytesHi;
+}
+
 int rank_screen_stages(int d) {
     const int nkb = (int)ceil_div(d, 64);
-    return tcb::sub_fits(nkb, 1, 2) ? tcb::stages_for(nkb, 0, 232448 - 128, tcb::kStageBytesHi) : 0;
+    return tcb::sub_fits(nkb, 1, 2) ? tcb::stages_for(nkb, 0, 232448 - 128, screen_stage_bytes(d)) : 0;
 }
 
 __global__ void __launch_bounds__(tcb::kThreads, 1) k_rank_screen(RankArgs a, int stages) {
     extern __shared__ unsigned char smem_raw[];
     tcb::run_bulk<RankScreenMode>(a, smem_raw, stages);
+}
+
+__global__ void __launch_bounds__(tcb::kThreads, 1) k_rank_screen192(RankArgs a, int stages) {
+    extern __shared__ unsigned char smem_raw[];
+    tcb::run_bulk<RankScreen192Mode>(a, smem_raw, stages);
 }
 
 constexpr int kSelectWarps = 4;  // warps (queries) per block of the final selection
@@ -948,8 +965,9 @@ cudaError_t prepare_rank_tc(int nprobe, int d) {
                                  (int)tcb::smem_bytes(pair, 0));
     const int scr = rank_screen_stages(d);
     if (e == cudaSuccess && scr)
-        e = cudaFuncSetAttribute(k_rank_screen, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)tcb::smem_bytes(scr, 0, tcb::kStageBytesHi));
+        e = cudaFuncSetAttribute(screen_wide(d) ? k_rank_screen192 : k_rank_screen,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)tcb::smem_bytes(scr, 0, screen_stage_bytes(d)));
     if (e == cudaSuccess) e = set_final_attr<2>();
     if (e == cudaSuccess) e = set_final_attr<4>();
     if (e == cudaSuccess) e = set_final_attr<8>();
@@ -1090,7 +1108,10 @@ cudaError_t enqueue_rank_tc(const float *Q, int64_t nq, const float *C, int64_t 
         const int tiles = (int)(ceil_div(n, (two ? 2 : 1) * tcp::kM) * L.nranges);
         const unsigned grid = (unsigned)std::min(tiles, num_sms());
         const size_t bsm = tcb::smem_bytes(bulk_stages, kRankEpiBytes);
-        if (scr)
+        if (scr && screen_wide(d))
+            k_rank_screen192<<<grid, tcb::kThreads, tcb::smem_bytes(screen_stages, 0, screen_stage_bytes(d)),
+                               st>>>(a, screen_stages);
+        else if (scr)
             k_rank_screen<<<grid, tcb::kThreads, tcb::smem_bytes(screen_stages, 0, tcb::kStageBytesHi),
                             st>>>(a, screen_stages);
         else if (mode == kRankStreamInit && pair_stages)

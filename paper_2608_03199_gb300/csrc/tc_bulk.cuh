@@ -119,6 +119,17 @@ struct mma_products { static constexpr int value = b_has_lo<Mode>::value ? 3 : 2
 template <class Mode>
 struct mma_products<Mode, decltype((void)Mode::kProducts)> { static constexpr int value = Mode::kProducts; };
 
+// B rows per chunk (the MMA's N): Mode::kNB if given, else 128 (one block of
+// the tensor layout).  192 is for a screen of two sub-tiles at d <= 128: its
+// A (2 x 64 columns) and two 192-column accumulators fill tensor memory, and
+// each MMA instruction covers half as many columns again -- the issuing
+// thread, not the tensor pipe, bounds such a screen.  A 192-row chunk spans
+// two layout blocks: rows 0-127 or 64-127 of one and the start of the next.
+template <class Mode, class = void>
+struct chunk_rows { static constexpr int value = kN; };
+template <class Mode>
+struct chunk_rows<Mode, decltype((void)Mode::kNB)> { static constexpr int value = Mode::kNB; };
+
 // sub-tiles of 128 A rows per tile: Mode::kSub if given (1 or 2), else 1
 template <class Mode, class = void>
 struct sub_tiles { static constexpr int value = 1; };
@@ -183,11 +194,11 @@ __device__ __forceinline__ void hand(Epi &epi, const Args &a, const Tile &T, int
 // acc_first: whether the first MMA accumulates (0 at a chunk's first K step).
 // One straight run of MMAs with their operands a constant off two bases: the
 // single issuing thread keeps up with the tensor pipe.
-template <int kProd, int K1, int K2>
+template <int kProd, int K1, int K2, uint32_t kKbStageBytes>
 __device__ __forceinline__ void issue_stage(uint32_t dt, uint32_t a0, uint64_t b0, uint32_t acc_first,
                                             uint32_t idesc) {
     constexpr uint32_t kAKbT = kProd == 1 ? 32 : 64;                       // A columns per K-block
-    constexpr uint64_t kKbDesc = (kProd == 3 ? kKbBytes : kKbBytesHi) >> 4;  // B K-block in 16-byte units
+    constexpr uint64_t kKbDesc = kKbStageBytes >> 4;                         // B K-block in 16-byte units
     constexpr uint64_t kLoDesc = (kKbBytes / 2) >> 4;                        // hi to lo of a split K-block
 #pragma unroll
     for (int j = 0; j < K1 + K2; ++j) {
@@ -210,18 +221,19 @@ __device__ __forceinline__ void issue_stage(uint32_t dt, uint32_t a0, uint64_t b
 
 // issue_stage for a run-time K-step pattern: a stage's first K-block has k1
 // steps (1..4) and its second k2 (0..4, only after a full first block)
-template <int kProd>
+template <int kProd, uint32_t kKbStageBytes>
 __device__ __forceinline__ void issue_stage_rt(int k1, int k2, uint32_t dt, uint32_t a0, uint64_t b0,
                                                uint32_t acc_first, uint32_t idesc) {
+    constexpr uint32_t B = kKbStageBytes;
     switch (k1 * 8 + k2) {
-        case 4 * 8 + 4: issue_stage<kProd, 4, 4>(dt, a0, b0, acc_first, idesc); break;
-        case 4 * 8 + 3: issue_stage<kProd, 4, 3>(dt, a0, b0, acc_first, idesc); break;
-        case 4 * 8 + 2: issue_stage<kProd, 4, 2>(dt, a0, b0, acc_first, idesc); break;
-        case 4 * 8 + 1: issue_stage<kProd, 4, 1>(dt, a0, b0, acc_first, idesc); break;
-        case 4 * 8 + 0: issue_stage<kProd, 4, 0>(dt, a0, b0, acc_first, idesc); break;
-        case 3 * 8 + 0: issue_stage<kProd, 3, 0>(dt, a0, b0, acc_first, idesc); break;
-        case 2 * 8 + 0: issue_stage<kProd, 2, 0>(dt, a0, b0, acc_first, idesc); break;
-        default: issue_stage<kProd, 1, 0>(dt, a0, b0, acc_first, idesc); break;
+        case 4 * 8 + 4: issue_stage<kProd, 4, 4, B>(dt, a0, b0, acc_first, idesc); break;
+        case 4 * 8 + 3: issue_stage<kProd, 4, 3, B>(dt, a0, b0, acc_first, idesc); break;
+        case 4 * 8 + 2: issue_stage<kProd, 4, 2, B>(dt, a0, b0, acc_first, idesc); break;
+        case 4 * 8 + 1: issue_stage<kProd, 4, 1, B>(dt, a0, b0, acc_first, idesc); break;
+        case 4 * 8 + 0: issue_stage<kProd, 4, 0, B>(dt, a0, b0, acc_first, idesc); break;
+        case 3 * 8 + 0: issue_stage<kProd, 3, 0, B>(dt, a0, b0, acc_first, idesc); break;
+        case 2 * 8 + 0: issue_stage<kProd, 2, 0, B>(dt, a0, b0, acc_first, idesc); break;
+        default: issue_stage<kProd, 1, 0, B>(dt, a0, b0, acc_first, idesc); break;
     }
 }
 
@@ -234,10 +246,12 @@ __device__ __forceinline__ void issue_stage_rt(int k1, int k2, uint32_t dt, uint
 template <class Mode>
 __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned char *smem_raw,
                                          int stages) {
-    constexpr uint32_t kIdesc = tc::idesc_f16(tcp::kM, kN);
+    constexpr int kNB = chunk_rows<Mode>::value;               // B rows per chunk = MMA N
+    constexpr uint32_t kIdesc = tc::idesc_f16(tcp::kM, kNB);
     constexpr int kProd = mma_products<Mode>::value;
     constexpr bool kLo = kProd == 3;                          // B's lo half in the stage
-    constexpr uint32_t kKbB = kLo ? kKbBytes : kKbBytesHi;     // bytes of one K-block of B
+    // bytes of one K-block of B in a stage (kNB rows)
+    constexpr uint32_t kKbB = (kLo ? kKbBytes : kKbBytesHi) / kN * kNB;
     // bytes of one K-block of B in global memory: a screen copies the hi half
     // of each K-block of the split layout, one copy per K-block
     constexpr uint32_t kSrcKb = b_has_lo<Mode>::value ? kKbBytes : kKbBytesHi;
@@ -248,6 +262,8 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
     constexpr uint32_t kStage = kKs * kKbB;                    // bytes of one B stage
     constexpr int kSub = sub_tiles<Mode>::value;
     static_assert(kSub == 1 || kSub == 2, "one or two sub-tiles");
+    static_assert(kNB == kN || (kNB == 192 && kProd == 1 && kSub == 2 && kSrcKb == kKbBytes),
+                  "192-row chunks: a screen of two sub-tiles over the split layout");
     // warp roles: A writers, producer, MMA issuer, epilogue (4 warps per sub-tile)
     constexpr int kAW = kSub == 1 ? kAWriterWarps : 4;
     constexpr int kAWGroups = kAW / 4;                         // K-block classes of A writers
@@ -270,7 +286,8 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
     int *status = Mode::status(a);
     // a d whose A does not fit tensor memory (the host never launches one):
     // report it and leave before any barrier or tensor memory is set up
-    if (!sub_fits(nkb, kProd, kSub)) {
+    if (!sub_fits(nkb, kProd, kSub) ||
+        (uint32_t)kSub * a_cols(nkb, kProd) + 2u * (uint32_t)kNB > kTmemCols) {
         if (threadIdx.x == 0) atomicExch(status, SIEVE_EINVAL);
         return;
     }
@@ -306,7 +323,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
     __syncthreads();
     tc::fence_after_sync();
     const uint32_t tmem = tmem_slot;
-    const uint32_t tA = tmem + nacc * kN;                      // A after the accumulators
+    const uint32_t tA = tmem + nacc * kNB;                     // A after the accumulators
 
     auto wait_n = [&](uint64_t *bar, uint32_t parity, uint32_t polls) -> bool {
         // a phase that has completed already is seen by a non-blocking test:
@@ -410,8 +427,37 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                 if (!(ok = publish(i + 1, nxt))) break;
                 const typename Mode::Tile T = Mode::tile(a, cur);
                 cur = nxt;
-                const int nch = (int)ceil_div(T.nb, kN);
+                const int nch = (int)ceil_div(T.nb, kNB);
+                const int nblk = (int)ceil_div(T.nb, kN);             // layout blocks of the tile's B
                 for (int ch = 0; ok && ch < nch; ++ch) {
+                    if constexpr (kNB != kN) {
+                        // a 192-row chunk: rows r0 .. r0 + 191 of the tile's B, from
+                        // block r0 / 128 (from its row r0 % 128) and the next block
+                        // (while it exists: rows past the tile's blocks are not
+                        // copied, and their columns are never read); the hi half of
+                        // each K-block, rows at 128 bytes, lands at the chunk row
+                        const int r0 = ch * kNB, b0 = r0 / kN, o0 = r0 % kN;
+                        const uint32_t n0 = (uint32_t)(kN - o0);
+                        const uint32_t n1 = b0 + 1 < nblk ? (uint32_t)kNB - n0 : 0u;
+                        const unsigned char *p0 = Mode::b_block(a, T, b0);
+                        const unsigned char *p1 = n1 ? Mode::b_block(a, T, b0 + 1) : nullptr;
+                        for (int kb = 0; kb < nkb; kb += kKs) {
+                            const uint32_t st = s % stages, sph = (s / stages) & 1u;
+                            const int nk = nkb - kb < kKs ? nkb - kb : kKs;
+                            if (!(ok = wait(&b_empty[st], sph ^ 1u))) break;
+                            tc::mbar_arrive_expect_tx(&b_full[st], (uint32_t)nk * (n0 + n1) * 128u);
+                            for (int j = 0; j < nk; ++j) {
+                                unsigned char *dst = Bst + (size_t)st * kStage + (size_t)j * kKbB;
+                                tc::bulk_g2s(dst, p0 + (size_t)(kb + j) * kSrcKb + (size_t)o0 * 128u, n0 * 128u,
+                                             &b_full[st]);
+                                if (n1)
+                                    tc::bulk_g2s(dst + (size_t)n0 * 128u, p1 + (size_t)(kb + j) * kSrcKb, n1 * 128u,
+                                                 &b_full[st]);
+                            }
+                            ++s;
+                        }
+                        continue;
+                    }
                     // a block's K-blocks are contiguous: a stage is one copy
                     const unsigned char *src = Mode::b_block(a, T, ch);
                     for (int kb = 0; kb < nkb; kb += kKs) {
@@ -454,7 +500,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                 tc::mbar_arrive(&ring_empty[slot]);
                 if (t < 0) break;
                 const typename Mode::Tile T = Mode::tile(a, t);
-                const int nch = (int)ceil_div(T.nb, kN);
+                const int nch = (int)ceil_div(T.nb, kNB);
                 if (nch == 0) continue;
                 for (int ch = 0; ok && ch < nch; ++ch, c += kSub) {
                     if constexpr (kSub == 1) {   // the chunk's accumulator
@@ -480,9 +526,9 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                                 if (!(ok = wait(&dempty_bar[(c + h) % nacc], (((c + h) / nacc) & 1u) ^ 1u))) break;
                                 tc::fence_after_sync();
                             }
-                            const uint32_t dt = tmem + ((c + h) % nacc) * kN;
-                            issue_stage_rt<kProd>(k1, k2, dt, tA + (uint32_t)h * aTile + (uint32_t)kb0 * kAKb,
-                                                  b_stage, kb0 > 0 ? 1u : 0u, kIdesc);
+                            const uint32_t dt = tmem + ((c + h) % nacc) * kNB;
+                            issue_stage_rt<kProd, kKbB>(k1, k2, dt, tA + (uint32_t)h * aTile + (uint32_t)kb0 * kAKb,
+                                                        b_stage, kb0 > 0 ? 1u : 0u, kIdesc);
                             // with two sub-tiles, the first sub-tile's accumulator is
                             // handed over before the second's MMAs are issued
                             if (kSub > 1 && last && h + 1 < kSub) tc::mma_commit(&dfull_bar[(c + h) % nacc]);
@@ -515,7 +561,7 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
             int t;
             if (!ring_take_warp(i, t) || t < 0) break;
             const typename Mode::Tile T = Mode::tile(a, t);
-            const int nch = (int)ceil_div(T.nb, kN);
+            const int nch = (int)ceil_div(T.nb, kNB);
             epi.begin(a, T, slot, epi_smem);
             for (int ch = 0; ch < nch; ++ch, c += kSub) {
                 const uint32_t buf = c % nacc, dph = (c / nacc) & 1u;
@@ -524,26 +570,25 @@ __device__ __forceinline__ void run_bulk(const typename Mode::Args &a, unsigned 
                 if (!ok) break;
                 epi.start(a, T, ch);
                 tc::fence_after_sync();
-                // two pairs of 32-column loads, each pair in flight together;
-                // the accumulator is released as soon as the second pair has
-                // landed, before its columns are handed to the mode
-                const uint32_t taddr = tmem + ((uint32_t)(quarter * 32) << 16) + buf * kN;
-                const int64_t col0 = (int64_t)ch * kN;
+                // pairs of 32-column loads, each pair in flight together; the
+                // accumulator is released as soon as the last pair has landed,
+                // before its columns are handed to the mode
+                const uint32_t taddr = tmem + ((uint32_t)(quarter * 32) << 16) + buf * kNB;
+                const int64_t col0 = (int64_t)ch * kNB;
                 uint32_t ra[32], rb[32];
-                tc::tmem_ld32_issue(taddr, ra);
-                tc::tmem_ld32_issue(taddr + 32, rb);
-                tc::tmem_ld_wait(ra);
-                tc::tmem_ld_wait(rb);
-                hand(epi, a, T, col0, ra);
-                hand(epi, a, T, col0 + 32, rb);
-                tc::tmem_ld32_issue(taddr + 64, ra);
-                tc::tmem_ld32_issue(taddr + 96, rb);
-                tc::tmem_ld_wait(ra);
-                tc::tmem_ld_wait(rb);
-                tc::fence_before_sync();
-                tc::mbar_arrive(&dempty_bar[buf]);
-                hand(epi, a, T, col0 + 64, ra);
-                hand(epi, a, T, col0 + 96, rb);
+#pragma unroll
+                for (int pr = 0; pr < kNB / 64; ++pr) {
+                    tc::tmem_ld32_issue(taddr + pr * 64, ra);
+                    tc::tmem_ld32_issue(taddr + pr * 64 + 32, rb);
+                    tc::tmem_ld_wait(ra);
+                    tc::tmem_ld_wait(rb);
+                    if (pr == kNB / 64 - 1) {
+                        tc::fence_before_sync();
+                        tc::mbar_arrive(&dempty_bar[buf]);
+                    }
+                    hand(epi, a, T, col0 + pr * 64, ra);
+                    hand(epi, a, T, col0 + pr * 64 + 32, rb);
+                }
             }
             if (!ok) break;
             epi.end(a, T);
