@@ -90,3 +90,23 @@ def test_scan_path_values_without_gpu():
         p = sieve._params(0.9, 10, 8, 4, True, 0, 0, scan_path=path)
         assert lib.sieve_search_workspace_size(ctypes.byref(v), 100, ctypes.byref(p), 0,
                                                ctypes.byref(n)) == -1
+
+
+def test_screen_scores_rejects_bad_arguments_without_gpu():
+    """sieve_screen_scores checks its arguments on the host before any device
+    work: it needs the centroids' tensor layout and d <= 256, and its output
+    rows must hold every centroid at a 32-float stride (SIEVE_EINVAL)."""
+    lib = sieve.lib()
+    ok = dict(n=1000, nlist=100, d=64, vectors=16, ids=16, list_offsets=16, centroids=16,
+              tc_centroids=16)
+    q, out = ctypes.c_void_p(256), ctypes.c_void_p(512)
+    v = sieve.IndexViewC(**{**ok, "tc_centroids": None})
+    assert lib.sieve_screen_scores(ctypes.byref(v), q, 10, out, 128, None) == -1   # no layout
+    v = sieve.IndexViewC(**{**ok, "d": 260})
+    assert lib.sieve_screen_scores(ctypes.byref(v), q, 10, out, 128, None) == -1   # d > 256
+    v = sieve.IndexViewC(**ok)
+    assert lib.sieve_screen_scores(ctypes.byref(v), q, 10, out, 96, None) == -1    # ld < nlist
+    assert lib.sieve_screen_scores(ctypes.byref(v), q, 10, out, 112, None) == -1   # ld % 32
+    assert lib.sieve_screen_scores(ctypes.byref(v), q, -1, out, 128, None) == -1   # nq < 0
+    assert lib.sieve_screen_scores(ctypes.byref(v), ctypes.c_void_p(260), 10, out, 128, None) == -1
+    assert lib.sieve_screen_scores(ctypes.byref(v), q, 10, None, 128, None) == -1
